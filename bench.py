@@ -1,0 +1,334 @@
+#!/usr/bin/env python
+"""Throughput of the xPress refinement pass on GB300 (refined draft blocks/s).
+
+One step = one refinement call (Algorithm 1 to convergence, device-side loop)
+plus acceptance against the target logits, over one batch of synthetic blocks
+already resident in HBM.  Default workload: the Qwen3-8B shape at batch 1,
+block 16, greedy (``qwen3_8b_greedy``).  L2 is flushed (a 512 MB write)
+between timed steps; steps are timed with CUDA events on the launching stream.
+
+Also reported on the same JSON line:
+  e2e           the same metric with host (pinned) inputs copied in and the
+                results copied out inside the timed region;
+  roofline      the Read + Correct + selection kernel launched alone (cold L2)
+                against the measured HBM copy bandwidth;
+  cpu_baseline  the CPU oracle on one block of the same workload;
+  clocks        nvidia-smi samples taken during the timed steps.
+
+``--impl reference`` times the CPU oracle instead (the reference arm).
+Multi-GPU: one process per GPU (torchrun); blocks are independent, so every
+rank runs its own batch (weak scaling) and the job time is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "refined draft blocks/s (Qwen3-8B shape, block 16)"
+READ_SOURCES = ["paper_2608_02438_gb300/csrc/read_tc.cu", "paper_2608_02438_gb300/csrc/common.cuh"]
+PROFILE_SUMMARY = "profiles/read_tc_qwen3_8b_greedy.txt"
+
+
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), int(os.environ.get("LOCAL_RANK", 0))
+
+
+def source_hash(paths):
+    h = hashlib.sha256()
+    for p in paths:
+        with open(os.path.join(ROOT, p), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(bytes_hash: str):
+    """dram bytes per Read launch from the committed ncu summary, if it was
+    taken on the current kernel sources."""
+    path = os.path.join(ROOT, PROFILE_SUMMARY)
+    if not os.path.exists(path):
+        return None
+    kv = {}
+    for line in open(path):
+        if ":" in line and not line.startswith("#"):
+            k, v = line.split(":", 1)
+            kv[k.strip()] = v.strip()
+    if kv.get("source_hash") != bytes_hash or "dram_bytes_per_launch" not in kv:
+        return None
+    try:
+        return float(kv["dram_bytes_per_launch"])
+    except ValueError:
+        return None
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        d = json.load(open(path))
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), "measured"
+    return 6800.0, 1900.0, "fallback"
+
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.out = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "50"], stdout=self.out,
+                                         stderr=subprocess.DEVNULL)
+        except (OSError, ValueError):
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        self.out.flush()
+        self.out.seek(0)
+        sms, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.out.read().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sms.append(float(parts[0]))
+                mx = max(mx, float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower() in ("active", "0x1", "1"):
+                    reasons.add(n)
+        if not sms:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": float(np.median(sms)), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sms)}
+
+
+def cpu_baseline(name: str, budget_s: float = 30.0):
+    """The CPU oracle as it stands, on whole blocks of the same workload."""
+    import oracle as O
+    from paper_2608_02438_gb300 import workloads as W
+    cfg, w, inp = W.make_workload(name, b=1)
+    m = O.Model(w, cfg.H, cfg.V, cfg.r, cfg.B, O.BF16 if cfg.dtype == W.BF16 else O.F32)
+    n, t0 = 0, time.perf_counter()
+    while True:
+        res = O.jacobi(m, inp["h"][0], inp["s"][0], int(inp["anchor"][0]), inp["draft"][0],
+                       float(inp["temperature"][0]), int(inp["seed"][0]), inp["offset"], cfg.K_max)
+        O.accept(m, inp["target"][0], inp["s"][0], res["tokens"], res["lse"], res["sel"], res["z_final"],
+                 float(inp["temperature"][0]), int(inp["seed"][0]), inp["offset"])
+        n += 1
+        el = time.perf_counter() - t0
+        if el > budget_s / 3 or n >= 50:
+            break
+    return n / el, n, el
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    from paper_2608_02438_gb300 import workloads as W
+    cfg = W.CONFIGS[args.config]
+    t0 = time.perf_counter()
+    val, n, el = cpu_baseline(args.config, budget_s=min(120.0, 20.0 * max(1, args.steps)))
+    line = {"impl": "reference", "metric": METRIC, "value": val, "unit": "blocks/s", "n_gpus": args.gpus,
+            "steps": n, "steps_requested": args.steps, "warmup": 0, "ms_per_step": 1000.0 * el / n,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": cfg.name, "batch": 1, "block": cfg.B, "hidden": cfg.H, "vocab": cfg.V,
+                       "rank": cfg.r, "K_max": cfg.K_max},
+            "cpu_baseline": {"value": val, "unit": "blocks/s", "cores": 1, "kind": "oracle",
+                             "sample": f"{n} whole block(s) of {cfg.name} (Algorithm 1 + acceptance), fp64, one thread"},
+            "e2e": {"value": val, "unit": "blocks/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "wall_s": time.perf_counter() - t0}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_xpress(args):
+    import torch
+    from paper_2608_02438_gb300 import binding as X
+    from paper_2608_02438_gb300 import build as BLD
+    from paper_2608_02438_gb300 import workloads as W
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(dev)
+    BLD.build()
+    cfg, w, inp = W.make_workload(args.config, seed_offset=rank)
+    dt = X.XPRESS_BF16 if cfg.dtype == W.BF16 else X.XPRESS_F32
+    ref = X.Refiner({k: X.to_device(v, dt) for k, v in w.items()}, cfg.H, cfg.V, cfg.r, cfg.B, dt)
+    stream = ref.stream
+    b = inp["h"].shape[0]
+    host = {"h": inp["h"], "s": inp["s"], "target": inp["target"], "draft": inp["draft"], "anchor": inp["anchor"],
+            "temperature": inp["temperature"], "seed": inp["seed"].view(np.int64)}
+    d = {k: (X.to_device(v, dt) if k in ("h", "s", "target") else torch.from_numpy(np.ascontiguousarray(v)).cuda())
+         for k, v in host.items()}
+    out = ref.alloc_outputs(b)
+    acc = dict(accept_len=torch.empty(b, dtype=torch.int32, device=dev),
+               out_tokens=torch.empty((b, cfg.B + 1), dtype=torch.int32, device=dev))
+    flush = torch.empty(512 * 2 ** 20, dtype=torch.uint8, device=dev)
+
+    def step():
+        ref.refine_block(d["h"], d["s"], d["draft"], d["anchor"], d["temperature"], d["seed"], inp["offset"],
+                         cfg.K_max, out=out)
+        ref.accept(d["target"], d["s"], out["tokens"], out["lse"], out["logit_sel"], out["z_final"],
+                   d["temperature"], d["seed"], inp["offset"], out=acc)
+
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, args.warmup)):
+            step()
+        torch.cuda.synchronize()
+        if ref.device_status("refine", b) != X.XPRESS_OK or ref.device_status("accept", b) != X.XPRESS_OK:
+            raise RuntimeError("device status error")
+        passes = ref.pass_count(b)
+        per_step_launches = 1 + (0) + 2 + 1 + 3 * passes + 4
+        starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize()
+        with ClockSampler(dev.index) as clk:
+            for i in range(args.steps):
+                flush.zero_()
+                starts[i].record(stream)
+                step()
+                ends[i].record(stream)
+            torch.cuda.synchronize()
+        ms = float(sum(s.elapsed_time(e) for s, e in zip(starts, ends)))
+        if world > 1:
+            tt = torch.tensor([ms], device=dev, dtype=torch.float64)
+            torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+            ms = float(tt.item())
+        value = world * b * args.steps / (ms / 1000.0)
+
+        # e2e: pinned host inputs in, results out, inside the timed region
+        pin = {k: torch.from_numpy(np.ascontiguousarray(v).view(np.int16) if k in ("h", "s", "target") and dt ==
+                                   X.XPRESS_BF16 else np.ascontiguousarray(v)).pin_memory()
+               for k, v in host.items()}
+        res_host = {"tokens": torch.empty((b, cfg.B), dtype=torch.int32).pin_memory(),
+                    "accept_len": torch.empty(b, dtype=torch.int32).pin_memory(),
+                    "out_tokens": torch.empty((b, cfg.B + 1), dtype=torch.int32).pin_memory()}
+        dview = {k: (v.view(torch.int16) if k in ("h", "s", "target") and dt == X.XPRESS_BF16 else v)
+                 for k, v in d.items()}
+        h2d = sum(t.numel() * t.element_size() for t in pin.values())
+        d2h = sum(t.numel() * t.element_size() for t in res_host.values())
+        n_e2e = max(10, min(args.steps, 300))
+        e_s = [torch.cuda.Event(enable_timing=True) for _ in range(n_e2e)]
+        e_e = [torch.cuda.Event(enable_timing=True) for _ in range(n_e2e)]
+        for i in range(n_e2e):
+            flush.zero_()
+            e_s[i].record(stream)
+            for k in pin:
+                dview[k].copy_(pin[k], non_blocking=True)
+            step()
+            res_host["tokens"].copy_(out["tokens"], non_blocking=True)
+            res_host["accept_len"].copy_(acc["accept_len"], non_blocking=True)
+            res_host["out_tokens"].copy_(acc["out_tokens"], non_blocking=True)
+            e_e[i].record(stream)
+        torch.cuda.synchronize()
+        ms_e2e = float(sum(s.elapsed_time(e) for s, e in zip(e_s, e_e)))
+        if world > 1:
+            tt = torch.tensor([ms_e2e], device=dev, dtype=torch.float64)
+            torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+            ms_e2e = float(tt.item())
+        e2e_value = world * b * n_e2e / (ms_e2e / 1000.0)
+
+        # roofline of the dominant kernel: Read + Correct + selection, alone,
+        # cold L2, over all b * B positions (a first pass)
+        step()
+        torch.cuda.synchronize()
+        ws_ptr, _ = ref.workspace("refine", b)
+        n_tok = b * cfg.B
+        reps = 50
+        r_s = [torch.cuda.Event(enable_timing=True) for _ in range(reps)]
+        r_e = [torch.cuda.Event(enable_timing=True) for _ in range(reps)]
+        for i in range(reps):
+            X.xpress_profile_read_prepare(ref.handle, ws_ptr, b, n_tok, stream.cuda_stream)
+            flush.zero_()
+            r_s[i].record(stream)
+            X.xpress_profile_read(ref.handle, ws_ptr, b, stream.cuda_stream)
+            r_e[i].record(stream)
+        torch.cuda.synchronize()
+        read_ms = float(np.mean([s.elapsed_time(e) for s, e in zip(r_s, r_e)]))
+    esz = 2 if dt == X.XPRESS_BF16 else 4
+    S = min(ref.torch.cuda.get_device_properties(dev).multi_processor_count, (cfg.V + 255) // 256)
+    read_bytes = cfg.V * cfg.r * esz + n_tok * cfg.V * esz + n_tok * cfg.r * esz + S * n_tok * 16
+    hbm, tc_peak, src = peaks()
+    achieved = read_bytes / (read_ms / 1000.0) / 1e9
+    rhash = source_hash(READ_SOURCES)
+    traffic = profiled_traffic(rhash)
+
+    if rank == 0:
+        cpu_val, cpu_n, cpu_el = cpu_baseline(args.config)
+        line = {
+            "metric": METRIC, "value": value, "unit": "blocks/s", "n_gpus": world, "steps": args.steps,
+            "warmup": max(3, args.warmup), "ms_per_step": ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if dt == X.XPRESS_BF16 else "f32",
+            "data": "synthetic",
+            "config": {"workload": cfg.name, "batch_per_gpu": b, "block": cfg.B, "hidden": cfg.H, "vocab": cfg.V,
+                       "rank": cfg.r, "K_max": cfg.K_max, "temperature": float(inp["temperature"][0]),
+                       "l2": "flushed between steps (512 MB write)"},
+            "tokens_per_s": value * cfg.B,
+            "passes_per_step": passes,
+            "e2e": {"value": e2e_value, "unit": "blocks/s", "h2d_bytes_per_step": int(h2d),
+                    "d2h_bytes_per_step": int(d2h), "steps": n_e2e},
+            "gpu_launches": per_step_launches * args.steps,
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                         "frac": achieved / hbm, "traffic": traffic, "peak_source": src,
+                         "kernel": "k_read_tc", "bytes_per_launch": read_bytes, "launch_ms": read_ms,
+                         "tokens_per_launch": n_tok, "source_hash": rhash},
+            "cpu_baseline": {"value": cpu_val, "unit": "blocks/s", "cores": 1, "kind": "oracle",
+                             "sample": f"{cpu_n} whole block(s) of {cfg.name} (Algorithm 1 + acceptance), fp64, "
+                                       f"one thread, {cpu_el:.1f} s"},
+            "clocks": clk.summary(),
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="xpress", choices=["xpress", "reference"])
+    ap.add_argument("--config", default="qwen3_8b_greedy")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_xpress(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

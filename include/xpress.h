@@ -1,0 +1,201 @@
+/*
+ * xpress.h -- C ABI of the GB300 (sm_103a) implementation of the xPress
+ * parallel refinement pass (arXiv 2608.02438, "xPress: Parallel Refinement for
+ * Diffusion Drafters in Speculative Decoding").
+ *
+ * Conventions for every entry point
+ *   - Tensors are DEVICE pointers to row-major, contiguous arrays owned by the
+ *     caller; the library never frees them and keeps no reference to them
+ *     after a call returns, except the weights given to xpress_refiner_create
+ *     (which must outlive the refiner).
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *     Calls are asynchronous on that stream; results are valid after the
+ *     stream is synchronised.
+ *   - The return value reports argument validation and launch errors only
+ *     (xpress_status).  Errors detected by the kernels themselves (a token id
+ *     out of range, a bounded wait that timed out) are recorded in a status
+ *     word inside the workspace; read it with xpress_get_device_status after
+ *     synchronising.
+ *   - Storage dtype: XPRESS_BF16 (bf16 bit patterns, 2 bytes) or XPRESS_F32.
+ *     Weights, drafter hidden states h, base logits s and target logits all
+ *     use the refiner's dtype.  Accumulation is fp32 throughout.  In the bf16
+ *     case the activations that feed a tensor-core product are rounded to bf16
+ *     (round to nearest even): c before W_1, sigma(W_1 c) before W_2, z before
+ *     W_r.  Logits l = s + delta, log-sum-exp and sampling are fp32.
+ *   - Supported shapes: r = 256, 1 <= B <= 32, V >= 32, V % 8 == 0,
+ *     H % 8 == 0; otherwise XPRESS_ERR_UNSUPPORTED.
+ *   - A refiner handle is not thread-safe: calls that use the same handle from
+ *     several host threads must be serialised by the caller.
+ */
+#ifndef XPRESS_H
+#define XPRESS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum { XPRESS_F32 = 0, XPRESS_BF16 = 1 } xpress_dtype;
+
+/* sigma in Trans (Sec. 4.1 calls it "a pointwise nonlinearity"). */
+typedef enum { XPRESS_ACT_SILU = 0, XPRESS_ACT_GELU = 1, XPRESS_ACT_RELU = 2 } xpress_act;
+
+typedef enum {
+    XPRESS_OK = 0,
+    XPRESS_ERR_INVALID_ARG = -1,   /* NULL pointer, bad size, misaligned pointer */
+    XPRESS_ERR_UNSUPPORTED = -2,   /* shape or dtype outside the supported set */
+    XPRESS_ERR_CUDA = -3,          /* a CUDA runtime call failed */
+    XPRESS_ERR_WORKSPACE = -4,     /* workspace NULL, too small or misaligned */
+    XPRESS_ERR_TIMEOUT = -5,       /* device: a bounded wait gave up */
+    XPRESS_ERR_DEVICE_CHECK = -6   /* device: an input failed a bounds check */
+} xpress_status;
+
+/* Opaque refiner: derived device tensors built once from the weights. */
+typedef struct xpress_refiner xpress_refiner;
+
+/* Refiner weights R_theta (Sec. 4.1, Eq. fuse / mix / mlp / read), device
+ * pointers in the refiner dtype, row-major:
+ *   W_e  [V, r]    token embedding; row x is the paper's column W_e[x]
+ *   W_h  [r, H]    down-projection of h_k
+ *   W_g  [r, H]    down-projection of the block mean g
+ *   W_in [r, 3r]   fusion of [W_h h_k || W_g g || W_e[x_{k-1}]] (in that order)
+ *   L    [r, B, B] per-channel causal mixer, L[d][k][j] = L^(d)_{k,j}; only the
+ *                  strictly lower triangle (j < k) is read
+ *   W1   [2r, r], W2 [r, 2r]   Trans MLP
+ *   W_r  [V, r]    readout head (shared over positions, not tied to W_e)   */
+typedef struct {
+    int H, V, r, B;
+    int dtype; /* xpress_dtype */
+    int act;   /* xpress_act */
+    const void *W_e, *W_h, *W_g, *W_in, *L, *W1, *W2, *W_r;
+} xpress_weights;
+
+/* Builds the derived tensors (the folded embedding E' = W_in[:, 2r:3r] W_e,
+ * fp32 [V, r], and the TMA descriptors) on `stream` and synchronises it.
+ * Allocates device memory (released by xpress_refiner_destroy).
+ * Errors: INVALID_ARG (NULL), UNSUPPORTED (shape/dtype), CUDA. */
+int xpress_refiner_create(const xpress_weights *w, void *stream, xpress_refiner **out);
+int xpress_refiner_destroy(xpress_refiner *refiner);
+
+/* One refinement call over b independent blocks (Sec. 4.2, Algorithm 1).
+ *   h           [b, B, H]   drafter hidden states h_1..h_B (Sec. 4.1)
+ *   s           [b, B, V]   drafter base logits s_k (Eq. correct)
+ *   draft       [b, B]      Y^(0), int32 token ids; NULL => argmax_v s_k,v
+ *                           (Algorithm 1's seed)
+ *   anchor      [b]         x_0, the fixed anchor token (the last verified token)
+ *   temperature [b]         T per sequence; T <= 0 re-selects by argmax
+ *                           (Algorithm 1), T > 0 by the fixed-noise
+ *                           hierarchical Gumbel-max draw of softmax(l/T)
+ *   seed        [b]         Philox4x32-10 key per sequence
+ *   offset                  per speculative round (counter word 3)
+ *   K_max                   maximum number of refiner passes, >= 1
+ *   fixed_K                 0: stop a block when a pass leaves it unchanged
+ *                           (Algorithm 1's break); 1: run exactly K_max
+ *                           passes on every block (Table 3 style timing)   */
+typedef struct {
+    int b;
+    const void *h;
+    const void *s;
+    const int32_t *draft;
+    const int32_t *anchor;
+    const float *temperature;
+    const uint64_t *seed;
+    uint32_t offset;
+    int K_max;
+    int fixed_K;
+} xpress_block_in;
+
+/* Outputs (device pointers; each may be NULL except tokens):
+ *   tokens    [b, B]  refined block Y (int32)
+ *   iters     [b]     refiner passes executed for the block (1..K_max)
+ *   converged [b]     1 if the last pass left the block unchanged
+ *   lse       [b, B]  T > 0: log sum_v exp(l_k,v / T) of the pass that last
+ *                     evaluated position k; T <= 0: NaN
+ *   logit_sel [b, B]  l_k,y / T at the selected token (T <= 0: l_k,y)
+ *   z_final   [b, B, r] fp32 z_k of that pass (the W_r operand before rounding)
+ *   refined_logits [b, B, V] fp32 l_k (debug; slows the pass down)          */
+typedef struct {
+    int32_t *tokens;
+    int32_t *iters;
+    int32_t *converged;
+    float *lse;
+    float *logit_sel;
+    float *z_final;
+    float *refined_logits;
+} xpress_block_out;
+
+/* Bytes of device workspace xpress_refine_block needs for b blocks. */
+size_t xpress_refine_workspace_size(const xpress_refiner *refiner, int b);
+
+/* Runs Algorithm 1 on all b blocks with no host synchronisation: the
+ * iteration loop runs on the device (a CUDA graph with a device-updated WHILE
+ * condition); blocks that have converged drop out of later passes, and a pass
+ * re-evaluates only the positions after the first token the previous pass
+ * changed (by Theorem 1 the others cannot change).  workspace: >= the size
+ * above, 256-byte aligned, owned by the caller, not shared by concurrent calls.
+ * Errors: INVALID_ARG, UNSUPPORTED, WORKSPACE, CUDA. */
+int xpress_refine_block(const xpress_refiner *refiner, const xpress_block_in *in,
+                        const xpress_block_out *out, void *workspace, size_t ws_bytes,
+                        void *stream);
+
+/* Acceptance of refined blocks against the target's logits (Sec. 3.1).
+ *   target      [b, B+1, V] target logits for positions 1..B and the bonus
+ *   s, tokens, lse, logit_sel, z_final: as passed to / returned by
+ *               xpress_refine_block for the same blocks
+ *   temperature [b] T <= 0: greedy -- accept the longest prefix equal to the
+ *               target argmax, then emit the target's token;  T > 0: lossless
+ *               rejection sampling -- accept y_k when u_k q_k(y_k) < p_k(y_k),
+ *               else emit a draw of max(0, p_k - q_k) (p_k if that is empty);
+ *               after B acceptances emit a draw of p_{B+1}
+ *   seed, offset: as for refinement (streams 2 and 3)
+ * All input pointers are required (lossless draws read lse, logit_sel, z_final
+ * and s).
+ * Outputs: accept_len [b] (0..B accepted draft tokens) and out_tokens
+ * [b, B+1] (accepted tokens, then the correction or bonus token, then -1).
+ * Errors: INVALID_ARG, WORKSPACE, CUDA. */
+typedef struct {
+    int b;
+    const void *target;
+    const void *s;
+    const int32_t *tokens;
+    const float *lse;
+    const float *logit_sel;
+    const float *z_final;
+    const float *temperature;
+    const uint64_t *seed;
+    uint32_t offset;
+} xpress_accept_in;
+
+size_t xpress_accept_workspace_size(const xpress_refiner *refiner, int b);
+int xpress_accept(const xpress_refiner *refiner, const xpress_accept_in *in, int32_t *accept_len,
+                  int32_t *out_tokens, void *workspace, size_t ws_bytes, void *stream);
+
+/* Synchronises `stream`, then reads (and clears) the device status word kept
+ * in `workspace` by xpress_refine_block / xpress_accept.  *status_out is an
+ * xpress_status (XPRESS_OK, XPRESS_ERR_TIMEOUT or XPRESS_ERR_DEVICE_CHECK). */
+int xpress_get_device_status(void *workspace, void *stream, int32_t *status_out);
+
+/* Synchronises `stream`, then reads how many refiner passes the device loop
+ * of the last xpress_refine_block call on `workspace` executed (the largest
+ * per-block pass count that involved a kernel launch). */
+int xpress_get_pass_count(void *workspace, void *stream, int32_t *passes_out);
+
+/* Profiling hooks (benchmarks only).  After an xpress_refine_block call on
+ * `workspace`, _prepare marks the first n_tokens positions of the b blocks as
+ * evaluated, and xpress_profile_read launches the Read + Correct + selection
+ * kernel alone on `stream` (its results overwrite the call's scratch), so
+ * that it can be timed with CUDA events.  The inputs of that call must still
+ * be alive.  Errors: INVALID_ARG, WORKSPACE, CUDA. */
+int xpress_profile_read_prepare(const xpress_refiner *refiner, void *workspace, int b, int n_tokens,
+                                void *stream);
+int xpress_profile_read(const xpress_refiner *refiner, void *workspace, int b, void *stream);
+
+const char *xpress_status_string(int status);
+int xpress_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* XPRESS_H */

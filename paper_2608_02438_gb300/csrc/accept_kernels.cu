@@ -1,0 +1,169 @@
+// accept_kernels.cu -- speculative acceptance of refined blocks (Sec. 3.1).
+//
+//   k_acc_rows    per target row (block position k = 1..B+1) and vocabulary
+//                 chunk: argmax (T <= 0) or the running max / sum of exp of
+//                 target / T (T > 0)
+//   k_acc_decide  per block: greedy -- longest prefix equal to the target
+//                 argmax plus the target's next token;  lossless -- accept y_k
+//                 while u_k q_k(y_k) < p_k(y_k), q from the refinement pass
+//                 (exp(l_y/T - lse)), p = softmax(target_k / T)
+//   k_acc_sample  per block with a draw to make and vocabulary chunk:
+//                 Gumbel-max over log max(0, p_k - q_k) at the first rejected
+//                 position (q_k recomputed from z_final through W_r), with the
+//                 draw from p_k alongside for an empty residual; or the bonus
+//                 draw from p_{B+1} after B acceptances
+//   k_acc_finish  combine the chunk partials and emit the last token
+#include "common.cuh"
+#include "kernels.h"
+
+namespace xp {
+
+__global__ void __launch_bounds__(256) k_acc_rows(AcceptParams p)
+{
+    const int row = blockIdx.x;                   // seq * (B + 1) + k
+    const int seq = row / (p.B + 1);
+    const int chunks = gridDim.y, c = blockIdx.y;
+    const int v0 = (int)((long long)p.V * c / chunks), v1 = (int)((long long)p.V * (c + 1) / chunks);
+    const float T = p.temperature[seq];
+    const float invT = T > 0.0f ? 1.0f / T : 0.0f;
+    Partial a{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
+    for (int v = v0 + threadIdx.x; v < v1; v += blockDim.x) {
+        const float x = ld_any(p.target, p.dtype, (size_t)row * p.V + v);
+        if (invT <= 0.0f) {
+            merge_argmax(a.best, a.idx, x, v);
+        } else {
+            merge_lse(a.m, a.s, x * invT, 1.0f);
+        }
+    }
+    __shared__ Partial sp[256];
+    sp[threadIdx.x] = a;
+    __syncthreads();
+    for (int w = 128; w > 0; w >>= 1) {
+        if (threadIdx.x < w) {
+            Partial x = sp[threadIdx.x];
+            merge_partial(x, sp[threadIdx.x + w], invT > 0.0f);
+            sp[threadIdx.x] = x;
+        }
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) p.rowpart[(size_t)row * chunks + c] = sp[0];
+}
+
+__device__ Partial combine_row(const AcceptParams &p, int row, int chunks, bool sampling)
+{
+    Partial a{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
+    for (int c = 0; c < chunks; ++c) merge_partial(a, p.rowpart[(size_t)row * chunks + c], sampling);
+    return a;
+}
+
+// one thread per block (sequence)
+__global__ void k_acc_decide(AcceptParams p, int chunks)
+{
+    const int seq = blockIdx.x * blockDim.x + threadIdx.x;
+    if (seq >= p.b) return;
+    const int B = p.B;
+    const float T = p.temperature[seq];
+    int32_t *out = p.out_tokens + (size_t)seq * (B + 1);
+    for (int k = 0; k <= B; ++k) out[k] = -1;
+    int n = 0;
+    if (T <= 0.0f) {
+        for (;;) {
+            const Partial a = combine_row(p, seq * (B + 1) + n, chunks, false);
+            if (n < B && p.tokens[(size_t)seq * B + n] == a.idx) { out[n] = a.idx; ++n; continue; }
+            out[n] = a.idx;
+            break;
+        }
+        p.job[seq] = -1;
+    } else {
+        const float invT = 1.0f / T;
+        int job = B;
+        for (; n < B; ++n) {
+            const int row = seq * (B + 1) + n;
+            const Partial a = combine_row(p, row, chunks, true);
+            const float lse_p = a.m + logf(a.s);
+            int y = p.tokens[(size_t)seq * B + n];
+            if (y < 0 || y >= p.V) { set_status(p.status, ST_BOUNDS); y = 0; }
+            const float p_y = expf(ld_any(p.target, p.dtype, (size_t)row * p.V + y) * invT - lse_p);
+            const float q_y = expf(p.logit_sel[(size_t)seq * B + n] - p.lse[(size_t)seq * B + n]);
+            const float u = uniform01(p.seed[seq], 0u, (uint32_t)n, STREAM_ACCEPT, p.offset);
+            if (u * q_y < p_y) { out[n] = y; continue; }
+            job = n;
+            p.jobf[seq] = lse_p;
+            break;
+        }
+        p.job[seq] = job;
+    }
+    p.accept_len[seq] = n;
+}
+
+// grid (b, chunks), 256 threads.  Writes two argmax partials per chunk: the
+// residual draw (best, idx) and the draw from p (m, s reused as score, idx).
+__global__ void __launch_bounds__(256) k_acc_sample(AcceptParams p)
+{
+    const int seq = blockIdx.x, chunks = gridDim.y, c = blockIdx.y;
+    const int k = p.job[seq];
+    if (k < 0) return;
+    const int B = p.B;
+    const float invT = 1.0f / p.temperature[seq];
+    const int v0 = (int)((long long)p.V * c / chunks), v1 = (int)((long long)p.V * (c + 1) / chunks);
+    __shared__ float zop[RANK];
+    const bool resid = k < B;
+    if (resid)
+        for (int d = threadIdx.x; d < RANK; d += blockDim.x)
+            zop[d] = round_op(p.z_final[((size_t)seq * B + k) * RANK + d], p.dtype);
+    __syncthreads();
+    const unsigned long long seed = p.seed[seq];
+    const size_t trow = (size_t)seq * (B + 1) + k;
+    const float lse_p = resid ? p.jobf[seq] : 0.0f;
+    const float lse_q = resid ? p.lse[(size_t)seq * B + k] : 0.0f;
+    float rb = -INFINITY, pb = -INFINITY;
+    int ri = 0x7fffffff, pi = 0x7fffffff;
+    for (int v = v0 + threadIdx.x; v < v1; v += blockDim.x) {
+        const float tx = ld_any(p.target, p.dtype, trow * p.V + v) * invT;
+        const float g = gumbel(seed, (uint32_t)v, (uint32_t)k, STREAM_RESID, p.offset);
+        merge_argmax(pb, pi, tx + g, v);
+        if (resid) {
+            float acc = 0.0f;
+            for (int d = 0; d < RANK; ++d) acc = fmaf(ld_any(p.W_r, p.dtype, (size_t)v * RANK + d), zop[d], acc);
+            const float lx = (acc + ld_any(p.s, p.dtype, ((size_t)seq * B + k) * p.V + v)) * invT;
+            const float res = expf(tx - lse_p) - expf(lx - lse_q);
+            if (res > 0.0f) merge_argmax(rb, ri, logf(res) + g, v);
+        }
+    }
+    __shared__ float sb[2][256];
+    __shared__ int si[2][256];
+    sb[0][threadIdx.x] = rb; si[0][threadIdx.x] = ri;
+    sb[1][threadIdx.x] = pb; si[1][threadIdx.x] = pi;
+    __syncthreads();
+    for (int w = 128; w > 0; w >>= 1) {
+        if (threadIdx.x < w)
+            for (int h = 0; h < 2; ++h) {
+                float b0 = sb[h][threadIdx.x];
+                int i0 = si[h][threadIdx.x];
+                merge_argmax(b0, i0, sb[h][threadIdx.x + w], si[h][threadIdx.x + w]);
+                sb[h][threadIdx.x] = b0;
+                si[h][threadIdx.x] = i0;
+            }
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) p.spart[(size_t)seq * chunks + c] = Partial{sb[0][0], si[0][0], sb[1][0], __int_as_float(si[1][0])};
+}
+
+__global__ void k_acc_finish(AcceptParams p, int chunks)
+{
+    const int seq = blockIdx.x * blockDim.x + threadIdx.x;
+    if (seq >= p.b) return;
+    const int k = p.job[seq];
+    if (k < 0) return;
+    float rb = -INFINITY, pb = -INFINITY;
+    int ri = 0x7fffffff, pi = 0x7fffffff;
+    for (int c = 0; c < chunks; ++c) {
+        const Partial a = p.spart[(size_t)seq * chunks + c];
+        merge_argmax(rb, ri, a.best, a.idx);
+        merge_argmax(pb, pi, a.m, __float_as_int(a.s));
+    }
+    const bool use_resid = k < p.B && rb > -INFINITY;
+    p.out_tokens[(size_t)seq * (p.B + 1) + k] = use_resid ? ri : pi;
+}
+
+}  // namespace xp

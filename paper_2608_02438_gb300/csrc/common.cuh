@@ -1,0 +1,366 @@
+// common.cuh -- device helpers shared by the xPress kernels (sm_103a).
+//
+// Contents: problem constants, the device parameter block, bf16 conversion,
+// Philox4x32-10 (Salmon et al., SC'11) with the counter layout the library
+// uses, and thin inline-PTX wrappers for mbarrier, TMA and tcgen05.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace xp {
+
+constexpr int RANK = 256;        // refiner rank r (Sec. 4.1 fixes r = 256)
+constexpr int GROUP = 32;        // vocabulary group of the hierarchical Gumbel-max
+constexpr int MAX_B = 32;        // largest block the kernels support
+constexpr int STREAM_GROUP = 0;  // Philox counter word 2: which draw
+constexpr int STREAM_ELEM = 1;
+constexpr int STREAM_ACCEPT = 2;
+constexpr int STREAM_RESID = 3;
+
+// device status word bits (xpress_get_device_status maps them to xpress_status)
+constexpr int ST_TIMEOUT = 1;
+constexpr int ST_BOUNDS = 2;
+
+// control block slots (int32, in the workspace)
+constexpr int CTL_NACT = 0;     // tokens evaluated by the next pass
+constexpr int CTL_DONE = 1;     // last-block-done ticket of the reduce kernel
+constexpr int CTL_PASS = 2;     // passes executed so far
+constexpr int CTL_ACC_DONE = 3; // ticket of the accept kernels
+constexpr int CTL_WORDS = 8;
+
+struct SeqState {
+    int active;     // takes part in the next pass
+    int m;          // the next pass evaluates positions k > m (0-based; -1 = all)
+    int iters;      // passes executed
+    int converged;  // the last pass left the block unchanged
+    int off;        // packed index of the first evaluated position in the next pass
+    int cnt;        // number of evaluated positions in the next pass
+    int pad0, pad1;
+};
+
+// One split-vocabulary partial per (vocab range, evaluated token).
+// T <= 0: best = max logit, idx = its token id (smallest on ties).
+// T  > 0: best = max group score (lse_g + Gumbel), idx = that group,
+//         (m, s) = running max and sum of exp(x - m) of x = l / T.
+struct Partial {
+    float best;
+    int idx;
+    float m;
+    float s;
+};
+
+// Everything a call needs on the device; written by the init kernel from the
+// by-value copy the host places in the graph's first node.
+struct Params {
+    int b, B, H, V, N;           // N = b * B
+    int dtype, act;              // 0 f32, 1 bf16;  0 SiLU, 1 GELU, 2 ReLU
+    int K_max, fixed_K;
+    uint32_t offset;
+    int S;                       // vocabulary ranges of the Read kernel
+    int ksplit;                  // split-K factor of the hidden projection
+    // inputs (caller-owned)
+    const void *h, *s;
+    const int32_t *draft, *anchor;
+    const float *temperature;
+    const unsigned long long *seed;
+    // weights (caller-owned) and derived tensors (refiner-owned)
+    const void *W_h, *W_g, *W_in, *L, *W1, *W2, *W_r;
+    const float *Ep;             // E' = W_in[:, 2r:3r] W_e, fp32 [V, r]
+    // outputs (caller-owned; NULL allowed except tokens)
+    int32_t *tokens, *iters, *converged;
+    float *lse, *logit_sel, *z_final, *logits;
+    // workspace
+    int32_t *status;
+    int32_t *ctl;
+    SeqState *st;
+    float *Upart;                // [ksplit, N, 2r] partial sums of h [W_h; W_g]^T
+    float *Pc;                   // [N, r] token-independent part of c after Mix
+    int32_t *Ynew;               // [N]
+    int32_t *act_tok;            // [N] packed evaluated tokens (global token ids)
+    void *zpack;                 // [N, r] W_r operand of the evaluated tokens
+    float *zbuf;                 // [N, r] fp32 z when the caller passes no z_final
+    Partial *part;               // [S, N]
+};
+
+// ------------------------------------------------------------------ numbers
+
+__device__ __forceinline__ float bf2f(uint16_t b) { return __uint_as_float((uint32_t)b << 16); }
+__device__ __forceinline__ uint16_t f2bf(float f) { return __bfloat16_as_ushort(__float2bfloat16_rn(f)); }
+__device__ __forceinline__ float round_op(float x, int dtype) { return dtype ? bf2f(f2bf(x)) : x; }
+
+template <typename T> __device__ __forceinline__ float ldf(const T *p, size_t i);
+template <> __device__ __forceinline__ float ldf<float>(const float *p, size_t i) { return p[i]; }
+template <> __device__ __forceinline__ float ldf<uint16_t>(const uint16_t *p, size_t i) { return bf2f(p[i]); }
+
+__device__ __forceinline__ float ld_any(const void *p, int dtype, size_t i)
+{
+    return dtype ? bf2f(static_cast<const uint16_t *>(p)[i]) : static_cast<const float *>(p)[i];
+}
+
+__device__ __forceinline__ float act_fn(int act, float t)
+{
+    if (act == 2) return fmaxf(t, 0.0f);
+    if (act == 1) return 0.5f * t * (1.0f + erff(t * 0.70710678118654752f));
+    return t / (1.0f + expf(-t));
+}
+
+// Philox4x32-10, written from its published definition (10 rounds of two
+// 32x32->64 multiplies and Weyl key bumps).
+__device__ __forceinline__ uint4 philox10(uint4 c, uint32_t k0, uint32_t k1)
+{
+#pragma unroll
+    for (int i = 0; i < 10; ++i) {
+        const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
+        const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
+        c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+        k0 += 0x9E3779B9u;
+        k1 += 0xBB67AE85u;
+    }
+    return c;
+}
+
+// Counter layout shared with the CPU oracle: (index >> 2, position, stream,
+// offset), output word index & 3; u = ((x >> 9) + 0.5) 2^-23 in (0, 1).
+__device__ __forceinline__ float uniform01(unsigned long long seed, uint32_t index, uint32_t pos,
+                                           uint32_t stream, uint32_t offset)
+{
+    const uint4 o = philox10(make_uint4(index >> 2, pos, stream, offset), (uint32_t)seed,
+                             (uint32_t)(seed >> 32));
+    const uint32_t w = (index & 3u) == 0 ? o.x : (index & 3u) == 1 ? o.y : (index & 3u) == 2 ? o.z : o.w;
+    return ((float)(w >> 9) + 0.5f) * (1.0f / 8388608.0f);
+}
+
+__device__ __forceinline__ float gumbel(unsigned long long seed, uint32_t index, uint32_t pos, uint32_t stream,
+                                        uint32_t offset)
+{
+    return -logf(-logf(uniform01(seed, index, pos, stream, offset)));
+}
+
+__device__ __forceinline__ void set_status(int32_t *status, int bit)
+{
+    if (status) atomicOr(status, bit);
+}
+
+// ---------------------------------------------------- split-vocab combining
+
+// T <= 0 argmax merge: larger value wins, equal values keep the smaller id.
+__device__ __forceinline__ void merge_argmax(float &best, int &idx, float ob, int oi)
+{
+    if (ob > best || (ob == best && oi < idx)) { best = ob; idx = oi; }
+}
+
+// log-sum-exp merge of (m, s) pairs, s = sum exp(x - m).
+__device__ __forceinline__ void merge_lse(float &m, float &s, float om, float os)
+{
+    if (om == -INFINITY) return;
+    if (m == -INFINITY) { m = om; s = os; return; }
+    if (om > m) { s = s * __expf(m - om) + os; m = om; }
+    else { s += os * __expf(om - m); }
+}
+
+__device__ __forceinline__ void merge_partial(Partial &a, const Partial &b, bool sampling)
+{
+    merge_argmax(a.best, a.idx, b.best, b.idx);
+    if (sampling) merge_lse(a.m, a.s, b.m, b.s);
+}
+
+// Per-token selection state over a run of 32-wide vocabulary groups.
+struct SelState {
+    float best; int idx; float m; float s;
+    __device__ __forceinline__ void init() { best = -INFINITY; idx = 0x7fffffff; m = -INFINITY; s = 0.0f; }
+};
+
+// Fold one group of 32 corrected logits l[v0 .. v0+31] (entries j >= valid
+// are ignored) into the state.  T <= 0: argmax.  T > 0: x = l * invT, the
+// group's log-sum-exp plus its Gumbel noise competes for the group draw, and
+// (m, s) accumulate the full log-sum-exp.
+__device__ __forceinline__ void select_group(SelState &st, const float *l, int v0, int valid, float invT,
+                                             unsigned long long seed, uint32_t pos, uint32_t offset)
+{
+    if (valid <= 0) return;
+    if (invT <= 0.0f) {
+        float mx = -INFINITY;
+#pragma unroll
+        for (int j = 0; j < GROUP; ++j)
+            if (j < valid) mx = fmaxf(mx, l[j]);
+        if (mx > st.best) {
+            int at = 0;
+#pragma unroll
+            for (int j = GROUP - 1; j >= 0; --j)
+                if (j < valid && l[j] == mx) at = j;
+            st.best = mx;
+            st.idx = v0 + at;
+        }
+        return;
+    }
+    float x[GROUP];
+    float mx = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < GROUP; ++j) {
+        x[j] = l[j] * invT;
+        if (j < valid) mx = fmaxf(mx, x[j]);
+    }
+    float sum = 0.0f;
+#pragma unroll
+    for (int j = 0; j < GROUP; ++j)
+        if (j < valid) sum += __expf(x[j] - mx);
+    const uint32_t g = (uint32_t)v0 / GROUP;
+    const float score = mx + __logf(sum) + gumbel(seed, g, pos, STREAM_GROUP, offset);
+    if (score > st.best) { st.best = score; st.idx = (int)g; }
+    merge_lse(st.m, st.s, mx, sum);
+}
+
+// ------------------------------------------------------------- PTX wrappers
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p)
+{
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ unsigned long long globaltimer()
+{
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t *bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar)
+{
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Bounded wait: gives up after `limit_ns` of wall time or as soon as another
+// role raised *abort; returns false then (the caller unwinds).
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volatile int *abort,
+                                          unsigned long long limit_ns = 2000000000ull)
+{
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = globaltimer();
+    for (uint32_t it = 1;; ++it) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((it & 63u) == 0) {
+            if (*abort) return false;
+            if (globaltimer() - t0 > limit_ns) { *abort = 1; return false; }
+        }
+    }
+}
+
+__device__ __forceinline__ void fence_barrier_init()
+{
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void tma_load_2d(void *smem_dst, const CUtensorMap *map, uint64_t *bar, int x, int y)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+        ::"r"(smem_u32(smem_dst)), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
+        : "memory");
+}
+
+__device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap *map)
+{
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+// tcgen05 (5th-generation tensor core, accumulators in tensor memory)
+__device__ __forceinline__ void tmem_alloc(uint32_t *dst_smem, uint32_t ncols)
+{
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst_smem)),
+                 "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish()
+{
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols)
+{
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// D[tmem] (+)= A[smem] * B[smem]^T, kind::f16 (bf16 inputs, fp32 accumulate)
+__device__ __forceinline__ void tc_mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                            uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+        ::"r"(d_tmem), "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// Arrive on `bar` once every tcgen05.mma issued so far by this thread is done.
+__device__ __forceinline__ void tc_commit(uint64_t *bar)
+{
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                     smem_u32(bar))
+                 : "memory");
+}
+
+// 32 lanes x 32 consecutive fp32 columns; thread t gets lane (base + t).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32])
+{
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, "
+        "%14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]),
+          "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]),
+          "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Shared-memory matrix descriptor for a K-major operand stored with the
+// 128-byte swizzle (rows of 64 bf16 at a 128-byte pitch, 8-row groups 1024
+// bytes apart): start address, leading offset 16 B, stride offset 1024 B,
+// descriptor version 1, layout type 2 (SWIZZLE_128B).
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr)
+{
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
+           ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+// Instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, both
+// K-major, N >> 3 at bit 17, M >> 4 at bit 24.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N)
+{
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+}  // namespace xp

@@ -1,0 +1,51 @@
+// kernels.h -- declarations of the kernels launched by the host code.
+#pragma once
+
+#include "common.cuh"
+
+namespace xp {
+
+struct AcceptParams {
+    int b, B, V, dtype;
+    const void *target, *s;
+    const int32_t *tokens;
+    const float *lse, *logit_sel, *z_final, *temperature;
+    const unsigned long long *seed;
+    uint32_t offset;
+    const void *W_r;
+    int32_t *accept_len, *out_tokens;
+    int32_t *status;
+    Partial *rowpart;   // [b * (B + 1), chunks]
+    int32_t *job;       // [b] position of the draw (-1: none, B: bonus)
+    float *jobf;        // [b] log-sum-exp of target / T at that position
+    Partial *spart;     // [b, chunks]
+};
+
+// refine_kernels.cu
+__global__ void k_init(Params pin, Params *pdev, cudaGraphConditionalHandle handle);
+__global__ void k_rowmax(const Params *pp);
+__global__ void k_pre_gemm(const Params *pp, int which, int kchunk);
+__global__ void k_pre_mix(const Params *pp);
+__global__ void k_mix_mlp(const Params *pp);
+__global__ void k_read_simt(const Params *pp);
+__global__ void k_reduce(const Params *pp, cudaGraphConditionalHandle handle);
+__global__ void k_prof_prepare(int32_t *ctl, int32_t *act_tok, int n);
+__global__ void k_build_ep(const void *W_e, const void *W_in, float *Ep, int V, int dtype);
+
+// read_tc.cu
+__global__ void k_read_tc(const Params *pp, const __grid_constant__ CUtensorMap tmap_wr,
+                          const __grid_constant__ CUtensorMap tmap_z);
+extern const size_t kReadTcSmemBytes;
+extern const int kReadTcThreads;
+
+// accept_kernels.cu
+__global__ void k_acc_rows(AcceptParams p);
+__global__ void k_acc_decide(AcceptParams p, int chunks);
+__global__ void k_acc_sample(AcceptParams p);
+__global__ void k_acc_finish(AcceptParams p, int chunks);
+
+constexpr int MIX_MLP_DYN_SMEM = (MAX_B * RANK + MAX_B * 2 * RANK) * 4;
+constexpr int READ_SIMT_DYN_SMEM = (32 * (RANK + 1) + 8 * 32 * 33) * 4;
+inline int pre_mix_smem(int B) { return (B * 2 * RANK + RANK + B * 32) * 4; }
+
+}  // namespace xp

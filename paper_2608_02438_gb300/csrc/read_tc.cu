@@ -1,0 +1,280 @@
+// read_tc.cu -- Read + Correct + selection on the 5th-generation tensor cores.
+//
+// Computes, for every evaluated token z_k (the W_r operand, bf16) and every
+// vocabulary id v,  l_k,v = s_k,v + (W_r z_k)_v  (Sec. 4.1, Eq. read and
+// Eq. correct) and folds it straight into the token's selection state
+// (Algorithm 1's argmax at T = 0, the group draw of the hierarchical
+// Gumbel-max at T > 0).  The logits never travel to HBM.
+//
+// GEMM view: D[token, v] = z[token, :] . W_r[v, :], M = tokens (128 per tile),
+// N = vocabulary (256 per tile), K = r = 256.  Tokens sit in TMEM lanes so that
+// each epilogue thread owns one token and reduces over vocabulary columns
+// without any cross-thread traffic.
+//
+// Roles (320 threads, one CTA per SM, persistent over a contiguous vocabulary
+// range):
+//   warp 0      TMA producer: the token tile (A, kept for the whole range) and
+//               a 4-stage ring of W_r K-chunks (B, 32 KB each)
+//   warp 1      TMEM allocator and tcgen05.mma issuer (one thread)
+//   warps 2-9   epilogue: tcgen05.ld 32 columns, add s, select_group
+// Two TMEM accumulators of 256 columns let the MMA of tile t+1 overlap the
+// epilogue of tile t.  With <= 32 evaluated tokens the 32 token rows are
+// replicated into all four TMEM lane quarters, so that all four SM
+// sub-partitions share the epilogue (each warp takes one 32-id group).
+#include "common.cuh"
+#include "kernels.h"
+
+namespace xp {
+
+constexpr int TC_BM = 128;
+constexpr int TC_BN = 256;
+constexpr int TC_BK = 64;                     // one 128-byte swizzle row of bf16
+constexpr int TC_KCH = RANK / TC_BK;          // 4 K-chunks
+constexpr int TC_STAGES = 4;
+constexpr int TC_EPI_WARPS = 8;
+constexpr int TC_THREADS = 32 * (2 + TC_EPI_WARPS);
+constexpr uint32_t TC_A_CHUNK = TC_BM * TC_BK * 2;       // 16 KB
+constexpr uint32_t TC_A_BYTES = TC_A_CHUNK * TC_KCH;      // 64 KB
+constexpr uint32_t TC_B_STAGE = TC_BN * TC_BK * 2;       // 32 KB
+constexpr uint32_t TC_TMEM_COLS = 2 * TC_BN;              // two accumulators
+constexpr uint32_t TC_IDESC = idesc_bf16(TC_BM, TC_BN);
+
+struct TcShared {
+    uint64_t full[TC_STAGES];
+    uint64_t empty[TC_STAGES];
+    uint64_t a_full, a_empty;
+    uint64_t tfull[2], tempty[2];
+    uint64_t drain;
+    uint32_t tmem_base;
+    int abort;
+    SelState st[TC_EPI_WARPS][32];
+};
+
+constexpr size_t TC_SMEM_BYTES = 1024 + TC_A_BYTES + TC_STAGES * TC_B_STAGE + sizeof(TcShared);
+const size_t kReadTcSmemBytes = TC_SMEM_BYTES;
+const int kReadTcThreads = TC_THREADS;
+
+__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+
+// Named barrier over the 8 epilogue warps that also ORs a predicate, so that
+// every epilogue warp takes the same decision to stop after an abort.
+__device__ __forceinline__ bool epi_bar_or(bool pred)
+{
+    uint32_t res;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "bar.red.or.pred q, 1, 256, p;\n\t"
+        "selp.u32 %0, 1, 0, q;\n\t}"
+        : "=r"(res)
+        : "r"((uint32_t)pred)
+        : "memory");
+    return res != 0;
+}
+
+__global__ void __launch_bounds__(TC_THREADS, 1)
+    k_read_tc(const Params *__restrict__ pp, const __grid_constant__ CUtensorMap tmap_wr,
+              const __grid_constant__ CUtensorMap tmap_z)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *sA = base;
+    uint8_t *sB = base + TC_A_BYTES;
+    TcShared &sh = *reinterpret_cast<TcShared *>(sB + TC_STAGES * TC_B_STAGE);
+    const Params &p = *pp;
+    const int n = p.ctl[CTL_NACT];
+    if (n == 0) return;
+    const bool small = n <= 32;
+    const int MT = small ? 1 : (n + TC_BM - 1) / TC_BM;
+    const int NVT = (p.V + TC_BN - 1) / TC_BN;
+    const int S = gridDim.x, r = blockIdx.x;
+    const int vt0 = (int)((long long)NVT * r / S), vt1 = (int)((long long)NVT * (r + 1) / S);
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < TC_STAGES; ++i) { mbar_init(&sh.full[i], 1); mbar_init(&sh.empty[i], 1); }
+        mbar_init(&sh.a_full, 1);
+        mbar_init(&sh.a_empty, 1);
+        for (int i = 0; i < 2; ++i) { mbar_init(&sh.tfull[i], 1); mbar_init(&sh.tempty[i], TC_EPI_WARPS); }
+        mbar_init(&sh.drain, 1);
+        sh.abort = 0;
+        fence_barrier_init();
+    }
+    if (warp == 1) { tmem_alloc(&sh.tmem_base, TC_TMEM_COLS); tmem_relinquish(); }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = sh.tmem_base;
+    volatile int *abort = &sh.abort;
+
+    if (warp == 0) {
+        // ------------------------------------------------------- producer
+        if (lane == 0) {
+            tma_prefetch_desc(&tmap_wr);
+            tma_prefetch_desc(&tmap_z);
+            int stage = 0;
+            uint32_t phase = 0, pending = 0, pend_par = 0;
+            for (int j = 0; j < MT && !*abort; ++j) {
+                if (!mbar_wait(&sh.a_empty, (j & 1) ^ 1, abort)) break;
+                mbar_expect_tx(&sh.a_full, TC_A_BYTES);
+                for (int kc = 0; kc < TC_KCH; ++kc)
+                    for (int q = 0; q < 4; ++q)
+                        tma_load_2d(sA + kc * TC_A_CHUNK + q * 4096, &tmap_z, &sh.a_full, kc * TC_BK,
+                                    small ? 0 : j * TC_BM + 32 * q);
+                for (int vt = vt0; vt < vt1 && !*abort; ++vt)
+                    for (int kc = 0; kc < TC_KCH; ++kc) {
+                        if (!mbar_wait(&sh.empty[stage], phase ^ 1, abort)) break;
+                        mbar_expect_tx(&sh.full[stage], TC_B_STAGE);
+                        tma_load_2d(sB + stage * TC_B_STAGE, &tmap_wr, &sh.full[stage], kc * TC_BK, vt * TC_BN);
+                        pending |= 1u << stage;
+                        pend_par = (pend_par & ~(1u << stage)) | (phase << stage);
+                        if (++stage == TC_STAGES) { stage = 0; phase ^= 1; }
+                    }
+            }
+            if (*abort) {
+                // let the copies already issued land before the CTA goes away
+                for (int st = 0; st < TC_STAGES; ++st)
+                    if (pending & (1u << st)) {
+                        int dummy = 0;
+                        mbar_wait(&sh.full[st], (pend_par >> st) & 1, &dummy, 10000000ull);
+                    }
+            }
+        }
+    } else if (warp == 1) {
+        // ---------------------------------------------------- MMA issuer
+        if (lane == 0) {
+            int stage = 0, t = 0;
+            uint32_t phase = 0;
+            for (int j = 0; j < MT && !*abort; ++j) {
+                if (!mbar_wait(&sh.a_full, j & 1, abort)) break;
+                tc_fence_after();
+                const uint32_t a0 = smem_u32(sA);
+                for (int vt = vt0; vt < vt1 && !*abort; ++vt, ++t) {
+                    const int buf = t & 1;
+                    if (!mbar_wait(&sh.tempty[buf], ((t >> 1) & 1) ^ 1, abort)) break;
+                    tc_fence_after();
+                    const uint32_t d = tmem + buf * TC_BN;
+                    for (int kc = 0; kc < TC_KCH; ++kc) {
+                        if (!mbar_wait(&sh.full[stage], phase, abort)) break;
+                        tc_fence_after();
+                        const uint32_t b0 = smem_u32(sB + stage * TC_B_STAGE);
+#pragma unroll
+                        for (int kk = 0; kk < TC_BK / 16; ++kk)
+                            tc_mma_bf16(d, smem_desc_sw128(a0 + kc * TC_A_CHUNK + kk * 32),
+                                        smem_desc_sw128(b0 + kk * 32), TC_IDESC, (kc | kk) != 0);
+                        tc_commit(&sh.empty[stage]);
+                        if (++stage == TC_STAGES) { stage = 0; phase ^= 1; }
+                    }
+                    tc_commit(&sh.tfull[buf]);
+                }
+                tc_commit(&sh.a_empty);
+            }
+            // every MMA issued above has finished before the CTA tears down
+            tc_commit(&sh.drain);
+            int dummy = 0;
+            mbar_wait(&sh.drain, 0, &dummy, 100000000ull);
+        }
+    } else {
+        // ------------------------------------------------------ epilogue
+        const int ew = warp - 2;
+        const int q = warp & 3;              // TMEM lane quarter this warp may access
+        const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+        const int g_first = small ? ew : (ew >> 2) * 4;
+        const int g_count = small ? 1 : 4;
+        int t = 0;
+        for (int j = 0; j < MT; ++j) {
+            bool ok = true;
+            const int slot = small ? lane : q * 32 + lane;
+            const int i = small ? lane : j * TC_BM + slot;
+            const bool valid = i < n;
+            int tok = 0, pos = 0, seq = 0;
+            float invT = 0.0f;
+            unsigned long long seed = 0;
+            if (valid) {
+                tok = p.act_tok[i];
+                seq = tok / p.B;
+                pos = tok % p.B;
+                const float T = p.temperature[seq];
+                invT = T > 0.0f ? 1.0f / T : 0.0f;
+                seed = p.seed[seq];
+            }
+            const uint16_t *srow = static_cast<const uint16_t *>(p.s) + (size_t)tok * p.V;
+            SelState sel;
+            sel.init();
+            for (int vt = vt0; vt < vt1; ++vt, ++t) {
+                const int buf = t & 1;
+                if (!mbar_wait(&sh.tfull[buf], (t >> 1) & 1, abort)) { ok = false; break; }
+                tc_fence_after();
+                for (int gl = g_first; gl < g_first + g_count; ++gl) {
+                    const int v0 = vt * TC_BN + gl * GROUP;
+                    const int nv = min(GROUP, p.V - v0);
+                    float sv[GROUP];
+                    if (valid && nv == GROUP) {
+                        const uint4 *src = reinterpret_cast<const uint4 *>(srow + v0);
+#pragma unroll
+                        for (int c = 0; c < 4; ++c) {
+                            const uint4 w = __ldg(src + c);
+                            const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) {
+                                sv[c * 8 + 2 * e] = __uint_as_float(ww[e] << 16);
+                                sv[c * 8 + 2 * e + 1] = __uint_as_float(ww[e] & 0xFFFF0000u);
+                            }
+                        }
+                    } else {
+#pragma unroll
+                        for (int jj = 0; jj < GROUP; ++jj) sv[jj] = (valid && jj < nv) ? bf2f(srow[v0 + jj]) : 0.0f;
+                    }
+                    float acc[GROUP];
+                    tmem_ld32(tmem + lane_base + buf * TC_BN + gl * GROUP, acc);
+                    if (valid && nv > 0) {
+#pragma unroll
+                        for (int jj = 0; jj < GROUP; ++jj) acc[jj] += sv[jj];
+                        if (p.logits) {
+                            float *dst = p.logits + (size_t)tok * p.V + v0;
+#pragma unroll
+                            for (int jj = 0; jj < GROUP; ++jj)
+                                if (jj < nv) dst[jj] = acc[jj];
+                        }
+                        select_group(sel, acc, v0, nv, invT, seed, (uint32_t)pos, p.offset);
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&sh.tempty[buf]);
+            }
+            sh.st[ew][lane] = sel;
+            const bool stop = epi_bar_or(!ok || *abort);
+            if (!stop) {
+                if (small) {
+                    if (ew == 0 && lane < n) {
+                        Partial a{sh.st[0][lane].best, sh.st[0][lane].idx, sh.st[0][lane].m, sh.st[0][lane].s};
+                        for (int w = 1; w < TC_EPI_WARPS; ++w) {
+                            const Partial b{sh.st[w][lane].best, sh.st[w][lane].idx, sh.st[w][lane].m,
+                                            sh.st[w][lane].s};
+                            merge_partial(a, b, invT > 0.0f);
+                        }
+                        p.part[(size_t)r * p.N + lane] = a;
+                    }
+                } else if (ew < 4 && valid) {
+                    Partial a{sh.st[ew][lane].best, sh.st[ew][lane].idx, sh.st[ew][lane].m, sh.st[ew][lane].s};
+                    const Partial b{sh.st[ew + 4][lane].best, sh.st[ew + 4][lane].idx, sh.st[ew + 4][lane].m,
+                                    sh.st[ew + 4][lane].s};
+                    merge_partial(a, b, invT > 0.0f);
+                    p.part[(size_t)r * p.N + i] = a;
+                }
+            }
+            epi_bar();
+            if (stop) break;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, TC_TMEM_COLS);
+    }
+    if (threadIdx.x == 0 && sh.abort) set_status(p.status, ST_TIMEOUT);
+}
+
+}  // namespace xp

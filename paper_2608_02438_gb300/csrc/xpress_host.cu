@@ -1,0 +1,569 @@
+// xpress_host.cu -- the C ABI (include/xpress.h): argument checks, workspace
+// layout, TMA descriptors, and the CUDA graph that runs Algorithm 1 with its
+// iteration loop on the device (a WHILE conditional node whose condition the
+// reduce kernel updates after every pass).
+#include <cudaTypedefs.h>
+
+#include <cstdint>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <new>
+
+#include "kernels.h"
+#include "xpress.h"
+
+using namespace xp;
+
+namespace {
+
+constexpr int XPRESS_VERSION = 1;
+constexpr int CACHE_SLOTS = 8;
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *f = nullptr;
+        cudaDriverEntryPointQueryResult q{};
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+    });
+    return fn;
+}
+
+// 2-D bf16 tensor [outer][inner], 128-byte swizzle, zero fill out of bounds.
+bool make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t inner, uint64_t outer, uint32_t box_inner,
+                    uint32_t box_outer)
+{
+    auto enc = tensor_map_encoder();
+    if (!enc) return false;
+    cuuint64_t dims[2] = {inner, outer};
+    cuuint64_t strides[1] = {inner * 2};
+    cuuint32_t box[2] = {box_inner, box_outer};
+    cuuint32_t es[2] = {1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+struct GraphEntry {
+    bool used = false;
+    void *ws = nullptr;
+    size_t ws_bytes = 0;
+    int b = 0;
+    bool draft_null = false;
+    cudaGraph_t graph = nullptr;
+    cudaGraphExec_t exec = nullptr;
+    cudaGraphNode_t init_node = nullptr;
+    cudaGraphConditionalHandle handle = 0;
+    dim3 init_grid;
+    uint64_t stamp = 0;
+};
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+struct Layout {
+    size_t status = 0, ctl = 64, params = 256, st = 0, upart = 0, pc = 0, ynew = 0, acttok = 0, zpack = 0,
+           zbuf = 0, part = 0, total = 0;
+    int ksplit = 1, kchunk = 0, S = 1;
+};
+
+}  // namespace
+
+struct xpress_refiner {
+    xpress_weights w{};
+    float *Ep = nullptr;
+    CUtensorMap tmap_wr{};
+    int device = 0;
+    int num_sms = 0;
+    bool use_tc = false;
+    cudaStream_t cs = nullptr;
+    GraphEntry cache[CACHE_SLOTS];
+    uint64_t clock = 0;
+};
+
+namespace {
+
+int read_S(const xpress_refiner *R)
+{
+    if (R->use_tc) {
+        const int nvt = (R->w.V + 255) / 256;
+        return nvt < R->num_sms ? nvt : R->num_sms;
+    }
+    const int ng = (R->w.V + GROUP - 1) / GROUP;
+    return ng < 2 * R->num_sms ? ng : 2 * R->num_sms;
+}
+
+Layout make_layout(const xpress_refiner *R, int b)
+{
+    Layout L;
+    const int B = R->w.B, N = b * B;
+    const size_t esz = R->w.dtype == XPRESS_BF16 ? 2 : 4;
+    size_t o = align256(L.params + sizeof(Params));
+    L.st = o;
+    o = align256(o + (size_t)b * sizeof(SeqState));
+    const int mt = (N + 63) / 64;
+    const int ctas = mt * (RANK / 64) * 2;
+    int ks = (2 * R->num_sms + ctas - 1) / ctas;
+    const int kmax = R->w.H / 256 > 0 ? R->w.H / 256 : 1;
+    ks = ks < 1 ? 1 : (ks > kmax ? kmax : ks);
+    L.kchunk = ((R->w.H + ks - 1) / ks + 15) / 16 * 16;
+    L.ksplit = (R->w.H + L.kchunk - 1) / L.kchunk;
+    L.upart = o;
+    o = align256(o + (size_t)L.ksplit * N * 2 * RANK * 4);
+    L.pc = o;
+    o = align256(o + (size_t)N * RANK * 4);
+    L.ynew = o;
+    o = align256(o + (size_t)N * 4);
+    L.acttok = o;
+    o = align256(o + (size_t)N * 4);
+    L.zpack = o;
+    o = align256(o + (size_t)N * RANK * esz);
+    L.zbuf = o;
+    o = align256(o + (size_t)N * RANK * 4);
+    L.S = read_S(R);
+    L.part = o;
+    o = align256(o + (size_t)L.S * N * sizeof(Partial));
+    L.total = o;
+    return L;
+}
+
+Params make_params(const xpress_refiner *R, const xpress_block_in *in, const xpress_block_out *out, void *ws,
+                   const Layout &L)
+{
+    Params P{};
+    char *w = static_cast<char *>(ws);
+    P.b = in->b;
+    P.B = R->w.B;
+    P.H = R->w.H;
+    P.V = R->w.V;
+    P.N = in->b * R->w.B;
+    P.dtype = R->w.dtype;
+    P.act = R->w.act;
+    P.K_max = in->K_max;
+    P.fixed_K = in->fixed_K ? 1 : 0;
+    P.offset = in->offset;
+    P.S = L.S;
+    P.ksplit = L.ksplit;
+    P.h = in->h;
+    P.s = in->s;
+    P.draft = in->draft;
+    P.anchor = in->anchor;
+    P.temperature = in->temperature;
+    P.seed = reinterpret_cast<const unsigned long long *>(in->seed);
+    P.W_h = R->w.W_h;
+    P.W_g = R->w.W_g;
+    P.W_in = R->w.W_in;
+    P.L = R->w.L;
+    P.W1 = R->w.W1;
+    P.W2 = R->w.W2;
+    P.W_r = R->w.W_r;
+    P.Ep = R->Ep;
+    P.tokens = out->tokens;
+    P.iters = out->iters;
+    P.converged = out->converged;
+    P.lse = out->lse;
+    P.logit_sel = out->logit_sel;
+    P.z_final = out->z_final;
+    P.logits = out->refined_logits;
+    P.status = reinterpret_cast<int32_t *>(w + L.status);
+    P.ctl = reinterpret_cast<int32_t *>(w + L.ctl);
+    P.st = reinterpret_cast<SeqState *>(w + L.st);
+    P.Upart = reinterpret_cast<float *>(w + L.upart);
+    P.Pc = reinterpret_cast<float *>(w + L.pc);
+    P.Ynew = reinterpret_cast<int32_t *>(w + L.ynew);
+    P.act_tok = reinterpret_cast<int32_t *>(w + L.acttok);
+    P.zpack = w + L.zpack;
+    P.zbuf = reinterpret_cast<float *>(w + L.zbuf);
+    P.part = reinterpret_cast<Partial *>(w + L.part);
+    return P;
+}
+
+#define XP_CUDA(call)                                                                                          \
+    do {                                                                                                       \
+        if ((call) != cudaSuccess) {                                                                           \
+            (void)cudaGetLastError();                                                                          \
+            return XPRESS_ERR_CUDA;                                                                            \
+        }                                                                                                      \
+    } while (0)
+
+int set_kernel_attributes()
+{
+    static int rc = -1;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        rc = XPRESS_OK;
+        if (cudaFuncSetAttribute(k_read_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kReadTcSmemBytes) !=
+                cudaSuccess ||
+            cudaFuncSetAttribute(k_mix_mlp, cudaFuncAttributeMaxDynamicSharedMemorySize, MIX_MLP_DYN_SMEM) !=
+                cudaSuccess ||
+            cudaFuncSetAttribute(k_read_simt, cudaFuncAttributeMaxDynamicSharedMemorySize, READ_SIMT_DYN_SMEM) !=
+                cudaSuccess ||
+            cudaFuncSetAttribute(k_pre_mix, cudaFuncAttributeMaxDynamicSharedMemorySize, pre_mix_smem(MAX_B)) !=
+                cudaSuccess) {
+            (void)cudaGetLastError();
+            rc = XPRESS_ERR_CUDA;
+        }
+    });
+    return rc;
+}
+
+void destroy_entry(GraphEntry &e)
+{
+    if (e.exec) cudaGraphExecDestroy(e.exec);
+    if (e.graph) cudaGraphDestroy(e.graph);
+    e = GraphEntry{};
+}
+
+// Builds the per-(workspace, b) graph:
+//   memset(status) -> k_init -> [k_rowmax] -> k_pre_gemm x2 -> k_pre_mix ->
+//   WHILE (cond) { k_mix_mlp -> k_read_{tc,simt} -> k_reduce (updates cond) }
+int build_graph(xpress_refiner *R, GraphEntry &e, const Params &P, const Layout &L, void *ws)
+{
+    const int b = P.b, N = P.N;
+    Params *pdev = reinterpret_cast<Params *>(static_cast<char *>(ws) + L.params);
+    CUtensorMap tmap_z{};
+    if (R->use_tc && !make_tmap_bf16(&tmap_z, P.zpack, RANK, (uint64_t)N, 64, 32)) return XPRESS_ERR_CUDA;
+
+    cudaGraph_t g = nullptr;
+    XP_CUDA(cudaGraphCreate(&g, 0));
+    e.graph = g;
+    cudaMemsetParams ms{};
+    ms.dst = P.status;
+    ms.value = 0;
+    ms.elementSize = 4;
+    ms.width = 1;
+    ms.height = 1;
+    cudaGraphNode_t mnode = nullptr;
+    XP_CUDA(cudaGraphAddMemsetNode(&mnode, g, nullptr, 0, &ms));
+    e.init_grid = dim3((unsigned)((N > b ? N : b) + 255) / 256);
+    XP_CUDA(cudaGraphConditionalHandleCreate(&e.handle, g, 0, cudaGraphCondAssignDefault));
+    cudaGraphConditionalHandle handle = e.handle;
+    {
+        Params Pc = P;
+        void *args[] = {&Pc, &pdev, &handle};
+        cudaKernelNodeParams kp{};
+        kp.func = reinterpret_cast<void *>(k_init);
+        kp.gridDim = e.init_grid;
+        kp.blockDim = dim3(256);
+        kp.kernelParams = args;
+        XP_CUDA(cudaGraphAddKernelNode(&e.init_node, g, &mnode, 1, &kp));
+    }
+
+    cudaStream_t cs = R->cs;
+    XP_CUDA(cudaStreamBeginCaptureToGraph(cs, g, &e.init_node, nullptr, 1, cudaStreamCaptureModeThreadLocal));
+    if (!P.draft) k_rowmax<<<N, 256, 0, cs>>>(pdev);
+    {
+        const dim3 grid(RANK / 64, (N + 63) / 64, L.ksplit);
+        k_pre_gemm<<<grid, 256, 0, cs>>>(pdev, 0, L.kchunk);
+        k_pre_gemm<<<grid, 256, 0, cs>>>(pdev, 1, L.kchunk);
+    }
+    k_pre_mix<<<dim3(b, RANK / 32), 256, pre_mix_smem(P.B), cs>>>(pdev);
+    cudaStreamCaptureStatus cst;
+    const cudaGraphNode_t *deps = nullptr;
+    size_t ndeps = 0;
+    cudaGraph_t capg = nullptr;
+    if (cudaStreamGetCaptureInfo(cs, &cst, nullptr, &capg, &deps, nullptr, &ndeps) != cudaSuccess) {
+        cudaGraph_t tmp;
+        cudaStreamEndCapture(cs, &tmp);
+        (void)cudaGetLastError();
+        return XPRESS_ERR_CUDA;
+    }
+    cudaGraphNodeParams cp{};
+    cp.type = cudaGraphNodeTypeConditional;
+    cp.conditional.handle = handle;
+    cp.conditional.type = cudaGraphCondTypeWhile;
+    cp.conditional.size = 1;
+    cudaGraphNode_t cnode = nullptr;
+    const cudaError_t add_err = cudaGraphAddNode(&cnode, capg, deps, nullptr, ndeps, &cp);
+    cudaError_t upd_err = cudaErrorUnknown;
+    if (add_err == cudaSuccess)
+        upd_err = cudaStreamUpdateCaptureDependencies(cs, &cnode, nullptr, 1, cudaStreamSetCaptureDependencies);
+    cudaGraph_t outer = nullptr;
+    const cudaError_t end_err = cudaStreamEndCapture(cs, &outer);
+    if (add_err != cudaSuccess || upd_err != cudaSuccess || end_err != cudaSuccess) {
+        (void)cudaGetLastError();
+        return XPRESS_ERR_CUDA;
+    }
+    cudaGraph_t body = cp.conditional.phGraph_out[0];
+    XP_CUDA(cudaStreamBeginCaptureToGraph(cs, body, nullptr, nullptr, 0, cudaStreamCaptureModeThreadLocal));
+    k_mix_mlp<<<dim3(8, b), 256, MIX_MLP_DYN_SMEM, cs>>>(pdev);
+    if (R->use_tc)
+        k_read_tc<<<L.S, kReadTcThreads, kReadTcSmemBytes, cs>>>(pdev, R->tmap_wr, tmap_z);
+    else
+        k_read_simt<<<L.S, 256, READ_SIMT_DYN_SMEM, cs>>>(pdev);
+    k_reduce<<<b, 1024, 0, cs>>>(pdev, handle);
+    cudaGraph_t body_out = nullptr;
+    XP_CUDA(cudaStreamEndCapture(cs, &body_out));
+    XP_CUDA(cudaGraphInstantiate(&e.exec, g, 0));
+    return XPRESS_OK;
+}
+
+int check_ws(void *ws, size_t ws_bytes, size_t need)
+{
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255) || ws_bytes < need) return XPRESS_ERR_WORKSPACE;
+    return XPRESS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int xpress_version(void) { return XPRESS_VERSION; }
+
+const char *xpress_status_string(int s)
+{
+    switch (s) {
+    case XPRESS_OK: return "ok";
+    case XPRESS_ERR_INVALID_ARG: return "invalid argument";
+    case XPRESS_ERR_UNSUPPORTED: return "unsupported shape or dtype";
+    case XPRESS_ERR_CUDA: return "CUDA runtime error";
+    case XPRESS_ERR_WORKSPACE: return "workspace missing, too small or misaligned";
+    case XPRESS_ERR_TIMEOUT: return "device wait timed out";
+    case XPRESS_ERR_DEVICE_CHECK: return "device bounds check failed";
+    default: return "unknown status";
+    }
+}
+
+int xpress_refiner_create(const xpress_weights *w, void *stream, xpress_refiner **out)
+{
+    if (!w || !out) return XPRESS_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (!w->W_e || !w->W_h || !w->W_g || !w->W_in || !w->L || !w->W1 || !w->W2 || !w->W_r)
+        return XPRESS_ERR_INVALID_ARG;
+    if (w->r != RANK || w->B < 1 || w->B > MAX_B || w->V < GROUP || (w->V % 8) || w->H < 8 || (w->H % 8) ||
+        (w->dtype != XPRESS_F32 && w->dtype != XPRESS_BF16) || w->act < 0 || w->act > 2)
+        return XPRESS_ERR_UNSUPPORTED;
+    if (set_kernel_attributes() != XPRESS_OK) return XPRESS_ERR_CUDA;
+    xpress_refiner *R = new (std::nothrow) xpress_refiner();
+    if (!R) return XPRESS_ERR_CUDA;
+    R->w = *w;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    int rc = XPRESS_OK;
+    do {
+        if (cudaGetDevice(&R->device) != cudaSuccess ||
+            cudaDeviceGetAttribute(&R->num_sms, cudaDevAttrMultiProcessorCount, R->device) != cudaSuccess) {
+            rc = XPRESS_ERR_CUDA;
+            break;
+        }
+        R->use_tc = w->dtype == XPRESS_BF16;
+        if (R->use_tc && !make_tmap_bf16(&R->tmap_wr, w->W_r, RANK, (uint64_t)w->V, 64, 256)) {
+            rc = XPRESS_ERR_CUDA;
+            break;
+        }
+        if (cudaMalloc(&R->Ep, (size_t)w->V * RANK * sizeof(float)) != cudaSuccess ||
+            cudaStreamCreateWithFlags(&R->cs, cudaStreamNonBlocking) != cudaSuccess) {
+            rc = XPRESS_ERR_CUDA;
+            break;
+        }
+        const dim3 grid(RANK / 64, (w->V + 63) / 64);
+        k_build_ep<<<grid, 256, 0, st>>>(w->W_e, w->W_in, R->Ep, w->V, w->dtype);
+        if (cudaGetLastError() != cudaSuccess || cudaStreamSynchronize(st) != cudaSuccess) rc = XPRESS_ERR_CUDA;
+    } while (0);
+    if (rc != XPRESS_OK) {
+        (void)cudaGetLastError();
+        xpress_refiner_destroy(R);
+        return rc;
+    }
+    *out = R;
+    return XPRESS_OK;
+}
+
+int xpress_refiner_destroy(xpress_refiner *R)
+{
+    if (!R) return XPRESS_ERR_INVALID_ARG;
+    for (auto &e : R->cache) destroy_entry(e);
+    if (R->Ep) cudaFree(R->Ep);
+    if (R->cs) cudaStreamDestroy(R->cs);
+    delete R;
+    return XPRESS_OK;
+}
+
+size_t xpress_refine_workspace_size(const xpress_refiner *R, int b)
+{
+    if (!R || b < 1) return 0;
+    return make_layout(R, b).total;
+}
+
+int xpress_refine_block(const xpress_refiner *Rc, const xpress_block_in *in, const xpress_block_out *out,
+                        void *ws, size_t ws_bytes, void *stream)
+{
+    xpress_refiner *R = const_cast<xpress_refiner *>(Rc);
+    if (!R || !in || !out) return XPRESS_ERR_INVALID_ARG;
+    if (in->b < 1 || in->K_max < 1 || !in->h || !in->s || !in->anchor || !in->temperature || !in->seed ||
+        !out->tokens)
+        return XPRESS_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(in->s) & 15) || (reinterpret_cast<uintptr_t>(in->h) & 15))
+        return XPRESS_ERR_INVALID_ARG;
+    const Layout L = make_layout(R, in->b);
+    if (const int rc = check_ws(ws, ws_bytes, L.total)) return rc;
+    Params P = make_params(R, in, out, ws, L);
+    const bool draft_null = in->draft == nullptr;
+    GraphEntry *hit = nullptr, *victim = &R->cache[0];
+    for (auto &e : R->cache) {
+        if (e.used && e.ws == ws && e.ws_bytes == ws_bytes && e.b == in->b && e.draft_null == draft_null) {
+            hit = &e;
+            break;
+        }
+        if (!e.used) victim = &e;
+        else if (victim->used && e.stamp < victim->stamp) victim = &e;
+    }
+    if (!hit) {
+        destroy_entry(*victim);
+        victim->used = true;
+        victim->ws = ws;
+        victim->ws_bytes = ws_bytes;
+        victim->b = in->b;
+        victim->draft_null = draft_null;
+        if (const int rc = build_graph(R, *victim, P, L, ws)) {
+            destroy_entry(*victim);
+            return rc;
+        }
+        hit = victim;
+    }
+    hit->stamp = ++R->clock;
+    Params *pdev = reinterpret_cast<Params *>(static_cast<char *>(ws) + L.params);
+    cudaGraphConditionalHandle handle = hit->handle;
+    void *args[] = {&P, &pdev, &handle};
+    cudaKernelNodeParams kp{};
+    kp.func = reinterpret_cast<void *>(k_init);
+    kp.gridDim = hit->init_grid;
+    kp.blockDim = dim3(256);
+    kp.kernelParams = args;
+    XP_CUDA(cudaGraphExecKernelNodeSetParams(hit->exec, hit->init_node, &kp));
+    XP_CUDA(cudaGraphLaunch(hit->exec, static_cast<cudaStream_t>(stream)));
+    return XPRESS_OK;
+}
+
+// ------------------------------------------------------------------ accept
+
+namespace {
+struct AcceptLayout {
+    size_t status = 0, rowpart = 256, job = 0, jobf = 0, spart = 0, total = 0;
+    int chunks = 1, chunks2 = 1;
+};
+
+AcceptLayout accept_layout(const xpress_refiner *R, int b)
+{
+    AcceptLayout A;
+    const int rows = b * (R->w.B + 1);
+    int c = (2 * R->num_sms + rows - 1) / rows;
+    A.chunks = c < 1 ? 1 : (c > 64 ? 64 : c);
+    int c2 = (2 * R->num_sms + b - 1) / b;
+    A.chunks2 = c2 < 1 ? 1 : (c2 > 512 ? 512 : c2);
+    size_t o = A.rowpart + align256((size_t)rows * A.chunks * sizeof(Partial));
+    A.job = o;
+    o += align256((size_t)b * 4);
+    A.jobf = o;
+    o += align256((size_t)b * 4);
+    A.spart = o;
+    o += align256((size_t)b * A.chunks2 * sizeof(Partial));
+    A.total = o;
+    return A;
+}
+}  // namespace
+
+size_t xpress_accept_workspace_size(const xpress_refiner *R, int b)
+{
+    if (!R || b < 1) return 0;
+    return accept_layout(R, b).total;
+}
+
+int xpress_accept(const xpress_refiner *R, const xpress_accept_in *in, int32_t *accept_len, int32_t *out_tokens,
+                  void *ws, size_t ws_bytes, void *stream)
+{
+    if (!R || !in || !accept_len || !out_tokens) return XPRESS_ERR_INVALID_ARG;
+    if (in->b < 1 || !in->target || !in->tokens || !in->temperature || !in->seed || !in->s || !in->lse ||
+        !in->logit_sel || !in->z_final)
+        return XPRESS_ERR_INVALID_ARG;
+    const AcceptLayout A = accept_layout(R, in->b);
+    if (const int rc = check_ws(ws, ws_bytes, A.total)) return rc;
+    char *w = static_cast<char *>(ws);
+    AcceptParams P{};
+    P.b = in->b;
+    P.B = R->w.B;
+    P.V = R->w.V;
+    P.dtype = R->w.dtype;
+    P.target = in->target;
+    P.s = in->s;
+    P.tokens = in->tokens;
+    P.lse = in->lse;
+    P.logit_sel = in->logit_sel;
+    P.z_final = in->z_final;
+    P.temperature = in->temperature;
+    P.seed = reinterpret_cast<const unsigned long long *>(in->seed);
+    P.offset = in->offset;
+    P.W_r = R->w.W_r;
+    P.accept_len = accept_len;
+    P.out_tokens = out_tokens;
+    P.status = reinterpret_cast<int32_t *>(w + A.status);
+    P.rowpart = reinterpret_cast<Partial *>(w + A.rowpart);
+    P.job = reinterpret_cast<int32_t *>(w + A.job);
+    P.jobf = reinterpret_cast<float *>(w + A.jobf);
+    P.spart = reinterpret_cast<Partial *>(w + A.spart);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    XP_CUDA(cudaMemsetAsync(P.status, 0, 4, st));
+    k_acc_rows<<<dim3(in->b * (R->w.B + 1), A.chunks), 256, 0, st>>>(P);
+    k_acc_decide<<<(in->b + 127) / 128, 128, 0, st>>>(P, A.chunks);
+    k_acc_sample<<<dim3(in->b, A.chunks2), 256, 0, st>>>(P);
+    k_acc_finish<<<(in->b + 127) / 128, 128, 0, st>>>(P, A.chunks2);
+    XP_CUDA(cudaGetLastError());
+    return XPRESS_OK;
+}
+
+int xpress_get_device_status(void *ws, void *stream, int32_t *status_out)
+{
+    if (!ws || !status_out) return XPRESS_ERR_INVALID_ARG;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    int32_t v = 0;
+    XP_CUDA(cudaStreamSynchronize(st));
+    XP_CUDA(cudaMemcpy(&v, ws, 4, cudaMemcpyDeviceToHost));
+    XP_CUDA(cudaMemset(ws, 0, 4));
+    *status_out = (v & ST_TIMEOUT) ? XPRESS_ERR_TIMEOUT : (v & ST_BOUNDS) ? XPRESS_ERR_DEVICE_CHECK : XPRESS_OK;
+    return XPRESS_OK;
+}
+
+int xpress_profile_read_prepare(const xpress_refiner *R, void *ws, int b, int n_tokens, void *stream)
+{
+    if (!R || b < 1 || n_tokens < 1 || n_tokens > b * R->w.B) return XPRESS_ERR_INVALID_ARG;
+    const Layout L = make_layout(R, b);
+    if (const int rc = check_ws(ws, L.total, L.total)) return rc;
+    char *w = static_cast<char *>(ws);
+    k_prof_prepare<<<(n_tokens + 255) / 256, 256, 0, static_cast<cudaStream_t>(stream)>>>(
+        reinterpret_cast<int32_t *>(w + L.ctl), reinterpret_cast<int32_t *>(w + L.acttok), n_tokens);
+    XP_CUDA(cudaGetLastError());
+    return XPRESS_OK;
+}
+
+int xpress_profile_read(const xpress_refiner *R, void *ws, int b, void *stream)
+{
+    if (!R || b < 1) return XPRESS_ERR_INVALID_ARG;
+    const Layout L = make_layout(R, b);
+    if (const int rc = check_ws(ws, L.total, L.total)) return rc;
+    char *w = static_cast<char *>(ws);
+    const Params *pdev = reinterpret_cast<const Params *>(w + L.params);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (R->use_tc) {
+        CUtensorMap tmap_z{};
+        if (!make_tmap_bf16(&tmap_z, w + L.zpack, RANK, (uint64_t)b * R->w.B, 64, 32)) return XPRESS_ERR_CUDA;
+        k_read_tc<<<L.S, kReadTcThreads, kReadTcSmemBytes, st>>>(pdev, R->tmap_wr, tmap_z);
+    } else {
+        k_read_simt<<<L.S, 256, READ_SIMT_DYN_SMEM, st>>>(pdev);
+    }
+    XP_CUDA(cudaGetLastError());
+    return XPRESS_OK;
+}
+
+int xpress_get_pass_count(void *ws, void *stream, int32_t *passes_out)
+{
+    if (!ws || !passes_out) return XPRESS_ERR_INVALID_ARG;
+    XP_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+    XP_CUDA(cudaMemcpy(passes_out, static_cast<char *>(ws) + 64 + CTL_PASS * 4, 4, cudaMemcpyDeviceToHost));
+    return XPRESS_OK;
+}
+
+}  // extern "C"

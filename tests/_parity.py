@@ -1,0 +1,83 @@
+"""Shared helpers for the GPU-vs-oracle parity tests.
+
+Parity rule: token outputs, pass counts, convergence flags and accept lengths
+must match bit-exactly.  A mismatching block is excused only at a documented
+near-tie: the oracle's smallest top-2 decision margin on that block's
+trajectory is below NEAR_TIE (1e-3 in the units of the decision: logits, or
+logits / T plus Gumbel noise); at most max(1, 1%) of the blocks may be excused.
+Float outputs: refined logits within 2e-2 (bf16) or 1e-4 (fp32) absolute.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+import oracle as O
+from paper_2608_02438_gb300 import workloads as W
+
+NEAR_TIE = 1e-3
+LOGIT_TOL = {W.BF16: 2e-2, W.F32: 1e-4}
+Z_TOL = {W.BF16: 5e-3, W.F32: 1e-5}
+
+
+def oracle_model(cfg, weights, act=O.SILU):
+    return O.Model(weights, cfg.H, cfg.V, cfg.r, cfg.B, O.BF16 if cfg.dtype == W.BF16 else O.F32, act)
+
+
+def device_inputs(refiner_dtype, inp, sel=None):
+    """Torch device tensors for the sequences `sel` (default: all)."""
+    import torch
+    from paper_2608_02438_gb300 import binding as X
+    idx = np.arange(inp["h"].shape[0]) if sel is None else np.asarray(sel)
+    d = dict(
+        h=X.to_device(inp["h"][idx], refiner_dtype), s=X.to_device(inp["s"][idx], refiner_dtype),
+        target=X.to_device(inp["target"][idx], refiner_dtype),
+        draft=torch.from_numpy(np.ascontiguousarray(inp["draft"][idx])).cuda(),
+        anchor=torch.from_numpy(np.ascontiguousarray(inp["anchor"][idx])).cuda(),
+        temperature=torch.from_numpy(np.ascontiguousarray(inp["temperature"][idx])).cuda(),
+        seed=torch.from_numpy(np.ascontiguousarray(inp["seed"][idx]).view(np.int64)).cuda())
+    return d
+
+
+def run_oracle(m, inp, i, K_max, fixed_K=False):
+    return O.jacobi(m, inp["h"][i], inp["s"][i], int(inp["anchor"][i]), inp["draft"][i],
+                    float(inp["temperature"][i]), int(inp["seed"][i]), inp["offset"], K_max, fixed_K,
+                    trajectory=True)
+
+
+def compare_blocks(gpu: dict, orc: dict, seqs, dtype, check_logits=None, m=None, inp=None):
+    """Returns (n_excused, report lines); raises AssertionError on a real mismatch."""
+    excused, lines = 0, []
+    for j, i in enumerate(seqs):
+        o = orc[i]
+        tok = gpu["tokens"][j]
+        same = (np.array_equal(tok, o["tokens"]) and int(gpu["iters"][j]) == o["iters"]
+                and int(gpu["converged"][j]) == o["converged"])
+        if not same:
+            msg = (f"block {i}: gpu tokens {tok.tolist()} iters {int(gpu['iters'][j])} conv "
+                   f"{int(gpu['converged'][j])} | oracle {o['tokens'].tolist()} iters {o['iters']} conv "
+                   f"{o['converged']} min margin {o['min_margin']:.3g}")
+            if o["min_margin"] < NEAR_TIE:
+                excused += 1
+                lines.append("excused near-tie: " + msg)
+                continue
+            raise AssertionError(msg)
+        # float outputs of the last pass
+        zt = Z_TOL[dtype]
+        np.testing.assert_allclose(gpu["z_final"][j], o["z_final"], atol=zt, rtol=zt,
+                                   err_msg=f"z_final block {i}")
+        T = float(inp["temperature"][i]) if inp is not None else 0.0
+        lt = LOGIT_TOL[dtype]
+        np.testing.assert_allclose(gpu["logit_sel"][j], o["sel"], atol=lt * (1.0 / T if T > 0 else 1.0),
+                                   err_msg=f"logit_sel block {i}")
+        if T > 0:
+            np.testing.assert_allclose(gpu["lse"][j], o["lse"], atol=1e-3 * max(1.0, 1.0 / T),
+                                       err_msg=f"lse block {i}")
+        if check_logits is not None and m is not None:
+            traj = o["trajectory"]
+            x = np.concatenate([[int(inp["anchor"][i])], traj[o["iters"] - 1, :-1]]).astype(np.int32)
+            ell, _, _ = O.forward(m, inp["h"][i], inp["s"][i], x)
+            err = np.abs(check_logits[j].astype(np.float64) - ell).max()
+            assert err <= lt, f"refined logits block {i}: max abs err {err:.3g} > {lt}"
+    limit = max(1, int(0.01 * len(seqs)))
+    assert excused <= limit, f"{excused} excused blocks > {limit}:\n" + "\n".join(lines)
+    return excused, lines
