@@ -18,21 +18,59 @@
 
 namespace xp {
 
+// 8 consecutive values of a row as fp32 (zeros past `n`).
+__device__ __forceinline__ void load8(float (&x)[8], const void *base, int dtype, size_t i, int n)
+{
+    if (n >= 8) {
+        if (dtype) {
+            const uint4 w = __ldg(reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(base) + i));
+            const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                x[2 * q] = __uint_as_float(ww[q] << 16);
+                x[2 * q + 1] = __uint_as_float(ww[q] & 0xFFFF0000u);
+            }
+        } else {
+            const float4 a = __ldg(reinterpret_cast<const float4 *>(static_cast<const float *>(base) + i));
+            const float4 b = __ldg(reinterpret_cast<const float4 *>(static_cast<const float *>(base) + i + 4));
+            x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w; x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+        }
+        return;
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) x[j] = j < n ? ld_any(base, dtype, i + j) : 0.0f;
+}
+
+// grid (b * (B + 1), chunks); chunk boundaries are multiples of 8 ids.
 __global__ void __launch_bounds__(256) k_acc_rows(AcceptParams p)
 {
     const int row = blockIdx.x;                   // seq * (B + 1) + k
     const int seq = row / (p.B + 1);
     const int chunks = gridDim.y, c = blockIdx.y;
-    const int v0 = (int)((long long)p.V * c / chunks), v1 = (int)((long long)p.V * (c + 1) / chunks);
+    const int V8 = (p.V + 7) / 8;
+    const int v0 = 8 * (int)((long long)V8 * c / chunks), v1 = min(p.V, 8 * (int)((long long)V8 * (c + 1) / chunks));
     const float T = p.temperature[seq];
     const float invT = T > 0.0f ? 1.0f / T : 0.0f;
     Partial a{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
-    for (int v = v0 + threadIdx.x; v < v1; v += blockDim.x) {
-        const float x = ld_any(p.target, p.dtype, (size_t)row * p.V + v);
+    const size_t base = (size_t)row * p.V;
+    for (int v = v0 + 8 * threadIdx.x; v < v1; v += 8 * blockDim.x) {
+        float x[8];
+        const int nv = min(8, v1 - v);
+        load8(x, p.target, p.dtype, base + v, nv);
         if (invT <= 0.0f) {
-            merge_argmax(a.best, a.idx, x, v);
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+                if (j < nv && x[j] > a.best) { a.best = x[j]; a.idx = v + j; }
         } else {
-            merge_lse(a.m, a.s, x * invT, 1.0f);
+            float mx = -INFINITY;
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+                if (j < nv) mx = fmaxf(mx, x[j] * invT);
+            float sum = 0.0f;
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+                if (j < nv) sum += __expf(x[j] * invT - mx);
+            merge_lse(a.m, a.s, mx, sum);
         }
     }
     __shared__ Partial sp[256];
@@ -49,51 +87,57 @@ __global__ void __launch_bounds__(256) k_acc_rows(AcceptParams p)
     if (threadIdx.x == 0) p.rowpart[(size_t)row * chunks + c] = sp[0];
 }
 
-__device__ Partial combine_row(const AcceptParams &p, int row, int chunks, bool sampling)
+// one warp per block (sequence): lane k combines the chunk partials of target
+// row k and takes the accept decision of position k; a ballot finds the first
+// position that is not accepted.
+__global__ void __launch_bounds__(32) k_acc_decide(AcceptParams p, int chunks)
 {
-    Partial a{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
-    for (int c = 0; c < chunks; ++c) merge_partial(a, p.rowpart[(size_t)row * chunks + c], sampling);
-    return a;
-}
-
-// one thread per block (sequence)
-__global__ void k_acc_decide(AcceptParams p, int chunks)
-{
-    const int seq = blockIdx.x * blockDim.x + threadIdx.x;
-    if (seq >= p.b) return;
+    const int seq = blockIdx.x, lane = threadIdx.x;
     const int B = p.B;
     const float T = p.temperature[seq];
-    int32_t *out = p.out_tokens + (size_t)seq * (B + 1);
-    for (int k = 0; k <= B; ++k) out[k] = -1;
-    int n = 0;
-    if (T <= 0.0f) {
-        for (;;) {
-            const Partial a = combine_row(p, seq * (B + 1) + n, chunks, false);
-            if (n < B && p.tokens[(size_t)seq * B + n] == a.idx) { out[n] = a.idx; ++n; continue; }
-            out[n] = a.idx;
-            break;
-        }
-        p.job[seq] = -1;
-    } else {
-        const float invT = 1.0f / T;
-        int job = B;
-        for (; n < B; ++n) {
-            const int row = seq * (B + 1) + n;
-            const Partial a = combine_row(p, row, chunks, true);
-            const float lse_p = a.m + logf(a.s);
-            int y = p.tokens[(size_t)seq * B + n];
-            if (y < 0 || y >= p.V) { set_status(p.status, ST_BOUNDS); y = 0; }
-            const float p_y = expf(ld_any(p.target, p.dtype, (size_t)row * p.V + y) * invT - lse_p);
-            const float q_y = expf(p.logit_sel[(size_t)seq * B + n] - p.lse[(size_t)seq * B + n]);
-            const float u = uniform01(p.seed[seq], 0u, (uint32_t)n, STREAM_ACCEPT, p.offset);
-            if (u * q_y < p_y) { out[n] = y; continue; }
-            job = n;
-            p.jobf[seq] = lse_p;
-            break;
-        }
-        p.job[seq] = job;
+    const bool sampling = T > 0.0f;
+    const float invT = sampling ? 1.0f / T : 0.0f;
+    __shared__ Partial rows[MAX_B + 1];
+    for (int k = lane; k <= B; k += 32) {
+        Partial a{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
+        const size_t r = (size_t)seq * (B + 1) + k;
+#pragma unroll 4
+        for (int c = 0; c < chunks; ++c) merge_partial(a, p.rowpart[r * chunks + c], sampling);
+        rows[k] = a;
     }
-    p.accept_len[seq] = n;
+    __syncwarp();
+    int y = -1;
+    bool ok = false;
+    float lse_p = 0.0f;
+    if (lane < B) {
+        y = p.tokens[(size_t)seq * B + lane];
+        if (y < 0 || y >= p.V) { set_status(p.status, ST_BOUNDS); y = 0; }
+        if (!sampling) {
+            ok = y == rows[lane].idx;
+        } else {
+            const int row = seq * (B + 1) + lane;
+            lse_p = rows[lane].m + logf(rows[lane].s);
+            const float p_y = expf(ld_any(p.target, p.dtype, (size_t)row * p.V + y) * invT - lse_p);
+            const float q_y = expf(p.logit_sel[(size_t)seq * B + lane] - p.lse[(size_t)seq * B + lane]);
+            const float u = uniform01(p.seed[seq], 0u, (uint32_t)lane, STREAM_ACCEPT, p.offset);
+            ok = u * q_y < p_y;
+        }
+    }
+    const unsigned rejected = __ballot_sync(0xffffffffu, lane < B && !ok);
+    const int n = rejected ? __ffs(rejected) - 1 : B;
+    int32_t *out = p.out_tokens + (size_t)seq * (B + 1);
+    for (int k = lane; k <= B; k += 32) out[k] = k < n ? p.tokens[(size_t)seq * B + k] : -1;
+    __syncwarp();
+    if (lane == 0) {
+        if (!sampling) {
+            out[n] = rows[n].idx;
+            p.job[seq] = -1;
+        } else {
+            p.job[seq] = n;
+            if (n < B) p.jobf[seq] = rows[n].m + logf(rows[n].s);
+        }
+        p.accept_len[seq] = n;
+    }
 }
 
 // grid (b, chunks), 256 threads.  Writes two argmax partials per chunk: the

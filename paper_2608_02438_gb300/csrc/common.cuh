@@ -60,6 +60,7 @@ struct Params {
     int K_max, fixed_K;
     uint32_t offset;
     int S;                       // vocabulary ranges of the Read kernel
+    int use_graph;               // 1: the pass loop is a graph WHILE node
     int ksplit;                  // split-K factor of the hidden projection
     // inputs (caller-owned)
     const void *h, *s;

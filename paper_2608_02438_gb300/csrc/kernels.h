@@ -25,6 +25,7 @@ struct AcceptParams {
 __global__ void k_init(Params pin, Params *pdev, cudaGraphConditionalHandle handle);
 __global__ void k_rowmax(const Params *pp);
 __global__ void k_pre_gemm(const Params *pp, int which, int kchunk);
+__global__ void k_pre_gemv(const Params *pp, int kslice);
 __global__ void k_pre_mix(const Params *pp);
 __global__ void k_mix_mlp(const Params *pp);
 __global__ void k_read_simt(const Params *pp);
@@ -44,8 +45,15 @@ __global__ void k_acc_decide(AcceptParams p, int chunks);
 __global__ void k_acc_sample(AcceptParams p);
 __global__ void k_acc_finish(AcceptParams p, int chunks);
 
-constexpr int MIX_MLP_DYN_SMEM = (MAX_B * RANK + MAX_B * 2 * RANK) * 4;
+// fp32: c and sigma(W_1 c) of up to 32 tokens in fp32; bf16: the same as
+// bf16 tensor-core operands plus this CTA's share of sigma(W_1 c)
+constexpr int MIX_MLP_DYN_SMEM_MAX = (MAX_B * 3 * RANK) * 4;
+inline int mix_mlp_smem(int dtype)
+{
+    return dtype ? (32 * (RANK + 8) + 32 * (2 * RANK + 8) + 32 * (64 + 8)) * 2 : MIX_MLP_DYN_SMEM_MAX;
+}
+constexpr int GEMV_SMEM = 128 * 1024;
 constexpr int READ_SIMT_DYN_SMEM = (32 * (RANK + 1) + 8 * 32 * 33) * 4;
-inline int pre_mix_smem(int B) { return (B * 2 * RANK + RANK + B * 32) * 4; }
+inline int pre_mix_smem(int B) { return (B * 2 * RANK + RANK + 32 * (2 * RANK + 1) + B * 32) * 4; }
 
 }  // namespace xp

@@ -72,6 +72,28 @@ __device__ __forceinline__ bool epi_bar_or(bool pred)
     return res != 0;
 }
 
+// s[v0 .. v0 + 31] of one token as raw bf16 pairs (zeros past V or for an
+// invalid thread).
+__device__ __forceinline__ void load_s_group(uint4 (&r)[4], const uint16_t *row, int v0, int V, bool valid)
+{
+    if (valid && v0 + GROUP <= V) {
+        const uint4 *src = reinterpret_cast<const uint4 *>(row + v0);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) r[c] = __ldg(src + c);
+        return;
+    }
+    uint32_t w[16];
+#pragma unroll
+    for (int q = 0; q < 16; ++q) {
+        const int j = v0 + 2 * q;
+        const uint32_t lo = (valid && j < V) ? row[j] : 0u;
+        const uint32_t hi = (valid && j + 1 < V) ? row[j + 1] : 0u;
+        w[q] = lo | (hi << 16);
+    }
+#pragma unroll
+    for (int c = 0; c < 4; ++c) r[c] = make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
+}
+
 __global__ void __launch_bounds__(TC_THREADS, 1)
     k_read_tc(const Params *__restrict__ pp, const __grid_constant__ CUtensorMap tmap_wr,
               const __grid_constant__ CUtensorMap tmap_z)
@@ -201,47 +223,52 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             const uint16_t *srow = static_cast<const uint16_t *>(p.s) + (size_t)tok * p.V;
             SelState sel;
             sel.init();
-            for (int vt = vt0; vt < vt1; ++vt, ++t) {
+            // (tile, group) work items in order; s of item i + 1 is loaded
+            // while item i is processed
+            const int items = (vt1 - vt0) * g_count;
+            uint4 cur[4], nxt[4];
+            load_s_group(cur, srow, vt0 * TC_BN + g_first * GROUP, p.V, valid);
+            for (int it = 0; it < items; ++it) {
+                const int vt = vt0 + it / g_count, gl = g_first + it % g_count;
                 const int buf = t & 1;
-                if (!mbar_wait(&sh.tfull[buf], (t >> 1) & 1, abort)) { ok = false; break; }
-                tc_fence_after();
-                for (int gl = g_first; gl < g_first + g_count; ++gl) {
-                    const int v0 = vt * TC_BN + gl * GROUP;
-                    const int nv = min(GROUP, p.V - v0);
-                    float sv[GROUP];
-                    if (valid && nv == GROUP) {
-                        const uint4 *src = reinterpret_cast<const uint4 *>(srow + v0);
-#pragma unroll
-                        for (int c = 0; c < 4; ++c) {
-                            const uint4 w = __ldg(src + c);
-                            const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-                            for (int e = 0; e < 4; ++e) {
-                                sv[c * 8 + 2 * e] = __uint_as_float(ww[e] << 16);
-                                sv[c * 8 + 2 * e + 1] = __uint_as_float(ww[e] & 0xFFFF0000u);
-                            }
-                        }
-                    } else {
-#pragma unroll
-                        for (int jj = 0; jj < GROUP; ++jj) sv[jj] = (valid && jj < nv) ? bf2f(srow[v0 + jj]) : 0.0f;
-                    }
-                    float acc[GROUP];
-                    tmem_ld32(tmem + lane_base + buf * TC_BN + gl * GROUP, acc);
-                    if (valid && nv > 0) {
-#pragma unroll
-                        for (int jj = 0; jj < GROUP; ++jj) acc[jj] += sv[jj];
-                        if (p.logits) {
-                            float *dst = p.logits + (size_t)tok * p.V + v0;
-#pragma unroll
-                            for (int jj = 0; jj < GROUP; ++jj)
-                                if (jj < nv) dst[jj] = acc[jj];
-                        }
-                        select_group(sel, acc, v0, nv, invT, seed, (uint32_t)pos, p.offset);
-                    }
+                if (gl == g_first) {
+                    if (!mbar_wait(&sh.tfull[buf], (t >> 1) & 1, abort)) { ok = false; break; }
+                    tc_fence_after();
                 }
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&sh.tempty[buf]);
+                if (it + 1 < items) {
+                    const int vn = vt0 + (it + 1) / g_count, gn = g_first + (it + 1) % g_count;
+                    load_s_group(nxt, srow, vn * TC_BN + gn * GROUP, p.V, valid);
+                }
+                const int v0 = vt * TC_BN + gl * GROUP;
+                const int nv = min(GROUP, p.V - v0);
+                float acc[GROUP];
+                tmem_ld32(tmem + lane_base + buf * TC_BN + gl * GROUP, acc);
+                if (valid && nv > 0) {
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) {
+                        const uint32_t ww[4] = {cur[c].x, cur[c].y, cur[c].z, cur[c].w};
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            acc[c * 8 + 2 * q] += __uint_as_float(ww[q] << 16);
+                            acc[c * 8 + 2 * q + 1] += __uint_as_float(ww[q] & 0xFFFF0000u);
+                        }
+                    }
+                    if (p.logits) {
+                        float *dst = p.logits + (size_t)tok * p.V + v0;
+#pragma unroll
+                        for (int jj = 0; jj < GROUP; ++jj)
+                            if (jj < nv) dst[jj] = acc[jj];
+                    }
+                    select_group(sel, acc, v0, nv, invT, seed, (uint32_t)pos, p.offset);
+                }
+#pragma unroll
+                for (int c = 0; c < 4; ++c) cur[c] = nxt[c];
+                if (gl == g_first + g_count - 1) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&sh.tempty[buf]);
+                    ++t;
+                }
             }
             sh.st[ew][lane] = sel;
             const bool stop = epi_bar_or(!ok || *abort);

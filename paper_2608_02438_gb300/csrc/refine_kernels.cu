@@ -39,7 +39,7 @@ __global__ void k_init(Params pin, Params *pdev, cudaGraphConditionalHandle hand
         p.ctl[CTL_NACT] = p.N;
         p.ctl[CTL_DONE] = 0;
         p.ctl[CTL_PASS] = 0;
-        cudaGraphSetConditional(handle, 1u);
+        if (p.use_graph) cudaGraphSetConditional(handle, 1u);
     }
     if (t < p.N) {
         p.act_tok[t] = t;
@@ -151,6 +151,71 @@ __global__ void __launch_bounds__(256) k_pre_gemm(const Params *__restrict__ pp,
                      RANK, kb, ke, blockIdx.y * 64, blockIdx.x * 64);
 }
 
+// Sum over the 32 lanes of v[0..31] (one value per token), scattered so that
+// lane t ends with the total of token t in v[0] (recursive halving, 31 shuffles).
+__device__ __forceinline__ float reduce_scatter32(float (&v)[32], int lane)
+{
+#pragma unroll
+    for (int s = 16; s >= 1; s >>= 1) {
+        const bool upper = (lane & s) != 0;
+#pragma unroll
+        for (int j = 0; j < s; ++j) {
+            const float send = upper ? v[j] : v[j + s];
+            const float keep = upper ? v[j + s] : v[j];
+            v[j] = keep + __shfl_xor_sync(0xffffffffu, send, s);
+        }
+    }
+    return v[0];
+}
+
+__device__ __forceinline__ void bf16x8_to_f32(const uint4 &w, float (&x)[8])
+{
+    const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        x[2 * q] = __uint_as_float(ww[q] << 16);
+        x[2 * q + 1] = __uint_as_float(ww[q] & 0xFFFF0000u);
+    }
+}
+
+// bf16, at most 32 tokens: Upart[z][t][o] = h[t][K-slice z] . [W_h; W_g][o][K-slice z].
+// grid (2r / 8, KS), 256 threads: warp w owns output row o = 8 x + w; the
+// CTA stages its K-slice of every token's h in shared memory ([N][kslice]).
+__global__ void __launch_bounds__(256) k_pre_gemv(const Params *__restrict__ pp, int kslice)
+{
+    const Params &p = *pp;
+    extern __shared__ __align__(16) uint16_t hs[];
+    const int N = p.N, H = p.H, warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const int kb = blockIdx.y * kslice, ke = min(H, kb + kslice), kl = ke - kb;
+    const uint16_t *h = static_cast<const uint16_t *>(p.h);
+    for (int i = threadIdx.x; i < N * (kl / 8); i += blockDim.x) {
+        const int t = i / (kl / 8), c = i % (kl / 8);
+        reinterpret_cast<uint4 *>(hs + (size_t)t * kslice)[c] =
+            __ldg(reinterpret_cast<const uint4 *>(h + (size_t)t * H + kb) + c);
+    }
+    const int o = blockIdx.x * 8 + warp;
+    const uint16_t *W = static_cast<const uint16_t *>(o < RANK ? p.W_h : p.W_g) + (size_t)(o % RANK) * H + kb;
+    float v[32];
+#pragma unroll
+    for (int t = 0; t < 32; ++t) v[t] = 0.0f;
+    __syncthreads();
+    for (int k0 = 8 * lane; k0 < kl; k0 += 256) {
+        float w[8];
+        bf16x8_to_f32(__ldg(reinterpret_cast<const uint4 *>(W + k0)), w);
+#pragma unroll
+        for (int t = 0; t < 32; ++t) {
+            if (t < N) {
+                float x[8];
+                bf16x8_to_f32(*reinterpret_cast<const uint4 *>(hs + (size_t)t * kslice + k0), x);
+#pragma unroll
+                for (int j = 0; j < 8; ++j) v[t] = fmaf(w[j], x[j], v[t]);
+            }
+        }
+    }
+    const float sum = reduce_scatter32(v, lane);
+    if (lane < N) p.Upart[((size_t)blockIdx.y * N + lane) * 2 * RANK + o] = sum;
+}
+
 // Folded embedding E'[v][d] = sum_e W_in[d][2r + e] W_e[v][e] (Sec. 4.1: Fuse
 // is linear, so the token slot folds into one table).  grid (r/64, ceil(V/64)).
 __global__ void __launch_bounds__(256) k_build_ep(const void *W_e, const void *W_in, float *Ep, int V, int dtype)
@@ -165,21 +230,56 @@ __global__ void __launch_bounds__(256) k_build_ep(const void *W_e, const void *W
 
 // -------------------------------------------------------------- k_pre_mix
 
-// grid (b, RANK / 32): block s, channels [32 y, 32 y + 32).
+// grid (b, RANK / 32): block s, channels [32 y, 32 y + 32).  Dynamic shared
+// memory: U [B][2r], u_g [r], W_in rows [32][2r + 1], P [B][32].
 __global__ void __launch_bounds__(256) k_pre_mix(const Params *__restrict__ pp)
 {
     const Params &p = *pp;
     extern __shared__ float sm[];
     const int B = p.B, s = blockIdx.x, d0 = blockIdx.y * 32;
-    float *U = sm;                     // [B][2r]   W_h h_k | W_g h_k
-    float *ug = U + B * 2 * RANK;      // [r]       W_g g
-    float *P = ug + RANK;              // [B][32]   P for this channel slice
+    float *U = sm;                         // [B][2r]   W_h h_k | W_g h_k
+    float *ug = U + B * 2 * RANK;          // [r]       W_g g
+    float *Ws = ug + RANK;                 // [32][2r + 1]  W_in[d0 + dd][0:2r]
+    float *P = Ws + 32 * (2 * RANK + 1);   // [B][32]   P for this channel slice
     const size_t tok0 = (size_t)s * B;
-    for (int i = threadIdx.x; i < B * 2 * RANK; i += blockDim.x) {
-        const int k = i / (2 * RANK), o = i % (2 * RANK);
-        float acc = 0.0f;
-        for (int z = 0; z < p.ksplit; ++z) acc += p.Upart[((size_t)z * p.N + tok0 + k) * 2 * RANK + o];
-        U[i] = acc;
+    if (p.dtype) {
+        for (int i = threadIdx.x; i < 32 * 2 * RANK / 8; i += blockDim.x) {
+            const int dd = i / (2 * RANK / 8), c = i % (2 * RANK / 8);
+            float x[8];
+            bf16x8_to_f32(__ldg(reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.W_in) +
+                                                                 (size_t)(d0 + dd) * 3 * RANK) + c), x);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) Ws[dd * (2 * RANK + 1) + 8 * c + j] = x[j];
+        }
+    } else {
+        for (int i = threadIdx.x; i < 32 * 2 * RANK; i += blockDim.x) {
+            const int dd = i / (2 * RANK), e = i % (2 * RANK);
+            Ws[dd * (2 * RANK + 1) + e] = ld_any(p.W_in, p.dtype, (size_t)(d0 + dd) * 3 * RANK + e);
+        }
+    }
+    {
+        // U = sum of the K-slice partials; each thread issues its loads as one batch
+        const int ks = p.ksplit, NN = p.N;
+        const float *up = p.Upart + tok0 * 2 * RANK;
+        for (int i0 = 0; i0 < B * 2 * RANK; i0 += 8 * 256) {
+            float v[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const int i = i0 + q * 256 + threadIdx.x;
+                v[q] = i < B * 2 * RANK ? up[i] : 0.0f;
+            }
+            for (int z = 1; z < ks; ++z)
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    const int i = i0 + q * 256 + threadIdx.x;
+                    if (i < B * 2 * RANK) v[q] += up[(size_t)z * NN * 2 * RANK + i];
+                }
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const int i = i0 + q * 256 + threadIdx.x;
+                if (i < B * 2 * RANK) U[i] = v[q];
+            }
+        }
     }
     __syncthreads();
     for (int e = threadIdx.x; e < RANK; e += blockDim.x) {
@@ -189,20 +289,30 @@ __global__ void __launch_bounds__(256) k_pre_mix(const Params *__restrict__ pp)
     }
     __syncthreads();
     // P[k][d] = sum_e W_in[d][e] u_h,k[e] + sum_e W_in[d][r + e] u_g[e]
-    for (int i = threadIdx.x; i < B * 32; i += blockDim.x) {
-        const int k = i / 32, dd = i % 32, d = d0 + dd;
-        float acc = 0.0f;
-        const size_t wrow = (size_t)d * 3 * RANK;
-        for (int e = 0; e < RANK; ++e) acc = fmaf(ld_any(p.W_in, p.dtype, wrow + e), U[k * 2 * RANK + e], acc);
-        for (int e = 0; e < RANK; ++e) acc = fmaf(ld_any(p.W_in, p.dtype, wrow + RANK + e), ug[e], acc);
-        P[k * 32 + dd] = acc;
+    {
+        const int dd = threadIdx.x % 32, kg = threadIdx.x / 32;
+        const float *w = Ws + dd * (2 * RANK + 1);
+        float gpart = 0.0f;
+        for (int e = 0; e < RANK; ++e) gpart = fmaf(w[RANK + e], ug[e], gpart);
+        for (int k = kg; k < B; k += 8) {
+            float acc = gpart;
+            const float *u = U + k * 2 * RANK;
+            for (int e = 0; e < RANK; ++e) acc = fmaf(w[e], u[e], acc);
+            P[k * 32 + dd] = acc;
+        }
     }
     __syncthreads();
     // Pc = (I + L) P, channel by channel (Eq. mix)
     for (int i = threadIdx.x; i < B * 32; i += blockDim.x) {
         const int k = i / 32, dd = i % 32, d = d0 + dd;
+        float lrow[MAX_B];
+        const size_t lb = ((size_t)d * B + k) * B;
+#pragma unroll
+        for (int j = 0; j < MAX_B; ++j) lrow[j] = j < k ? ld_any(p.L, p.dtype, lb + j) : 0.0f;
         float acc = P[k * 32 + dd];
-        for (int j = 0; j < k; ++j) acc = fmaf(ld_any(p.L, p.dtype, ((size_t)d * B + k) * B + j), P[j * 32 + dd], acc);
+#pragma unroll
+        for (int j = 0; j < MAX_B; ++j)
+            if (j < k) acc = fmaf(lrow[j], P[j * 32 + dd], acc);
         p.Pc[(tok0 + k) * RANK + d] = acc;
     }
 }
@@ -210,60 +320,76 @@ __global__ void __launch_bounds__(256) k_pre_mix(const Params *__restrict__ pp)
 // -------------------------------------------------------------- k_mix_mlp
 
 constexpr int MLP_CLUSTER = 8;
+constexpr int W1S_LD = RANK + 2;        // padded row strides (in elements) so that
+constexpr int W2S_LD = 2 * RANK + 2;    // 32 rows hit 32 different banks
 
-// grid (8, b), cluster (8, 1, 1), 256 threads.  CTA `rank` of block s owns
-// channels [32 rank, +32) of c and z, and rows [64 rank, +64) of W_1.
-__global__ void __cluster_dims__(MLP_CLUSTER, 1, 1) __launch_bounds__(256) k_mix_mlp(const Params *__restrict__ pp)
+// Trans for the cluster's tokens, one CTA's share:  u rows [64 rank, +64) of
+// sigma(W_1 c) and z channels [32 rank, +32) of c + W_2 u.  The CTA's W_1 and
+// W_2 rows are staged in shared memory (T = storage type of the weights).
+// STAGE = false reads the rows straight from global memory (fp32 weights,
+// which would not fit next to the activations).
+template <typename T, bool STAGE>
+__device__ __forceinline__ void mlp_share(const Params &p, cg::cluster_group &cluster, int rank, int cnt, int m,
+                                          int s, int off, float (*cown)[32], float (*uown)[64], float *cop,
+                                          float *uop, T *stage)
 {
-    const Params &p = *pp;
-    cg::cluster_group cluster = cg::this_cluster();
-    const int rank = (int)cluster.block_rank();
-    const int s = blockIdx.y, B = p.B;
-    const SeqState st = p.st[s];
-    if (!st.active) return;            // uniform over the cluster
-    const int m = st.m, cnt = B - 1 - m, off = st.off;
-    const int d0 = rank * 32;
-
-    __shared__ float e[MAX_B][32];      // gathered E' rows, own channel slice
-    __shared__ float cown[MAX_B][32];   // c, own channel slice (unrounded)
-    __shared__ float uown[MAX_B][64];   // sigma(W_1 c), own rows, operand-rounded
-    extern __shared__ float dyn[];
-    float *cop = dyn;                   // [cnt][RANK]    all of c, operand-rounded
-    float *uop = dyn + MAX_B * RANK;    // [cnt][2 RANK]  all of sigma(W_1 c)
-
-    // Fuse (token part) + Mix for the own channel slice
-    for (int i = threadIdx.x; i < B * 32; i += blockDim.x) {
-        const int j = i / 32, dd = i % 32;
-        int x = j == 0 ? p.anchor[s] : p.tokens[(size_t)s * B + j - 1];
-        if (x < 0 || x >= p.V) x = 0;   // reported by k_init
-        e[j][dd] = p.Ep[(size_t)x * RANK + d0 + dd];
+    const int B = p.B, d0 = rank * 32;
+    const T *W1 = static_cast<const T *>(p.W1) + (size_t)rank * 64 * RANK;
+    const T *W2 = static_cast<const T *>(p.W2) + (size_t)d0 * 2 * RANK;
+    const T *w1s = W1, *w2s = W2;
+    int ld1 = RANK, ld2 = 2 * RANK;
+    if constexpr (STAGE) {
+        // bf16 rows, 16-byte loads issued back to back; the padded smem rows are
+        // written as 4-byte pairs
+        T *s1 = stage, *s2 = stage + 64 * W1S_LD;
+        constexpr int N1 = 64 * RANK / 8, N2 = 32 * 2 * RANK / 8;
+        uint4 r1[N1 / 256], r2[N2 / 256];
+#pragma unroll
+        for (int q = 0; q < N1 / 256; ++q) r1[q] = __ldg(reinterpret_cast<const uint4 *>(W1) + threadIdx.x + 256 * q);
+#pragma unroll
+        for (int q = 0; q < N2 / 256; ++q) r2[q] = __ldg(reinterpret_cast<const uint4 *>(W2) + threadIdx.x + 256 * q);
+#pragma unroll
+        for (int q = 0; q < N1 / 256; ++q) {
+            const int i = threadIdx.x + 256 * q, row = i / (RANK / 8), c = i % (RANK / 8);
+            uint32_t *dst = reinterpret_cast<uint32_t *>(s1 + row * W1S_LD + 8 * c);
+            dst[0] = r1[q].x; dst[1] = r1[q].y; dst[2] = r1[q].z; dst[3] = r1[q].w;
+        }
+#pragma unroll
+        for (int q = 0; q < N2 / 256; ++q) {
+            const int i = threadIdx.x + 256 * q, row = i / (2 * RANK / 8), c = i % (2 * RANK / 8);
+            uint32_t *dst = reinterpret_cast<uint32_t *>(s2 + row * W2S_LD + 8 * c);
+            dst[0] = r2[q].x; dst[1] = r2[q].y; dst[2] = r2[q].z; dst[3] = r2[q].w;
+        }
+        w1s = s1;
+        w2s = s2;
+        ld1 = W1S_LD;
+        ld2 = W2S_LD;
     }
-    __syncthreads();
-    for (int i = threadIdx.x; i < cnt * 32; i += blockDim.x) {
-        const int t = i / 32, dd = i % 32, k = m + 1 + t, d = d0 + dd;
-        float acc = p.Pc[((size_t)s * B + k) * RANK + d] + e[k][dd];
-        for (int j = 0; j < k; ++j) acc = fmaf(ld_any(p.L, p.dtype, ((size_t)d * B + k) * B + j), e[j][dd], acc);
-        cown[t][dd] = acc;
-    }
-    cluster.sync();
-    for (int i = threadIdx.x; i < cnt * RANK; i += blockDim.x) {
-        const int t = i / RANK, d = i % RANK;
-        const float *peer = cluster.map_shared_rank(&cown[0][0], d / 32);
-        cop[t * RANK + d] = round_op(peer[t * 32 + (d % 32)], p.dtype);
+    // all of c from the 8 CTAs of the cluster (float4 loads of peer shared memory)
+    for (int i = threadIdx.x; i < cnt * RANK / 4; i += blockDim.x) {
+        const int t = i / (RANK / 4), d = 4 * (i % (RANK / 4));
+        const float4 *peer = reinterpret_cast<const float4 *>(cluster.map_shared_rank(&cown[0][0], d / 32));
+        const float4 c4 = peer[(t * 32 + (d % 32)) / 4];
+        float *dst = cop + t * RANK + d;
+        dst[0] = round_op(c4.x, p.dtype);
+        dst[1] = round_op(c4.y, p.dtype);
+        dst[2] = round_op(c4.z, p.dtype);
+        dst[3] = round_op(c4.w, p.dtype);
     }
     __syncthreads();
     // t = W_1 c for rows [64 rank, +64): thread (row, token group of 4)
     {
-        const int row = threadIdx.x % 64, tg = threadIdx.x / 64, o = rank * 64 + row;
+        const int row = threadIdx.x % 64, tg = threadIdx.x / 64;
+        const T *w = w1s + row * ld1;
         float acc[8];
 #pragma unroll
         for (int q = 0; q < 8; ++q) acc[q] = 0.0f;
         for (int d = 0; d < RANK; ++d) {
-            const float w = ld_any(p.W1, p.dtype, (size_t)o * RANK + d);
+            const float wv = ldf(w, d);
 #pragma unroll
             for (int q = 0; q < 8; ++q) {
                 const int t = tg + 4 * q;
-                if (t < cnt) acc[q] = fmaf(w, cop[t * RANK + d], acc[q]);
+                if (t < cnt) acc[q] = fmaf(wv, cop[t * RANK + d], acc[q]);
             }
         }
 #pragma unroll
@@ -273,24 +399,25 @@ __global__ void __cluster_dims__(MLP_CLUSTER, 1, 1) __launch_bounds__(256) k_mix
         }
     }
     cluster.sync();
-    for (int i = threadIdx.x; i < cnt * 2 * RANK; i += blockDim.x) {
-        const int t = i / (2 * RANK), f = i % (2 * RANK);
-        const float *peer = cluster.map_shared_rank(&uown[0][0], f / 64);
-        uop[t * 2 * RANK + f] = peer[t * 64 + (f % 64)];
+    for (int i = threadIdx.x; i < cnt * 2 * RANK / 4; i += blockDim.x) {
+        const int t = i / (2 * RANK / 4), f = 4 * (i % (2 * RANK / 4));
+        const float4 *peer = reinterpret_cast<const float4 *>(cluster.map_shared_rank(&uown[0][0], f / 64));
+        reinterpret_cast<float4 *>(uop + t * 2 * RANK)[f / 4] = peer[(t * 64 + (f % 64)) / 4];
     }
     __syncthreads();
     // z = c + W_2 u for channels [32 rank, +32): thread (row, token group of 8)
     {
         const int row = threadIdx.x % 32, tg = threadIdx.x / 32, d = d0 + row;
+        const T *w = w2s + row * ld2;
         float acc[4];
 #pragma unroll
         for (int q = 0; q < 4; ++q) acc[q] = 0.0f;
         for (int f = 0; f < 2 * RANK; ++f) {
-            const float w = ld_any(p.W2, p.dtype, (size_t)d * 2 * RANK + f);
+            const float wv = ldf(w, f);
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 const int t = tg + 8 * q;
-                if (t < cnt) acc[q] = fmaf(w, uop[t * 2 * RANK + f], acc[q]);
+                if (t < cnt) acc[q] = fmaf(wv, uop[t * 2 * RANK + f], acc[q]);
             }
         }
         float *zf = p.z_final ? p.z_final : p.zbuf;
@@ -306,6 +433,181 @@ __global__ void __cluster_dims__(MLP_CLUSTER, 1, 1) __launch_bounds__(256) k_mix
                 else static_cast<float *>(p.zpack)[zi] = z;
             }
         }
+    }
+}
+
+// D (16x8, fp32) += A (16x16, bf16, row-major) * B (16x8, bf16, column-major):
+// the m16n8k16 warp-level tensor-core product (used for the small Trans GEMMs;
+// the vocabulary readout uses tcgen05).
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1)
+{
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+        "{%0, %1, %2, %3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+constexpr int COP_LD = RANK + 8;        // bf16 row strides of the A operands in
+constexpr int UOP_LD = 2 * RANK + 8;    // shared memory (8-row fragments hit distinct banks)
+constexpr int UOWN_LD = 64 + 8;
+
+// Trans on tensor cores for bf16 refiners (operands are bf16 by the precision
+// contract).  Tokens are the M dimension (two 16-row tiles cover up to 32),
+// W_1 / W_2 rows the N dimension, features the K dimension.
+__device__ __forceinline__ void mlp_share_mma(const Params &p, cg::cluster_group &cluster, int rank, int cnt, int m,
+                                              int s, int off, float (*cown)[32], uint16_t *cop, uint16_t *uop,
+                                              uint16_t *uown)
+{
+    const int B = p.B, d0 = rank * 32, warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const int g = lane >> 2, tq = lane & 3;      // fragment row group, thread in group
+    const uint16_t *W1 = static_cast<const uint16_t *>(p.W1);
+    const uint16_t *W2 = static_cast<const uint16_t *>(p.W2);
+    // B fragments straight from global memory, issued before the exchange:
+    // warp w owns W_1 rows [64 rank + 8 w, +8) and W_2 rows [32 rank + 8 (w % 4), +8)
+    const uint32_t *w1row = reinterpret_cast<const uint32_t *>(W1 + (size_t)(rank * 64 + 8 * warp + g) * RANK);
+    const uint32_t *w2row = reinterpret_cast<const uint32_t *>(W2 + (size_t)(d0 + 8 * (warp & 3) + g) * 2 * RANK);
+    uint32_t b1f[RANK / 16][2], b2f[2 * RANK / 16 / 2][2];
+#pragma unroll
+    for (int ks = 0; ks < RANK / 16; ++ks) {
+        b1f[ks][0] = __ldg(w1row + ks * 8 + tq);
+        b1f[ks][1] = __ldg(w1row + ks * 8 + 4 + tq);
+    }
+    // the W_2 product splits K in two halves over warps w and w + 4
+    const int khalf = warp >> 2;
+#pragma unroll
+    for (int ks = 0; ks < RANK / 16; ++ks) {
+        const int kk = khalf * (RANK / 16) + ks;
+        b2f[ks][0] = __ldg(w2row + kk * 8 + tq);
+        b2f[ks][1] = __ldg(w2row + kk * 8 + 4 + tq);
+    }
+    // all of c from the cluster, rounded to bf16 (rows past cnt are zero)
+    for (int i = threadIdx.x; i < 32 * RANK / 4; i += blockDim.x) {
+        const int t = i / (RANK / 4), d = 4 * (i % (RANK / 4));
+        float4 c4 = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (t < cnt) {
+            const float4 *peer = reinterpret_cast<const float4 *>(cluster.map_shared_rank(&cown[0][0], d / 32));
+            c4 = peer[(t * 32 + (d % 32)) / 4];
+        }
+        uint32_t *dst = reinterpret_cast<uint32_t *>(cop + t * COP_LD + d);
+        dst[0] = (uint32_t)f2bf(c4.x) | ((uint32_t)f2bf(c4.y) << 16);
+        dst[1] = (uint32_t)f2bf(c4.z) | ((uint32_t)f2bf(c4.w) << 16);
+    }
+    __syncthreads();
+    // u = sigma(W_1 c): warp w -> 8 output rows, both token tiles
+    for (int mt = 0; mt * 16 < cnt; ++mt) {
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+        const uint16_t *arow0 = cop + (mt * 16 + g) * COP_LD, *arow1 = arow0 + 8 * COP_LD;
+#pragma unroll
+        for (int ks = 0; ks < RANK / 16; ++ks) {
+            uint32_t a[4];
+            a[0] = *reinterpret_cast<const uint32_t *>(arow0 + ks * 16 + 2 * tq);
+            a[1] = *reinterpret_cast<const uint32_t *>(arow1 + ks * 16 + 2 * tq);
+            a[2] = *reinterpret_cast<const uint32_t *>(arow0 + ks * 16 + 8 + 2 * tq);
+            a[3] = *reinterpret_cast<const uint32_t *>(arow1 + ks * 16 + 8 + 2 * tq);
+            mma_bf16_16816(acc, a, b1f[ks][0], b1f[ks][1]);
+        }
+        const int col = 8 * warp + 2 * tq;          // local W_1 row (0..63)
+        const int t0 = mt * 16 + g, t1 = t0 + 8;
+        *reinterpret_cast<uint32_t *>(uown + t0 * UOWN_LD + col) =
+            (uint32_t)f2bf(act_fn(p.act, acc[0])) | ((uint32_t)f2bf(act_fn(p.act, acc[1])) << 16);
+        *reinterpret_cast<uint32_t *>(uown + t1 * UOWN_LD + col) =
+            (uint32_t)f2bf(act_fn(p.act, acc[2])) | ((uint32_t)f2bf(act_fn(p.act, acc[3])) << 16);
+    }
+    cluster.sync();
+    // all of u from the cluster (16-byte pieces of the peers' rows)
+    for (int i = threadIdx.x; i < cnt * (2 * RANK / 8); i += blockDim.x) {
+        const int t = i / (2 * RANK / 8), f = 8 * (i % (2 * RANK / 8));
+        const uint16_t *peer = cluster.map_shared_rank(uown, f / 64);
+        *reinterpret_cast<uint4 *>(uop + t * UOP_LD + f) =
+            *reinterpret_cast<const uint4 *>(peer + t * UOWN_LD + (f % 64));
+    }
+    for (int i = threadIdx.x; i < (32 - cnt) * (2 * RANK / 8); i += blockDim.x) {
+        const int t = cnt + i / (2 * RANK / 8), f = 8 * (i % (2 * RANK / 8));
+        *reinterpret_cast<uint4 *>(uop + t * UOP_LD + f) = make_uint4(0, 0, 0, 0);
+    }
+    __syncthreads();
+    // z = c + W_2 u: warp w -> 8 channels (w % 4), half of K (w / 4); the two
+    // halves meet in shared memory
+    __shared__ float zhalf[2][32][32];
+    for (int mt = 0; mt * 16 < cnt; ++mt) {
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+        const uint16_t *arow0 = uop + (mt * 16 + g) * UOP_LD + khalf * RANK, *arow1 = arow0 + 8 * UOP_LD;
+#pragma unroll
+        for (int ks = 0; ks < RANK / 16; ++ks) {
+            uint32_t a[4];
+            a[0] = *reinterpret_cast<const uint32_t *>(arow0 + ks * 16 + 2 * tq);
+            a[1] = *reinterpret_cast<const uint32_t *>(arow1 + ks * 16 + 2 * tq);
+            a[2] = *reinterpret_cast<const uint32_t *>(arow0 + ks * 16 + 8 + 2 * tq);
+            a[3] = *reinterpret_cast<const uint32_t *>(arow1 + ks * 16 + 8 + 2 * tq);
+            mma_bf16_16816(acc, a, b2f[ks][0], b2f[ks][1]);
+        }
+        const int col = 8 * (warp & 3) + 2 * tq;
+        const int t0 = mt * 16 + g;
+        zhalf[khalf][t0][col] = acc[0];
+        zhalf[khalf][t0][col + 1] = acc[1];
+        zhalf[khalf][t0 + 8][col] = acc[2];
+        zhalf[khalf][t0 + 8][col + 1] = acc[3];
+    }
+    __syncthreads();
+    float *zf = p.z_final ? p.z_final : p.zbuf;
+    for (int i = threadIdx.x; i < cnt * 32; i += blockDim.x) {
+        const int t = i / 32, dd = i % 32, k = m + 1 + t, d = d0 + dd;
+        const float z = cown[t][dd] + (zhalf[0][t][dd] + zhalf[1][t][dd]);
+        zf[((size_t)s * B + k) * RANK + d] = z;
+        static_cast<uint16_t *>(p.zpack)[(size_t)(off + t) * RANK + d] = f2bf(z);
+    }
+}
+
+// grid (8, b), cluster (8, 1, 1), 256 threads.  CTA `rank` of block s owns
+// channels [32 rank, +32) of c and z, and rows [64 rank, +64) of W_1; c and
+// sigma(W_1 c) are exchanged through distributed shared memory.
+__global__ void __cluster_dims__(MLP_CLUSTER, 1, 1) __launch_bounds__(256) k_mix_mlp(const Params *__restrict__ pp)
+{
+    const Params &p = *pp;
+    cg::cluster_group cluster = cg::this_cluster();
+    const int rank = (int)cluster.block_rank();
+    const int s = blockIdx.y, B = p.B;
+    const SeqState st = p.st[s];
+    if (!st.active) return;            // uniform over the cluster
+    const int m = st.m, cnt = B - 1 - m, off = st.off;
+    const int d0 = rank * 32;
+
+    __shared__ float e[MAX_B][32];                     // gathered E' rows, own channel slice
+    __shared__ __align__(16) float cown[MAX_B][32];    // c, own channel slice (unrounded)
+    __shared__ __align__(16) float uown[MAX_B][64];    // sigma(W_1 c), own rows (fp32 path)
+    extern __shared__ __align__(16) float dyn[];
+
+    // Fuse (token part) + Mix for the own channel slice
+    for (int i = threadIdx.x; i < B * 32; i += blockDim.x) {
+        const int j = i / 32, dd = i % 32;
+        int x = j == 0 ? p.anchor[s] : p.tokens[(size_t)s * B + j - 1];
+        if (x < 0 || x >= p.V) x = 0;   // reported by k_init
+        e[j][dd] = p.Ep[(size_t)x * RANK + d0 + dd];
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < cnt * 32; i += blockDim.x) {
+        const int t = i / 32, dd = i % 32, k = m + 1 + t, d = d0 + dd;
+        float lrow[MAX_B];
+        const size_t lb = ((size_t)d * B + k) * B;
+#pragma unroll
+        for (int j = 0; j < MAX_B; ++j) lrow[j] = j < k ? ld_any(p.L, p.dtype, lb + j) : 0.0f;
+        float acc = p.Pc[((size_t)s * B + k) * RANK + d] + e[k][dd];
+#pragma unroll
+        for (int j = 0; j < MAX_B; ++j)
+            if (j < k) acc = fmaf(lrow[j], e[j][dd], acc);
+        cown[t][dd] = acc;
+    }
+    cluster.sync();
+    if (p.dtype) {
+        uint16_t *cop = reinterpret_cast<uint16_t *>(dyn);
+        uint16_t *uop = cop + 32 * COP_LD;
+        uint16_t *uo = uop + 32 * UOP_LD;
+        mlp_share_mma(p, cluster, rank, cnt, m, s, off, cown, cop, uop, uo);
+    } else {
+        float *cop = dyn;
+        float *uop = dyn + MAX_B * RANK;
+        mlp_share<float, false>(p, cluster, rank, cnt, m, s, off, cown, uown, cop, uop, nullptr);
     }
     cluster.sync();                     // peers may still read our shared memory
 }
@@ -406,13 +708,15 @@ __global__ void __launch_bounds__(1024) k_reduce(const Params *__restrict__ pp, 
     const int s = blockIdx.x, B = p.B, warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const SeqState st = p.st[s];
     __shared__ int last;
-    __shared__ int ynew[MAX_B];
+    __shared__ int ynew[MAX_B], yold[MAX_B];
     const float T = p.temperature[s];
     const float invT = T > 0.0f ? 1.0f / T : 0.0f;
     const bool sampling = invT > 0.0f;
     if (st.active && warp < B && warp > st.m) {
         const int k = warp, i = st.off + (k - st.m - 1), tok = s * B + k;
+        if (lane == 0) yold[k] = p.tokens[tok];
         Partial a{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
+#pragma unroll 4
         for (int r = lane; r < p.S; r += 32) merge_partial(a, p.part[(size_t)r * p.N + i], sampling);
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
@@ -435,9 +739,24 @@ __global__ void __launch_bounds__(1024) k_reduce(const Params *__restrict__ pp, 
             float x = -INFINITY, score = -INFINITY;
             if (v < p.V) {
                 float acc = 0.0f;
-                for (int d = 0; d < RANK; ++d)
-                    acc = fmaf(ld_any(p.W_r, p.dtype, (size_t)v * RANK + d),
-                               ld_any(p.zpack, p.dtype, (size_t)i * RANK + d), acc);
+                if (p.dtype) {
+                    const uint4 *wr = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.W_r) +
+                                                                      (size_t)v * RANK);
+                    const uint4 *zr = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.zpack) +
+                                                                      (size_t)i * RANK);
+#pragma unroll 8
+                    for (int c = 0; c < RANK / 8; ++c) {
+                        float w8[8], z8[8];
+                        bf16x8_to_f32(__ldg(wr + c), w8);
+                        bf16x8_to_f32(zr[c], z8);
+#pragma unroll
+                        for (int j = 0; j < 8; ++j) acc = fmaf(w8[j], z8[j], acc);
+                    }
+                } else {
+                    for (int d = 0; d < RANK; ++d)
+                        acc = fmaf(ld_any(p.W_r, 0, (size_t)v * RANK + d), ld_any(p.zpack, 0, (size_t)i * RANK + d),
+                                   acc);
+                }
                 x = (acc + ld_any(p.s, p.dtype, (size_t)tok * p.V + v)) * invT;
                 score = x + gumbel(p.seed[s], (uint32_t)v, (uint32_t)k, STREAM_ELEM, p.offset);
             }
@@ -457,17 +776,15 @@ __global__ void __launch_bounds__(1024) k_reduce(const Params *__restrict__ pp, 
             ynew[k] = y;
             if (p.lse) p.lse[tok] = lse;
             if (p.logit_sel) p.logit_sel[tok] = sel;
+            p.tokens[tok] = y;
         }
     }
     __syncthreads();
     if (threadIdx.x == 0) {
         if (st.active) {
             int first = -1;
-            for (int k = st.m + 1; k < B; ++k) {
-                const int old = p.tokens[(size_t)s * B + k];
-                if (ynew[k] != old && first < 0) first = k;
-                p.tokens[(size_t)s * B + k] = ynew[k];
-            }
+            for (int k = st.m + 1; k < B; ++k)
+                if (ynew[k] != yold[k]) { first = k; break; }
             SeqState ns = st;
             ns.iters = st.iters + 1;
             ns.converged = first < 0;
@@ -529,7 +846,7 @@ __global__ void __launch_bounds__(1024) k_reduce(const Params *__restrict__ pp, 
         p.ctl[CTL_PASS] = passes;
         // no block can take part in more than K_max passes; the cap also bounds
         // the loop should the per-block bookkeeping ever disagree
-        cudaGraphSetConditional(handle, (total > 0 && passes < p.K_max) ? 1u : 0u);
+        if (p.use_graph) cudaGraphSetConditional(handle, (total > 0 && passes < p.K_max) ? 1u : 0u);
     }
 }
 

@@ -5,6 +5,7 @@
 #include <cudaTypedefs.h>
 
 #include <cstdint>
+#include <cstdio>
 #include <cstdlib>
 #include <cstring>
 #include <mutex>
@@ -70,6 +71,7 @@ struct Layout {
     size_t status = 0, ctl = 64, params = 256, st = 0, upart = 0, pc = 0, ynew = 0, acttok = 0, zpack = 0,
            zbuf = 0, part = 0, total = 0;
     int ksplit = 1, kchunk = 0, S = 1;
+    bool gemv = false;
 };
 
 }  // namespace
@@ -106,13 +108,22 @@ Layout make_layout(const xpress_refiner *R, int b)
     size_t o = align256(L.params + sizeof(Params));
     L.st = o;
     o = align256(o + (size_t)b * sizeof(SeqState));
-    const int mt = (N + 63) / 64;
-    const int ctas = mt * (RANK / 64) * 2;
-    int ks = (2 * R->num_sms + ctas - 1) / ctas;
-    const int kmax = R->w.H / 256 > 0 ? R->w.H / 256 : 1;
-    ks = ks < 1 ? 1 : (ks > kmax ? kmax : ks);
-    L.kchunk = ((R->w.H + ks - 1) / ks + 15) / 16 * 16;
-    L.ksplit = (R->w.H + L.kchunk - 1) / L.kchunk;
+    L.gemv = R->w.dtype == XPRESS_BF16 && N <= 32;
+    if (L.gemv) {
+        // the largest K-slice (multiple of 256) whose h fits in 128 KB of shared memory
+        int ks = (GEMV_SMEM / (2 * N)) / 256 * 256;
+        const int H256 = (R->w.H + 255) / 256 * 256;
+        L.kchunk = ks < H256 ? ks : H256;
+        L.ksplit = (R->w.H + L.kchunk - 1) / L.kchunk;
+    } else {
+        const int mt = (N + 63) / 64;
+        const int ctas = mt * (RANK / 64) * 2;
+        int ks = (2 * R->num_sms + ctas - 1) / ctas;
+        const int kmax = R->w.H / 256 > 0 ? R->w.H / 256 : 1;
+        ks = ks < 1 ? 1 : (ks > kmax ? kmax : ks);
+        L.kchunk = ((R->w.H + ks - 1) / ks + 15) / 16 * 16;
+        L.ksplit = (R->w.H + L.kchunk - 1) / L.kchunk;
+    }
     L.upart = o;
     o = align256(o + (size_t)L.ksplit * N * 2 * RANK * 4);
     L.pc = o;
@@ -148,6 +159,7 @@ Params make_params(const xpress_refiner *R, const xpress_block_in *in, const xpr
     P.fixed_K = in->fixed_K ? 1 : 0;
     P.offset = in->offset;
     P.S = L.S;
+    P.use_graph = 1;
     P.ksplit = L.ksplit;
     P.h = in->h;
     P.s = in->s;
@@ -199,17 +211,30 @@ int set_kernel_attributes()
         rc = XPRESS_OK;
         if (cudaFuncSetAttribute(k_read_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kReadTcSmemBytes) !=
                 cudaSuccess ||
-            cudaFuncSetAttribute(k_mix_mlp, cudaFuncAttributeMaxDynamicSharedMemorySize, MIX_MLP_DYN_SMEM) !=
+            cudaFuncSetAttribute(k_mix_mlp, cudaFuncAttributeMaxDynamicSharedMemorySize, MIX_MLP_DYN_SMEM_MAX) !=
                 cudaSuccess ||
             cudaFuncSetAttribute(k_read_simt, cudaFuncAttributeMaxDynamicSharedMemorySize, READ_SIMT_DYN_SMEM) !=
                 cudaSuccess ||
             cudaFuncSetAttribute(k_pre_mix, cudaFuncAttributeMaxDynamicSharedMemorySize, pre_mix_smem(MAX_B)) !=
+                cudaSuccess ||
+            cudaFuncSetAttribute(k_pre_gemv, cudaFuncAttributeMaxDynamicSharedMemorySize, GEMV_SMEM) !=
                 cudaSuccess) {
             (void)cudaGetLastError();
             rc = XPRESS_ERR_CUDA;
         }
     });
     return rc;
+}
+
+void launch_pre_gemm(const Layout &L, int N, Params *pdev, cudaStream_t st)
+{
+    if (L.gemv) {
+        k_pre_gemv<<<dim3(2 * RANK / 8, L.ksplit), 256, N * L.kchunk * 2, st>>>(pdev, L.kchunk);
+    } else {
+        const dim3 grid(RANK / 64, (N + 63) / 64, L.ksplit);
+        k_pre_gemm<<<grid, 256, 0, st>>>(pdev, 0, L.kchunk);
+        k_pre_gemm<<<grid, 256, 0, st>>>(pdev, 1, L.kchunk);
+    }
 }
 
 void destroy_entry(GraphEntry &e)
@@ -257,11 +282,7 @@ int build_graph(xpress_refiner *R, GraphEntry &e, const Params &P, const Layout 
     cudaStream_t cs = R->cs;
     XP_CUDA(cudaStreamBeginCaptureToGraph(cs, g, &e.init_node, nullptr, 1, cudaStreamCaptureModeThreadLocal));
     if (!P.draft) k_rowmax<<<N, 256, 0, cs>>>(pdev);
-    {
-        const dim3 grid(RANK / 64, (N + 63) / 64, L.ksplit);
-        k_pre_gemm<<<grid, 256, 0, cs>>>(pdev, 0, L.kchunk);
-        k_pre_gemm<<<grid, 256, 0, cs>>>(pdev, 1, L.kchunk);
-    }
+    launch_pre_gemm(L, N, pdev, cs);
     k_pre_mix<<<dim3(b, RANK / 32), 256, pre_mix_smem(P.B), cs>>>(pdev);
     cudaStreamCaptureStatus cst;
     const cudaGraphNode_t *deps = nullptr;
@@ -291,7 +312,7 @@ int build_graph(xpress_refiner *R, GraphEntry &e, const Params &P, const Layout 
     }
     cudaGraph_t body = cp.conditional.phGraph_out[0];
     XP_CUDA(cudaStreamBeginCaptureToGraph(cs, body, nullptr, nullptr, 0, cudaStreamCaptureModeThreadLocal));
-    k_mix_mlp<<<dim3(8, b), 256, MIX_MLP_DYN_SMEM, cs>>>(pdev);
+    k_mix_mlp<<<dim3(8, b), 256, mix_mlp_smem(P.dtype), cs>>>(pdev);
     if (R->use_tc)
         k_read_tc<<<L.S, kReadTcThreads, kReadTcSmemBytes, cs>>>(pdev, R->tmap_wr, tmap_z);
     else
@@ -301,6 +322,107 @@ int build_graph(xpress_refiner *R, GraphEntry &e, const Params &P, const Layout 
     XP_CUDA(cudaStreamEndCapture(cs, &body_out));
     XP_CUDA(cudaGraphInstantiate(&e.exec, g, 0));
     return XPRESS_OK;
+}
+
+// Profiling mode (XPRESS_EAGER=1 in the environment): the same kernels
+// launched one by one from the host, with a host read of the pass count after
+// every pass, so that per-kernel profilers see each launch.  Not for serving.
+// Per-kernel CUDA-event timer of the profiling mode (XPRESS_EAGER=2).
+struct KernelTimer {
+    cudaStream_t st;
+    bool on;
+    struct Rec { const char *name; cudaEvent_t a, b; };
+    Rec recs[256];
+    int n = 0;
+    KernelTimer(cudaStream_t s, bool enable) : st(s), on(enable) {}
+    void start(const char *name)
+    {
+        if (!on || n >= 256) return;
+        recs[n].name = name;
+        cudaEventCreate(&recs[n].a);
+        cudaEventCreate(&recs[n].b);
+        cudaEventRecord(recs[n].a, st);
+    }
+    void stop()
+    {
+        if (!on || n >= 256) return;
+        cudaEventRecord(recs[n].b, st);
+        ++n;
+    }
+    void report()
+    {
+        if (!on) return;
+        cudaStreamSynchronize(st);
+        std::fprintf(stderr, "xpress-timing:");
+        for (int i = 0; i < n; ++i) {
+            float ms = 0.0f;
+            cudaEventElapsedTime(&ms, recs[i].a, recs[i].b);
+            std::fprintf(stderr, " %s=%.2f", recs[i].name, 1000.0f * ms);
+            cudaEventDestroy(recs[i].a);
+            cudaEventDestroy(recs[i].b);
+        }
+        std::fprintf(stderr, "\n");
+    }
+};
+
+// Profiling mode (XPRESS_EAGER=1 in the environment): the same kernels
+// launched one by one from the host, with a host read of the pass count after
+// every pass, so that per-kernel profilers see each launch; XPRESS_EAGER=2
+// also prints CUDA-event times of every launch (microseconds) to stderr.
+// Not for serving.
+int run_eager(xpress_refiner *R, Params P, const Layout &L, void *ws, cudaStream_t st, bool timed)
+{
+    P.use_graph = 0;
+    const int b = P.b, N = P.N;
+    Params *pdev = reinterpret_cast<Params *>(static_cast<char *>(ws) + L.params);
+    CUtensorMap tmap_z{};
+    if (R->use_tc && !make_tmap_bf16(&tmap_z, P.zpack, RANK, (uint64_t)N, 64, 32)) return XPRESS_ERR_CUDA;
+    KernelTimer kt(st, timed);
+    XP_CUDA(cudaMemsetAsync(P.status, 0, 4, st));
+    kt.start("init");
+    k_init<<<((N > b ? N : b) + 255) / 256, 256, 0, st>>>(P, pdev, 0);
+    kt.stop();
+    if (!P.draft) {
+        kt.start("rowmax");
+        k_rowmax<<<N, 256, 0, st>>>(pdev);
+        kt.stop();
+    }
+    kt.start("pre_gemm");
+    launch_pre_gemm(L, N, pdev, st);
+    kt.stop();
+    kt.start("pre_mix");
+    k_pre_mix<<<dim3(b, RANK / 32), 256, pre_mix_smem(P.B), st>>>(pdev);
+    kt.stop();
+    for (int pass = 0; pass < P.K_max; ++pass) {
+        kt.start("mix_mlp");
+        k_mix_mlp<<<dim3(8, b), 256, mix_mlp_smem(P.dtype), st>>>(pdev);
+        kt.stop();
+        kt.start("read");
+        if (R->use_tc)
+            k_read_tc<<<L.S, kReadTcThreads, kReadTcSmemBytes, st>>>(pdev, R->tmap_wr, tmap_z);
+        else
+            k_read_simt<<<L.S, 256, READ_SIMT_DYN_SMEM, st>>>(pdev);
+        kt.stop();
+        kt.start("reduce");
+        k_reduce<<<b, 1024, 0, st>>>(pdev, 0);
+        kt.stop();
+        int32_t nact = 0;
+        XP_CUDA(cudaMemcpyAsync(&nact, P.ctl + CTL_NACT, 4, cudaMemcpyDeviceToHost, st));
+        XP_CUDA(cudaStreamSynchronize(st));
+        if (nact == 0) break;
+    }
+    kt.report();
+    XP_CUDA(cudaGetLastError());
+    return XPRESS_OK;
+}
+
+int eager_mode()
+{
+    static const int mode = [] {
+        const char *e = std::getenv("XPRESS_EAGER");
+        return (e && (e[0] == '1' || e[0] == '2')) ? e[0] - '0' : 0;
+    }();
+    return mode;
 }
 
 int check_ws(void *ws, size_t ws_bytes, size_t need)
@@ -402,6 +524,7 @@ int xpress_refine_block(const xpress_refiner *Rc, const xpress_block_in *in, con
     const Layout L = make_layout(R, in->b);
     if (const int rc = check_ws(ws, ws_bytes, L.total)) return rc;
     Params P = make_params(R, in, out, ws, L);
+    if (eager_mode()) return run_eager(R, P, L, ws, static_cast<cudaStream_t>(stream), eager_mode() == 2);
     const bool draft_null = in->draft == nullptr;
     GraphEntry *hit = nullptr, *victim = &R->cache[0];
     for (auto &e : R->cache) {
@@ -508,7 +631,7 @@ int xpress_accept(const xpress_refiner *R, const xpress_accept_in *in, int32_t *
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     XP_CUDA(cudaMemsetAsync(P.status, 0, 4, st));
     k_acc_rows<<<dim3(in->b * (R->w.B + 1), A.chunks), 256, 0, st>>>(P);
-    k_acc_decide<<<(in->b + 127) / 128, 128, 0, st>>>(P, A.chunks);
+    k_acc_decide<<<in->b, 32, 0, st>>>(P, A.chunks);
     k_acc_sample<<<dim3(in->b, A.chunks2), 256, 0, st>>>(P);
     k_acc_finish<<<(in->b + 127) / 128, 128, 0, st>>>(P, A.chunks2);
     XP_CUDA(cudaGetLastError());
