@@ -61,6 +61,7 @@ struct Params {
     uint32_t offset;
     int S;                       // vocabulary ranges of the Read kernel
     int use_graph;               // 1: the pass loop is a graph WHILE node
+    unsigned long long *trace;   // optional kernel timeline (profiling), else NULL
     int ksplit;                  // split-K factor of the hidden projection
     // inputs (caller-owned)
     const void *h, *s;
@@ -216,6 +217,32 @@ __device__ __forceinline__ void select_group(SelState &st, const float *l, int v
 
 // ------------------------------------------------------------- PTX wrappers
 
+__device__ __forceinline__ unsigned long long globaltimer_ns()
+{
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Optional timeline of a refinement call (enabled by the host for profiling):
+// trace[slot] = earliest start, trace[TRACE_SLOTS + slot] = latest end over
+// the kernel's blocks (globaltimer, ns).  Slots: 0 init, 1 argmax seed,
+// 2 precompute GEMM, 3 precompute Fuse/Mix, 8 + 4 j + {0 Trans, 1 Read,
+// 2 reduce} for pass j.
+constexpr int TRACE_SLOTS = 256;
+__device__ __forceinline__ void trace_mark(unsigned long long *tr, int slot, unsigned long long t0)
+{
+    if (tr && slot < TRACE_SLOTS) {
+        atomicMin(tr + slot, t0);
+        atomicMax(tr + TRACE_SLOTS + slot, globaltimer_ns());
+    }
+}
+
+// Programmatic dependent launch: wait for the preceding kernel of the stream
+// (no-op when launched without the attribute) / let the next one start.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 __device__ __forceinline__ uint32_t smem_u32(const void *p)
 {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -284,6 +311,31 @@ __device__ __forceinline__ void tma_load_2d(void *smem_dst, const CUtensorMap *m
         "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
         ::"r"(smem_u32(smem_dst)), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
         : "memory");
+}
+
+// Same, with an L2 cache policy (e.g. keep the readout weights resident
+// across the passes of one call).
+__device__ __forceinline__ void tma_load_2d_hint(void *smem_dst, const CUtensorMap *map, uint64_t *bar, int x, int y,
+                                                 uint64_t policy)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1, {%2, "
+        "%3}], [%4], %5;" ::"r"(smem_u32(smem_dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar)), "l"(policy)
+        : "memory");
+}
+
+// Bulk prefetch of [addr, addr + bytes) into L2 (16-byte aligned, multiple of 16).
+__device__ __forceinline__ void prefetch_l2_bulk(const void *addr, uint32_t bytes)
+{
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(addr), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ uint64_t policy_evict_last()
+{
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
 }
 
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap *map)

@@ -35,7 +35,7 @@ __global__ void k_build_ep(const void *W_e, const void *W_in, float *Ep, int V, 
 
 // read_tc.cu
 __global__ void k_read_tc(const Params *pp, const __grid_constant__ CUtensorMap tmap_wr,
-                          const __grid_constant__ CUtensorMap tmap_z);
+                          const __grid_constant__ CUtensorMap tmap_z, int V);
 extern const size_t kReadTcSmemBytes;
 extern const int kReadTcThreads;
 

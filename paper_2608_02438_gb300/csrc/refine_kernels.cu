@@ -33,6 +33,7 @@ namespace xp {
 __global__ void k_init(Params pin, Params *pdev, cudaGraphConditionalHandle handle)
 {
     const Params &p = pin;
+    const unsigned long long t_start = globaltimer_ns();
     const int t = blockIdx.x * blockDim.x + threadIdx.x;
     if (t == 0) {
         *pdev = pin;
@@ -57,6 +58,7 @@ __global__ void k_init(Params pin, Params *pdev, cudaGraphConditionalHandle hand
         if (p.iters) p.iters[t] = 0;
         if (p.converged) p.converged[t] = 0;
     }
+    if (threadIdx.x == 0) trace_mark(p.trace, 0, t_start);
 }
 
 // --------------------------------------------------------------- k_rowmax
@@ -183,25 +185,47 @@ __device__ __forceinline__ void bf16x8_to_f32(const uint4 &w, float (&x)[8])
 // CTA stages its K-slice of every token's h in shared memory ([N][kslice]).
 __global__ void __launch_bounds__(256) k_pre_gemv(const Params *__restrict__ pp, int kslice)
 {
+    const unsigned long long t_start = globaltimer_ns();
     const Params &p = *pp;
     extern __shared__ __align__(16) uint16_t hs[];
     const int N = p.N, H = p.H, warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const int kb = blockIdx.y * kslice, ke = min(H, kb + kslice), kl = ke - kb;
     const uint16_t *h = static_cast<const uint16_t *>(p.h);
-    for (int i = threadIdx.x; i < N * (kl / 8); i += blockDim.x) {
-        const int t = i / (kl / 8), c = i % (kl / 8);
-        reinterpret_cast<uint4 *>(hs + (size_t)t * kslice)[c] =
-            __ldg(reinterpret_cast<const uint4 *>(h + (size_t)t * H + kb) + c);
-    }
+    // this warp's weight row: 16-byte pieces k0 = 8 lane + 256 q of the K-slice,
+    // the next piece requested while the current one is used
     const int o = blockIdx.x * 8 + warp;
     const uint16_t *W = static_cast<const uint16_t *>(o < RANK ? p.W_h : p.W_g) + (size_t)(o % RANK) * H + kb;
+    uint4 wcur = make_uint4(0, 0, 0, 0), wnext = make_uint4(0, 0, 0, 0);
+    if (8 * lane < kl) wcur = __ldg(reinterpret_cast<const uint4 *>(W + 8 * lane));
+    if (8 * lane + 256 < kl) wnext = __ldg(reinterpret_cast<const uint4 *>(W + 8 * lane + 256));
+    {
+        // stage h[:, K-slice] in batches of 8 16-byte loads per thread
+        const int per = kl / 8, total = N * per;
+        for (int i0 = 0; i0 < total; i0 += 8 * 256) {
+            uint4 hv[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const int i = i0 + q * 256 + threadIdx.x;
+                if (i < total)
+                    hv[q] = __ldg(reinterpret_cast<const uint4 *>(h + (size_t)(i / per) * H + kb) + (i % per));
+            }
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const int i = i0 + q * 256 + threadIdx.x;
+                if (i < total) reinterpret_cast<uint4 *>(hs + (size_t)(i / per) * kslice)[i % per] = hv[q];
+            }
+        }
+    }
+    __syncthreads();
     float v[32];
 #pragma unroll
     for (int t = 0; t < 32; ++t) v[t] = 0.0f;
-    __syncthreads();
+#pragma unroll 1
     for (int k0 = 8 * lane; k0 < kl; k0 += 256) {
         float w[8];
-        bf16x8_to_f32(__ldg(reinterpret_cast<const uint4 *>(W + k0)), w);
+        bf16x8_to_f32(wcur, w);
+        wcur = wnext;
+        if (k0 + 512 < kl) wnext = __ldg(reinterpret_cast<const uint4 *>(W + k0 + 512));
 #pragma unroll
         for (int t = 0; t < 32; ++t) {
             if (t < N) {
@@ -214,6 +238,8 @@ __global__ void __launch_bounds__(256) k_pre_gemv(const Params *__restrict__ pp,
     }
     const float sum = reduce_scatter32(v, lane);
     if (lane < N) p.Upart[((size_t)blockIdx.y * N + lane) * 2 * RANK + o] = sum;
+    __syncthreads();
+    if (threadIdx.x == 0) trace_mark(p.trace, 2, t_start);
 }
 
 // Folded embedding E'[v][d] = sum_e W_in[d][2r + e] W_e[v][e] (Sec. 4.1: Fuse
@@ -234,6 +260,7 @@ __global__ void __launch_bounds__(256) k_build_ep(const void *W_e, const void *W
 // memory: U [B][2r], u_g [r], W_in rows [32][2r + 1], P [B][32].
 __global__ void __launch_bounds__(256) k_pre_mix(const Params *__restrict__ pp)
 {
+    const unsigned long long t_start = globaltimer_ns();
     const Params &p = *pp;
     extern __shared__ float sm[];
     const int B = p.B, s = blockIdx.x, d0 = blockIdx.y * 32;
@@ -243,11 +270,19 @@ __global__ void __launch_bounds__(256) k_pre_mix(const Params *__restrict__ pp)
     float *P = Ws + 32 * (2 * RANK + 1);   // [B][32]   P for this channel slice
     const size_t tok0 = (size_t)s * B;
     if (p.dtype) {
-        for (int i = threadIdx.x; i < 32 * 2 * RANK / 8; i += blockDim.x) {
-            const int dd = i / (2 * RANK / 8), c = i % (2 * RANK / 8);
+        constexpr int PER = 32 * 2 * RANK / 8 / 256;   // 8 16-byte pieces per thread
+        uint4 wv[PER];
+#pragma unroll
+        for (int q = 0; q < PER; ++q) {
+            const int i = threadIdx.x + 256 * q, dd = i / (2 * RANK / 8), c = i % (2 * RANK / 8);
+            wv[q] = __ldg(reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.W_in) +
+                                                          (size_t)(d0 + dd) * 3 * RANK) + c);
+        }
+#pragma unroll
+        for (int q = 0; q < PER; ++q) {
+            const int i = threadIdx.x + 256 * q, dd = i / (2 * RANK / 8), c = i % (2 * RANK / 8);
             float x[8];
-            bf16x8_to_f32(__ldg(reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.W_in) +
-                                                                 (size_t)(d0 + dd) * 3 * RANK) + c), x);
+            bf16x8_to_f32(wv[q], x);
 #pragma unroll
             for (int j = 0; j < 8; ++j) Ws[dd * (2 * RANK + 1) + 8 * c + j] = x[j];
         }
@@ -315,6 +350,8 @@ __global__ void __launch_bounds__(256) k_pre_mix(const Params *__restrict__ pp)
             if (j < k) acc = fmaf(lrow[j], P[j * 32 + dd], acc);
         p.Pc[(tok0 + k) * RANK + d] = acc;
     }
+    __syncthreads();
+    if (threadIdx.x == 0) trace_mark(p.trace, 3, t_start);
 }
 
 // -------------------------------------------------------------- k_mix_mlp
@@ -455,43 +492,57 @@ constexpr int UOWN_LD = 64 + 8;
 // Trans on tensor cores for bf16 refiners (operands are bf16 by the precision
 // contract).  Tokens are the M dimension (two 16-row tiles cover up to 32),
 // W_1 / W_2 rows the N dimension, features the K dimension.
-__device__ __forceinline__ void mlp_share_mma(const Params &p, cg::cluster_group &cluster, int rank, int cnt, int m,
-                                              int s, int off, float (*cown)[32], uint16_t *cop, uint16_t *uop,
-                                              uint16_t *uown)
+// Tensor-core operand fragments of the CTA's W_1 / W_2 rows (static weights,
+// fetched before the kernel waits for its predecessor): warp w owns W_1 rows
+// [64 rank + 8 w, +8) and W_2 rows [32 rank + 8 (w % 4), +8) over K half w / 4.
+struct MlpFrags {
+    uint32_t b1[RANK / 16][2], b2[RANK / 16][2];
+};
+
+__device__ __forceinline__ void load_mlp_frags(const Params &p, int rank, MlpFrags &f)
 {
-    const int B = p.B, d0 = rank * 32, warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-    const int g = lane >> 2, tq = lane & 3;      // fragment row group, thread in group
-    const uint16_t *W1 = static_cast<const uint16_t *>(p.W1);
-    const uint16_t *W2 = static_cast<const uint16_t *>(p.W2);
-    // B fragments straight from global memory, issued before the exchange:
-    // warp w owns W_1 rows [64 rank + 8 w, +8) and W_2 rows [32 rank + 8 (w % 4), +8)
-    const uint32_t *w1row = reinterpret_cast<const uint32_t *>(W1 + (size_t)(rank * 64 + 8 * warp + g) * RANK);
-    const uint32_t *w2row = reinterpret_cast<const uint32_t *>(W2 + (size_t)(d0 + 8 * (warp & 3) + g) * 2 * RANK);
-    uint32_t b1f[RANK / 16][2], b2f[2 * RANK / 16 / 2][2];
-#pragma unroll
-    for (int ks = 0; ks < RANK / 16; ++ks) {
-        b1f[ks][0] = __ldg(w1row + ks * 8 + tq);
-        b1f[ks][1] = __ldg(w1row + ks * 8 + 4 + tq);
-    }
-    // the W_2 product splits K in two halves over warps w and w + 4
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32, g = lane >> 2, tq = lane & 3;
+    const uint32_t *w1row = reinterpret_cast<const uint32_t *>(static_cast<const uint16_t *>(p.W1) +
+                                                               (size_t)(rank * 64 + 8 * warp + g) * RANK);
+    const uint32_t *w2row = reinterpret_cast<const uint32_t *>(static_cast<const uint16_t *>(p.W2) +
+                                                               (size_t)(rank * 32 + 8 * (warp & 3) + g) * 2 * RANK);
     const int khalf = warp >> 2;
 #pragma unroll
     for (int ks = 0; ks < RANK / 16; ++ks) {
+        f.b1[ks][0] = __ldg(w1row + ks * 8 + tq);
+        f.b1[ks][1] = __ldg(w1row + ks * 8 + 4 + tq);
         const int kk = khalf * (RANK / 16) + ks;
-        b2f[ks][0] = __ldg(w2row + kk * 8 + tq);
-        b2f[ks][1] = __ldg(w2row + kk * 8 + 4 + tq);
+        f.b2[ks][0] = __ldg(w2row + kk * 8 + tq);
+        f.b2[ks][1] = __ldg(w2row + kk * 8 + 4 + tq);
     }
+}
+
+__device__ __forceinline__ void mlp_share_mma(const Params &p, cg::cluster_group &cluster, int rank, int cnt, int m,
+                                              int s, int off, float (*cown)[32], uint16_t *cop, uint16_t *uop,
+                                              uint16_t *uown, const MlpFrags &fr)
+{
+    const int B = p.B, d0 = rank * 32, warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const int g = lane >> 2, tq = lane & 3;      // fragment row group, thread in group
+    const int khalf = warp >> 2;                 // W_2: K half of this warp
     // all of c from the cluster, rounded to bf16 (rows past cnt are zero)
-    for (int i = threadIdx.x; i < 32 * RANK / 4; i += blockDim.x) {
-        const int t = i / (RANK / 4), d = 4 * (i % (RANK / 4));
-        float4 c4 = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (t < cnt) {
-            const float4 *peer = reinterpret_cast<const float4 *>(cluster.map_shared_rank(&cown[0][0], d / 32));
-            c4 = peer[(t * 32 + (d % 32)) / 4];
+    {
+        constexpr int PER = 32 * RANK / 4 / 256;     // 8 float4 per thread
+        float4 c4[PER];
+#pragma unroll
+        for (int q = 0; q < PER; ++q) {
+            const int i = threadIdx.x + 256 * q, t = i / (RANK / 4), d = 4 * (i % (RANK / 4));
+            c4[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (t < cnt)
+                c4[q] = reinterpret_cast<const float4 *>(cluster.map_shared_rank(&cown[0][0], d / 32))[
+                    (t * 32 + (d % 32)) / 4];
         }
-        uint32_t *dst = reinterpret_cast<uint32_t *>(cop + t * COP_LD + d);
-        dst[0] = (uint32_t)f2bf(c4.x) | ((uint32_t)f2bf(c4.y) << 16);
-        dst[1] = (uint32_t)f2bf(c4.z) | ((uint32_t)f2bf(c4.w) << 16);
+#pragma unroll
+        for (int q = 0; q < PER; ++q) {
+            const int i = threadIdx.x + 256 * q, t = i / (RANK / 4), d = 4 * (i % (RANK / 4));
+            uint32_t *dst = reinterpret_cast<uint32_t *>(cop + t * COP_LD + d);
+            dst[0] = (uint32_t)f2bf(c4[q].x) | ((uint32_t)f2bf(c4[q].y) << 16);
+            dst[1] = (uint32_t)f2bf(c4[q].z) | ((uint32_t)f2bf(c4[q].w) << 16);
+        }
     }
     __syncthreads();
     // u = sigma(W_1 c): warp w -> 8 output rows, both token tiles
@@ -505,7 +556,7 @@ __device__ __forceinline__ void mlp_share_mma(const Params &p, cg::cluster_group
             a[1] = *reinterpret_cast<const uint32_t *>(arow1 + ks * 16 + 2 * tq);
             a[2] = *reinterpret_cast<const uint32_t *>(arow0 + ks * 16 + 8 + 2 * tq);
             a[3] = *reinterpret_cast<const uint32_t *>(arow1 + ks * 16 + 8 + 2 * tq);
-            mma_bf16_16816(acc, a, b1f[ks][0], b1f[ks][1]);
+            mma_bf16_16816(acc, a, fr.b1[ks][0], fr.b1[ks][1]);
         }
         const int col = 8 * warp + 2 * tq;          // local W_1 row (0..63)
         const int t0 = mt * 16 + g, t1 = t0 + 8;
@@ -516,15 +567,22 @@ __device__ __forceinline__ void mlp_share_mma(const Params &p, cg::cluster_group
     }
     cluster.sync();
     // all of u from the cluster (16-byte pieces of the peers' rows)
-    for (int i = threadIdx.x; i < cnt * (2 * RANK / 8); i += blockDim.x) {
-        const int t = i / (2 * RANK / 8), f = 8 * (i % (2 * RANK / 8));
-        const uint16_t *peer = cluster.map_shared_rank(uown, f / 64);
-        *reinterpret_cast<uint4 *>(uop + t * UOP_LD + f) =
-            *reinterpret_cast<const uint4 *>(peer + t * UOWN_LD + (f % 64));
-    }
-    for (int i = threadIdx.x; i < (32 - cnt) * (2 * RANK / 8); i += blockDim.x) {
-        const int t = cnt + i / (2 * RANK / 8), f = 8 * (i % (2 * RANK / 8));
-        *reinterpret_cast<uint4 *>(uop + t * UOP_LD + f) = make_uint4(0, 0, 0, 0);
+    {
+        constexpr int PER = 32 * (2 * RANK / 8) / 256;   // 8 uint4 per thread
+        uint4 u4[PER];
+#pragma unroll
+        for (int q = 0; q < PER; ++q) {
+            const int i = threadIdx.x + 256 * q, t = i / (2 * RANK / 8), f = 8 * (i % (2 * RANK / 8));
+            u4[q] = make_uint4(0, 0, 0, 0);
+            if (t < cnt)
+                u4[q] = *reinterpret_cast<const uint4 *>(cluster.map_shared_rank(uown, f / 64) + t * UOWN_LD +
+                                                         (f % 64));
+        }
+#pragma unroll
+        for (int q = 0; q < PER; ++q) {
+            const int i = threadIdx.x + 256 * q, t = i / (2 * RANK / 8), f = 8 * (i % (2 * RANK / 8));
+            *reinterpret_cast<uint4 *>(uop + t * UOP_LD + f) = u4[q];
+        }
     }
     __syncthreads();
     // z = c + W_2 u: warp w -> 8 channels (w % 4), half of K (w / 4); the two
@@ -540,7 +598,7 @@ __device__ __forceinline__ void mlp_share_mma(const Params &p, cg::cluster_group
             a[1] = *reinterpret_cast<const uint32_t *>(arow1 + ks * 16 + 2 * tq);
             a[2] = *reinterpret_cast<const uint32_t *>(arow0 + ks * 16 + 8 + 2 * tq);
             a[3] = *reinterpret_cast<const uint32_t *>(arow1 + ks * 16 + 8 + 2 * tq);
-            mma_bf16_16816(acc, a, b2f[ks][0], b2f[ks][1]);
+            mma_bf16_16816(acc, a, fr.b2[ks][0], fr.b2[ks][1]);
         }
         const int col = 8 * (warp & 3) + 2 * tq;
         const int t0 = mt * 16 + g;
@@ -564,10 +622,15 @@ __device__ __forceinline__ void mlp_share_mma(const Params &p, cg::cluster_group
 // sigma(W_1 c) are exchanged through distributed shared memory.
 __global__ void __cluster_dims__(MLP_CLUSTER, 1, 1) __launch_bounds__(256) k_mix_mlp(const Params *__restrict__ pp)
 {
+    const unsigned long long t_start = globaltimer_ns();
+    pdl_trigger();                     // the Read kernel may start its prologue
     const Params &p = *pp;
     cg::cluster_group cluster = cg::this_cluster();
     const int rank = (int)cluster.block_rank();
     const int s = blockIdx.y, B = p.B;
+    MlpFrags fr;
+    if (p.dtype) load_mlp_frags(p, rank, fr);
+    pdl_wait();                        // the previous pass (or the precompute) is complete
     const SeqState st = p.st[s];
     if (!st.active) return;            // uniform over the cluster
     const int m = st.m, cnt = B - 1 - m, off = st.off;
@@ -603,13 +666,14 @@ __global__ void __cluster_dims__(MLP_CLUSTER, 1, 1) __launch_bounds__(256) k_mix
         uint16_t *cop = reinterpret_cast<uint16_t *>(dyn);
         uint16_t *uop = cop + 32 * COP_LD;
         uint16_t *uo = uop + 32 * UOP_LD;
-        mlp_share_mma(p, cluster, rank, cnt, m, s, off, cown, cop, uop, uo);
+        mlp_share_mma(p, cluster, rank, cnt, m, s, off, cown, cop, uop, uo, fr);
     } else {
         float *cop = dyn;
         float *uop = dyn + MAX_B * RANK;
         mlp_share<float, false>(p, cluster, rank, cnt, m, s, off, cown, uown, cop, uop, nullptr);
     }
     cluster.sync();                     // peers may still read our shared memory
+    if (threadIdx.x == 0 && p.trace) trace_mark(p.trace, 8 + 4 * p.ctl[CTL_PASS], t_start);
 }
 
 // ------------------------------------------------------------ k_read_simt
@@ -704,8 +768,11 @@ __global__ void __launch_bounds__(256) k_read_simt(const Params *__restrict__ pp
 // and sets the WHILE condition of the graph.
 __global__ void __launch_bounds__(1024) k_reduce(const Params *__restrict__ pp, cudaGraphConditionalHandle handle)
 {
+    const unsigned long long t_start = globaltimer_ns();
+    pdl_wait();
     const Params &p = *pp;
     const int s = blockIdx.x, B = p.B, warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const int tr_slot = 8 + 4 * p.ctl[CTL_PASS] + 2;
     const SeqState st = p.st[s];
     __shared__ int last;
     __shared__ int ynew[MAX_B], yold[MAX_B];
@@ -809,44 +876,61 @@ __global__ void __launch_bounds__(1024) k_reduce(const Params *__restrict__ pp, 
         }
         __threadfence();
         last = atomicAdd(&p.ctl[CTL_DONE], 1) == p.b - 1;
+        if (!last) trace_mark(p.trace, tr_slot, t_start);
     }
     __syncthreads();
     if (!last) return;
     __threadfence();
-    __shared__ int total;
-    // pack the positions of the next pass (b <= 1024 blocks per call)
-    if (threadIdx.x == 0) {
-        int acc = 0;
-        for (int q = 0; q < p.b; ++q) {
-            SeqState ns;
+    // pack the positions of the next pass: states read in parallel, block-wide
+    // exclusive scan of the counts, then the packed token list
+    __shared__ int wsum[32];
+    int carry = 0;
+    for (int q0 = 0; q0 < p.b; q0 += 1024) {
+        const int q = q0 + threadIdx.x;
+        SeqState ns{};
+        int c = 0;
+        if (q < p.b) {
             const volatile int *src = reinterpret_cast<const volatile int *>(&p.st[q]);
             ns.active = src[0]; ns.m = src[1]; ns.iters = src[2]; ns.converged = src[3];
-            ns.pad0 = ns.pad1 = 0;
-            if (ns.active) {
-                ns.off = acc;
-                ns.cnt = B - 1 - ns.m;
-                acc += ns.cnt;
-            } else {
-                ns.cnt = 0;
-            }
-            p.st[q] = ns;
+            c = ns.active ? B - 1 - ns.m : 0;
         }
-        total = acc;
-    }
-    __syncthreads();
-    for (int q = warp; q < p.b; q += 32) {
-        const SeqState ns = p.st[q];
-        if (ns.active)
-            for (int t = lane; t < ns.cnt; t += 32) p.act_tok[ns.off + t] = q * B + ns.m + 1 + t;
+        int incl = c;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += v;
+        }
+        if (lane == 31) wsum[warp] = incl;
+        __syncthreads();
+        if (warp == 0) {
+            int w = wsum[lane];
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int v = __shfl_up_sync(0xffffffffu, w, o);
+                if (lane >= o) w += v;
+            }
+            wsum[lane] = w;
+        }
+        __syncthreads();
+        const int off = carry + (warp ? wsum[warp - 1] : 0) + incl - c;
+        if (q < p.b) {
+            ns.off = off;
+            ns.cnt = c;
+            p.st[q] = ns;
+            for (int t = 0; t < c; ++t) p.act_tok[off + t] = q * B + ns.m + 1 + t;
+        }
+        carry += wsum[31];
+        __syncthreads();
     }
     if (threadIdx.x == 0) {
         const int passes = p.ctl[CTL_PASS] + 1;
-        p.ctl[CTL_NACT] = total;
+        p.ctl[CTL_NACT] = carry;
         p.ctl[CTL_DONE] = 0;
         p.ctl[CTL_PASS] = passes;
         // no block can take part in more than K_max passes; the cap also bounds
         // the loop should the per-block bookkeeping ever disagree
-        if (p.use_graph) cudaGraphSetConditional(handle, (total > 0 && passes < p.K_max) ? 1u : 0u);
+        if (p.use_graph) cudaGraphSetConditional(handle, (carry > 0 && passes < p.K_max) ? 1u : 0u);
+        trace_mark(p.trace, tr_slot, t_start);
     }
 }
 

@@ -79,6 +79,7 @@ struct Layout {
 struct xpress_refiner {
     xpress_weights w{};
     float *Ep = nullptr;
+    unsigned long long *trace = nullptr;   // profiling timeline (XPRESS_TRACE=1)
     CUtensorMap tmap_wr{};
     int device = 0;
     int num_sms = 0;
@@ -160,6 +161,7 @@ Params make_params(const xpress_refiner *R, const xpress_block_in *in, const xpr
     P.offset = in->offset;
     P.S = L.S;
     P.use_graph = 1;
+    P.trace = R->trace;
     P.ksplit = L.ksplit;
     P.h = in->h;
     P.s = in->s;
@@ -224,6 +226,25 @@ int set_kernel_attributes()
         }
     });
     return rc;
+}
+
+// Launch with programmatic stream serialization: the kernel may start while
+// its predecessor finishes and waits for it with griddepcontrol.wait.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       Args... args)
+{
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
 void launch_pre_gemm(const Layout &L, int N, Params *pdev, cudaStream_t st)
@@ -312,12 +333,13 @@ int build_graph(xpress_refiner *R, GraphEntry &e, const Params &P, const Layout 
     }
     cudaGraph_t body = cp.conditional.phGraph_out[0];
     XP_CUDA(cudaStreamBeginCaptureToGraph(cs, body, nullptr, nullptr, 0, cudaStreamCaptureModeThreadLocal));
-    k_mix_mlp<<<dim3(8, b), 256, mix_mlp_smem(P.dtype), cs>>>(pdev);
+    XP_CUDA(launch_pdl(k_mix_mlp, dim3(8, b), dim3(256), mix_mlp_smem(P.dtype), cs, (const Params *)pdev));
     if (R->use_tc)
-        k_read_tc<<<L.S, kReadTcThreads, kReadTcSmemBytes, cs>>>(pdev, R->tmap_wr, tmap_z);
+        XP_CUDA(launch_pdl(k_read_tc, dim3(L.S), dim3(kReadTcThreads), kReadTcSmemBytes, cs, (const Params *)pdev,
+                           R->tmap_wr, tmap_z, R->w.V));
     else
         k_read_simt<<<L.S, 256, READ_SIMT_DYN_SMEM, cs>>>(pdev);
-    k_reduce<<<b, 1024, 0, cs>>>(pdev, handle);
+    XP_CUDA(launch_pdl(k_reduce, dim3(b), dim3(1024), 0, cs, (const Params *)pdev, handle));
     cudaGraph_t body_out = nullptr;
     XP_CUDA(cudaStreamEndCapture(cs, &body_out));
     XP_CUDA(cudaGraphInstantiate(&e.exec, g, 0));
@@ -399,7 +421,7 @@ int run_eager(xpress_refiner *R, Params P, const Layout &L, void *ws, cudaStream
         kt.stop();
         kt.start("read");
         if (R->use_tc)
-            k_read_tc<<<L.S, kReadTcThreads, kReadTcSmemBytes, st>>>(pdev, R->tmap_wr, tmap_z);
+            k_read_tc<<<L.S, kReadTcThreads, kReadTcSmemBytes, st>>>(pdev, R->tmap_wr, tmap_z, R->w.V);
         else
             k_read_simt<<<L.S, 256, READ_SIMT_DYN_SMEM, st>>>(pdev);
         kt.stop();
@@ -423,6 +445,31 @@ int eager_mode()
         return (e && (e[0] == '1' || e[0] == '2')) ? e[0] - '0' : 0;
     }();
     return mode;
+}
+
+// Prints the device timeline of the call just launched (XPRESS_TRACE=1):
+// per kernel, start and end in microseconds from the first kernel's start.
+void print_trace(xpress_refiner *R, cudaStream_t st)
+{
+    unsigned long long h[2 * TRACE_SLOTS];
+    if (cudaMemcpyAsync(h, R->trace, sizeof(h), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+        cudaStreamSynchronize(st) != cudaSuccess)
+        return;
+    unsigned long long t0 = ~0ull;
+    for (int i = 0; i < TRACE_SLOTS; ++i)
+        if (h[i] < t0) t0 = h[i];
+    static const char *pre[4] = {"init", "seed", "pregemm", "premix"};
+    static const char *body[3] = {"mlp", "read", "reduce"};
+    std::fprintf(stderr, "xpress-trace:");
+    for (int i = 0; i < TRACE_SLOTS; ++i) {
+        if (h[i] == ~0ull) continue;
+        char name[32];
+        if (i >= 200) std::snprintf(name, sizeof(name), "readphase%d", i - 200);
+        else if (i < 8) std::snprintf(name, sizeof(name), "%s", i < 4 ? pre[i] : "?");
+        else std::snprintf(name, sizeof(name), "%s%d", (i - 8) % 4 < 3 ? body[(i - 8) % 4] : "?", (i - 8) / 4);
+        std::fprintf(stderr, " %s=[%.1f,%.1f]", name, (h[i] - t0) / 1000.0, (h[TRACE_SLOTS + i] - t0) / 1000.0);
+    }
+    std::fprintf(stderr, "\n");
 }
 
 int check_ws(void *ws, size_t ws_bytes, size_t need)
@@ -477,6 +524,11 @@ int xpress_refiner_create(const xpress_weights *w, void *stream, xpress_refiner 
             rc = XPRESS_ERR_CUDA;
             break;
         }
+        if (const char *tr = std::getenv("XPRESS_TRACE"))
+            if (tr[0] == '1' && cudaMalloc(&R->trace, 2 * TRACE_SLOTS * sizeof(unsigned long long)) != cudaSuccess) {
+                rc = XPRESS_ERR_CUDA;
+                break;
+            }
         if (cudaMalloc(&R->Ep, (size_t)w->V * RANK * sizeof(float)) != cudaSuccess ||
             cudaStreamCreateWithFlags(&R->cs, cudaStreamNonBlocking) != cudaSuccess) {
             rc = XPRESS_ERR_CUDA;
@@ -501,6 +553,7 @@ int xpress_refiner_destroy(xpress_refiner *R)
     for (auto &e : R->cache) destroy_entry(e);
     if (R->Ep) cudaFree(R->Ep);
     if (R->cs) cudaStreamDestroy(R->cs);
+    if (R->trace) cudaFree(R->trace);
     delete R;
     return XPRESS_OK;
 }
@@ -558,7 +611,13 @@ int xpress_refine_block(const xpress_refiner *Rc, const xpress_block_in *in, con
     kp.blockDim = dim3(256);
     kp.kernelParams = args;
     XP_CUDA(cudaGraphExecKernelNodeSetParams(hit->exec, hit->init_node, &kp));
-    XP_CUDA(cudaGraphLaunch(hit->exec, static_cast<cudaStream_t>(stream)));
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (R->trace) {
+        XP_CUDA(cudaMemsetAsync(R->trace, 0xFF, TRACE_SLOTS * sizeof(unsigned long long), st));
+        XP_CUDA(cudaMemsetAsync(R->trace + TRACE_SLOTS, 0, TRACE_SLOTS * sizeof(unsigned long long), st));
+    }
+    XP_CUDA(cudaGraphLaunch(hit->exec, st));
+    if (R->trace) print_trace(R, st);
     return XPRESS_OK;
 }
 
@@ -673,7 +732,7 @@ int xpress_profile_read(const xpress_refiner *R, void *ws, int b, void *stream)
     if (R->use_tc) {
         CUtensorMap tmap_z{};
         if (!make_tmap_bf16(&tmap_z, w + L.zpack, RANK, (uint64_t)b * R->w.B, 64, 32)) return XPRESS_ERR_CUDA;
-        k_read_tc<<<L.S, kReadTcThreads, kReadTcSmemBytes, st>>>(pdev, R->tmap_wr, tmap_z);
+        k_read_tc<<<L.S, kReadTcThreads, kReadTcSmemBytes, st>>>(pdev, R->tmap_wr, tmap_z, R->w.V);
     } else {
         k_read_simt<<<L.S, 256, READ_SIMT_DYN_SMEM, st>>>(pdev);
     }
