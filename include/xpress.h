@@ -172,6 +172,31 @@ size_t xpress_accept_workspace_size(const xpress_refiner *refiner, int b);
 int xpress_accept(const xpress_refiner *refiner, const xpress_accept_in *in, int32_t *accept_len,
                   int32_t *out_tokens, void *workspace, size_t ws_bytes, void *stream);
 
+/* xpress_accept for callers that cannot allocate device memory (code that
+ * runs while another thread captures a CUDA graph, allocators that forbid
+ * device allocations after start-up, hosts that only hand out pre-registered
+ * buffers).  It takes no workspace: the acceptance kernels keep their scratch
+ * in a fixed 256 KiB array inside this library (a file-scope __device__
+ * array, held by every GPU that loads the library until the process exits).
+ * The paper has no counterpart to this entry point; it exists for such
+ * callers only.
+ *   - Same inputs, outputs and results as xpress_accept.
+ *   - Size limit: the scratch of the batch must fit the array, which holds
+ *     any batch with b * (B + 1) <= 8192 target rows on a 152-SM GB300;
+ *     larger batches return XPRESS_ERR_UNSUPPORTED (use xpress_accept).
+ *   - Allocates nothing: no cudaMalloc, no cudaFree, no allocating library
+ *     call.  Its first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress, once per device, with that device current);
+ *     make that first call before any stream capture.
+ *   - Every call shares the one array, which keeps the previous call's
+ *     contents: calls that overlap on the GPU (other streams, other threads)
+ *     race on it and must be serialised by the caller.  The device status of
+ *     these calls is not reported (xpress_get_device_status needs a
+ *     workspace).
+ * Errors: INVALID_ARG, UNSUPPORTED (batch too large), CUDA. */
+int xpress_accept_noalloc(const xpress_refiner *refiner, const xpress_accept_in *in, int32_t *accept_len,
+                          int32_t *out_tokens, void *stream);
+
 /* Synchronises `stream`, then reads (and clears) the device status word kept
  * in `workspace` by xpress_refine_block / xpress_accept.  *status_out is an
  * xpress_status (XPRESS_OK, XPRESS_ERR_TIMEOUT or XPRESS_ERR_DEVICE_CHECK). */

@@ -86,6 +86,8 @@ def load(path: str = LIB_PATH):
     lib.xpress_get_device_status.restype = I
     lib.xpress_get_pass_count.argtypes = [P, P, C.POINTER(C.c_int32)]
     lib.xpress_get_pass_count.restype = I
+    lib.xpress_accept_noalloc.argtypes = [P, C.POINTER(XpressAcceptIn), P, P, P]
+    lib.xpress_accept_noalloc.restype = I
     lib.xpress_profile_read_prepare.argtypes = [P, P, I, I, P]
     lib.xpress_profile_read_prepare.restype = I
     lib.xpress_profile_read.argtypes = [P, P, I, P]
@@ -141,6 +143,12 @@ def xpress_accept(handle, acc_in: XpressAcceptIn, accept_len_ptr: int, out_token
     _check("xpress_accept", load().xpress_accept(handle, C.byref(acc_in), C.c_void_p(accept_len_ptr),
                                                  C.c_void_p(out_tokens_ptr), C.c_void_p(ws_ptr), ws_bytes,
                                                  C.c_void_p(stream)))
+
+
+def xpress_accept_noalloc(handle, acc_in: XpressAcceptIn, accept_len_ptr: int, out_tokens_ptr: int,
+                          stream: int) -> None:
+    _check("xpress_accept_noalloc", load().xpress_accept_noalloc(handle, C.byref(acc_in), C.c_void_p(accept_len_ptr),
+                                                                 C.c_void_p(out_tokens_ptr), C.c_void_p(stream)))
 
 
 def xpress_get_device_status(ws_ptr: int, stream: int) -> int:

@@ -2,6 +2,7 @@
 #pragma once
 
 #include "common.cuh"
+#include "xpress.h"
 
 namespace xp {
 
@@ -53,6 +54,12 @@ inline int mix_mlp_smem(int dtype)
     return dtype ? (32 * (RANK + 8) + 32 * (2 * RANK + 8) + 32 * (64 + 8)) * 2 : MIX_MLP_DYN_SMEM_MAX;
 }
 constexpr int GEMV_SMEM = 128 * 1024;
+
+// acceptance launch shared by xpress_accept and xpress_accept_noalloc
+// (xpress_host.cu); `ws` holds the scratch laid out by accept_scratch_bytes
+size_t accept_scratch_bytes(const xpress_refiner *R, int b);
+int accept_launch(const xpress_refiner *R, const xpress_accept_in *in, int32_t *accept_len, int32_t *out_tokens,
+                  void *ws, size_t ws_bytes, void *stream);
 constexpr int READ_SIMT_DYN_SMEM = (32 * (RANK + 1) + 8 * 32 * 33) * 4;
 inline int pre_mix_smem(int B) { return (B * 2 * RANK + RANK + 32 * (2 * RANK + 1) + B * 32) * 4; }
 

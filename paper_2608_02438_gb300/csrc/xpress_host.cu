@@ -649,13 +649,17 @@ AcceptLayout accept_layout(const xpress_refiner *R, int b)
 }
 }  // namespace
 
-size_t xpress_accept_workspace_size(const xpress_refiner *R, int b)
+}  // extern "C"
+
+namespace xp {
+
+size_t accept_scratch_bytes(const xpress_refiner *R, int b)
 {
     if (!R || b < 1) return 0;
     return accept_layout(R, b).total;
 }
 
-int xpress_accept(const xpress_refiner *R, const xpress_accept_in *in, int32_t *accept_len, int32_t *out_tokens,
+int accept_launch(const xpress_refiner *R, const xpress_accept_in *in, int32_t *accept_len, int32_t *out_tokens,
                   void *ws, size_t ws_bytes, void *stream)
 {
     if (!R || !in || !accept_len || !out_tokens) return XPRESS_ERR_INVALID_ARG;
@@ -695,6 +699,23 @@ int xpress_accept(const xpress_refiner *R, const xpress_accept_in *in, int32_t *
     k_acc_finish<<<(in->b + 127) / 128, 128, 0, st>>>(P, A.chunks2);
     XP_CUDA(cudaGetLastError());
     return XPRESS_OK;
+}
+
+}  // namespace xp
+
+extern "C" {
+
+
+size_t xpress_accept_workspace_size(const xpress_refiner *R, int b)
+{
+    if (!R || b < 1) return 0;
+    return accept_layout(R, b).total;
+}
+
+int xpress_accept(const xpress_refiner *R, const xpress_accept_in *in, int32_t *accept_len, int32_t *out_tokens,
+                  void *ws, size_t ws_bytes, void *stream)
+{
+    return xp::accept_launch(R, in, accept_len, out_tokens, ws, ws_bytes, stream);
 }
 
 int xpress_get_device_status(void *ws, void *stream, int32_t *status_out)
