@@ -126,7 +126,8 @@ def _lm_head_logits(rng, h32: np.ndarray, V: int) -> np.ndarray:
 
 def _gumbel_sample(rng, logits: np.ndarray) -> np.ndarray:
     """Drafter-side sampling of Y^(0) from softmax(s) (the drafter, not the refiner)."""
-    g = -np.log(-np.log(rng.uniform(1e-12, 1.0, size=logits.shape).astype(np.float32)))
+    u = rng.random(size=logits.shape) * (1.0 - 2e-12) + 1e-12      # float64, strictly inside (0, 1)
+    g = (-np.log(-np.log(u))).astype(np.float32)
     return np.argmax(logits + g, axis=-1).astype(np.int32)
 
 

@@ -172,3 +172,48 @@ def test_accept_tiny(X, temps):
 def test_accept_qwen3_shape(X, name):
     cfg, w, inp = W.make_workload(name)
     _accept_check(X, cfg, w, inp)
+
+
+# ------------------------------------------------- full-size batched configs
+
+def _consistent_drafts(cfg, w, inp):
+    """Blocks flagged `consistent` get the oracle's fixed point as their draft
+    (so they converge in one pass); computed by the oracle only."""
+    m = oracle_model(cfg, w)
+    for i in np.nonzero(inp["consistent"])[0]:
+        o = O.jacobi(m, inp["h"][i], inp["s"][i], int(inp["anchor"][i]), inp["draft"][i],
+                     float(inp["temperature"][i]), int(inp["seed"][i]), inp["offset"], cfg.B)
+        inp["draft"][i] = o["tokens"]
+    return inp
+
+
+@pytest.mark.parametrize("name,sample", [("serving_b32", (0, 5, 17, 31)), ("long_b64", (0, 1, 38, 63))])
+def test_batched_full_size_sampled(X, name, sample):
+    cfg, w, inp = W.make_workload(name)
+    if cfg.consistent_frac > 0:
+        inp = _consistent_drafts(cfg, w, inp)
+        sample = tuple(sorted(set(sample) | {int(np.nonzero(inp["consistent"])[0][0])}))
+    ref, d, g = _run(X, cfg, w, inp)
+    m = oracle_model(cfg, w)
+    orc = {i: run_oracle(m, inp, i, cfg.K_max) for i in sample}
+    sub = {k: (v[list(sample)] if v is not None else None) for k, v in g.items()}
+    compare_blocks(sub, orc, list(sample), cfg.dtype, inp=inp)
+    # properties over every block: pass counts within [1, K_max]; blocks whose
+    # draft is already the fixed point converge in exactly one pass
+    assert (g["iters"] >= 1).all() and (g["iters"] <= cfg.K_max).all()
+    if cfg.consistent_frac > 0:
+        cons = inp["consistent"]
+        assert (g["iters"][cons] == 1).all() and (g["converged"][cons] == 1).all()
+        np.testing.assert_array_equal(g["tokens"][cons], inp["draft"][cons])
+    # acceptance on the same blocks
+    out_dev = ref.refine_block(d["h"], d["s"], d["draft"], d["anchor"], d["temperature"], d["seed"], inp["offset"],
+                               cfg.K_max)
+    acc = ref.accept(d["target"], d["s"], out_dev["tokens"], out_dev["lse"], out_dev["logit_sel"],
+                     out_dev["z_final"], d["temperature"], d["seed"], inp["offset"])
+    torch.cuda.synchronize()
+    alen, otok = acc["accept_len"].cpu().numpy(), acc["out_tokens"].cpu().numpy()
+    for i in sample:
+        o = orc[i]
+        n, out, mg = O.accept(m, inp["target"][i], inp["s"][i], o["tokens"], o["lse"], o["sel"], o["z_final"],
+                              float(inp["temperature"][i]), int(inp["seed"][i]), inp["offset"])
+        assert (int(alen[i]) == n and otok[i].tolist() == out.tolist()) or mg < 1e-3, (i, alen[i], n)
