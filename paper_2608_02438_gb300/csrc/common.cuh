@@ -62,6 +62,7 @@ struct Params {
     int S;                       // vocabulary ranges of the Read kernel
     int use_graph;               // 1: the pass loop is a graph WHILE node
     unsigned long long *trace;   // optional kernel timeline (profiling), else NULL
+    int read_flags;              // experiments: bit 0 = no L2 bulk prefetch of W_r
     int ksplit;                  // split-K factor of the hidden projection
     // inputs (caller-owned)
     const void *h, *s;

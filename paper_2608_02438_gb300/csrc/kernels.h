@@ -40,6 +40,14 @@ __global__ void k_read_tc(const Params *pp, const __grid_constant__ CUtensorMap 
 extern const size_t kReadTcSmemBytes;
 extern const int kReadTcThreads;
 
+// read_tcv.cu (at most 32 evaluated tokens: vocabulary rows as the MMA M)
+__global__ void k_read_tcv(const Params *pp, const __grid_constant__ CUtensorMap tmap_wr128,
+                           const __grid_constant__ CUtensorMap tmap_z, int V, int fuse,
+                           cudaGraphConditionalHandle handle);
+extern const size_t kReadTcvSmemBytes;
+extern const int kReadTcvThreads;
+constexpr int TCV_MAX_TOKENS = 32;
+
 // accept_kernels.cu
 __global__ void k_acc_rows(AcceptParams p);
 __global__ void k_acc_decide(AcceptParams p, int chunks);

@@ -1,0 +1,238 @@
+// reduce_common.cuh -- the end-of-pass step shared by k_reduce and the fused
+// reduce of k_read_tcv: combine the split-vocabulary partials of a token,
+// finish the T > 0 draw inside the winning group, apply Algorithm 1's
+// stopping rule to a block, and pack the positions of the next pass.
+#pragma once
+
+#include "common.cuh"
+
+namespace xp {
+
+__device__ __forceinline__ void bf16x8_to_float(const uint4 &w, float (&x)[8])
+{
+    const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        x[2 * q] = __uint_as_float(ww[q] << 16);
+        x[2 * q + 1] = __uint_as_float(ww[q] & 0xFFFF0000u);
+    }
+}
+
+struct TokenResult {
+    int y;
+    float sel, lse;
+};
+
+// Warp-collective: the re-selected token of packed token i (global token id
+// tok = seq * B + k).  Combines the S partials in a fixed tree (deterministic);
+// T > 0 recomputes l = s + W_r z over the 32 members of the drawn group and
+// draws one by Gumbel-max (the second level of the hierarchical draw).
+__device__ __forceinline__ TokenResult reduce_token(const Params &p, int i, int tok, float invT,
+                                                    unsigned long long seed)
+{
+    const int lane = threadIdx.x % 32, k = tok % p.B;
+    const bool sampling = invT > 0.0f;
+    Partial a{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
+    // the lane's partials (ranges lane, lane + 32, ...) requested together
+    constexpr int PER = 8;
+    for (int r0 = 0; r0 < p.S; r0 += 32 * PER) {
+        Partial pv[PER];
+#pragma unroll
+        for (int j = 0; j < PER; ++j) {
+            const int r = r0 + lane + 32 * j;
+            pv[j] = r < p.S ? p.part[(size_t)r * p.N + i] : Partial{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
+        }
+#pragma unroll
+        for (int j = 0; j < PER; ++j) merge_partial(a, pv[j], sampling);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        Partial b;
+        b.best = __shfl_xor_sync(0xffffffffu, a.best, o);
+        b.idx = __shfl_xor_sync(0xffffffffu, a.idx, o);
+        b.m = __shfl_xor_sync(0xffffffffu, a.m, o);
+        b.s = __shfl_xor_sync(0xffffffffu, a.s, o);
+        merge_partial(a, b, sampling);
+    }
+    TokenResult res;
+    if (!sampling) {
+        res.y = a.idx;
+        res.sel = a.best;
+        res.lse = __int_as_float(0x7fc00000);
+        return res;
+    }
+    const int v = a.idx * GROUP + lane;
+    float x = -INFINITY, score = -INFINITY;
+    if (v < p.V) {
+        float acc = 0.0f;
+        if (p.dtype) {
+            const uint4 *wr = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.W_r) + (size_t)v * RANK);
+            const uint4 *zr = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.zpack) + (size_t)i * RANK);
+#pragma unroll 8
+            for (int c = 0; c < RANK / 8; ++c) {
+                float w8[8], z8[8];
+                bf16x8_to_float(__ldg(wr + c), w8);
+                bf16x8_to_float(zr[c], z8);
+#pragma unroll
+                for (int j = 0; j < 8; ++j) acc = fmaf(w8[j], z8[j], acc);
+            }
+        } else {
+            for (int d = 0; d < RANK; ++d)
+                acc = fmaf(ld_any(p.W_r, 0, (size_t)v * RANK + d), ld_any(p.zpack, 0, (size_t)i * RANK + d), acc);
+        }
+        x = (acc + ld_any(p.s, p.dtype, (size_t)tok * p.V + v)) * invT;
+        score = x + gumbel(seed, (uint32_t)v, (uint32_t)k, STREAM_ELEM, p.offset);
+    }
+    float bs = score;
+    int bi = v;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float os = __shfl_xor_sync(0xffffffffu, bs, o);
+        const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+        merge_argmax(bs, bi, os, oi);
+    }
+    res.y = bi;
+    res.sel = __shfl_sync(0xffffffffu, x, (bi - a.idx * GROUP) & (GROUP - 1));
+    res.lse = a.m + logf(a.s);
+    return res;
+}
+
+// Algorithm 1's stopping rule for block s after a pass that evaluated
+// positions m+1..B-1: ynew[base + k] / yold[base + k] hold the new and the
+// previous token of evaluated position k.  Single thread.
+__device__ __forceinline__ SeqState converge_state(const Params &p, const SeqState &st, const int *ynew,
+                                                   const int *yold, int base)
+{
+    const int B = p.B;
+    int first = -1;
+    for (int k = st.m + 1; k < B; ++k)
+        if (ynew[base + k] != yold[base + k]) { first = k; break; }
+    SeqState ns = st;
+    ns.iters = st.iters + 1;
+    ns.converged = first < 0;
+    if (p.fixed_K) {
+        ns.active = ns.iters < p.K_max;
+        ns.m = -1;
+    } else if (first < 0 || ns.iters >= p.K_max) {
+        ns.active = 0;
+    } else if (first == B - 1) {
+        // the next pass would evaluate no position and change nothing:
+        // it is Algorithm 1's final, unchanged pass
+        ns.iters += 1;
+        ns.converged = 1;
+        ns.active = 0;
+    } else {
+        ns.active = 1;
+        ns.m = first;
+    }
+    return ns;
+}
+
+__device__ __forceinline__ void converge_block(const Params &p, int s, const SeqState &st, const int *ynew,
+                                               const int *yold, int base)
+{
+    const SeqState ns = converge_state(p, st, ynew, yold, base);
+    p.st[s] = ns;
+    if (p.iters) p.iters[s] = ns.iters;
+    if (p.converged) p.converged[s] = ns.converged;
+}
+
+// Warp-collective version of converge + pack for at most 32 blocks whose
+// states sit in shared memory (lane q: block q): applies the stopping rule,
+// scans the counts, writes the states, the packed token list and the control
+// words, and sets the loop condition.
+__device__ __forceinline__ void converge_pack_small(const Params &p, const SeqState *st_in, const int *ynew,
+                                                    const int *yold, int passes_before,
+                                                    cudaGraphConditionalHandle handle)
+{
+    const int q = threadIdx.x % 32, B = p.B;
+    SeqState ns{};
+    int c = 0;
+    if (q < p.b) {
+        const SeqState st = st_in[q];
+        ns = st.active ? converge_state(p, st, ynew, yold, st.off - st.m - 1) : st;
+        if (st.active) {
+            if (p.iters) p.iters[q] = ns.iters;
+            if (p.converged) p.converged[q] = ns.converged;
+        }
+        c = ns.active ? B - 1 - ns.m : 0;
+    }
+    int incl = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int v = __shfl_up_sync(0xffffffffu, incl, o);
+        if (q >= o) incl += v;
+    }
+    const int total = __shfl_sync(0xffffffffu, incl, 31);
+    if (q < p.b) {
+        ns.off = incl - c;
+        ns.cnt = c;
+        p.st[q] = ns;
+        for (int t = 0; t < c; ++t) p.act_tok[ns.off + t] = q * B + ns.m + 1 + t;
+    }
+    if (q == 0) {
+        const int passes = passes_before + 1;
+        p.ctl[CTL_NACT] = total;
+        p.ctl[CTL_DONE] = 0;
+        p.ctl[CTL_PASS] = passes;
+        if (p.use_graph) cudaGraphSetConditional(handle, (total > 0 && passes < p.K_max) ? 1u : 0u);
+    }
+}
+
+// Block-collective (any multiple of 32 threads): packs the positions of the
+// next pass (exclusive scan of the per-block counts), updates the control
+// words and sets the graph's loop condition.  Call after every block state of
+// this pass is final and visible.
+__device__ __forceinline__ void pack_next_pass(const Params &p, cudaGraphConditionalHandle handle, int *wsum)
+{
+    const int B = p.B, warp = threadIdx.x / 32, lane = threadIdx.x % 32, nwarps = blockDim.x / 32;
+    int carry = 0;
+    for (int q0 = 0; q0 < p.b; q0 += blockDim.x) {
+        const int q = q0 + threadIdx.x;
+        SeqState ns{};
+        int c = 0;
+        if (q < p.b) {
+            const volatile int *src = reinterpret_cast<const volatile int *>(&p.st[q]);
+            ns.active = src[0]; ns.m = src[1]; ns.iters = src[2]; ns.converged = src[3];
+            c = ns.active ? B - 1 - ns.m : 0;
+        }
+        int incl = c;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += v;
+        }
+        if (lane == 31) wsum[warp] = incl;
+        __syncthreads();
+        if (warp == 0) {
+            int w = lane < nwarps ? wsum[lane] : 0;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int v = __shfl_up_sync(0xffffffffu, w, o);
+                if (lane >= o) w += v;
+            }
+            wsum[lane] = w;
+        }
+        __syncthreads();
+        const int off = carry + (warp ? wsum[warp - 1] : 0) + incl - c;
+        if (q < p.b) {
+            ns.off = off;
+            ns.cnt = c;
+            p.st[q] = ns;
+            for (int t = 0; t < c; ++t) p.act_tok[off + t] = q * B + ns.m + 1 + t;
+        }
+        carry += wsum[nwarps - 1];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) {
+        const int passes = p.ctl[CTL_PASS] + 1;
+        p.ctl[CTL_NACT] = carry;
+        p.ctl[CTL_DONE] = 0;
+        p.ctl[CTL_PASS] = passes;
+        // no block can take part in more than K_max passes; the cap also bounds
+        // the loop should the per-block bookkeeping ever disagree
+        if (p.use_graph) cudaGraphSetConditional(handle, (carry > 0 && passes < p.K_max) ? 1u : 0u);
+    }
+}
+
+}  // namespace xp

@@ -20,6 +20,7 @@
 
 #include "common.cuh"
 #include "kernels.h"
+#include "reduce_common.cuh"
 
 namespace cg = cooperative_groups;
 
@@ -631,6 +632,9 @@ __global__ void __cluster_dims__(MLP_CLUSTER, 1, 1) __launch_bounds__(256) k_mix
     MlpFrags fr;
     if (p.dtype) load_mlp_frags(p, rank, fr);
     pdl_wait();                        // the previous pass (or the precompute) is complete
+    const int trs = (p.trace && s == 0 && rank == 0 && threadIdx.x == 0 && p.ctl[CTL_PASS] < 2)
+                        ? 210 + 8 * p.ctl[CTL_PASS] : 0;
+    if (trs) trace_mark(p.trace, trs, t_start);
     const SeqState st = p.st[s];
     if (!st.active) return;            // uniform over the cluster
     const int m = st.m, cnt = B - 1 - m, off = st.off;
@@ -649,6 +653,7 @@ __global__ void __cluster_dims__(MLP_CLUSTER, 1, 1) __launch_bounds__(256) k_mix
         e[j][dd] = p.Ep[(size_t)x * RANK + d0 + dd];
     }
     __syncthreads();
+    if (trs) trace_mark(p.trace, trs + 1, t_start);
     for (int i = threadIdx.x; i < cnt * 32; i += blockDim.x) {
         const int t = i / 32, dd = i % 32, k = m + 1 + t, d = d0 + dd;
         float lrow[MAX_B];
@@ -661,7 +666,9 @@ __global__ void __cluster_dims__(MLP_CLUSTER, 1, 1) __launch_bounds__(256) k_mix
             if (j < k) acc = fmaf(lrow[j], e[j][dd], acc);
         cown[t][dd] = acc;
     }
+    if (trs) trace_mark(p.trace, trs + 2, t_start);
     cluster.sync();
+    if (trs) trace_mark(p.trace, trs + 3, t_start);
     if (p.dtype) {
         uint16_t *cop = reinterpret_cast<uint16_t *>(dyn);
         uint16_t *uop = cop + 32 * COP_LD;
@@ -672,7 +679,9 @@ __global__ void __cluster_dims__(MLP_CLUSTER, 1, 1) __launch_bounds__(256) k_mix
         float *uop = dyn + MAX_B * RANK;
         mlp_share<float, false>(p, cluster, rank, cnt, m, s, off, cown, uown, cop, uop, nullptr);
     }
+    if (trs) trace_mark(p.trace, trs + 4, t_start);
     cluster.sync();                     // peers may still read our shared memory
+    if (trs) trace_mark(p.trace, trs + 5, t_start);
     if (threadIdx.x == 0 && p.trace) trace_mark(p.trace, 8 + 4 * p.ctl[CTL_PASS], t_start);
 }
 
@@ -776,104 +785,22 @@ __global__ void __launch_bounds__(1024) k_reduce(const Params *__restrict__ pp, 
     const SeqState st = p.st[s];
     __shared__ int last;
     __shared__ int ynew[MAX_B], yold[MAX_B];
-    const float T = p.temperature[s];
-    const float invT = T > 0.0f ? 1.0f / T : 0.0f;
-    const bool sampling = invT > 0.0f;
+    __shared__ int wsum[32];
     if (st.active && warp < B && warp > st.m) {
         const int k = warp, i = st.off + (k - st.m - 1), tok = s * B + k;
         if (lane == 0) yold[k] = p.tokens[tok];
-        Partial a{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
-#pragma unroll 4
-        for (int r = lane; r < p.S; r += 32) merge_partial(a, p.part[(size_t)r * p.N + i], sampling);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            Partial b;
-            b.best = __shfl_xor_sync(0xffffffffu, a.best, o);
-            b.idx = __shfl_xor_sync(0xffffffffu, a.idx, o);
-            b.m = __shfl_xor_sync(0xffffffffu, a.m, o);
-            b.s = __shfl_xor_sync(0xffffffffu, a.s, o);
-            merge_partial(a, b, sampling);
-        }
-        int y;
-        float sel, lse;
-        if (!sampling) {
-            y = a.idx;
-            sel = a.best;
-            lse = __int_as_float(0x7fc00000);
-        } else {
-            // second stage: Gumbel-max over the members of the drawn group
-            const int v = a.idx * GROUP + lane;
-            float x = -INFINITY, score = -INFINITY;
-            if (v < p.V) {
-                float acc = 0.0f;
-                if (p.dtype) {
-                    const uint4 *wr = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.W_r) +
-                                                                      (size_t)v * RANK);
-                    const uint4 *zr = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.zpack) +
-                                                                      (size_t)i * RANK);
-#pragma unroll 8
-                    for (int c = 0; c < RANK / 8; ++c) {
-                        float w8[8], z8[8];
-                        bf16x8_to_f32(__ldg(wr + c), w8);
-                        bf16x8_to_f32(zr[c], z8);
-#pragma unroll
-                        for (int j = 0; j < 8; ++j) acc = fmaf(w8[j], z8[j], acc);
-                    }
-                } else {
-                    for (int d = 0; d < RANK; ++d)
-                        acc = fmaf(ld_any(p.W_r, 0, (size_t)v * RANK + d), ld_any(p.zpack, 0, (size_t)i * RANK + d),
-                                   acc);
-                }
-                x = (acc + ld_any(p.s, p.dtype, (size_t)tok * p.V + v)) * invT;
-                score = x + gumbel(p.seed[s], (uint32_t)v, (uint32_t)k, STREAM_ELEM, p.offset);
-            }
-            float bs = score;
-            int bi = v;
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                const float os = __shfl_xor_sync(0xffffffffu, bs, o);
-                const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-                merge_argmax(bs, bi, os, oi);
-            }
-            y = bi;
-            sel = __shfl_sync(0xffffffffu, x, (bi - a.idx * GROUP) & (GROUP - 1));
-            lse = a.m + logf(a.s);
-        }
+        const float T = p.temperature[s];
+        const TokenResult res = reduce_token(p, i, tok, T > 0.0f ? 1.0f / T : 0.0f, p.seed[s]);
         if (lane == 0) {
-            ynew[k] = y;
-            if (p.lse) p.lse[tok] = lse;
-            if (p.logit_sel) p.logit_sel[tok] = sel;
-            p.tokens[tok] = y;
+            ynew[k] = res.y;
+            if (p.lse) p.lse[tok] = res.lse;
+            if (p.logit_sel) p.logit_sel[tok] = res.sel;
+            p.tokens[tok] = res.y;
         }
     }
     __syncthreads();
     if (threadIdx.x == 0) {
-        if (st.active) {
-            int first = -1;
-            for (int k = st.m + 1; k < B; ++k)
-                if (ynew[k] != yold[k]) { first = k; break; }
-            SeqState ns = st;
-            ns.iters = st.iters + 1;
-            ns.converged = first < 0;
-            if (p.fixed_K) {
-                ns.active = ns.iters < p.K_max;
-                ns.m = -1;
-            } else if (first < 0 || ns.iters >= p.K_max) {
-                ns.active = 0;
-            } else if (first == B - 1) {
-                // the next pass would evaluate no position and change nothing:
-                // it is Algorithm 1's final, unchanged pass
-                ns.iters += 1;
-                ns.converged = 1;
-                ns.active = 0;
-            } else {
-                ns.active = 1;
-                ns.m = first;
-            }
-            p.st[s] = ns;
-            if (p.iters) p.iters[s] = ns.iters;
-            if (p.converged) p.converged[s] = ns.converged;
-        }
+        if (st.active) converge_block(p, s, st, ynew, yold, 0);
         __threadfence();
         last = atomicAdd(&p.ctl[CTL_DONE], 1) == p.b - 1;
         if (!last) trace_mark(p.trace, tr_slot, t_start);
@@ -881,57 +808,8 @@ __global__ void __launch_bounds__(1024) k_reduce(const Params *__restrict__ pp, 
     __syncthreads();
     if (!last) return;
     __threadfence();
-    // pack the positions of the next pass: states read in parallel, block-wide
-    // exclusive scan of the counts, then the packed token list
-    __shared__ int wsum[32];
-    int carry = 0;
-    for (int q0 = 0; q0 < p.b; q0 += 1024) {
-        const int q = q0 + threadIdx.x;
-        SeqState ns{};
-        int c = 0;
-        if (q < p.b) {
-            const volatile int *src = reinterpret_cast<const volatile int *>(&p.st[q]);
-            ns.active = src[0]; ns.m = src[1]; ns.iters = src[2]; ns.converged = src[3];
-            c = ns.active ? B - 1 - ns.m : 0;
-        }
-        int incl = c;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int v = __shfl_up_sync(0xffffffffu, incl, o);
-            if (lane >= o) incl += v;
-        }
-        if (lane == 31) wsum[warp] = incl;
-        __syncthreads();
-        if (warp == 0) {
-            int w = wsum[lane];
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const int v = __shfl_up_sync(0xffffffffu, w, o);
-                if (lane >= o) w += v;
-            }
-            wsum[lane] = w;
-        }
-        __syncthreads();
-        const int off = carry + (warp ? wsum[warp - 1] : 0) + incl - c;
-        if (q < p.b) {
-            ns.off = off;
-            ns.cnt = c;
-            p.st[q] = ns;
-            for (int t = 0; t < c; ++t) p.act_tok[off + t] = q * B + ns.m + 1 + t;
-        }
-        carry += wsum[31];
-        __syncthreads();
-    }
-    if (threadIdx.x == 0) {
-        const int passes = p.ctl[CTL_PASS] + 1;
-        p.ctl[CTL_NACT] = carry;
-        p.ctl[CTL_DONE] = 0;
-        p.ctl[CTL_PASS] = passes;
-        // no block can take part in more than K_max passes; the cap also bounds
-        // the loop should the per-block bookkeeping ever disagree
-        if (p.use_graph) cudaGraphSetConditional(handle, (carry > 0 && passes < p.K_max) ? 1u : 0u);
-        trace_mark(p.trace, tr_slot, t_start);
-    }
+    pack_next_pass(p, handle, wsum);
+    if (threadIdx.x == 0) trace_mark(p.trace, tr_slot, t_start);
 }
 
 // Profiling hook: the next Read pass evaluates tokens 0..n-1.

@@ -72,6 +72,7 @@ struct Layout {
            zbuf = 0, part = 0, total = 0;
     int ksplit = 1, kchunk = 0, S = 1;
     bool gemv = false;
+    bool tcv = false;
 };
 
 }  // namespace
@@ -80,7 +81,8 @@ struct xpress_refiner {
     xpress_weights w{};
     float *Ep = nullptr;
     unsigned long long *trace = nullptr;   // profiling timeline (XPRESS_TRACE=1)
-    CUtensorMap tmap_wr{};
+    CUtensorMap tmap_wr{};                 // W_r boxes of 256 rows (k_read_tc)
+    CUtensorMap tmap_wr128{};              // W_r boxes of 128 rows (k_read_tcv)
     int device = 0;
     int num_sms = 0;
     bool use_tc = false;
@@ -91,10 +93,14 @@ struct xpress_refiner {
 
 namespace {
 
-int read_S(const xpress_refiner *R)
+// k_read_tcv serves calls that evaluate at most 32 tokens (b * B <= 32)
+bool use_tcv(const xpress_refiner *R, int b) { return R->use_tc && b * R->w.B <= TCV_MAX_TOKENS; }
+
+int read_S(const xpress_refiner *R, int b)
 {
     if (R->use_tc) {
-        const int nvt = (R->w.V + 255) / 256;
+        const int rows = use_tcv(R, b) ? 128 : 256;
+        const int nvt = (R->w.V + rows - 1) / rows;
         return nvt < R->num_sms ? nvt : R->num_sms;
     }
     const int ng = (R->w.V + GROUP - 1) / GROUP;
@@ -137,7 +143,8 @@ Layout make_layout(const xpress_refiner *R, int b)
     o = align256(o + (size_t)N * RANK * esz);
     L.zbuf = o;
     o = align256(o + (size_t)N * RANK * 4);
-    L.S = read_S(R);
+    L.S = read_S(R, b);
+    L.tcv = use_tcv(R, b);
     L.part = o;
     o = align256(o + (size_t)L.S * N * sizeof(Partial));
     L.total = o;
@@ -162,6 +169,13 @@ Params make_params(const xpress_refiner *R, const xpress_block_in *in, const xpr
     P.S = L.S;
     P.use_graph = 1;
     P.trace = R->trace;
+    {
+        static const int flags = [] {
+            const char *e = std::getenv("XPRESS_READ_FLAGS");
+            return e ? std::atoi(e) : 0;
+        }();
+        P.read_flags = flags;
+    }
     P.ksplit = L.ksplit;
     P.h = in->h;
     P.s = in->s;
@@ -220,6 +234,8 @@ int set_kernel_attributes()
             cudaFuncSetAttribute(k_pre_mix, cudaFuncAttributeMaxDynamicSharedMemorySize, pre_mix_smem(MAX_B)) !=
                 cudaSuccess ||
             cudaFuncSetAttribute(k_pre_gemv, cudaFuncAttributeMaxDynamicSharedMemorySize, GEMV_SMEM) !=
+                cudaSuccess ||
+            cudaFuncSetAttribute(k_read_tcv, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kReadTcvSmemBytes) !=
                 cudaSuccess) {
             (void)cudaGetLastError();
             rc = XPRESS_ERR_CUDA;
@@ -334,12 +350,18 @@ int build_graph(xpress_refiner *R, GraphEntry &e, const Params &P, const Layout 
     cudaGraph_t body = cp.conditional.phGraph_out[0];
     XP_CUDA(cudaStreamBeginCaptureToGraph(cs, body, nullptr, nullptr, 0, cudaStreamCaptureModeThreadLocal));
     XP_CUDA(launch_pdl(k_mix_mlp, dim3(8, b), dim3(256), mix_mlp_smem(P.dtype), cs, (const Params *)pdev));
-    if (R->use_tc)
-        XP_CUDA(launch_pdl(k_read_tc, dim3(L.S), dim3(kReadTcThreads), kReadTcSmemBytes, cs, (const Params *)pdev,
-                           R->tmap_wr, tmap_z, R->w.V));
-    else
-        k_read_simt<<<L.S, 256, READ_SIMT_DYN_SMEM, cs>>>(pdev);
-    XP_CUDA(launch_pdl(k_reduce, dim3(b), dim3(1024), 0, cs, (const Params *)pdev, handle));
+    if (L.tcv) {
+        // the small-batch Read kernel also ends the pass (fused reduce)
+        XP_CUDA(launch_pdl(k_read_tcv, dim3(L.S), dim3(kReadTcvThreads), kReadTcvSmemBytes, cs, (const Params *)pdev,
+                           R->tmap_wr128, tmap_z, R->w.V, 1, handle));
+    } else {
+        if (R->use_tc)
+            XP_CUDA(launch_pdl(k_read_tc, dim3(L.S), dim3(kReadTcThreads), kReadTcSmemBytes, cs,
+                               (const Params *)pdev, R->tmap_wr, tmap_z, R->w.V));
+        else
+            k_read_simt<<<L.S, 256, READ_SIMT_DYN_SMEM, cs>>>(pdev);
+        XP_CUDA(launch_pdl(k_reduce, dim3(b), dim3(1024), 0, cs, (const Params *)pdev, handle));
+    }
     cudaGraph_t body_out = nullptr;
     XP_CUDA(cudaStreamEndCapture(cs, &body_out));
     XP_CUDA(cudaGraphInstantiate(&e.exec, g, 0));
@@ -420,14 +442,18 @@ int run_eager(xpress_refiner *R, Params P, const Layout &L, void *ws, cudaStream
         k_mix_mlp<<<dim3(8, b), 256, mix_mlp_smem(P.dtype), st>>>(pdev);
         kt.stop();
         kt.start("read");
-        if (R->use_tc)
+        if (L.tcv)
+            k_read_tcv<<<L.S, kReadTcvThreads, kReadTcvSmemBytes, st>>>(pdev, R->tmap_wr128, tmap_z, R->w.V, 1, 0);
+        else if (R->use_tc)
             k_read_tc<<<L.S, kReadTcThreads, kReadTcSmemBytes, st>>>(pdev, R->tmap_wr, tmap_z, R->w.V);
         else
             k_read_simt<<<L.S, 256, READ_SIMT_DYN_SMEM, st>>>(pdev);
         kt.stop();
-        kt.start("reduce");
-        k_reduce<<<b, 1024, 0, st>>>(pdev, 0);
-        kt.stop();
+        if (!L.tcv) {
+            kt.start("reduce");
+            k_reduce<<<b, 1024, 0, st>>>(pdev, 0);
+            kt.stop();
+        }
         int32_t nact = 0;
         XP_CUDA(cudaMemcpyAsync(&nact, P.ctl + CTL_NACT, 4, cudaMemcpyDeviceToHost, st));
         XP_CUDA(cudaStreamSynchronize(st));
@@ -464,7 +490,8 @@ void print_trace(xpress_refiner *R, cudaStream_t st)
     for (int i = 0; i < TRACE_SLOTS; ++i) {
         if (h[i] == ~0ull) continue;
         char name[32];
-        if (i >= 200) std::snprintf(name, sizeof(name), "readphase%d", i - 200);
+        if (i >= 210) std::snprintf(name, sizeof(name), "mlp%dphase%d", (i - 210) / 8, (i - 210) % 8);
+        else if (i >= 200) std::snprintf(name, sizeof(name), "readphase%d", i - 200);
         else if (i < 8) std::snprintf(name, sizeof(name), "%s", i < 4 ? pre[i] : "?");
         else std::snprintf(name, sizeof(name), "%s%d", (i - 8) % 4 < 3 ? body[(i - 8) % 4] : "?", (i - 8) / 4);
         std::fprintf(stderr, " %s=[%.1f,%.1f]", name, (h[i] - t0) / 1000.0, (h[TRACE_SLOTS + i] - t0) / 1000.0);
@@ -520,7 +547,8 @@ int xpress_refiner_create(const xpress_weights *w, void *stream, xpress_refiner 
             break;
         }
         R->use_tc = w->dtype == XPRESS_BF16;
-        if (R->use_tc && !make_tmap_bf16(&R->tmap_wr, w->W_r, RANK, (uint64_t)w->V, 64, 256)) {
+        if (R->use_tc && (!make_tmap_bf16(&R->tmap_wr, w->W_r, RANK, (uint64_t)w->V, 64, 256) ||
+                          !make_tmap_bf16(&R->tmap_wr128, w->W_r, RANK, (uint64_t)w->V, 64, 128))) {
             rc = XPRESS_ERR_CUDA;
             break;
         }
@@ -753,7 +781,10 @@ int xpress_profile_read(const xpress_refiner *R, void *ws, int b, void *stream)
     if (R->use_tc) {
         CUtensorMap tmap_z{};
         if (!make_tmap_bf16(&tmap_z, w + L.zpack, RANK, (uint64_t)b * R->w.B, 64, 32)) return XPRESS_ERR_CUDA;
-        k_read_tc<<<L.S, kReadTcThreads, kReadTcSmemBytes, st>>>(pdev, R->tmap_wr, tmap_z, R->w.V);
+        if (L.tcv)
+            k_read_tcv<<<L.S, kReadTcvThreads, kReadTcvSmemBytes, st>>>(pdev, R->tmap_wr128, tmap_z, R->w.V, 0, 0);
+        else
+            k_read_tc<<<L.S, kReadTcThreads, kReadTcSmemBytes, st>>>(pdev, R->tmap_wr, tmap_z, R->w.V);
     } else {
         k_read_simt<<<L.S, 256, READ_SIMT_DYN_SMEM, st>>>(pdev);
     }
