@@ -30,6 +30,7 @@ constexpr int CTL_DONE = 1;     // last-block-done ticket of the reduce kernel
 constexpr int CTL_PASS = 2;     // passes executed so far
 constexpr int CTL_ACC_DONE = 3; // ticket of the accept kernels
 constexpr int CTL_WORDS = 8;
+constexpr int RMAX_SEG = 32;    // vocabulary segments of the argmax-s scan
 
 struct SeqState {
     int active;     // takes part in the next pass
@@ -50,6 +51,31 @@ struct Partial {
     int idx;
     float m;
     float s;
+};
+
+// Counters through which the CTAs of the persistent small-batch kernel hand
+// work to one another (one 128-byte line each).  They only grow during a
+// call; STOP_BIT set in a counter tells its waiters to leave.  A call uses one
+// of two blocks (named by the area's parity word) and clears the other, which
+// the next call uses.
+constexpr unsigned STOP_BIT = 1u << 30;
+struct alignas(128) CtlLine {
+    unsigned v;
+    unsigned pad[31];
+};
+struct SmallCtl {
+    CtlLine pre_done;    // Read CTAs done with the precompute
+    CtlLine c_ready;     // Trans CTAs that published their slice of c (8 per pass)
+    CtlLine u_ready;     // ... of sigma(W_1 c)
+    CtlLine z_ready;     // ... of z
+    CtlLine pass_done;   // passes whose end (reduce, stopping rule, pack) is written
+    CtlLine read_done;   // Read CTAs done with their partials (ticket)
+    CtlLine exit_cnt;    // CTAs that left (ticket)
+    CtlLine status;      // device status bits of the call
+};
+struct SmallCtlArea {
+    CtlLine parity;      // which block the next call uses (flipped by each call's last CTA)
+    SmallCtl blk[2];
 };
 
 // Everything a call needs on the device; written by the init kernel from the
@@ -86,6 +112,12 @@ struct Params {
     void *zpack;                 // [N, r] W_r operand of the evaluated tokens
     float *zbuf;                 // [N, r] fp32 z when the caller passes no z_final
     Partial *part;               // [S, N]
+    // persistent small-batch kernel only
+    const float *Fhg;            // [2r, H] fp32: rows W_in[:, 0:r] W_h, then W_in[:, r:2r] W_g
+    int pre_kslice, pre_ks;      // K-slice width of the hidden projection and the number of slices
+    uint16_t *cx, *ux;           // [32, r] c and [32, 2r] sigma(W_1 c), bf16, exchanged by the Trans CTAs
+    Partial *rmax;               // [N, RMAX_SEG] argmax-s partials (calls without a draft)
+    SmallCtlArea *sctl;          // control blocks of the persistent kernel
 };
 
 // ------------------------------------------------------------------ numbers
@@ -237,6 +269,36 @@ __device__ __forceinline__ void trace_mark(unsigned long long *tr, int slot, uns
         atomicMin(tr + slot, t0);
         atomicMax(tr + TRACE_SLOTS + slot, globaltimer_ns());
     }
+}
+
+// Inter-CTA signalling in global memory at GPU scope.
+__device__ __forceinline__ unsigned ld_acquire_gpu(const unsigned *p)
+{
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ unsigned ld_relaxed_gpu(const unsigned *p)
+{
+    unsigned v;
+    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void red_add_release_gpu(unsigned *p, unsigned v)
+{
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ unsigned atom_add_acq_rel_gpu(unsigned *p, unsigned v)
+{
+    unsigned old;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
+// Orders this thread's generic-proxy global accesses with its later
+// async-proxy (TMA) accesses.
+__device__ __forceinline__ void fence_proxy_async_global()
+{
+    asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
 // Programmatic dependent launch: wait for the preceding kernel of the stream

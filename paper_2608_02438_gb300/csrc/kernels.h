@@ -48,6 +48,14 @@ extern const size_t kReadTcvSmemBytes;
 extern const int kReadTcvThreads;
 constexpr int TCV_MAX_TOKENS = 32;
 
+// refine_small.cu (at most 32 evaluated tokens, bf16: the whole call in one
+// persistent cooperative kernel of S Read CTAs + SMALL_TRANS_CTAS Trans CTAs)
+__global__ void k_refine_small(const __grid_constant__ Params p, const __grid_constant__ CUtensorMap tmap_wr128,
+                               const __grid_constant__ CUtensorMap tmap_z);
+__global__ void k_fold_hidden(const uint16_t *W_h, const uint16_t *W_g, const uint16_t *W_in, float *Fhg, int H);
+extern const size_t kRefineSmallSmemBytes;
+constexpr int SMALL_TRANS_CTAS = 8;
+
 // accept_kernels.cu
 __global__ void k_acc_rows(AcceptParams p);
 __global__ void k_acc_decide(AcceptParams p, int chunks);

@@ -22,22 +22,9 @@
 #include "common.cuh"
 #include "kernels.h"
 #include "reduce_common.cuh"
+#include "tcv_common.cuh"
 
 namespace xp {
-
-constexpr int TV_BM = 128;                    // vocabulary rows per block (MMA M)
-constexpr int TV_BN = 32;                     // token columns (MMA N)
-constexpr int TV_BK = 64;
-constexpr int TV_KCH = RANK / TV_BK;
-constexpr int TV_STAGES = 8;
-constexpr int TV_NBUF = 4;
-constexpr int TV_EPI_WARPS = 8;
-constexpr int TV_THREADS = 32 * (2 + TV_EPI_WARPS);
-constexpr uint32_t TV_A_STAGE = TV_BM * TV_BK * 2;        // 16 KB of W_r
-constexpr uint32_t TV_Z_CHUNK = TV_BN * TV_BK * 2;        // 4 KB of z
-constexpr uint32_t TV_Z_BYTES = TV_Z_CHUNK * TV_KCH;      // 16 KB
-constexpr uint32_t TV_TMEM_COLS = TV_NBUF * TV_BN;        // 128
-constexpr uint32_t TV_IDESC = idesc_bf16(TV_BM, TV_BN);
 
 struct TvShared {
     uint64_t full[TV_STAGES];
@@ -61,44 +48,6 @@ struct TvShared {
 constexpr size_t TV_SMEM_BYTES = 1024 + TV_STAGES * TV_A_STAGE + TV_Z_BYTES + sizeof(TvShared);
 const size_t kReadTcvSmemBytes = TV_SMEM_BYTES;
 const int kReadTcvThreads = TV_THREADS;
-
-__device__ __forceinline__ void tv_epi_bar() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
-
-__device__ __forceinline__ bool tv_epi_bar_or(bool pred)
-{
-    uint32_t res;
-    asm volatile(
-        "{\n\t.reg .pred p, q;\n\t"
-        "setp.ne.u32 p, %1, 0;\n\t"
-        "bar.red.or.pred q, 1, 256, p;\n\t"
-        "selp.u32 %0, 1, 0, q;\n\t}"
-        : "=r"(res)
-        : "r"((uint32_t)pred)
-        : "memory");
-    return res != 0;
-}
-
-// s[v0 .. v0 + 31] of one token as raw bf16 pairs (zeros past V or for an
-// invalid lane).
-__device__ __forceinline__ void load_s_group(uint4 (&r)[4], const uint16_t *row, int v0, int V, bool valid)
-{
-    if (valid && v0 + GROUP <= V) {
-        const uint4 *src = reinterpret_cast<const uint4 *>(row + v0);
-#pragma unroll
-        for (int c = 0; c < 4; ++c) r[c] = __ldg(src + c);
-        return;
-    }
-    uint32_t w[16];
-#pragma unroll
-    for (int q = 0; q < 16; ++q) {
-        const int j = v0 + 2 * q;
-        const uint32_t lo = (valid && j < V) ? row[j] : 0u;
-        const uint32_t hi = (valid && j + 1 < V) ? row[j + 1] : 0u;
-        w[q] = lo | (hi << 16);
-    }
-#pragma unroll
-    for (int c = 0; c < 4; ++c) r[c] = make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
-}
 
 __global__ void __launch_bounds__(TV_THREADS, 1)
     k_read_tcv(const Params *__restrict__ pp, const __grid_constant__ CUtensorMap tmap_wr128,

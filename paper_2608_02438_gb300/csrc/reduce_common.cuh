@@ -27,6 +27,12 @@ struct TokenResult {
 // tok = seq * B + k).  Combines the S partials in a fixed tree (deterministic);
 // T > 0 recomputes l = s + W_r z over the 32 members of the drawn group and
 // draws one by Gumbel-max (the second level of the hierarchical draw).
+__device__ __forceinline__ Partial ldcg_partial(const Partial *q)
+{
+    const float4 v = __ldcg(reinterpret_cast<const float4 *>(q));
+    return Partial{v.x, __float_as_int(v.y), v.z, v.w};
+}
+
 __device__ __forceinline__ TokenResult reduce_token(const Params &p, int i, int tok, float invT,
                                                     unsigned long long seed)
 {
@@ -40,7 +46,9 @@ __device__ __forceinline__ TokenResult reduce_token(const Params &p, int i, int 
 #pragma unroll
         for (int j = 0; j < PER; ++j) {
             const int r = r0 + lane + 32 * j;
-            pv[j] = r < p.S ? p.part[(size_t)r * p.N + i] : Partial{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
+            // through L2: a CTA of the persistent kernel may reduce several passes
+            pv[j] = r < p.S ? ldcg_partial(p.part + (size_t)r * p.N + i)
+                            : Partial{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
         }
 #pragma unroll
         for (int j = 0; j < PER; ++j) merge_partial(a, pv[j], sampling);
@@ -140,8 +148,9 @@ __device__ __forceinline__ void converge_block(const Params &p, int s, const Seq
 // Warp-collective version of converge + pack for at most 32 blocks whose
 // states sit in shared memory (lane q: block q): applies the stopping rule,
 // scans the counts, writes the states, the packed token list and the control
-// words, and sets the loop condition.
-__device__ __forceinline__ void converge_pack_small(const Params &p, const SeqState *st_in, const int *ynew,
+// words, and sets the loop condition.  Returns (in every lane) whether another
+// pass follows.
+__device__ __forceinline__ bool converge_pack_small(const Params &p, const SeqState *st_in, const int *ynew,
                                                     const int *yold, int passes_before,
                                                     cudaGraphConditionalHandle handle)
 {
@@ -170,13 +179,15 @@ __device__ __forceinline__ void converge_pack_small(const Params &p, const SeqSt
         p.st[q] = ns;
         for (int t = 0; t < c; ++t) p.act_tok[ns.off + t] = q * B + ns.m + 1 + t;
     }
+    const int passes = passes_before + 1;
+    const bool more = total > 0 && passes < p.K_max;
     if (q == 0) {
-        const int passes = passes_before + 1;
         p.ctl[CTL_NACT] = total;
         p.ctl[CTL_DONE] = 0;
         p.ctl[CTL_PASS] = passes;
-        if (p.use_graph) cudaGraphSetConditional(handle, (total > 0 && passes < p.K_max) ? 1u : 0u);
+        if (p.use_graph) cudaGraphSetConditional(handle, more ? 1u : 0u);
     }
+    return more;
 }
 
 // Block-collective (any multiple of 32 threads): packs the positions of the

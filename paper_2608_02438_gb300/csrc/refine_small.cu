@@ -1,0 +1,826 @@
+// refine_small.cu -- Algorithm 1 for small batches as one persistent kernel.
+//
+// Calls that evaluate at most 32 tokens (b * B <= 32) with a bf16 refiner run
+// the whole refinement -- the token-independent part of Fuse and Mix (Sec. 4.1,
+// hoisted out of the loop because h and g do not change between passes), every
+// Jacobi pass of Algorithm 1 and its stopping rule -- in one cooperative launch
+// of S + 8 CTAs, at most one per SM, so that no pass pays a kernel launch, a
+// graph-node switch or a cold start.
+//
+//   Read CTAs (blockIdx < S).  Before the first pass they compute partial sums
+//     of P_k = F_h h_k + F_g g over K-slices of the folded projection
+//     F = [W_in[:, 0:r] W_h ; W_in[:, r:2r] W_g] (fp32, built once per refiner:
+//     Fuse is linear, and F_g g is the block mean of F_g h_k), and, for a call
+//     without a draft, partial argmaxes of s (Algorithm 1's Y^(0)).  In every
+//     pass they run Read + Correct + selection (Eq. read / correct, the argmax
+//     or the fixed-noise group draw) over a fixed range of 128-row vocabulary
+//     blocks: W_r rows are the tcgen05 M dimension, the <= 32 tokens N, and an
+//     8-stage TMA ring streams W_r, running ahead into the next pass while the
+//     Trans CTAs work.  The CTA that finishes a pass last combines the
+//     per-range partials, applies the stopping rule and packs the next pass.
+//   Trans CTAs (S .. S + 7).  CTA j owns channels [32 j, 32 j + 32).  Once per
+//     call they finish Pc = (I + L) P for their channels (Eq. mix); in every
+//     pass they gather E' rows for the current tokens, mix (Eq. fuse / mix) and
+//     run Trans z = c + W_2 sigma(W_1 c) (Eq. mlp) on tensor cores, exchanging
+//     c and sigma(W_1 c) through L2.
+//
+// The roles hand work to one another through monotone counters (SmallCtl,
+// release / acquire at GPU scope).  Every wait is bounded: a wait that runs
+// out records ST_TIMEOUT and sets the stop bit in every counter, so that all
+// CTAs leave, each after draining its own copies in flight.
+#include "common.cuh"
+#include "kernels.h"
+#include "mlp_common.cuh"
+#include "reduce_common.cuh"
+#include "tcv_common.cuh"
+
+namespace xp {
+
+namespace {
+
+// ------------------------------------------------------------- shared memory
+
+struct RsShared {                              // Read CTA, after the W_r stages and z
+    uint64_t full[TV_STAGES], empty[TV_STAGES];
+    uint64_t z_full, z_empty, go;
+    uint64_t tfull[TV_NBUF], tempty[TV_NBUF];
+    uint64_t drain;
+    uint32_t tmem_base;
+    int abort;
+    int pass_n, pass_stop;                     // published by the producer with `go`
+    int last, passes;
+    int tok[TV_BN], pos[TV_BN];
+    float invT[TV_BN];
+    unsigned long long seed[TV_BN];
+    int ynew[TV_BN], yold[TV_BN];
+    SeqState seq[TV_BN];
+    SelState sel[TV_EPI_WARPS][32];
+    float tile[TV_EPI_WARPS][TV_BN][33];       // per-warp transpose: [token][vocabulary row]
+};
+
+struct TsShared {                              // Trans CTA
+    float e[MAX_B][32];                        // E' rows of all b*B positions, own channels
+    float pc[MAX_B][32];                       // Pc of all b*B positions, own channels
+    float cown[MAX_B][32];                     // c of the evaluated tokens, own channels (fp32)
+    float zhalf[2][MAX_B][32];                 // W_2 u, the two K halves
+    int tok[MAX_B];                            // evaluated tokens of the pass (global ids)
+    int x[MAX_B];                              // current tokens Y
+    int n, go;
+};
+
+constexpr size_t RS_BYTES = 1024 + TV_STAGES * TV_A_STAGE + TV_Z_BYTES + sizeof(RsShared);
+constexpr size_t TS_HEAD = (sizeof(TsShared) + 127) / 128 * 128;
+constexpr size_t TS_BYTES = 1024 + TS_HEAD + 32 * COP_LD * 2 + 32 * UOP_LD * 2 + 32 * MAX_B * MAX_B * 2;
+constexpr size_t SMALL_SMEM = RS_BYTES > TS_BYTES ? RS_BYTES : TS_BYTES;
+
+// ------------------------------------------------------------- signalling
+
+// Records `bits` (if any) and sets the stop bit of every counter.
+__device__ void raise_stop(SmallCtl *c, int bits)
+{
+    if (bits) atomicOr(reinterpret_cast<int *>(&c->status.v), bits);
+    __threadfence();
+    atomicOr(&c->pre_done.v, STOP_BIT);
+    atomicOr(&c->c_ready.v, STOP_BIT);
+    atomicOr(&c->u_ready.v, STOP_BIT);
+    atomicOr(&c->z_ready.v, STOP_BIT);
+    atomicOr(&c->pass_done.v, STOP_BIT);
+}
+
+// One thread: waits until *ctr >= target (true).  false once the stop bit is
+// set, or after about 2 s (the timeout is recorded and every role stops).
+// Relaxed polls with a short sleep keep ~150 pollers from crowding the line's
+// L2 slice; the fence after the last poll makes it an acquire.
+__device__ bool wait_count(SmallCtl *c, const unsigned *ctr, unsigned target)
+{
+    const unsigned long long t0 = globaltimer();
+    for (uint32_t it = 0; it < (1u << 26); ++it) {
+        const unsigned v = ld_relaxed_gpu(ctr);
+        if (v & STOP_BIT) { __threadfence(); return false; }
+        if (v >= target) { __threadfence(); return true; }
+        if (it >= 2) __nanosleep(32);
+        if ((it & 63u) == 63u && globaltimer() - t0 > 2000000000ull) break;
+    }
+    raise_stop(c, ST_TIMEOUT);
+    return false;
+}
+
+// One thread per CTA, last action on the control area: the CTA that leaves
+// last publishes the call's status and hands the other block to the next call.
+__device__ void leave(const Params &p, SmallCtlArea *a, SmallCtl *c, int par)
+{
+    __threadfence();
+    if (atomicAdd(&c->exit_cnt.v, 1u) == gridDim.x - 1) {
+        __threadfence();
+        *p.status = (int32_t)__ldcg(reinterpret_cast<const int *>(&c->status.v));
+        a->parity.v = (unsigned)(par ^ 1);
+    }
+}
+
+// ------------------------------------------------------------- precompute
+
+// Sum over the 32 lanes of v[0..NT-1] (NT = 16 or 32 token slots); lane t
+// (t < NT) ends with the total of slot t.
+template <int NT>
+__device__ __forceinline__ float reduce_scatter_n(float (&v)[NT], int lane)
+{
+#pragma unroll
+    for (int s = NT / 2; s >= 1; s >>= 1) {
+        const bool upper = (lane & s) != 0;
+#pragma unroll
+        for (int j = 0; j < s; ++j) {
+            const float send = upper ? v[j] : v[j + s];
+            const float keep = upper ? v[j + s] : v[j];
+            v[j] = keep + __shfl_xor_sync(0xffffffffu, send, s);
+        }
+    }
+    float r = v[0];
+#pragma unroll
+    for (int s = NT; s < 32; s <<= 1) r += __shfl_xor_sync(0xffffffffu, r, s);
+    return r;
+}
+
+// Work item of the hidden projection: Upart[ks][t][o] = sum over K-slice ks of
+// F[o][k] h[t][k] for the 8 R rows o of row group rg (warp w: R rows).  h's
+// slice is staged in `hs` (bf16 [N][pre_kslice]).  The 8 epilogue warps call
+// this together.
+template <int NT>
+__device__ void pre_item(const Params &p, int item, uint16_t *hs, int w, int lane)
+{
+    constexpr int R = 64 / NT, ROWS = 8 * R, NG = 2 * RANK / ROWS;
+    const int rg = item % NG, ks = item / NG;
+    const int N = p.N, H = p.H, pitch = p.pre_kslice;
+    const int kb = ks * pitch, kl = min(H, kb + pitch) - kb;
+    const uint16_t *h = static_cast<const uint16_t *>(p.h);
+    {
+        const int per = kl / 8, total = N * per, tid = w * 32 + lane;
+        for (int i0 = 0; i0 < total; i0 += 8 * 256) {
+            uint4 v[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const int i = i0 + q * 256 + tid;
+                if (i < total) v[q] = __ldg(reinterpret_cast<const uint4 *>(h + (size_t)(i / per) * H + kb) + i % per);
+            }
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const int i = i0 + q * 256 + tid;
+                if (i < total) reinterpret_cast<uint4 *>(hs + (size_t)(i / per) * pitch)[i % per] = v[q];
+            }
+        }
+    }
+    tv_epi_bar();
+    const int row0 = rg * ROWS + w * R;
+    const float *F = p.Fhg + (size_t)row0 * H + kb;
+    float acc[R][NT];
+#pragma unroll
+    for (int r = 0; r < R; ++r)
+#pragma unroll
+        for (int t = 0; t < NT; ++t) acc[r][t] = 0.0f;
+    for (int c0 = 0; c0 < kl; c0 += 512) {
+        float4 wv[R][4];
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int k = c0 + 128 * i + 4 * lane;
+                wv[r][i] = k < kl ? __ldg(reinterpret_cast<const float4 *>(F + (size_t)r * H + k))
+                                  : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int k = c0 + 128 * i + 4 * lane;
+            if (k >= kl) continue;
+#pragma unroll
+            for (int t = 0; t < NT; ++t) {
+                if (t >= N) continue;
+                const uint2 hv = *reinterpret_cast<const uint2 *>(hs + (size_t)t * pitch + k);
+                const float h0 = __uint_as_float(hv.x << 16), h1 = __uint_as_float(hv.x & 0xFFFF0000u);
+                const float h2 = __uint_as_float(hv.y << 16), h3 = __uint_as_float(hv.y & 0xFFFF0000u);
+#pragma unroll
+                for (int r = 0; r < R; ++r) {
+                    float a = acc[r][t];
+                    a = fmaf(wv[r][i].x, h0, a);
+                    a = fmaf(wv[r][i].y, h1, a);
+                    a = fmaf(wv[r][i].z, h2, a);
+                    a = fmaf(wv[r][i].w, h3, a);
+                    acc[r][t] = a;
+                }
+            }
+        }
+    }
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        const float s = reduce_scatter_n<NT>(acc[r], lane);
+        if (lane < N) p.Upart[((size_t)ks * N + lane) * 2 * RANK + row0 + r] = s;
+    }
+    tv_epi_bar();                              // hs is restaged by the next item
+}
+
+// Partial argmax of s[t, segment] (fp32 compare of the bf16 values, smallest
+// id among equal maxima).  One warp.
+__device__ void rowmax_item(const Params &p, int item, int lane)
+{
+    const int t = item / RMAX_SEG, seg = item % RMAX_SEG, V = p.V;
+    const int v0 = (int)((long long)V * seg / RMAX_SEG), v1 = (int)((long long)V * (seg + 1) / RMAX_SEG);
+    const uint16_t *row = static_cast<const uint16_t *>(p.s) + (size_t)t * V;
+    float best = -INFINITY;
+    int idx = 0x7fffffff;
+#pragma unroll 4
+    for (int v = v0 + lane; v < v1; v += 32) {
+        const float x = bf2f(__ldg(row + v));
+        if (x > best || (x == best && v < idx)) { best = x; idx = v; }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+        const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
+        if (ob > best || (ob == best && oi < idx)) { best = ob; idx = oi; }
+    }
+    if (lane == 0) p.rmax[item] = Partial{best, idx, 0.0f, 0.0f};
+}
+
+// ------------------------------------------------------------- Read role
+
+__device__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUtensorMap *tmap_z, SmallCtl *c,
+                          uint8_t *base, unsigned long long t_start)
+{
+    uint8_t *sA = base;                                    // W_r stages (h slices before the first pass)
+    uint8_t *sZ = base + TV_STAGES * TV_A_STAGE;           // z, 4 K-chunks
+    RsShared &sh = *reinterpret_cast<RsShared *>(sZ + TV_Z_BYTES);
+    const int V = p.V, S = p.S, r = blockIdx.x, N = p.N, B = p.B;
+    const int NVB = (V + TV_BM - 1) / TV_BM;
+    const int vb0 = (int)((long long)NVB * r / S), vb1 = (int)((long long)NVB * (r + 1) / S);
+    const int nblk = vb1 - vb0;                            // >= 1: S <= NVB
+    const int per_pass = nblk * TV_KCH;                    // W_r chunks per pass
+    const int ahead = min(TV_STAGES, per_pass);
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const bool tr = p.trace && r == 0;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < TV_STAGES; ++i) { mbar_init(&sh.full[i], 1); mbar_init(&sh.empty[i], 1); }
+        mbar_init(&sh.z_full, 1);
+        mbar_init(&sh.z_empty, 1);
+        mbar_init(&sh.go, 1);
+        for (int i = 0; i < TV_NBUF; ++i) { mbar_init(&sh.tfull[i], 1); mbar_init(&sh.tempty[i], 4); }
+        mbar_init(&sh.drain, 1);
+        sh.abort = 0;
+        fence_barrier_init();
+    }
+    if (warp == 1) { tmem_alloc(&sh.tmem_base, TV_TMEM_COLS); tmem_relinquish(); }
+    const uint64_t keep = policy_evict_last();
+    if (warp == 0 && lane == 0) {
+        tma_prefetch_desc(tmap_wr);
+        tma_prefetch_desc(tmap_z);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = sh.tmem_base;
+    volatile int *abort = &sh.abort;
+
+    // ---- precompute (epilogue warps), h slices staged in the W_r stages
+    if (warp >= 2) {
+        const int w = warp - 2;
+        const int ng = N <= 16 ? 16 : 32;                  // row groups (8 R rows each, R = 64 / NT)
+        const int items = ng * p.pre_ks;
+        uint16_t *hs = reinterpret_cast<uint16_t *>(sA);
+        for (int item = r; item < items; item += S) {
+            if (N <= 16) pre_item<16>(p, item, hs, w, lane);
+            else pre_item<32>(p, item, hs, w, lane);
+        }
+        if (!p.draft)
+            for (int item = r * TV_EPI_WARPS + w; item < N * RMAX_SEG; item += S * TV_EPI_WARPS)
+                rowmax_item(p, item, lane);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        red_add_release_gpu(&c->pre_done.v, 1u);
+        if (tr) trace_mark(p.trace, 2, t_start);
+        // this CTA's W_r range into L2 while Pc and the first Trans run (after
+        // the precompute, whose reads it would otherwise slow down)
+        if (!(p.read_flags & 1)) {
+            const char *wr = static_cast<const char *>(p.W_r);
+            const int rows = min(vb1 * TV_BM, V) - vb0 * TV_BM;
+            for (int r0 = 0; r0 < rows; r0 += 64)
+                prefetch_l2_bulk(wr + (size_t)(vb0 * TV_BM + r0) * RANK * 2,
+                                 (uint32_t)min(64, rows - r0) * RANK * 2);
+        }
+    }
+
+    if (warp == 0) {
+        // ------------------------------------------------------- producer
+        if (lane == 0) {
+            uint32_t pending = 0, pend_par = 0;            // last issue per stage (for the drain)
+            bool z_issued = false;
+            uint32_t z_par = 0;
+            auto issue = [&](long long ci) -> bool {
+                const int stage = (int)(ci % TV_STAGES);
+                const uint32_t ph = (uint32_t)((ci / TV_STAGES) & 1);
+                if (!mbar_wait(&sh.empty[stage], ph ^ 1, abort)) return false;
+                const int within = (int)(ci % per_pass);
+                mbar_expect_tx(&sh.full[stage], TV_A_STAGE);
+                tma_load_2d_hint(sA + stage * TV_A_STAGE, tmap_wr, &sh.full[stage], (within % TV_KCH) * TV_BK,
+                                 (vb0 + within / TV_KCH) * TV_BM, keep);
+                pending |= 1u << stage;
+                pend_par = (pend_par & ~(1u << stage)) | (ph << stage);
+                return true;
+            };
+            long long next = 0;
+            bool ok = true;
+            for (; next < ahead && ok; ++next) ok = issue(next);
+            for (int pass = 0; ok; ++pass) {
+                const bool go = wait_count(c, &c->z_ready.v, (unsigned)(8 * (pass + 1)));
+                if (go) {
+                    fence_proxy_async_global();
+                    sh.pass_n = min(__ldcg(p.ctl + CTL_NACT), TV_BN);
+                }
+                sh.pass_stop = go ? 0 : 1;
+                mbar_arrive(&sh.go);
+                if (!go) break;
+                // z of this pass, once the previous pass's MMAs are done with it
+                if (pass > 0 && !mbar_wait(&sh.z_empty, (uint32_t)((pass - 1) & 1), abort)) { ok = false; break; }
+                mbar_expect_tx(&sh.z_full, TV_Z_BYTES);
+                for (int kc = 0; kc < TV_KCH; ++kc) tma_load_2d(sZ + kc * TV_Z_CHUNK, tmap_z, &sh.z_full, kc * TV_BK, 0);
+                z_issued = true;
+                z_par = (uint32_t)(pass & 1);
+                // the rest of this pass, then the first chunks of the next one
+                const long long end = (long long)(pass + 1) * per_pass + ahead;
+                for (; next < end; ++next)
+                    if (!issue(next)) { ok = false; break; }
+            }
+            // no copy may still be landing when the CTA leaves
+            int dummy = 0;
+            for (int st = 0; st < TV_STAGES; ++st)
+                if (pending & (1u << st)) mbar_wait(&sh.full[st], (pend_par >> st) & 1, &dummy, 100000000ull);
+            if (z_issued) mbar_wait(&sh.z_full, z_par, &dummy, 100000000ull);
+        }
+    } else if (warp == 1) {
+        // ---------------------------------------------------- MMA issuer
+        if (lane == 0) {
+            const uint32_t z0 = smem_u32(sZ);
+            for (int pass = 0;; ++pass) {
+                if (!mbar_wait(&sh.go, (uint32_t)(pass & 1), abort)) break;
+                if (*reinterpret_cast<volatile int *>(&sh.pass_stop)) break;
+                if (!mbar_wait(&sh.z_full, (uint32_t)(pass & 1), abort)) break;
+                tc_fence_after();
+                bool ok = true;
+                for (int i = 0; i < nblk && ok; ++i) {
+                    const int ib = pass * nblk + i, buf = ib % TV_NBUF;
+                    if (!mbar_wait(&sh.tempty[buf], (uint32_t)(((ib / TV_NBUF) & 1) ^ 1), abort)) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t d = tmem + buf * TV_BN;
+                    for (int kc = 0; kc < TV_KCH; ++kc) {
+                        const long long ci = (long long)pass * per_pass + i * TV_KCH + kc;
+                        const int stage = (int)(ci % TV_STAGES);
+                        if (!mbar_wait(&sh.full[stage], (uint32_t)((ci / TV_STAGES) & 1), abort)) { ok = false; break; }
+                        tc_fence_after();
+                        const uint32_t a0 = smem_u32(sA + stage * TV_A_STAGE);
+#pragma unroll
+                        for (int kk = 0; kk < TV_BK / 16; ++kk)
+                            tc_mma_bf16(d, smem_desc_sw128(a0 + kk * 32), smem_desc_sw128(z0 + kc * TV_Z_CHUNK + kk * 32),
+                                        TV_IDESC, (kc | kk) != 0);
+                        tc_commit(&sh.empty[stage]);
+                    }
+                    if (ok) tc_commit(&sh.tfull[buf]);
+                }
+                if (!ok) break;
+                tc_commit(&sh.z_empty);
+            }
+            tc_commit(&sh.drain);
+            int dummy = 0;
+            mbar_wait(&sh.drain, 0, &dummy, 100000000ull);
+        }
+    } else {
+        // ------------------------------------------------------ epilogue
+        const int ew = warp - 2, q = warp & 3, half = ew >> 2;
+        const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+        float (*tile)[33] = sh.tile[ew];
+        for (int pass = 0;; ++pass) {
+            // every epilogue thread takes the same decision (the named
+            // barriers below need all 256)
+            const bool got = mbar_wait(&sh.go, (uint32_t)(pass & 1), abort);
+            if (tv_epi_bar_or(!got || *abort || *reinterpret_cast<volatile int *>(&sh.pass_stop))) break;
+            const unsigned long long t_go = globaltimer_ns();
+            const int n = *reinterpret_cast<volatile int *>(&sh.pass_n);
+            if (ew == 0) {
+                __threadfence();
+                const int t = lane;
+                int tok = 0, pos = 0;
+                float invT = 0.0f;
+                unsigned long long seed = 0;
+                if (t < n) {
+                    tok = __ldcg(p.act_tok + t);
+                    const int s = tok / B;
+                    pos = tok % B;
+                    const float T = p.temperature[s];
+                    invT = T > 0.0f ? 1.0f / T : 0.0f;
+                    seed = p.seed[s];
+                    sh.yold[t] = __ldcg(p.tokens + tok);
+                }
+                sh.tok[t] = tok;
+                sh.pos[t] = pos;
+                sh.invT[t] = invT;
+                sh.seed[t] = seed;
+                if (t < p.b) {
+                    const int4 *src = reinterpret_cast<const int4 *>(p.st + t);
+                    const int4 a = __ldcg(src), b2 = __ldcg(src + 1);
+                    sh.seq[t] = SeqState{a.x, a.y, a.z, a.w, b2.x, b2.y, b2.z, b2.w};
+                }
+                if (t == 0) sh.passes = __ldcg(p.ctl + CTL_PASS);
+            }
+            tv_epi_bar();
+            const int my_tok = sh.tok[lane], my_pos = sh.pos[lane];
+            const float my_invT = sh.invT[lane];
+            const unsigned long long my_seed = sh.seed[lane];
+            const bool tvalid = lane < n;
+            const uint16_t *srow = static_cast<const uint16_t *>(p.s) + (size_t)my_tok * V;
+            SelState sel;
+            sel.init();
+            bool ok = true;
+            uint4 cur[4], nxt[4];
+            if (half < nblk) load_s_group(cur, srow, (vb0 + half) * TV_BM + q * 32, V, tvalid);
+            for (int i = half; i < nblk; i += 2) {
+                const int ib = pass * nblk + i, buf = ib % TV_NBUF;
+                const int v0 = (vb0 + i) * TV_BM + q * 32;
+                if (i + 2 < nblk) load_s_group(nxt, srow, (vb0 + i + 2) * TV_BM + q * 32, V, tvalid);
+                if (!mbar_wait(&sh.tfull[buf], (uint32_t)((ib / TV_NBUF) & 1), abort)) { ok = false; break; }
+                tc_fence_after();
+                float acc[TV_BN];
+                tmem_ld32(tmem + lane_base + buf * TV_BN, acc);
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&sh.tempty[buf]);
+#pragma unroll
+                for (int t2 = 0; t2 < TV_BN; ++t2) tile[t2][lane] = acc[t2];
+                __syncwarp();
+                const int nv = min(GROUP, V - v0);
+                if (tvalid && nv > 0) {
+                    float l[GROUP];
+#pragma unroll
+                    for (int cc = 0; cc < 4; ++cc) {
+                        const uint32_t ww[4] = {cur[cc].x, cur[cc].y, cur[cc].z, cur[cc].w};
+#pragma unroll
+                        for (int e2 = 0; e2 < 4; ++e2) {
+                            l[cc * 8 + 2 * e2] = tile[lane][cc * 8 + 2 * e2] + __uint_as_float(ww[e2] << 16);
+                            l[cc * 8 + 2 * e2 + 1] =
+                                tile[lane][cc * 8 + 2 * e2 + 1] + __uint_as_float(ww[e2] & 0xFFFF0000u);
+                        }
+                    }
+                    if (p.logits) {
+                        float *dst = p.logits + (size_t)my_tok * V + v0;
+#pragma unroll
+                        for (int jj = 0; jj < GROUP; ++jj)
+                            if (jj < nv) dst[jj] = l[jj];
+                    }
+                    select_group(sel, l, v0, nv, my_invT, my_seed, (uint32_t)my_pos, p.offset);
+                }
+                __syncwarp();
+#pragma unroll
+                for (int cc = 0; cc < 4; ++cc) cur[cc] = nxt[cc];
+            }
+            sh.sel[ew][lane] = sel;
+            if (tv_epi_bar_or(!ok || *abort)) break;
+            if (ew == 0 && lane < n) {
+                Partial a{sh.sel[0][lane].best, sh.sel[0][lane].idx, sh.sel[0][lane].m, sh.sel[0][lane].s};
+                for (int w2 = 1; w2 < TV_EPI_WARPS; ++w2) {
+                    const Partial b2{sh.sel[w2][lane].best, sh.sel[w2][lane].idx, sh.sel[w2][lane].m,
+                                     sh.sel[w2][lane].s};
+                    merge_partial(a, b2, my_invT > 0.0f);
+                }
+                p.part[(size_t)r * N + lane] = a;
+            }
+            tv_epi_bar();
+            if (ew == 0 && lane == 0) {
+                __threadfence();
+                sh.last = atom_add_acq_rel_gpu(&c->read_done.v, 1u) == (unsigned)(S * (pass + 1) - 1);
+                if (tr) trace_mark(p.trace, 8 + 4 * pass + 1, t_go);
+            }
+            tv_epi_bar();
+            if (sh.last) {
+                // end of the pass: combine the partials of every evaluated
+                // token, apply the stopping rule, pack the next pass
+                __threadfence();
+                const unsigned long long t_last = globaltimer_ns();
+                for (int t = ew; t < n; t += TV_EPI_WARPS) {
+                    const int tok = sh.tok[t];
+                    const TokenResult res = reduce_token(p, t, tok, sh.invT[t], sh.seed[t]);
+                    if (lane == 0) {
+                        sh.ynew[t] = res.y;
+                        if (p.lse) p.lse[tok] = res.lse;
+                        if (p.logit_sel) p.logit_sel[tok] = res.sel;
+                        p.tokens[tok] = res.y;
+                    }
+                }
+                tv_epi_bar();
+                if (ew == 0) {
+                    const bool more = converge_pack_small(p, sh.seq, sh.ynew, sh.yold, sh.passes, 0);
+                    __syncwarp();
+                    if (lane == 0) {
+                        __threadfence();
+                        if (more) red_add_release_gpu(&c->pass_done.v, 1u);
+                        else raise_stop(c, 0);
+                        if (p.trace) trace_mark(p.trace, 8 + 4 * pass + 2, t_last);
+                    }
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, TV_TMEM_COLS);
+    }
+    if (threadIdx.x == 0 && sh.abort) raise_stop(c, ST_TIMEOUT);
+}
+
+// ------------------------------------------------------------- Trans role
+
+__device__ void trans_role(const Params &p, SmallCtl *c, uint8_t *base, unsigned long long t_start)
+{
+    TsShared &sh = *reinterpret_cast<TsShared *>(base);
+    uint16_t *cop = reinterpret_cast<uint16_t *>(base + TS_HEAD);
+    uint16_t *uop = cop + 32 * COP_LD;
+    uint16_t *Ls = uop + 32 * UOP_LD;
+    const int rank = blockIdx.x - p.S, d0 = rank * 32;
+    const int N = p.N, B = p.B, b = p.b, V = p.V;
+    const int tid = threadIdx.x, nth = blockDim.x, warp = tid / 32, lane = tid % 32;
+    const int g = lane >> 2, tq = lane & 3, khalf = (warp >> 2) & 1;
+    const bool lead = rank == 0;
+
+    // static operands: W_1 / W_2 fragments (warps 0-7) and the CTA's slice of L
+    MlpFrags fr;
+    if (warp < 8) load_mlp_frags(p, rank, fr);
+    {
+        const int n16 = 32 * B * B * 2 / 16;
+        const uint4 *src = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.L) + (size_t)d0 * B * B);
+        for (int i = tid; i < n16; i += nth) reinterpret_cast<uint4 *>(Ls)[i] = __ldg(src + i);
+    }
+    // Y^(0) from the draft; the lead CTA writes the state of the first pass
+    if (tid < N) {
+        int y = 0;
+        if (p.draft) {
+            y = p.draft[tid];
+            if (y < 0 || y >= V) {
+                if (lead) atomicOr(reinterpret_cast<int *>(&c->status.v), ST_BOUNDS);
+                y = 0;
+            }
+        }
+        sh.x[tid] = y;
+        sh.tok[tid] = tid;
+    }
+    if (lead) {
+        if (tid < N) {
+            p.act_tok[tid] = tid;
+            if (p.draft) p.tokens[tid] = sh.x[tid];
+        }
+        if (tid < b) {
+            SeqState s{};
+            s.active = 1; s.m = -1; s.iters = 0; s.converged = 0; s.off = tid * B; s.cnt = B;
+            p.st[tid] = s;
+            if (p.anchor[tid] < 0 || p.anchor[tid] >= V) atomicOr(reinterpret_cast<int *>(&c->status.v), ST_BOUNDS);
+            if (p.iters) p.iters[tid] = 0;
+            if (p.converged) p.converged[tid] = 0;
+        }
+        if (tid == 0) { p.ctl[CTL_NACT] = N; p.ctl[CTL_DONE] = 0; p.ctl[CTL_PASS] = 0; }
+    }
+    if (tid == 0) sh.go = wait_count(c, &c->pre_done.v, (unsigned)p.S);
+    __syncthreads();
+    if (!sh.go) return;
+    if (!p.draft) {
+        // Y^(0) = argmax s (Algorithm 1), from the Read CTAs' partials
+        for (int t = warp; t < N; t += nth / 32) {
+            const Partial q = ldcg_partial(p.rmax + (size_t)t * RMAX_SEG + lane);
+            float best = q.best;
+            int idx = q.idx;
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+                const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
+                if (ob > best || (ob == best && oi < idx)) { best = ob; idx = oi; }
+            }
+            if (lane == 0) {
+                if (idx < 0 || idx >= V) idx = 0;
+                sh.x[t] = idx;
+                if (lead) p.tokens[t] = idx;
+            }
+        }
+    }
+    // Pc = (I + L) P for the own channels (Eq. mix); P_k = F_h h_k + mean_j F_g h_j
+    {
+        float(*P)[32] = sh.e;                                  // scratch until the first gather
+        float(*G)[32] = sh.cown;
+        const int ks = p.pre_ks;
+        for (int i = tid; i < N * 32; i += nth) {
+            const int t = i / 32, dd = i % 32;
+            const float *u = p.Upart + (size_t)t * 2 * RANK + d0 + dd;
+            float a = 0.0f, gsum = 0.0f;
+#pragma unroll 4
+            for (int z = 0; z < ks; ++z) {
+                a += __ldcg(u + (size_t)z * N * 2 * RANK);
+                gsum += __ldcg(u + (size_t)z * N * 2 * RANK + RANK);
+            }
+            P[t][dd] = a;
+            G[t][dd] = gsum;
+        }
+        __syncthreads();
+        for (int i = tid; i < N * 32; i += nth) {
+            const int t = i / 32, dd = i % 32, s = t / B;
+            float gs = 0.0f;
+            for (int k = 0; k < B; ++k) gs += G[s * B + k][dd];
+            sh.pc[t][dd] = P[t][dd] + gs / (float)B;           // P, complete
+        }
+        __syncthreads();
+        for (int i = tid; i < N * 32; i += nth) {
+            const int t = i / 32, dd = i % 32, s = t / B, k = t % B;
+            float a = sh.pc[t][dd];
+            for (int j = 0; j < k; ++j) a = fmaf(bf2f(Ls[(dd * B + k) * B + j]), sh.pc[s * B + j][dd], a);
+            P[t][dd] = a;
+        }
+        __syncthreads();
+        for (int i = tid; i < N * 32; i += nth) sh.pc[i / 32][i % 32] = P[i / 32][i % 32];
+        __syncthreads();
+    }
+    if (lead && tid == 0 && p.trace) trace_mark(p.trace, 3, t_start);
+
+    float *zf = p.z_final ? p.z_final : p.zbuf;
+    uint16_t *zpack = static_cast<uint16_t *>(p.zpack);
+    for (int pass = 0;; ++pass) {
+        const unsigned long long t_pass = globaltimer_ns();
+        const int trs = (lead && tid == 0 && p.trace && pass < 3) ? 210 + 8 * pass : 0;
+        int n = N;
+        if (pass > 0) {
+            if (tid == 0) sh.go = wait_count(c, &c->pass_done.v, (unsigned)pass);
+            __syncthreads();
+            if (!sh.go) break;
+            n = min(__ldcg(p.ctl + CTL_NACT), MAX_B);
+            if (tid < n) sh.tok[tid] = __ldcg(p.act_tok + tid);
+            if (tid < N) sh.x[tid] = __ldcg(p.tokens + tid);
+            __syncthreads();
+        }
+        if (trs) trace_mark(p.trace, trs, t_pass);
+        // Fuse, token part: e_j = E'[x_{j-1}] (x_{-1} = anchor) for every position
+        for (int i = tid; i < N * 32; i += nth) {
+            const int j = i / 32, dd = i % 32, k = j % B, s = j / B;
+            int x = k == 0 ? p.anchor[s] : sh.x[j - 1];
+            if (x < 0 || x >= V) x = 0;                        // reported at the start
+            sh.e[j][dd] = __ldg(p.Ep + (size_t)x * RANK + d0 + dd);
+        }
+        __syncthreads();
+        if (trs) trace_mark(p.trace, trs + 1, t_pass);
+        // Mix for the evaluated tokens; c leaves rounded to bf16 (the W_1 operand)
+        for (int i = tid; i < n * 32; i += nth) {
+            const int t = i / 32, dd = i % 32, tok = sh.tok[t], s = tok / B, k = tok % B;
+            float a = sh.pc[tok][dd] + sh.e[tok][dd];
+            for (int j = 0; j < k; ++j) a = fmaf(bf2f(Ls[(dd * B + k) * B + j]), sh.e[s * B + j][dd], a);
+            sh.cown[t][dd] = a;
+            p.cx[(size_t)t * RANK + d0 + dd] = f2bf(a);
+        }
+        __syncthreads();
+        if (tid == 0) {
+            __threadfence();
+            red_add_release_gpu(&c->c_ready.v, 1u);
+            sh.go = wait_count(c, &c->c_ready.v, (unsigned)(8 * (pass + 1)));
+            if (trs) trace_mark(p.trace, trs + 2, t_pass);
+        }
+        __syncthreads();
+        if (!sh.go) break;
+        for (int i = tid; i < 32 * (RANK / 8); i += nth) {
+            const int t = i / (RANK / 8), cc = i % (RANK / 8);
+            uint4 v = make_uint4(0, 0, 0, 0);
+            if (t < n) v = __ldcg(reinterpret_cast<const uint4 *>(p.cx + (size_t)t * RANK) + cc);
+            *reinterpret_cast<uint4 *>(cop + t * COP_LD + 8 * cc) = v;
+        }
+        __syncthreads();
+        // u = sigma(W_1 c), rows [64 rank, +64): warp w -> 8 rows
+        if (warp < 8) {
+            for (int mt = 0; mt * 16 < n; ++mt) {
+                float acc[4] = {0.f, 0.f, 0.f, 0.f};
+                const uint16_t *arow0 = cop + (mt * 16 + g) * COP_LD, *arow1 = arow0 + 8 * COP_LD;
+#pragma unroll
+                for (int ks = 0; ks < RANK / 16; ++ks) {
+                    uint32_t a[4];
+                    a[0] = *reinterpret_cast<const uint32_t *>(arow0 + ks * 16 + 2 * tq);
+                    a[1] = *reinterpret_cast<const uint32_t *>(arow1 + ks * 16 + 2 * tq);
+                    a[2] = *reinterpret_cast<const uint32_t *>(arow0 + ks * 16 + 8 + 2 * tq);
+                    a[3] = *reinterpret_cast<const uint32_t *>(arow1 + ks * 16 + 8 + 2 * tq);
+                    mma_bf16_16816(acc, a, fr.b1[ks][0], fr.b1[ks][1]);
+                }
+                const int f = 64 * rank + 8 * warp + 2 * tq;
+                const int t0 = mt * 16 + g, t1 = t0 + 8;
+                if (t0 < n)
+                    *reinterpret_cast<uint32_t *>(p.ux + (size_t)t0 * 2 * RANK + f) =
+                        (uint32_t)f2bf(act_fn(p.act, acc[0])) | ((uint32_t)f2bf(act_fn(p.act, acc[1])) << 16);
+                if (t1 < n)
+                    *reinterpret_cast<uint32_t *>(p.ux + (size_t)t1 * 2 * RANK + f) =
+                        (uint32_t)f2bf(act_fn(p.act, acc[2])) | ((uint32_t)f2bf(act_fn(p.act, acc[3])) << 16);
+            }
+        }
+        __syncthreads();
+        if (tid == 0) {
+            __threadfence();
+            red_add_release_gpu(&c->u_ready.v, 1u);
+            sh.go = wait_count(c, &c->u_ready.v, (unsigned)(8 * (pass + 1)));
+            if (trs) trace_mark(p.trace, trs + 3, t_pass);
+        }
+        __syncthreads();
+        if (!sh.go) break;
+        for (int i = tid; i < 32 * (2 * RANK / 8); i += nth) {
+            const int t = i / (2 * RANK / 8), cc = i % (2 * RANK / 8);
+            uint4 v = make_uint4(0, 0, 0, 0);
+            if (t < n) v = __ldcg(reinterpret_cast<const uint4 *>(p.ux + (size_t)t * 2 * RANK) + cc);
+            *reinterpret_cast<uint4 *>(uop + t * UOP_LD + 8 * cc) = v;
+        }
+        __syncthreads();
+        // z = c + W_2 u for channels [32 rank, +32): warp w -> 8 channels, K half w / 4
+        if (warp < 8) {
+            for (int mt = 0; mt * 16 < n; ++mt) {
+                float acc[4] = {0.f, 0.f, 0.f, 0.f};
+                const uint16_t *arow0 = uop + (mt * 16 + g) * UOP_LD + khalf * RANK, *arow1 = arow0 + 8 * UOP_LD;
+#pragma unroll
+                for (int ks = 0; ks < RANK / 16; ++ks) {
+                    uint32_t a[4];
+                    a[0] = *reinterpret_cast<const uint32_t *>(arow0 + ks * 16 + 2 * tq);
+                    a[1] = *reinterpret_cast<const uint32_t *>(arow1 + ks * 16 + 2 * tq);
+                    a[2] = *reinterpret_cast<const uint32_t *>(arow0 + ks * 16 + 8 + 2 * tq);
+                    a[3] = *reinterpret_cast<const uint32_t *>(arow1 + ks * 16 + 8 + 2 * tq);
+                    mma_bf16_16816(acc, a, fr.b2[ks][0], fr.b2[ks][1]);
+                }
+                const int col = 8 * (warp & 3) + 2 * tq, t0 = mt * 16 + g;
+                sh.zhalf[khalf][t0][col] = acc[0];
+                sh.zhalf[khalf][t0][col + 1] = acc[1];
+                sh.zhalf[khalf][t0 + 8][col] = acc[2];
+                sh.zhalf[khalf][t0 + 8][col + 1] = acc[3];
+            }
+        }
+        __syncthreads();
+        for (int i = tid; i < n * 32; i += nth) {
+            const int t = i / 32, dd = i % 32, tok = sh.tok[t];
+            const float z = sh.cown[t][dd] + (sh.zhalf[0][t][dd] + sh.zhalf[1][t][dd]);
+            zf[(size_t)tok * RANK + d0 + dd] = z;
+            zpack[(size_t)t * RANK + d0 + dd] = f2bf(z);
+        }
+        fence_proxy_async_global();                            // z is read by TMA
+        __syncthreads();
+        if (tid == 0) {
+            __threadfence();
+            red_add_release_gpu(&c->z_ready.v, 1u);
+            if (lead && p.trace) trace_mark(p.trace, 8 + 4 * pass, t_pass);
+        }
+    }
+}
+
+}  // namespace
+
+const size_t kRefineSmallSmemBytes = SMALL_SMEM;
+
+// grid S + 8 (cooperative), TV_THREADS threads, SMALL_SMEM dynamic shared memory.
+__global__ void __launch_bounds__(TV_THREADS, 1)
+    k_refine_small(const __grid_constant__ Params p, const __grid_constant__ CUtensorMap tmap_wr128,
+                   const __grid_constant__ CUtensorMap tmap_z)
+{
+    const unsigned long long t_start = globaltimer_ns();
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    SmallCtlArea *area = p.sctl;
+    const int par = (int)(__ldcg(&area->parity.v) & 1u);
+    SmallCtl *c = &area->blk[par];
+    if (blockIdx.x == 0 && threadIdx.x < 8) {
+        // the next call's block (this call's other one) starts from zero
+        CtlLine *nxt = reinterpret_cast<CtlLine *>(&area->blk[par ^ 1]);
+        nxt[threadIdx.x].v = 0;
+    }
+    if ((int)blockIdx.x < p.S) read_role(p, &tmap_wr128, &tmap_z, c, base, t_start);
+    else trans_role(p, c, base, t_start);
+    __syncthreads();
+    if (threadIdx.x == 0) leave(p, area, c, par);
+}
+
+// Folded hidden projection (Fuse is linear): Fhg[o][i] = sum_e W_in[o][e] W_h[e][i]
+// for o < r and sum_e W_in[o - r][r + e] W_g[e][i] for o >= r, fp32 accumulation.
+// grid (ceil(H / 256), 2r / 8), 256 threads.
+__global__ void __launch_bounds__(256) k_fold_hidden(const uint16_t *W_h, const uint16_t *W_g, const uint16_t *W_in,
+                                                     float *Fhg, int H)
+{
+    __shared__ float win[8][RANK];
+    const int o0 = blockIdx.y * 8, i = blockIdx.x * 256 + threadIdx.x;
+    const bool gpart = o0 >= RANK;
+    for (int q = threadIdx.x; q < 8 * RANK; q += 256) {
+        const int rr = q / RANK, e = q % RANK, o = o0 + rr;
+        win[rr][e] = bf2f(W_in[(size_t)(o % RANK) * 3 * RANK + (gpart ? RANK : 0) + e]);
+    }
+    __syncthreads();
+    if (i >= H) return;
+    const uint16_t *W = gpart ? W_g : W_h;
+    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    for (int e = 0; e < RANK; ++e) {
+        const float x = bf2f(W[(size_t)e * H + i]);
+#pragma unroll
+        for (int rr = 0; rr < 8; ++rr) acc[rr] = fmaf(win[rr][e], x, acc[rr]);
+    }
+#pragma unroll
+    for (int rr = 0; rr < 8; ++rr) Fhg[(size_t)(o0 + rr) * H + i] = acc[rr];
+}
+
+}  // namespace xp

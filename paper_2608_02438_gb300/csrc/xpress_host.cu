@@ -70,9 +70,12 @@ size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 struct Layout {
     size_t status = 0, ctl = 64, params = 256, st = 0, upart = 0, pc = 0, ynew = 0, acttok = 0, zpack = 0,
            zbuf = 0, part = 0, total = 0;
+    size_t sctl = 0, cx = 0, ux = 0, rmax = 0;
     int ksplit = 1, kchunk = 0, S = 1;
+    int pre_kslice = 0, pre_ks = 0;
     bool gemv = false;
     bool tcv = false;
+    bool small = false;      // persistent small-batch kernel
 };
 
 }  // namespace
@@ -87,6 +90,10 @@ struct xpress_refiner {
     int num_sms = 0;
     bool use_tc = false;
     cudaStream_t cs = nullptr;
+    float *Fhg = nullptr;                  // [2r, H] folded hidden projection (small-batch kernel)
+    bool small_ok = false;                 // the small-batch kernel can run co-resident on this GPU
+    void *small_ws[CACHE_SLOTS] = {};      // workspaces whose control area this refiner has cleared
+    int small_ws_next = 0;
     GraphEntry cache[CACHE_SLOTS];
     uint64_t clock = 0;
 };
@@ -96,12 +103,24 @@ namespace {
 // k_read_tcv serves calls that evaluate at most 32 tokens (b * B <= 32)
 bool use_tcv(const xpress_refiner *R, int b) { return R->use_tc && b * R->w.B <= TCV_MAX_TOKENS; }
 
+// The persistent kernel serves the same calls unless XPRESS_SMALL=0 (the
+// multi-kernel graph path then runs them).
+bool use_small(const xpress_refiner *R, int b)
+{
+    static const bool enabled = [] {
+        const char *e = std::getenv("XPRESS_SMALL");
+        return !(e && e[0] == '0');
+    }();
+    return enabled && R->small_ok && use_tcv(R, b);
+}
+
 int read_S(const xpress_refiner *R, int b)
 {
     if (R->use_tc) {
         const int rows = use_tcv(R, b) ? 128 : 256;
         const int nvt = (R->w.V + rows - 1) / rows;
-        return nvt < R->num_sms ? nvt : R->num_sms;
+        const int sms = use_small(R, b) ? R->num_sms - SMALL_TRANS_CTAS : R->num_sms;
+        return nvt < sms ? nvt : sms;
     }
     const int ng = (R->w.V + GROUP - 1) / GROUP;
     return ng < 2 * R->num_sms ? ng : 2 * R->num_sms;
@@ -113,6 +132,8 @@ Layout make_layout(const xpress_refiner *R, int b)
     const int B = R->w.B, N = b * B;
     const size_t esz = R->w.dtype == XPRESS_BF16 ? 2 : 4;
     size_t o = align256(L.params + sizeof(Params));
+    L.sctl = o;                                    // same offset for every b
+    o = align256(o + sizeof(SmallCtlArea));
     L.st = o;
     o = align256(o + (size_t)b * sizeof(SeqState));
     L.gemv = R->w.dtype == XPRESS_BF16 && N <= 32;
@@ -131,8 +152,23 @@ Layout make_layout(const xpress_refiner *R, int b)
         L.kchunk = ((R->w.H + ks - 1) / ks + 15) / 16 * 16;
         L.ksplit = (R->w.H + L.kchunk - 1) / L.kchunk;
     }
+    L.S = read_S(R, b);
+    L.small = use_small(R, b);
+    int upart_ks = L.ksplit;
+    if (L.small) {
+        // K-slices of the folded projection: about one work item per Read CTA,
+        // h's slice within the W_r stages (128 KB)
+        const int ng = N <= 16 ? 16 : 32;
+        const int ks_max = L.S / ng > 1 ? L.S / ng : 1;
+        int kslice = ((R->w.H + ks_max - 1) / ks_max + 127) / 128 * 128;
+        const int kcap = (128 * 1024 / (2 * N)) / 128 * 128;
+        if (kslice > kcap) kslice = kcap;
+        L.pre_kslice = kslice;
+        L.pre_ks = (R->w.H + kslice - 1) / kslice;
+        if (L.pre_ks > upart_ks) upart_ks = L.pre_ks;
+    }
     L.upart = o;
-    o = align256(o + (size_t)L.ksplit * N * 2 * RANK * 4);
+    o = align256(o + (size_t)upart_ks * N * 2 * RANK * 4);
     L.pc = o;
     o = align256(o + (size_t)N * RANK * 4);
     L.ynew = o;
@@ -143,10 +179,17 @@ Layout make_layout(const xpress_refiner *R, int b)
     o = align256(o + (size_t)N * RANK * esz);
     L.zbuf = o;
     o = align256(o + (size_t)N * RANK * 4);
-    L.S = read_S(R, b);
     L.tcv = use_tcv(R, b);
     L.part = o;
     o = align256(o + (size_t)L.S * N * sizeof(Partial));
+    if (L.small) {
+        L.cx = o;
+        o = align256(o + (size_t)32 * RANK * 2);
+        L.ux = o;
+        o = align256(o + (size_t)32 * 2 * RANK * 2);
+        L.rmax = o;
+        o = align256(o + (size_t)N * RMAX_SEG * sizeof(Partial));
+    }
     L.total = o;
     return L;
 }
@@ -208,6 +251,16 @@ Params make_params(const xpress_refiner *R, const xpress_block_in *in, const xpr
     P.zpack = w + L.zpack;
     P.zbuf = reinterpret_cast<float *>(w + L.zbuf);
     P.part = reinterpret_cast<Partial *>(w + L.part);
+    if (L.small) {
+        P.use_graph = 0;
+        P.Fhg = R->Fhg;
+        P.pre_kslice = L.pre_kslice;
+        P.pre_ks = L.pre_ks;
+        P.cx = reinterpret_cast<uint16_t *>(w + L.cx);
+        P.ux = reinterpret_cast<uint16_t *>(w + L.ux);
+        P.rmax = reinterpret_cast<Partial *>(w + L.rmax);
+        P.sctl = reinterpret_cast<SmallCtlArea *>(w + L.sctl);
+    }
     return P;
 }
 
@@ -236,7 +289,9 @@ int set_kernel_attributes()
             cudaFuncSetAttribute(k_pre_gemv, cudaFuncAttributeMaxDynamicSharedMemorySize, GEMV_SMEM) !=
                 cudaSuccess ||
             cudaFuncSetAttribute(k_read_tcv, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kReadTcvSmemBytes) !=
-                cudaSuccess) {
+                cudaSuccess ||
+            cudaFuncSetAttribute(k_refine_small, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)kRefineSmallSmemBytes) != cudaSuccess) {
             (void)cudaGetLastError();
             rc = XPRESS_ERR_CUDA;
         }
@@ -464,6 +519,41 @@ int run_eager(xpress_refiner *R, Params P, const Layout &L, void *ws, cudaStream
     return XPRESS_OK;
 }
 
+void print_trace(xpress_refiner *R, cudaStream_t st);
+
+// One call of the persistent small-batch kernel.  The control area's two
+// blocks and parity word are cleared the first time this refiner meets the
+// workspace; from then on each call clears the block the next call uses.
+int run_small(xpress_refiner *R, const Params &P, const Layout &L, void *ws, cudaStream_t st)
+{
+    bool seen = false;
+    for (void *s : R->small_ws) seen = seen || s == ws;
+    if (!seen) {
+        XP_CUDA(cudaMemsetAsync(static_cast<char *>(ws) + L.sctl, 0, sizeof(SmallCtlArea), st));
+        R->small_ws[R->small_ws_next] = ws;
+        R->small_ws_next = (R->small_ws_next + 1) % CACHE_SLOTS;
+    }
+    CUtensorMap tmap_z{};
+    if (!make_tmap_bf16(&tmap_z, P.zpack, RANK, (uint64_t)P.N, 64, 32)) return XPRESS_ERR_CUDA;
+    if (R->trace) {
+        XP_CUDA(cudaMemsetAsync(R->trace, 0xFF, TRACE_SLOTS * sizeof(unsigned long long), st));
+        XP_CUDA(cudaMemsetAsync(R->trace + TRACE_SLOTS, 0, TRACE_SLOTS * sizeof(unsigned long long), st));
+    }
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3((unsigned)(L.S + SMALL_TRANS_CTAS));
+    cfg.blockDim = dim3(32 * (2 + 8));
+    cfg.dynamicSmemBytes = kRefineSmallSmemBytes;
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    XP_CUDA(cudaLaunchKernelEx(&cfg, k_refine_small, P, R->tmap_wr128, tmap_z));
+    if (R->trace) print_trace(R, st);
+    return XPRESS_OK;
+}
+
 int eager_mode()
 {
     static const int mode = [] {
@@ -484,7 +574,7 @@ void print_trace(xpress_refiner *R, cudaStream_t st)
     unsigned long long t0 = ~0ull;
     for (int i = 0; i < TRACE_SLOTS; ++i)
         if (h[i] < t0) t0 = h[i];
-    static const char *pre[4] = {"init", "seed", "pregemm", "premix"};
+    static const char *pre[4] = {"init", "seed", "precompute", "pc"};
     static const char *body[3] = {"mlp", "read", "reduce"};
     std::fprintf(stderr, "xpress-trace:");
     for (int i = 0; i < TRACE_SLOTS; ++i) {
@@ -564,6 +654,26 @@ int xpress_refiner_create(const xpress_weights *w, void *stream, xpress_refiner 
         }
         const dim3 grid(RANK / 64, (w->V + 63) / 64);
         k_build_ep<<<grid, 256, 0, st>>>(w->W_e, w->W_in, R->Ep, w->V, w->dtype);
+        if (R->use_tc) {
+            // persistent small-batch kernel: every CTA must be resident at once
+            int coop = 0, per_sm = 0;
+            if (cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, R->device) != cudaSuccess ||
+                cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_refine_small, 32 * (2 + 8),
+                                                              kRefineSmallSmemBytes) != cudaSuccess) {
+                (void)cudaGetLastError();
+                coop = 0;
+            }
+            if (coop && per_sm >= 1 && R->num_sms > SMALL_TRANS_CTAS) {
+                if (cudaMalloc(&R->Fhg, (size_t)2 * RANK * w->H * sizeof(float)) != cudaSuccess) {
+                    rc = XPRESS_ERR_CUDA;
+                    break;
+                }
+                k_fold_hidden<<<dim3((w->H + 255) / 256, 2 * RANK / 8), 256, 0, st>>>(
+                    static_cast<const uint16_t *>(w->W_h), static_cast<const uint16_t *>(w->W_g),
+                    static_cast<const uint16_t *>(w->W_in), R->Fhg, w->H);
+                R->small_ok = true;
+            }
+        }
         if (cudaGetLastError() != cudaSuccess || cudaStreamSynchronize(st) != cudaSuccess) rc = XPRESS_ERR_CUDA;
     } while (0);
     if (rc != XPRESS_OK) {
@@ -580,6 +690,7 @@ int xpress_refiner_destroy(xpress_refiner *R)
     if (!R) return XPRESS_ERR_INVALID_ARG;
     for (auto &e : R->cache) destroy_entry(e);
     if (R->Ep) cudaFree(R->Ep);
+    if (R->Fhg) cudaFree(R->Fhg);
     if (R->cs) cudaStreamDestroy(R->cs);
     if (R->trace) cudaFree(R->trace);
     delete R;
@@ -605,6 +716,7 @@ int xpress_refine_block(const xpress_refiner *Rc, const xpress_block_in *in, con
     const Layout L = make_layout(R, in->b);
     if (const int rc = check_ws(ws, ws_bytes, L.total)) return rc;
     Params P = make_params(R, in, out, ws, L);
+    if (L.small && !eager_mode()) return run_small(R, P, L, ws, static_cast<cudaStream_t>(stream));
     if (eager_mode()) return run_eager(R, P, L, ws, static_cast<cudaStream_t>(stream), eager_mode() == 2);
     const bool draft_null = in->draft == nullptr;
     GraphEntry *hit = nullptr, *victim = &R->cache[0];
