@@ -294,6 +294,8 @@ __device__ __forceinline__ unsigned atom_add_acq_rel_gpu(unsigned *p, unsigned v
     asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
     return old;
 }
+// Makes a preceding relaxed read an acquire (and later writes ordered after it).
+__device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
 // Orders this thread's generic-proxy global accesses with its later
 // async-proxy (TMA) accesses.
 __device__ __forceinline__ void fence_proxy_async_global()

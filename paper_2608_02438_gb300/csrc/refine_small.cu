@@ -96,8 +96,8 @@ __device__ bool wait_count(SmallCtl *c, const unsigned *ctr, unsigned target)
     const unsigned long long t0 = globaltimer();
     for (uint32_t it = 0; it < (1u << 26); ++it) {
         const unsigned v = ld_relaxed_gpu(ctr);
-        if (v & STOP_BIT) { __threadfence(); return false; }
-        if (v >= target) { __threadfence(); return true; }
+        if (v & STOP_BIT) { fence_acq_rel_gpu(); return false; }
+        if (v >= target) { fence_acq_rel_gpu(); return true; }
         if (it >= 2) __nanosleep(32);
         if ((it & 63u) == 63u && globaltimer() - t0 > 2000000000ull) break;
     }
@@ -293,8 +293,8 @@ __device__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUt
                 rowmax_item(p, item, lane);
     }
     __syncthreads();
+    // (release: the other threads' writes precede it through the barrier)
     if (threadIdx.x == 0) {
-        __threadfence();
         red_add_release_gpu(&c->pre_done.v, 1u);
         if (tr) trace_mark(p.trace, 2, t_start);
         // this CTA's W_r range into L2 while Pc and the first Trans run (after
@@ -404,7 +404,6 @@ __device__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUt
             const unsigned long long t_go = globaltimer_ns();
             const int n = *reinterpret_cast<volatile int *>(&sh.pass_n);
             if (ew == 0) {
-                __threadfence();
                 const int t = lane;
                 int tok = 0, pos = 0;
                 float invT = 0.0f;
@@ -492,7 +491,6 @@ __device__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUt
             }
             tv_epi_bar();
             if (ew == 0 && lane == 0) {
-                __threadfence();
                 sh.last = atom_add_acq_rel_gpu(&c->read_done.v, 1u) == (unsigned)(S * (pass + 1) - 1);
                 if (tr) trace_mark(p.trace, 8 + 4 * pass + 1, t_go);
             }
@@ -500,7 +498,6 @@ __device__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUt
             if (sh.last) {
                 // end of the pass: combine the partials of every evaluated
                 // token, apply the stopping rule, pack the next pass
-                __threadfence();
                 const unsigned long long t_last = globaltimer_ns();
                 for (int t = ew; t < n; t += TV_EPI_WARPS) {
                     const int tok = sh.tok[t];
@@ -517,7 +514,6 @@ __device__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUt
                     const bool more = converge_pack_small(p, sh.seq, sh.ynew, sh.yold, sh.passes, 0);
                     __syncwarp();
                     if (lane == 0) {
-                        __threadfence();
                         if (more) red_add_release_gpu(&c->pass_done.v, 1u);
                         else raise_stop(c, 0);
                         if (p.trace) trace_mark(p.trace, 8 + 4 * pass + 2, t_last);
@@ -679,7 +675,6 @@ __device__ void trans_role(const Params &p, SmallCtl *c, uint8_t *base, unsigned
         }
         __syncthreads();
         if (tid == 0) {
-            __threadfence();
             red_add_release_gpu(&c->c_ready.v, 1u);
             sh.go = wait_count(c, &c->c_ready.v, (unsigned)(8 * (pass + 1)));
             if (trs) trace_mark(p.trace, trs + 2, t_pass);
@@ -719,7 +714,6 @@ __device__ void trans_role(const Params &p, SmallCtl *c, uint8_t *base, unsigned
         }
         __syncthreads();
         if (tid == 0) {
-            __threadfence();
             red_add_release_gpu(&c->u_ready.v, 1u);
             sh.go = wait_count(c, &c->u_ready.v, (unsigned)(8 * (pass + 1)));
             if (trs) trace_mark(p.trace, trs + 3, t_pass);
@@ -764,7 +758,6 @@ __device__ void trans_role(const Params &p, SmallCtl *c, uint8_t *base, unsigned
         fence_proxy_async_global();                            // z is read by TMA
         __syncthreads();
         if (tid == 0) {
-            __threadfence();
             red_add_release_gpu(&c->z_ready.v, 1u);
             if (lead && p.trace) trace_mark(p.trace, 8 + 4 * pass, t_pass);
         }
