@@ -10,8 +10,10 @@ between timed steps; steps are timed with CUDA events on the launching stream.
 Also reported on the same JSON line:
   e2e           the same metric with host (pinned) inputs copied in and the
                 results copied out inside the timed region;
-  roofline      the Read + Correct + selection kernel launched alone (cold L2)
-                against the measured HBM copy bandwidth;
+  roofline      the dominant kernel launched alone (cold L2) against the
+                measured HBM copy bandwidth: for bf16 calls of at most 32
+                tokens the persistent kernel that runs the whole refinement,
+                otherwise the Read + Correct + selection kernel;
   cpu_baseline  the CPU oracle on one block of the same workload;
   clocks        nvidia-smi samples taken during the timed steps.
 
@@ -36,8 +38,13 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "refined draft blocks/s (Qwen3-8B shape, block 16)"
-READ_SOURCES = ["paper_2608_02438_gb300/csrc/read_tc.cu", "paper_2608_02438_gb300/csrc/common.cuh"]
-PROFILE_SUMMARY = "profiles/read_tc_qwen3_8b_greedy.txt"
+CSRC = "paper_2608_02438_gb300/csrc/"
+# sources of the kernel the roofline reports, and the ncu summary taken on them
+SMALL_SOURCES = [CSRC + f for f in ("refine_small.cu", "tcv_common.cuh", "mlp_common.cuh", "reduce_common.cuh",
+                                    "common.cuh")]
+SMALL_SUMMARY = "profiles/k_refine_small_qwen3_8b_greedy.txt"
+READ_SOURCES = [CSRC + "read_tc.cu", CSRC + "common.cuh"]
+READ_SUMMARY = "profiles/k_read_tc_serving_b32.txt"
 
 
 def dist_env():
@@ -52,10 +59,10 @@ def source_hash(paths):
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(bytes_hash: str):
-    """dram bytes per Read launch from the committed ncu summary, if it was
-    taken on the current kernel sources."""
-    path = os.path.join(ROOT, PROFILE_SUMMARY)
+def profiled_traffic(summary: str, bytes_hash: str):
+    """dram bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel sources."""
+    path = os.path.join(ROOT, summary)
     if not os.path.exists(path):
         return None
     kv = {}
@@ -210,11 +217,18 @@ def run_xpress(args):
         if ref.device_status("refine", b) != X.XPRESS_OK or ref.device_status("accept", b) != X.XPRESS_OK:
             raise RuntimeError("device status error")
         passes = ref.pass_count(b)
+        ctl = ref.control_words(b)
+        evaluated = ctl[4]                       # tokens evaluated over all passes
+        # bf16 calls of at most 32 tokens run as one persistent kernel (unless
+        # XPRESS_SMALL=0); others: init + precompute (two split-K GEMMs) +
+        # Fuse/Mix, then per pass Trans + Read + reduce.  Then the four
+        # acceptance kernels.
+        persistent = (dt == X.XPRESS_BF16 and b * cfg.B <= 32 and os.environ.get("XPRESS_SMALL", "1") != "0")
         small = b * cfg.B <= 32
-        # init + precompute (one GEMV, or two split-K GEMMs) + Fuse/Mix, then per
-        # pass Trans + Read (+ reduce unless fused into the small-batch Read),
-        # then the four acceptance kernels
-        per_step_launches = 1 + (1 if small else 2) + 1 + passes * (2 if small else 3) + 4
+        if persistent:
+            per_step_launches = 1 + 4
+        else:
+            per_step_launches = 1 + (1 if small else 2) + 1 + passes * (2 if small else 3) + 4
         starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
         ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
         if world > 1:
@@ -266,8 +280,8 @@ def run_xpress(args):
             ms_e2e = float(tt.item())
         e2e_value = world * b * n_e2e / (ms_e2e / 1000.0)
 
-        # roofline of the dominant kernel: Read + Correct + selection, alone,
-        # cold L2, over all b * B positions (a first pass)
+        # roofline of the dominant kernel, launched alone with L2 flushed
+        # before it (and, for context, with the previous launch's data in L2)
         step()
         torch.cuda.synchronize()
         ws_ptr, _ = ref.workspace("refine", b)
@@ -275,33 +289,50 @@ def run_xpress(args):
         reps = 50
         r_s = [torch.cuda.Event(enable_timing=True) for _ in range(reps)]
         r_e = [torch.cuda.Event(enable_timing=True) for _ in range(reps)]
-        for i in range(reps):
-            X.xpress_profile_read_prepare(ref.handle, ws_ptr, b, n_tok, stream.cuda_stream)
-            flush.zero_()
-            r_s[i].record(stream)
-            X.xpress_profile_read(ref.handle, ws_ptr, b, stream.cuda_stream)
-            r_e[i].record(stream)
-        torch.cuda.synchronize()
-        read_ms = float(np.mean([s.elapsed_time(e) for s, e in zip(r_s, r_e)]))
-        # the same launch with W_r left in L2 by the previous one (the state
-        # of passes 2.. of a call), for context
-        for i in range(reps):
-            X.xpress_profile_read_prepare(ref.handle, ws_ptr, b, n_tok, stream.cuda_stream)
-            r_s[i].record(stream)
-            X.xpress_profile_read(ref.handle, ws_ptr, b, stream.cuda_stream)
-            r_e[i].record(stream)
-        torch.cuda.synchronize()
-        read_warm_ms = float(np.median([s.elapsed_time(e) for s, e in zip(r_s, r_e)][2:]))
+
+        def dominant():
+            if persistent:       # the whole refinement is this one launch
+                ref.refine_block(d["h"], d["s"], d["draft"], d["anchor"], d["temperature"], d["seed"],
+                                 inp["offset"], cfg.K_max, out=out)
+            else:                # Read + Correct + selection over all b * B positions
+                X.xpress_profile_read(ref.handle, ws_ptr, b, stream.cuda_stream)
+
+        for cold in (True, False):
+            for i in range(reps):
+                if not persistent:
+                    X.xpress_profile_read_prepare(ref.handle, ws_ptr, b, n_tok, stream.cuda_stream)
+                if cold:
+                    flush.zero_()
+                r_s[i].record(stream)
+                dominant()
+                r_e[i].record(stream)
+            torch.cuda.synchronize()
+            times = [s.elapsed_time(e) for s, e in zip(r_s, r_e)]
+            if cold:
+                read_ms = float(np.mean(times))
+            else:
+                read_warm_ms = float(np.median(times[2:]))
     esz = 2 if dt == X.XPRESS_BF16 else 4
-    small = b * cfg.B <= 32
-    read_kernel = "k_read_tcv" if small else "k_read_tc"
-    rows = 128 if small else 256
-    S = min(ref.torch.cuda.get_device_properties(dev).multi_processor_count, (cfg.V + rows - 1) // rows)
-    read_bytes = cfg.V * cfg.r * esz + n_tok * cfg.V * esz + n_tok * cfg.r * esz + S * n_tok * 16
+    sms = ref.torch.cuda.get_device_properties(dev).multi_processor_count
+    if persistent:
+        # algorithmic bytes of one call: the folded projection [2r, H] fp32 and
+        # h once; per pass W_r; per evaluated token its s row, its E' row, its
+        # z operand and 16-byte partial per vocabulary range
+        read_kernel = "k_refine_small"
+        S = min(sms - 8, (cfg.V + 127) // 128)
+        read_bytes = (2 * cfg.r * cfg.H * 4 + n_tok * cfg.H * esz + passes * cfg.V * cfg.r * esz
+                      + evaluated * (cfg.V * esz + cfg.r * 4 + cfg.r * esz + 2 * S * 16))
+        summary, srcs = SMALL_SUMMARY, SMALL_SOURCES
+    else:
+        read_kernel = "k_read_tcv" if small else "k_read_tc"
+        rows = 128 if small else 256
+        S = min(sms, (cfg.V + rows - 1) // rows)
+        read_bytes = cfg.V * cfg.r * esz + n_tok * cfg.V * esz + n_tok * cfg.r * esz + S * n_tok * 16
+        summary, srcs = READ_SUMMARY, READ_SOURCES
     hbm, tc_peak, src = peaks()
     achieved = read_bytes / (read_ms / 1000.0) / 1e9
-    rhash = source_hash(READ_SOURCES)
-    traffic = profiled_traffic(rhash)
+    rhash = source_hash(srcs)
+    traffic = profiled_traffic(summary, rhash)
 
     if rank == 0:
         cpu_val, cpu_n, cpu_el = cpu_baseline(args.config)
@@ -322,7 +353,9 @@ def run_xpress(args):
                          "frac": achieved / hbm, "traffic": traffic, "peak_source": src,
                          "kernel": read_kernel, "bytes_per_launch": read_bytes, "launch_ms": read_ms,
                          "launch_ms_l2_warm": read_warm_ms,
-                         "tokens_per_launch": n_tok, "source_hash": rhash},
+                         "tokens_per_launch": n_tok, "passes_per_launch": passes if persistent else 1,
+                         "tokens_evaluated_per_launch": evaluated if persistent else n_tok,
+                         "source_hash": rhash},
             "cpu_baseline": {"value": cpu_val, "unit": "blocks/s", "cores": 1, "kind": "oracle",
                              "sample": f"{cpu_n} whole block(s) of {cfg.name} (Algorithm 1 + acceptance), fp64, "
                                        f"one thread, {cpu_el:.1f} s"},

@@ -256,6 +256,15 @@ class Refiner:
         ws, _ = self.workspace(kind, b)
         return xpress_get_device_status(ws, self.stream.cuda_stream)
 
+    def control_words(self, b: int):
+        """The refine workspace's control words (passes run, tokens evaluated
+        over all passes, ...), read after a synchronize; for measurement."""
+        self.torch.cuda.synchronize()
+        ws, _ = self.workspace("refine", b)
+        buf = self._ws[("refine", b)]
+        off = ws - buf.data_ptr() + 64
+        return buf[off:off + 32].view(self.torch.int32).cpu().tolist()
+
     def pass_count(self, b: int) -> int:
         ws, _ = self.workspace("refine", b)
         return xpress_get_pass_count(ws, self.stream.cuda_stream)

@@ -29,6 +29,7 @@ constexpr int CTL_NACT = 0;     // tokens evaluated by the next pass
 constexpr int CTL_DONE = 1;     // last-block-done ticket of the reduce kernel
 constexpr int CTL_PASS = 2;     // passes executed so far
 constexpr int CTL_ACC_DONE = 3; // ticket of the accept kernels
+constexpr int CTL_EVAL = 4;     // tokens evaluated by all passes so far (sum over passes)
 constexpr int CTL_WORDS = 8;
 constexpr int RMAX_SEG = 32;    // vocabulary segments of the argmax-s scan
 

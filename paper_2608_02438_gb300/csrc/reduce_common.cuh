@@ -185,6 +185,7 @@ __device__ __forceinline__ bool converge_pack_small(const Params &p, const SeqSt
         p.ctl[CTL_NACT] = total;
         p.ctl[CTL_DONE] = 0;
         p.ctl[CTL_PASS] = passes;
+        if (more) p.ctl[CTL_EVAL] += total;
         if (p.use_graph) cudaGraphSetConditional(handle, more ? 1u : 0u);
     }
     return more;
@@ -240,6 +241,7 @@ __device__ __forceinline__ void pack_next_pass(const Params &p, cudaGraphConditi
         p.ctl[CTL_NACT] = carry;
         p.ctl[CTL_DONE] = 0;
         p.ctl[CTL_PASS] = passes;
+        if (carry > 0 && passes < p.K_max) p.ctl[CTL_EVAL] += carry;
         // no block can take part in more than K_max passes; the cap also bounds
         // the loop should the per-block bookkeeping ever disagree
         if (p.use_graph) cudaGraphSetConditional(handle, (carry > 0 && passes < p.K_max) ? 1u : 0u);

@@ -42,6 +42,7 @@ __global__ void k_init(Params pin, Params *pdev, cudaGraphConditionalHandle hand
         p.ctl[CTL_NACT] = p.N;
         p.ctl[CTL_DONE] = 0;
         p.ctl[CTL_PASS] = 0;
+        p.ctl[CTL_EVAL] = p.N;
         if (p.use_graph) cudaGraphSetConditional(handle, 1u);
     }
     if (t < p.N) {

@@ -579,7 +579,7 @@ __device__ void trans_role(const Params &p, SmallCtl *c, uint8_t *base, unsigned
             if (p.iters) p.iters[tid] = 0;
             if (p.converged) p.converged[tid] = 0;
         }
-        if (tid == 0) { p.ctl[CTL_NACT] = N; p.ctl[CTL_DONE] = 0; p.ctl[CTL_PASS] = 0; }
+        if (tid == 0) { p.ctl[CTL_NACT] = N; p.ctl[CTL_DONE] = 0; p.ctl[CTL_PASS] = 0; p.ctl[CTL_EVAL] = N; }
     }
     if (tid == 0) sh.go = wait_count(c, &c->pre_done.v, (unsigned)p.S);
     __syncthreads();
