@@ -317,17 +317,17 @@ def run_xpress(args):
     if persistent:
         # algorithmic bytes of one call: the folded projection [2r, H] fp32 and
         # h once; per pass W_r; per evaluated token its s row, its E' row, its
-        # z operand and 16-byte partial per vocabulary range
+        # z operand and a 32-byte partial per vocabulary range (written, read)
         read_kernel = "k_refine_small"
         S = min(sms - 8, (cfg.V + 127) // 128)
         read_bytes = (2 * cfg.r * cfg.H * 4 + n_tok * cfg.H * esz + passes * cfg.V * cfg.r * esz
-                      + evaluated * (cfg.V * esz + cfg.r * 4 + cfg.r * esz + 2 * S * 16))
+                      + evaluated * (cfg.V * esz + cfg.r * 4 + cfg.r * esz + 2 * S * 32))
         summary, srcs = SMALL_SUMMARY, SMALL_SOURCES
     else:
         read_kernel = "k_read_tcv" if small else "k_read_tc"
         rows = 128 if small else 256
         S = min(sms, (cfg.V + rows - 1) // rows)
-        read_bytes = cfg.V * cfg.r * esz + n_tok * cfg.V * esz + n_tok * cfg.r * esz + S * n_tok * 16
+        read_bytes = cfg.V * cfg.r * esz + n_tok * cfg.V * esz + n_tok * cfg.r * esz + S * n_tok * 32
         summary, srcs = READ_SUMMARY, READ_SOURCES
     hbm, tc_peak, src = peaks()
     achieved = read_bytes / (read_ms / 1000.0) / 1e9

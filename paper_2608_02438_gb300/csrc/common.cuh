@@ -54,6 +54,21 @@ struct Partial {
     float s;
 };
 
+// One split-vocabulary partial of the Read (per vocabulary range and evaluated
+// token): Partial's fields plus, for T > 0, the member draw of the range's
+// best group -- y (token id) and sel = l_y / T -- taken when that group became
+// the range's best, so that combining the ranges needs no second pass over the
+// winning group.
+struct alignas(16) RPartial {
+    float best;
+    int idx;
+    float m;
+    float s;
+    int y;
+    float sel;
+    int pad0, pad1;
+};
+
 // Counters through which the CTAs of the persistent small-batch kernel hand
 // work to one another (one 128-byte line each).  They only grow during a
 // call; STOP_BIT set in a counter tells its waiters to leave.  A call uses one
@@ -69,8 +84,7 @@ struct SmallCtl {
     CtlLine c_ready;     // Trans CTAs that published their slice of c (8 per pass)
     CtlLine u_ready;     // ... of sigma(W_1 c)
     CtlLine z_ready;     // ... of z
-    CtlLine pass_done;   // passes whose end (reduce, stopping rule, pack) is written
-    CtlLine read_done;   // Read CTAs done with their partials (ticket)
+    CtlLine read_done;   // Read CTAs done with their partials (S per pass)
     CtlLine exit_cnt;    // CTAs that left (ticket)
     CtlLine status;      // device status bits of the call
 };
@@ -112,13 +126,14 @@ struct Params {
     int32_t *act_tok;            // [N] packed evaluated tokens (global token ids)
     void *zpack;                 // [N, r] W_r operand of the evaluated tokens
     float *zbuf;                 // [N, r] fp32 z when the caller passes no z_final
-    Partial *part;               // [S, N]
+    RPartial *part;              // [S, N]
     // persistent small-batch kernel only
     const float *Fhg;            // [2r, H] fp32: rows W_in[:, 0:r] W_h, then W_in[:, r:2r] W_g
     int pre_kslice, pre_ks;      // K-slice width of the hidden projection and the number of slices
     uint16_t *cx, *ux;           // [32, r] c and [32, 2r] sigma(W_1 c), bf16, exchanged by the Trans CTAs
     Partial *rmax;               // [N, RMAX_SEG] argmax-s partials (calls without a draft)
     SmallCtlArea *sctl;          // control blocks of the persistent kernel
+    unsigned long long *best64;  // [2][32] per pass parity: max over ranges of argmax_key (greedy tokens)
 };
 
 // ------------------------------------------------------------------ numbers
@@ -203,11 +218,45 @@ __device__ __forceinline__ void merge_partial(Partial &a, const Partial &b, bool
     if (sampling) merge_lse(a.m, a.s, b.m, b.s);
 }
 
+// Greedy selection as one 64-bit key whose unsigned maximum is the argmax with
+// the smallest id among equal values: the fp32 value mapped to an
+// order-preserving unsigned word (high half), the inverted id (low half).
+__device__ __forceinline__ unsigned long long argmax_key(float best, int idx)
+{
+    const uint32_t b = __float_as_uint(best);
+    const uint32_t u = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+    return ((unsigned long long)u << 32) | (unsigned long long)(0xFFFFFFFFu - (uint32_t)idx);
+}
+__device__ __forceinline__ void argmax_unkey(unsigned long long key, float &best, int &idx)
+{
+    const uint32_t u = (uint32_t)(key >> 32);
+    best = __uint_as_float((u & 0x80000000u) ? (u & 0x7FFFFFFFu) : ~u);
+    idx = (int)(0xFFFFFFFFu - (uint32_t)key);
+}
+
+// Combining two Read partials: the argmax side carries its member draw.
+__device__ __forceinline__ void merge_rpartial(RPartial &a, const RPartial &b, bool sampling)
+{
+    if (b.best > a.best || (b.best == a.best && b.idx < a.idx)) {
+        a.best = b.best; a.idx = b.idx; a.y = b.y; a.sel = b.sel;
+    }
+    if (sampling) merge_lse(a.m, a.s, b.m, b.s);
+}
+
 // Per-token selection state over a run of 32-wide vocabulary groups.
 struct SelState {
     float best; int idx; float m; float s;
-    __device__ __forceinline__ void init() { best = -INFINITY; idx = 0x7fffffff; m = -INFINITY; s = 0.0f; }
+    int y; float sel;                         // T > 0: member draw of the best group
+    __device__ __forceinline__ void init()
+    {
+        best = -INFINITY; idx = 0x7fffffff; m = -INFINITY; s = 0.0f; y = 0x7fffffff; sel = -INFINITY;
+    }
+    __device__ __forceinline__ RPartial partial() const { return RPartial{best, idx, m, s, y, sel, 0, 0}; }
 };
+__device__ __forceinline__ RPartial rpartial_identity()
+{
+    return RPartial{-INFINITY, 0x7fffffff, -INFINITY, 0.0f, 0x7fffffff, -INFINITY, 0, 0};
+}
 
 // Fold one group of 32 corrected logits l[v0 .. v0+31] (entries j >= valid
 // are ignored) into the state.  T <= 0: argmax.  T > 0: x = l * invT, the
@@ -245,7 +294,31 @@ __device__ __forceinline__ void select_group(SelState &st, const float *l, int v
         if (j < valid) sum += __expf(x[j] - mx);
     const uint32_t g = (uint32_t)v0 / GROUP;
     const float score = mx + __logf(sum) + gumbel(seed, g, pos, STREAM_GROUP, offset);
-    if (score > st.best) { st.best = score; st.idx = (int)g; }
+    if (score > st.best) {
+        // the group is this range's best so far: draw its member now (Gumbel-max
+        // over the members, smallest id on ties), one Philox call per 4 ids
+        st.best = score;
+        st.idx = (int)g;
+        float bsc = -INFINITY, bx = x[0];
+        int bj = 0;
+#pragma unroll
+        for (int c = 0; c < GROUP / 4; ++c) {
+            const uint4 o = philox10(make_uint4(((uint32_t)v0 >> 2) + c, pos, STREAM_ELEM, offset), (uint32_t)seed,
+                                     (uint32_t)(seed >> 32));
+            const uint32_t w4[4] = {o.x, o.y, o.z, o.w};
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int j = 4 * c + q;
+                if (j < valid) {
+                    const float u = ((float)(w4[q] >> 9) + 0.5f) * (1.0f / 8388608.0f);
+                    const float sc = x[j] - logf(-logf(u));
+                    if (sc > bsc) { bsc = sc; bj = j; bx = x[j]; }
+                }
+            }
+        }
+        st.y = v0 + bj;
+        st.sel = bx;
+    }
     merge_lse(st.m, st.s, mx, sum);
 }
 

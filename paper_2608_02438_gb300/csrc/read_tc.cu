@@ -313,19 +313,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             if (!stop) {
                 if (small) {
                     if (ew == 0 && lane < n) {
-                        Partial a{sh.st[0][lane].best, sh.st[0][lane].idx, sh.st[0][lane].m, sh.st[0][lane].s};
-                        for (int w = 1; w < TC_EPI_WARPS; ++w) {
-                            const Partial b{sh.st[w][lane].best, sh.st[w][lane].idx, sh.st[w][lane].m,
-                                            sh.st[w][lane].s};
-                            merge_partial(a, b, invT > 0.0f);
-                        }
+                        RPartial a = sh.st[0][lane].partial();
+                        for (int w = 1; w < TC_EPI_WARPS; ++w) merge_rpartial(a, sh.st[w][lane].partial(), invT > 0.0f);
                         p.part[(size_t)r * p.N + lane] = a;
                     }
                 } else if (ew < 4 && valid) {
-                    Partial a{sh.st[ew][lane].best, sh.st[ew][lane].idx, sh.st[ew][lane].m, sh.st[ew][lane].s};
-                    const Partial b{sh.st[ew + 4][lane].best, sh.st[ew + 4][lane].idx, sh.st[ew + 4][lane].m,
-                                    sh.st[ew + 4][lane].s};
-                    merge_partial(a, b, invT > 0.0f);
+                    RPartial a = sh.st[ew][lane].partial();
+                    merge_rpartial(a, sh.st[ew + 4][lane].partial(), invT > 0.0f);
                     p.part[(size_t)r * p.N + i] = a;
                 }
             }

@@ -255,11 +255,8 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
         sh.st[ew][lane] = sel;
         const bool stop = tv_epi_bar_or(!ok || *abort);
         if (!stop && ew == 0 && lane < n) {
-            Partial a{sh.st[0][lane].best, sh.st[0][lane].idx, sh.st[0][lane].m, sh.st[0][lane].s};
-            for (int w = 1; w < TV_EPI_WARPS; ++w) {
-                const Partial b{sh.st[w][lane].best, sh.st[w][lane].idx, sh.st[w][lane].m, sh.st[w][lane].s};
-                merge_partial(a, b, my_invT > 0.0f);
-            }
+            RPartial a = sh.st[0][lane].partial();
+            for (int w = 1; w < TV_EPI_WARPS; ++w) merge_rpartial(a, sh.st[w][lane].partial(), my_invT > 0.0f);
             p.part[(size_t)r * p.N + lane] = a;
         }
     }
@@ -288,7 +285,7 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
             if (tr0 && threadIdx.x == 0) trace_mark(p.trace, 204, t_wait);
             for (int t = warp; t < n; t += TV_THREADS / 32) {
                 const int tok = sh.tok[t];
-                const TokenResult res = reduce_token(p, t, tok, sh.invT[t], sh.seed[t]);
+                const TokenResult res = reduce_token(p, t, sh.invT[t]);
                 if (lane == 0) {
                     sh.ynew[t] = res.y;
                     if (p.lse) p.lse[tok] = res.lse;

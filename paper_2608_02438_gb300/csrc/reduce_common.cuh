@@ -8,16 +8,6 @@
 
 namespace xp {
 
-__device__ __forceinline__ void bf16x8_to_float(const uint4 &w, float (&x)[8])
-{
-    const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        x[2 * q] = __uint_as_float(ww[q] << 16);
-        x[2 * q + 1] = __uint_as_float(ww[q] & 0xFFFF0000u);
-    }
-}
-
 struct TokenResult {
     int y;
     float sel, lse;
@@ -33,76 +23,65 @@ __device__ __forceinline__ Partial ldcg_partial(const Partial *q)
     return Partial{v.x, __float_as_int(v.y), v.z, v.w};
 }
 
-__device__ __forceinline__ TokenResult reduce_token(const Params &p, int i, int tok, float invT,
-                                                    unsigned long long seed)
+// A Read partial through L2 (a CTA of the persistent kernel may combine
+// several passes, so L1 could hold an older copy).
+__device__ __forceinline__ RPartial ldcg_rpartial(const RPartial *q)
 {
-    const int lane = threadIdx.x % 32, k = tok % p.B;
-    const bool sampling = invT > 0.0f;
-    Partial a{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
-    // the lane's partials (ranges lane, lane + 32, ...) requested together
-    constexpr int PER = 8;
-    for (int r0 = 0; r0 < p.S; r0 += 32 * PER) {
-        Partial pv[PER];
-#pragma unroll
-        for (int j = 0; j < PER; ++j) {
-            const int r = r0 + lane + 32 * j;
-            // through L2: a CTA of the persistent kernel may reduce several passes
-            pv[j] = r < p.S ? ldcg_partial(p.part + (size_t)r * p.N + i)
-                            : Partial{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
-        }
-#pragma unroll
-        for (int j = 0; j < PER; ++j) merge_partial(a, pv[j], sampling);
-    }
+    const float4 a = __ldcg(reinterpret_cast<const float4 *>(q));
+    const float4 b = __ldcg(reinterpret_cast<const float4 *>(q) + 1);
+    return RPartial{a.x, __float_as_int(a.y), a.z, a.w, __float_as_int(b.x), b.y, 0, 0};
+}
+
+// Second half of reduce_token: combines the lane partials `a` of one evaluated
+// token across the warp.  T <= 0: the argmax and its logit.  T > 0: the drawn
+// group's member draw (taken by the Read when the group became its range's
+// best), l_y / T, and log sum exp(l / T).  Warp-collective.
+__device__ __forceinline__ TokenResult finish_token(RPartial a, bool sampling)
+{
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
-        Partial b;
+        RPartial b;
         b.best = __shfl_xor_sync(0xffffffffu, a.best, o);
         b.idx = __shfl_xor_sync(0xffffffffu, a.idx, o);
         b.m = __shfl_xor_sync(0xffffffffu, a.m, o);
         b.s = __shfl_xor_sync(0xffffffffu, a.s, o);
-        merge_partial(a, b, sampling);
+        b.y = __shfl_xor_sync(0xffffffffu, a.y, o);
+        b.sel = __shfl_xor_sync(0xffffffffu, a.sel, o);
+        merge_rpartial(a, b, sampling);
     }
     TokenResult res;
     if (!sampling) {
         res.y = a.idx;
         res.sel = a.best;
         res.lse = __int_as_float(0x7fc00000);
-        return res;
+    } else {
+        res.y = a.y;
+        res.sel = a.sel;
+        res.lse = a.m + logf(a.s);
     }
-    const int v = a.idx * GROUP + lane;
-    float x = -INFINITY, score = -INFINITY;
-    if (v < p.V) {
-        float acc = 0.0f;
-        if (p.dtype) {
-            const uint4 *wr = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.W_r) + (size_t)v * RANK);
-            const uint4 *zr = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.zpack) + (size_t)i * RANK);
-#pragma unroll 8
-            for (int c = 0; c < RANK / 8; ++c) {
-                float w8[8], z8[8];
-                bf16x8_to_float(__ldg(wr + c), w8);
-                bf16x8_to_float(zr[c], z8);
-#pragma unroll
-                for (int j = 0; j < 8; ++j) acc = fmaf(w8[j], z8[j], acc);
-            }
-        } else {
-            for (int d = 0; d < RANK; ++d)
-                acc = fmaf(ld_any(p.W_r, 0, (size_t)v * RANK + d), ld_any(p.zpack, 0, (size_t)i * RANK + d), acc);
-        }
-        x = (acc + ld_any(p.s, p.dtype, (size_t)tok * p.V + v)) * invT;
-        score = x + gumbel(seed, (uint32_t)v, (uint32_t)k, STREAM_ELEM, p.offset);
-    }
-    float bs = score;
-    int bi = v;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        const float os = __shfl_xor_sync(0xffffffffu, bs, o);
-        const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-        merge_argmax(bs, bi, os, oi);
-    }
-    res.y = bi;
-    res.sel = __shfl_sync(0xffffffffu, x, (bi - a.idx * GROUP) & (GROUP - 1));
-    res.lse = a.m + logf(a.s);
     return res;
+}
+
+// Combines the S Read partials of evaluated token i.  Warp-collective.
+__device__ __forceinline__ TokenResult reduce_token(const Params &p, int i, float invT)
+{
+    const int lane = threadIdx.x % 32;
+    const bool sampling = invT > 0.0f;
+    RPartial a = rpartial_identity();
+    // the lane's partials (ranges lane, lane + 32, ...) requested together
+    // (one round for up to 160 ranges)
+    constexpr int PER = 5;
+    for (int r0 = 0; r0 < p.S; r0 += 32 * PER) {
+        RPartial pv[PER];
+#pragma unroll
+        for (int j = 0; j < PER; ++j) {
+            const int r = r0 + lane + 32 * j;
+            pv[j] = r < p.S ? ldcg_rpartial(p.part + (size_t)r * p.N + i) : rpartial_identity();
+        }
+#pragma unroll
+        for (int j = 0; j < PER; ++j) merge_rpartial(a, pv[j], sampling);
+    }
+    return finish_token(a, sampling);
 }
 
 // Algorithm 1's stopping rule for block s after a pass that evaluated

@@ -690,11 +690,8 @@ __global__ void __launch_bounds__(256) k_read_simt(const Params *__restrict__ pp
         __syncthreads();
         if (warp == 0 && lane < nt) {
             const bool sampling = invT > 0.0f;
-            Partial a{sst[0][lane].best, sst[0][lane].idx, sst[0][lane].m, sst[0][lane].s};
-            for (int w = 1; w < 8; ++w) {
-                const Partial b{sst[w][lane].best, sst[w][lane].idx, sst[w][lane].m, sst[w][lane].s};
-                merge_partial(a, b, sampling);
-            }
+            RPartial a = sst[0][lane].partial();
+            for (int w = 1; w < 8; ++w) merge_rpartial(a, sst[w][lane].partial(), sampling);
             p.part[(size_t)blockIdx.x * p.N + t0 + lane] = a;
         }
         __syncthreads();
@@ -721,7 +718,7 @@ __global__ void __launch_bounds__(1024) k_reduce(const Params *__restrict__ pp, 
         const int k = warp, i = st.off + (k - st.m - 1), tok = s * B + k;
         if (lane == 0) yold[k] = p.tokens[tok];
         const float T = p.temperature[s];
-        const TokenResult res = reduce_token(p, i, tok, T > 0.0f ? 1.0f / T : 0.0f, p.seed[s]);
+        const TokenResult res = reduce_token(p, i, T > 0.0f ? 1.0f / T : 0.0f);
         if (lane == 0) {
             ynew[k] = res.y;
             if (p.lse) p.lse[tok] = res.lse;

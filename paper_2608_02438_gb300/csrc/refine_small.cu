@@ -16,13 +16,16 @@
 //     or the fixed-noise group draw) over a fixed range of 128-row vocabulary
 //     blocks: W_r rows are the tcgen05 M dimension, the <= 32 tokens N, and an
 //     8-stage TMA ring streams W_r, running ahead into the next pass while the
-//     Trans CTAs work.  The CTA that finishes a pass last combines the
-//     per-range partials, applies the stopping rule and packs the next pass.
+//     Trans CTAs work.  Each range leaves one partial per token (for T > 0
+//     with the member draw of its best group already taken).
 //   Trans CTAs (S .. S + 7).  CTA j owns channels [32 j, 32 j + 32).  Once per
 //     call they finish Pc = (I + L) P for their channels (Eq. mix); in every
 //     pass they gather E' rows for the current tokens, mix (Eq. fuse / mix) and
 //     run Trans z = c + W_2 sigma(W_1 c) (Eq. mlp) on tensor cores, exchanging
-//     c and sigma(W_1 c) through L2.
+//     c and sigma(W_1 c) through L2.  Then each of them combines the Read
+//     partials, applies Algorithm 1's stopping rule and packs the next pass
+//     (the same result in all eight; the first one publishes it), so the next
+//     pass starts without another hand-off.
 //
 // The roles hand work to one another through monotone counters (SmallCtl,
 // release / acquire at GPU scope).  Every wait is bounded: a wait that runs
@@ -48,12 +51,9 @@ struct RsShared {                              // Read CTA, after the W_r stages
     uint32_t tmem_base;
     int abort;
     int pass_n, pass_stop;                     // published by the producer with `go`
-    int last, passes;
     int tok[TV_BN], pos[TV_BN];
     float invT[TV_BN];
     unsigned long long seed[TV_BN];
-    int ynew[TV_BN], yold[TV_BN];
-    SeqState seq[TV_BN];
     SelState sel[TV_EPI_WARPS][32];
     float tile[TV_EPI_WARPS][TV_BN][33];       // per-warp transpose: [token][vocabulary row]
 };
@@ -65,7 +65,11 @@ struct TsShared {                              // Trans CTA
     float zhalf[2][MAX_B][32];                 // W_2 u, the two K halves
     int tok[MAX_B];                            // evaluated tokens of the pass (global ids)
     int x[MAX_B];                              // current tokens Y
-    int n, go;
+    int ynew[MAX_B], yold[MAX_B];              // per evaluated token: new / previous token
+    int tok2[MAX_B];                           // evaluated tokens of the next pass
+    SeqState st[MAX_B];                        // per block: Algorithm 1 state
+    float invT[MAX_B];                         // per block: 1 / T (0 for greedy)
+    int n, n2, go, more;
 };
 
 constexpr size_t RS_BYTES = 1024 + TV_STAGES * TV_A_STAGE + TV_Z_BYTES + sizeof(RsShared);
@@ -76,7 +80,7 @@ constexpr size_t SMALL_SMEM = RS_BYTES > TS_BYTES ? RS_BYTES : TS_BYTES;
 // ------------------------------------------------------------- signalling
 
 // Records `bits` (if any) and sets the stop bit of every counter.
-__device__ void raise_stop(SmallCtl *c, int bits)
+__device__ __forceinline__ void raise_stop(SmallCtl *c, int bits)
 {
     if (bits) atomicOr(reinterpret_cast<int *>(&c->status.v), bits);
     __threadfence();
@@ -84,14 +88,14 @@ __device__ void raise_stop(SmallCtl *c, int bits)
     atomicOr(&c->c_ready.v, STOP_BIT);
     atomicOr(&c->u_ready.v, STOP_BIT);
     atomicOr(&c->z_ready.v, STOP_BIT);
-    atomicOr(&c->pass_done.v, STOP_BIT);
+    atomicOr(&c->read_done.v, STOP_BIT);
 }
 
 // One thread: waits until *ctr >= target (true).  false once the stop bit is
 // set, or after about 2 s (the timeout is recorded and every role stops).
 // Relaxed polls with a short sleep keep ~150 pollers from crowding the line's
 // L2 slice; the fence after the last poll makes it an acquire.
-__device__ bool wait_count(SmallCtl *c, const unsigned *ctr, unsigned target)
+__device__ __forceinline__ bool wait_count(SmallCtl *c, const unsigned *ctr, unsigned target)
 {
     const unsigned long long t0 = globaltimer();
     for (uint32_t it = 0; it < (1u << 26); ++it) {
@@ -107,7 +111,7 @@ __device__ bool wait_count(SmallCtl *c, const unsigned *ctr, unsigned target)
 
 // One thread per CTA, last action on the control area: the CTA that leaves
 // last publishes the call's status and hands the other block to the next call.
-__device__ void leave(const Params &p, SmallCtlArea *a, SmallCtl *c, int par)
+__device__ __forceinline__ void leave(const Params &p, SmallCtlArea *a, SmallCtl *c, int par)
 {
     __threadfence();
     if (atomicAdd(&c->exit_cnt.v, 1u) == gridDim.x - 1) {
@@ -145,7 +149,7 @@ __device__ __forceinline__ float reduce_scatter_n(float (&v)[NT], int lane)
 // slice is staged in `hs` (bf16 [N][pre_kslice]).  The 8 epilogue warps call
 // this together.
 template <int NT>
-__device__ void pre_item(const Params &p, int item, uint16_t *hs, int w, int lane)
+__device__ __forceinline__ void pre_item(const Params &p, int item, uint16_t *hs, int w, int lane)
 {
     constexpr int R = 64 / NT, ROWS = 8 * R, NG = 2 * RANK / ROWS;
     const int rg = item % NG, ks = item / NG;
@@ -218,7 +222,7 @@ __device__ void pre_item(const Params &p, int item, uint16_t *hs, int w, int lan
 
 // Partial argmax of s[t, segment] (fp32 compare of the bf16 values, smallest
 // id among equal maxima).  One warp.
-__device__ void rowmax_item(const Params &p, int item, int lane)
+__device__ __forceinline__ void rowmax_item(const Params &p, int item, int lane)
 {
     const int t = item / RMAX_SEG, seg = item % RMAX_SEG, V = p.V;
     const int v0 = (int)((long long)V * seg / RMAX_SEG), v1 = (int)((long long)V * (seg + 1) / RMAX_SEG);
@@ -241,7 +245,7 @@ __device__ void rowmax_item(const Params &p, int item, int lane)
 
 // ------------------------------------------------------------- Read role
 
-__device__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUtensorMap *tmap_z, SmallCtl *c,
+__device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUtensorMap *tmap_z, SmallCtl *c,
                           uint8_t *base, unsigned long long t_start)
 {
     uint8_t *sA = base;                                    // W_r stages (h slices before the first pass)
@@ -328,7 +332,9 @@ __device__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUt
             };
             long long next = 0;
             bool ok = true;
-            for (; next < ahead && ok; ++next) ok = issue(next);
+            const bool lookahead = !(p.read_flags & 2);
+            if (lookahead)
+                for (; next < ahead && ok; ++next) ok = issue(next);
             for (int pass = 0; ok; ++pass) {
                 const bool go = wait_count(c, &c->z_ready.v, (unsigned)(8 * (pass + 1)));
                 if (go) {
@@ -336,6 +342,7 @@ __device__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUt
                     sh.pass_n = min(__ldcg(p.ctl + CTL_NACT), TV_BN);
                 }
                 sh.pass_stop = go ? 0 : 1;
+                if (p.trace && pass == 1) { const unsigned long long tn = globaltimer_ns(); trace_mark(p.trace, 201, tn); }
                 mbar_arrive(&sh.go);
                 if (!go) break;
                 // z of this pass, once the previous pass's MMAs are done with it
@@ -345,7 +352,7 @@ __device__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUt
                 z_issued = true;
                 z_par = (uint32_t)(pass & 1);
                 // the rest of this pass, then the first chunks of the next one
-                const long long end = (long long)(pass + 1) * per_pass + ahead;
+                const long long end = (long long)(pass + 1) * per_pass + (lookahead ? ahead : 0);
                 for (; next < end; ++next)
                     if (!issue(next)) { ok = false; break; }
             }
@@ -364,6 +371,7 @@ __device__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUt
                 if (*reinterpret_cast<volatile int *>(&sh.pass_stop)) break;
                 if (!mbar_wait(&sh.z_full, (uint32_t)(pass & 1), abort)) break;
                 tc_fence_after();
+                if (p.trace && pass == 1) { const unsigned long long tn = globaltimer_ns(); trace_mark(p.trace, 202, tn); }
                 bool ok = true;
                 for (int i = 0; i < nblk && ok; ++i) {
                     const int ib = pass * nblk + i, buf = ib % TV_NBUF;
@@ -386,6 +394,7 @@ __device__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUt
                 }
                 if (!ok) break;
                 tc_commit(&sh.z_empty);
+                if (p.trace && pass == 1) { const unsigned long long tn = globaltimer_ns(); trace_mark(p.trace, 203, tn); }
             }
             tc_commit(&sh.drain);
             int dummy = 0;
@@ -415,18 +424,11 @@ __device__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUt
                     const float T = p.temperature[s];
                     invT = T > 0.0f ? 1.0f / T : 0.0f;
                     seed = p.seed[s];
-                    sh.yold[t] = __ldcg(p.tokens + tok);
                 }
                 sh.tok[t] = tok;
                 sh.pos[t] = pos;
                 sh.invT[t] = invT;
                 sh.seed[t] = seed;
-                if (t < p.b) {
-                    const int4 *src = reinterpret_cast<const int4 *>(p.st + t);
-                    const int4 a = __ldcg(src), b2 = __ldcg(src + 1);
-                    sh.seq[t] = SeqState{a.x, a.y, a.z, a.w, b2.x, b2.y, b2.z, b2.w};
-                }
-                if (t == 0) sh.passes = __ldcg(p.ctl + CTL_PASS);
             }
             tv_epi_bar();
             const int my_tok = sh.tok[lane], my_pos = sh.pos[lane];
@@ -479,46 +481,20 @@ __device__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUt
                 for (int cc = 0; cc < 4; ++cc) cur[cc] = nxt[cc];
             }
             sh.sel[ew][lane] = sel;
+            if (p.trace && pass == 1 && lane == 0) { const unsigned long long tn = globaltimer_ns(); trace_mark(p.trace, 204, tn); }
             if (tv_epi_bar_or(!ok || *abort)) break;
             if (ew == 0 && lane < n) {
-                Partial a{sh.sel[0][lane].best, sh.sel[0][lane].idx, sh.sel[0][lane].m, sh.sel[0][lane].s};
-                for (int w2 = 1; w2 < TV_EPI_WARPS; ++w2) {
-                    const Partial b2{sh.sel[w2][lane].best, sh.sel[w2][lane].idx, sh.sel[w2][lane].m,
-                                     sh.sel[w2][lane].s};
-                    merge_partial(a, b2, my_invT > 0.0f);
-                }
-                p.part[(size_t)r * N + lane] = a;
+                RPartial a = sh.sel[0][lane].partial();
+                for (int w2 = 1; w2 < TV_EPI_WARPS; ++w2) merge_rpartial(a, sh.sel[w2][lane].partial(), my_invT > 0.0f);
+                if (my_invT > 0.0f) p.part[(size_t)r * N + lane] = a;
+                else atomicMax(p.best64 + 32 * (pass & 1) + lane, argmax_key(a.best, a.idx));   // greedy: one key
             }
             tv_epi_bar();
+            // partials of this range are written: the Trans CTAs end the pass
             if (ew == 0 && lane == 0) {
-                sh.last = atom_add_acq_rel_gpu(&c->read_done.v, 1u) == (unsigned)(S * (pass + 1) - 1);
+                red_add_release_gpu(&c->read_done.v, 1u);
+                if (p.trace && pass < 2) { const unsigned long long tn = globaltimer_ns(); trace_mark(p.trace, 205 + pass, tn); }
                 if (tr) trace_mark(p.trace, 8 + 4 * pass + 1, t_go);
-            }
-            tv_epi_bar();
-            if (sh.last) {
-                // end of the pass: combine the partials of every evaluated
-                // token, apply the stopping rule, pack the next pass
-                const unsigned long long t_last = globaltimer_ns();
-                for (int t = ew; t < n; t += TV_EPI_WARPS) {
-                    const int tok = sh.tok[t];
-                    const TokenResult res = reduce_token(p, t, tok, sh.invT[t], sh.seed[t]);
-                    if (lane == 0) {
-                        sh.ynew[t] = res.y;
-                        if (p.lse) p.lse[tok] = res.lse;
-                        if (p.logit_sel) p.logit_sel[tok] = res.sel;
-                        p.tokens[tok] = res.y;
-                    }
-                }
-                tv_epi_bar();
-                if (ew == 0) {
-                    const bool more = converge_pack_small(p, sh.seq, sh.ynew, sh.yold, sh.passes, 0);
-                    __syncwarp();
-                    if (lane == 0) {
-                        if (more) red_add_release_gpu(&c->pass_done.v, 1u);
-                        else raise_stop(c, 0);
-                        if (p.trace) trace_mark(p.trace, 8 + 4 * pass + 2, t_last);
-                    }
-                }
             }
         }
     }
@@ -533,7 +509,7 @@ __device__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUt
 
 // ------------------------------------------------------------- Trans role
 
-__device__ void trans_role(const Params &p, SmallCtl *c, uint8_t *base, unsigned long long t_start)
+__device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t *base, unsigned long long t_start)
 {
     TsShared &sh = *reinterpret_cast<TsShared *>(base);
     uint16_t *cop = reinterpret_cast<uint16_t *>(base + TS_HEAD);
@@ -580,6 +556,14 @@ __device__ void trans_role(const Params &p, SmallCtl *c, uint8_t *base, unsigned
             if (p.converged) p.converged[tid] = 0;
         }
         if (tid == 0) { p.ctl[CTL_NACT] = N; p.ctl[CTL_DONE] = 0; p.ctl[CTL_PASS] = 0; p.ctl[CTL_EVAL] = N; }
+        if (tid < 64) p.best64[tid] = 0ull;                    // both parities, before pass 0's z
+    }
+    if (tid < b) {
+        SeqState s{};
+        s.active = 1; s.m = -1; s.iters = 0; s.converged = 0; s.off = tid * B; s.cnt = B;
+        sh.st[tid] = s;
+        const float T = p.temperature[tid];
+        sh.invT[tid] = T > 0.0f ? 1.0f / T : 0.0f;
     }
     if (tid == 0) sh.go = wait_count(c, &c->pre_done.v, (unsigned)p.S);
     __syncthreads();
@@ -642,19 +626,10 @@ __device__ void trans_role(const Params &p, SmallCtl *c, uint8_t *base, unsigned
 
     float *zf = p.z_final ? p.z_final : p.zbuf;
     uint16_t *zpack = static_cast<uint16_t *>(p.zpack);
+    int n = N;                                                 // evaluated tokens of this pass
     for (int pass = 0;; ++pass) {
         const unsigned long long t_pass = globaltimer_ns();
         const int trs = (lead && tid == 0 && p.trace && pass < 3) ? 210 + 8 * pass : 0;
-        int n = N;
-        if (pass > 0) {
-            if (tid == 0) sh.go = wait_count(c, &c->pass_done.v, (unsigned)pass);
-            __syncthreads();
-            if (!sh.go) break;
-            n = min(__ldcg(p.ctl + CTL_NACT), MAX_B);
-            if (tid < n) sh.tok[tid] = __ldcg(p.act_tok + tid);
-            if (tid < N) sh.x[tid] = __ldcg(p.tokens + tid);
-            __syncthreads();
-        }
         if (trs) trace_mark(p.trace, trs, t_pass);
         // Fuse, token part: e_j = E'[x_{j-1}] (x_{-1} = anchor) for every position
         for (int i = tid; i < N * 32; i += nth) {
@@ -720,6 +695,9 @@ __device__ void trans_role(const Params &p, SmallCtl *c, uint8_t *base, unsigned
         }
         __syncthreads();
         if (!sh.go) break;
+        // every Trans CTA has read the previous pass's keys (before its u was
+        // published): clear them for the pass after this one (same parity)
+        if (lead && pass > 0 && tid < 32) p.best64[32 * ((pass - 1) & 1) + tid] = 0ull;
         for (int i = tid; i < 32 * (2 * RANK / 8); i += nth) {
             const int t = i / (2 * RANK / 8), cc = i % (2 * RANK / 8);
             uint4 v = make_uint4(0, 0, 0, 0);
@@ -760,6 +738,102 @@ __device__ void trans_role(const Params &p, SmallCtl *c, uint8_t *base, unsigned
         if (tid == 0) {
             red_add_release_gpu(&c->z_ready.v, 1u);
             if (lead && p.trace) trace_mark(p.trace, 8 + 4 * pass, t_pass);
+            sh.go = wait_count(c, &c->read_done.v, (unsigned)(p.S * (pass + 1)));
+        }
+        __syncthreads();
+        if (!sh.go) break;
+        const unsigned long long t_end = globaltimer_ns();
+        if (lead && tid == 0 && p.trace && pass < 2) trace_mark(p.trace, 240 + 4 * pass, t_end);
+        // ---- end of the pass, in every Trans CTA (identical results; the lead
+        // CTA publishes them): combine the Read partials of each evaluated
+        // token, apply Algorithm 1's stopping rule, pack the next pass
+        if (warp == 0) {
+            // greedy tokens: the Read CTAs left one argmax key per token
+            const int t = lane;
+            if (t < n && sh.invT[sh.tok[t] / B] <= 0.0f) {
+                const int tok = sh.tok[t];
+                float best;
+                int idx;
+                argmax_unkey(__ldcg(p.best64 + 32 * (pass & 1) + t), best, idx);
+                sh.ynew[t] = idx;
+                sh.yold[t] = sh.x[tok];
+                if (lead) {
+                    if (p.lse) p.lse[tok] = __int_as_float(0x7fc00000);
+                    if (p.logit_sel) p.logit_sel[tok] = best;
+                    p.tokens[tok] = idx;
+                }
+            }
+        }
+        // T > 0 tokens: warp w combines the partials of tokens w, w + 10, ...
+        for (int t = warp; t < n; t += nth / 32) {
+            const int tok = sh.tok[t];
+            const float invT = sh.invT[tok / B];               // warp-uniform
+            if (invT <= 0.0f) continue;
+            const TokenResult res = reduce_token(p, t, invT);
+            if (lane == 0) {
+                sh.ynew[t] = res.y;
+                sh.yold[t] = sh.x[tok];
+                if (lead) {
+                    if (p.lse) p.lse[tok] = res.lse;
+                    if (p.logit_sel) p.logit_sel[tok] = res.sel;
+                    p.tokens[tok] = res.y;
+                }
+            }
+        }
+        if (lead && lane == 0 && p.trace && pass < 2) trace_mark(p.trace, 240 + 4 * pass + 1, t_end);
+        __syncthreads();
+        if (lead && tid == 0 && p.trace && pass < 2) trace_mark(p.trace, 240 + 4 * pass + 2, t_end);
+        if (warp == 0) {
+            // lane q: block q (b <= 32)
+            SeqState ns{};
+            int cnt = 0;
+            if (lane < b) {
+                const SeqState st = sh.st[lane];
+                ns = st.active ? converge_state(p, st, sh.ynew, sh.yold, st.off - st.m - 1) : st;
+                if (st.active && lead) {
+                    if (p.iters) p.iters[lane] = ns.iters;
+                    if (p.converged) p.converged[lane] = ns.converged;
+                }
+                cnt = ns.active ? B - 1 - ns.m : 0;
+            }
+            int incl = cnt;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int v = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += v;
+            }
+            const int total = __shfl_sync(0xffffffffu, incl, 31);
+            if (lane < b) {
+                ns.off = incl - cnt;
+                ns.cnt = cnt;
+                sh.st[lane] = ns;
+                for (int q = 0; q < cnt; ++q) sh.tok2[ns.off + q] = lane * B + ns.m + 1 + q;
+            }
+            if (lane == 0) {
+                sh.n2 = total;
+                sh.more = total > 0 && pass + 1 < p.K_max;
+            }
+        } else {
+            for (int t = tid - 32; t < n; t += nth - 32) sh.x[sh.tok[t]] = sh.ynew[t];
+        }
+        __syncthreads();
+        if (lead && tid == 0 && p.trace && pass < 2) trace_mark(p.trace, 240 + 4 * pass + 3, t_end);
+        n = sh.n2;
+        const bool more = sh.more;
+        if (tid < n) sh.tok[tid] = sh.tok2[tid];
+        if (lead) {
+            if (tid < n) p.act_tok[tid] = sh.tok2[tid];
+            if (tid == 0) {
+                p.ctl[CTL_NACT] = n;
+                p.ctl[CTL_PASS] = pass + 1;
+                if (more) p.ctl[CTL_EVAL] += n;
+            }
+        }
+        __syncthreads();
+        if (lead && tid == 0 && p.trace) trace_mark(p.trace, 8 + 4 * pass + 2, t_end);
+        if (!more) {
+            if (lead && tid == 0) raise_stop(c, 0);            // after the lead's writes
+            break;
         }
     }
 }
@@ -768,7 +842,9 @@ __device__ void trans_role(const Params &p, SmallCtl *c, uint8_t *base, unsigned
 
 const size_t kRefineSmallSmemBytes = SMALL_SMEM;
 
-// grid S + 8 (cooperative), TV_THREADS threads, SMALL_SMEM dynamic shared memory.
+// grid S + 8 (cooperative), TV_THREADS threads, SMALL_SMEM dynamic shared memory,
+// one CTA per SM (10 warps: 3 on some of the 4 sub-partitions, hence <= 168
+// registers per thread).
 __global__ void __launch_bounds__(TV_THREADS, 1)
     k_refine_small(const __grid_constant__ Params p, const __grid_constant__ CUtensorMap tmap_wr128,
                    const __grid_constant__ CUtensorMap tmap_z)
@@ -779,7 +855,7 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
     SmallCtlArea *area = p.sctl;
     const int par = (int)(__ldcg(&area->parity.v) & 1u);
     SmallCtl *c = &area->blk[par];
-    if (blockIdx.x == 0 && threadIdx.x < 8) {
+    if (blockIdx.x == 0 && threadIdx.x < (int)(sizeof(SmallCtl) / sizeof(CtlLine))) {
         // the next call's block (this call's other one) starts from zero
         CtlLine *nxt = reinterpret_cast<CtlLine *>(&area->blk[par ^ 1]);
         nxt[threadIdx.x].v = 0;

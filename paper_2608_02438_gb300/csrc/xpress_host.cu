@@ -70,7 +70,7 @@ size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 struct Layout {
     size_t status = 0, ctl = 64, params = 256, st = 0, upart = 0, pc = 0, ynew = 0, acttok = 0, zpack = 0,
            zbuf = 0, part = 0, total = 0;
-    size_t sctl = 0, cx = 0, ux = 0, rmax = 0;
+    size_t sctl = 0, cx = 0, ux = 0, rmax = 0, best64 = 0;
     int ksplit = 1, kchunk = 0, S = 1;
     int pre_kslice = 0, pre_ks = 0;
     bool gemv = false;
@@ -181,7 +181,7 @@ Layout make_layout(const xpress_refiner *R, int b)
     o = align256(o + (size_t)N * RANK * 4);
     L.tcv = use_tcv(R, b);
     L.part = o;
-    o = align256(o + (size_t)L.S * N * sizeof(Partial));
+    o = align256(o + (size_t)L.S * N * sizeof(RPartial));
     if (L.small) {
         L.cx = o;
         o = align256(o + (size_t)32 * RANK * 2);
@@ -189,6 +189,8 @@ Layout make_layout(const xpress_refiner *R, int b)
         o = align256(o + (size_t)32 * 2 * RANK * 2);
         L.rmax = o;
         o = align256(o + (size_t)N * RMAX_SEG * sizeof(Partial));
+        L.best64 = o;
+        o = align256(o + 64 * sizeof(unsigned long long));
     }
     L.total = o;
     return L;
@@ -250,7 +252,7 @@ Params make_params(const xpress_refiner *R, const xpress_block_in *in, const xpr
     P.act_tok = reinterpret_cast<int32_t *>(w + L.acttok);
     P.zpack = w + L.zpack;
     P.zbuf = reinterpret_cast<float *>(w + L.zbuf);
-    P.part = reinterpret_cast<Partial *>(w + L.part);
+    P.part = reinterpret_cast<RPartial *>(w + L.part);
     if (L.small) {
         P.use_graph = 0;
         P.Fhg = R->Fhg;
@@ -260,6 +262,7 @@ Params make_params(const xpress_refiner *R, const xpress_block_in *in, const xpr
         P.ux = reinterpret_cast<uint16_t *>(w + L.ux);
         P.rmax = reinterpret_cast<Partial *>(w + L.rmax);
         P.sctl = reinterpret_cast<SmallCtlArea *>(w + L.sctl);
+        P.best64 = reinterpret_cast<unsigned long long *>(w + L.best64);
     }
     return P;
 }
@@ -580,7 +583,8 @@ void print_trace(xpress_refiner *R, cudaStream_t st)
     for (int i = 0; i < TRACE_SLOTS; ++i) {
         if (h[i] == ~0ull) continue;
         char name[32];
-        if (i >= 210) std::snprintf(name, sizeof(name), "mlp%dphase%d", (i - 210) / 8, (i - 210) % 8);
+        if (i >= 240 && i < 248) std::snprintf(name, sizeof(name), "end%dphase%d", (i - 240) / 4, (i - 240) % 4);
+        else if (i >= 210) std::snprintf(name, sizeof(name), "mlp%dphase%d", (i - 210) / 8, (i - 210) % 8);
         else if (i >= 200) std::snprintf(name, sizeof(name), "readphase%d", i - 200);
         else if (i < 8) std::snprintf(name, sizeof(name), "%s", i < 4 ? pre[i] : "?");
         else std::snprintf(name, sizeof(name), "%s%d", (i - 8) % 4 < 3 ? body[(i - 8) % 4] : "?", (i - 8) / 4);
