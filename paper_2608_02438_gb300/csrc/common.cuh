@@ -126,7 +126,7 @@ struct Params {
     int32_t *act_tok;            // [N] packed evaluated tokens (global token ids)
     void *zpack;                 // [N, r] W_r operand of the evaluated tokens
     float *zbuf;                 // [N, r] fp32 z when the caller passes no z_final
-    RPartial *part;              // [S, N]
+    RPartial *part;              // [N, S] token-major (a token's ranges are contiguous)
     // persistent small-batch kernel only
     const float *Fhg;            // [2r, H] fp32: rows W_in[:, 0:r] W_h, then W_in[:, r:2r] W_g
     int pre_kslice, pre_ks;      // K-slice width of the hidden projection and the number of slices
@@ -262,8 +262,43 @@ __device__ __forceinline__ RPartial rpartial_identity()
 // are ignored) into the state.  T <= 0: argmax.  T > 0: x = l * invT, the
 // group's log-sum-exp plus its Gumbel noise competes for the group draw, and
 // (m, s) accumulate the full log-sum-exp.
+// The member draw of the hierarchical Gumbel-max inside group [v0, v0 + 32):
+// argmax over the members j < valid of x_j + Gumbel(seed, v0 + j, pos,
+// STREAM_ELEM, offset), smallest id on ties; one Philox call per 4 ids.  x is
+// read as x[XS * j] (XS = 1: a register array; 32: a lane's column in shared
+// memory).
+template <int XS = 1>
+__device__ __forceinline__ void member_draw(const float *x, int valid, int v0, unsigned long long seed, uint32_t pos,
+                                            uint32_t offset, int &y, float &sel)
+{
+    float bsc = -INFINITY, bx = x[0];
+    int bj = 0;
+#pragma unroll
+    for (int c = 0; c < GROUP / 4; ++c) {
+        const uint4 o = philox10(make_uint4(((uint32_t)v0 >> 2) + c, pos, STREAM_ELEM, offset), (uint32_t)seed,
+                                 (uint32_t)(seed >> 32));
+        const uint32_t w4[4] = {o.x, o.y, o.z, o.w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int j = 4 * c + q;
+            if (j < valid) {
+                const float u = ((float)(w4[q] >> 9) + 0.5f) * (1.0f / 8388608.0f);
+                const float xj = x[XS * j];
+                const float sc = xj - logf(-logf(u));
+                if (sc > bsc) { bsc = sc; bj = j; bx = xj; }
+            }
+        }
+    }
+    y = v0 + bj;
+    sel = bx;
+}
+
+// xsave (T > 0 only): when given, the x of the best group so far are stored at
+// xsave[32 j] instead of drawing its member at once (the caller draws once,
+// for the group that ends up best).
 __device__ __forceinline__ void select_group(SelState &st, const float *l, int v0, int valid, float invT,
-                                             unsigned long long seed, uint32_t pos, uint32_t offset)
+                                             unsigned long long seed, uint32_t pos, uint32_t offset,
+                                             float *xsave = nullptr)
 {
     if (valid <= 0) return;
     if (invT <= 0.0f) {
@@ -295,29 +330,16 @@ __device__ __forceinline__ void select_group(SelState &st, const float *l, int v
     const uint32_t g = (uint32_t)v0 / GROUP;
     const float score = mx + __logf(sum) + gumbel(seed, g, pos, STREAM_GROUP, offset);
     if (score > st.best) {
-        // the group is this range's best so far: draw its member now (Gumbel-max
-        // over the members, smallest id on ties), one Philox call per 4 ids
         st.best = score;
         st.idx = (int)g;
-        float bsc = -INFINITY, bx = x[0];
-        int bj = 0;
+        if (xsave) {
+            // keep the group's x for one member draw at the end of the range
 #pragma unroll
-        for (int c = 0; c < GROUP / 4; ++c) {
-            const uint4 o = philox10(make_uint4(((uint32_t)v0 >> 2) + c, pos, STREAM_ELEM, offset), (uint32_t)seed,
-                                     (uint32_t)(seed >> 32));
-            const uint32_t w4[4] = {o.x, o.y, o.z, o.w};
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int j = 4 * c + q;
-                if (j < valid) {
-                    const float u = ((float)(w4[q] >> 9) + 0.5f) * (1.0f / 8388608.0f);
-                    const float sc = x[j] - logf(-logf(u));
-                    if (sc > bsc) { bsc = sc; bj = j; bx = x[j]; }
-                }
-            }
+            for (int j = 0; j < GROUP; ++j) xsave[32 * j] = x[j];
+        } else {
+            // draw the member now
+            member_draw(x, valid, v0, seed, pos, offset, st.y, st.sel);
         }
-        st.y = v0 + bj;
-        st.sel = bx;
     }
     merge_lse(st.m, st.s, mx, sum);
 }

@@ -315,12 +315,12 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     if (ew == 0 && lane < n) {
                         RPartial a = sh.st[0][lane].partial();
                         for (int w = 1; w < TC_EPI_WARPS; ++w) merge_rpartial(a, sh.st[w][lane].partial(), invT > 0.0f);
-                        p.part[(size_t)r * p.N + lane] = a;
+                        p.part[(size_t)lane * p.S + r] = a;
                     }
                 } else if (ew < 4 && valid) {
                     RPartial a = sh.st[ew][lane].partial();
                     merge_rpartial(a, sh.st[ew + 4][lane].partial(), invT > 0.0f);
-                    p.part[(size_t)r * p.N + i] = a;
+                    p.part[(size_t)i * p.S + r] = a;
                 }
             }
             epi_bar();

@@ -257,7 +257,7 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
         if (!stop && ew == 0 && lane < n) {
             RPartial a = sh.st[0][lane].partial();
             for (int w = 1; w < TV_EPI_WARPS; ++w) merge_rpartial(a, sh.st[w][lane].partial(), my_invT > 0.0f);
-            p.part[(size_t)r * p.N + lane] = a;
+            p.part[(size_t)lane * p.S + r] = a;
         }
     }
     if (tr0 && threadIdx.x == 64) trace_mark(p.trace, 203, t_wait);

@@ -76,7 +76,7 @@ __device__ __forceinline__ TokenResult reduce_token(const Params &p, int i, floa
 #pragma unroll
         for (int j = 0; j < PER; ++j) {
             const int r = r0 + lane + 32 * j;
-            pv[j] = r < p.S ? ldcg_rpartial(p.part + (size_t)r * p.N + i) : rpartial_identity();
+            pv[j] = r < p.S ? ldcg_rpartial(p.part + (size_t)i * p.S + r) : rpartial_identity();
         }
 #pragma unroll
         for (int j = 0; j < PER; ++j) merge_rpartial(a, pv[j], sampling);

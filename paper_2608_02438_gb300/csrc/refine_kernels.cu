@@ -692,7 +692,7 @@ __global__ void __launch_bounds__(256) k_read_simt(const Params *__restrict__ pp
             const bool sampling = invT > 0.0f;
             RPartial a = sst[0][lane].partial();
             for (int w = 1; w < 8; ++w) merge_rpartial(a, sst[w][lane].partial(), sampling);
-            p.part[(size_t)blockIdx.x * p.N + t0 + lane] = a;
+            p.part[(size_t)(t0 + lane) * p.S + blockIdx.x] = a;
         }
         __syncthreads();
     }

@@ -56,6 +56,7 @@ struct RsShared {                              // Read CTA, after the W_r stages
     unsigned long long seed[TV_BN];
     SelState sel[TV_EPI_WARPS][32];
     float tile[TV_EPI_WARPS][TV_BN][33];       // per-warp transpose: [token][vocabulary row]
+    float bestx[TV_EPI_WARPS][GROUP][32];      // T > 0: x of each (warp, token)'s best group, [j][token]
 };
 
 struct TsShared {                              // Trans CTA
@@ -474,7 +475,7 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
                         for (int jj = 0; jj < GROUP; ++jj)
                             if (jj < nv) dst[jj] = l[jj];
                     }
-                    select_group(sel, l, v0, nv, my_invT, my_seed, (uint32_t)my_pos, p.offset);
+                    select_group(sel, l, v0, nv, my_invT, my_seed, (uint32_t)my_pos, p.offset, &sh.bestx[ew][0][lane]);
                 }
                 __syncwarp();
 #pragma unroll
@@ -485,8 +486,19 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
             if (tv_epi_bar_or(!ok || *abort)) break;
             if (ew == 0 && lane < n) {
                 RPartial a = sh.sel[0][lane].partial();
-                for (int w2 = 1; w2 < TV_EPI_WARPS; ++w2) merge_rpartial(a, sh.sel[w2][lane].partial(), my_invT > 0.0f);
-                if (my_invT > 0.0f) p.part[(size_t)r * N + lane] = a;
+                int wbest = 0;
+                for (int w2 = 1; w2 < TV_EPI_WARPS; ++w2) {
+                    const RPartial b2 = sh.sel[w2][lane].partial();
+                    if (b2.best > a.best || (b2.best == a.best && b2.idx < a.idx)) wbest = w2;
+                    merge_rpartial(a, b2, my_invT > 0.0f);
+                }
+                if (my_invT > 0.0f && a.idx != 0x7fffffff) {
+                    // the member draw of this range's best group, once
+                    const int v0 = a.idx * GROUP;
+                    member_draw<32>(&sh.bestx[wbest][0][lane], min(GROUP, V - v0), v0, my_seed, (uint32_t)my_pos,
+                                    p.offset, a.y, a.sel);
+                }
+                if (my_invT > 0.0f) p.part[(size_t)lane * S + r] = a;
                 else atomicMax(p.best64 + 32 * (pass & 1) + lane, argmax_key(a.best, a.idx));   // greedy: one key
             }
             tv_epi_bar();
