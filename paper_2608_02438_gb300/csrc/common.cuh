@@ -294,8 +294,9 @@ __device__ __forceinline__ void member_draw(const float *x, int valid, int v0, u
 }
 
 // xsave (T > 0 only): when given, the x of the best group so far are stored at
-// xsave[32 j] instead of drawing its member at once (the caller draws once,
-// for the group that ends up best).
+// xsave[32 j], so that the caller can draw the member of the group that ends
+// up best once (member_draw).  Without it the partial carries no member and
+// the end of the pass draws it (draw_in_group).
 __device__ __forceinline__ void select_group(SelState &st, const float *l, int v0, int valid, float invT,
                                              unsigned long long seed, uint32_t pos, uint32_t offset,
                                              float *xsave = nullptr)
@@ -336,9 +337,6 @@ __device__ __forceinline__ void select_group(SelState &st, const float *l, int v
             // keep the group's x for one member draw at the end of the range
 #pragma unroll
             for (int j = 0; j < GROUP; ++j) xsave[32 * j] = x[j];
-        } else {
-            // draw the member now
-            member_draw(x, valid, v0, seed, pos, offset, st.y, st.sel);
         }
     }
     merge_lse(st.m, st.s, mx, sum);

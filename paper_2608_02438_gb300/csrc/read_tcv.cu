@@ -285,7 +285,7 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
             if (tr0 && threadIdx.x == 0) trace_mark(p.trace, 204, t_wait);
             for (int t = warp; t < n; t += TV_THREADS / 32) {
                 const int tok = sh.tok[t];
-                const TokenResult res = reduce_token(p, t, sh.invT[t]);
+                const TokenResult res = reduce_token(p, t, tok, sh.invT[t], sh.seed[t]);
                 if (lane == 0) {
                     sh.ynew[t] = res.y;
                     if (p.lse) p.lse[tok] = res.lse;

@@ -8,9 +8,20 @@
 
 namespace xp {
 
+__device__ __forceinline__ void bf16x8_to_float(const uint4 &w, float (&x)[8])
+{
+    const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        x[2 * q] = __uint_as_float(ww[q] << 16);
+        x[2 * q + 1] = __uint_as_float(ww[q] & 0xFFFF0000u);
+    }
+}
+
 struct TokenResult {
     int y;
     float sel, lse;
+    int grp;                     // T > 0: the drawn group
 };
 
 // Warp-collective: the re-selected token of packed token i (global token id
@@ -59,11 +70,57 @@ __device__ __forceinline__ TokenResult finish_token(RPartial a, bool sampling)
         res.sel = a.sel;
         res.lse = a.m + logf(a.s);
     }
+    res.grp = a.idx;
     return res;
 }
 
-// Combines the S Read partials of evaluated token i.  Warp-collective.
-__device__ __forceinline__ TokenResult reduce_token(const Params &p, int i, float invT)
+// T > 0 member draw of a token whose Read partials carry none (the graph
+// path's epilogues leave it out): recompute the 32 logits of the drawn group
+// g, l_v = s_v + W_r[v] . z_i, and take the Gumbel-max over its members.
+// Warp-collective (lane = member).
+__device__ __forceinline__ void draw_in_group(const Params &p, int i, int tok, int g, float invT,
+                                              unsigned long long seed, TokenResult &res)
+{
+    const int lane = threadIdx.x % 32, k = tok % p.B;
+    const int v = g * GROUP + lane;
+    float x = -INFINITY, score = -INFINITY;
+    if (v < p.V) {
+        float acc = 0.0f;
+        if (p.dtype) {
+            const uint4 *wr = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.W_r) + (size_t)v * RANK);
+            const uint4 *zr = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.zpack) + (size_t)i * RANK);
+#pragma unroll 8
+            for (int c = 0; c < RANK / 8; ++c) {
+                float w8[8], z8[8];
+                bf16x8_to_float(__ldg(wr + c), w8);
+                bf16x8_to_float(__ldcg(zr + c), z8);
+#pragma unroll
+                for (int j = 0; j < 8; ++j) acc = fmaf(w8[j], z8[j], acc);
+            }
+        } else {
+            for (int d = 0; d < RANK; ++d)
+                acc = fmaf(ld_any(p.W_r, 0, (size_t)v * RANK + d), ld_any(p.zpack, 0, (size_t)i * RANK + d), acc);
+        }
+        x = (acc + ld_any(p.s, p.dtype, (size_t)tok * p.V + v)) * invT;
+        score = x + gumbel(seed, (uint32_t)v, (uint32_t)k, STREAM_ELEM, p.offset);
+    }
+    float bs = score;
+    int bi = v;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float os = __shfl_xor_sync(0xffffffffu, bs, o);
+        const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+        merge_argmax(bs, bi, os, oi);
+    }
+    res.y = bi;
+    res.sel = __shfl_sync(0xffffffffu, x, (bi - g * GROUP) & (GROUP - 1));
+}
+
+// Combines the S Read partials of evaluated token i (global id tok).  For
+// T > 0 the member of the drawn group comes with the partials when the Read
+// drew it, else it is drawn here.  Warp-collective.
+__device__ __forceinline__ TokenResult reduce_token(const Params &p, int i, int tok, float invT,
+                                                    unsigned long long seed)
 {
     const int lane = threadIdx.x % 32;
     const bool sampling = invT > 0.0f;
@@ -81,7 +138,9 @@ __device__ __forceinline__ TokenResult reduce_token(const Params &p, int i, floa
 #pragma unroll
         for (int j = 0; j < PER; ++j) merge_rpartial(a, pv[j], sampling);
     }
-    return finish_token(a, sampling);
+    TokenResult res = finish_token(a, sampling);
+    if (sampling && res.y == 0x7fffffff) draw_in_group(p, i, tok, res.grp, invT, seed, res);
+    return res;
 }
 
 // Algorithm 1's stopping rule for block s after a pass that evaluated

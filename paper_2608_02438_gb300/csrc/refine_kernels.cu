@@ -718,7 +718,7 @@ __global__ void __launch_bounds__(1024) k_reduce(const Params *__restrict__ pp, 
         const int k = warp, i = st.off + (k - st.m - 1), tok = s * B + k;
         if (lane == 0) yold[k] = p.tokens[tok];
         const float T = p.temperature[s];
-        const TokenResult res = reduce_token(p, i, T > 0.0f ? 1.0f / T : 0.0f);
+        const TokenResult res = reduce_token(p, i, tok, T > 0.0f ? 1.0f / T : 0.0f, p.seed[s]);
         if (lane == 0) {
             ynew[k] = res.y;
             if (p.lse) p.lse[tok] = res.lse;

@@ -781,7 +781,7 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
             const int tok = sh.tok[t];
             const float invT = sh.invT[tok / B];               // warp-uniform
             if (invT <= 0.0f) continue;
-            const TokenResult res = reduce_token(p, t, invT);
+            const TokenResult res = reduce_token(p, t, tok, invT, p.seed[tok / B]);
             if (lane == 0) {
                 sh.ynew[t] = res.y;
                 sh.yold[t] = sh.x[tok];
