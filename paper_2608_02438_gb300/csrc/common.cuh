@@ -81,6 +81,7 @@ struct alignas(128) CtlLine {
 };
 struct SmallCtl {
     CtlLine pre_done;    // Read CTAs done with the precompute
+    CtlLine pc_ready;    // Trans CTAs that published their slice of Pc (8 per call)
     CtlLine c_ready;     // Trans CTAs that published their slice of c (8 per pass)
     CtlLine u_ready;     // ... of sigma(W_1 c)
     CtlLine z_ready;     // ... of z
@@ -131,6 +132,8 @@ struct Params {
     const float *Fhg;            // [2r, H] fp32: rows W_in[:, 0:r] W_h, then W_in[:, r:2r] W_g
     int pre_kslice, pre_ks;      // K-slice width of the hidden projection and the number of slices
     uint16_t *cx, *ux;           // [32, r] c and [32, 2r] sigma(W_1 c), bf16, exchanged by the Trans CTAs
+    float *pcx;                  // [32, r] Pc, fp32, exchanged once per call (blocks of at most 16)
+    const uint16_t *Lpk;         // [B(B-1)/2, r] bf16: L's strictly lower part, row q = k(k-1)/2 + j
     Partial *rmax;               // [N, RMAX_SEG] argmax-s partials (calls without a draft)
     SmallCtlArea *sctl;          // control blocks of the persistent kernel
     unsigned long long *best64;  // [2][32] per pass parity: max over ranges of argmax_key (greedy tokens)

@@ -59,15 +59,21 @@ struct RsShared {                              // Read CTA, after the W_r stages
     float bestx[TV_EPI_WARPS][GROUP][32];      // T > 0: x of each (warp, token)'s best group, [j][token]
 };
 
-struct TsShared {                              // Trans CTA
-    float e[MAX_B][32];                        // E' rows of all b*B positions, own channels
-    float pc[MAX_B][32];                       // Pc of all b*B positions, own channels
+// Trans CTA.  With blocks of at most 16 positions every Trans CTA keeps all
+// r channels of E' rows, Pc and L (so it forms c itself: no exchange of c);
+// with larger blocks only its own 32 channels (c is exchanged).  Dynamic
+// shared memory after the head: cop [32][COP_LD] and uop [32][UOP_LD] bf16,
+// e [32][CH] and pc [32][CH] fp32, Lp [B(B-1)/2][CH] bf16 (L's strictly
+// lower part, channel innermost).
+constexpr int FULL_C_MAX_B = 16;
+struct TsShared {
     float cown[MAX_B][32];                     // c of the evaluated tokens, own channels (fp32)
     float zhalf[2][MAX_B][32];                 // W_2 u, the two K halves
     int tok[MAX_B];                            // evaluated tokens of the pass (global ids)
     int x[MAX_B];                              // current tokens Y
     int ynew[MAX_B], yold[MAX_B];              // per evaluated token: new / previous token
     int tok2[MAX_B];                           // evaluated tokens of the next pass
+    int tpos[MAX_B], tseq[MAX_B];              // per global token id: position k, block s
     SeqState st[MAX_B];                        // per block: Algorithm 1 state
     float invT[MAX_B];                         // per block: 1 / T (0 for greedy)
     int n, n2, go, more;
@@ -75,7 +81,10 @@ struct TsShared {                              // Trans CTA
 
 constexpr size_t RS_BYTES = 1024 + TV_STAGES * TV_A_STAGE + TV_Z_BYTES + sizeof(RsShared);
 constexpr size_t TS_HEAD = (sizeof(TsShared) + 127) / 128 * 128;
-constexpr size_t TS_BYTES = 1024 + TS_HEAD + 32 * COP_LD * 2 + 32 * UOP_LD * 2 + 32 * MAX_B * MAX_B * 2;
+constexpr size_t TS_TAIL_FULL = 2 * 32 * RANK * 4 + RANK * (FULL_C_MAX_B * (FULL_C_MAX_B - 1) / 2) * 2;
+constexpr size_t TS_TAIL_OWN = 2 * 32 * 32 * 4 + 32 * (MAX_B * (MAX_B - 1) / 2) * 2;
+constexpr size_t TS_BYTES = 1024 + TS_HEAD + 32 * COP_LD * 2 + 32 * UOP_LD * 2 +
+                            (TS_TAIL_FULL > TS_TAIL_OWN ? TS_TAIL_FULL : TS_TAIL_OWN);
 constexpr size_t SMALL_SMEM = RS_BYTES > TS_BYTES ? RS_BYTES : TS_BYTES;
 
 // ------------------------------------------------------------- signalling
@@ -524,23 +533,29 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
 __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t *base, unsigned long long t_start)
 {
     TsShared &sh = *reinterpret_cast<TsShared *>(base);
-    uint16_t *cop = reinterpret_cast<uint16_t *>(base + TS_HEAD);
-    uint16_t *uop = cop + 32 * COP_LD;
-    uint16_t *Ls = uop + 32 * UOP_LD;
     const int rank = blockIdx.x - p.S, d0 = rank * 32;
     const int N = p.N, B = p.B, b = p.b, V = p.V;
+    const bool full = B <= FULL_C_MAX_B;                   // this CTA forms all of c
+    const int CH = full ? RANK : 32, cb = full ? 0 : d0;   // channels kept, first one
+    const int TRI = B * (B - 1) / 2;
+    uint16_t *cop = reinterpret_cast<uint16_t *>(base + TS_HEAD);
+    uint16_t *uop = cop + 32 * COP_LD;
+    float *e = reinterpret_cast<float *>(uop + 32 * UOP_LD);   // [32][CH]
+    float *pc = e + 32 * CH;                                   // [32][CH]
+    uint16_t *Lp = reinterpret_cast<uint16_t *>(pc + 32 * CH);  // [TRI][CH]
     const int tid = threadIdx.x, nth = blockDim.x, warp = tid / 32, lane = tid % 32;
     const int g = lane >> 2, tq = lane & 3, khalf = (warp >> 2) & 1;
     const bool lead = rank == 0;
 
-    // static operands: W_1 / W_2 fragments (warps 0-7) and the CTA's slice of L
+    // static operands: W_1 / W_2 fragments (warps 0-7) and L's strictly lower
+    // part for the kept channels
     MlpFrags fr;
     if (warp < 8) load_mlp_frags(p, rank, fr);
-    {
-        const int n16 = 32 * B * B * 2 / 16;
-        const uint4 *src = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.L) + (size_t)d0 * B * B);
-        for (int i = tid; i < n16; i += nth) reinterpret_cast<uint4 *>(Ls)[i] = __ldg(src + i);
+    for (int i = tid; i < TRI * CH / 8; i += nth) {            // 16-byte pieces of the kept channels
+        const int q = i / (CH / 8), c8 = i % (CH / 8);
+        reinterpret_cast<uint4 *>(Lp)[i] = __ldg(reinterpret_cast<const uint4 *>(p.Lpk + (size_t)q * RANK + cb) + c8);
     }
+    if (tid < N) { sh.tpos[tid] = tid % B; sh.tseq[tid] = tid / B; }
     // Y^(0) from the draft; the lead CTA writes the state of the first pass
     if (tid < N) {
         int y = 0;
@@ -601,8 +616,9 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
     }
     // Pc = (I + L) P for the own channels (Eq. mix); P_k = F_h h_k + mean_j F_g h_j
     {
-        float(*P)[32] = sh.e;                                  // scratch until the first gather
-        float(*G)[32] = sh.cown;
+        float(*P)[32] = sh.cown;                               // scratch until the first pass
+        float(*G)[32] = sh.zhalf[0];
+        float(*Q)[32] = sh.zhalf[1];
         const int ks = p.pre_ks;
         for (int i = tid; i < N * 32; i += nth) {
             const int t = i / 32, dd = i % 32;
@@ -621,18 +637,31 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
             const int t = i / 32, dd = i % 32, s = t / B;
             float gs = 0.0f;
             for (int k = 0; k < B; ++k) gs += G[s * B + k][dd];
-            sh.pc[t][dd] = P[t][dd] + gs / (float)B;           // P, complete
+            Q[t][dd] = P[t][dd] + gs / (float)B;               // P, complete
         }
         __syncthreads();
+        const int lb = full ? d0 : 0;                          // own channels within the kept ones
         for (int i = tid; i < N * 32; i += nth) {
             const int t = i / 32, dd = i % 32, s = t / B, k = t % B;
-            float a = sh.pc[t][dd];
-            for (int j = 0; j < k; ++j) a = fmaf(bf2f(Ls[(dd * B + k) * B + j]), sh.pc[s * B + j][dd], a);
-            P[t][dd] = a;
+            float a = Q[t][dd];
+            for (int j2 = 0; j2 < k; ++j2)
+                a = fmaf(bf2f(Lp[(k * (k - 1) / 2 + j2) * CH + lb + dd]), Q[s * B + j2][dd], a);
+            if (full) p.pcx[(size_t)t * RANK + d0 + dd] = a;
+            else pc[t * CH + dd] = a;
         }
         __syncthreads();
-        for (int i = tid; i < N * 32; i += nth) sh.pc[i / 32][i % 32] = P[i / 32][i % 32];
-        __syncthreads();
+        if (full) {
+            // every Trans CTA needs Pc for all channels: one exchange per call
+            if (tid == 0) {
+                red_add_release_gpu(&c->pc_ready.v, 1u);
+                sh.go = wait_count(c, &c->pc_ready.v, 8u);
+            }
+            __syncthreads();
+            if (!sh.go) return;
+            for (int i = tid; i < N * RANK / 4; i += nth)
+                reinterpret_cast<float4 *>(pc)[i] = __ldcg(reinterpret_cast<const float4 *>(p.pcx) + i);
+            __syncthreads();
+        }
     }
     if (lead && tid == 0 && p.trace) trace_mark(p.trace, 3, t_start);
 
@@ -643,38 +672,79 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
         const unsigned long long t_pass = globaltimer_ns();
         const int trs = (lead && tid == 0 && p.trace && pass < 3) ? 210 + 8 * pass : 0;
         if (trs) trace_mark(p.trace, trs, t_pass);
-        // Fuse, token part: e_j = E'[x_{j-1}] (x_{-1} = anchor) for every position
-        for (int i = tid; i < N * 32; i += nth) {
-            const int j = i / 32, dd = i % 32, k = j % B, s = j / B;
+        // Fuse, token part: e_j = E'[x_{j-1}] (x_{-1} = anchor) for every
+        // position, kept channels (16-byte pieces)
+        for (int i = tid; i < N * CH / 4; i += nth) {
+            const int j = i / (CH / 4), q = i % (CH / 4), k = j % B, s = j / B;
             int x = k == 0 ? p.anchor[s] : sh.x[j - 1];
             if (x < 0 || x >= V) x = 0;                        // reported at the start
-            sh.e[j][dd] = __ldg(p.Ep + (size_t)x * RANK + d0 + dd);
+            reinterpret_cast<float4 *>(e)[i] = __ldg(reinterpret_cast<const float4 *>(p.Ep + (size_t)x * RANK + cb) + q);
         }
         __syncthreads();
         if (trs) trace_mark(p.trace, trs + 1, t_pass);
-        // Mix for the evaluated tokens; c leaves rounded to bf16 (the W_1 operand)
-        for (int i = tid; i < n * 32; i += nth) {
-            const int t = i / 32, dd = i % 32, tok = sh.tok[t], s = tok / B, k = tok % B;
-            float a = sh.pc[tok][dd] + sh.e[tok][dd];
-            for (int j = 0; j < k; ++j) a = fmaf(bf2f(Ls[(dd * B + k) * B + j]), sh.e[s * B + j][dd], a);
-            sh.cown[t][dd] = a;
-            p.cx[(size_t)t * RANK + d0 + dd] = f2bf(a);
+        // Mix for the evaluated tokens; c enters W_1 rounded to bf16.
+        if (full) {
+            // thread = channel; a block's E' values sit in registers and both
+            // loops are unrolled (B <= 16), predicated on the block's frontier
+            const int dd = tid;
+            if (dd < RANK)
+                for (int s = 0; s < b; ++s) {
+                    const SeqState st = sh.st[s];
+                    if (!st.active) continue;
+                    float er[FULL_C_MAX_B];
+#pragma unroll
+                    for (int j2 = 0; j2 < FULL_C_MAX_B; ++j2) er[j2] = j2 < B ? e[(s * B + j2) * CH + dd] : 0.0f;
+#pragma unroll
+                    for (int k = 0; k < FULL_C_MAX_B; ++k) {
+                        if (k < B && k > st.m) {
+                            float a = pc[(s * B + k) * CH + dd] + er[k];
+#pragma unroll
+                            for (int j2 = 0; j2 < k; ++j2)
+                                a = fmaf(bf2f(Lp[(k * (k - 1) / 2 + j2) * CH + dd]), er[j2], a);
+                            const int t = st.off + k - st.m - 1;
+                            cop[t * COP_LD + dd] = f2bf(a);
+                            if ((dd >> 5) == rank) sh.cown[t][dd & 31] = a;
+                        }
+                    }
+                }
+        } else {
+            // thread (channel dd of the own 32, token phase t0)
+            const int tstep = nth / CH;                        // 10 token phases
+            const int dd = tid % CH, t0 = tid / CH;
+            if (t0 < tstep)
+                for (int t = t0; t < n; t += tstep) {
+                    const int tok = sh.tok[t], s = sh.tseq[tok], k = sh.tpos[tok];
+                    float a = pc[tok * CH + dd] + e[tok * CH + dd];
+                    const uint16_t *lrow = Lp + (k * (k - 1) / 2) * CH + dd;
+                    const float *erow = e + (s * B) * CH + dd;
+                    for (int j2 = 0; j2 < k; ++j2) a = fmaf(bf2f(lrow[j2 * CH]), erow[j2 * CH], a);
+                    sh.cown[t][dd] = a;
+                    p.cx[(size_t)t * RANK + d0 + dd] = f2bf(a);
+                }
         }
-        __syncthreads();
-        if (tid == 0) {
-            red_add_release_gpu(&c->c_ready.v, 1u);
-            sh.go = wait_count(c, &c->c_ready.v, (unsigned)(8 * (pass + 1)));
+        if (full) {
+            // rows past n of the last 16-row tile: zero operands
+            for (int i = tid; i < ((n + 15) / 16 * 16 - n) * RANK; i += nth)
+                cop[(n + i / RANK) * COP_LD + i % RANK] = 0;
+            __syncthreads();
             if (trs) trace_mark(p.trace, trs + 2, t_pass);
+        } else {
+            __syncthreads();
+            if (tid == 0) {
+                red_add_release_gpu(&c->c_ready.v, 1u);
+                sh.go = wait_count(c, &c->c_ready.v, (unsigned)(8 * (pass + 1)));
+                if (trs) trace_mark(p.trace, trs + 2, t_pass);
+            }
+            __syncthreads();
+            if (!sh.go) break;
+            for (int i = tid; i < 32 * (RANK / 8); i += nth) {
+                const int t = i / (RANK / 8), cc = i % (RANK / 8);
+                uint4 v = make_uint4(0, 0, 0, 0);
+                if (t < n) v = __ldcg(reinterpret_cast<const uint4 *>(p.cx + (size_t)t * RANK) + cc);
+                *reinterpret_cast<uint4 *>(cop + t * COP_LD + 8 * cc) = v;
+            }
+            __syncthreads();
         }
-        __syncthreads();
-        if (!sh.go) break;
-        for (int i = tid; i < 32 * (RANK / 8); i += nth) {
-            const int t = i / (RANK / 8), cc = i % (RANK / 8);
-            uint4 v = make_uint4(0, 0, 0, 0);
-            if (t < n) v = __ldcg(reinterpret_cast<const uint4 *>(p.cx + (size_t)t * RANK) + cc);
-            *reinterpret_cast<uint4 *>(cop + t * COP_LD + 8 * cc) = v;
-        }
-        __syncthreads();
         // u = sigma(W_1 c), rows [64 rank, +64): warp w -> 8 rows
         if (warp < 8) {
             for (int mt = 0; mt * 16 < n; ++mt) {
@@ -902,6 +972,20 @@ __global__ void __launch_bounds__(256) k_fold_hidden(const uint16_t *W_h, const 
     }
 #pragma unroll
     for (int rr = 0; rr < 8; ++rr) Fhg[(size_t)(o0 + rr) * H + i] = acc[rr];
+}
+
+// Packs L's strictly lower part channel-innermost: Lpk[k(k-1)/2 + j][d] =
+// L[d][k][j] (j < k), so that a warp reading one (k, j) for 32 consecutive
+// channels reads 64 contiguous bytes.  grid (ceil(B(B-1)/2 / 8)), 256 threads.
+__global__ void __launch_bounds__(256) k_pack_L(const uint16_t *L, uint16_t *Lpk, int B)
+{
+    const int TRI = B * (B - 1) / 2, d = threadIdx.x;
+    for (int q = blockIdx.x * 8; q < min(TRI, blockIdx.x * 8 + 8); ++q) {
+        int k = 1;
+        while ((k + 1) * k / 2 <= q) ++k;
+        const int j = q - k * (k - 1) / 2;
+        Lpk[(size_t)q * RANK + d] = L[((size_t)d * B + k) * B + j];
+    }
 }
 
 }  // namespace xp

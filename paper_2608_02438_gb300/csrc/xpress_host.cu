@@ -70,7 +70,7 @@ size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 struct Layout {
     size_t status = 0, ctl = 64, params = 256, st = 0, upart = 0, pc = 0, ynew = 0, acttok = 0, zpack = 0,
            zbuf = 0, part = 0, total = 0;
-    size_t sctl = 0, cx = 0, ux = 0, rmax = 0, best64 = 0;
+    size_t sctl = 0, cx = 0, ux = 0, pcx = 0, rmax = 0, best64 = 0;
     int ksplit = 1, kchunk = 0, S = 1;
     int pre_kslice = 0, pre_ks = 0;
     bool gemv = false;
@@ -91,6 +91,7 @@ struct xpress_refiner {
     bool use_tc = false;
     cudaStream_t cs = nullptr;
     float *Fhg = nullptr;                  // [2r, H] folded hidden projection (small-batch kernel)
+    uint16_t *Lpk = nullptr;               // [B(B-1)/2, r] L's strictly lower part, channel innermost
     bool small_ok = false;                 // the small-batch kernel can run co-resident on this GPU
     void *small_ws[CACHE_SLOTS] = {};      // workspaces whose control area this refiner has cleared
     int small_ws_next = 0;
@@ -187,6 +188,8 @@ Layout make_layout(const xpress_refiner *R, int b)
         o = align256(o + (size_t)32 * RANK * 2);
         L.ux = o;
         o = align256(o + (size_t)32 * 2 * RANK * 2);
+        L.pcx = o;
+        o = align256(o + (size_t)32 * RANK * 4);
         L.rmax = o;
         o = align256(o + (size_t)N * RMAX_SEG * sizeof(Partial));
         L.best64 = o;
@@ -260,6 +263,8 @@ Params make_params(const xpress_refiner *R, const xpress_block_in *in, const xpr
         P.pre_ks = L.pre_ks;
         P.cx = reinterpret_cast<uint16_t *>(w + L.cx);
         P.ux = reinterpret_cast<uint16_t *>(w + L.ux);
+        P.pcx = reinterpret_cast<float *>(w + L.pcx);
+        P.Lpk = R->Lpk;
         P.rmax = reinterpret_cast<Partial *>(w + L.rmax);
         P.sctl = reinterpret_cast<SmallCtlArea *>(w + L.sctl);
         P.best64 = reinterpret_cast<unsigned long long *>(w + L.best64);
@@ -675,6 +680,13 @@ int xpress_refiner_create(const xpress_weights *w, void *stream, xpress_refiner 
                 k_fold_hidden<<<dim3((w->H + 255) / 256, 2 * RANK / 8), 256, 0, st>>>(
                     static_cast<const uint16_t *>(w->W_h), static_cast<const uint16_t *>(w->W_g),
                     static_cast<const uint16_t *>(w->W_in), R->Fhg, w->H);
+                const int tri = w->B * (w->B - 1) / 2;
+                if (cudaMalloc(&R->Lpk, (size_t)(tri > 0 ? tri : 1) * RANK * 2) != cudaSuccess) {
+                    rc = XPRESS_ERR_CUDA;
+                    break;
+                }
+                if (tri > 0)
+                    k_pack_L<<<(tri + 7) / 8, 256, 0, st>>>(static_cast<const uint16_t *>(w->L), R->Lpk, w->B);
                 R->small_ok = true;
             }
         }
@@ -695,6 +707,7 @@ int xpress_refiner_destroy(xpress_refiner *R)
     for (auto &e : R->cache) destroy_entry(e);
     if (R->Ep) cudaFree(R->Ep);
     if (R->Fhg) cudaFree(R->Fhg);
+    if (R->Lpk) cudaFree(R->Lpk);
     if (R->cs) cudaStreamDestroy(R->cs);
     if (R->trace) cudaFree(R->trace);
     delete R;

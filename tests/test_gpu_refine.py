@@ -77,7 +77,11 @@ def test_tiny_fp32_strong_coupling(X, temps):
     assert max(o["iters"] for o in orc.values()) >= 3      # multi-pass trajectories were exercised
 
 
-@pytest.mark.parametrize("b,B,temps", [(1, 16, (0.0,)), (3, 8, (1.0,)), (5, 8, (0.0, 1.0)), (20, 8, (1.0, 0.0)),
+# b * B <= 32 runs the persistent kernel: blocks of at most 16 form c in every
+# Trans CTA ((1, 16), (3, 8), (2, 16)), larger blocks exchange it ((1, 32),
+# (1, 24)); the others run the multi-kernel graph.
+@pytest.mark.parametrize("b,B,temps", [(1, 16, (0.0,)), (3, 8, (1.0,)), (2, 16, (0.0, 1.0)), (1, 32, (0.0,)),
+                                       (1, 24, (1.0,)), (5, 8, (0.0, 1.0)), (20, 8, (1.0, 0.0)),
                                        (9, 32, (0.0, 0.8))])
 def test_bf16_tensor_core_path(X, b, B, temps):
     cfg = W.tiny_config("bf16s", b=b, B=B, H=128, V=2080, r=256, dtype=W.BF16, temps=temps, seed=1000 + b)
