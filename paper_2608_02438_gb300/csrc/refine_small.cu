@@ -530,6 +530,19 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
 
 // ------------------------------------------------------------- Trans role
 
+// Fuse, token part: e_j = E'[x_{j-1}] (x_{-1} = the anchor) for every position
+// j of every block, channels [cb, cb + CH) (16-byte pieces).
+__device__ __forceinline__ void gather_e(const Params &p, const int *x, float *e, int CH, int cb, int tid, int nth)
+{
+    const int N = p.N, B = p.B, V = p.V;
+    for (int i = tid; i < N * CH / 4; i += nth) {
+        const int j = i / (CH / 4), q = i % (CH / 4), k = j % B, s = j / B;
+        int tk = k == 0 ? p.anchor[s] : x[j - 1];
+        if (tk < 0 || tk >= V) tk = 0;                         // reported at the start
+        reinterpret_cast<float4 *>(e)[i] = __ldg(reinterpret_cast<const float4 *>(p.Ep + (size_t)tk * RANK + cb) + q);
+    }
+}
+
 __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t *base, unsigned long long t_start)
 {
     TsShared &sh = *reinterpret_cast<TsShared *>(base);
@@ -591,6 +604,12 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
         sh.st[tid] = s;
         const float T = p.temperature[tid];
         sh.invT[tid] = T > 0.0f ? 1.0f / T : 0.0f;
+    }
+    // with a draft, pass 0's tokens are known now: gather its E' rows while
+    // the Read CTAs run the precompute
+    if (p.draft) {
+        __syncthreads();
+        gather_e(p, sh.x, e, CH, cb, tid, nth);
     }
     if (tid == 0) sh.go = wait_count(c, &c->pre_done.v, (unsigned)p.S);
     __syncthreads();
@@ -672,15 +691,10 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
         const unsigned long long t_pass = globaltimer_ns();
         const int trs = (lead && tid == 0 && p.trace && pass < 3) ? 210 + 8 * pass : 0;
         if (trs) trace_mark(p.trace, trs, t_pass);
-        // Fuse, token part: e_j = E'[x_{j-1}] (x_{-1} = anchor) for every
-        // position, kept channels (16-byte pieces)
-        for (int i = tid; i < N * CH / 4; i += nth) {
-            const int j = i / (CH / 4), q = i % (CH / 4), k = j % B, s = j / B;
-            int x = k == 0 ? p.anchor[s] : sh.x[j - 1];
-            if (x < 0 || x >= V) x = 0;                        // reported at the start
-            reinterpret_cast<float4 *>(e)[i] = __ldg(reinterpret_cast<const float4 *>(p.Ep + (size_t)x * RANK + cb) + q);
+        if (pass > 0 || !p.draft) {
+            gather_e(p, sh.x, e, CH, cb, tid, nth);
+            __syncthreads();
         }
-        __syncthreads();
         if (trs) trace_mark(p.trace, trs + 1, t_pass);
         // Mix for the evaluated tokens; c enters W_1 rounded to bf16.
         if (full) {
@@ -815,8 +829,7 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
             zf[(size_t)tok * RANK + d0 + dd] = z;
             zpack[(size_t)t * RANK + d0 + dd] = f2bf(z);
         }
-        fence_proxy_async_global();                            // z is read by TMA
-        __syncthreads();
+        __syncthreads();                                       // (the Read CTAs fence before their TMA of z)
         if (tid == 0) {
             red_add_release_gpu(&c->z_ready.v, 1u);
             if (lead && p.trace) trace_mark(p.trace, 8 + 4 * pass, t_pass);
