@@ -261,10 +261,6 @@ __device__ __forceinline__ RPartial rpartial_identity()
     return RPartial{-INFINITY, 0x7fffffff, -INFINITY, 0.0f, 0x7fffffff, -INFINITY, 0, 0};
 }
 
-// Fold one group of 32 corrected logits l[v0 .. v0+31] (entries j >= valid
-// are ignored) into the state.  T <= 0: argmax.  T > 0: x = l * invT, the
-// group's log-sum-exp plus its Gumbel noise competes for the group draw, and
-// (m, s) accumulate the full log-sum-exp.
 // The member draw of the hierarchical Gumbel-max inside group [v0, v0 + 32):
 // argmax over the members j < valid of x_j + Gumbel(seed, v0 + j, pos,
 // STREAM_ELEM, offset), smallest id on ties; one Philox call per 4 ids.  x is
@@ -296,25 +292,38 @@ __device__ __forceinline__ void member_draw(const float *x, int valid, int v0, u
     sel = bx;
 }
 
-// xsave (T > 0 only): when given, the x of the best group so far are stored at
-// xsave[32 j], so that the caller can draw the member of the group that ends
-// up best once (member_draw).  Without it the partial carries no member and
-// the end of the pass draws it (draw_in_group).
-__device__ __forceinline__ void select_group(SelState &st, const float *l, int v0, int valid, float invT,
-                                             unsigned long long seed, uint32_t pos, uint32_t offset,
-                                             float *xsave = nullptr)
+// Gumbel noise of the 4 consecutive vocabulary groups 4 g4 .. 4 g4 + 3 of one
+// position (stream STREAM_GROUP): one Philox call, word q for group 4 g4 + q
+// (the counter layout of uniform01), -log(-log u) with the fast logarithm.
+__device__ __forceinline__ void group_noise4(unsigned long long seed, uint32_t g4, uint32_t pos, uint32_t offset,
+                                             float (&gn)[4])
 {
-    if (valid <= 0) return;
+    const uint4 o = philox10(make_uint4(g4, pos, STREAM_GROUP, offset), (uint32_t)seed, (uint32_t)(seed >> 32));
+    const uint32_t w[4] = {o.x, o.y, o.z, o.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) gn[q] = -__logf(-__logf(((float)(w[q] >> 9) + 0.5f) * (1.0f / 8388608.0f)));
+}
+__device__ __forceinline__ float group_noise(unsigned long long seed, uint32_t g, uint32_t pos, uint32_t offset)
+{
+    float gn[4];
+    group_noise4(seed, g >> 2, pos, offset, gn);
+    return gn[g & 3];
+}
+
+template <bool FULL>
+__device__ __forceinline__ void select_group_impl(SelState &st, const float *l, int v0, int valid, float invT,
+                                                  float gnoise, float *xsave)
+{
     if (invT <= 0.0f) {
         float mx = -INFINITY;
 #pragma unroll
         for (int j = 0; j < GROUP; ++j)
-            if (j < valid) mx = fmaxf(mx, l[j]);
+            if (FULL || j < valid) mx = fmaxf(mx, l[j]);
         if (mx > st.best) {
             int at = 0;
 #pragma unroll
             for (int j = GROUP - 1; j >= 0; --j)
-                if (j < valid && l[j] == mx) at = j;
+                if ((FULL || j < valid) && l[j] == mx) at = j;
             st.best = mx;
             st.idx = v0 + at;
         }
@@ -325,17 +334,16 @@ __device__ __forceinline__ void select_group(SelState &st, const float *l, int v
 #pragma unroll
     for (int j = 0; j < GROUP; ++j) {
         x[j] = l[j] * invT;
-        if (j < valid) mx = fmaxf(mx, x[j]);
+        if (FULL || j < valid) mx = fmaxf(mx, x[j]);
     }
     float sum = 0.0f;
 #pragma unroll
     for (int j = 0; j < GROUP; ++j)
-        if (j < valid) sum += __expf(x[j] - mx);
-    const uint32_t g = (uint32_t)v0 / GROUP;
-    const float score = mx + __logf(sum) + gumbel(seed, g, pos, STREAM_GROUP, offset);
+        if (FULL || j < valid) sum += __expf(x[j] - mx);
+    const float score = mx + __logf(sum) + gnoise;
     if (score > st.best) {
         st.best = score;
-        st.idx = (int)g;
+        st.idx = v0 / GROUP;
         if (xsave) {
             // keep the group's x for one member draw at the end of the range
 #pragma unroll
@@ -343,6 +351,21 @@ __device__ __forceinline__ void select_group(SelState &st, const float *l, int v
         }
     }
     merge_lse(st.m, st.s, mx, sum);
+}
+
+// Fold one group of 32 corrected logits l[v0 .. v0+31] (entries j >= valid
+// are ignored) into the state.  T <= 0: argmax.  T > 0: x = l * invT, the
+// group's log-sum-exp plus its Gumbel noise `gnoise` (group_noise) competes for
+// the group draw, and (m, s) accumulate the full log-sum-exp.  xsave (T > 0
+// only): when given, the x of the best group so far are stored at xsave[32 j],
+// so that the caller can draw the member of the group that ends up best once
+// (member_draw).  Without it the partial carries no member and the end of the
+// pass draws it (draw_in_group).
+__device__ __forceinline__ void select_group(SelState &st, const float *l, int v0, int valid, float invT,
+                                             float gnoise, float *xsave = nullptr)
+{
+    if (valid >= GROUP) select_group_impl<true>(st, l, v0, GROUP, invT, gnoise, xsave);
+    else if (valid > 0) select_group_impl<false>(st, l, v0, valid, invT, gnoise, xsave);
 }
 
 // ------------------------------------------------------------- PTX wrappers

@@ -264,12 +264,25 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             // (tile, group) work items in order; s of item i + 1 is loaded
             // while item i is processed
             const int items = (vt1 - vt0) * g_count;
+            // this thread's s segment of vocabulary tile vt into L2 (bulk, no
+            // registers): the register loads one group ahead then hit L2
+            auto prefetch_s = [&](int vt) {
+                const int v0 = vt * TC_BN + g_first * GROUP;
+                if (valid && vt < vt1 && v0 < p.V)
+                    prefetch_l2_bulk(srow + v0, (uint32_t)min(g_count * GROUP, p.V - v0) * 2u);
+            };
+            prefetch_s(vt0);
+            prefetch_s(vt0 + 1);
             uint4 cur[4], nxt[4];
+            float gn[4] = {0.f, 0.f, 0.f, 0.f};     // T > 0: Gumbel noise of the tile's group quad
             load_s_group(cur, srow, vt0 * TC_BN + g_first * GROUP, p.V, valid);
             for (int it = 0; it < items; ++it) {
                 const int vt = vt0 + it / g_count, gl = g_first + it % g_count;
                 const int buf = t & 1;
                 if (gl == g_first) {
+                    prefetch_s(vt + 2);
+                    if (valid && invT > 0.0f)
+                        group_noise4(seed, (uint32_t)(vt * (TC_BN / GROUP) + g_first) >> 2, (uint32_t)pos, p.offset, gn);
                     if (!mbar_wait(&sh.tfull[buf], (t >> 1) & 1, abort)) { ok = false; break; }
                     tc_fence_after();
                 }
@@ -297,7 +310,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                         for (int jj = 0; jj < GROUP; ++jj)
                             if (jj < nv) dst[jj] = acc[jj];
                     }
-                    select_group(sel, acc, v0, nv, invT, seed, (uint32_t)pos, p.offset);
+                    select_group(sel, acc, v0, nv, invT, gn[(v0 / GROUP) & 3]);
                 }
 #pragma unroll
                 for (int c = 0; c < 4; ++c) cur[c] = nxt[c];

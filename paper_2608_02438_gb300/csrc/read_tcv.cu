@@ -246,7 +246,8 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
                     for (int jj = 0; jj < GROUP; ++jj)
                         if (jj < nv) dst[jj] = l[jj];
                 }
-                select_group(sel, l, v0, nv, my_invT, my_seed, (uint32_t)my_pos, p.offset);
+                const float gz = my_invT > 0.0f ? group_noise(my_seed, (uint32_t)(v0 / GROUP), (uint32_t)my_pos, p.offset) : 0.0f;
+                select_group(sel, l, v0, nv, my_invT, gz);
             }
             __syncwarp();
 #pragma unroll

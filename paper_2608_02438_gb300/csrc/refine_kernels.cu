@@ -682,7 +682,8 @@ __global__ void __launch_bounds__(256) k_read_simt(const Params *__restrict__ pp
                 float row[32];
 #pragma unroll
                 for (int j = 0; j < 32; ++j) row[j] = ls[warp][lane][j];
-                select_group(sel, row, g * GROUP, min(GROUP, p.V - g * GROUP), invT, seed, pos, p.offset);
+                select_group(sel, row, g * GROUP, min(GROUP, p.V - g * GROUP), invT,
+                             invT > 0.0f ? group_noise(seed, (uint32_t)g, pos, p.offset) : 0.0f);
             }
             __syncwarp();
         }

@@ -484,7 +484,9 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
                         for (int jj = 0; jj < GROUP; ++jj)
                             if (jj < nv) dst[jj] = l[jj];
                     }
-                    select_group(sel, l, v0, nv, my_invT, my_seed, (uint32_t)my_pos, p.offset, &sh.bestx[ew][0][lane]);
+                    const float gz =
+                        my_invT > 0.0f ? group_noise(my_seed, (uint32_t)(v0 / GROUP), (uint32_t)my_pos, p.offset) : 0.0f;
+                    select_group(sel, l, v0, nv, my_invT, gz, &sh.bestx[ew][0][lane]);
                 }
                 __syncwarp();
 #pragma unroll
