@@ -314,11 +314,14 @@ template <bool FULL>
 __device__ __forceinline__ void select_group_impl(SelState &st, const float *l, int v0, int valid, float invT,
                                                   float gnoise, float *xsave)
 {
+    // four independent chains for the max and the sum, so that few warps
+    // still keep the pipes busy
     if (invT <= 0.0f) {
-        float mx = -INFINITY;
+        float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
         for (int j = 0; j < GROUP; ++j)
-            if (FULL || j < valid) mx = fmaxf(mx, l[j]);
+            if (FULL || j < valid) m4[j & 3] = fmaxf(m4[j & 3], l[j]);
+        const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
         if (mx > st.best) {
             int at = 0;
 #pragma unroll
@@ -330,16 +333,18 @@ __device__ __forceinline__ void select_group_impl(SelState &st, const float *l, 
         return;
     }
     float x[GROUP];
-    float mx = -INFINITY;
+    float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
     for (int j = 0; j < GROUP; ++j) {
         x[j] = l[j] * invT;
-        if (FULL || j < valid) mx = fmaxf(mx, x[j]);
+        if (FULL || j < valid) m4[j & 3] = fmaxf(m4[j & 3], x[j]);
     }
-    float sum = 0.0f;
+    const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+    float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int j = 0; j < GROUP; ++j)
-        if (FULL || j < valid) sum += __expf(x[j] - mx);
+        if (FULL || j < valid) s4[j & 3] += __expf(x[j] - mx);
+    const float sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
     const float score = mx + __logf(sum) + gnoise;
     if (score > st.best) {
         st.best = score;
@@ -469,6 +474,22 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity)
     return ok != 0;
 }
 
+// try_wait with a suspend-time hint: the thread sleeps until the phase
+// completes or about `hint_ns` pass, instead of spinning on issue slots that
+// the other warps of its sub-partition need.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t *bar, uint32_t parity, uint32_t hint_ns)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity), "r"(hint_ns)
+        : "memory");
+    return ok != 0;
+}
+
 // Bounded wait: gives up after `limit_ns` of wall time or as soon as another
 // role raised *abort; returns false then (the caller unwinds).
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volatile int *abort,
@@ -477,8 +498,8 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volati
     if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = globaltimer();
     for (uint32_t it = 1;; ++it) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if ((it & 63u) == 0) {
+        if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
+        if ((it & 7u) == 0) {
             if (*abort) return false;
             if (globaltimer() - t0 > limit_ns) { *abort = 1; return false; }
         }
@@ -514,6 +535,20 @@ __device__ __forceinline__ void tma_load_2d_hint(void *smem_dst, const CUtensorM
 __device__ __forceinline__ void prefetch_l2_bulk(const void *addr, uint32_t bytes)
 {
     asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(addr), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ uint64_t policy_evict_first()
+{
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+
+// Same as prefetch_l2_bulk, with an L2 cache policy.
+__device__ __forceinline__ void prefetch_l2_bulk_hint(const void *addr, uint32_t bytes, uint64_t policy)
+{
+    asm volatile("cp.async.bulk.prefetch.L2.global.L2::cache_hint [%0], %1, %2;" ::"l"(addr), "r"(bytes), "l"(policy)
+                 : "memory");
 }
 
 __device__ __forceinline__ uint64_t policy_evict_last()

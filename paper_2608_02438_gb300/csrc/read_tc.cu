@@ -73,13 +73,13 @@ __device__ __forceinline__ bool epi_bar_or(bool pred)
 }
 
 // s[v0 .. v0 + 31] of one token as raw bf16 pairs (zeros past V or for an
-// invalid thread).
+// invalid thread); streaming loads (s is read once, evict it first).
 __device__ __forceinline__ void load_s_group(uint4 (&r)[4], const uint16_t *row, int v0, int V, bool valid)
 {
     if (valid && v0 + GROUP <= V) {
         const uint4 *src = reinterpret_cast<const uint4 *>(row + v0);
 #pragma unroll
-        for (int c = 0; c < 4; ++c) r[c] = __ldg(src + c);
+        for (int c = 0; c < 4; ++c) r[c] = __ldcs(src + c);
         return;
     }
     uint32_t w[16];
@@ -266,10 +266,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             const int items = (vt1 - vt0) * g_count;
             // this thread's s segment of vocabulary tile vt into L2 (bulk, no
             // registers): the register loads one group ahead then hit L2
+            // s is read once: evict it first, so that W_r (re-read for every
+            // token tile, evict_last) stays in L2
+            const uint64_t once = policy_evict_first();
             auto prefetch_s = [&](int vt) {
                 const int v0 = vt * TC_BN + g_first * GROUP;
                 if (valid && vt < vt1 && v0 < p.V)
-                    prefetch_l2_bulk(srow + v0, (uint32_t)min(g_count * GROUP, p.V - v0) * 2u);
+                    prefetch_l2_bulk_hint(srow + v0, (uint32_t)min(g_count * GROUP, p.V - v0) * 2u, once);
             };
             prefetch_s(vt0);
             prefetch_s(vt0 + 1);
