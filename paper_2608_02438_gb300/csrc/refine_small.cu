@@ -352,7 +352,7 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
                     sh.pass_n = min(__ldcg(p.ctl + CTL_NACT), TV_BN);
                 }
                 sh.pass_stop = go ? 0 : 1;
-                if (p.trace && pass == 1) { const unsigned long long tn = globaltimer_ns(); trace_mark(p.trace, 201, tn); }
+                if (p.trace && pass < 2) { const unsigned long long tn = globaltimer_ns(); trace_mark(p.trace, pass ? 201 : 231, tn); }
                 mbar_arrive(&sh.go);
                 if (!go) break;
                 // z of this pass, once the previous pass's MMAs are done with it
@@ -381,7 +381,7 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
                 if (*reinterpret_cast<volatile int *>(&sh.pass_stop)) break;
                 if (!mbar_wait(&sh.z_full, (uint32_t)(pass & 1), abort)) break;
                 tc_fence_after();
-                if (p.trace && pass == 1) { const unsigned long long tn = globaltimer_ns(); trace_mark(p.trace, 202, tn); }
+                if (p.trace && pass < 2) { const unsigned long long tn = globaltimer_ns(); trace_mark(p.trace, pass ? 202 : 232, tn); }
                 bool ok = true;
                 for (int i = 0; i < nblk && ok; ++i) {
                     const int ib = pass * nblk + i, buf = ib % TV_NBUF;
@@ -404,7 +404,7 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
                 }
                 if (!ok) break;
                 tc_commit(&sh.z_empty);
-                if (p.trace && pass == 1) { const unsigned long long tn = globaltimer_ns(); trace_mark(p.trace, 203, tn); }
+                if (p.trace && pass < 2) { const unsigned long long tn = globaltimer_ns(); trace_mark(p.trace, pass ? 203 : 233, tn); }
             }
             tc_commit(&sh.drain);
             int dummy = 0;
@@ -493,7 +493,7 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
                 for (int cc = 0; cc < 4; ++cc) cur[cc] = nxt[cc];
             }
             sh.sel[ew][lane] = sel;
-            if (p.trace && pass == 1 && lane == 0) { const unsigned long long tn = globaltimer_ns(); trace_mark(p.trace, 204, tn); }
+            if (p.trace && pass < 2 && lane == 0) { const unsigned long long tn = globaltimer_ns(); trace_mark(p.trace, pass ? 204 : 234, tn); }
             if (tv_epi_bar_or(!ok || *abort)) break;
             if (ew == 0 && lane < n) {
                 RPartial a = sh.sel[0][lane].partial();
@@ -710,17 +710,18 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
                     float er[FULL_C_MAX_B];
 #pragma unroll
                     for (int j2 = 0; j2 < FULL_C_MAX_B; ++j2) er[j2] = j2 < B ? e[(s * B + j2) * CH + dd] : 0.0f;
+                    // k rolled (short code: the first pass runs it cold), j unrolled
+                    // so that er stays in registers
+#pragma unroll 1
+                    for (int k = st.m + 1; k < B; ++k) {
+                        float a = pc[(s * B + k) * CH + dd] + e[(s * B + k) * CH + dd];
+                        const uint16_t *lrow = Lp + (k * (k - 1) / 2) * CH + dd;
 #pragma unroll
-                    for (int k = 0; k < FULL_C_MAX_B; ++k) {
-                        if (k < B && k > st.m) {
-                            float a = pc[(s * B + k) * CH + dd] + er[k];
-#pragma unroll
-                            for (int j2 = 0; j2 < k; ++j2)
-                                a = fmaf(bf2f(Lp[(k * (k - 1) / 2 + j2) * CH + dd]), er[j2], a);
-                            const int t = st.off + k - st.m - 1;
-                            cop[t * COP_LD + dd] = f2bf(a);
-                            if ((dd >> 5) == rank) sh.cown[t][dd & 31] = a;
-                        }
+                        for (int j2 = 0; j2 < FULL_C_MAX_B - 1; ++j2)
+                            if (j2 < k) a = fmaf(bf2f(lrow[j2 * CH]), er[j2], a);
+                        const int t = st.off + k - st.m - 1;
+                        cop[t * COP_LD + dd] = f2bf(a);
+                        if ((dd >> 5) == rank) sh.cown[t][dd & 31] = a;
                     }
                 }
         } else {

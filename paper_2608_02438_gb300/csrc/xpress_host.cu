@@ -589,6 +589,7 @@ void print_trace(xpress_refiner *R, cudaStream_t st)
         if (h[i] == ~0ull) continue;
         char name[32];
         if (i >= 240 && i < 248) std::snprintf(name, sizeof(name), "end%dphase%d", (i - 240) / 4, (i - 240) % 4);
+        else if (i >= 230 && i < 240) std::snprintf(name, sizeof(name), "read0phase%d", i - 230);
         else if (i >= 210) std::snprintf(name, sizeof(name), "mlp%dphase%d", (i - 210) / 8, (i - 210) % 8);
         else if (i >= 200) std::snprintf(name, sizeof(name), "readphase%d", i - 200);
         else if (i < 8) std::snprintf(name, sizeof(name), "%s", i < 4 ? pre[i] : "?");
