@@ -609,9 +609,31 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
     }
     // with a draft, pass 0's tokens are known now: gather its E' rows while
     // the Read CTAs run the precompute
+    float *mixe = reinterpret_cast<float *>(uop);             // [32][RANK] fp32 (full mode, pass 0 only)
     if (p.draft) {
         __syncthreads();
         gather_e(p, sh.x, e, CH, cb, tid, nth);
+        if (full) {
+            // the token part of pass 0's Mix, e_k + sum_{j<k} L_kj e_j, while
+            // the Read CTAs run the precompute (uop is free until W_1)
+            __syncthreads();
+            const int dd = tid;
+            if (dd < RANK)
+                for (int s = 0; s < b; ++s) {
+                    float er[FULL_C_MAX_B];
+#pragma unroll
+                    for (int j2 = 0; j2 < FULL_C_MAX_B; ++j2) er[j2] = j2 < B ? e[(s * B + j2) * CH + dd] : 0.0f;
+#pragma unroll 1
+                    for (int k = 0; k < B; ++k) {
+                        float a = e[(s * B + k) * CH + dd];
+                        const uint16_t *lrow = Lp + (k * (k - 1) / 2) * CH + dd;
+#pragma unroll
+                        for (int j2 = 0; j2 < FULL_C_MAX_B - 1; ++j2)
+                            if (j2 < k) a = fmaf(bf2f(lrow[j2 * CH]), er[j2], a);
+                        mixe[(s * B + k) * CH + dd] = a;
+                    }
+                }
+        }
     }
     if (tid == 0) sh.go = wait_count(c, &c->pre_done.v, (unsigned)p.S);
     __syncthreads();
@@ -703,6 +725,7 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
             // thread = channel; a block's E' values sit in registers and both
             // loops are unrolled (B <= 16), predicated on the block's frontier
             const int dd = tid;
+            const bool pre_mixed = pass == 0 && p.draft;       // e_k + sum_j L e_j formed during the precompute
             if (dd < RANK)
                 for (int s = 0; s < b; ++s) {
                     const SeqState st = sh.st[s];
@@ -714,12 +737,18 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
                     // so that er stays in registers
 #pragma unroll 1
                     for (int k = st.m + 1; k < B; ++k) {
-                        float a = pc[(s * B + k) * CH + dd] + e[(s * B + k) * CH + dd];
-                        const uint16_t *lrow = Lp + (k * (k - 1) / 2) * CH + dd;
-#pragma unroll
-                        for (int j2 = 0; j2 < FULL_C_MAX_B - 1; ++j2)
-                            if (j2 < k) a = fmaf(bf2f(lrow[j2 * CH]), er[j2], a);
                         const int t = st.off + k - st.m - 1;
+                        float a;
+                        if (pre_mixed) {
+                            a = mixe[(s * B + k) * CH + dd];
+                        } else {
+                            a = e[(s * B + k) * CH + dd];
+                            const uint16_t *lrow = Lp + (k * (k - 1) / 2) * CH + dd;
+#pragma unroll
+                            for (int j2 = 0; j2 < FULL_C_MAX_B - 1; ++j2)
+                                if (j2 < k) a = fmaf(bf2f(lrow[j2 * CH]), er[j2], a);
+                        }
+                        a = pc[(s * B + k) * CH + dd] + a;
                         cop[t * COP_LD + dd] = f2bf(a);
                         if ((dd >> 5) == rank) sh.cown[t][dd & 31] = a;
                     }
@@ -731,10 +760,11 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
             if (t0 < tstep)
                 for (int t = t0; t < n; t += tstep) {
                     const int tok = sh.tok[t], s = sh.tseq[tok], k = sh.tpos[tok];
-                    float a = pc[tok * CH + dd] + e[tok * CH + dd];
+                    float a = e[tok * CH + dd];
                     const uint16_t *lrow = Lp + (k * (k - 1) / 2) * CH + dd;
                     const float *erow = e + (s * B) * CH + dd;
                     for (int j2 = 0; j2 < k; ++j2) a = fmaf(bf2f(lrow[j2 * CH]), erow[j2 * CH], a);
+                    a = pc[tok * CH + dd] + a;
                     sh.cown[t][dd] = a;
                     p.cx[(size_t)t * RANK + d0 + dd] = f2bf(a);
                 }
