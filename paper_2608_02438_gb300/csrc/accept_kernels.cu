@@ -42,8 +42,13 @@ __device__ __forceinline__ void load8(float (&x)[8], const void *base, int dtype
 }
 
 // grid (b * (B + 1), chunks); chunk boundaries are multiples of 8 ids.
+// The four kernels are chained with programmatic dependent launch: each lets
+// the next one start early and waits (griddepcontrol.wait) for its
+// predecessor's results right before reading them.
 __global__ void __launch_bounds__(256) k_acc_rows(AcceptParams p)
 {
+    pdl_trigger();
+    if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) *p.status = 0;
     const int row = blockIdx.x;                   // seq * (B + 1) + k
     const int seq = row / (p.B + 1);
     const int chunks = gridDim.y, c = blockIdx.y;
@@ -92,6 +97,8 @@ __global__ void __launch_bounds__(256) k_acc_rows(AcceptParams p)
 // position that is not accepted.
 __global__ void __launch_bounds__(32) k_acc_decide(AcceptParams p, int chunks)
 {
+    pdl_trigger();
+    pdl_wait();                                   // the row partials
     const int seq = blockIdx.x, lane = threadIdx.x;
     const int B = p.B;
     const float T = p.temperature[seq];
@@ -144,6 +151,8 @@ __global__ void __launch_bounds__(32) k_acc_decide(AcceptParams p, int chunks)
 // residual draw (best, idx) and the draw from p (m, s reused as score, idx).
 __global__ void __launch_bounds__(256) k_acc_sample(AcceptParams p)
 {
+    pdl_trigger();
+    pdl_wait();                                   // the decisions
     const int seq = blockIdx.x, chunks = gridDim.y, c = blockIdx.y;
     const int k = p.job[seq];
     if (k < 0) return;
@@ -195,6 +204,7 @@ __global__ void __launch_bounds__(256) k_acc_sample(AcceptParams p)
 
 __global__ void k_acc_finish(AcceptParams p, int chunks)
 {
+    pdl_wait();                                   // the draw partials
     const int seq = blockIdx.x * blockDim.x + threadIdx.x;
     if (seq >= p.b) return;
     const int k = p.job[seq];
