@@ -44,7 +44,10 @@ __device__ __forceinline__ void load8(float (&x)[8], const void *base, int dtype
 // grid (b * (B + 1), chunks); chunk boundaries are multiples of 8 ids.
 // The four kernels are chained with programmatic dependent launch: each lets
 // the next one start early and waits (griddepcontrol.wait) for its
-// predecessor's results right before reading them.
+// predecessor's results right before reading them.  k_acc_rows reads only the
+// target logits and temperatures, so it may run while the preceding kernel of
+// the stream (the refinement) finishes; it waits for that kernel before it
+// exits, so that the later kernels' waits cover it too.
 __global__ void __launch_bounds__(256) k_acc_rows(AcceptParams p)
 {
     pdl_trigger();
@@ -90,6 +93,7 @@ __global__ void __launch_bounds__(256) k_acc_rows(AcceptParams p)
         __syncthreads();
     }
     if (threadIdx.x == 0) p.rowpart[(size_t)row * chunks + c] = sp[0];
+    pdl_wait();
 }
 
 // one warp per block (sequence): lane k combines the chunk partials of target

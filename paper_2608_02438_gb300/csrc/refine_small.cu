@@ -978,6 +978,10 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
                    const __grid_constant__ CUtensorMap tmap_z)
 {
     const unsigned long long t_start = globaltimer_ns();
+    // a kernel launched after this one with programmatic dependent launch may
+    // start now (the acceptance's first kernel reads none of our outputs; a
+    // dependent must wait with griddepcontrol.wait before reading them)
+    pdl_trigger();
     extern __shared__ uint8_t smem_raw[];
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     SmallCtlArea *area = p.sctl;

@@ -850,9 +850,9 @@ int accept_launch(const xpress_refiner *R, const xpress_accept_in *in, int32_t *
     P.jobf = reinterpret_cast<float *>(w + A.jobf);
     P.spart = reinterpret_cast<Partial *>(w + A.spart);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    // k_acc_rows clears the status word; the others are chained to their
-    // predecessor with programmatic dependent launch
-    k_acc_rows<<<dim3(in->b * (R->w.B + 1), A.chunks), 256, 0, st>>>(P);
+    // all four are chained to their predecessor with programmatic dependent
+    // launch (k_acc_rows clears the status word)
+    XP_CUDA(launch_pdl(k_acc_rows, dim3(in->b * (R->w.B + 1), A.chunks), dim3(256), 0, st, P));
     XP_CUDA(launch_pdl(k_acc_decide, dim3(in->b), dim3(32), 0, st, P, A.chunks));
     XP_CUDA(launch_pdl(k_acc_sample, dim3(in->b, A.chunks2), dim3(256), 0, st, P));
     XP_CUDA(launch_pdl(k_acc_finish, dim3((in->b + 127) / 128), dim3(128), 0, st, P, A.chunks2));
