@@ -551,6 +551,20 @@ __device__ __forceinline__ void prefetch_l2_bulk_hint(const void *addr, uint32_t
                  : "memory");
 }
 
+// 16-byte asynchronous copy global -> shared (L2 only; bytes < 16 zero-fill
+// the rest) with an L2 cache policy, and its commit / wait groups.
+__device__ __forceinline__ void cp_async16(void *smem_dst, const void *gsrc, uint32_t bytes, uint64_t policy)
+{
+    asm volatile("cp.async.cg.shared.global.L2::cache_hint [%0], [%1], 16, %2, %3;" ::"r"(smem_u32(smem_dst)),
+                 "l"(gsrc), "r"(bytes), "l"(policy)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N> __device__ __forceinline__ void cp_async_wait()
+{
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
 __device__ __forceinline__ uint64_t policy_evict_last()
 {
     uint64_t pol;

@@ -30,7 +30,8 @@ constexpr int TC_BM = 128;
 constexpr int TC_BN = 256;
 constexpr int TC_BK = 64;                     // one 128-byte swizzle row of bf16
 constexpr int TC_KCH = RANK / TC_BK;          // 4 K-chunks
-constexpr int TC_STAGES = 4;
+constexpr int TC_STAGES = 2;                  // W_r stays in L2 (evict_last): 2 stages in flight suffice
+constexpr int TC_SPF = 4;                     // s groups in flight per epilogue thread (cp.async ring)
 constexpr int TC_EPI_WARPS = 8;
 constexpr int TC_THREADS = 32 * (2 + TC_EPI_WARPS);
 constexpr uint32_t TC_A_CHUNK = TC_BM * TC_BK * 2;       // 16 KB
@@ -50,7 +51,8 @@ struct TcShared {
     SelState st[TC_EPI_WARPS][32];
 };
 
-constexpr size_t TC_SMEM_BYTES = 1024 + TC_A_BYTES + TC_STAGES * TC_B_STAGE + sizeof(TcShared);
+constexpr uint32_t TC_S_BYTES = TC_SPF * 4 * (TC_EPI_WARPS * 32) * 16;   // [slot][chunk][thread] 16 B
+constexpr size_t TC_SMEM_BYTES = 1024 + TC_A_BYTES + TC_STAGES * TC_B_STAGE + TC_S_BYTES + sizeof(TcShared);
 const size_t kReadTcSmemBytes = TC_SMEM_BYTES;
 const int kReadTcThreads = TC_THREADS;
 
@@ -103,7 +105,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sA = base;
     uint8_t *sB = base + TC_A_BYTES;
-    TcShared &sh = *reinterpret_cast<TcShared *>(sB + TC_STAGES * TC_B_STAGE);
+    uint4 *sS = reinterpret_cast<uint4 *>(sB + TC_STAGES * TC_B_STAGE);   // epilogue s ring
+    TcShared &sh = *reinterpret_cast<TcShared *>(sB + TC_STAGES * TC_B_STAGE + TC_S_BYTES);
     const Params &p = *pp;
     const int NVT = (V + TC_BN - 1) / TC_BN;
     const int S = gridDim.x, r = blockIdx.x;
@@ -276,9 +279,25 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             };
             prefetch_s(vt0);
             prefetch_s(vt0 + 1);
-            uint4 cur[4], nxt[4];
             float gn[4] = {0.f, 0.f, 0.f, 0.f};     // T > 0: Gumbel noise of the tile's group quad
-            load_s_group(cur, srow, vt0 * TC_BN + g_first * GROUP, p.V, valid);
+            // s of item k into ring slot k % TC_SPF (cp.async, L2 only; zero-filled
+            // past V or for an invalid thread), one commit group per item
+            const int et = threadIdx.x - 64;
+            auto issue_s = [&](int k) {
+                if (k < items) {
+                    const int v0 = (vt0 + k / g_count) * TC_BN + (g_first + k % g_count) * GROUP;
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) {
+                        const int vv = v0 + 8 * c;
+                        const bool in = valid && vv < p.V;
+                        cp_async16(&sS[((k % TC_SPF) * 4 + c) * (TC_EPI_WARPS * 32) + et], in ? srow + vv : srow,
+                                   in ? 16u : 0u, once);
+                    }
+                }
+                cp_async_commit();
+            };
+#pragma unroll
+            for (int k = 0; k < TC_SPF - 1; ++k) issue_s(k);
             for (int it = 0; it < items; ++it) {
                 const int vt = vt0 + it / g_count, gl = g_first + it % g_count;
                 const int buf = t & 1;
@@ -289,10 +308,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     if (!mbar_wait(&sh.tfull[buf], (t >> 1) & 1, abort)) { ok = false; break; }
                     tc_fence_after();
                 }
-                if (it + 1 < items) {
-                    const int vn = vt0 + (it + 1) / g_count, gn = g_first + (it + 1) % g_count;
-                    load_s_group(nxt, srow, vn * TC_BN + gn * GROUP, p.V, valid);
-                }
+                issue_s(it + TC_SPF - 1);
+                cp_async_wait<TC_SPF - 1>();        // item it has landed
+                uint4 cur[4];
+#pragma unroll
+                for (int c = 0; c < 4; ++c) cur[c] = sS[((it % TC_SPF) * 4 + c) * (TC_EPI_WARPS * 32) + et];
                 const int v0 = vt * TC_BN + gl * GROUP;
                 const int nv = min(GROUP, p.V - v0);
                 float acc[GROUP];
@@ -315,8 +335,6 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     }
                     select_group(sel, acc, v0, nv, invT, gn[(v0 / GROUP) & 3]);
                 }
-#pragma unroll
-                for (int c = 0; c < 4; ++c) cur[c] = nxt[c];
                 if (gl == g_first + g_count - 1) {
                     tc_fence_before();
                     __syncwarp();
@@ -324,6 +342,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     ++t;
                 }
             }
+            cp_async_wait<0>();                      // nothing in flight into the ring
             sh.st[ew][lane] = sel;
             const bool stop = epi_bar_or(!ok || *abort);
             if (!stop) {
