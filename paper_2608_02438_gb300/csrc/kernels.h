@@ -57,6 +57,12 @@ __global__ void k_pack_L(const uint16_t *L, uint16_t *Lpk, int B);
 extern const size_t kRefineSmallSmemBytes;
 constexpr int SMALL_TRANS_CTAS = 8;
 
+// pre_tc.cu (bf16, more than 32 tokens: the hidden projection on tcgen05)
+__global__ void k_pre_tc(const Params *pp, const __grid_constant__ CUtensorMap tmap_h,
+                         const __grid_constant__ CUtensorMap tmap_wh, const __grid_constant__ CUtensorMap tmap_wg,
+                         int kslice);
+extern const size_t kPreTcSmemBytes;
+
 // accept_kernels.cu
 __global__ void k_acc_rows(AcceptParams p);
 __global__ void k_acc_decide(AcceptParams p, int chunks);

@@ -60,6 +60,7 @@ struct GraphEntry {
     cudaGraph_t graph = nullptr;
     cudaGraphExec_t exec = nullptr;
     cudaGraphNode_t init_node = nullptr;
+    cudaGraphNode_t pre_node = nullptr;    // k_pre_tc (its h tensor map changes per call)
     cudaGraphConditionalHandle handle = 0;
     dim3 init_grid;
     uint64_t stamp = 0;
@@ -76,6 +77,7 @@ struct Layout {
     bool gemv = false;
     bool tcv = false;
     bool small = false;      // persistent small-batch kernel
+    bool pre_tc = false;     // hidden projection on tcgen05 (bf16, more than 32 tokens)
 };
 
 }  // namespace
@@ -86,6 +88,7 @@ struct xpress_refiner {
     unsigned long long *trace = nullptr;   // profiling timeline (XPRESS_TRACE=1)
     CUtensorMap tmap_wr{};                 // W_r boxes of 256 rows (k_read_tc)
     CUtensorMap tmap_wr128{};              // W_r boxes of 128 rows (k_read_tcv)
+    CUtensorMap tmap_wh{}, tmap_wg{};      // W_h, W_g boxes of 256 rows x 64 (k_pre_tc)
     int device = 0;
     int num_sms = 0;
     bool use_tc = false;
@@ -143,6 +146,15 @@ Layout make_layout(const xpress_refiner *R, int b)
         int ks = (GEMV_SMEM / (2 * N)) / 256 * 256;
         const int H256 = (R->w.H + 255) / 256 * 256;
         L.kchunk = ks < H256 ? ks : H256;
+        L.ksplit = (R->w.H + L.kchunk - 1) / L.kchunk;
+    } else if (R->use_tc) {
+        // k_pre_tc: 128-token x 256-row tiles, split over K to about one wave
+        L.pre_tc = true;
+        const int tiles = 2 * ((N + 127) / 128);
+        int ks = (R->num_sms + tiles / 2) / tiles;
+        const int kmax = (R->w.H + 63) / 64;
+        ks = ks < 1 ? 1 : (ks > kmax ? kmax : ks);
+        L.kchunk = ((R->w.H + ks - 1) / ks + 63) / 64 * 64;
         L.ksplit = (R->w.H + L.kchunk - 1) / L.kchunk;
     } else {
         const int mt = (N + 63) / 64;
@@ -299,7 +311,9 @@ int set_kernel_attributes()
             cudaFuncSetAttribute(k_read_tcv, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kReadTcvSmemBytes) !=
                 cudaSuccess ||
             cudaFuncSetAttribute(k_refine_small, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)kRefineSmallSmemBytes) != cudaSuccess) {
+                                 (int)kRefineSmallSmemBytes) != cudaSuccess ||
+            cudaFuncSetAttribute(k_pre_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kPreTcSmemBytes) !=
+                cudaSuccess) {
             (void)cudaGetLastError();
             rc = XPRESS_ERR_CUDA;
         }
@@ -325,6 +339,35 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
+
+// Arguments of a k_pre_tc launch (kept alive for cudaGraphAddKernelNode /
+// cudaGraphExecKernelNodeSetParams, which read them through kernelParams).
+struct PreTcArgs {
+    const Params *pdev;
+    CUtensorMap th;
+    CUtensorMap wh, wg;
+    int kslice;
+    void *ptrs[5];
+    bool make(const xpress_refiner *R, const Params &P, const Layout &L, Params *pd)
+    {
+        pdev = pd;
+        wh = R->tmap_wh;
+        wg = R->tmap_wg;
+        kslice = L.kchunk;
+        ptrs[0] = &pdev; ptrs[1] = &th; ptrs[2] = &wh; ptrs[3] = &wg; ptrs[4] = &kslice;
+        return make_tmap_bf16(&th, P.h, (uint64_t)P.H, (uint64_t)P.N, 64, 128);
+    }
+    cudaKernelNodeParams node(const Layout &L, int N)
+    {
+        cudaKernelNodeParams kp{};
+        kp.func = reinterpret_cast<void *>(k_pre_tc);
+        kp.gridDim = dim3((unsigned)((N + 127) / 128), 2, (unsigned)L.ksplit);
+        kp.blockDim = dim3(320);
+        kp.sharedMemBytes = (unsigned)kPreTcSmemBytes;
+        kp.kernelParams = ptrs;
+        return kp;
+    }
+};
 
 void launch_pre_gemm(const Layout &L, int N, Params *pdev, cudaStream_t st)
 {
@@ -379,10 +422,18 @@ int build_graph(xpress_refiner *R, GraphEntry &e, const Params &P, const Layout 
         XP_CUDA(cudaGraphAddKernelNode(&e.init_node, g, &mnode, 1, &kp));
     }
 
+    cudaGraphNode_t cap_dep = e.init_node;
+    if (L.pre_tc) {
+        PreTcArgs a;
+        if (!a.make(R, P, L, pdev)) return XPRESS_ERR_CUDA;
+        cudaKernelNodeParams kp = a.node(L, N);
+        XP_CUDA(cudaGraphAddKernelNode(&e.pre_node, g, &e.init_node, 1, &kp));
+        cap_dep = e.pre_node;
+    }
     cudaStream_t cs = R->cs;
-    XP_CUDA(cudaStreamBeginCaptureToGraph(cs, g, &e.init_node, nullptr, 1, cudaStreamCaptureModeThreadLocal));
+    XP_CUDA(cudaStreamBeginCaptureToGraph(cs, g, &cap_dep, nullptr, 1, cudaStreamCaptureModeThreadLocal));
     if (!P.draft) k_rowmax<<<N, 256, 0, cs>>>(pdev);
-    launch_pre_gemm(L, N, pdev, cs);
+    if (!L.pre_tc) launch_pre_gemm(L, N, pdev, cs);
     k_pre_mix<<<dim3(b, RANK / 32), 256, pre_mix_smem(P.B), cs>>>(pdev);
     cudaStreamCaptureStatus cst;
     const cudaGraphNode_t *deps = nullptr;
@@ -495,7 +546,14 @@ int run_eager(xpress_refiner *R, Params P, const Layout &L, void *ws, cudaStream
         kt.stop();
     }
     kt.start("pre_gemm");
-    launch_pre_gemm(L, N, pdev, st);
+    if (L.pre_tc) {
+        PreTcArgs a;
+        if (!a.make(R, P, L, pdev)) return XPRESS_ERR_CUDA;
+        k_pre_tc<<<dim3((unsigned)((N + 127) / 128), 2, (unsigned)L.ksplit), 320, kPreTcSmemBytes, st>>>(
+            pdev, a.th, a.wh, a.wg, a.kslice);
+    } else {
+        launch_pre_gemm(L, N, pdev, st);
+    }
     kt.stop();
     kt.start("pre_mix");
     k_pre_mix<<<dim3(b, RANK / 32), 256, pre_mix_smem(P.B), st>>>(pdev);
@@ -648,7 +706,9 @@ int xpress_refiner_create(const xpress_weights *w, void *stream, xpress_refiner 
         }
         R->use_tc = w->dtype == XPRESS_BF16;
         if (R->use_tc && (!make_tmap_bf16(&R->tmap_wr, w->W_r, RANK, (uint64_t)w->V, 64, 256) ||
-                          !make_tmap_bf16(&R->tmap_wr128, w->W_r, RANK, (uint64_t)w->V, 64, 128))) {
+                          !make_tmap_bf16(&R->tmap_wr128, w->W_r, RANK, (uint64_t)w->V, 64, 128) ||
+                          !make_tmap_bf16(&R->tmap_wh, w->W_h, (uint64_t)w->H, RANK, 64, 256) ||
+                          !make_tmap_bf16(&R->tmap_wg, w->W_g, (uint64_t)w->H, RANK, 64, 256))) {
             rc = XPRESS_ERR_CUDA;
             break;
         }
@@ -769,6 +829,12 @@ int xpress_refine_block(const xpress_refiner *Rc, const xpress_block_in *in, con
     kp.blockDim = dim3(256);
     kp.kernelParams = args;
     XP_CUDA(cudaGraphExecKernelNodeSetParams(hit->exec, hit->init_node, &kp));
+    if (L.pre_tc) {
+        PreTcArgs a;
+        if (!a.make(R, P, L, pdev)) return XPRESS_ERR_CUDA;
+        cudaKernelNodeParams pk = a.node(L, P.N);
+        XP_CUDA(cudaGraphExecKernelNodeSetParams(hit->exec, hit->pre_node, &pk));
+    }
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (R->trace) {
         XP_CUDA(cudaMemsetAsync(R->trace, 0xFF, TRACE_SLOTS * sizeof(unsigned long long), st));
