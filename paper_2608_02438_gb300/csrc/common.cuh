@@ -310,6 +310,14 @@ __device__ __forceinline__ float group_noise(unsigned long long seed, uint32_t g
     return gn[g & 3];
 }
 
+// 2^x with the hardware approximation (as exp's own fast path uses).
+__device__ __forceinline__ float ex2_approx(float x)
+{
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
 template <bool FULL>
 __device__ __forceinline__ void select_group_impl(SelState &st, const float *l, int v0, int valid, float invT,
                                                   float gnoise, float *xsave)
@@ -332,19 +340,20 @@ __device__ __forceinline__ void select_group_impl(SelState &st, const float *l, 
         }
         return;
     }
-    float x[GROUP];
+    // x = l / T: the max is taken on l (1/T > 0 keeps the order) and
+    // exp(x - max x) = 2^(l c - max l c) with c = log2(e) / T, one FMA each
     float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-    for (int j = 0; j < GROUP; ++j) {
-        x[j] = l[j] * invT;
-        if (FULL || j < valid) m4[j & 3] = fmaxf(m4[j & 3], x[j]);
-    }
-    const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+    for (int j = 0; j < GROUP; ++j)
+        if (FULL || j < valid) m4[j & 3] = fmaxf(m4[j & 3], l[j]);
+    const float ml = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+    const float cl = invT * 1.4426950408889634f, off2 = -ml * cl;
     float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int j = 0; j < GROUP; ++j)
-        if (FULL || j < valid) s4[j & 3] += __expf(x[j] - mx);
+        if (FULL || j < valid) s4[j & 3] += ex2_approx(fmaf(l[j], cl, off2));
     const float sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+    const float mx = ml * invT;
     const float score = mx + __logf(sum) + gnoise;
     if (score > st.best) {
         st.best = score;
@@ -352,7 +361,7 @@ __device__ __forceinline__ void select_group_impl(SelState &st, const float *l, 
         if (xsave) {
             // keep the group's x for one member draw at the end of the range
 #pragma unroll
-            for (int j = 0; j < GROUP; ++j) xsave[32 * j] = x[j];
+            for (int j = 0; j < GROUP; ++j) xsave[32 * j] = l[j] * invT;
         }
     }
     merge_lse(st.m, st.s, mx, sum);

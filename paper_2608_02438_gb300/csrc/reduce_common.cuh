@@ -237,14 +237,19 @@ __device__ __forceinline__ void pack_next_pass(const Params &p, cudaGraphConditi
 {
     const int B = p.B, warp = threadIdx.x / 32, lane = threadIdx.x % 32, nwarps = blockDim.x / 32;
     int carry = 0;
+    // greedy blocks first, then sampling ones: the Read's warps then mostly
+    // see one kind of selection
+    for (int cls = 0; cls < 2; ++cls)
     for (int q0 = 0; q0 < p.b; q0 += blockDim.x) {
         const int q = q0 + threadIdx.x;
         SeqState ns{};
         int c = 0;
+        bool mine = false;
         if (q < p.b) {
             const volatile int *src = reinterpret_cast<const volatile int *>(&p.st[q]);
             ns.active = src[0]; ns.m = src[1]; ns.iters = src[2]; ns.converged = src[3];
-            c = ns.active ? B - 1 - ns.m : 0;
+            mine = (p.temperature[q] > 0.0f) == (cls == 1);
+            c = (mine && ns.active) ? B - 1 - ns.m : 0;
         }
         int incl = c;
 #pragma unroll
@@ -265,7 +270,7 @@ __device__ __forceinline__ void pack_next_pass(const Params &p, cudaGraphConditi
         }
         __syncthreads();
         const int off = carry + (warp ? wsum[warp - 1] : 0) + incl - c;
-        if (q < p.b) {
+        if (q < p.b && mine) {
             ns.off = off;
             ns.cnt = c;
             p.st[q] = ns;
