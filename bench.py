@@ -221,14 +221,14 @@ def run_xpress(args):
         evaluated = ctl[4]                       # tokens evaluated over all passes
         # bf16 calls of at most 32 tokens run as one persistent kernel (unless
         # XPRESS_SMALL=0); others: init + precompute (two split-K GEMMs) +
-        # Fuse/Mix, then per pass Trans + Read + reduce.  Then the four
+        # Fuse/Mix, then per pass Trans + Read + reduce.  Then the two
         # acceptance kernels.
         persistent = (dt == X.XPRESS_BF16 and b * cfg.B <= 32 and os.environ.get("XPRESS_SMALL", "1") != "0")
         small = b * cfg.B <= 32
         if persistent:
-            per_step_launches = 1 + 4
+            per_step_launches = 1 + 2
         else:
-            per_step_launches = 1 + (1 if small else 2) + 1 + passes * (2 if small else 3) + 4
+            per_step_launches = 1 + (1 if small else 2) + 1 + passes * (2 if small else 3) + 2
         starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
         ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
         if world > 1:

@@ -3,16 +3,16 @@
 //   k_acc_rows    per target row (block position k = 1..B+1) and vocabulary
 //                 chunk: argmax (T <= 0) or the running max / sum of exp of
 //                 target / T (T > 0)
-//   k_acc_decide  per block: greedy -- longest prefix equal to the target
-//                 argmax plus the target's next token;  lossless -- accept y_k
-//                 while u_k q_k(y_k) < p_k(y_k), q from the refinement pass
-//                 (exp(l_y/T - lse)), p = softmax(target_k / T)
-//   k_acc_sample  per block with a draw to make and vocabulary chunk:
-//                 Gumbel-max over log max(0, p_k - q_k) at the first rejected
-//                 position (q_k recomputed from z_final through W_r), with the
-//                 draw from p_k alongside for an empty residual; or the bonus
-//                 draw from p_{B+1} after B acceptances
-//   k_acc_finish  combine the chunk partials and emit the last token
+//   k_acc_finalize per block and vocabulary chunk: the decision (greedy --
+//                 longest prefix equal to the target argmax plus the target's
+//                 next token; lossless -- accept y_k while u_k q_k(y_k) <
+//                 p_k(y_k), q from the refinement pass (exp(l_y/T - lse)),
+//                 p = softmax(target_k / T)), then for a sampling block the
+//                 draw over the chunk: Gumbel-max over log max(0, p_k - q_k)
+//                 at the first rejected position (q_k recomputed from z_final
+//                 through W_r), with the draw from p_k alongside for an empty
+//                 residual, or the bonus draw from p_{B+1} after B acceptances;
+//                 the block's last chunk combines the draws and emits the token
 #include "common.cuh"
 #include "kernels.h"
 
@@ -41,6 +41,12 @@ __device__ __forceinline__ void load8(float (&x)[8], const void *base, int dtype
     for (int j = 0; j < 8; ++j) x[j] = j < n ? ld_any(base, dtype, i + j) : 0.0f;
 }
 
+__device__ __forceinline__ Partial ldcg_partial16(const Partial *q)
+{
+    const float4 v = __ldcg(reinterpret_cast<const float4 *>(q));
+    return Partial{v.x, __float_as_int(v.y), v.z, v.w};
+}
+
 // grid (b * (B + 1), chunks); chunk boundaries are multiples of 8 ids.
 // The four kernels are chained with programmatic dependent launch: each lets
 // the next one start early and waits (griddepcontrol.wait) for its
@@ -51,7 +57,10 @@ __device__ __forceinline__ void load8(float (&x)[8], const void *base, int dtype
 __global__ void __launch_bounds__(256) k_acc_rows(AcceptParams p)
 {
     pdl_trigger();
-    if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) *p.status = 0;
+    if (blockIdx.x == 0 && blockIdx.y == 0) {
+        if (threadIdx.x == 0) *p.status = 0;
+        for (int q = threadIdx.x; q < p.b; q += blockDim.x) p.ticket[q] = 0;
+    }
     const int row = blockIdx.x;                   // seq * (B + 1) + k
     const int seq = row / (p.B + 1);
     const int chunks = gridDim.y, c = blockIdx.y;
@@ -96,73 +105,78 @@ __global__ void __launch_bounds__(256) k_acc_rows(AcceptParams p)
     pdl_wait();
 }
 
-// one warp per block (sequence): lane k combines the chunk partials of target
-// row k and takes the accept decision of position k; a ballot finds the first
-// position that is not accepted.
-__global__ void __launch_bounds__(32) k_acc_decide(AcceptParams p, int chunks)
+// grid (b, chunks2), 256 threads.  Warp 0 of every CTA takes block seq's
+// decision: lane k combines the chunk partials of target row k and decides
+// position k (greedy: y_k equals the target argmax; lossless: u_k q_k(y_k) <
+// p_k(y_k), q from the refinement pass, p = softmax(target_k / T)); a ballot
+// finds the first position not accepted.  Chunk 0 publishes the accepted
+// prefix (and, greedy, the target's token after it).  For a sampling block
+// every CTA then draws over its vocabulary chunk -- Gumbel-max over
+// log max(0, p_k - q_k) at the first rejected position (q_k recomputed from
+// z_final through W_r), with the draw from p_k alongside for an empty
+// residual, or the bonus draw from p_{B+1} after B acceptances -- and the last
+// CTA of the block (ticket) combines the chunks and emits the token.
+__global__ void __launch_bounds__(256) k_acc_finalize(AcceptParams p, int chunks)
 {
-    pdl_trigger();
-    pdl_wait();                                   // the row partials
-    const int seq = blockIdx.x, lane = threadIdx.x;
+    pdl_wait();                                   // the row partials (and the refinement before them)
+    const int seq = blockIdx.x, c = blockIdx.y, nch = gridDim.y;
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const int B = p.B;
     const float T = p.temperature[seq];
     const bool sampling = T > 0.0f;
     const float invT = sampling ? 1.0f / T : 0.0f;
     __shared__ Partial rows[MAX_B + 1];
-    for (int k = lane; k <= B; k += 32) {
-        Partial a{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
-        const size_t r = (size_t)seq * (B + 1) + k;
+    __shared__ int s_n;
+    __shared__ float s_lsep;
+    __shared__ int s_last;
+    if (warp == 0) {
+        for (int k = lane; k <= B; k += 32) {
+            Partial a{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
+            const size_t r = (size_t)seq * (B + 1) + k;
 #pragma unroll 4
-        for (int c = 0; c < chunks; ++c) merge_partial(a, p.rowpart[r * chunks + c], sampling);
-        rows[k] = a;
-    }
-    __syncwarp();
-    int y = -1;
-    bool ok = false;
-    float lse_p = 0.0f;
-    if (lane < B) {
-        y = p.tokens[(size_t)seq * B + lane];
-        if (y < 0 || y >= p.V) { set_status(p.status, ST_BOUNDS); y = 0; }
-        if (!sampling) {
-            ok = y == rows[lane].idx;
-        } else {
-            const int row = seq * (B + 1) + lane;
-            lse_p = rows[lane].m + logf(rows[lane].s);
-            const float p_y = expf(ld_any(p.target, p.dtype, (size_t)row * p.V + y) * invT - lse_p);
-            const float q_y = expf(p.logit_sel[(size_t)seq * B + lane] - p.lse[(size_t)seq * B + lane]);
-            const float u = uniform01(p.seed[seq], 0u, (uint32_t)lane, STREAM_ACCEPT, p.offset);
-            ok = u * q_y < p_y;
+            for (int cc = 0; cc < chunks; ++cc) merge_partial(a, p.rowpart[r * chunks + cc], sampling);
+            rows[k] = a;
+        }
+        __syncwarp();
+        int y = -1;
+        bool ok = false;
+        if (lane < B) {
+            y = p.tokens[(size_t)seq * B + lane];
+            if (y < 0 || y >= p.V) {
+                if (c == 0) set_status(p.status, ST_BOUNDS);
+                y = 0;
+            }
+            if (!sampling) {
+                ok = y == rows[lane].idx;
+            } else {
+                const int row = seq * (B + 1) + lane;
+                const float lse_p = rows[lane].m + logf(rows[lane].s);
+                const float p_y = expf(ld_any(p.target, p.dtype, (size_t)row * p.V + y) * invT - lse_p);
+                const float q_y = expf(p.logit_sel[(size_t)seq * B + lane] - p.lse[(size_t)seq * B + lane]);
+                const float u = uniform01(p.seed[seq], 0u, (uint32_t)lane, STREAM_ACCEPT, p.offset);
+                ok = u * q_y < p_y;
+            }
+        }
+        const unsigned rejected = __ballot_sync(0xffffffffu, lane < B && !ok);
+        const int n = rejected ? __ffs(rejected) - 1 : B;
+        if (c == 0) {
+            int32_t *out = p.out_tokens + (size_t)seq * (B + 1);
+            for (int k = lane; k <= B; k += 32) out[k] = k < n ? p.tokens[(size_t)seq * B + k] : -1;
+            __syncwarp();
+            if (lane == 0) {
+                if (!sampling) out[n] = rows[n].idx;
+                p.accept_len[seq] = n;
+            }
+        }
+        if (lane == 0) {
+            s_n = n;
+            s_lsep = (sampling && n < B) ? rows[n].m + logf(rows[n].s) : 0.0f;
         }
     }
-    const unsigned rejected = __ballot_sync(0xffffffffu, lane < B && !ok);
-    const int n = rejected ? __ffs(rejected) - 1 : B;
-    int32_t *out = p.out_tokens + (size_t)seq * (B + 1);
-    for (int k = lane; k <= B; k += 32) out[k] = k < n ? p.tokens[(size_t)seq * B + k] : -1;
-    __syncwarp();
-    if (lane == 0) {
-        if (!sampling) {
-            out[n] = rows[n].idx;
-            p.job[seq] = -1;
-        } else {
-            p.job[seq] = n;
-            if (n < B) p.jobf[seq] = rows[n].m + logf(rows[n].s);
-        }
-        p.accept_len[seq] = n;
-    }
-}
-
-// grid (b, chunks), 256 threads.  Writes two argmax partials per chunk: the
-// residual draw (best, idx) and the draw from p (m, s reused as score, idx).
-__global__ void __launch_bounds__(256) k_acc_sample(AcceptParams p)
-{
-    pdl_trigger();
-    pdl_wait();                                   // the decisions
-    const int seq = blockIdx.x, chunks = gridDim.y, c = blockIdx.y;
-    const int k = p.job[seq];
-    if (k < 0) return;
-    const int B = p.B;
-    const float invT = 1.0f / p.temperature[seq];
-    const int v0 = (int)((long long)p.V * c / chunks), v1 = (int)((long long)p.V * (c + 1) / chunks);
+    __syncthreads();
+    if (!sampling) return;
+    const int k = s_n;
+    const int v0 = (int)((long long)p.V * c / nch), v1 = (int)((long long)p.V * (c + 1) / nch);
     __shared__ float zop[RANK];
     const bool resid = k < B;
     if (resid)
@@ -171,7 +185,7 @@ __global__ void __launch_bounds__(256) k_acc_sample(AcceptParams p)
     __syncthreads();
     const unsigned long long seed = p.seed[seq];
     const size_t trow = (size_t)seq * (B + 1) + k;
-    const float lse_p = resid ? p.jobf[seq] : 0.0f;
+    const float lse_p = s_lsep;
     const float lse_q = resid ? p.lse[(size_t)seq * B + k] : 0.0f;
     float rb = -INFINITY, pb = -INFINITY;
     int ri = 0x7fffffff, pi = 0x7fffffff;
@@ -203,25 +217,25 @@ __global__ void __launch_bounds__(256) k_acc_sample(AcceptParams p)
             }
         __syncthreads();
     }
-    if (threadIdx.x == 0) p.spart[(size_t)seq * chunks + c] = Partial{sb[0][0], si[0][0], sb[1][0], __int_as_float(si[1][0])};
-}
-
-__global__ void k_acc_finish(AcceptParams p, int chunks)
-{
-    pdl_wait();                                   // the draw partials
-    const int seq = blockIdx.x * blockDim.x + threadIdx.x;
-    if (seq >= p.b) return;
-    const int k = p.job[seq];
-    if (k < 0) return;
-    float rb = -INFINITY, pb = -INFINITY;
-    int ri = 0x7fffffff, pi = 0x7fffffff;
-    for (int c = 0; c < chunks; ++c) {
-        const Partial a = p.spart[(size_t)seq * chunks + c];
-        merge_argmax(rb, ri, a.best, a.idx);
-        merge_argmax(pb, pi, a.m, __float_as_int(a.s));
+    if (threadIdx.x == 0) {
+        p.spart[(size_t)seq * nch + c] = Partial{sb[0][0], si[0][0], sb[1][0], __int_as_float(si[1][0])};
+        __threadfence();
+        s_last = atomicAdd(p.ticket + seq, 1) == nch - 1;
     }
-    const bool use_resid = k < p.B && rb > -INFINITY;
-    p.out_tokens[(size_t)seq * (p.B + 1) + k] = use_resid ? ri : pi;
+    __syncthreads();
+    if (s_last && threadIdx.x == 0) {
+        // every chunk of this block has drawn: combine and emit
+        __threadfence();
+        float cb = -INFINITY, cp = -INFINITY;
+        int ci = 0x7fffffff, cpi = 0x7fffffff;
+        for (int cc = 0; cc < nch; ++cc) {
+            const Partial a = ldcg_partial16(p.spart + (size_t)seq * nch + cc);
+            merge_argmax(cb, ci, a.best, a.idx);
+            merge_argmax(cp, cpi, a.m, __float_as_int(a.s));
+        }
+        const bool use_resid = k < B && cb > -INFINITY;
+        p.out_tokens[(size_t)seq * (B + 1) + k] = use_resid ? ci : cpi;
+    }
 }
 
 }  // namespace xp

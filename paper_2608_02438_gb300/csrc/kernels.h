@@ -17,8 +17,7 @@ struct AcceptParams {
     int32_t *accept_len, *out_tokens;
     int32_t *status;
     Partial *rowpart;   // [b * (B + 1), chunks]
-    int32_t *job;       // [b] position of the draw (-1: none, B: bonus)
-    float *jobf;        // [b] log-sum-exp of target / T at that position
+    int32_t *ticket;    // [b] draw chunks done (cleared by k_acc_rows)
     Partial *spart;     // [b, chunks]
 };
 
@@ -65,9 +64,7 @@ extern const size_t kPreTcSmemBytes;
 
 // accept_kernels.cu
 __global__ void k_acc_rows(AcceptParams p);
-__global__ void k_acc_decide(AcceptParams p, int chunks);
-__global__ void k_acc_sample(AcceptParams p);
-__global__ void k_acc_finish(AcceptParams p, int chunks);
+__global__ void k_acc_finalize(AcceptParams p, int chunks);
 
 // fp32: c and sigma(W_1 c) of up to 32 tokens in fp32; bf16: the same as
 // bf16 tensor-core operands plus this CTA's share of sigma(W_1 c)

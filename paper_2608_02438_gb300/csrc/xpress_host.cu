@@ -849,7 +849,7 @@ int xpress_refine_block(const xpress_refiner *Rc, const xpress_block_in *in, con
 
 namespace {
 struct AcceptLayout {
-    size_t status = 0, rowpart = 256, job = 0, jobf = 0, spart = 0, total = 0;
+    size_t status = 0, rowpart = 256, ticket = 0, spart = 0, total = 0;
     int chunks = 1, chunks2 = 1;
 };
 
@@ -862,9 +862,7 @@ AcceptLayout accept_layout(const xpress_refiner *R, int b)
     int c2 = (2 * R->num_sms + b - 1) / b;
     A.chunks2 = c2 < 1 ? 1 : (c2 > 512 ? 512 : c2);
     size_t o = A.rowpart + align256((size_t)rows * A.chunks * sizeof(Partial));
-    A.job = o;
-    o += align256((size_t)b * 4);
-    A.jobf = o;
+    A.ticket = o;
     o += align256((size_t)b * 4);
     A.spart = o;
     o += align256((size_t)b * A.chunks2 * sizeof(Partial));
@@ -912,16 +910,13 @@ int accept_launch(const xpress_refiner *R, const xpress_accept_in *in, int32_t *
     P.out_tokens = out_tokens;
     P.status = reinterpret_cast<int32_t *>(w + A.status);
     P.rowpart = reinterpret_cast<Partial *>(w + A.rowpart);
-    P.job = reinterpret_cast<int32_t *>(w + A.job);
-    P.jobf = reinterpret_cast<float *>(w + A.jobf);
+    P.ticket = reinterpret_cast<int32_t *>(w + A.ticket);
     P.spart = reinterpret_cast<Partial *>(w + A.spart);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    // all four are chained to their predecessor with programmatic dependent
-    // launch (k_acc_rows clears the status word)
+    // both are chained to their predecessor with programmatic dependent
+    // launch (k_acc_rows clears the status word and the draw tickets)
     XP_CUDA(launch_pdl(k_acc_rows, dim3(in->b * (R->w.B + 1), A.chunks), dim3(256), 0, st, P));
-    XP_CUDA(launch_pdl(k_acc_decide, dim3(in->b), dim3(32), 0, st, P, A.chunks));
-    XP_CUDA(launch_pdl(k_acc_sample, dim3(in->b, A.chunks2), dim3(256), 0, st, P));
-    XP_CUDA(launch_pdl(k_acc_finish, dim3((in->b + 127) / 128), dim3(128), 0, st, P, A.chunks2));
+    XP_CUDA(launch_pdl(k_acc_finalize, dim3(in->b, A.chunks2), dim3(256), 0, st, P, A.chunks));
     XP_CUDA(cudaGetLastError());
     return XPRESS_OK;
 }
