@@ -80,8 +80,7 @@ struct alignas(128) CtlLine {
     unsigned pad[31];
 };
 struct SmallCtl {
-    CtlLine pre_done;    // Read CTAs done with the precompute
-    CtlLine pc_ready;    // Trans CTAs that published their slice of Pc (8 per call)
+    CtlLine pre_done;    // Read CTAs done with the precompute (Pc and the first c)
     CtlLine c_ready;     // Trans CTAs that published their slice of c (8 per pass)
     CtlLine u_ready;     // ... of sigma(W_1 c)
     CtlLine z_ready;     // ... of z
@@ -129,10 +128,11 @@ struct Params {
     float *zbuf;                 // [N, r] fp32 z when the caller passes no z_final
     RPartial *part;              // [N, S] token-major (a token's ranges are contiguous)
     // persistent small-batch kernel only
-    const float *Fhg;            // [2r, H] fp32: rows W_in[:, 0:r] W_h, then W_in[:, r:2r] W_g
-    int pre_kslice, pre_ks;      // K-slice width of the hidden projection and the number of slices
+    const uint16_t *Fhl;         // [2][2r, H] bf16: hi then lo term of the fp32 rows W_in[:, 0:r] W_h,
+                                 // then W_in[:, r:2r] W_g (hi + lo carries about 16 significant bits)
+    float *c0x;                  // [32, r] c of the first pass (with a draft), fp32
     uint16_t *cx, *ux;           // [32, r] c and [32, 2r] sigma(W_1 c), bf16, exchanged by the Trans CTAs
-    float *pcx;                  // [32, r] Pc, fp32, exchanged once per call (blocks of at most 16)
+    float *pcx;                  // [32, r] Pc = (I + L) P, fp32
     const uint16_t *Lpk;         // [B(B-1)/2, r] bf16: L's strictly lower part, row q = k(k-1)/2 + j
     Partial *rmax;               // [N, RMAX_SEG] argmax-s partials (calls without a draft)
     SmallCtlArea *sctl;          // control blocks of the persistent kernel
@@ -518,6 +518,15 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volati
 __device__ __forceinline__ void fence_barrier_init()
 {
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+// Untiled bulk copy global -> shared memory, completing on `bar` (both
+// addresses 16-byte aligned, bytes a multiple of 16).
+__device__ __forceinline__ void bulk_load_1d(void *smem_dst, const void *src, uint32_t bytes, uint64_t *bar)
+{
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 ::"r"(smem_u32(smem_dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar))
+                 : "memory");
 }
 
 __device__ __forceinline__ void tma_load_2d(void *smem_dst, const CUtensorMap *map, uint64_t *bar, int x, int y)

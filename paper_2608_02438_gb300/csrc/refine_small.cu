@@ -48,6 +48,7 @@ struct RsShared {                              // Read CTA, after the W_r stages
     uint64_t z_full, z_empty, go;
     uint64_t tfull[TV_NBUF], tempty[TV_NBUF];
     uint64_t drain;
+    uint64_t pfull[3], pempty[3];              // precompute ring (h and F chunks)
     uint32_t tmem_base;
     int abort;
     int pass_n, pass_stop;                     // published by the producer with `go`
@@ -132,102 +133,174 @@ __device__ __forceinline__ void leave(const Params &p, SmallCtlArea *a, SmallCtl
 }
 
 // ------------------------------------------------------------- precompute
-
-// Sum over the 32 lanes of v[0..NT-1] (NT = 16 or 32 token slots); lane t
-// (t < NT) ends with the total of slot t.
+//
+// Read CTAs, before the first pass: the token-independent part of Fuse and
+// Mix for pairs of channels, unit u -> channels d0 = 2u, d0 + 1 (128 units).
+//   U[t][o] = sum_k h[t][k] F[o][k] over all of K for the unit's four rows o
+//   (the h slot W_in[:, 0:r] W_h and the g slot W_in[:, r:2r] W_g of both
+//   channels), on tensor cores: F as two bf16 terms (hi + lo, so that the
+//   products with the bf16 h are exact and only the fp32 sums round);
+//   P_k = U_h,k + (1/B) sum_j U_g,j (the g slot is the block mean), and
+//   Pc_k = P_k + sum_{j<k} L_kj P_j (Eq. mix, per channel), written to pcx;
+//   with a draft also the first pass's c_k = Pc_k + e_k + sum_{j<k} L_kj e_j
+//   (e_k = E'[x_{k-1}], Eq. fuse / mix), written to c0x.
+// K is streamed through a 3-buffer ring of bulk copies (warp 0 issues them):
+// per chunk the unit's 8 F rows ([lo][slot h / g][channel]) and the N rows of
+// h, each row at a pitch of 64 mod 128 bytes so that the fragment loads below
+// hit distinct banks.
+constexpr int PC_BUFS = 3;
+constexpr int PC_ROWS = 8;
 template <int NT>
-__device__ __forceinline__ float reduce_scatter_n(float (&v)[NT], int lane)
+struct PcShape {
+    static constexpr int KC = NT <= 16 ? 768 : 512;          // K per chunk (a multiple of 8 warps x 32)
+    static constexpr int PITCH = 2 * KC + 64;                // bytes per row
+    static constexpr int BUF = (PC_ROWS + NT) * PITCH;
+};
+static_assert(PC_BUFS * PcShape<16>::BUF <= (int)(TV_STAGES * TV_A_STAGE + TV_Z_BYTES), "precompute ring");
+static_assert(PC_BUFS * PcShape<32>::BUF <= (int)(TV_STAGES * TV_A_STAGE + TV_Z_BYTES), "precompute ring");
+
+// Warp 0, one lane: the chunk copies of every unit of this CTA.
+template <int NT>
+__device__ __forceinline__ void pc_produce(const Params &p, uint8_t *ring, RsShared &sh, int r, int S,
+                                           volatile int *abort)
 {
-#pragma unroll
-    for (int s = NT / 2; s >= 1; s >>= 1) {
-        const bool upper = (lane & s) != 0;
-#pragma unroll
-        for (int j = 0; j < s; ++j) {
-            const float send = upper ? v[j] : v[j + s];
-            const float keep = upper ? v[j + s] : v[j];
-            v[j] = keep + __shfl_xor_sync(0xffffffffu, send, s);
+    using Sh = PcShape<NT>;
+    const int H = p.H, N = p.N, nchk = (H + Sh::KC - 1) / Sh::KC;
+    const uint16_t *h = static_cast<const uint16_t *>(p.h);
+    const size_t lo_off = (size_t)2 * RANK * H;
+    uint32_t pending = 0, pend_par = 0;
+    int ci = 0;
+    bool ok = true;
+    for (int unit = r; unit < RANK / 2 && ok; unit += S)
+        for (int kc = 0; kc < nchk; ++kc, ++ci) {
+            const int buf = ci % PC_BUFS;
+            const uint32_t ph = (uint32_t)((ci / PC_BUFS) & 1);
+            if (!mbar_wait(&sh.pempty[buf], ph ^ 1, abort)) { ok = false; break; }
+            const int kb = kc * Sh::KC, kl = min(Sh::KC, H - kb);
+            const uint32_t bytes = (uint32_t)kl * 2;
+            uint8_t *dst = ring + buf * Sh::BUF;
+            mbar_expect_tx(&sh.pfull[buf], bytes * (uint32_t)(PC_ROWS + N));
+            for (int m = 0; m < PC_ROWS; ++m) {
+                const int lo = m >> 2, slot = (m >> 1) & 1, ch = m & 1;
+                bulk_load_1d(dst + m * Sh::PITCH, p.Fhl + lo * lo_off + (size_t)(slot * RANK + 2 * unit + ch) * H + kb,
+                             bytes, &sh.pfull[buf]);
+            }
+            for (int t = 0; t < N; ++t)
+                bulk_load_1d(dst + (PC_ROWS + t) * Sh::PITCH, h + (size_t)t * H + kb, bytes, &sh.pfull[buf]);
+            pending |= 1u << buf;
+            pend_par = (pend_par & ~(1u << buf)) | (ph << buf);
         }
-    }
-    float r = v[0];
-#pragma unroll
-    for (int s = NT; s < 32; s <<= 1) r += __shfl_xor_sync(0xffffffffu, r, s);
-    return r;
+    // no copy may still be landing when the ring is reused
+    int dummy = 0;
+    for (int b2 = 0; b2 < PC_BUFS; ++b2)
+        if (pending & (1u << b2)) mbar_wait(&sh.pfull[b2], (pend_par >> b2) & 1, &dummy, 100000000ull);
 }
 
-// Work item of the hidden projection: Upart[ks][t][o] = sum over K-slice ks of
-// F[o][k] h[t][k] for the 8 R rows o of row group rg (warp w: R rows).  h's
-// slice is staged in `hs` (bf16 [N][pre_kslice]).  The 8 epilogue warps call
-// this together.
+// The 8 epilogue warps (w = 0..7): per unit, warp w takes the 32-wide K steps
+// w, w + 8, ... of every chunk (m16n8k16: A = the unit's F rows, hi in rows
+// 0-7 and lo in rows 8-15, B = h, tokens in 8-column tiles).  The 16 K values
+// of one product are taken from 32 consecutive ones, the same for A and B, so
+// each operand is one 16-byte load per lane.
 template <int NT>
-__device__ __forceinline__ void pre_item(const Params &p, int item, uint16_t *hs, int w, int lane)
+__device__ __forceinline__ void pc_consume(const Params &p, uint8_t *ring, RsShared &sh, int r, int S, int w,
+                                           int lane, volatile int *abort, bool tm, unsigned long long t_start)
 {
-    constexpr int R = 64 / NT, ROWS = 8 * R, NG = 2 * RANK / ROWS;
-    const int rg = item % NG, ks = item / NG;
-    const int N = p.N, H = p.H, pitch = p.pre_kslice;
-    const int kb = ks * pitch, kl = min(H, kb + pitch) - kb;
-    const uint16_t *h = static_cast<const uint16_t *>(p.h);
-    {
-        const int per = kl / 8, total = N * per, tid = w * 32 + lane;
-        for (int i0 = 0; i0 < total; i0 += 8 * 256) {
-            uint4 v[8];
-#pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                const int i = i0 + q * 256 + tid;
-                if (i < total) v[q] = __ldg(reinterpret_cast<const uint4 *>(h + (size_t)(i / per) * H + kb) + i % per);
-            }
-#pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                const int i = i0 + q * 256 + tid;
-                if (i < total) reinterpret_cast<uint4 *>(hs + (size_t)(i / per) * pitch)[i % per] = v[q];
-            }
+    using Sh = PcShape<NT>;
+    const int H = p.H, N = p.N, B = p.B, V = p.V, nchk = (H + Sh::KC - 1) / Sh::KC;
+    const int g = lane >> 2, tq = lane & 3, et = w * 32 + lane;
+    const int TRI = B * (B - 1) / 2;
+    float *us = &sh.bestx[0][0][0];                               // U [4][32]: rows (slot, channel)
+    float2 *es = reinterpret_cast<float2 *>(us + 4 * 32);         // E' entries of the first pass [32]
+    uint32_t *ls = reinterpret_cast<uint32_t *>(es + 32);         // L pairs [B(B-1)/2] (both channels)
+    int ci = 0;
+    bool ok = true;
+    for (int unit = r; unit < RANK / 2; unit += S) {
+        const int d0 = 2 * unit;
+        // L of the two channels and the first pass's E' entries (latency
+        // overlapped with the first chunk's copies)
+        for (int q = et; q < TRI; q += 256) ls[q] = __ldg(reinterpret_cast<const uint32_t *>(p.Lpk + (size_t)q * RANK + d0));
+        if (p.draft && et < N) {
+            const int s = et / B, k = et % B;
+            int tk = k == 0 ? p.anchor[s] : p.draft[et - 1];
+            if (tk < 0 || tk >= V) tk = 0;                        // reported by the Trans CTAs
+            es[et] = __ldg(reinterpret_cast<const float2 *>(p.Ep + (size_t)tk * RANK + d0));
         }
-    }
-    tv_epi_bar();
-    const int row0 = rg * ROWS + w * R;
-    const float *F = p.Fhg + (size_t)row0 * H + kb;
-    float acc[R][NT];
+        float acc[NT / 8][4];
 #pragma unroll
-    for (int r = 0; r < R; ++r)
+        for (int nt = 0; nt < NT / 8; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.0f;
+        for (int kc = 0; kc < nchk; ++kc, ++ci) {
+            const int buf = ci % PC_BUFS;
+            if (ok && !mbar_wait(&sh.pfull[buf], (uint32_t)((ci / PC_BUFS) & 1), abort)) ok = false;
+            if (ok) {
+                if (tm && kc == 0) trace_mark(p.trace, 5, t_start);
+                const int kl = min(Sh::KC, H - kc * Sh::KC);
+                const uint8_t *fb = ring + buf * Sh::BUF;
+                const uint8_t *fhi = fb + (g & 3) * Sh::PITCH, *flo = fb + (4 + (g & 3)) * Sh::PITCH;
+                const uint8_t *hr = fb + (PC_ROWS + g) * Sh::PITCH;
+#pragma unroll 1
+                for (int ks = w; ks * 32 < kl; ks += 8) {
+                    const int ko = ks * 32 + 8 * tq;
+                    const bool v = ko < kl;
+                    const uint4 z4 = make_uint4(0u, 0u, 0u, 0u);
+                    const uint4 ah = v ? *reinterpret_cast<const uint4 *>(fhi + 2 * ko) : z4;
+                    const uint4 al = v ? *reinterpret_cast<const uint4 *>(flo + 2 * ko) : z4;
+                    const uint32_t a0[4] = {ah.x, al.x, ah.y, al.y}, a1[4] = {ah.z, al.z, ah.w, al.w};
 #pragma unroll
-        for (int t = 0; t < NT; ++t) acc[r][t] = 0.0f;
-    for (int c0 = 0; c0 < kl; c0 += 512) {
-        float4 wv[R][4];
-#pragma unroll
-        for (int r = 0; r < R; ++r)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int k = c0 + 128 * i + 4 * lane;
-                wv[r][i] = k < kl ? __ldg(reinterpret_cast<const float4 *>(F + (size_t)r * H + k))
-                                  : make_float4(0.f, 0.f, 0.f, 0.f);
-            }
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const int k = c0 + 128 * i + 4 * lane;
-            if (k >= kl) continue;
-#pragma unroll
-            for (int t = 0; t < NT; ++t) {
-                if (t >= N) continue;
-                const uint2 hv = *reinterpret_cast<const uint2 *>(hs + (size_t)t * pitch + k);
-                const float h0 = __uint_as_float(hv.x << 16), h1 = __uint_as_float(hv.x & 0xFFFF0000u);
-                const float h2 = __uint_as_float(hv.y << 16), h3 = __uint_as_float(hv.y & 0xFFFF0000u);
-#pragma unroll
-                for (int r = 0; r < R; ++r) {
-                    float a = acc[r][t];
-                    a = fmaf(wv[r][i].x, h0, a);
-                    a = fmaf(wv[r][i].y, h1, a);
-                    a = fmaf(wv[r][i].z, h2, a);
-                    a = fmaf(wv[r][i].w, h3, a);
-                    acc[r][t] = a;
+                    for (int nt = 0; nt < NT / 8; ++nt) {
+                        const uint4 bb = (v && nt * 8 + g < N)
+                                             ? *reinterpret_cast<const uint4 *>(hr + nt * 8 * Sh::PITCH + 2 * ko)
+                                             : z4;
+                        mma_bf16_16816(acc[nt], a0, bb.x, bb.y);
+                        mma_bf16_16816(acc[nt], a1, bb.z, bb.w);
+                    }
                 }
             }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sh.pempty[buf]);
         }
-    }
+        if (tm && unit == r) trace_mark(p.trace, 6, t_start);
+        // the 8 warps' sums (row g < 4: hi + lo of row (slot g / 2, channel g % 2))
+        if (g < 4)
 #pragma unroll
-    for (int r = 0; r < R; ++r) {
-        const float s = reduce_scatter_n<NT>(acc[r], lane);
-        if (lane < N) p.Upart[((size_t)ks * N + lane) * 2 * RANK + row0 + r] = s;
+            for (int nt = 0; nt < NT / 8; ++nt) {
+                const int t0 = nt * 8 + 2 * tq;
+                sh.tile[w][t0][g] = acc[nt][0] + acc[nt][2];
+                sh.tile[w][t0 + 1][g] = acc[nt][1] + acc[nt][3];
+            }
+        tv_epi_bar();
+        if (et < 4 * N) {
+            const int t = et >> 2, row = et & 3;
+            float u = 0.0f;
+#pragma unroll
+            for (int w2 = 0; w2 < TV_EPI_WARPS; ++w2) u += sh.tile[w2][t][row];
+            us[row * 32 + t] = u;
+        }
+        tv_epi_bar();
+        if (ok && et < 2 * N) {
+            const int t = et >> 1, ch = et & 1, s = t / B, k = t % B;
+            const float *uh = us + ch * 32 + s * B, *ug = us + (2 + ch) * 32 + s * B;
+            float gs = 0.0f;
+            for (int j = 0; j < B; ++j) gs += ug[j];
+            const float gm = gs / (float)B;
+            const int lrow = k * (k - 1) / 2;
+            float a = uh[k] + gm;
+            for (int j = 0; j < k; ++j) {
+                const uint32_t lw = ls[lrow + j];
+                a = fmaf(__uint_as_float(ch ? (lw & 0xFFFF0000u) : (lw << 16)), uh[j] + gm, a);
+            }
+            p.pcx[(size_t)t * RANK + d0 + ch] = a;
+            if (p.draft) {
+                const float2 *eb = es + s * B;
+                float m = ch ? eb[k].y : eb[k].x;
+                for (int j = 0; j < k; ++j) {
+                    const uint32_t lw = ls[lrow + j];
+                    m = fmaf(__uint_as_float(ch ? (lw & 0xFFFF0000u) : (lw << 16)), ch ? eb[j].y : eb[j].x, m);
+                }
+                p.c0x[(size_t)t * RANK + d0 + ch] = a + m;
+            }
+        }
+        tv_epi_bar();                                             // tile, us, es and ls are reused
     }
-    tv_epi_bar();                              // hs is restaged by the next item
 }
 
 // Partial argmax of s[t, segment] (fp32 compare of the bf16 values, smallest
@@ -277,6 +350,7 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
         mbar_init(&sh.go, 1);
         for (int i = 0; i < TV_NBUF; ++i) { mbar_init(&sh.tfull[i], 1); mbar_init(&sh.tempty[i], 4); }
         mbar_init(&sh.drain, 1);
+        for (int i = 0; i < PC_BUFS; ++i) { mbar_init(&sh.pfull[i], 1); mbar_init(&sh.pempty[i], TV_EPI_WARPS); }
         sh.abort = 0;
         fence_barrier_init();
     }
@@ -292,27 +366,33 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
     const uint32_t tmem = sh.tmem_base;
     volatile int *abort = &sh.abort;
 
-    // ---- precompute (epilogue warps), h slices staged in the W_r stages
-    if (warp >= 2) {
-        const int w = warp - 2;
-        const int ng = N <= 16 ? 16 : 32;                  // row groups (8 R rows each, R = 64 / NT)
-        const int items = ng * p.pre_ks;
-        uint16_t *hs = reinterpret_cast<uint16_t *>(sA);
-        for (int item = r; item < items; item += S) {
-            if (N <= 16) pre_item<16>(p, item, hs, w, lane);
-            else pre_item<32>(p, item, hs, w, lane);
+    // ---- precompute: Pc (and the first pass's c) for this CTA's channel
+    // pairs, through a ring in the W_r stages; without a draft also partial
+    // argmaxes of s
+    if (warp == 0) {
+        if (lane == 0) {
+            if (N <= 16) pc_produce<16>(p, sA, sh, r, S, abort);
+            else pc_produce<32>(p, sA, sh, r, S, abort);
         }
+    } else if (warp >= 2) {
+        const int w = warp - 2;
+        const bool tm = tr && w == 0 && lane == 0;
+        if (tm) trace_mark(p.trace, 4, t_start);
+        if (N <= 16) pc_consume<16>(p, sA, sh, r, S, w, lane, abort, tm, t_start);
+        else pc_consume<32>(p, sA, sh, r, S, w, lane, abort, tm, t_start);
         if (!p.draft)
             for (int item = r * TV_EPI_WARPS + w; item < N * RMAX_SEG; item += S * TV_EPI_WARPS)
                 rowmax_item(p, item, lane);
+        if (tm) trace_mark(p.trace, 7, t_start);
     }
     __syncthreads();
     // (release: the other threads' writes precede it through the barrier)
     if (threadIdx.x == 0) {
-        red_add_release_gpu(&c->pre_done.v, 1u);
+        if (sh.abort) raise_stop(c, ST_TIMEOUT);
+        else red_add_release_gpu(&c->pre_done.v, 1u);
         if (tr) trace_mark(p.trace, 2, t_start);
-        // this CTA's W_r range into L2 while Pc and the first Trans run (after
-        // the precompute, whose reads it would otherwise slow down)
+        // this CTA's W_r range into L2 while the first Trans runs (after the
+        // precompute, whose reads it would otherwise slow down)
         if (!(p.read_flags & 1)) {
             const char *wr = static_cast<const char *>(p.W_r);
             const int rows = min(vb1 * TV_BM, V) - vb0 * TV_BM;
@@ -511,6 +591,10 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
                 }
                 if (my_invT > 0.0f) p.part[(size_t)lane * S + r] = a;
                 else atomicMax(p.best64 + 32 * (pass & 1) + lane, argmax_key(a.best, a.idx));   // greedy: one key
+                // this range's candidate for the token: its E' row into L2 for
+                // the next pass's gather (the winner is one of the candidates)
+                const int cand = my_invT > 0.0f ? a.y : a.idx;
+                if (cand >= 0 && cand < V) prefetch_l2_bulk(p.Ep + (size_t)cand * RANK, RANK * 4);
             }
             tv_epi_bar();
             // partials of this range are written: the Trans CTAs end the pass
@@ -607,37 +691,11 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
         const float T = p.temperature[tid];
         sh.invT[tid] = T > 0.0f ? 1.0f / T : 0.0f;
     }
-    // with a draft, pass 0's tokens are known now: gather its E' rows while
-    // the Read CTAs run the precompute
-    float *mixe = reinterpret_cast<float *>(uop);             // [32][RANK] fp32 (full mode, pass 0 only)
-    if (p.draft) {
-        __syncthreads();
-        gather_e(p, sh.x, e, CH, cb, tid, nth);
-        if (full) {
-            // the token part of pass 0's Mix, e_k + sum_{j<k} L_kj e_j, while
-            // the Read CTAs run the precompute (uop is free until W_1)
-            __syncthreads();
-            const int dd = tid;
-            if (dd < RANK)
-                for (int s = 0; s < b; ++s) {
-                    float er[FULL_C_MAX_B];
-#pragma unroll
-                    for (int j2 = 0; j2 < FULL_C_MAX_B; ++j2) er[j2] = j2 < B ? e[(s * B + j2) * CH + dd] : 0.0f;
-#pragma unroll 1
-                    for (int k = 0; k < B; ++k) {
-                        float a = e[(s * B + k) * CH + dd];
-                        const uint16_t *lrow = Lp + (k * (k - 1) / 2) * CH + dd;
-#pragma unroll
-                        for (int j2 = 0; j2 < FULL_C_MAX_B - 1; ++j2)
-                            if (j2 < k) a = fmaf(bf2f(lrow[j2 * CH]), er[j2], a);
-                        mixe[(s * B + k) * CH + dd] = a;
-                    }
-                }
-        }
-    }
+    if (lead && tid == 0 && p.trace) trace_mark(p.trace, 250, t_start);
     if (tid == 0) sh.go = wait_count(c, &c->pre_done.v, (unsigned)p.S);
     __syncthreads();
     if (!sh.go) return;
+    if (lead && tid == 0 && p.trace) trace_mark(p.trace, 251, t_start);
     if (!p.draft) {
         // Y^(0) = argmax s (Algorithm 1), from the Read CTAs' partials
         for (int t = warp; t < N; t += nth / 32) {
@@ -657,55 +715,12 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
             }
         }
     }
-    // Pc = (I + L) P for the own channels (Eq. mix); P_k = F_h h_k + mean_j F_g h_j
-    {
-        float(*P)[32] = sh.cown;                               // scratch until the first pass
-        float(*G)[32] = sh.zhalf[0];
-        float(*Q)[32] = sh.zhalf[1];
-        const int ks = p.pre_ks;
-        for (int i = tid; i < N * 32; i += nth) {
-            const int t = i / 32, dd = i % 32;
-            const float *u = p.Upart + (size_t)t * 2 * RANK + d0 + dd;
-            float a = 0.0f, gsum = 0.0f;
-#pragma unroll 4
-            for (int z = 0; z < ks; ++z) {
-                a += __ldcg(u + (size_t)z * N * 2 * RANK);
-                gsum += __ldcg(u + (size_t)z * N * 2 * RANK + RANK);
-            }
-            P[t][dd] = a;
-            G[t][dd] = gsum;
-        }
-        __syncthreads();
-        for (int i = tid; i < N * 32; i += nth) {
-            const int t = i / 32, dd = i % 32, s = t / B;
-            float gs = 0.0f;
-            for (int k = 0; k < B; ++k) gs += G[s * B + k][dd];
-            Q[t][dd] = P[t][dd] + gs / (float)B;               // P, complete
-        }
-        __syncthreads();
-        const int lb = full ? d0 : 0;                          // own channels within the kept ones
-        for (int i = tid; i < N * 32; i += nth) {
-            const int t = i / 32, dd = i % 32, s = t / B, k = t % B;
-            float a = Q[t][dd];
-            for (int j2 = 0; j2 < k; ++j2)
-                a = fmaf(bf2f(Lp[(k * (k - 1) / 2 + j2) * CH + lb + dd]), Q[s * B + j2][dd], a);
-            if (full) p.pcx[(size_t)t * RANK + d0 + dd] = a;
-            else pc[t * CH + dd] = a;
-        }
-        __syncthreads();
-        if (full) {
-            // every Trans CTA needs Pc for all channels: one exchange per call
-            if (tid == 0) {
-                red_add_release_gpu(&c->pc_ready.v, 1u);
-                sh.go = wait_count(c, &c->pc_ready.v, 8u);
-            }
-            __syncthreads();
-            if (!sh.go) return;
-            for (int i = tid; i < N * RANK / 4; i += nth)
-                reinterpret_cast<float4 *>(pc)[i] = __ldcg(reinterpret_cast<const float4 *>(p.pcx) + i);
-            __syncthreads();
-        }
+    // Pc = (I + L) P (Eq. mix) of the kept channels, from the Read CTAs
+    for (int i = tid; i < N * CH / 4; i += nth) {
+        const int t = i / (CH / 4), q = i % (CH / 4);
+        reinterpret_cast<float4 *>(pc)[i] = __ldcg(reinterpret_cast<const float4 *>(p.pcx + (size_t)t * RANK + cb) + q);
     }
+    __syncthreads();
     if (lead && tid == 0 && p.trace) trace_mark(p.trace, 3, t_start);
 
     float *zf = p.z_final ? p.z_final : p.zbuf;
@@ -715,42 +730,67 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
         const unsigned long long t_pass = globaltimer_ns();
         const int trs = (lead && tid == 0 && p.trace && pass < 3) ? 210 + 8 * pass : 0;
         if (trs) trace_mark(p.trace, trs, t_pass);
-        if (pass > 0 || !p.draft) {
+        const bool first_c = pass == 0 && p.draft;             // c formed by the Read CTAs
+        if (!first_c) {
             gather_e(p, sh.x, e, CH, cb, tid, nth);
             __syncthreads();
         }
         if (trs) trace_mark(p.trace, trs + 1, t_pass);
         // Mix for the evaluated tokens; c enters W_1 rounded to bf16.
-        if (full) {
-            // thread = channel; a block's E' values sit in registers and both
-            // loops are unrolled (B <= 16), predicated on the block's frontier
-            const int dd = tid;
-            const bool pre_mixed = pass == 0 && p.draft;       // e_k + sum_j L e_j formed during the precompute
-            if (dd < RANK)
+        if (first_c) {
+            for (int i = tid; i < n * (RANK / 4); i += nth) {
+                const int t = i / (RANK / 4), q = i % (RANK / 4);
+                const float4 v = __ldcg(reinterpret_cast<const float4 *>(p.c0x + (size_t)t * RANK) + q);
+                *reinterpret_cast<uint2 *>(cop + t * COP_LD + 4 * q) =
+                    make_uint2((uint32_t)f2bf(v.x) | ((uint32_t)f2bf(v.y) << 16),
+                               (uint32_t)f2bf(v.z) | ((uint32_t)f2bf(v.w) << 16));
+                if ((q >> 3) == rank) *reinterpret_cast<float4 *>(&sh.cown[t][4 * (q & 7)]) = v;
+            }
+            for (int i = tid; i < ((n + 15) / 16 * 16 - n) * RANK; i += nth)
+                cop[(n + i / RANK) * COP_LD + i % RANK] = 0;
+            __syncthreads();
+            if (trs) trace_mark(p.trace, trs + 2, t_pass);
+        } else if (full) {
+            // thread (channel pair 2 cp, 2 cp + 1; half kh of the positions,
+            // dealt ABBA from the last one so that both halves get about the
+            // same number of L terms): a block's E' values sit in registers,
+            // the j loop is unrolled (B <= 16) and predicated on k, and two
+            // partial sums per channel shorten the dependency chains
+            const int cp = tid & 127, kh = tid >> 7, d = 2 * cp;
+            if (kh < 2)
                 for (int s = 0; s < b; ++s) {
                     const SeqState st = sh.st[s];
                     if (!st.active) continue;
-                    float er[FULL_C_MAX_B];
+                    float2 er[FULL_C_MAX_B];
 #pragma unroll
-                    for (int j2 = 0; j2 < FULL_C_MAX_B; ++j2) er[j2] = j2 < B ? e[(s * B + j2) * CH + dd] : 0.0f;
-                    // k rolled (short code: the first pass runs it cold), j unrolled
-                    // so that er stays in registers
+                    for (int j2 = 0; j2 < FULL_C_MAX_B; ++j2)
+                        er[j2] = j2 < B ? *reinterpret_cast<const float2 *>(e + (s * B + j2) * CH + d)
+                                        : make_float2(0.0f, 0.0f);
 #pragma unroll 1
                     for (int k = st.m + 1; k < B; ++k) {
+                        if ((((B - 1 - k + 1) >> 1) & 1) != kh) continue;
                         const int t = st.off + k - st.m - 1;
-                        float a;
-                        if (pre_mixed) {
-                            a = mixe[(s * B + k) * CH + dd];
-                        } else {
-                            a = e[(s * B + k) * CH + dd];
-                            const uint16_t *lrow = Lp + (k * (k - 1) / 2) * CH + dd;
+                        float2 a0 = *reinterpret_cast<const float2 *>(e + (s * B + k) * CH + d);
+                        float2 a1 = make_float2(0.0f, 0.0f);
+                        const uint32_t *lrow = reinterpret_cast<const uint32_t *>(Lp + (k * (k - 1) / 2) * CH + d);
 #pragma unroll
-                            for (int j2 = 0; j2 < FULL_C_MAX_B - 1; ++j2)
-                                if (j2 < k) a = fmaf(bf2f(lrow[j2 * CH]), er[j2], a);
-                        }
-                        a = pc[(s * B + k) * CH + dd] + a;
-                        cop[t * COP_LD + dd] = f2bf(a);
-                        if ((dd >> 5) == rank) sh.cown[t][dd & 31] = a;
+                        for (int j2 = 0; j2 < FULL_C_MAX_B - 1; ++j2)
+                            if (j2 < k) {
+                                const uint32_t lw = lrow[j2 * (CH / 2)];
+                                const float lx = __uint_as_float(lw << 16), ly = __uint_as_float(lw & 0xFFFF0000u);
+                                if (j2 & 1) {
+                                    a1.x = fmaf(lx, er[j2].x, a1.x);
+                                    a1.y = fmaf(ly, er[j2].y, a1.y);
+                                } else {
+                                    a0.x = fmaf(lx, er[j2].x, a0.x);
+                                    a0.y = fmaf(ly, er[j2].y, a0.y);
+                                }
+                            }
+                        const float2 pcv = *reinterpret_cast<const float2 *>(pc + (s * B + k) * CH + d);
+                        const float cx0 = pcv.x + (a0.x + a1.x), cx1 = pcv.y + (a0.y + a1.y);
+                        *reinterpret_cast<uint32_t *>(cop + t * COP_LD + d) =
+                            (uint32_t)f2bf(cx0) | ((uint32_t)f2bf(cx1) << 16);
+                        if ((d >> 5) == rank) *reinterpret_cast<float2 *>(&sh.cown[t][d & 31]) = make_float2(cx0, cx1);
                     }
                 }
         } else {
@@ -769,7 +809,8 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
                     p.cx[(size_t)t * RANK + d0 + dd] = f2bf(a);
                 }
         }
-        if (full) {
+        if (first_c) {
+        } else if (full) {
             // rows past n of the last 16-row tile: zero operands
             for (int i = tid; i < ((n + 15) / 16 * 16 - n) * RANK; i += nth)
                 cop[(n + i / RANK) * COP_LD + i % RANK] = 0;
@@ -779,7 +820,7 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
             __syncthreads();
             if (tid == 0) {
                 red_add_release_gpu(&c->c_ready.v, 1u);
-                sh.go = wait_count(c, &c->c_ready.v, (unsigned)(8 * (pass + 1)));
+                sh.go = wait_count(c, &c->c_ready.v, (unsigned)(8 * (pass + (p.draft ? 0 : 1))));
                 if (trs) trace_mark(p.trace, trs + 2, t_pass);
             }
             __syncthreads();
@@ -998,11 +1039,13 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
     if (threadIdx.x == 0) leave(p, area, c, par);
 }
 
-// Folded hidden projection (Fuse is linear): Fhg[o][i] = sum_e W_in[o][e] W_h[e][i]
-// for o < r and sum_e W_in[o - r][r + e] W_g[e][i] for o >= r, fp32 accumulation.
+// Folded hidden projection (Fuse is linear): F[o][i] = sum_e W_in[o][e] W_h[e][i]
+// for o < r and sum_e W_in[o - r][r + e] W_g[e][i] for o >= r, fp32 accumulation,
+// stored as two bf16 terms: Fhl[0] = hi = bf16(F), Fhl[1] = lo = bf16(F - hi)
+// (F - hi is exact in fp32; hi + lo is F to about 2^-17 relative).
 // grid (ceil(H / 256), 2r / 8), 256 threads.
 __global__ void __launch_bounds__(256) k_fold_hidden(const uint16_t *W_h, const uint16_t *W_g, const uint16_t *W_in,
-                                                     float *Fhg, int H)
+                                                     uint16_t *Fhl, int H)
 {
     __shared__ float win[8][RANK];
     const int o0 = blockIdx.y * 8, i = blockIdx.x * 256 + threadIdx.x;
@@ -1021,7 +1064,11 @@ __global__ void __launch_bounds__(256) k_fold_hidden(const uint16_t *W_h, const 
         for (int rr = 0; rr < 8; ++rr) acc[rr] = fmaf(win[rr][e], x, acc[rr]);
     }
 #pragma unroll
-    for (int rr = 0; rr < 8; ++rr) Fhg[(size_t)(o0 + rr) * H + i] = acc[rr];
+    for (int rr = 0; rr < 8; ++rr) {
+        const uint16_t hi = f2bf(acc[rr]);
+        Fhl[(size_t)(o0 + rr) * H + i] = hi;
+        Fhl[(size_t)(2 * RANK + o0 + rr) * H + i] = f2bf(acc[rr] - bf2f(hi));
+    }
 }
 
 // Packs L's strictly lower part channel-innermost: Lpk[k(k-1)/2 + j][d] =

@@ -71,9 +71,8 @@ size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 struct Layout {
     size_t status = 0, ctl = 64, params = 256, st = 0, upart = 0, pc = 0, ynew = 0, acttok = 0, zpack = 0,
            zbuf = 0, part = 0, total = 0;
-    size_t sctl = 0, cx = 0, ux = 0, pcx = 0, rmax = 0, best64 = 0;
+    size_t sctl = 0, cx = 0, ux = 0, pcx = 0, c0x = 0, rmax = 0, best64 = 0;
     int ksplit = 1, kchunk = 0, S = 1;
-    int pre_kslice = 0, pre_ks = 0;
     bool gemv = false;
     bool tcv = false;
     bool small = false;      // persistent small-batch kernel
@@ -93,7 +92,7 @@ struct xpress_refiner {
     int num_sms = 0;
     bool use_tc = false;
     cudaStream_t cs = nullptr;
-    float *Fhg = nullptr;                  // [2r, H] folded hidden projection (small-batch kernel)
+    uint16_t *Fhl = nullptr;               // [2][2r, H] folded hidden projection, bf16 hi / lo (small-batch kernel)
     uint16_t *Lpk = nullptr;               // [B(B-1)/2, r] L's strictly lower part, channel innermost
     bool small_ok = false;                 // the small-batch kernel can run co-resident on this GPU
     void *small_ws[CACHE_SLOTS] = {};      // workspaces whose control area this refiner has cleared
@@ -168,18 +167,6 @@ Layout make_layout(const xpress_refiner *R, int b)
     L.S = read_S(R, b);
     L.small = use_small(R, b);
     int upart_ks = L.ksplit;
-    if (L.small) {
-        // K-slices of the folded projection: about one work item per Read CTA,
-        // h's slice within the W_r stages (128 KB)
-        const int ng = N <= 16 ? 16 : 32;
-        const int ks_max = L.S / ng > 1 ? L.S / ng : 1;
-        int kslice = ((R->w.H + ks_max - 1) / ks_max + 127) / 128 * 128;
-        const int kcap = (128 * 1024 / (2 * N)) / 128 * 128;
-        if (kslice > kcap) kslice = kcap;
-        L.pre_kslice = kslice;
-        L.pre_ks = (R->w.H + kslice - 1) / kslice;
-        if (L.pre_ks > upart_ks) upart_ks = L.pre_ks;
-    }
     L.upart = o;
     o = align256(o + (size_t)upart_ks * N * 2 * RANK * 4);
     L.pc = o;
@@ -201,6 +188,8 @@ Layout make_layout(const xpress_refiner *R, int b)
         L.ux = o;
         o = align256(o + (size_t)32 * 2 * RANK * 2);
         L.pcx = o;
+        o = align256(o + (size_t)32 * RANK * 4);
+        L.c0x = o;
         o = align256(o + (size_t)32 * RANK * 4);
         L.rmax = o;
         o = align256(o + (size_t)N * RMAX_SEG * sizeof(Partial));
@@ -270,9 +259,8 @@ Params make_params(const xpress_refiner *R, const xpress_block_in *in, const xpr
     P.part = reinterpret_cast<RPartial *>(w + L.part);
     if (L.small) {
         P.use_graph = 0;
-        P.Fhg = R->Fhg;
-        P.pre_kslice = L.pre_kslice;
-        P.pre_ks = L.pre_ks;
+        P.Fhl = R->Fhl;
+        P.c0x = reinterpret_cast<float *>(w + L.c0x);
         P.cx = reinterpret_cast<uint16_t *>(w + L.cx);
         P.ux = reinterpret_cast<uint16_t *>(w + L.ux);
         P.pcx = reinterpret_cast<float *>(w + L.pcx);
@@ -646,7 +634,9 @@ void print_trace(xpress_refiner *R, cudaStream_t st)
     for (int i = 0; i < TRACE_SLOTS; ++i) {
         if (h[i] == ~0ull) continue;
         char name[32];
-        if (i >= 240 && i < 248) std::snprintf(name, sizeof(name), "end%dphase%d", (i - 240) / 4, (i - 240) % 4);
+        if (i >= 248) std::snprintf(name, sizeof(name), "transsetup%d", i - 248);
+        else if (i >= 4 && i < 8) std::snprintf(name, sizeof(name), "readsetup%d", i - 4);
+        else if (i >= 240 && i < 248) std::snprintf(name, sizeof(name), "end%dphase%d", (i - 240) / 4, (i - 240) % 4);
         else if (i >= 230 && i < 240) std::snprintf(name, sizeof(name), "read0phase%d", i - 230);
         else if (i >= 210) std::snprintf(name, sizeof(name), "mlp%dphase%d", (i - 210) / 8, (i - 210) % 8);
         else if (i >= 200) std::snprintf(name, sizeof(name), "readphase%d", i - 200);
@@ -734,13 +724,13 @@ int xpress_refiner_create(const xpress_weights *w, void *stream, xpress_refiner 
                 coop = 0;
             }
             if (coop && per_sm >= 1 && R->num_sms > SMALL_TRANS_CTAS) {
-                if (cudaMalloc(&R->Fhg, (size_t)2 * RANK * w->H * sizeof(float)) != cudaSuccess) {
+                if (cudaMalloc(&R->Fhl, (size_t)2 * 2 * RANK * w->H * sizeof(uint16_t)) != cudaSuccess) {
                     rc = XPRESS_ERR_CUDA;
                     break;
                 }
                 k_fold_hidden<<<dim3((w->H + 255) / 256, 2 * RANK / 8), 256, 0, st>>>(
                     static_cast<const uint16_t *>(w->W_h), static_cast<const uint16_t *>(w->W_g),
-                    static_cast<const uint16_t *>(w->W_in), R->Fhg, w->H);
+                    static_cast<const uint16_t *>(w->W_in), R->Fhl, w->H);
                 const int tri = w->B * (w->B - 1) / 2;
                 if (cudaMalloc(&R->Lpk, (size_t)(tri > 0 ? tri : 1) * RANK * 2) != cudaSuccess) {
                     rc = XPRESS_ERR_CUDA;
@@ -767,7 +757,7 @@ int xpress_refiner_destroy(xpress_refiner *R)
     if (!R) return XPRESS_ERR_INVALID_ARG;
     for (auto &e : R->cache) destroy_entry(e);
     if (R->Ep) cudaFree(R->Ep);
-    if (R->Fhg) cudaFree(R->Fhg);
+    if (R->Fhl) cudaFree(R->Fhl);
     if (R->Lpk) cudaFree(R->Lpk);
     if (R->cs) cudaStreamDestroy(R->cs);
     if (R->trace) cudaFree(R->trace);
