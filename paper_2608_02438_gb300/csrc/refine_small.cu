@@ -76,6 +76,7 @@ struct TsShared {
     int tok2[MAX_B];                           // evaluated tokens of the next pass
     int tpos[MAX_B], tseq[MAX_B];              // per global token id: position k, block s
     SeqState st[MAX_B];                        // per block: Algorithm 1 state
+    int anch[MAX_B];                           // per block: anchor token (bounds-checked)
     float invT[MAX_B];                         // per block: 1 / T (0 for greedy)
     int n, n2, go, more;
 };
@@ -618,14 +619,26 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
 
 // Fuse, token part: e_j = E'[x_{j-1}] (x_{-1} = the anchor) for every position
 // j of every block, channels [cb, cb + CH) (16-byte pieces).
-__device__ __forceinline__ void gather_e(const Params &p, const int *x, float *e, int CH, int cb, int tid, int nth)
+__device__ __forceinline__ void gather_e(const Params &p, const int *x, const int *anch, float *e, int CH, int cb,
+                                         int tid, int nth)
 {
-    const int N = p.N, B = p.B, V = p.V;
-    for (int i = tid; i < N * CH / 4; i += nth) {
-        const int j = i / (CH / 4), q = i % (CH / 4), k = j % B, s = j / B;
-        int tk = k == 0 ? p.anchor[s] : x[j - 1];
-        if (tk < 0 || tk >= V) tk = 0;                         // reported at the start
-        reinterpret_cast<float4 *>(e)[i] = __ldg(reinterpret_cast<const float4 *>(p.Ep + (size_t)tk * RANK + cb) + q);
+    const int N = p.N, B = p.B, V = p.V, total = N * CH / 4;
+    constexpr int GU = 4;                                      // loads in flight per thread
+    for (int i0 = tid; i0 < total; i0 += GU * nth) {
+        float4 v[GU];
+#pragma unroll
+        for (int u = 0; u < GU; ++u) {
+            const int i = i0 + u * nth;
+            if (i < total) {
+                const int j = i / (CH / 4), q = i % (CH / 4), k = j % B, s = j / B;
+                int tk = k == 0 ? anch[s] : x[j - 1];
+                if (tk < 0 || tk >= V) tk = 0;                 // reported at the start
+                v[u] = __ldg(reinterpret_cast<const float4 *>(p.Ep + (size_t)tk * RANK + cb) + q);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < GU; ++u)
+            if (i0 + u * nth < total) reinterpret_cast<float4 *>(e)[i0 + u * nth] = v[u];
     }
 }
 
@@ -688,6 +701,7 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
         SeqState s{};
         s.active = 1; s.m = -1; s.iters = 0; s.converged = 0; s.off = tid * B; s.cnt = B;
         sh.st[tid] = s;
+        sh.anch[tid] = p.anchor[tid];
         const float T = p.temperature[tid];
         sh.invT[tid] = T > 0.0f ? 1.0f / T : 0.0f;
     }
@@ -732,7 +746,7 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
         if (trs) trace_mark(p.trace, trs, t_pass);
         const bool first_c = pass == 0 && p.draft;             // c formed by the Read CTAs
         if (!first_c) {
-            gather_e(p, sh.x, e, CH, cb, tid, nth);
+            gather_e(p, sh.x, sh.anch, e, CH, cb, tid, nth);
             __syncthreads();
         }
         if (trs) trace_mark(p.trace, trs + 1, t_pass);
@@ -754,8 +768,10 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
             // thread (channel pair 2 cp, 2 cp + 1; half kh of the positions,
             // dealt ABBA from the last one so that both halves get about the
             // same number of L terms): a block's E' values sit in registers,
-            // the j loop is unrolled (B <= 16) and predicated on k, and two
-            // partial sums per channel shorten the dependency chains
+            // the j loop is unrolled (B <= 16) with unconditional loads (row
+            // k(k-1)/2 + j2 stays inside the 120 rows reserved for Lp) and the
+            // terms j2 >= k selected away, and two partial sums per channel
+            // shorten the dependency chains
             const int cp = tid & 127, kh = tid >> 7, d = 2 * cp;
             if (kh < 2)
                 for (int s = 0; s < b; ++s) {
@@ -773,10 +789,12 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
                         float2 a0 = *reinterpret_cast<const float2 *>(e + (s * B + k) * CH + d);
                         float2 a1 = make_float2(0.0f, 0.0f);
                         const uint32_t *lrow = reinterpret_cast<const uint32_t *>(Lp + (k * (k - 1) / 2) * CH + d);
+                        uint32_t lw2[FULL_C_MAX_B - 1];
 #pragma unroll
-                        for (int j2 = 0; j2 < FULL_C_MAX_B - 1; ++j2)
-                            if (j2 < k) {
-                                const uint32_t lw = lrow[j2 * (CH / 2)];
+                        for (int j2 = 0; j2 < FULL_C_MAX_B - 1; ++j2) lw2[j2] = lrow[j2 * (CH / 2)];
+#pragma unroll
+                        for (int j2 = 0; j2 < FULL_C_MAX_B - 1; ++j2) {
+                                const uint32_t lw = j2 < k ? lw2[j2] : 0u;
                                 const float lx = __uint_as_float(lw << 16), ly = __uint_as_float(lw & 0xFFFF0000u);
                                 if (j2 & 1) {
                                     a1.x = fmaf(lx, er[j2].x, a1.x);
