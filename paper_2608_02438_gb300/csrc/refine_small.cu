@@ -576,19 +576,62 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
             sh.sel[ew][lane] = sel;
             if (p.trace && pass < 2 && lane == 0) { const unsigned long long tn = globaltimer_ns(); trace_mark(p.trace, pass ? 204 : 234, tn); }
             if (tv_epi_bar_or(!ok || *abort)) break;
-            if (ew == 0 && lane < n) {
-                RPartial a = sh.sel[0][lane].partial();
-                int wbest = 0;
+            // T > 0: the member draw of this range's best group, once per
+            // token, its 32 members split over the 8 warps (warp w: members
+            // 4w .. 4w + 3, one Philox call); every warp merges the partials
+            // of the 8 warps to find that group (the same result in each)
+            RPartial a{};
+            int wbest = 0;
+            const bool draw = tv_epi_bar_or(lane < n && my_invT > 0.0f);
+            if (draw && lane < n) {
+                a = sh.sel[0][lane].partial();
                 for (int w2 = 1; w2 < TV_EPI_WARPS; ++w2) {
                     const RPartial b2 = sh.sel[w2][lane].partial();
                     if (b2.best > a.best || (b2.best == a.best && b2.idx < a.idx)) wbest = w2;
                     merge_rpartial(a, b2, my_invT > 0.0f);
                 }
+                float bsc = -INFINITY, bx = 0.0f;
+                int bj = 0x7fffffff;
                 if (my_invT > 0.0f && a.idx != 0x7fffffff) {
-                    // the member draw of this range's best group, once
-                    const int v0 = a.idx * GROUP;
-                    member_draw<32>(&sh.bestx[wbest][0][lane], min(GROUP, V - v0), v0, my_seed, (uint32_t)my_pos,
-                                    p.offset, a.y, a.sel);
+                    const int v0 = a.idx * GROUP, valid = min(GROUP, V - v0);
+                    const uint4 o = philox10(make_uint4(((uint32_t)v0 >> 2) + ew, (uint32_t)my_pos, STREAM_ELEM, p.offset),
+                                             (uint32_t)my_seed, (uint32_t)(my_seed >> 32));
+                    const uint32_t w4[4] = {o.x, o.y, o.z, o.w};
+#pragma unroll
+                    for (int q2 = 0; q2 < 4; ++q2) {
+                        const int j = 4 * ew + q2;
+                        if (j < valid) {
+                            const float u = ((float)(w4[q2] >> 9) + 0.5f) * (1.0f / 8388608.0f);
+                            const float xj = sh.bestx[wbest][j][lane];
+                            const float sc = xj - logf(-logf(u));
+                            if (sc > bsc) { bsc = sc; bj = j; bx = xj; }
+                        }
+                    }
+                }
+                tile[0][lane] = bsc;
+                tile[1][lane] = __int_as_float(bj);
+                tile[2][lane] = bx;
+            }
+            if (draw) tv_epi_bar();
+            if (ew == 0 && lane < n) {
+                if (my_invT > 0.0f) {
+                    if (a.idx != 0x7fffffff) {
+                        // members in order, the first of equal scores
+                        float bsc = -INFINITY, bx = 0.0f;
+                        int bj = 0;
+                        for (int w2 = 0; w2 < TV_EPI_WARPS; ++w2)
+                            if (sh.tile[w2][0][lane] > bsc) {
+                                bsc = sh.tile[w2][0][lane];
+                                bj = __float_as_int(sh.tile[w2][1][lane]);
+                                bx = sh.tile[w2][2][lane];
+                            }
+                        if (bsc == -INFINITY) bx = sh.bestx[wbest][0][lane];
+                        a.y = a.idx * GROUP + bj;
+                        a.sel = bx;
+                    }
+                } else {
+                    a = sh.sel[0][lane].partial();
+                    for (int w2 = 1; w2 < TV_EPI_WARPS; ++w2) merge_rpartial(a, sh.sel[w2][lane].partial(), false);
                 }
                 if (my_invT > 0.0f) p.part[(size_t)lane * S + r] = a;
                 else atomicMax(p.best64 + 32 * (pass & 1) + lane, argmax_key(a.best, a.idx));   // greedy: one key
@@ -639,6 +682,47 @@ __device__ __forceinline__ void gather_e(const Params &p, const int *x, const in
 #pragma unroll
         for (int u = 0; u < GU; ++u)
             if (i0 + u * nth < total) reinterpret_cast<float4 *>(e)[i0 + u * nth] = v[u];
+    }
+}
+
+// Mix of one block of B = 16 positions for the channel pair d, d + 1 (full-c
+// mode): c_k = Pc_k + e_k + sum_{j<k} L_kj e_j (Eq. fuse / mix) for the
+// positions k > m of half KH (dealt ABBA from the last position, so that both
+// halves get 60 of the 120 L terms).  Every (k, j) term is a compile-time
+// slot: no per-term predicate or index arithmetic.  e and pc point at the
+// block's first row; c goes to cop (bf16, row t = off + k - m - 1) and, for
+// the CTA's own channels, to cown (fp32).
+//
+// Not inlined: the Trans CTAs run it once on scratch operands while they wait
+// for the precompute, so that its code (about 600 instructions, a cold fetch
+// from DRAM after the caches have been flushed) is cached before the first
+// pass that mixes.
+template <int KH>
+__device__ __noinline__ void mix_block16(const float *e, const uint16_t *Lp, const float *pc, uint16_t *cop,
+                                         float (*cown)[32], int d, int m, int off, int rank)
+{
+    constexpr int BB = FULL_C_MAX_B;
+    float2 er[BB];
+#pragma unroll
+    for (int j = 0; j < BB; ++j) er[j] = *reinterpret_cast<const float2 *>(e + j * RANK + d);
+#pragma unroll
+    for (int q = 0; q < BB / 2; ++q) {
+        const int k = BB - 1 - ((q >> 1) * 4 + (KH ? 1 + (q & 1) : (q & 1) * 3));
+        if (k <= m) continue;
+        float2 a0 = er[k], a1 = make_float2(0.0f, 0.0f);
+        const uint32_t *lrow = reinterpret_cast<const uint32_t *>(Lp + (k * (k - 1) / 2) * RANK + d);
+#pragma unroll
+        for (int j = 0; j < k; ++j) {
+            const uint32_t lw = lrow[j * (RANK / 2)];
+            float2 &a = (j & 1) ? a1 : a0;
+            a.x = fmaf(__uint_as_float(lw << 16), er[j].x, a.x);
+            a.y = fmaf(__uint_as_float(lw & 0xFFFF0000u), er[j].y, a.y);
+        }
+        const int t = off + k - m - 1;
+        const float2 pcv = *reinterpret_cast<const float2 *>(pc + k * RANK + d);
+        const float c0 = pcv.x + (a0.x + a1.x), c1 = pcv.y + (a0.y + a1.y);
+        *reinterpret_cast<uint32_t *>(cop + t * COP_LD + d) = (uint32_t)f2bf(c0) | ((uint32_t)f2bf(c1) << 16);
+        if ((d >> 5) == rank) *reinterpret_cast<float2 *>(&cown[t][d & 31]) = make_float2(c0, c1);
     }
 }
 
@@ -704,6 +788,13 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
         sh.anch[tid] = p.anchor[tid];
         const float T = p.temperature[tid];
         sh.invT[tid] = T > 0.0f ? 1.0f / T : 0.0f;
+    }
+    if (full && B == FULL_C_MAX_B && tid < 2 * 128) {
+        // warm the mix's code on scratch operands (cop and cown are rewritten
+        // before their first use; e and pc hold whatever is there)
+        const int d = 2 * (tid & 127);
+        if (tid < 128) mix_block16<0>(e, Lp, pc, cop, sh.cown, d, -1, 0, rank);
+        else mix_block16<1>(e, Lp, pc, cop, sh.cown, d, -1, 0, rank);
     }
     if (lead && tid == 0 && p.trace) trace_mark(p.trace, 250, t_start);
     if (tid == 0) sh.go = wait_count(c, &c->pre_done.v, (unsigned)p.S);
@@ -773,7 +864,15 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
             // terms j2 >= k selected away, and two partial sums per channel
             // shorten the dependency chains
             const int cp = tid & 127, kh = tid >> 7, d = 2 * cp;
-            if (kh < 2)
+            if (B == FULL_C_MAX_B) {
+                for (int s = 0; s < b; ++s) {
+                    const SeqState st = sh.st[s];
+                    if (!st.active) continue;
+                    if (kh == 0) mix_block16<0>(e + s * B * CH, Lp, pc + s * B * CH, cop, sh.cown, d, st.m, st.off, rank);
+                    else if (kh == 1)
+                        mix_block16<1>(e + s * B * CH, Lp, pc + s * B * CH, cop, sh.cown, d, st.m, st.off, rank);
+                }
+            } else if (kh < 2)
                 for (int s = 0; s < b; ++s) {
                     const SeqState st = sh.st[s];
                     if (!st.active) continue;
@@ -886,11 +985,24 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
         // every Trans CTA has read the previous pass's keys (before its u was
         // published): clear them for the pass after this one (same parity)
         if (lead && pass > 0 && tid < 32) p.best64[32 * ((pass - 1) & 1) + tid] = 0ull;
-        for (int i = tid; i < 32 * (2 * RANK / 8); i += nth) {
-            const int t = i / (2 * RANK / 8), cc = i % (2 * RANK / 8);
-            uint4 v = make_uint4(0, 0, 0, 0);
-            if (t < n) v = __ldcg(reinterpret_cast<const uint4 *>(p.ux + (size_t)t * 2 * RANK) + cc);
-            *reinterpret_cast<uint4 *>(uop + t * UOP_LD + 8 * cc) = v;
+        {
+            // the rows of W_2's 16-row tiles: u of the evaluated tokens, zeros
+            // past n; four loads in flight per thread
+            const int total = (n + 15) / 16 * 16 * (2 * RANK / 8);
+            for (int i0 = tid; i0 < total; i0 += 4 * nth) {
+                uint4 v[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int i = i0 + u * nth, t = i / (2 * RANK / 8), cc = i % (2 * RANK / 8);
+                    v[u] = make_uint4(0, 0, 0, 0);
+                    if (i < total && t < n) v[u] = __ldcg(reinterpret_cast<const uint4 *>(p.ux + (size_t)t * 2 * RANK) + cc);
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int i = i0 + u * nth, t = i / (2 * RANK / 8), cc = i % (2 * RANK / 8);
+                    if (i < total) *reinterpret_cast<uint4 *>(uop + t * UOP_LD + 8 * cc) = v[u];
+                }
+            }
         }
         __syncthreads();
         // z = c + W_2 u for channels [32 rank, +32): warp w -> 8 channels, K half w / 4
