@@ -121,6 +121,34 @@ __device__ __forceinline__ bool wait_count(SmallCtl *c, const unsigned *ctr, uns
     return false;
 }
 
+// wait_count that, while it waits, streams [pf, pf + bytes) into L2 one
+// slice every gap_ns: DRAM stays busy without queues deep enough to stall the
+// latency-bound accesses of the other role (its first-pass code and operands).
+__device__ __forceinline__ bool wait_count_prefetch(SmallCtl *c, const unsigned *ctr, unsigned target, const char *pf,
+                                                    uint32_t bytes, uint32_t slice, unsigned gap_ns)
+{
+    const unsigned long long t0 = globaltimer();
+    unsigned long long t_next = t0;
+    uint32_t done = 0;
+    for (uint32_t it = 0; it < (1u << 26); ++it) {
+        const unsigned v = ld_relaxed_gpu(ctr);
+        if (v & STOP_BIT) { fence_acq_rel_gpu(); return false; }
+        if (v >= target) { fence_acq_rel_gpu(); return true; }
+        if (done < bytes) {
+            const unsigned long long now = globaltimer();
+            if (now >= t_next) {
+                prefetch_l2_bulk(pf + done, min(slice, bytes - done));
+                done += slice;
+                t_next = now + gap_ns;
+            }
+        }
+        if (it >= 2) __nanosleep(32);
+        if ((it & 63u) == 63u && globaltimer() - t0 > 2000000000ull) break;
+    }
+    raise_stop(c, ST_TIMEOUT);
+    return false;
+}
+
 // One thread per CTA, last action on the control area: the CTA that leaves
 // last publishes the call's status and hands the other block to the next call.
 __device__ __forceinline__ void leave(const Params &p, SmallCtlArea *a, SmallCtl *c, int par)
@@ -392,15 +420,6 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
         if (sh.abort) raise_stop(c, ST_TIMEOUT);
         else red_add_release_gpu(&c->pre_done.v, 1u);
         if (tr) trace_mark(p.trace, 2, t_start);
-        // this CTA's W_r range into L2 while the first Trans runs (after the
-        // precompute, whose reads it would otherwise slow down)
-        if (!(p.read_flags & 1)) {
-            const char *wr = static_cast<const char *>(p.W_r);
-            const int rows = min(vb1 * TV_BM, V) - vb0 * TV_BM;
-            for (int r0 = 0; r0 < rows; r0 += 64)
-                prefetch_l2_bulk(wr + (size_t)(vb0 * TV_BM + r0) * RANK * 2,
-                                 (uint32_t)min(64, rows - r0) * RANK * 2);
-        }
     }
 
     if (warp == 0) {
@@ -426,8 +445,18 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
             const bool lookahead = !(p.read_flags & 2);
             if (lookahead)
                 for (; next < ahead && ok; ++next) ok = issue(next);
+            // while the first Trans runs, the rest of this CTA's W_r range
+            // (past the chunks the ring holds) goes into L2 a slice at a time
+            const int pf_row0 = vb0 * TV_BM + (lookahead ? ahead / TV_KCH : 0) * TV_BM;
+            const int pf_rows = max(0, min(vb1 * TV_BM, V) - pf_row0);
+            const uint32_t pf_bytes = (p.read_flags & 1) ? 0u : (uint32_t)pf_rows * RANK * 2;
             for (int pass = 0; ok; ++pass) {
-                const bool go = wait_count(c, &c->z_ready.v, (unsigned)(8 * (pass + 1)));
+                const bool go = pass == 0
+                                    ? wait_count_prefetch(c, &c->z_ready.v, 8u, static_cast<const char *>(p.W_r) +
+                                                                                   (size_t)pf_row0 * RANK * 2,
+                                                          pf_bytes, 64 * RANK * 2,
+                                                          (p.read_flags >> 8) ? (unsigned)(p.read_flags >> 8) * 100u : 1000u)
+                                    : wait_count(c, &c->z_ready.v, (unsigned)(8 * (pass + 1)));
                 if (go) {
                     fence_proxy_async_global();
                     sh.pass_n = min(__ldcg(p.ctl + CTL_NACT), TV_BN);
