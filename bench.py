@@ -44,7 +44,7 @@ SMALL_SOURCES = [CSRC + f for f in ("refine_small.cu", "tcv_common.cuh", "mlp_co
                                     "common.cuh")]
 SMALL_SUMMARY = "profiles/k_refine_small_qwen3_8b_greedy.txt"
 READ_SOURCES = [CSRC + "read_tc.cu", CSRC + "common.cuh"]
-READ_SUMMARY = "profiles/k_read_tc_serving_b32.txt"
+READ_SUMMARIES = {"long_b64": "profiles/k_read_tc_long_b64.txt"}
 
 
 def dist_env():
@@ -62,8 +62,8 @@ def source_hash(paths):
 def profiled_traffic(summary: str, bytes_hash: str):
     """dram bytes per launch from the committed ncu summary, if it was taken
     on the current kernel sources."""
-    path = os.path.join(ROOT, summary)
-    if not os.path.exists(path):
+    path = os.path.join(ROOT, summary) if summary else ""
+    if not path or not os.path.isfile(path):
         return None
     kv = {}
     for line in open(path):
@@ -351,9 +351,14 @@ def run_xpress(args):
         rows = 128 if small else 256
         S = min(sms, (cfg.V + rows - 1) // rows)
         read_bytes = cfg.V * cfg.r * esz + n_tok * cfg.V * esz + n_tok * cfg.r * esz + S * n_tok * 32
-        summary, srcs = READ_SUMMARY, READ_SOURCES
+        summary, srcs = READ_SUMMARIES.get(cfg.name, ""), READ_SOURCES
     hbm, tc_peak, src = peaks()
     achieved = read_bytes / (read_ms / 1000.0) / 1e9
+    # large token counts: the LM-head product 2 V r N is what the kernel does
+    # most of, so its roofline is the tensor pipe (bf16 dense, measured)
+    tensor_bound = (not persistent) and (not small)
+    read_flops = 2.0 * cfg.V * cfg.r * n_tok
+    achieved_tf = read_flops / (read_ms / 1000.0) / 1e12
     rhash = source_hash(srcs)
     traffic = profiled_traffic(summary, rhash)
 
@@ -372,8 +377,11 @@ def run_xpress(args):
             "e2e": {"value": e2e_value, "unit": "blocks/s", "h2d_bytes_per_step": int(h2d),
                     "d2h_bytes_per_step": int(d2h), "steps": n_e2e},
             "gpu_launches": per_step_launches * args.steps,
-            "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                         "frac": achieved / hbm, "traffic": traffic, "peak_source": src,
+            "roofline": {"bound": "tensor" if tensor_bound else "hbm",
+                         "achieved": achieved_tf if tensor_bound else achieved,
+                         "peak": tc_peak if tensor_bound else hbm, "unit": "TFLOP/s" if tensor_bound else "GB/s",
+                         "frac": (achieved_tf / tc_peak) if tensor_bound else achieved / hbm,
+                         "hbm_frac": achieved / hbm, "traffic": traffic, "peak_source": src,
                          "kernel": read_kernel, "bytes_per_launch": read_bytes, "launch_ms": read_ms,
                          "launch_ms_l2_warm": read_warm_ms,
                          "tokens_per_launch": n_tok, "passes_per_launch": passes if persistent else 1,
