@@ -354,10 +354,11 @@ def run_xpress(args):
         summary, srcs = READ_SUMMARIES.get(cfg.name, ""), READ_SOURCES
     hbm, tc_peak, src = peaks()
     achieved = read_bytes / (read_ms / 1000.0) / 1e9
-    # large token counts: the LM-head product 2 V r N is what the kernel does
-    # most of, so its roofline is the tensor pipe (bf16 dense, measured)
-    tensor_bound = (not persistent) and (not small)
+    # large token counts: the LM-head product 2 V r N; the roofline is the
+    # tensor pipe (bf16 dense, measured) when its arithmetic intensity is near
+    # the ridge (batch 64 x block 32: 224 of 284 flop/byte), else HBM
     read_flops = 2.0 * cfg.V * cfg.r * n_tok
+    tensor_bound = (not persistent) and (not small) and read_flops / read_bytes >= 0.75 * tc_peak * 1e3 / hbm
     achieved_tf = read_flops / (read_ms / 1000.0) / 1e12
     rhash = source_hash(srcs)
     traffic = profiled_traffic(summary, rhash)

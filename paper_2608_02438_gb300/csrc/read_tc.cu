@@ -11,16 +11,19 @@
 // each epilogue thread owns one token and reduces over vocabulary columns
 // without any cross-thread traffic.
 //
-// Roles (320 threads, one CTA per SM, persistent over a contiguous vocabulary
+// Roles (576 threads, one CTA per SM, persistent over a contiguous vocabulary
 // range):
 //   warp 0      TMA producer: the token tile (A, kept for the whole range) and
-//               a 4-stage ring of W_r K-chunks (B, 32 KB each)
+//               a 2-stage ring of W_r K-chunks (B, 32 KB each)
 //   warp 1      TMEM allocator and tcgen05.mma issuer (one thread)
-//   warps 2-9   epilogue: tcgen05.ld 32 columns, add s, select_group
+//   warps 2-17  epilogue: tcgen05.ld 32 columns, add s (a 2-slot cp.async ring
+//               per thread), select_group; 4 warps per SM sub-partition, so
+//               that the dependent chains of the fold are hidden
 // Two TMEM accumulators of 256 columns let the MMA of tile t+1 overlap the
-// epilogue of tile t.  With <= 32 evaluated tokens the 32 token rows are
-// replicated into all four TMEM lane quarters, so that all four SM
-// sub-partitions share the epilogue (each warp takes one 32-id group).
+// epilogue of tile t.  The 4 warps of a TMEM lane quarter split the 8 groups of
+// a tile.  With <= 32 evaluated tokens the 32 token rows are replicated into
+// all four TMEM lane quarters, and warps 0-7 of the epilogue take one 32-id
+// group each (the others only hand the accumulators back).
 #include "common.cuh"
 #include "kernels.h"
 
@@ -31,8 +34,9 @@ constexpr int TC_BN = 256;
 constexpr int TC_BK = 64;                     // one 128-byte swizzle row of bf16
 constexpr int TC_KCH = RANK / TC_BK;          // 4 K-chunks
 constexpr int TC_STAGES = 2;                  // W_r stays in L2 (evict_last): 2 stages in flight suffice
-constexpr int TC_SPF = 4;                     // s groups in flight per epilogue thread (cp.async ring)
-constexpr int TC_EPI_WARPS = 8;
+constexpr int TC_SPF = 2;                     // s groups in flight per epilogue thread (cp.async ring)
+constexpr int TC_EPI_WARPS = 16;                // 4 per SM sub-partition (latency hiding)
+constexpr int TC_WPQ = TC_EPI_WARPS / 4;       // epilogue warps per TMEM lane quarter
 constexpr int TC_THREADS = 32 * (2 + TC_EPI_WARPS);
 constexpr uint32_t TC_A_CHUNK = TC_BM * TC_BK * 2;       // 16 KB
 constexpr uint32_t TC_A_BYTES = TC_A_CHUNK * TC_KCH;      // 64 KB
@@ -56,7 +60,7 @@ constexpr size_t TC_SMEM_BYTES = 1024 + TC_A_BYTES + TC_STAGES * TC_B_STAGE + TC
 const size_t kReadTcSmemBytes = TC_SMEM_BYTES;
 const int kReadTcThreads = TC_THREADS;
 
-__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, %0;" ::"n"(TC_EPI_WARPS * 32) : "memory"); }
 
 // Named barrier over the 8 epilogue warps that also ORs a predicate, so that
 // every epilogue warp takes the same decision to stop after an abort.
@@ -66,10 +70,10 @@ __device__ __forceinline__ bool epi_bar_or(bool pred)
     asm volatile(
         "{\n\t.reg .pred p, q;\n\t"
         "setp.ne.u32 p, %1, 0;\n\t"
-        "bar.red.or.pred q, 1, 256, p;\n\t"
+        "bar.red.or.pred q, 1, %2, p;\n\t"
         "selp.u32 %0, 1, 0, q;\n\t}"
         : "=r"(res)
-        : "r"((uint32_t)pred)
+        : "r"((uint32_t)pred), "n"(TC_EPI_WARPS * 32)
         : "memory");
     return res != 0;
 }
@@ -242,8 +246,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         const int ew = warp - 2;
         const int q = warp & 3;              // TMEM lane quarter this warp may access
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
-        const int g_first = small ? ew : (ew >> 2) * 4;
-        const int g_count = small ? 1 : 4;
+        // large: the TC_WPQ warps of a lane quarter split the 8 groups of a
+        // tile; small (<= 32 tokens, replicated in every quarter): warp ew < 8
+        // takes group ew, the others only hand the accumulators back
+        const int g_first = small ? (ew & 7) : (ew >> 2) * (8 / TC_WPQ);
+        const int g_count = small ? (ew < 8 ? 1 : 0) : 8 / TC_WPQ;
         int t = 0;
         for (int j = 0; j < MT; ++j) {
             bool ok = true;
@@ -267,18 +274,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             // (tile, group) work items in order; s of item i + 1 is loaded
             // while item i is processed
             const int items = (vt1 - vt0) * g_count;
-            // this thread's s segment of vocabulary tile vt into L2 (bulk, no
-            // registers): the register loads one group ahead then hit L2
             // s is read once: evict it first, so that W_r (re-read for every
-            // token tile, evict_last) stays in L2
+            // token tile, evict_last) stays in L2.  (An L2 bulk prefetch of s
+            // ahead of the ring measured slower: many small prefetches.)
             const uint64_t once = policy_evict_first();
-            auto prefetch_s = [&](int vt) {
-                const int v0 = vt * TC_BN + g_first * GROUP;
-                if (valid && vt < vt1 && v0 < p.V)
-                    prefetch_l2_bulk_hint(srow + v0, (uint32_t)min(g_count * GROUP, p.V - v0) * 2u, once);
-            };
-            prefetch_s(vt0);
-            prefetch_s(vt0 + 1);
             float gn[4] = {0.f, 0.f, 0.f, 0.f};     // T > 0: Gumbel noise of the tile's group quad
             // s of item k into ring slot k % TC_SPF (cp.async, L2 only; zero-filled
             // past V or for an invalid thread), one commit group per item
@@ -298,11 +297,20 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             };
 #pragma unroll
             for (int k = 0; k < TC_SPF - 1; ++k) issue_s(k);
+            if (g_count == 0)
+                for (int vt = vt0; vt < vt1; ++vt) {
+                    const int buf = t & 1;
+                    if (!mbar_wait(&sh.tfull[buf], (t >> 1) & 1, abort)) { ok = false; break; }
+                    tc_fence_after();
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&sh.tempty[buf]);
+                    ++t;
+                }
             for (int it = 0; it < items; ++it) {
                 const int vt = vt0 + it / g_count, gl = g_first + it % g_count;
                 const int buf = t & 1;
                 if (gl == g_first) {
-                    prefetch_s(vt + 2);
                     if (valid && invT > 0.0f)
                         group_noise4(seed, (uint32_t)(vt * (TC_BN / GROUP) + g_first) >> 2, (uint32_t)pos, p.offset, gn);
                     if (!mbar_wait(&sh.tfull[buf], (t >> 1) & 1, abort)) { ok = false; break; }
@@ -354,7 +362,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     }
                 } else if (ew < 4 && valid) {
                     RPartial a = sh.st[ew][lane].partial();
-                    merge_rpartial(a, sh.st[ew + 4][lane].partial(), invT > 0.0f);
+                    for (int w = 1; w < TC_WPQ; ++w) merge_rpartial(a, sh.st[ew + 4 * w][lane].partial(), invT > 0.0f);
                     p.part[(size_t)i * p.S + r] = a;
                 }
             }
