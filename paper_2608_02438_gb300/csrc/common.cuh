@@ -120,7 +120,9 @@ struct Params {
     int32_t *status;
     int32_t *ctl;
     SeqState *st;
-    float *Upart;                // [ksplit, N, 2r] partial sums of h [W_h; W_g]^T
+    float *Upart;                // [ksplit, N, 2r] partial sums of h [W_h; W_g]^T (pre_folded: of h F^T,
+                                 // F = [W_in[:, 0:r] W_h ; W_in[:, r:2r] W_g])
+    int pre_folded;              // Upart holds the folded projection (k_pre_tc)
     float *Pc;                   // [N, r] token-independent part of c after Mix
     int32_t *Ynew;               // [N]
     int32_t *act_tok;            // [N] packed evaluated tokens (global token ids)

@@ -82,5 +82,8 @@ int accept_launch(const xpress_refiner *R, const xpress_accept_in *in, int32_t *
                   void *ws, size_t ws_bytes, void *stream);
 constexpr int READ_SIMT_DYN_SMEM = (32 * (RANK + 1) + 8 * 32 * 33) * 4;
 inline int pre_mix_smem(int B) { return (B * 2 * RANK + RANK + 32 * (2 * RANK + 1) + B * 32) * 4; }
+// k_pre_mix after k_pre_tc, whose partials already carry W_in (folded): the
+// block's h and g slot values of the 32 channels, and P
+inline int pre_mix_smem_folded(int B) { return 3 * B * 32 * 4; }
 
 }  // namespace xp

@@ -1,10 +1,12 @@
 // pre_tc.cu -- the hidden projection of Fuse on tcgen05 for large batches.
 //
-// U[t][o] = sum_k h[t][k] W[o][k] with W = [W_h ; W_g] (Sec. 4.1, Eq. fuse: the
-// h and g slots before W_in; g's slot is the block mean of W_g h_k, taken by
-// the Fuse/Mix precompute).  bf16 operands (exact products), fp32
-// accumulation in TMEM; each CTA computes one 128-token x 256-row tile over
-// one K-slice and writes it as a split-K partial Upart[slice][t][o].
+// U[t][o] = sum_k h[t][k] F[o][k] with F = [W_in[:, 0:r] W_h ; W_in[:, r:2r] W_g]
+// (Sec. 4.1, Eq. fuse: Fuse is linear, so the h and g slots are folded through
+// W_in once per refiner; g's slot is the block mean of F_g h_k, taken by the
+// Fuse/Mix precompute).  F is stored as two bf16 terms hi + lo, run as a
+// doubled K loop into the same accumulator: bf16 operands (exact products),
+// fp32 accumulation in TMEM.  Each CTA computes one 128-token x 256-row tile
+// over one K-slice and writes it as a split-K partial Upart[slice][t][o].
 //
 // Roles (320 threads): warp 0 TMA producer (a 4-stage ring of h and W
 // K-chunks), warp 1 TMEM allocator and MMA issuer, warps 2-9 epilogue
@@ -38,7 +40,7 @@ const size_t kPreTcSmemBytes = 1024 + PT_STAGES * PT_STAGE + sizeof(PtShared);
 
 __global__ void __launch_bounds__(320, 1)
     k_pre_tc(const Params *__restrict__ pp, const __grid_constant__ CUtensorMap tmap_h,
-             const __grid_constant__ CUtensorMap tmap_wh, const __grid_constant__ CUtensorMap tmap_wg, int kslice)
+             const __grid_constant__ CUtensorMap tmap_fhi, const __grid_constant__ CUtensorMap tmap_flo, int kslice)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -47,8 +49,7 @@ __global__ void __launch_bounds__(320, 1)
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const int t0 = blockIdx.x * PT_BM, which = blockIdx.y, ks = blockIdx.z;
     const int kb = ks * kslice, ke = min(p.H, kb + kslice);
-    const int nch = (ke - kb + PT_BK - 1) / PT_BK;
-    const CUtensorMap *tmap_w = which ? &tmap_wg : &tmap_wh;
+    const int nch = (ke - kb + PT_BK - 1) / PT_BK;         // K-chunks of the slice, each taken twice (hi, lo)
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < PT_STAGES; ++i) { mbar_init(&sh.full[i], 1); mbar_init(&sh.empty[i], 1); }
@@ -66,16 +67,18 @@ __global__ void __launch_bounds__(320, 1)
     if (warp == 0) {
         if (lane == 0) {
             tma_prefetch_desc(&tmap_h);
-            tma_prefetch_desc(tmap_w);
+            tma_prefetch_desc(&tmap_fhi);
+            tma_prefetch_desc(&tmap_flo);
             uint32_t pending = 0, pend_par = 0;
-            for (int c = 0; c < nch; ++c) {
+            for (int c = 0; c < 2 * nch; ++c) {
                 const int st = c % PT_STAGES;
                 const uint32_t ph = (uint32_t)((c / PT_STAGES) & 1);
                 if (!mbar_wait(&sh.empty[st], ph ^ 1, abort)) break;
                 uint8_t *sa = base + st * PT_STAGE;
                 mbar_expect_tx(&sh.full[st], PT_STAGE);
-                tma_load_2d(sa, &tmap_h, &sh.full[st], kb + c * PT_BK, t0);
-                tma_load_2d(sa + PT_A_STAGE, tmap_w, &sh.full[st], kb + c * PT_BK, 0);
+                const int kc = kb + (c % nch) * PT_BK;
+                tma_load_2d(sa, &tmap_h, &sh.full[st], kc, t0);
+                tma_load_2d(sa + PT_A_STAGE, c < nch ? &tmap_fhi : &tmap_flo, &sh.full[st], kc, which * RANK);
                 pending |= 1u << st;
                 pend_par = (pend_par & ~(1u << st)) | (ph << st);
             }
@@ -87,7 +90,7 @@ __global__ void __launch_bounds__(320, 1)
     } else if (warp == 1) {
         if (lane == 0) {
             bool ok = true;
-            for (int c = 0; c < nch && ok; ++c) {
+            for (int c = 0; c < 2 * nch && ok; ++c) {
                 const int st = c % PT_STAGES;
                 if (!mbar_wait(&sh.full[st], (uint32_t)((c / PT_STAGES) & 1), abort)) { ok = false; break; }
                 tc_fence_after();

@@ -240,79 +240,103 @@ __global__ void __launch_bounds__(256) k_pre_mix(const Params *__restrict__ pp)
     const Params &p = *pp;
     extern __shared__ float sm[];
     const int B = p.B, s = blockIdx.x, d0 = blockIdx.y * 32;
-    float *U = sm;                         // [B][2r]   W_h h_k | W_g h_k
-    float *ug = U + B * 2 * RANK;          // [r]       W_g g
-    float *Ws = ug + RANK;                 // [32][2r + 1]  W_in[d0 + dd][0:2r]
-    float *P = Ws + 32 * (2 * RANK + 1);   // [B][32]   P for this channel slice
     const size_t tok0 = (size_t)s * B;
-    if (p.dtype) {
-        constexpr int PER = 32 * 2 * RANK / 8 / 256;   // 8 16-byte pieces per thread
-        uint4 wv[PER];
-#pragma unroll
-        for (int q = 0; q < PER; ++q) {
-            const int i = threadIdx.x + 256 * q, dd = i / (2 * RANK / 8), c = i % (2 * RANK / 8);
-            wv[q] = __ldg(reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.W_in) +
-                                                          (size_t)(d0 + dd) * 3 * RANK) + c);
-        }
-#pragma unroll
-        for (int q = 0; q < PER; ++q) {
-            const int i = threadIdx.x + 256 * q, dd = i / (2 * RANK / 8), c = i % (2 * RANK / 8);
-            float x[8];
-            bf16x8_to_f32(wv[q], x);
-#pragma unroll
-            for (int j = 0; j < 8; ++j) Ws[dd * (2 * RANK + 1) + 8 * c + j] = x[j];
-        }
-    } else {
-        for (int i = threadIdx.x; i < 32 * 2 * RANK; i += blockDim.x) {
-            const int dd = i / (2 * RANK), e = i % (2 * RANK);
-            Ws[dd * (2 * RANK + 1) + e] = ld_any(p.W_in, p.dtype, (size_t)(d0 + dd) * 3 * RANK + e);
-        }
-    }
-    {
-        // U = sum of the K-slice partials; each thread issues its loads as one batch
+    float *P;                              // [B][32]   P for this channel slice
+    if (p.pre_folded) {
+        // the partials already are h F^T: P_k = F_h h_k + mean_j F_g h_j for
+        // the 32 channels (the h slot at column d, the g slot at r + d)
+        float *Uh = sm, *Ug = Uh + B * 32;
+        P = Ug + B * 32;
         const int ks = p.ksplit, NN = p.N;
-        const float *up = p.Upart + tok0 * 2 * RANK;
-        for (int i0 = 0; i0 < B * 2 * RANK; i0 += 8 * 256) {
-            float v[8];
+        for (int i = threadIdx.x; i < B * 64; i += blockDim.x) {
+            const int k = i / 64, c = i % 64, slot = c / 32, dd = c % 32;
+            const float *up = p.Upart + (tok0 + k) * 2 * RANK + slot * RANK + d0 + dd;
+            float v = 0.0f;
+            for (int z = 0; z < ks; ++z) v += __ldcg(up + (size_t)z * NN * 2 * RANK);
+            (slot ? Ug : Uh)[k * 32 + dd] = v;
+        }
+        __syncthreads();
+        for (int i = threadIdx.x; i < B * 32; i += blockDim.x) {
+            const int k = i / 32, dd = i % 32;
+            float gs = 0.0f;
+            for (int j = 0; j < B; ++j) gs += Ug[j * 32 + dd];
+            P[k * 32 + dd] = Uh[k * 32 + dd] + gs / (float)B;
+        }
+        __syncthreads();
+    } else {
+        float *U = sm;                         // [B][2r]   W_h h_k | W_g h_k
+        float *ug = U + B * 2 * RANK;          // [r]       W_g g
+        float *Ws = ug + RANK;                 // [32][2r + 1]  W_in[d0 + dd][0:2r]
+        P = Ws + 32 * (2 * RANK + 1);
+        if (p.dtype) {
+            constexpr int PER = 32 * 2 * RANK / 8 / 256;   // 8 16-byte pieces per thread
+            uint4 wv[PER];
 #pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                const int i = i0 + q * 256 + threadIdx.x;
-                v[q] = i < B * 2 * RANK ? up[i] : 0.0f;
+            for (int q = 0; q < PER; ++q) {
+                const int i = threadIdx.x + 256 * q, dd = i / (2 * RANK / 8), c = i % (2 * RANK / 8);
+                wv[q] = __ldg(reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.W_in) +
+                                                              (size_t)(d0 + dd) * 3 * RANK) + c);
             }
-            for (int z = 1; z < ks; ++z)
+#pragma unroll
+            for (int q = 0; q < PER; ++q) {
+                const int i = threadIdx.x + 256 * q, dd = i / (2 * RANK / 8), c = i % (2 * RANK / 8);
+                float x[8];
+                bf16x8_to_f32(wv[q], x);
+#pragma unroll
+                for (int j = 0; j < 8; ++j) Ws[dd * (2 * RANK + 1) + 8 * c + j] = x[j];
+            }
+        } else {
+            for (int i = threadIdx.x; i < 32 * 2 * RANK; i += blockDim.x) {
+                const int dd = i / (2 * RANK), e = i % (2 * RANK);
+                Ws[dd * (2 * RANK + 1) + e] = ld_any(p.W_in, p.dtype, (size_t)(d0 + dd) * 3 * RANK + e);
+            }
+        }
+        {
+            // U = sum of the K-slice partials; each thread issues its loads as one batch
+            const int ks = p.ksplit, NN = p.N;
+            const float *up = p.Upart + tok0 * 2 * RANK;
+            for (int i0 = 0; i0 < B * 2 * RANK; i0 += 8 * 256) {
+                float v[8];
 #pragma unroll
                 for (int q = 0; q < 8; ++q) {
                     const int i = i0 + q * 256 + threadIdx.x;
-                    if (i < B * 2 * RANK) v[q] += up[(size_t)z * NN * 2 * RANK + i];
+                    v[q] = i < B * 2 * RANK ? up[i] : 0.0f;
                 }
+                for (int z = 1; z < ks; ++z)
 #pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                const int i = i0 + q * 256 + threadIdx.x;
-                if (i < B * 2 * RANK) U[i] = v[q];
+                    for (int q = 0; q < 8; ++q) {
+                        const int i = i0 + q * 256 + threadIdx.x;
+                        if (i < B * 2 * RANK) v[q] += up[(size_t)z * NN * 2 * RANK + i];
+                    }
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    const int i = i0 + q * 256 + threadIdx.x;
+                    if (i < B * 2 * RANK) U[i] = v[q];
+                }
             }
         }
-    }
-    __syncthreads();
-    for (int e = threadIdx.x; e < RANK; e += blockDim.x) {
-        float acc = 0.0f;
-        for (int k = 0; k < B; ++k) acc += U[k * 2 * RANK + RANK + e];
-        ug[e] = acc / (float)B;
-    }
-    __syncthreads();
-    // P[k][d] = sum_e W_in[d][e] u_h,k[e] + sum_e W_in[d][r + e] u_g[e]
-    {
-        const int dd = threadIdx.x % 32, kg = threadIdx.x / 32;
-        const float *w = Ws + dd * (2 * RANK + 1);
-        float gpart = 0.0f;
-        for (int e = 0; e < RANK; ++e) gpart = fmaf(w[RANK + e], ug[e], gpart);
-        for (int k = kg; k < B; k += 8) {
-            float acc = gpart;
-            const float *u = U + k * 2 * RANK;
-            for (int e = 0; e < RANK; ++e) acc = fmaf(w[e], u[e], acc);
-            P[k * 32 + dd] = acc;
+        __syncthreads();
+        for (int e = threadIdx.x; e < RANK; e += blockDim.x) {
+            float acc = 0.0f;
+            for (int k = 0; k < B; ++k) acc += U[k * 2 * RANK + RANK + e];
+            ug[e] = acc / (float)B;
         }
+        __syncthreads();
+        // P[k][d] = sum_e W_in[d][e] u_h,k[e] + sum_e W_in[d][r + e] u_g[e]
+        {
+            const int dd = threadIdx.x % 32, kg = threadIdx.x / 32;
+            const float *w = Ws + dd * (2 * RANK + 1);
+            float gpart = 0.0f;
+            for (int e = 0; e < RANK; ++e) gpart = fmaf(w[RANK + e], ug[e], gpart);
+            for (int k = kg; k < B; k += 8) {
+                float acc = gpart;
+                const float *u = U + k * 2 * RANK;
+                for (int e = 0; e < RANK; ++e) acc = fmaf(w[e], u[e], acc);
+                P[k * 32 + dd] = acc;
+            }
+        }
+        __syncthreads();
     }
-    __syncthreads();
     // Pc = (I + L) P, channel by channel (Eq. mix)
     for (int i = threadIdx.x; i < B * 32; i += blockDim.x) {
         const int k = i / 32, dd = i % 32, d = d0 + dd;

@@ -87,12 +87,13 @@ struct xpress_refiner {
     unsigned long long *trace = nullptr;   // profiling timeline (XPRESS_TRACE=1)
     CUtensorMap tmap_wr{};                 // W_r boxes of 256 rows (k_read_tc)
     CUtensorMap tmap_wr128{};              // W_r boxes of 128 rows (k_read_tcv)
-    CUtensorMap tmap_wh{}, tmap_wg{};      // W_h, W_g boxes of 256 rows x 64 (k_pre_tc)
+    CUtensorMap tmap_wh{}, tmap_wg{};      // W_h, W_g boxes of 256 rows x 64
+    CUtensorMap tmap_fhi{}, tmap_flo{};    // folded projection, hi / lo term, boxes of 256 rows x 64 (k_pre_tc)
     int device = 0;
     int num_sms = 0;
     bool use_tc = false;
     cudaStream_t cs = nullptr;
-    uint16_t *Fhl = nullptr;               // [2][2r, H] folded hidden projection, bf16 hi / lo (small-batch kernel)
+    uint16_t *Fhl = nullptr;               // [2][2r, H] folded hidden projection, bf16 hi / lo (bf16 refiners)
     uint16_t *Lpk = nullptr;               // [B(B-1)/2, r] L's strictly lower part, channel innermost
     bool small_ok = false;                 // the small-batch kernel can run co-resident on this GPU
     void *small_ws[CACHE_SLOTS] = {};      // workspaces whose control area this refiner has cleared
@@ -251,6 +252,7 @@ Params make_params(const xpress_refiner *R, const xpress_block_in *in, const xpr
     P.ctl = reinterpret_cast<int32_t *>(w + L.ctl);
     P.st = reinterpret_cast<SeqState *>(w + L.st);
     P.Upart = reinterpret_cast<float *>(w + L.upart);
+    P.pre_folded = L.pre_tc ? 1 : 0;
     P.Pc = reinterpret_cast<float *>(w + L.pc);
     P.Ynew = reinterpret_cast<int32_t *>(w + L.ynew);
     P.act_tok = reinterpret_cast<int32_t *>(w + L.acttok);
@@ -339,8 +341,8 @@ struct PreTcArgs {
     bool make(const xpress_refiner *R, const Params &P, const Layout &L, Params *pd)
     {
         pdev = pd;
-        wh = R->tmap_wh;
-        wg = R->tmap_wg;
+        wh = R->tmap_fhi;
+        wg = R->tmap_flo;
         kslice = L.kchunk;
         ptrs[0] = &pdev; ptrs[1] = &th; ptrs[2] = &wh; ptrs[3] = &wg; ptrs[4] = &kslice;
         return make_tmap_bf16(&th, P.h, (uint64_t)P.H, (uint64_t)P.N, 64, 128);
@@ -422,7 +424,7 @@ int build_graph(xpress_refiner *R, GraphEntry &e, const Params &P, const Layout 
     XP_CUDA(cudaStreamBeginCaptureToGraph(cs, g, &cap_dep, nullptr, 1, cudaStreamCaptureModeThreadLocal));
     if (!P.draft) k_rowmax<<<N, 256, 0, cs>>>(pdev);
     if (!L.pre_tc) launch_pre_gemm(L, N, pdev, cs);
-    k_pre_mix<<<dim3(b, RANK / 32), 256, pre_mix_smem(P.B), cs>>>(pdev);
+    k_pre_mix<<<dim3(b, RANK / 32), 256, L.pre_tc ? pre_mix_smem_folded(P.B) : pre_mix_smem(P.B), cs>>>(pdev);
     cudaStreamCaptureStatus cst;
     const cudaGraphNode_t *deps = nullptr;
     size_t ndeps = 0;
@@ -544,7 +546,7 @@ int run_eager(xpress_refiner *R, Params P, const Layout &L, void *ws, cudaStream
     }
     kt.stop();
     kt.start("pre_mix");
-    k_pre_mix<<<dim3(b, RANK / 32), 256, pre_mix_smem(P.B), st>>>(pdev);
+    k_pre_mix<<<dim3(b, RANK / 32), 256, L.pre_tc ? pre_mix_smem_folded(P.B) : pre_mix_smem(P.B), st>>>(pdev);
     kt.stop();
     for (int pass = 0; pass < P.K_max; ++pass) {
         kt.start("mix_mlp");
@@ -723,14 +725,21 @@ int xpress_refiner_create(const xpress_weights *w, void *stream, xpress_refiner 
                 (void)cudaGetLastError();
                 coop = 0;
             }
+            // the folded hidden projection (both the persistent kernel and
+            // k_pre_tc take it)
+            if (cudaMalloc(&R->Fhl, (size_t)2 * 2 * RANK * w->H * sizeof(uint16_t)) != cudaSuccess) {
+                rc = XPRESS_ERR_CUDA;
+                break;
+            }
+            k_fold_hidden<<<dim3((w->H + 255) / 256, 2 * RANK / 8), 256, 0, st>>>(
+                static_cast<const uint16_t *>(w->W_h), static_cast<const uint16_t *>(w->W_g),
+                static_cast<const uint16_t *>(w->W_in), R->Fhl, w->H);
+            if (!make_tmap_bf16(&R->tmap_fhi, R->Fhl, (uint64_t)w->H, 2 * RANK, 64, 256) ||
+                !make_tmap_bf16(&R->tmap_flo, R->Fhl + (size_t)2 * RANK * w->H, (uint64_t)w->H, 2 * RANK, 64, 256)) {
+                rc = XPRESS_ERR_CUDA;
+                break;
+            }
             if (coop && per_sm >= 1 && R->num_sms > SMALL_TRANS_CTAS) {
-                if (cudaMalloc(&R->Fhl, (size_t)2 * 2 * RANK * w->H * sizeof(uint16_t)) != cudaSuccess) {
-                    rc = XPRESS_ERR_CUDA;
-                    break;
-                }
-                k_fold_hidden<<<dim3((w->H + 255) / 256, 2 * RANK / 8), 256, 0, st>>>(
-                    static_cast<const uint16_t *>(w->W_h), static_cast<const uint16_t *>(w->W_g),
-                    static_cast<const uint16_t *>(w->W_in), R->Fhl, w->H);
                 const int tri = w->B * (w->B - 1) / 2;
                 if (cudaMalloc(&R->Lpk, (size_t)(tri > 0 ? tri : 1) * RANK * 2) != cudaSuccess) {
                     rc = XPRESS_ERR_CUDA;
