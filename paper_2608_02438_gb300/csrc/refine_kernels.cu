@@ -341,9 +341,16 @@ __global__ void __launch_bounds__(256) k_pre_mix(const Params *__restrict__ pp)
     for (int i = threadIdx.x; i < B * 32; i += blockDim.x) {
         const int k = i / 32, dd = i % 32, d = d0 + dd;
         float lrow[MAX_B];
-        const size_t lb = ((size_t)d * B + k) * B;
+        if (p.Lpk) {
+            // packed L: a warp's 32 channels of one (k, j) are 64 contiguous bytes
+            const uint16_t *lp = p.Lpk + (size_t)(k * (k - 1) / 2) * RANK + d;
 #pragma unroll
-        for (int j = 0; j < MAX_B; ++j) lrow[j] = j < k ? ld_any(p.L, p.dtype, lb + j) : 0.0f;
+            for (int j = 0; j < MAX_B; ++j) lrow[j] = j < k ? bf2f(lp[(size_t)j * RANK]) : 0.0f;
+        } else {
+            const size_t lb = ((size_t)d * B + k) * B;
+#pragma unroll
+            for (int j = 0; j < MAX_B; ++j) lrow[j] = j < k ? ld_any(p.L, p.dtype, lb + j) : 0.0f;
+        }
         float acc = P[k * 32 + dd];
 #pragma unroll
         for (int j = 0; j < MAX_B; ++j)
@@ -576,7 +583,7 @@ __device__ __forceinline__ void mlp_share_mma(const Params &p, cg::cluster_group
 // grid (8, b), cluster (8, 1, 1), 256 threads.  CTA `rank` of block s owns
 // channels [32 rank, +32) of c and z, and rows [64 rank, +64) of W_1; c and
 // sigma(W_1 c) are exchanged through distributed shared memory.
-__global__ void __cluster_dims__(MLP_CLUSTER, 1, 1) __launch_bounds__(256) k_mix_mlp(const Params *__restrict__ pp)
+__global__ void __cluster_dims__(MLP_CLUSTER, 1, 1) __launch_bounds__(256, 2) k_mix_mlp(const Params *__restrict__ pp)
 {
     const unsigned long long t_start = globaltimer_ns();
     pdl_trigger();                     // the Read kernel may start its prologue
@@ -612,9 +619,15 @@ __global__ void __cluster_dims__(MLP_CLUSTER, 1, 1) __launch_bounds__(256) k_mix
     for (int i = threadIdx.x; i < cnt * 32; i += blockDim.x) {
         const int t = i / 32, dd = i % 32, k = m + 1 + t, d = d0 + dd;
         float lrow[MAX_B];
-        const size_t lb = ((size_t)d * B + k) * B;
+        if (p.Lpk) {
+            const uint16_t *lp = p.Lpk + (size_t)(k * (k - 1) / 2) * RANK + d;
 #pragma unroll
-        for (int j = 0; j < MAX_B; ++j) lrow[j] = j < k ? ld_any(p.L, p.dtype, lb + j) : 0.0f;
+            for (int j = 0; j < MAX_B; ++j) lrow[j] = j < k ? bf2f(lp[(size_t)j * RANK]) : 0.0f;
+        } else {
+            const size_t lb = ((size_t)d * B + k) * B;
+#pragma unroll
+            for (int j = 0; j < MAX_B; ++j) lrow[j] = j < k ? ld_any(p.L, p.dtype, lb + j) : 0.0f;
+        }
         float acc = p.Pc[((size_t)s * B + k) * RANK + d] + e[k][dd];
 #pragma unroll
         for (int j = 0; j < MAX_B; ++j)

@@ -253,6 +253,7 @@ Params make_params(const xpress_refiner *R, const xpress_block_in *in, const xpr
     P.st = reinterpret_cast<SeqState *>(w + L.st);
     P.Upart = reinterpret_cast<float *>(w + L.upart);
     P.pre_folded = L.pre_tc ? 1 : 0;
+    P.Lpk = R->Lpk;                        // null for fp32 refiners
     P.Pc = reinterpret_cast<float *>(w + L.pc);
     P.Ynew = reinterpret_cast<int32_t *>(w + L.ynew);
     P.act_tok = reinterpret_cast<int32_t *>(w + L.acttok);
@@ -266,7 +267,6 @@ Params make_params(const xpress_refiner *R, const xpress_block_in *in, const xpr
         P.cx = reinterpret_cast<uint16_t *>(w + L.cx);
         P.ux = reinterpret_cast<uint16_t *>(w + L.ux);
         P.pcx = reinterpret_cast<float *>(w + L.pcx);
-        P.Lpk = R->Lpk;
         P.rmax = reinterpret_cast<Partial *>(w + L.rmax);
         P.sctl = reinterpret_cast<SmallCtlArea *>(w + L.sctl);
         P.best64 = reinterpret_cast<unsigned long long *>(w + L.best64);
@@ -739,16 +739,15 @@ int xpress_refiner_create(const xpress_weights *w, void *stream, xpress_refiner 
                 rc = XPRESS_ERR_CUDA;
                 break;
             }
-            if (coop && per_sm >= 1 && R->num_sms > SMALL_TRANS_CTAS) {
-                const int tri = w->B * (w->B - 1) / 2;
-                if (cudaMalloc(&R->Lpk, (size_t)(tri > 0 ? tri : 1) * RANK * 2) != cudaSuccess) {
-                    rc = XPRESS_ERR_CUDA;
-                    break;
-                }
-                if (tri > 0)
-                    k_pack_L<<<(tri + 7) / 8, 256, 0, st>>>(static_cast<const uint16_t *>(w->L), R->Lpk, w->B);
-                R->small_ok = true;
+            // L's strictly lower part, channel innermost (coalesced mixes)
+            const int tri = w->B * (w->B - 1) / 2;
+            if (cudaMalloc(&R->Lpk, (size_t)(tri > 0 ? tri : 1) * RANK * 2) != cudaSuccess) {
+                rc = XPRESS_ERR_CUDA;
+                break;
             }
+            if (tri > 0)
+                k_pack_L<<<(tri + 7) / 8, 256, 0, st>>>(static_cast<const uint16_t *>(w->L), R->Lpk, w->B);
+            if (coop && per_sm >= 1 && R->num_sms > SMALL_TRANS_CTAS) R->small_ok = true;
         }
         if (cudaGetLastError() != cudaSuccess || cudaStreamSynchronize(st) != cudaSuccess) rc = XPRESS_ERR_CUDA;
     } while (0);
