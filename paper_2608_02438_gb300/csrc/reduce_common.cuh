@@ -84,20 +84,40 @@ __device__ __forceinline__ void draw_in_group(const Params &p, int i, int tok, i
     const int lane = threadIdx.x % 32, k = tok % p.B;
     const int v = g * GROUP + lane;
     float x = -INFINITY, score = -INFINITY;
-    if (v < p.V) {
-        float acc = 0.0f;
-        if (p.dtype) {
-            const uint4 *wr = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.W_r) + (size_t)v * RANK);
-            const uint4 *zr = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.zpack) + (size_t)i * RANK);
-#pragma unroll 8
-            for (int c = 0; c < RANK / 8; ++c) {
-                float w8[8], z8[8];
-                bf16x8_to_float(__ldg(wr + c), w8);
-                bf16x8_to_float(__ldcg(zr + c), z8);
+    float acc_bf = 0.0f;
+    if (p.dtype) {
+        // the warp takes the group's rows one at a time: lane l holds z[8l ..
+        // 8l + 7] and the same slice of the row (one coalesced 512-byte row
+        // per load), the partial products meet through shuffles
+        float z8[8];
+        bf16x8_to_float(__ldcg(reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.zpack) +
+                                                               (size_t)i * RANK) + lane), z8);
+        const uint16_t *wr0 = static_cast<const uint16_t *>(p.W_r);
+#pragma unroll 1
+        for (int r0 = 0; r0 < GROUP; r0 += 8) {
+            uint4 w[8];
 #pragma unroll
-                for (int j = 0; j < 8; ++j) acc = fmaf(w8[j], z8[j], acc);
+            for (int u = 0; u < 8; ++u) {
+                const int row = g * GROUP + r0 + u;
+                w[u] = row < p.V ? __ldg(reinterpret_cast<const uint4 *>(wr0 + (size_t)row * RANK) + lane)
+                                 : make_uint4(0, 0, 0, 0);
             }
-        } else {
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                float w8[8];
+                bf16x8_to_float(w[u], w8);
+                float part = 0.0f;
+#pragma unroll
+                for (int j = 0; j < 8; ++j) part = fmaf(w8[j], z8[j], part);
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+                if (lane == r0 + u) acc_bf = part;
+            }
+        }
+    }
+    if (v < p.V) {
+        float acc = acc_bf;
+        if (!p.dtype) {
             for (int d = 0; d < RANK; ++d)
                 acc = fmaf(ld_any(p.W_r, 0, (size_t)v * RANK + d), ld_any(p.zpack, 0, (size_t)i * RANK + d), acc);
         }
