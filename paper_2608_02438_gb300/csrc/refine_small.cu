@@ -357,16 +357,22 @@ __device__ __forceinline__ void rowmax_item(const Params &p, int item, int lane)
 
 // ------------------------------------------------------------- Read role
 
-__device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUtensorMap *tmap_z, SmallCtl *c,
+__device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUtensorMap *tmap_wr32,
+                                          const CUtensorMap *tmap_z, SmallCtl *c,
                           uint8_t *base, unsigned long long t_start)
 {
     uint8_t *sA = base;                                    // W_r stages (h slices before the first pass)
     uint8_t *sZ = base + TV_STAGES * TV_A_STAGE;           // z, 4 K-chunks
     RsShared &sh = *reinterpret_cast<RsShared *>(sZ + TV_Z_BYTES);
     const int V = p.V, S = p.S, r = blockIdx.x, N = p.N, B = p.B;
-    const int NVB = (V + TV_BM - 1) / TV_BM;
-    const int vb0 = (int)((long long)NVB * r / S), vb1 = (int)((long long)NVB * (r + 1) / S);
-    const int nblk = vb1 - vb0;                            // >= 1: S <= NVB
+    // vocabulary rows [R0, R1), cut at 32-row granularity so that the ranges
+    // differ by at most 32 rows; 128-row blocks, the last one possibly partial
+    // (its quarters come by 32-row boxes)
+    const int NQ = (V + 31) / 32;
+    const int R0 = 32 * (int)((long long)NQ * r / S);
+    const int R1 = min(32 * (int)((long long)NQ * (r + 1) / S), V);
+    const int nblk = (R1 - R0 + TV_BM - 1) / TV_BM;        // >= 1: S <= V / 128
+    const int last_q = (R1 - R0 - (nblk - 1) * TV_BM + 31) / 32;   // quarters of the last block (1..4)
     const int per_pass = nblk * TV_KCH;                    // W_r chunks per pass
     const int ahead = min(TV_STAGES, per_pass);
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
@@ -432,10 +438,18 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
                 const int stage = (int)(ci % TV_STAGES);
                 const uint32_t ph = (uint32_t)((ci / TV_STAGES) & 1);
                 if (!mbar_wait(&sh.empty[stage], ph ^ 1, abort)) return false;
-                const int within = (int)(ci % per_pass);
-                mbar_expect_tx(&sh.full[stage], TV_A_STAGE);
-                tma_load_2d_hint(sA + stage * TV_A_STAGE, tmap_wr, &sh.full[stage], (within % TV_KCH) * TV_BK,
-                                 (vb0 + within / TV_KCH) * TV_BM, keep);
+                const int within = (int)(ci % per_pass), blk = within / TV_KCH, kx = (within % TV_KCH) * TV_BK;
+                if (blk == nblk - 1 && last_q < 4) {
+                    // partial last block: its quarters only (the MMA's other rows
+                    // are stale and the epilogue leaves them out)
+                    mbar_expect_tx(&sh.full[stage], (uint32_t)last_q * (TV_A_STAGE / 4));
+                    for (int qq = 0; qq < last_q; ++qq)
+                        tma_load_2d_hint(sA + stage * TV_A_STAGE + qq * (TV_A_STAGE / 4), tmap_wr32, &sh.full[stage], kx,
+                                         R0 + blk * TV_BM + 32 * qq, keep);
+                } else {
+                    mbar_expect_tx(&sh.full[stage], TV_A_STAGE);
+                    tma_load_2d_hint(sA + stage * TV_A_STAGE, tmap_wr, &sh.full[stage], kx, R0 + blk * TV_BM, keep);
+                }
                 pending |= 1u << stage;
                 pend_par = (pend_par & ~(1u << stage)) | (ph << stage);
                 return true;
@@ -447,8 +461,8 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
                 for (; next < ahead && ok; ++next) ok = issue(next);
             // while the first Trans runs, the rest of this CTA's W_r range
             // (past the chunks the ring holds) goes into L2 a slice at a time
-            const int pf_row0 = vb0 * TV_BM + (lookahead ? ahead / TV_KCH : 0) * TV_BM;
-            const int pf_rows = max(0, min(vb1 * TV_BM, V) - pf_row0);
+            const int pf_row0 = R0 + (lookahead ? ahead / TV_KCH : 0) * TV_BM;
+            const int pf_rows = max(0, R1 - pf_row0);
             const uint32_t pf_bytes = (p.read_flags & 1) ? 0u : (uint32_t)pf_rows * RANK * 2;
             for (int pass = 0; ok; ++pass) {
                 const bool go = pass == 0
@@ -560,11 +574,11 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
             sel.init();
             bool ok = true;
             uint4 cur[4], nxt[4];
-            if (half < nblk) load_s_group(cur, srow, (vb0 + half) * TV_BM + q * 32, V, tvalid);
+            if (half < nblk) load_s_group(cur, srow, R0 + half * TV_BM + q * 32, V, tvalid);
             for (int i = half; i < nblk; i += 2) {
                 const int ib = pass * nblk + i, buf = ib % TV_NBUF;
-                const int v0 = (vb0 + i) * TV_BM + q * 32;
-                if (i + 2 < nblk) load_s_group(nxt, srow, (vb0 + i + 2) * TV_BM + q * 32, V, tvalid);
+                const int v0 = R0 + i * TV_BM + q * 32;
+                if (i + 2 < nblk) load_s_group(nxt, srow, R0 + (i + 2) * TV_BM + q * 32, V, tvalid);
                 if (!mbar_wait(&sh.tfull[buf], (uint32_t)((ib / TV_NBUF) & 1), abort)) { ok = false; break; }
                 tc_fence_after();
                 float acc[TV_BN];
@@ -575,7 +589,7 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
 #pragma unroll
                 for (int t2 = 0; t2 < TV_BN; ++t2) tile[t2][lane] = acc[t2];
                 __syncwarp();
-                const int nv = min(GROUP, V - v0);
+                const int nv = min(GROUP, R1 - v0);                // rows of this CTA's range
                 if (tvalid && nv > 0) {
                     float l[GROUP];
 #pragma unroll
@@ -1175,7 +1189,7 @@ const size_t kRefineSmallSmemBytes = SMALL_SMEM;
 // registers per thread).
 __global__ void __launch_bounds__(TV_THREADS, 1)
     k_refine_small(const __grid_constant__ Params p, const __grid_constant__ CUtensorMap tmap_wr128,
-                   const __grid_constant__ CUtensorMap tmap_z)
+                   const __grid_constant__ CUtensorMap tmap_wr32, const __grid_constant__ CUtensorMap tmap_z)
 {
     const unsigned long long t_start = globaltimer_ns();
     // a kernel launched after this one with programmatic dependent launch may
@@ -1192,7 +1206,7 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
         CtlLine *nxt = reinterpret_cast<CtlLine *>(&area->blk[par ^ 1]);
         nxt[threadIdx.x].v = 0;
     }
-    if ((int)blockIdx.x < p.S) read_role(p, &tmap_wr128, &tmap_z, c, base, t_start);
+    if ((int)blockIdx.x < p.S) read_role(p, &tmap_wr128, &tmap_wr32, &tmap_z, c, base, t_start);
     else trans_role(p, c, base, t_start);
     __syncthreads();
     if (threadIdx.x == 0) leave(p, area, c, par);

@@ -86,7 +86,8 @@ struct xpress_refiner {
     float *Ep = nullptr;
     unsigned long long *trace = nullptr;   // profiling timeline (XPRESS_TRACE=1)
     CUtensorMap tmap_wr{};                 // W_r boxes of 256 rows (k_read_tc)
-    CUtensorMap tmap_wr128{};              // W_r boxes of 128 rows (k_read_tcv)
+    CUtensorMap tmap_wr128{};              // W_r boxes of 128 rows (k_read_tcv, k_refine_small)
+    CUtensorMap tmap_wr32{};               // W_r boxes of 32 rows (k_refine_small, partial blocks)
     CUtensorMap tmap_wh{}, tmap_wg{};      // W_h, W_g boxes of 256 rows x 64
     CUtensorMap tmap_fhi{}, tmap_flo{};    // folded projection, hi / lo term, boxes of 256 rows x 64 (k_pre_tc)
     int device = 0;
@@ -605,7 +606,7 @@ int run_small(xpress_refiner *R, const Params &P, const Layout &L, void *ws, cud
     cfg.stream = st;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    XP_CUDA(cudaLaunchKernelEx(&cfg, k_refine_small, P, R->tmap_wr128, tmap_z));
+    XP_CUDA(cudaLaunchKernelEx(&cfg, k_refine_small, P, R->tmap_wr128, R->tmap_wr32, tmap_z));
     if (R->trace) print_trace(R, st);
     return XPRESS_OK;
 }
@@ -699,6 +700,7 @@ int xpress_refiner_create(const xpress_weights *w, void *stream, xpress_refiner 
         R->use_tc = w->dtype == XPRESS_BF16;
         if (R->use_tc && (!make_tmap_bf16(&R->tmap_wr, w->W_r, RANK, (uint64_t)w->V, 64, 256) ||
                           !make_tmap_bf16(&R->tmap_wr128, w->W_r, RANK, (uint64_t)w->V, 64, 128) ||
+                          !make_tmap_bf16(&R->tmap_wr32, w->W_r, RANK, (uint64_t)w->V, 64, 32) ||
                           !make_tmap_bf16(&R->tmap_wh, w->W_h, (uint64_t)w->H, RANK, 64, 256) ||
                           !make_tmap_bf16(&R->tmap_wg, w->W_g, (uint64_t)w->H, RANK, 64, 256))) {
             rc = XPRESS_ERR_CUDA;
