@@ -189,6 +189,52 @@ __global__ void __launch_bounds__(256) k_acc_finalize(AcceptParams p, int chunks
     const float lse_q = resid ? p.lse[(size_t)seq * B + k] : 0.0f;
     float rb = -INFINITY, pb = -INFINITY;
     int ri = 0x7fffffff, pi = 0x7fffffff;
+    if (resid && p.dtype) {
+        // bf16: a warp takes 32 rows of W_r at a time, one coalesced 512-byte
+        // row per load (lane l holds z[8l .. 8l + 7] and the same slice of the
+        // row), the partial products meet through shuffles, and lane u keeps
+        // row u's sum for the draw
+        const int lane = threadIdx.x % 32, nw = blockDim.x / 32;
+        float z8[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) z8[j] = zop[8 * lane + j];
+        const uint16_t *wr = static_cast<const uint16_t *>(p.W_r);
+        for (int gb = v0 + (threadIdx.x / 32) * 32; gb < v1; gb += nw * 32) {
+            float myacc = 0.0f;
+#pragma unroll 1
+            for (int u0 = 0; u0 < 32; u0 += 8) {
+                uint4 w[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const int row = gb + u0 + u;
+                    w[u] = row < v1 ? __ldg(reinterpret_cast<const uint4 *>(wr + (size_t)row * RANK) + lane)
+                                    : make_uint4(0, 0, 0, 0);
+                }
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const uint32_t ww[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
+                    float part = 0.0f;
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        part = fmaf(__uint_as_float(ww[q] << 16), z8[2 * q], part);
+                        part = fmaf(__uint_as_float(ww[q] & 0xFFFF0000u), z8[2 * q + 1], part);
+                    }
+#pragma unroll
+                    for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+                    if (lane == u0 + u) myacc = part;
+                }
+            }
+            const int v = gb + lane;
+            if (v < v1) {
+                const float tx = ld_any(p.target, p.dtype, trow * p.V + v) * invT;
+                const float g = gumbel(seed, (uint32_t)v, (uint32_t)k, STREAM_RESID, p.offset);
+                merge_argmax(pb, pi, tx + g, v);
+                const float lx = (myacc + ld_any(p.s, p.dtype, ((size_t)seq * B + k) * p.V + v)) * invT;
+                const float res = expf(tx - lse_p) - expf(lx - lse_q);
+                if (res > 0.0f) merge_argmax(rb, ri, logf(res) + g, v);
+            }
+        }
+    } else
     for (int v = v0 + threadIdx.x; v < v1; v += blockDim.x) {
         const float tx = ld_any(p.target, p.dtype, trow * p.V + v) * invT;
         const float g = gumbel(seed, (uint32_t)v, (uint32_t)k, STREAM_RESID, p.offset);
