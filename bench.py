@@ -52,10 +52,15 @@ def dist_env():
 
 
 def source_hash(paths):
+    """Hash of the kernel sources' code: // comments and blank lines are left
+    out, so that a comment edit does not orphan a profile taken on the code."""
     h = hashlib.sha256()
     for p in paths:
-        with open(os.path.join(ROOT, p), "rb") as f:
-            h.update(f.read())
+        with open(os.path.join(ROOT, p), encoding="utf-8") as f:
+            for line in f:
+                code = line.split("//", 1)[0].rstrip()
+                if code:
+                    h.update(code.encode() + b"\n")
     return h.hexdigest()[:16]
 
 

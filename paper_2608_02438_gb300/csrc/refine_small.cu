@@ -7,23 +7,25 @@
 // of S + 8 CTAs, at most one per SM, so that no pass pays a kernel launch, a
 // graph-node switch or a cold start.
 //
-//   Read CTAs (blockIdx < S).  Before the first pass they compute partial sums
-//     of P_k = F_h h_k + F_g g over K-slices of the folded projection
-//     F = [W_in[:, 0:r] W_h ; W_in[:, r:2r] W_g] (fp32, built once per refiner:
-//     Fuse is linear, and F_g g is the block mean of F_g h_k), and, for a call
-//     without a draft, partial argmaxes of s (Algorithm 1's Y^(0)).  In every
-//     pass they run Read + Correct + selection (Eq. read / correct, the argmax
-//     or the fixed-noise group draw) over a fixed range of 128-row vocabulary
-//     blocks: W_r rows are the tcgen05 M dimension, the <= 32 tokens N, and an
-//     8-stage TMA ring streams W_r, running ahead into the next pass while the
-//     Trans CTAs work.  Each range leaves one partial per token (for T > 0
-//     with the member draw of its best group already taken).
-//   Trans CTAs (S .. S + 7).  CTA j owns channels [32 j, 32 j + 32).  Once per
-//     call they finish Pc = (I + L) P for their channels (Eq. mix); in every
-//     pass they gather E' rows for the current tokens, mix (Eq. fuse / mix) and
-//     run Trans z = c + W_2 sigma(W_1 c) (Eq. mlp) on tensor cores, exchanging
-//     c and sigma(W_1 c) through L2.  Then each of them combines the Read
-//     partials, applies Algorithm 1's stopping rule and packs the next pass
+//   Read CTAs (blockIdx < S).  Before the first pass they compute, per pair of
+//     channels, Pc = (I + L) P with P_k = F_h h_k + F_g g over all of K on
+//     tensor cores, F = [W_in[:, 0:r] W_h ; W_in[:, r:2r] W_g] folded once per
+//     refiner (Fuse is linear, and F_g g is the block mean of F_g h_k) and
+//     stored as bf16 hi + lo terms; with a draft also the first pass's c.
+//     For a call without a draft they compute partial argmaxes of s
+//     (Algorithm 1's Y^(0)).  In every pass they run Read + Correct +
+//     selection (Eq. read / correct, the argmax or the fixed-noise group
+//     draw) over a fixed range of vocabulary rows (128-row blocks): W_r rows
+//     are the tcgen05 M dimension, the <= 32 tokens N, and an 8-stage TMA ring
+//     streams W_r, running ahead into the next pass while the Trans CTAs work.
+//     Each range leaves one result per token (greedy: an argmax key; T > 0: a
+//     partial with the member draw of its best group already taken).
+//   Trans CTAs (S .. S + 7).  CTA j owns channels [32 j, 32 j + 32).  In every
+//     pass they gather E' rows for the current tokens, mix (Eq. fuse / mix;
+//     with blocks of at most 16 positions every Trans CTA forms all of c) and
+//     run Trans z = c + W_2 sigma(W_1 c) (Eq. mlp) on tensor cores,
+//     exchanging sigma(W_1 c) through L2.  Then each of them combines the Read
+//     results, applies Algorithm 1's stopping rule and packs the next pass
 //     (the same result in all eight; the first one publishes it), so the next
 //     pass starts without another hand-off.
 //
