@@ -269,18 +269,34 @@ __global__ void __launch_bounds__(256) k_acc_finalize(AcceptParams p, int chunks
         s_last = atomicAdd(p.ticket + seq, 1) == nch - 1;
     }
     __syncthreads();
-    if (s_last && threadIdx.x == 0) {
-        // every chunk of this block has drawn: combine and emit
-        __threadfence();
-        float cb = -INFINITY, cp = -INFINITY;
-        int ci = 0x7fffffff, cpi = 0x7fffffff;
-        for (int cc = 0; cc < nch; ++cc) {
-            const Partial a = ldcg_partial16(p.spart + (size_t)seq * nch + cc);
-            merge_argmax(cb, ci, a.best, a.idx);
-            merge_argmax(cp, cpi, a.m, __float_as_int(a.s));
-        }
-        const bool use_resid = k < B && cb > -INFINITY;
-        p.out_tokens[(size_t)seq * (B + 1) + k] = use_resid ? ci : cpi;
+    if (!s_last) return;
+    // every chunk of this block has drawn: the last CTA combines the chunks'
+    // results (each thread a share, then the tree above) and emits the token
+    __threadfence();
+    float cb = -INFINITY, cp = -INFINITY;
+    int ci = 0x7fffffff, cpi = 0x7fffffff;
+    for (int cc = threadIdx.x; cc < nch; cc += blockDim.x) {
+        const Partial a = ldcg_partial16(p.spart + (size_t)seq * nch + cc);
+        merge_argmax(cb, ci, a.best, a.idx);
+        merge_argmax(cp, cpi, a.m, __float_as_int(a.s));
+    }
+    sb[0][threadIdx.x] = cb; si[0][threadIdx.x] = ci;
+    sb[1][threadIdx.x] = cp; si[1][threadIdx.x] = cpi;
+    __syncthreads();
+    for (int w = 128; w > 0; w >>= 1) {
+        if (threadIdx.x < w)
+            for (int h = 0; h < 2; ++h) {
+                float b0 = sb[h][threadIdx.x];
+                int i0 = si[h][threadIdx.x];
+                merge_argmax(b0, i0, sb[h][threadIdx.x + w], si[h][threadIdx.x + w]);
+                sb[h][threadIdx.x] = b0;
+                si[h][threadIdx.x] = i0;
+            }
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) {
+        const bool use_resid = k < B && sb[0][0] > -INFINITY;
+        p.out_tokens[(size_t)seq * (B + 1) + k] = use_resid ? si[0][0] : si[1][0];
     }
 }
 
