@@ -133,8 +133,16 @@ __global__ void __launch_bounds__(256) k_acc_finalize(AcceptParams p, int chunks
         for (int k = lane; k <= B; k += 32) {
             Partial a{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
             const size_t r = (size_t)seq * (B + 1) + k;
-#pragma unroll 4
-            for (int cc = 0; cc < chunks; ++cc) merge_partial(a, p.rowpart[r * chunks + cc], sampling);
+            // eight chunks' partials requested together per round
+            for (int c0 = 0; c0 < chunks; c0 += 8) {
+                Partial q[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u)
+                    q[u] = c0 + u < chunks ? ldcg_partial16(p.rowpart + r * chunks + c0 + u)
+                                           : Partial{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
+#pragma unroll
+                for (int u = 0; u < 8; ++u) merge_partial(a, q[u], sampling);
+            }
             rows[k] = a;
         }
         __syncwarp();
