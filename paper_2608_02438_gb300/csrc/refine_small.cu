@@ -771,6 +771,22 @@ __device__ __noinline__ void mix_block16(const float *e, const uint16_t *Lp, con
     }
 }
 
+// gather_e issued as asynchronous copies (one commit group; the caller waits
+// with cp_async_wait<0> before reading e).
+__device__ __forceinline__ void gather_e_async(const Params &p, const int *x, const int *anch, float *e, int CH,
+                                               int cb, int tid, int nth, uint64_t policy)
+{
+    const int N = p.N, B = p.B, V = p.V, total = N * CH / 4;
+    for (int i = tid; i < total; i += nth) {
+        const int j = i / (CH / 4), q = i % (CH / 4), k = j % B, s = j / B;
+        int tk = k == 0 ? anch[s] : x[j - 1];
+        if (tk < 0 || tk >= V) tk = 0;                         // reported at the start
+        cp_async16(reinterpret_cast<float4 *>(e) + i, reinterpret_cast<const float4 *>(p.Ep + (size_t)tk * RANK + cb) + q,
+                   16u, policy);
+    }
+    cp_async_commit();
+}
+
 __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t *base, unsigned long long t_start)
 {
     TsShared &sh = *reinterpret_cast<TsShared *>(base);
@@ -875,6 +891,7 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
 
     float *zf = p.z_final ? p.z_final : p.zbuf;
     uint16_t *zpack = static_cast<uint16_t *>(p.zpack);
+    const uint64_t eprow_policy = policy_evict_first();       // E' rows are read once per pass
     int n = N;                                                 // evaluated tokens of this pass
     for (int pass = 0;; ++pass) {
         const unsigned long long t_pass = globaltimer_ns();
@@ -882,7 +899,8 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
         if (trs) trace_mark(p.trace, trs, t_pass);
         const bool first_c = pass == 0 && p.draft;             // c formed by the Read CTAs
         if (!first_c) {
-            gather_e(p, sh.x, sh.anch, e, CH, cb, tid, nth);
+            if (pass > 0) cp_async_wait<0>();                  // issued at the end of the previous pass
+            else gather_e(p, sh.x, sh.anch, e, CH, cb, tid, nth);
             __syncthreads();
         }
         if (trs) trace_mark(p.trace, trs + 1, t_pass);
@@ -1127,6 +1145,11 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
         if (lead && lane == 0 && p.trace && pass < 2) trace_mark(p.trace, 240 + 4 * pass + 1, t_end);
         __syncthreads();
         if (lead && tid == 0 && p.trace && pass < 2) trace_mark(p.trace, 240 + 4 * pass + 2, t_end);
+        // the new tokens, then the next pass's E' rows in flight while the
+        // stopping rule and the packing run
+        for (int t = tid; t < n; t += nth) sh.x[sh.tok[t]] = sh.ynew[t];
+        __syncthreads();
+        gather_e_async(p, sh.x, sh.anch, e, CH, cb, tid, nth, eprow_policy);
         if (warp == 0) {
             // lane q: block q (b <= 32)
             SeqState ns{};
@@ -1157,8 +1180,6 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
                 sh.n2 = total;
                 sh.more = total > 0 && pass + 1 < p.K_max;
             }
-        } else {
-            for (int t = tid - 32; t < n; t += nth - 32) sh.x[sh.tok[t]] = sh.ynew[t];
         }
         __syncthreads();
         if (lead && tid == 0 && p.trace && pass < 2) trace_mark(p.trace, 240 + 4 * pass + 3, t_end);
@@ -1176,6 +1197,7 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
         __syncthreads();
         if (lead && tid == 0 && p.trace) trace_mark(p.trace, 8 + 4 * pass + 2, t_end);
         if (!more) {
+            cp_async_wait<0>();                                // no copy may land after the CTA leaves
             if (lead && tid == 0) raise_stop(c, 0);            // after the lead's writes
             break;
         }
