@@ -103,7 +103,9 @@ struct Params {
     int S;                       // vocabulary ranges of the Read kernel
     int use_graph;               // 1: the pass loop is a graph WHILE node
     unsigned long long *trace;   // optional kernel timeline (profiling), else NULL
-    int read_flags;              // experiments: bit 0 = no L2 bulk prefetch of W_r
+    int read_flags;              // tuning (XPRESS_READ_FLAGS): bit 0 = no L2 bulk prefetch of W_r, bit 1 = no
+                                 // lookahead of the W_r ring into the next pass, bits 8+ = the pacing of the
+                                 // first pass's W_r prefetch in units of 100 ns (0: 1 us per 32 KB slice)
     int ksplit;                  // split-K factor of the hidden projection
     // inputs (caller-owned)
     const void *h, *s;
