@@ -91,6 +91,17 @@ def test_bf16_tensor_core_path(X, b, B, temps):
     assert max(o["iters"] for o in orc.values()) >= 2
 
 
+# A vocabulary that is not a multiple of 32 (or of 128): the last Read range
+# ends in a partial 32-row quarter whose box reaches past V (zero-filled), and
+# the graph path's last 256-row tile is ragged.
+@pytest.mark.parametrize("b,B,temps", [(1, 16, (0.0,)), (2, 16, (1.0, 0.0)), (4, 16, (0.0, 1.0))])
+def test_bf16_ragged_vocabulary(X, b, B, temps):
+    cfg = W.tiny_config("bf16v", b=b, B=B, H=128, V=2088, r=256, dtype=W.BF16, temps=temps, seed=1500 + b)
+    w = W.make_weights(cfg.H, cfg.V, cfg.r, cfg.B, cfg.dtype, 2500 + b, "strong")
+    inp = W.make_inputs(cfg)
+    _check(X, cfg, w, inp)
+
+
 def test_bf16_fixed_k_and_cap(X):
     cfg = W.tiny_config("bf16k", b=6, B=16, H=128, V=2080, r=256, dtype=W.BF16, temps=(0.0, 1.0), seed=31)
     w = W.make_weights(cfg.H, cfg.V, cfg.r, cfg.B, cfg.dtype, 32, "strong")
