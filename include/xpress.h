@@ -115,7 +115,15 @@ typedef struct {
  *                     evaluated position k; T <= 0: NaN
  *   logit_sel [b, B]  l_k,y / T at the selected token (T <= 0: l_k,y)
  *   z_final   [b, B, r] fp32 z_k of that pass (the W_r operand before rounding)
- *   refined_logits [b, B, V] fp32 l_k (debug; slows the pass down)          */
+ *   refined_logits [b, B, V] fp32 l_k (debug; slows the pass down)
+ *   trajectory [b, K_max, B] int32 (debug): trajectory[s][j][k] is the token
+ *                     pass j + 1 selected for position k of block s, written
+ *                     only where that pass evaluated position k (a pass
+ *                     evaluates the positions after the first one the previous
+ *                     pass changed, Theorem 1); every other entry keeps what
+ *                     the caller stored there.  Y^(j) of Algorithm 1 is
+ *                     recovered by carrying each position's last written
+ *                     token forward from Y^(0).                             */
 typedef struct {
     int32_t *tokens;
     int32_t *iters;
@@ -124,17 +132,22 @@ typedef struct {
     float *logit_sel;
     float *z_final;
     float *refined_logits;
+    int32_t *trajectory;
 } xpress_block_out;
 
 /* Bytes of device workspace xpress_refine_block needs for b blocks. */
 size_t xpress_refine_workspace_size(const xpress_refiner *refiner, int b);
 
 /* Runs Algorithm 1 on all b blocks with no host synchronisation: the
- * iteration loop runs on the device (a CUDA graph with a device-updated WHILE
- * condition); blocks that have converged drop out of later passes, and a pass
- * re-evaluates only the positions after the first token the previous pass
- * changed (by Theorem 1 the others cannot change).  workspace: >= the size
- * above, 256-byte aligned, owned by the caller, not shared by concurrent calls.
+ * iteration loop runs on the device.  Calls of a bf16 refiner that evaluate at
+ * most 32 tokens (b * B <= 32) run as one persistent cooperative kernel whose
+ * CTAs apply the stopping rule themselves; other calls run a CUDA graph whose
+ * WHILE conditional node repeats the per-pass kernels until the device clears
+ * its condition.  Blocks that have converged drop out of later passes, and a
+ * pass re-evaluates only the positions after the first token the previous
+ * pass changed (by Theorem 1 the others cannot change).  workspace: >= the
+ * size above, 256-byte aligned, owned by the caller, not shared by concurrent
+ * calls.
  * Errors: INVALID_ARG, UNSUPPORTED, WORKSPACE, CUDA. */
 int xpress_refine_block(const xpress_refiner *refiner, const xpress_block_in *in,
                         const xpress_block_out *out, void *workspace, size_t ws_bytes,
@@ -188,9 +201,12 @@ int xpress_accept(const xpress_refiner *refiner, const xpress_accept_in *in, int
  *     call.  Its first call on a device looks up the array's device address
  *     (cudaGetSymbolAddress, once per device, with that device current);
  *     make that first call before any stream capture.
+ *   - The refiner's device must be the current device; a call made with
+ *     another device current returns XPRESS_ERR_INVALID_ARG.
  *   - Every call shares the one array, which keeps the previous call's
  *     contents: calls that overlap on the GPU (other streams, other threads)
- *     race on it and must be serialised by the caller.  The device status of
+ *     race on it and must be serialised by the caller.  Calls issued back to
+ *     back on one stream are serialised by that stream.  The device status of
  *     these calls is not reported (xpress_get_device_status needs a
  *     workspace).
  * Errors: INVALID_ARG, UNSUPPORTED (batch too large), CUDA. */
@@ -201,6 +217,18 @@ int xpress_accept_noalloc(const xpress_refiner *refiner, const xpress_accept_in 
  * in `workspace` by xpress_refine_block / xpress_accept.  *status_out is an
  * xpress_status (XPRESS_OK, XPRESS_ERR_TIMEOUT or XPRESS_ERR_DEVICE_CHECK). */
 int xpress_get_device_status(void *workspace, void *stream, int32_t *status_out);
+
+/* Failure detection: every wait of the persistent small-batch kernel for
+ * another CTA's progress (a monotone counter in the workspace) gives up after
+ * `limit_ns` nanoseconds of wall time (2 s by default, 0 <= limit_ns <= 60 s);
+ * the kernel then records XPRESS_ERR_TIMEOUT in the workspace's status word,
+ * every CTA lets its own copies and tensor-core work drain, frees its tensor
+ * memory and returns, and the next call on the workspace starts clean.  Waits
+ * of a CTA on its own copies keep their own bounds.  Applies to the calls
+ * made after it on this refiner (the paper has no counterpart; it exists so
+ * that the timeout path can be exercised).
+ * Errors: INVALID_ARG (NULL refiner, limit above 60 s). */
+int xpress_set_wait_limit(xpress_refiner *refiner, uint64_t limit_ns);
 
 /* Synchronises `stream`, then reads how many refiner passes the device loop
  * of the last xpress_refine_block call on `workspace` executed (the largest

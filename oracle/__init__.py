@@ -79,7 +79,7 @@ def _load():
             lib.xo_select.argtypes = [P, I, D, U64, U32, I, P, P, P, P]
             lib.xo_jacobi.argtypes = [MP, P, P, C.c_int32, P, D, U64, U32, I, I, P, P, P, P, P, P, P, P, P]
             lib.xo_sequential.argtypes = [MP, P, P, C.c_int32, D, U64, U32, P, P]
-            lib.xo_accept.argtypes = [MP, P, P, P, P, P, P, D, U64, U32, P, P, P]
+            lib.xo_accept.argtypes = [MP, P, P, P, P, P, P, D, U64, U32, P, P, P, P]
             lib.xo_jacobi_seeds.argtypes = [MP, P, P, C.c_int32, P, D, P, I, U32, I, P, P]
             lib.xo_refine_accept_seeds.argtypes = [MP, P, P, P, C.c_int32, P, D, P, I, U32, I, P, P]
             for f in ("xo_forward", "xo_select", "xo_jacobi", "xo_sequential", "xo_accept",
@@ -217,8 +217,12 @@ def sequential(m: Model, h, s, anchor, T=0.0, seed=0, offset=0):
     return y, mg
 
 
-def accept(m: Model, target, s, tokens, lse, sel, z_final, T, seed, offset):
-    """Acceptance (Sec. 3.1).  Returns (accept_len, out_tokens [B+1], margin)."""
+def accept(m: Model, target, s, tokens, lse, sel, z_final, T, seed, offset, with_gaps=False):
+    """Acceptance (Sec. 3.1).  Returns (accept_len, out_tokens [B+1], margin),
+    plus, with ``with_gaps``, the per-decision margins gaps [B+2]: gaps[k]
+    (k < B) of the decision at position k (T = 0: top-2 gap of target row k;
+    T > 0: |u q - p| / p of the accept test), gaps[B+1] of the final token's
+    draw (top-2 margin); +inf where nothing was decided."""
     tgt = m._a(target, (m.B + 1, m.V))
     s = m._a(s, (m.B, m.V))
     y = np.ascontiguousarray(tokens, dtype=np.int32)
@@ -228,9 +232,12 @@ def accept(m: Model, target, s, tokens, lse, sel, z_final, T, seed, offset):
     n = np.zeros(1, np.int32)
     out = np.zeros(m.B + 1, np.int32)
     mg = np.zeros(1)
+    gaps = np.zeros(m.B + 2)
     if _load().xo_accept(C.byref(m.c), _ptr(tgt), _ptr(s), _ptr(y), _ptr(lse), _ptr(sel), _ptr(z),
-                         float(T), int(seed), int(offset), _ptr(n), _ptr(out), _ptr(mg)):
+                         float(T), int(seed), int(offset), _ptr(n), _ptr(out), _ptr(mg), _ptr(gaps)):
         raise ValueError("invalid arguments")
+    if with_gaps:
+        return int(n[0]), out, float(mg[0]), gaps
     return int(n[0]), out, float(mg[0])
 
 

@@ -19,7 +19,7 @@
  *   lossless acceptance            Sec. 3.1 and Sec. 4.3 (accept w.p.
  *                                  min(1, p/q), else resample max(0, p-q))
  *
- * Readings of points the paper leaves open (each is listed in the design doc):
+ * Readings of points the paper leaves open:
  *   - sigma is selectable: SiLU (default), GELU(erf), ReLU (Sec. 4.1 says only
  *     "a pointwise nonlinearity");
  *   - no biases or norms (the equations have none);
@@ -439,10 +439,16 @@ int xo_sequential(const xo_model *M, const void *h, const void *s, int32_t ancho
  *         sample p_k); if all B are accepted, the bonus is a Gumbel-max draw
  *         from p_{B+1} (stream 3, position B).
  * out [B+1] = emitted tokens then -1; returns n in *accept_len.
- * margin: smallest decision margin (relative for the accept tests). */
+ * margin: smallest decision margin (relative for the accept tests).
+ * gaps [B+2] (optional): gaps[k] for k < B is the margin of the decision at
+ * position k (T = 0: the top-2 gap of target row k, for the rows examined;
+ * T > 0: |u q - p| / p of the accept test, for the positions tested), and
+ * gaps[B+1] the top-2 margin of the token drawn or taken at the end; entries
+ * not decided are +inf. */
 int xo_accept(const xo_model *M, const void *tgt, const void *s, const int32_t *y,
               const double *lse, const double *sel, const double *z_final, double T,
-              uint64_t seed, uint32_t offset, int32_t *accept_len, int32_t *out, double *margin)
+              uint64_t seed, uint32_t offset, int32_t *accept_len, int32_t *out, double *margin,
+              double *gaps)
 {
     const int B = M->B, V = M->V, r = M->r;
     double *row = (double *)malloc(sizeof(double) * V);
@@ -450,13 +456,17 @@ int xo_accept(const xo_model *M, const void *tgt, const void *s, const int32_t *
     double mg = INFINITY, m1;
     int n = 0;
     for (int k = 0; k <= B; ++k) out[k] = -1;
+    if (gaps)
+        for (int k = 0; k < B + 2; ++k) gaps[k] = INFINITY;
     if (T <= 0.0) {
         for (;;) {
             for (int v = 0; v < V; ++v) row[v] = ld(tgt, M->dtype, (size_t)n * V + v);
             int t = argmax_f32(row, V, &m1);
             if (m1 < mg) mg = m1;
+            if (gaps) gaps[n < B ? n : B + 1] = m1;
             if (n < B && y[n] == t) { out[n] = y[n]; ++n; continue; }
             out[n] = t;
+            if (gaps && n < B) gaps[B + 1] = m1;
             break;
         }
     } else {
@@ -474,6 +484,7 @@ int xo_accept(const xo_model *M, const void *tgt, const void *s, const int32_t *
             double u = xo_uniform(seed, 0u, (uint32_t)n, XO_STREAM_ACCEPT, offset);
             double rel = fabs(u * q_y - p_y) / (p_y > 0 ? p_y : 1e-300);
             if (rel < mg) mg = rel;
+            if (gaps) gaps[n] = rel;
             if ((float)(u * q_y) < (float)p_y) { out[n] = y[n]; continue; }
             rejected = 1;
             /* residual max(0, p - q) at position n */
@@ -500,6 +511,7 @@ int xo_accept(const xo_model *M, const void *tgt, const void *s, const int32_t *
                     sc[v] = row[v] + xo_gumbel(seed, (uint32_t)v, (uint32_t)n, XO_STREAM_RESID, offset);
             out[n] = argmax_f32(sc, V, &m1);
             if (m1 < mg) mg = m1;
+            if (gaps) gaps[B + 1] = m1;
             free(zop); free(ell);
             break;
         }
@@ -509,6 +521,7 @@ int xo_accept(const xo_model *M, const void *tgt, const void *s, const int32_t *
                         xo_gumbel(seed, (uint32_t)v, (uint32_t)B, XO_STREAM_RESID, offset);
             out[B] = argmax_f32(sc, V, &m1);
             if (m1 < mg) mg = m1;
+            if (gaps) gaps[B + 1] = m1;
         }
     }
     *accept_len = n;
@@ -555,7 +568,7 @@ int xo_refine_accept_seeds(const xo_model *M, const void *h, const void *s, cons
                            sel, z, NULL, NULL, NULL);
         if (!rc)
             rc = xo_accept(M, tgt, s, tok, lse, sel, z, T, seeds[i], offset, accept_len + i,
-                           out + (size_t)i * (B + 1), NULL);
+                           out + (size_t)i * (B + 1), NULL, NULL);
         if (rc) { free(tok); free(lse); free(sel); free(z); return rc; }
     }
     free(tok); free(lse); free(sel); free(z);

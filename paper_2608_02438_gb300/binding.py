@@ -40,7 +40,7 @@ class XpressBlockIn(C.Structure):
 
 class XpressBlockOut(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in ("tokens", "iters", "converged", "lse", "logit_sel", "z_final",
-                                          "refined_logits")]
+                                          "refined_logits", "trajectory")]
 
 
 class XpressAcceptIn(C.Structure):
@@ -88,6 +88,8 @@ def load(path: str = LIB_PATH):
     lib.xpress_get_pass_count.restype = I
     lib.xpress_accept_noalloc.argtypes = [P, C.POINTER(XpressAcceptIn), P, P, P]
     lib.xpress_accept_noalloc.restype = I
+    lib.xpress_set_wait_limit.argtypes = [P, C.c_uint64]
+    lib.xpress_set_wait_limit.restype = I
     lib.xpress_profile_read_prepare.argtypes = [P, P, I, I, P]
     lib.xpress_profile_read_prepare.restype = I
     lib.xpress_profile_read.argtypes = [P, P, I, P]
@@ -164,6 +166,10 @@ def xpress_get_pass_count(ws_ptr: int, stream: int) -> int:
     return v.value
 
 
+def xpress_set_wait_limit(handle, limit_ns: int) -> None:
+    _check("xpress_set_wait_limit", load().xpress_set_wait_limit(handle, limit_ns))
+
+
 def xpress_profile_read_prepare(handle, ws_ptr: int, b: int, n_tokens: int, stream: int) -> None:
     _check("xpress_profile_read_prepare", load().xpress_profile_read_prepare(handle, C.c_void_p(ws_ptr), b, n_tokens,
                                                                               C.c_void_p(stream)))
@@ -211,7 +217,9 @@ class Refiner:
         ptr = (buf.data_ptr() + 255) & ~255
         return ptr, buf.numel() - (ptr - buf.data_ptr())
 
-    def alloc_outputs(self, b: int, want_logits: bool = False) -> dict:
+    def alloc_outputs(self, b: int, want_logits: bool = False, traj_K: int = 0) -> dict:
+        """Output tensors; traj_K > 0 adds the debug trajectory [b, traj_K, B]
+        (traj_K must equal the call's K_max), filled with -1."""
         t = self.torch
         return dict(tokens=t.empty((b, self.B), dtype=t.int32, device="cuda"),
                     iters=t.empty(b, dtype=t.int32, device="cuda"),
@@ -220,18 +228,22 @@ class Refiner:
                     logit_sel=t.empty((b, self.B), dtype=t.float32, device="cuda"),
                     z_final=t.empty((b, self.B, self.r), dtype=t.float32, device="cuda"),
                     refined_logits=t.empty((b, self.B, self.V), dtype=t.float32, device="cuda") if want_logits
+                    else None,
+                    trajectory=t.full((b, traj_K, self.B), -1, dtype=t.int32, device="cuda") if traj_K > 0
                     else None)
 
     def refine_block(self, h, s, draft, anchor, temperature, seed, offset: int, K_max: int, fixed_K: bool = False,
-                     out: dict | None = None, want_logits: bool = False) -> dict:
+                     out: dict | None = None, want_logits: bool = False, want_traj: bool = False) -> dict:
         b = h.shape[0]
-        out = out if out is not None else self.alloc_outputs(b, want_logits)
+        out = out if out is not None else self.alloc_outputs(b, want_logits, K_max if want_traj else 0)
+        if out.get("trajectory") is not None and tuple(out["trajectory"].shape) != (b, K_max, self.B):
+            raise ValueError("trajectory must be [b, K_max, B]")
         blk_in = XpressBlockIn(b, h.data_ptr(), s.data_ptr(), None if draft is None else draft.data_ptr(),
                                anchor.data_ptr(), temperature.data_ptr(), seed.data_ptr(), offset, K_max,
                                int(bool(fixed_K)))
         blk_out = XpressBlockOut(*[None if out.get(n) is None else out[n].data_ptr() for n in
                                    ("tokens", "iters", "converged", "lse", "logit_sel", "z_final",
-                                    "refined_logits")])
+                                    "refined_logits", "trajectory")])
         ws, wsb = self.workspace("refine", b)
         xpress_refine_block(self.handle, blk_in, blk_out, ws, wsb, self.stream.cuda_stream)
         return out

@@ -116,6 +116,12 @@ __global__ void __launch_bounds__(256) k_acc_rows(AcceptParams p)
 // z_final through W_r), with the draw from p_k alongside for an empty
 // residual, or the bonus draw from p_{B+1} after B acceptances -- and the last
 // CTA of the block (ticket) combines the chunks and emits the token.
+//
+// k_acc_finalize never triggers its dependents early (no griddepcontrol.
+// launch_dependents): the next acceptance call's k_acc_rows, which may reuse
+// the same scratch (always, for xpress_accept_noalloc), clears the status
+// word and the tickets before its own dependency wait, so it must not start
+// until every CTA of this kernel has exited.
 __global__ void __launch_bounds__(256) k_acc_finalize(AcceptParams p, int chunks)
 {
     pdl_wait();                                   // the row partials (and the refinement before them)

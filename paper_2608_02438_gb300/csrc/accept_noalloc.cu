@@ -25,16 +25,13 @@ __device__ __align__(256) unsigned char g_accept_scratch[ACCEPT_NOALLOC_SCRATCH_
 std::mutex g_mutex;
 void *g_scratch_addr[MAX_DEVICES];   // device address of g_accept_scratch, per device
 
-// The address of the array as the current device sees it.  In host code the
-// name g_accept_scratch is only a host-side stand-in, so the device address
-// is queried once per device (with that device current) and cached.
-int scratch_address(void **out)
+// The address of the array on device `dev`, which must be the current
+// device.  In host code the name g_accept_scratch is only a host-side
+// stand-in, so the device address is queried once per device (with that
+// device current) and cached.
+int scratch_address(int dev, void **out)
 {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= MAX_DEVICES) {
-        (void)cudaGetLastError();
-        return XPRESS_ERR_CUDA;
-    }
+    if (dev < 0 || dev >= MAX_DEVICES) return XPRESS_ERR_CUDA;
     std::lock_guard<std::mutex> lock(g_mutex);
     if (!g_scratch_addr[dev]) {
         void *ptr = nullptr;
@@ -55,7 +52,16 @@ extern "C" int xpress_accept_noalloc(const xpress_refiner *refiner, const xpress
 {
     if (!refiner || !in || in->b < 1) return XPRESS_ERR_INVALID_ARG;
     if (xp::accept_scratch_bytes(refiner, in->b) > ACCEPT_NOALLOC_SCRATCH_BYTES) return XPRESS_ERR_UNSUPPORTED;
+    // the array used must be the one on the refiner's device: a call made with
+    // another device current would touch (and possibly create) that device's
+    // context instead, so it is refused
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return XPRESS_ERR_CUDA;
+    }
+    if (dev != xp::refiner_device(refiner)) return XPRESS_ERR_INVALID_ARG;
     void *scratch = nullptr;
-    if (const int rc = scratch_address(&scratch)) return rc;
+    if (const int rc = scratch_address(dev, &scratch)) return rc;
     return xp::accept_launch(refiner, in, accept_len, out_tokens, scratch, ACCEPT_NOALLOC_SCRATCH_BYTES, stream);
 }

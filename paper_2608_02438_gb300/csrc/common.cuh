@@ -102,10 +102,8 @@ struct Params {
     uint32_t offset;
     int S;                       // vocabulary ranges of the Read kernel
     int use_graph;               // 1: the pass loop is a graph WHILE node
+    unsigned long long wait_ns;  // persistent kernel: bound on each wait for another CTA (2 s by default)
     unsigned long long *trace;   // optional kernel timeline (profiling), else NULL
-    int read_flags;              // tuning (XPRESS_READ_FLAGS): bit 0 = no L2 bulk prefetch of W_r, bit 1 = no
-                                 // lookahead of the W_r ring into the next pass, bits 8+ = the pacing of the
-                                 // first pass's W_r prefetch in units of 100 ns (0: 1 us per 32 KB slice)
     int ksplit;                  // split-K factor of the hidden projection
     // inputs (caller-owned)
     const void *h, *s;
@@ -118,6 +116,7 @@ struct Params {
     // outputs (caller-owned; NULL allowed except tokens)
     int32_t *tokens, *iters, *converged;
     float *lse, *logit_sel, *z_final, *logits;
+    int32_t *traj;               // [b, K_max, B] optional: token selected at each evaluated (pass, position)
     // workspace
     int32_t *status;
     int32_t *ctl;
@@ -156,6 +155,13 @@ template <> __device__ __forceinline__ float ldf<uint16_t>(const uint16_t *p, si
 __device__ __forceinline__ float ld_any(const void *p, int dtype, size_t i)
 {
     return dtype ? bf2f(static_cast<const uint16_t *>(p)[i]) : static_cast<const float *>(p)[i];
+}
+
+// Optional trajectory output: the token pass `pass` (0-based) selected for
+// global token `tok` (block tok / B, position tok % B).
+__device__ __forceinline__ void record_traj(const Params &p, int tok, int pass, int y)
+{
+    if (p.traj && pass >= 0 && pass < p.K_max) p.traj[((size_t)(tok / p.B) * p.K_max + pass) * p.B + tok % p.B] = y;
 }
 
 __device__ __forceinline__ float act_fn(int act, float t)

@@ -78,6 +78,7 @@ constexpr int GEMV_SMEM = 128 * 1024;
 // acceptance launch shared by xpress_accept and xpress_accept_noalloc
 // (xpress_host.cu); `ws` holds the scratch laid out by accept_scratch_bytes
 size_t accept_scratch_bytes(const xpress_refiner *R, int b);
+int refiner_device(const xpress_refiner *R);   // the device the refiner was created on
 int accept_launch(const xpress_refiner *R, const xpress_accept_in *in, int32_t *accept_len, int32_t *out_tokens,
                   void *ws, size_t ws_bytes, void *stream);
 constexpr int READ_SIMT_DYN_SMEM = (32 * (RANK + 1) + 8 * 32 * 33) * 4;

@@ -144,7 +144,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         // L2 now, so that they stream while the previous kernel finishes
         const uint32_t row_bytes = RANK * 2;
         const char *wr = static_cast<const char *>(p.W_r);
-        for (int vt = vt0; vt < vt1 && !(p.read_flags & 1); ++vt) {
+        for (int vt = vt0; vt < vt1; ++vt) {
             const int rows = min(TC_BN, V - vt * TC_BN);
             for (int r0 = 0; r0 < rows; r0 += 64)
                 prefetch_l2_bulk(wr + (size_t)(vt * TC_BN + r0) * row_bytes, (uint32_t)min(64, rows - r0) * row_bytes);

@@ -90,9 +90,8 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
         tma_prefetch_desc(&tmap_z);
         const char *wr = static_cast<const char *>(p.W_r);
         const int rows = min(vb1 * TV_BM, V) - vb0 * TV_BM;
-        if (!(p.read_flags & 1))
-            for (int r0 = 0; r0 < rows; r0 += 64)
-                prefetch_l2_bulk(wr + (size_t)(vb0 * TV_BM + r0) * RANK * 2, (uint32_t)min(64, rows - r0) * RANK * 2);
+        for (int r0 = 0; r0 < rows; r0 += 64)
+            prefetch_l2_bulk(wr + (size_t)(vb0 * TV_BM + r0) * RANK * 2, (uint32_t)min(64, rows - r0) * RANK * 2);
         for (int i = 0; i < pre; ++i) {
             mbar_expect_tx(&sh.full[i], TV_A_STAGE);
             tma_load_2d_hint(sA + i * TV_A_STAGE, &tmap_wr128, &sh.full[i], (i % TV_KCH) * TV_BK,
@@ -292,6 +291,7 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
                     if (p.lse) p.lse[tok] = res.lse;
                     if (p.logit_sel) p.logit_sel[tok] = res.sel;
                     p.tokens[tok] = res.y;
+                    record_traj(p, tok, sh.passes, res.y);
                 }
             }
             __syncthreads();

@@ -747,7 +747,8 @@ __global__ void __launch_bounds__(1024) k_reduce(const Params *__restrict__ pp, 
     pdl_wait();
     const Params &p = *pp;
     const int s = blockIdx.x, B = p.B, warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-    const int tr_slot = 8 + 4 * p.ctl[CTL_PASS] + 2;
+    const int pass = p.ctl[CTL_PASS];               // passes before this one (updated by the last CTA)
+    const int tr_slot = 8 + 4 * pass + 2;
     const SeqState st = p.st[s];
     __shared__ int last;
     __shared__ int ynew[MAX_B], yold[MAX_B];
@@ -762,6 +763,7 @@ __global__ void __launch_bounds__(1024) k_reduce(const Params *__restrict__ pp, 
             if (p.lse) p.lse[tok] = res.lse;
             if (p.logit_sel) p.logit_sel[tok] = res.sel;
             p.tokens[tok] = res.y;
+            record_traj(p, tok, pass, res.y);
         }
     }
     __syncthreads();

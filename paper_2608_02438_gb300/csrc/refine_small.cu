@@ -106,10 +106,12 @@ __device__ __forceinline__ void raise_stop(SmallCtl *c, int bits)
 }
 
 // One thread: waits until *ctr >= target (true).  false once the stop bit is
-// set, or after about 2 s (the timeout is recorded and every role stops).
+// set, or after limit_ns of wall time (the caller's bound on waits for other
+// CTAs, 2 s by default: the timeout is recorded and every role stops).
 // Relaxed polls with a short sleep keep ~150 pollers from crowding the line's
 // L2 slice; the fence after the last poll makes it an acquire.
-__device__ __forceinline__ bool wait_count(SmallCtl *c, const unsigned *ctr, unsigned target)
+__device__ __forceinline__ bool wait_count(SmallCtl *c, const unsigned *ctr, unsigned target,
+                                           unsigned long long limit_ns)
 {
     const unsigned long long t0 = globaltimer();
     for (uint32_t it = 0; it < (1u << 26); ++it) {
@@ -117,7 +119,7 @@ __device__ __forceinline__ bool wait_count(SmallCtl *c, const unsigned *ctr, uns
         if (v & STOP_BIT) { fence_acq_rel_gpu(); return false; }
         if (v >= target) { fence_acq_rel_gpu(); return true; }
         if (it >= 2) __nanosleep(32);
-        if ((it & 63u) == 63u && globaltimer() - t0 > 2000000000ull) break;
+        if (globaltimer() - t0 > limit_ns) break;
     }
     raise_stop(c, ST_TIMEOUT);
     return false;
@@ -127,7 +129,8 @@ __device__ __forceinline__ bool wait_count(SmallCtl *c, const unsigned *ctr, uns
 // slice every gap_ns: DRAM stays busy without queues deep enough to stall the
 // latency-bound accesses of the other role (its first-pass code and operands).
 __device__ __forceinline__ bool wait_count_prefetch(SmallCtl *c, const unsigned *ctr, unsigned target, const char *pf,
-                                                    uint32_t bytes, uint32_t slice, unsigned gap_ns)
+                                                    uint32_t bytes, uint32_t slice, unsigned gap_ns,
+                                                    unsigned long long limit_ns)
 {
     const unsigned long long t0 = globaltimer();
     unsigned long long t_next = t0;
@@ -145,7 +148,7 @@ __device__ __forceinline__ bool wait_count_prefetch(SmallCtl *c, const unsigned 
             }
         }
         if (it >= 2) __nanosleep(32);
-        if ((it & 63u) == 63u && globaltimer() - t0 > 2000000000ull) break;
+        if (globaltimer() - t0 > limit_ns) break;
     }
     raise_stop(c, ST_TIMEOUT);
     return false;
@@ -458,21 +461,18 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
             };
             long long next = 0;
             bool ok = true;
-            const bool lookahead = !(p.read_flags & 2);
-            if (lookahead)
-                for (; next < ahead && ok; ++next) ok = issue(next);
+            for (; next < ahead && ok; ++next) ok = issue(next);
             // while the first Trans runs, the rest of this CTA's W_r range
             // (past the chunks the ring holds) goes into L2 a slice at a time
-            const int pf_row0 = R0 + (lookahead ? ahead / TV_KCH : 0) * TV_BM;
+            const int pf_row0 = R0 + (ahead / TV_KCH) * TV_BM;
             const int pf_rows = max(0, R1 - pf_row0);
-            const uint32_t pf_bytes = (p.read_flags & 1) ? 0u : (uint32_t)pf_rows * RANK * 2;
+            const uint32_t pf_bytes = (uint32_t)pf_rows * RANK * 2;
             for (int pass = 0; ok; ++pass) {
                 const bool go = pass == 0
                                     ? wait_count_prefetch(c, &c->z_ready.v, 8u, static_cast<const char *>(p.W_r) +
                                                                                    (size_t)pf_row0 * RANK * 2,
-                                                          pf_bytes, 64 * RANK * 2,
-                                                          (p.read_flags >> 8) ? (unsigned)(p.read_flags >> 8) * 100u : 1000u)
-                                    : wait_count(c, &c->z_ready.v, (unsigned)(8 * (pass + 1)));
+                                                          pf_bytes, 64 * RANK * 2, 1000u, p.wait_ns)
+                                    : wait_count(c, &c->z_ready.v, (unsigned)(8 * (pass + 1)), p.wait_ns);
                 if (go) {
                     fence_proxy_async_global();
                     sh.pass_n = min(__ldcg(p.ctl + CTL_NACT), TV_BN);
@@ -488,7 +488,7 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
                 z_issued = true;
                 z_par = (uint32_t)(pass & 1);
                 // the rest of this pass, then the first chunks of the next one
-                const long long end = (long long)(pass + 1) * per_pass + (lookahead ? ahead : 0);
+                const long long end = (long long)(pass + 1) * per_pass + ahead;
                 for (; next < end; ++next)
                     if (!issue(next)) { ok = false; break; }
             }
@@ -858,7 +858,7 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
         else mix_block16<1>(e, Lp, pc, cop, sh.cown, d, -1, 0, rank);
     }
     if (lead && tid == 0 && p.trace) trace_mark(p.trace, 250, t_start);
-    if (tid == 0) sh.go = wait_count(c, &c->pre_done.v, (unsigned)p.S);
+    if (tid == 0) sh.go = wait_count(c, &c->pre_done.v, (unsigned)p.S, p.wait_ns);
     __syncthreads();
     if (!sh.go) return;
     if (lead && tid == 0 && p.trace) trace_mark(p.trace, 251, t_start);
@@ -1000,7 +1000,7 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
             __syncthreads();
             if (tid == 0) {
                 red_add_release_gpu(&c->c_ready.v, 1u);
-                sh.go = wait_count(c, &c->c_ready.v, (unsigned)(8 * (pass + (p.draft ? 0 : 1))));
+                sh.go = wait_count(c, &c->c_ready.v, (unsigned)(8 * (pass + (p.draft ? 0 : 1))), p.wait_ns);
                 if (trs) trace_mark(p.trace, trs + 2, t_pass);
             }
             __syncthreads();
@@ -1040,7 +1040,7 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
         __syncthreads();
         if (tid == 0) {
             red_add_release_gpu(&c->u_ready.v, 1u);
-            sh.go = wait_count(c, &c->u_ready.v, (unsigned)(8 * (pass + 1)));
+            sh.go = wait_count(c, &c->u_ready.v, (unsigned)(8 * (pass + 1)), p.wait_ns);
             if (trs) trace_mark(p.trace, trs + 3, t_pass);
         }
         __syncthreads();
@@ -1100,7 +1100,7 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
         if (tid == 0) {
             red_add_release_gpu(&c->z_ready.v, 1u);
             if (lead && p.trace) trace_mark(p.trace, 8 + 4 * pass, t_pass);
-            sh.go = wait_count(c, &c->read_done.v, (unsigned)(p.S * (pass + 1)));
+            sh.go = wait_count(c, &c->read_done.v, (unsigned)(p.S * (pass + 1)), p.wait_ns);
         }
         __syncthreads();
         if (!sh.go) break;
@@ -1123,6 +1123,7 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
                     if (p.lse) p.lse[tok] = __int_as_float(0x7fc00000);
                     if (p.logit_sel) p.logit_sel[tok] = best;
                     p.tokens[tok] = idx;
+                    record_traj(p, tok, pass, idx);
                 }
             }
         }
@@ -1139,6 +1140,7 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
                     if (p.lse) p.lse[tok] = res.lse;
                     if (p.logit_sel) p.logit_sel[tok] = res.sel;
                     p.tokens[tok] = res.y;
+                    record_traj(p, tok, pass, res.y);
                 }
             }
         }

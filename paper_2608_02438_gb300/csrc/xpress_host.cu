@@ -92,6 +92,7 @@ struct xpress_refiner {
     CUtensorMap tmap_fhi{}, tmap_flo{};    // folded projection, hi / lo term, boxes of 256 rows x 64 (k_pre_tc)
     int device = 0;
     int num_sms = 0;
+    unsigned long long wait_ns = 2000000000ull;   // bound on the persistent kernel's waits for other CTAs
     bool use_tc = false;
     cudaStream_t cs = nullptr;
     uint16_t *Fhl = nullptr;               // [2][2r, H] folded hidden projection, bf16 hi / lo (bf16 refiners)
@@ -219,14 +220,8 @@ Params make_params(const xpress_refiner *R, const xpress_block_in *in, const xpr
     P.offset = in->offset;
     P.S = L.S;
     P.use_graph = 1;
+    P.wait_ns = R->wait_ns;
     P.trace = R->trace;
-    {
-        static const int flags = [] {
-            const char *e = std::getenv("XPRESS_READ_FLAGS");
-            return e ? std::atoi(e) : 0;
-        }();
-        P.read_flags = flags;
-    }
     P.ksplit = L.ksplit;
     P.h = in->h;
     P.s = in->s;
@@ -249,6 +244,7 @@ Params make_params(const xpress_refiner *R, const xpress_block_in *in, const xpr
     P.logit_sel = out->logit_sel;
     P.z_final = out->z_final;
     P.logits = out->refined_logits;
+    P.traj = out->trajectory;
     P.status = reinterpret_cast<int32_t *>(w + L.status);
     P.ctl = reinterpret_cast<int32_t *>(w + L.ctl);
     P.st = reinterpret_cast<SeqState *>(w + L.st);
@@ -875,6 +871,8 @@ AcceptLayout accept_layout(const xpress_refiner *R, int b)
 
 namespace xp {
 
+int refiner_device(const xpress_refiner *R) { return R ? R->device : -1; }
+
 size_t accept_scratch_bytes(const xpress_refiner *R, int b)
 {
     if (!R || b < 1) return 0;
@@ -981,6 +979,13 @@ int xpress_profile_read(const xpress_refiner *R, void *ws, int b, void *stream)
         k_read_simt<<<L.S, 256, READ_SIMT_DYN_SMEM, st>>>(pdev);
     }
     XP_CUDA(cudaGetLastError());
+    return XPRESS_OK;
+}
+
+int xpress_set_wait_limit(xpress_refiner *R, uint64_t limit_ns)
+{
+    if (!R || limit_ns > 60000000000ull) return XPRESS_ERR_INVALID_ARG;
+    R->wait_ns = limit_ns;
     return XPRESS_OK;
 }
 

@@ -2,12 +2,30 @@
 
 Parity rule: token outputs, pass counts, convergence flags and accept lengths
 must match bit-exactly.  A mismatching block is excused only at a documented
-near-tie: the oracle's smallest top-2 decision margin on that block's
-trajectory is below NEAR_TIE (1e-3 in the units of the decision: logits, or
-logits / T plus Gumbel noise); at most max(1, 1%) of the blocks may be excused.
+near-tie, judged at the FIRST divergence:
+
+* refinement: both sides start from the same Y^(0); the first pass j whose
+  iterate Y^(j) differs, and the first position k where it differs, name the
+  decision that went the other way (both sides took it from identical
+  inputs).  The block is excused only if the oracle's top-2 margin of that
+  decision (Algorithm 1's argmax, or the group / member Gumbel-max at T > 0)
+  is below NEAR_TIE.  The GPU's iterates come from its debug trajectory
+  output; the oracle's from its own trajectory and per-pass margins.
+* lossless acceptance: at the first position where the two accept lengths
+  part, only if |u q - p| < ACCEPT_TIE * p there (Sec. 3.1's accept test);
+  a differing final token only if the oracle's top-2 margin of that draw is
+  below NEAR_TIE.  Greedy acceptance compares bf16 target values exactly and
+  is never excused.
+
+Every excused block is recorded (EXCUSED, printed at the end of the session)
+and at most 1% of the blocks of a case may be excused (none in a case of
+fewer than 100 blocks).
 Float outputs: refined logits within 2e-2 (bf16) or 1e-4 (fp32) absolute.
 """
 from __future__ import annotations
+
+import hashlib
+import os
 
 import numpy as np
 
@@ -15,8 +33,12 @@ import oracle as O
 from paper_2608_02438_gb300 import workloads as W
 
 NEAR_TIE = 1e-3
+ACCEPT_TIE = 1e-4
 LOGIT_TOL = {W.BF16: 2e-2, W.F32: 1e-4}
 Z_TOL = {W.BF16: 5e-3, W.F32: 1e-5}
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+EXCUSED: list[str] = []
 
 
 def oracle_model(cfg, weights, act=O.SILU):
@@ -38,15 +60,45 @@ def device_inputs(refiner_dtype, inp, sel=None):
     return d
 
 
-def run_oracle(m, inp, i, K_max, fixed_K=False):
-    return O.jacobi(m, inp["h"][i], inp["s"][i], int(inp["anchor"][i]), inp["draft"][i],
+def run_oracle(m, inp, i, K_max, fixed_K=False, draft=True):
+    return O.jacobi(m, inp["h"][i], inp["s"][i], int(inp["anchor"][i]), inp["draft"][i] if draft else None,
                     float(inp["temperature"][i]), int(inp["seed"][i]), inp["offset"], K_max, fixed_K,
                     trajectory=True)
 
 
-def compare_blocks(gpu: dict, orc: dict, seqs, dtype, check_logits=None, m=None, inp=None):
-    """Returns (n_excused, report lines); raises AssertionError on a real mismatch."""
-    excused, lines = 0, []
+def gpu_iterates(y0, traj, iters):
+    """Y^(0..iters) of one block from the GPU's trajectory output (entries a
+    pass did not evaluate are -1 and keep the previous iterate's token)."""
+    ys = [np.asarray(y0, np.int32)]
+    for j in range(int(iters)):
+        row = traj[j]
+        ys.append(np.where(row >= 0, row, ys[-1]).astype(np.int32))
+    return np.stack(ys)
+
+
+def first_divergence(gy, oy):
+    """(pass j >= 1, position k) of the first differing iterate, or None."""
+    for j in range(1, min(len(gy), len(oy))):
+        diff = np.nonzero(gy[j] != oy[j])[0]
+        if diff.size:
+            return j, int(diff[0])
+    return None
+
+
+def _limit(n):
+    return int(0.01 * n)
+
+
+def _excuse(msg):
+    EXCUSED.append(msg)
+    print("excused near-tie: " + msg)
+
+
+def compare_blocks(gpu: dict, orc: dict, seqs, dtype, check_logits=None, m=None, inp=None, allow_excused=True):
+    """gpu: host arrays of the GPU call (row j = block seqs[j]; needs the
+    trajectory output); orc: oracle results keyed by block.  Returns the
+    excused report lines; raises AssertionError on a real mismatch."""
+    lines = []
     for j, i in enumerate(seqs):
         o = orc[i]
         tok = gpu["tokens"][j]
@@ -55,12 +107,20 @@ def compare_blocks(gpu: dict, orc: dict, seqs, dtype, check_logits=None, m=None,
         if not same:
             msg = (f"block {i}: gpu tokens {tok.tolist()} iters {int(gpu['iters'][j])} conv "
                    f"{int(gpu['converged'][j])} | oracle {o['tokens'].tolist()} iters {o['iters']} conv "
-                   f"{o['converged']} min margin {o['min_margin']:.3g}")
-            if o["min_margin"] < NEAR_TIE:
-                excused += 1
-                lines.append("excused near-tie: " + msg)
-                continue
-            raise AssertionError(msg)
+                   f"{o['converged']}")
+            traj = gpu.get("trajectory")
+            assert traj is not None, "parity needs the GPU trajectory to locate the first divergence: " + msg
+            oy = o["trajectory"]
+            gy = gpu_iterates(oy[0], traj[j], gpu["iters"][j])
+            fd = first_divergence(gy, oy)
+            assert fd is not None, "iterates agree but the outcome differs (stopping rule): " + msg
+            jp, k = fd
+            mg = float(o["margins"][jp - 1][k])
+            msg += f" | first divergence pass {jp} position {k}, oracle margin {mg:.3g}"
+            assert allow_excused and mg < NEAR_TIE, msg
+            lines.append(msg)
+            _excuse(msg)
+            continue
         # float outputs of the last pass
         zt = Z_TOL[dtype]
         np.testing.assert_allclose(gpu["z_final"][j], o["z_final"], atol=zt, rtol=zt,
@@ -78,6 +138,69 @@ def compare_blocks(gpu: dict, orc: dict, seqs, dtype, check_logits=None, m=None,
             ell, _, _ = O.forward(m, inp["h"][i], inp["s"][i], x)
             err = np.abs(check_logits[j].astype(np.float64) - ell).max()
             assert err <= lt, f"refined logits block {i}: max abs err {err:.3g} > {lt}"
-    limit = max(1, int(0.01 * len(seqs)))
-    assert excused <= limit, f"{excused} excused blocks > {limit}:\n" + "\n".join(lines)
-    return excused, lines
+    assert len(lines) <= _limit(len(seqs)), f"{len(lines)} excused blocks > {_limit(len(seqs))}:\n" + "\n".join(lines)
+    return lines
+
+
+def compare_accept(alen, otok, expect: dict, seqs, temps):
+    """alen [n], otok [n, B+1] from the GPU (row j = block seqs[j]);
+    expect[i] = (accept_len, out_tokens, gaps) from the oracle."""
+    lines = []
+    for j, i in enumerate(seqs):
+        n, out, gaps = expect[i]
+        B = len(out) - 1
+        gn, gout = int(alen[j]), otok[j].tolist()
+        if gn == n and gout == list(out):
+            continue
+        msg = f"block {i}: gpu accept {gn} {gout} | oracle {n} {list(out)}"
+        assert temps[i] > 0, "greedy acceptance must match exactly: " + msg
+        if gn != n:
+            k = min(gn, n)
+            ok = k < B and gaps[k] < ACCEPT_TIE
+            msg += f" | accept test at position {k}: |uq - p| / p = {gaps[k]:.3g}"
+        else:
+            ok = gaps[B + 1] < NEAR_TIE
+            msg += f" | final draw margin {gaps[B + 1]:.3g}"
+        assert ok, msg
+        lines.append(msg)
+        _excuse(msg)
+    assert len(lines) <= _limit(len(seqs)), f"{len(lines)} excused blocks > {_limit(len(seqs))}:\n" + "\n".join(lines)
+    return lines
+
+
+# ------------------------------------------------------------ stored goldens
+
+def input_digest(weights: dict, inp: dict) -> str:
+    """sha256 (first 16 hex digits) of a workload's weights and per-block
+    inputs (the draft as drawn, before any consistent-draft replacement);
+    tests/golden/make_goldens.py stores it with the goldens."""
+    h = hashlib.sha256()
+    for k in sorted(weights):
+        h.update(k.encode())
+        h.update(np.ascontiguousarray(weights[k]).tobytes())
+    for k in ("h", "s", "target", "draft", "anchor", "temperature", "seed"):
+        h.update(k.encode())
+        h.update(np.ascontiguousarray(inp[k]).tobytes())
+    h.update(str(inp["offset"]).encode())
+    return h.hexdigest()[:16]
+
+
+def load_golden(name: str, weights: dict, inp: dict) -> dict:
+    """The oracle's stored outputs for every block of a named workload;
+    refuses a file computed from other inputs.  Replaces inp["draft"] by the
+    stored drafts (consistent blocks get Y*)."""
+    path = os.path.join(GOLDEN, f"{name}.npz")
+    g = dict(np.load(path))
+    digest = input_digest(weights, inp)
+    assert str(g["digest"]) == digest, (f"{path} was computed from other inputs (digest {g['digest']} != {digest}); "
+                                        "regenerate it with tests/golden/make_goldens.py")
+    inp["draft"] = g["draft"].copy()
+    return g
+
+
+def golden_oracle(g: dict, i: int) -> dict:
+    """One block of a stored golden in the layout of oracle.jacobi's result."""
+    it = int(g["iters"][i])
+    return dict(tokens=g["tokens"][i], iters=it, converged=int(g["converged"][i]), lse=g["lse"][i].astype(np.float64),
+                sel=g["sel"][i].astype(np.float64), z_final=g["z_final"][i].astype(np.float64),
+                trajectory=g["trajectory"][i, : it + 1], margins=g["margins"][i, :it].astype(np.float64))

@@ -50,3 +50,7 @@ def test_unsupported_shapes_are_rejected(lib):
                        (4100 + 1, 151936, 256, 16)]:
         w = X.XpressWeights(H, V, r, B, X.XPRESS_BF16, 0, *dummy)
         assert lib.xpress_refiner_create(C.byref(w), None, C.byref(h)) == X.XPRESS_ERR_UNSUPPORTED
+
+
+def test_wait_limit_argument_checks(lib):
+    assert lib.xpress_set_wait_limit(None, 1000) == X.XPRESS_ERR_INVALID_ARG

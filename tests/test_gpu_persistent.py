@@ -40,15 +40,17 @@ def _setup(X, b, seed):
 def _call(X, ref, cfg, inp, ws):
     d = device_inputs(X.XPRESS_BF16, inp)
     b = d["h"].shape[0]
-    out = ref.alloc_outputs(b)
+    out = ref.alloc_outputs(b, traj_K=cfg.K_max)
     blk_in = X.XpressBlockIn(b, d["h"].data_ptr(), d["s"].data_ptr(), d["draft"].data_ptr(), d["anchor"].data_ptr(),
                              d["temperature"].data_ptr(), d["seed"].data_ptr(), inp["offset"], cfg.K_max, 0)
     blk_out = X.XpressBlockOut(*[None if out.get(n) is None else out[n].data_ptr() for n in
-                                 ("tokens", "iters", "converged", "lse", "logit_sel", "z_final", "refined_logits")])
+                                 ("tokens", "iters", "converged", "lse", "logit_sel", "z_final", "refined_logits",
+                                  "trajectory")])
     X.xpress_refine_block(ref.handle, blk_in, blk_out, ws.data_ptr(), ws.numel(), ref.stream.cuda_stream)
     torch.cuda.synchronize()
     assert X.xpress_get_device_status(ws.data_ptr(), ref.stream.cuda_stream) == X.XPRESS_OK
-    return {k: out[k].cpu().numpy().copy() for k in ("tokens", "iters", "converged", "lse", "logit_sel", "z_final")}
+    return {k: out[k].cpu().numpy().copy() for k in ("tokens", "iters", "converged", "lse", "logit_sel", "z_final",
+                                                     "trajectory")}
 
 
 def test_interleaved_workspaces_and_batch_sizes(X):

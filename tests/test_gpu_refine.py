@@ -17,7 +17,8 @@ import pytest
 import oracle as O
 from paper_2608_02438_gb300 import workloads as W
 
-from _parity import compare_blocks, device_inputs, oracle_model, run_oracle
+from _parity import (compare_accept, compare_blocks, device_inputs, golden_oracle, load_golden, oracle_model,
+                     run_oracle)
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
@@ -43,7 +44,7 @@ def _run(X, cfg, weights, inp, K_max=None, fixed_K=False, want_logits=False, seq
     ref, dt = _refiner(X, cfg, weights)
     d = device_inputs(dt, inp, seqs)
     out = ref.refine_block(d["h"], d["s"], d["draft"], d["anchor"], d["temperature"], d["seed"], inp["offset"],
-                           K_max or cfg.K_max, fixed_K=fixed_K, want_logits=want_logits)
+                           K_max or cfg.K_max, fixed_K=fixed_K, want_logits=want_logits, want_traj=True)
     torch.cuda.synchronize()
     assert ref.device_status("refine", d["h"].shape[0]) == X.XPRESS_OK
     host = {k: (v.cpu().numpy() if v is not None else None) for k, v in out.items()}
@@ -153,7 +154,7 @@ def test_qwen3_shape_batch1(X, name):
 
 def _accept_check(X, cfg, w, inp):
     ref, d, g, m, orc = _check(X, cfg, w, inp, logits=False)
-    b = cfg.b if inp["h"].shape[0] == cfg.b else inp["h"].shape[0]
+    b = inp["h"].shape[0]
     out_dev = ref.refine_block(d["h"], d["s"], d["draft"], d["anchor"], d["temperature"], d["seed"], inp["offset"],
                                cfg.K_max)
     acc = ref.accept(d["target"], d["s"], out_dev["tokens"], out_dev["lse"], out_dev["logit_sel"],
@@ -162,15 +163,13 @@ def _accept_check(X, cfg, w, inp):
     assert ref.device_status("accept", b) == X.XPRESS_OK
     alen = acc["accept_len"].cpu().numpy()
     otok = acc["out_tokens"].cpu().numpy()
-    excused = 0
+    expect = {}
     for i in range(b):
         o = orc[i]
-        n, out, mg = O.accept(m, inp["target"][i], inp["s"][i], o["tokens"], o["lse"], o["sel"], o["z_final"],
-                              float(inp["temperature"][i]), int(inp["seed"][i]), inp["offset"])
-        if int(alen[i]) != n or otok[i].tolist() != out.tolist():
-            assert mg < 1e-3, f"block {i}: gpu {int(alen[i])} {otok[i].tolist()} | oracle {n} {out.tolist()} margin {mg}"
-            excused += 1
-    assert excused <= max(1, b // 100)
+        n, out, _, gaps = O.accept(m, inp["target"][i], inp["s"][i], o["tokens"], o["lse"], o["sel"], o["z_final"],
+                                   float(inp["temperature"][i]), int(inp["seed"][i]), inp["offset"], with_gaps=True)
+        expect[i] = (n, out, gaps)
+    compare_accept(alen, otok, expect, list(range(b)), inp["temperature"])
     return alen
 
 
@@ -191,44 +190,32 @@ def test_accept_qwen3_shape(X, name):
 
 # ------------------------------------------------- full-size batched configs
 
-def _consistent_drafts(cfg, w, inp):
-    """Blocks flagged `consistent` get the oracle's fixed point as their draft
-    (so they converge in one pass); computed by the oracle only."""
-    m = oracle_model(cfg, w)
-    for i in np.nonzero(inp["consistent"])[0]:
-        o = O.jacobi(m, inp["h"][i], inp["s"][i], int(inp["anchor"][i]), inp["draft"][i],
-                     float(inp["temperature"][i]), int(inp["seed"][i]), inp["offset"], cfg.B)
-        inp["draft"][i] = o["tokens"]
-    return inp
-
-
-@pytest.mark.parametrize("name,sample", [("serving_b32", (0, 5, 17, 31)), ("long_b64", (0, 1, 38, 63))])
-def test_batched_full_size_sampled(X, name, sample):
+# Every block of the batch-32 and batch-64 workloads against the oracle's
+# stored outputs (tests/golden/make_goldens.py writes them with the oracle
+# alone; the file's input digest must match the inputs drawn here).  Blocks
+# flagged consistent carry the oracle's fixed point Y* as their draft and
+# must converge in one pass.
+@pytest.mark.parametrize("name", ["serving_b32", "long_b64"])
+def test_batched_full_size_all_blocks(X, name):
     cfg, w, inp = W.make_workload(name)
-    if cfg.consistent_frac > 0:
-        inp = _consistent_drafts(cfg, w, inp)
-        sample = tuple(sorted(set(sample) | {int(np.nonzero(inp["consistent"])[0][0])}))
+    gold = load_golden(name, w, inp)
     ref, d, g = _run(X, cfg, w, inp)
-    m = oracle_model(cfg, w)
-    orc = {i: run_oracle(m, inp, i, cfg.K_max) for i in sample}
-    sub = {k: (v[list(sample)] if v is not None else None) for k, v in g.items()}
-    compare_blocks(sub, orc, list(sample), cfg.dtype, inp=inp)
-    # properties over every block: pass counts within [1, K_max]; blocks whose
-    # draft is already the fixed point converge in exactly one pass
-    assert (g["iters"] >= 1).all() and (g["iters"] <= cfg.K_max).all()
+    b = inp["h"].shape[0]
+    orc = {i: golden_oracle(gold, i) for i in range(b)}
+    compare_blocks(g, orc, list(range(b)), cfg.dtype, inp=inp)
     if cfg.consistent_frac > 0:
         cons = inp["consistent"]
+        assert cons.any()
         assert (g["iters"][cons] == 1).all() and (g["converged"][cons] == 1).all()
         np.testing.assert_array_equal(g["tokens"][cons], inp["draft"][cons])
-    # acceptance on the same blocks
+    # acceptance on the same blocks, from the GPU's refinement outputs
     out_dev = ref.refine_block(d["h"], d["s"], d["draft"], d["anchor"], d["temperature"], d["seed"], inp["offset"],
                                cfg.K_max)
     acc = ref.accept(d["target"], d["s"], out_dev["tokens"], out_dev["lse"], out_dev["logit_sel"],
                      out_dev["z_final"], d["temperature"], d["seed"], inp["offset"])
     torch.cuda.synchronize()
-    alen, otok = acc["accept_len"].cpu().numpy(), acc["out_tokens"].cpu().numpy()
-    for i in sample:
-        o = orc[i]
-        n, out, mg = O.accept(m, inp["target"][i], inp["s"][i], o["tokens"], o["lse"], o["sel"], o["z_final"],
-                              float(inp["temperature"][i]), int(inp["seed"][i]), inp["offset"])
-        assert (int(alen[i]) == n and otok[i].tolist() == out.tolist()) or mg < 1e-3, (i, alen[i], n)
+    assert ref.device_status("accept", b) == X.XPRESS_OK
+    expect = {i: (int(gold["accept_len"][i]), gold["out_tokens"][i], gold["accept_gaps"][i].astype(np.float64))
+              for i in range(b)}
+    compare_accept(acc["accept_len"].cpu().numpy(), acc["out_tokens"].cpu().numpy(), expect, list(range(b)),
+                   inp["temperature"])

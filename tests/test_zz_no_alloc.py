@@ -6,9 +6,11 @@ forbids device allocations after start-up) use xpress_accept_noalloc, which
 keeps its scratch in a fixed array inside the library.  This test checks, on
 two calls in a row through the C ABI, that its accept lengths and emitted
 tokens equal those of xpress_accept on the same inputs (integer outputs, so
-the comparison is exact), for a greedy and a sampling batch.  It passes when
-run alone in a fresh process (the first call then does the one-time address
-lookup) and after the other tests.
+the comparison is exact), for a greedy and a sampling batch: first two calls
+each followed by a synchronisation, then two calls issued back to back on
+one stream with no synchronisation between them (the stream orders them on
+the shared array).  It passes when run alone in a fresh process (the first
+call then does the one-time address lookup) and after the other tests.
 """
 import numpy as np
 import pytest
@@ -58,14 +60,21 @@ def test_noalloc_accept_matches_workspace_accept_on_two_calls(X):
                           d["temperature"], d["seed"], inp["offset"])
         torch.cuda.synchronize()
         want = {k: v.cpu().numpy().copy() for k, v in want.items()}
-        for call in range(2):
-            alen = torch.full((cfg.b,), -7, dtype=torch.int32, device="cuda")
-            otok = torch.full((cfg.b, cfg.B + 1), -7, dtype=torch.int32, device="cuda")
-            X.xpress_accept_noalloc(ref.handle, _accept_in(X, cfg, inp, d, out), alen.data_ptr(), otok.data_ptr(),
-                                    ref.stream.cuda_stream)
+        for sync_between in (True, False):
+            outs = []
+            for call in range(2):
+                alen = torch.full((cfg.b,), -7, dtype=torch.int32, device="cuda")
+                otok = torch.full((cfg.b, cfg.B + 1), -7, dtype=torch.int32, device="cuda")
+                X.xpress_accept_noalloc(ref.handle, _accept_in(X, cfg, inp, d, out), alen.data_ptr(),
+                                        otok.data_ptr(), ref.stream.cuda_stream)
+                if sync_between:
+                    torch.cuda.synchronize()
+                outs.append((alen, otok))
             torch.cuda.synchronize()
-            np.testing.assert_array_equal(alen.cpu().numpy(), want["accept_len"], err_msg=f"call {call}")
-            np.testing.assert_array_equal(otok.cpu().numpy(), want["out_tokens"], err_msg=f"call {call}")
+            for call, (alen, otok) in enumerate(outs):
+                tag = f"call {call}, {'synchronised' if sync_between else 'back to back'}"
+                np.testing.assert_array_equal(alen.cpu().numpy(), want["accept_len"], err_msg=tag)
+                np.testing.assert_array_equal(otok.cpu().numpy(), want["out_tokens"], err_msg=tag)
         ref.close()
 
 
