@@ -16,6 +16,8 @@ What each entry point follows (see the C file for the details):
 * :func:`jacobi`      -- Algorithm 1 (Sec. 4.2).
 * :func:`sequential`  -- the sequential decode Y* of Theorem 1.
 * :func:`accept`      -- greedy / lossless acceptance (Sec. 3.1, Sec. 4.3).
+* :func:`lm_head`     -- the base logits s = W_lm h and Algorithm 1's
+  Y^(0) = argmax s (Sec. 4.1, Fig. 2a).
 * :func:`philox`, :func:`uniform`, :func:`gumbel` -- Philox4x32-10
   (Salmon et al., SC'11) and the counter layout shared by both sides.
 
@@ -82,8 +84,9 @@ def _load():
             lib.xo_accept.argtypes = [MP, P, P, P, P, P, P, D, U64, U32, P, P, P, P]
             lib.xo_jacobi_seeds.argtypes = [MP, P, P, C.c_int32, P, D, P, I, U32, I, P, P]
             lib.xo_refine_accept_seeds.argtypes = [MP, P, P, P, C.c_int32, P, D, P, I, U32, I, P, P]
+            lib.xo_lm_head.argtypes = [P, P, I, I, I, I, P, P, P]
             for f in ("xo_forward", "xo_select", "xo_jacobi", "xo_sequential", "xo_accept",
-                      "xo_jacobi_seeds", "xo_refine_accept_seeds"):
+                      "xo_jacobi_seeds", "xo_refine_accept_seeds", "xo_lm_head"):
                 getattr(lib, f).restype = I
             _lib = lib
     return _lib
@@ -239,6 +242,23 @@ def accept(m: Model, target, s, tokens, lse, sel, z_final, T, seed, offset, with
     if with_gaps:
         return int(n[0]), out, float(mg[0]), gaps
     return int(n[0]), out, float(mg[0])
+
+
+def lm_head(W_lm, h, dtype):
+    """Base logits s = W_lm h (Sec. 4.1, Fig. 2a) for W_lm [V, H] and h [N, H]
+    in the storage dtype (F32 or BF16).  Returns (s_exact [N, V] float64,
+    s_store [N, V] in the storage dtype, argmax [N] of the stored rows)."""
+    W_lm = _storage(W_lm, dtype)
+    h = _storage(h, dtype)
+    V, H = W_lm.shape
+    N = h.shape[0]
+    assert h.shape == (N, H)
+    s_exact = np.empty((N, V))
+    s_store = np.empty((N, V), np.float32 if dtype == F32 else np.uint16)
+    am = np.empty(N, np.int32)
+    if _load().xo_lm_head(_ptr(W_lm), _ptr(h), V, H, N, dtype, _ptr(s_exact), _ptr(s_store), _ptr(am)):
+        raise ValueError("invalid arguments")
+    return s_exact, s_store, am
 
 
 def jacobi_seeds(m: Model, h, s, anchor, draft, T, seeds, offset, K_max):

@@ -18,6 +18,9 @@
  *   greedy acceptance              Sec. 3.1 (longest matching prefix + 1)
  *   lossless acceptance            Sec. 3.1 and Sec. 4.3 (accept w.p.
  *                                  min(1, p/q), else resample max(0, p-q))
+ *   base logits s = W_lm h         Sec. 4.1 / Fig. 2a (the target-sized LM
+ *                                  head that produces s_k; Algorithm 1's
+ *                                  Y^(0) = argmax s)
  *
  * Readings of points the paper leaves open:
  *   - sigma is selectable: SiLU (default), GELU(erf), ReLU (Sec. 4.1 says only
@@ -527,6 +530,46 @@ int xo_accept(const xo_model *M, const void *tgt, const void *s, const int32_t *
     *accept_len = n;
     if (margin) *margin = mg;
     free(row); free(sc);
+    return 0;
+}
+
+/* ------------------------------------------------------------ base logits */
+
+/* s_n = W_lm h_n for N hidden states (Sec. 4.1, Fig. 2a: the LM head that
+ * produces the drafter's base logits s_k), W_lm [V, H] and h [N, H] in the
+ * storage dtype.  Outputs: s_exact [N, V] (fp64 sums, optional); s_store
+ * [N, V] in the storage dtype (bf16 bit patterns rounded to nearest even, or
+ * fp32); argmax [N] = first index of the maximum of the stored row (Algorithm
+ * 1's Y^(0) = argmax_v s_k,v, taken on s as stored). */
+int xo_lm_head(const void *W_lm, const void *h, int V, int H, int N, int dtype, double *s_exact, void *s_store,
+               int32_t *argmax)
+{
+    if (V < 1 || H < 1 || N < 1) return -1;
+    double *row = (double *)malloc(sizeof(double) * V);
+    for (int n = 0; n < N; ++n) {
+        for (int v = 0; v < V; ++v) {
+            double acc = 0.0;
+            for (int i = 0; i < H; ++i)
+                acc += ld(W_lm, dtype, (size_t)v * H + i) * ld(h, dtype, (size_t)n * H + i);
+            if (s_exact) s_exact[(size_t)n * V + v] = acc;
+            if (dtype == XO_BF16) {
+                const float f = (float)xo_round_bf16(acc);
+                uint32_t u;
+                memcpy(&u, &f, 4);
+                if (s_store) ((uint16_t *)s_store)[(size_t)n * V + v] = (uint16_t)(u >> 16);
+                row[v] = (double)f;
+            } else {
+                const float f = (float)acc;
+                if (s_store) ((float *)s_store)[(size_t)n * V + v] = f;
+                row[v] = (double)f;
+            }
+        }
+        int best = 0;
+        for (int v = 1; v < V; ++v)
+            if (row[v] > row[best]) best = v;
+        if (argmax) argmax[n] = best;
+    }
+    free(row);
     return 0;
 }
 
