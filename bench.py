@@ -413,21 +413,61 @@ def run_xpress(args):
             else:
                 read_warm_ms = float(np.median(times[2:]))
         # Table 3's shape: the refinement with exactly K passes on every block
-        # (no early exit), L2 flushed before each call
-        fixed_us = {}
-        for K in (1, 4, 6, 8):
-            fs = [torch.cuda.Event(enable_timing=True) for _ in range(12)]
-            fe = [torch.cuda.Event(enable_timing=True) for _ in range(12)]
-            for i in range(12):
+        # (no early exit), the sequential decode (B dependent passes) and the
+        # Markov-head comparison head decoded the same way; L2 flushed before
+        # each call
+        def timed_us(call, reps=12):
+            fs = [torch.cuda.Event(enable_timing=True) for _ in range(reps)]
+            fe = [torch.cuda.Event(enable_timing=True) for _ in range(reps)]
+            for i in range(reps):
                 flush.zero_()
                 fs[i].record(stream)
-                ref.refine_block(d["h"], d["s"], d["draft"], d["anchor"], d["temperature"], d["seed"], inp["offset"],
-                                 K, fixed_K=True, out=out)
+                call()
                 fe[i].record(stream)
             torch.cuda.synchronize()
-            fixed_us[K] = 1000.0 * float(np.mean([s.elapsed_time(e) for s, e in zip(fs[2:], fe[2:])]))
+            return 1000.0 * float(np.mean([s.elapsed_time(e) for s, e in zip(fs[2:], fe[2:])]))
+
+        fixed_us = {K: timed_us(lambda: ref.refine_block(d["h"], d["s"], d["draft"], d["anchor"], d["temperature"],
+                                                         d["seed"], inp["offset"], K, fixed_K=True, out=out))
+                    for K in (1, 4, 6, 8)}
+        seq_K = max(cfg.K_max, cfg.B)
+        seq_us = timed_us(lambda: ref.refine_block(d["h"], d["s"], d["draft"], d["anchor"], d["temperature"],
+                                                   d["seed"], inp["offset"], seq_K, out=out,
+                                                   mode=X.XPRESS_MODE_SEQUENTIAL))
         if ref.device_status("refine", b) != X.XPRESS_OK:
-            raise RuntimeError("device status error (fixed-K calls)")
+            raise RuntimeError("device status error (fixed-K / sequential calls)")
+        mref = X.Refiner({k: X.to_device(v, dt) for k, v in W.markov_head_weights(w).items()}, cfg.H, cfg.V, cfg.r,
+                         cfg.B, dt, stream=stream)
+        markov_us = timed_us(lambda: mref.refine_block(d["h"], d["s"], d["draft"], d["anchor"], d["temperature"],
+                                                       d["seed"], inp["offset"], seq_K, out=out,
+                                                       mode=X.XPRESS_MODE_SEQUENTIAL))
+        if mref.device_status("refine", b) != X.XPRESS_OK:
+            raise RuntimeError("device status error (Markov head)")
+        mref.close()
+
+        lm_us, lm_bytes = None, None
+        if dt == X.XPRESS_BF16:
+            # the base logits s = W_lm h of the same hidden states (Fig. 2a), with
+            # Y^(0) = argmax s: a tied-size LM head W_lm ~ N(0, 0.02^2) [V, H],
+            # drawn on the device with a seeded generator
+            gen = torch.Generator(device=dev)
+            gen.manual_seed(20260101)
+            W_lm = (torch.randn((cfg.V, cfg.H), generator=gen, device=dev, dtype=torch.float32) * 0.02).to(
+                torch.bfloat16)
+            h_flat = d["h"].reshape(b * cfg.B, cfg.H)
+            s_lm = torch.empty((b * cfg.B, cfg.V), dtype=W_lm.dtype, device=dev)
+            y0_lm = torch.empty(b * cfg.B, dtype=torch.int32, device=dev)
+            lm_ws = torch.empty(X.xpress_lm_head_workspace_size(cfg.V, b * cfg.B) + 256, dtype=torch.uint8, device=dev)
+            lm_ptr = (lm_ws.data_ptr() + 255) & ~255
+
+            def lm_call():
+                X.xpress_lm_head(W_lm.data_ptr(), cfg.V, cfg.H, h_flat.data_ptr(), b * cfg.B, s_lm.data_ptr(),
+                                 y0_lm.data_ptr(), lm_ptr, lm_ws.numel() - (lm_ptr - lm_ws.data_ptr()), stream.cuda_stream)
+
+            lm_call()
+            lm_us = timed_us(lm_call, reps=20)
+            lm_bytes = cfg.V * cfg.H * 2 + b * cfg.B * cfg.H * 2 + b * cfg.B * cfg.V * 2
+            del W_lm, s_lm
     esz = 2 if dt == X.XPRESS_BF16 else 4
     sms = ref.torch.cuda.get_device_properties(dev).multi_processor_count
     if persistent:
@@ -473,6 +513,13 @@ def run_xpress(args):
             "passes_per_step": passes,
             "fixed_K_us_per_call": {str(k): v for k, v in fixed_us.items()},
             "fixed_K_us_per_pass": (fixed_us[8] - fixed_us[1]) / 7.0,
+            "sequential_decode_us_per_call": seq_us,
+            "markov_head_us_per_call": markov_us,
+            "lm_head": None if lm_us is None else {
+                "kernel": "k_lm_head32" if b * cfg.B <= 32 else "k_lm_head256", "us_per_call": lm_us,
+                "bytes_per_call": lm_bytes, "achieved_gbs": lm_bytes / (lm_us * 1e-6) / 1e9,
+                "frac": lm_bytes / (lm_us * 1e-6) / 1e9 / hbm, "bound": "hbm", "peak_gbs": hbm,
+                "tokens": b * cfg.B, "note": "s = W_lm h (bf16 out) + Y^(0) = argmax s, L2 flushed"},
             "e2e": {"value": e2e_value, "unit": "blocks/s", "h2d_bytes_per_step": int(h2d),
                     "d2h_bytes_per_step": int(d2h), "steps": n_e2e},
             "gpu_launches": per_step_launches * args.steps,

@@ -93,7 +93,18 @@ int xpress_refiner_destroy(xpress_refiner *refiner);
  *   K_max                   maximum number of refiner passes, >= 1
  *   fixed_K                 0: stop a block when a pass leaves it unchanged
  *                           (Algorithm 1's break); 1: run exactly K_max
- *                           passes on every block (Table 3 style timing)   */
+ *                           passes on every block (Table 3 style timing)
+ *   mode                    XPRESS_MODE_JACOBI: Algorithm 1 (parallel passes);
+ *                           XPRESS_MODE_SEQUENTIAL: the sequential decode of
+ *                           Theorem 1, y*_k = Select(R(y*_<k))_k for
+ *                           k = 1..B, one position per pass (B dependent
+ *                           passes; needs K_max >= B; draft and fixed_K are
+ *                           not used; iters = B, converged = 1).  Both modes
+ *                           reach the same block (Theorem 1); the second is
+ *                           the serial baseline the paper compares against
+ *                           (Table 3).                                      */
+typedef enum { XPRESS_MODE_JACOBI = 0, XPRESS_MODE_SEQUENTIAL = 1 } xpress_mode;
+
 typedef struct {
     int b;
     const void *h;
@@ -105,6 +116,7 @@ typedef struct {
     uint32_t offset;
     int K_max;
     int fixed_K;
+    int mode; /* xpress_mode */
 } xpress_block_in;
 
 /* Outputs (device pointers; each may be NULL except tokens):
@@ -217,6 +229,27 @@ int xpress_accept_noalloc(const xpress_refiner *refiner, const xpress_accept_in 
  * in `workspace` by xpress_refine_block / xpress_accept.  *status_out is an
  * xpress_status (XPRESS_OK, XPRESS_ERR_TIMEOUT or XPRESS_ERR_DEVICE_CHECK). */
 int xpress_get_device_status(void *workspace, void *stream, int32_t *status_out);
+
+/* Base logits of the drafter (Sec. 4.1, Fig. 2a: the target-sized LM head
+ * that produces s_k, the Correct term of the refiner) and Algorithm 1's seed
+ * Y^(0) = argmax_v s_k,v, for N hidden states.
+ *   W_lm        [V, H] bf16, row v = the LM head's row for token v
+ *   h           [N, H] bf16 hidden states (e.g. [b, B, H] flattened)
+ *   s_out       [N, V] bf16 (may be NULL): s[n][v] = sum_i h[n][i] W_lm[v][i],
+ *               accumulated in fp32 on tensor cores and rounded once to bf16
+ *               (nearest even) -- the storage format xpress_refine_block
+ *               reads
+ *   argmax_out  [N] int32 (may be NULL): the first maximum of the stored s
+ *               row (smallest id on ties), as xpress_refine_block takes it
+ *               when no draft is given
+ * At least one output must be given.  bf16 only; H % 8 == 0; W_lm and h
+ * 16-byte aligned.  workspace: >= xpress_lm_head_workspace_size(V, N) bytes,
+ * 256-byte aligned (per-CTA partial maxima).  Asynchronous on `stream`; two
+ * kernel launches.
+ * Errors: INVALID_ARG, WORKSPACE, CUDA. */
+size_t xpress_lm_head_workspace_size(int V, int N);
+int xpress_lm_head(const void *W_lm, int V, int H, const void *h, int N, void *s_out, int32_t *argmax_out,
+                   void *workspace, size_t ws_bytes, void *stream);
 
 /* Failure detection: every wait of the persistent small-batch kernel for
  * another CTA's progress (a monotone counter in the workspace) gives up after

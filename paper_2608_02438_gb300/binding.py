@@ -22,6 +22,7 @@ HEADER = os.path.join(ROOT, "include", "xpress.h")
 
 XPRESS_F32, XPRESS_BF16 = 0, 1
 XPRESS_ACT_SILU, XPRESS_ACT_GELU, XPRESS_ACT_RELU = 0, 1, 2
+XPRESS_MODE_JACOBI, XPRESS_MODE_SEQUENTIAL = 0, 1
 XPRESS_OK = 0
 XPRESS_ERR_INVALID_ARG, XPRESS_ERR_UNSUPPORTED, XPRESS_ERR_CUDA = -1, -2, -3
 XPRESS_ERR_WORKSPACE, XPRESS_ERR_TIMEOUT, XPRESS_ERR_DEVICE_CHECK = -4, -5, -6
@@ -35,7 +36,7 @@ class XpressWeights(C.Structure):
 class XpressBlockIn(C.Structure):
     _fields_ = [("b", C.c_int), ("h", C.c_void_p), ("s", C.c_void_p), ("draft", C.c_void_p),
                 ("anchor", C.c_void_p), ("temperature", C.c_void_p), ("seed", C.c_void_p),
-                ("offset", C.c_uint32), ("K_max", C.c_int), ("fixed_K", C.c_int)]
+                ("offset", C.c_uint32), ("K_max", C.c_int), ("fixed_K", C.c_int), ("mode", C.c_int)]
 
 
 class XpressBlockOut(C.Structure):
@@ -88,6 +89,10 @@ def load(path: str = LIB_PATH):
     lib.xpress_get_pass_count.restype = I
     lib.xpress_accept_noalloc.argtypes = [P, C.POINTER(XpressAcceptIn), P, P, P]
     lib.xpress_accept_noalloc.restype = I
+    lib.xpress_lm_head_workspace_size.argtypes = [I, I]
+    lib.xpress_lm_head_workspace_size.restype = S
+    lib.xpress_lm_head.argtypes = [P, I, I, P, I, P, P, P, S, P]
+    lib.xpress_lm_head.restype = I
     lib.xpress_set_wait_limit.argtypes = [P, C.c_uint64]
     lib.xpress_set_wait_limit.restype = I
     lib.xpress_profile_read_prepare.argtypes = [P, P, I, I, P]
@@ -166,6 +171,35 @@ def xpress_get_pass_count(ws_ptr: int, stream: int) -> int:
     return v.value
 
 
+def xpress_lm_head_workspace_size(V: int, N: int) -> int:
+    return load().xpress_lm_head_workspace_size(V, N)
+
+
+def xpress_lm_head(W_lm_ptr: int, V: int, H: int, h_ptr: int, N: int, s_ptr, argmax_ptr, ws_ptr: int, ws_bytes: int,
+                   stream: int) -> None:
+    _check("xpress_lm_head", load().xpress_lm_head(C.c_void_p(W_lm_ptr), V, H, C.c_void_p(h_ptr), N,
+                                                   C.c_void_p(s_ptr) if s_ptr else None,
+                                                   C.c_void_p(argmax_ptr) if argmax_ptr else None,
+                                                   C.c_void_p(ws_ptr), ws_bytes, C.c_void_p(stream)))
+
+
+def lm_head(W_lm, h, s_out=None, argmax_out=None, stream=None) -> int:
+    """Base logits s = W_lm h (bf16 device tensors W_lm [V, H], h [N, H];
+    s_out [N, V] bf16 and / or argmax_out [N] int32 device tensors) on
+    `stream` (default: torch's current stream).  Returns XPRESS_OK."""
+    import torch
+    V, H = W_lm.shape
+    N = h.shape[0]
+    st = stream if stream is not None else torch.cuda.current_stream()
+    size = xpress_lm_head_workspace_size(V, N)
+    ws = torch.empty(size + 256, dtype=torch.uint8, device=W_lm.device)
+    ptr = (ws.data_ptr() + 255) & ~255
+    xpress_lm_head(W_lm.data_ptr(), V, H, h.data_ptr(), N, None if s_out is None else s_out.data_ptr(),
+                   None if argmax_out is None else argmax_out.data_ptr(), ptr, size, st.cuda_stream)
+    lm_head.workspace = ws                       # kept alive until the next call (the launch is asynchronous)
+    return XPRESS_OK
+
+
 def xpress_set_wait_limit(handle, limit_ns: int) -> None:
     _check("xpress_set_wait_limit", load().xpress_set_wait_limit(handle, limit_ns))
 
@@ -233,14 +267,15 @@ class Refiner:
                     else None)
 
     def refine_block(self, h, s, draft, anchor, temperature, seed, offset: int, K_max: int, fixed_K: bool = False,
-                     out: dict | None = None, want_logits: bool = False, want_traj: bool = False) -> dict:
+                     out: dict | None = None, want_logits: bool = False, want_traj: bool = False,
+                     mode: int = XPRESS_MODE_JACOBI) -> dict:
         b = h.shape[0]
         out = out if out is not None else self.alloc_outputs(b, want_logits, K_max if want_traj else 0)
         if out.get("trajectory") is not None and tuple(out["trajectory"].shape) != (b, K_max, self.B):
             raise ValueError("trajectory must be [b, K_max, B]")
         blk_in = XpressBlockIn(b, h.data_ptr(), s.data_ptr(), None if draft is None else draft.data_ptr(),
                                anchor.data_ptr(), temperature.data_ptr(), seed.data_ptr(), offset, K_max,
-                               int(bool(fixed_K)))
+                               int(bool(fixed_K)), int(mode))
         blk_out = XpressBlockOut(*[None if out.get(n) is None else out[n].data_ptr() for n in
                                    ("tokens", "iters", "converged", "lse", "logit_sel", "z_final",
                                     "refined_logits", "trajectory")])

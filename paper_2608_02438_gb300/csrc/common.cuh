@@ -99,6 +99,7 @@ struct Params {
     int b, B, H, V, N;           // N = b * B
     int dtype, act;              // 0 f32, 1 bf16;  0 SiLU, 1 GELU, 2 ReLU
     int K_max, fixed_K;
+    int sequential;              // 1: Theorem 1's sequential decode (pass j evaluates position j only)
     uint32_t offset;
     int S;                       // vocabulary ranges of the Read kernel
     int use_graph;               // 1: the pass loop is a graph WHILE node

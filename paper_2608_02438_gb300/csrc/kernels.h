@@ -62,6 +62,15 @@ __global__ void k_pre_tc(const Params *pp, const __grid_constant__ CUtensorMap t
                          int kslice);
 extern const size_t kPreTcSmemBytes;
 
+// lm_head.cu (base logits s = W_lm h and Y^(0) = argmax s; NT tokens per chunk, 32 or 256)
+__global__ void k_lm_head32(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_h, int V,
+                            int H, int N, uint16_t *s_out, Partial *part, int32_t *status);
+__global__ void k_lm_head256(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_h,
+                             int V, int H, int N, uint16_t *s_out, Partial *part, int32_t *status);
+__global__ void k_lm_head_argmax(const Partial *part, int G, int N, int32_t *argmax_out);
+extern const size_t kLmHeadSmemBytes[2];
+extern const int kLmHeadThreads;
+
 // accept_kernels.cu
 __global__ void k_acc_rows(AcceptParams p);
 __global__ void k_acc_finalize(AcceptParams p, int chunks);

@@ -170,11 +170,19 @@ __device__ __forceinline__ SeqState converge_state(const Params &p, const SeqSta
                                                    const int *yold, int base)
 {
     const int B = p.B;
+    SeqState ns = st;
+    ns.iters = st.iters + 1;
+    if (p.sequential) {
+        // sequential decode: the pass decided position m + 1 from the
+        // decided prefix; the block is complete after position B - 1
+        ns.m = st.m + 1;
+        ns.active = ns.m + 1 < B;
+        ns.converged = !ns.active;
+        return ns;
+    }
     int first = -1;
     for (int k = st.m + 1; k < B; ++k)
         if (ynew[base + k] != yold[base + k]) { first = k; break; }
-    SeqState ns = st;
-    ns.iters = st.iters + 1;
     ns.converged = first < 0;
     if (p.fixed_K) {
         ns.active = ns.iters < p.K_max;
@@ -192,6 +200,14 @@ __device__ __forceinline__ SeqState converge_state(const Params &p, const SeqSta
         ns.m = first;
     }
     return ns;
+}
+
+// Positions the next pass evaluates for a block in state ns: all after the
+// first one the last pass changed (Algorithm 1 with Theorem 1's frontier), or
+// the next one of the sequential decode.
+__device__ __forceinline__ int eval_count(const Params &p, const SeqState &ns)
+{
+    return ns.active ? (p.sequential ? 1 : p.B - 1 - ns.m) : 0;
 }
 
 __device__ __forceinline__ void converge_block(const Params &p, int s, const SeqState &st, const int *ynew,
@@ -222,7 +238,7 @@ __device__ __forceinline__ bool converge_pack_small(const Params &p, const SeqSt
             if (p.iters) p.iters[q] = ns.iters;
             if (p.converged) p.converged[q] = ns.converged;
         }
-        c = ns.active ? B - 1 - ns.m : 0;
+        c = eval_count(p, ns);
     }
     int incl = c;
 #pragma unroll
@@ -269,7 +285,7 @@ __device__ __forceinline__ void pack_next_pass(const Params &p, cudaGraphConditi
             const volatile int *src = reinterpret_cast<const volatile int *>(&p.st[q]);
             ns.active = src[0]; ns.m = src[1]; ns.iters = src[2]; ns.converged = src[3];
             mine = (p.temperature[q] > 0.0f) == (cls == 1);
-            c = (mine && ns.active) ? B - 1 - ns.m : 0;
+            c = mine ? eval_count(p, ns) : 0;
         }
         int incl = c;
 #pragma unroll

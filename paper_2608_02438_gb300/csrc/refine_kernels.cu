@@ -37,16 +37,17 @@ __global__ void k_init(Params pin, Params *pdev, cudaGraphConditionalHandle hand
     const Params &p = pin;
     const unsigned long long t_start = globaltimer_ns();
     const int t = blockIdx.x * blockDim.x + threadIdx.x;
+    const int n0 = p.sequential ? p.b : p.N;   // tokens of the first pass: all positions, or position 0
     if (t == 0) {
         *pdev = pin;
-        p.ctl[CTL_NACT] = p.N;
+        p.ctl[CTL_NACT] = n0;
         p.ctl[CTL_DONE] = 0;
         p.ctl[CTL_PASS] = 0;
-        p.ctl[CTL_EVAL] = p.N;
+        p.ctl[CTL_EVAL] = n0;
         if (p.use_graph) cudaGraphSetConditional(handle, 1u);
     }
+    if (t < n0) p.act_tok[t] = p.sequential ? t * p.B : t;
     if (t < p.N) {
-        p.act_tok[t] = t;
         if (p.draft) {
             int y = p.draft[t];
             if (y < 0 || y >= p.V) { set_status(p.status, ST_BOUNDS); y = 0; }
@@ -55,7 +56,8 @@ __global__ void k_init(Params pin, Params *pdev, cudaGraphConditionalHandle hand
     }
     if (t < p.b) {
         SeqState s{};
-        s.active = 1; s.m = -1; s.iters = 0; s.converged = 0; s.off = t * p.B; s.cnt = p.B;
+        s.active = 1; s.m = -1; s.iters = 0; s.converged = 0;
+        s.off = p.sequential ? t : t * p.B; s.cnt = p.sequential ? 1 : p.B;
         p.st[t] = s;
         if (p.anchor[t] < 0 || p.anchor[t] >= p.V) set_status(p.status, ST_BOUNDS);
         if (p.iters) p.iters[t] = 0;
@@ -599,7 +601,7 @@ __global__ void __cluster_dims__(MLP_CLUSTER, 1, 1) __launch_bounds__(256, 2) k_
     if (trs) trace_mark(p.trace, trs, t_start);
     const SeqState st = p.st[s];
     if (!st.active) return;            // uniform over the cluster
-    const int m = st.m, cnt = B - 1 - m, off = st.off;
+    const int m = st.m, cnt = st.cnt, off = st.off;
     const int d0 = rank * 32;
 
     __shared__ float e[MAX_B][32];                     // gathered E' rows, own channel slice
@@ -753,7 +755,7 @@ __global__ void __launch_bounds__(1024) k_reduce(const Params *__restrict__ pp, 
     __shared__ int last;
     __shared__ int ynew[MAX_B], yold[MAX_B];
     __shared__ int wsum[32];
-    if (st.active && warp < B && warp > st.m) {
+    if (st.active && warp < B && warp > st.m && warp <= st.m + st.cnt) {
         const int k = warp, i = st.off + (k - st.m - 1), tok = s * B + k;
         if (lane == 0) yold[k] = p.tokens[tok];
         const float T = p.temperature[s];

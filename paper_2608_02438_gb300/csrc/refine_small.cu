@@ -744,7 +744,7 @@ __device__ __forceinline__ void gather_e(const Params &p, const int *x, const in
 // pass that mixes.
 template <int KH>
 __device__ __noinline__ void mix_block16(const float *e, const uint16_t *Lp, const float *pc, uint16_t *cop,
-                                         float (*cown)[32], int d, int m, int off, int rank)
+                                         float (*cown)[32], int d, int m, int mlast, int off, int rank)
 {
     constexpr int BB = FULL_C_MAX_B;
     float2 er[BB];
@@ -753,7 +753,7 @@ __device__ __noinline__ void mix_block16(const float *e, const uint16_t *Lp, con
 #pragma unroll
     for (int q = 0; q < BB / 2; ++q) {
         const int k = BB - 1 - ((q >> 1) * 4 + (KH ? 1 + (q & 1) : (q & 1) * 3));
-        if (k <= m) continue;
+        if (k <= m || k > mlast) continue;
         float2 a0 = er[k], a1 = make_float2(0.0f, 0.0f);
         const uint32_t *lrow = reinterpret_cast<const uint32_t *>(Lp + (k * (k - 1) / 2) * RANK + d);
 #pragma unroll
@@ -824,27 +824,30 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
             }
         }
         sh.x[tid] = y;
-        sh.tok[tid] = tid;
+        sh.tok[tid] = p.sequential ? tid * B : tid;           // the first pass: all positions, or position 0
     }
+    const int n0 = p.sequential ? b : N;                       // tokens the first pass evaluates
     if (lead) {
+        if (tid < n0) p.act_tok[tid] = p.sequential ? tid * B : tid;
         if (tid < N) {
-            p.act_tok[tid] = tid;
             if (p.draft) p.tokens[tid] = sh.x[tid];
         }
         if (tid < b) {
             SeqState s{};
-            s.active = 1; s.m = -1; s.iters = 0; s.converged = 0; s.off = tid * B; s.cnt = B;
+            s.active = 1; s.m = -1; s.iters = 0; s.converged = 0;
+            s.off = p.sequential ? tid : tid * B; s.cnt = p.sequential ? 1 : B;
             p.st[tid] = s;
             if (p.anchor[tid] < 0 || p.anchor[tid] >= V) atomicOr(reinterpret_cast<int *>(&c->status.v), ST_BOUNDS);
             if (p.iters) p.iters[tid] = 0;
             if (p.converged) p.converged[tid] = 0;
         }
-        if (tid == 0) { p.ctl[CTL_NACT] = N; p.ctl[CTL_DONE] = 0; p.ctl[CTL_PASS] = 0; p.ctl[CTL_EVAL] = N; }
+        if (tid == 0) { p.ctl[CTL_NACT] = n0; p.ctl[CTL_DONE] = 0; p.ctl[CTL_PASS] = 0; p.ctl[CTL_EVAL] = n0; }
         if (tid < 64) p.best64[tid] = 0ull;                    // both parities, before pass 0's z
     }
     if (tid < b) {
         SeqState s{};
-        s.active = 1; s.m = -1; s.iters = 0; s.converged = 0; s.off = tid * B; s.cnt = B;
+        s.active = 1; s.m = -1; s.iters = 0; s.converged = 0;
+        s.off = p.sequential ? tid : tid * B; s.cnt = p.sequential ? 1 : B;
         sh.st[tid] = s;
         sh.anch[tid] = p.anchor[tid];
         const float T = p.temperature[tid];
@@ -854,8 +857,8 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
         // warm the mix's code on scratch operands (cop and cown are rewritten
         // before their first use; e and pc hold whatever is there)
         const int d = 2 * (tid & 127);
-        if (tid < 128) mix_block16<0>(e, Lp, pc, cop, sh.cown, d, -1, 0, rank);
-        else mix_block16<1>(e, Lp, pc, cop, sh.cown, d, -1, 0, rank);
+        if (tid < 128) mix_block16<0>(e, Lp, pc, cop, sh.cown, d, -1, B - 1, 0, rank);
+        else mix_block16<1>(e, Lp, pc, cop, sh.cown, d, -1, B - 1, 0, rank);
     }
     if (lead && tid == 0 && p.trace) trace_mark(p.trace, 250, t_start);
     if (tid == 0) sh.go = wait_count(c, &c->pre_done.v, (unsigned)p.S, p.wait_ns);
@@ -892,12 +895,12 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
     float *zf = p.z_final ? p.z_final : p.zbuf;
     uint16_t *zpack = static_cast<uint16_t *>(p.zpack);
     const uint64_t eprow_policy = policy_evict_first();       // E' rows are read once per pass
-    int n = N;                                                 // evaluated tokens of this pass
+    int n = n0;                                                // evaluated tokens of this pass
     for (int pass = 0;; ++pass) {
         const unsigned long long t_pass = globaltimer_ns();
         const int trs = (lead && tid == 0 && p.trace && pass < 3) ? 210 + 8 * pass : 0;
         if (trs) trace_mark(p.trace, trs, t_pass);
-        const bool first_c = pass == 0 && p.draft;             // c formed by the Read CTAs
+        const bool first_c = pass == 0 && p.draft && !p.sequential;   // c formed by the Read CTAs
         if (!first_c) {
             if (pass > 0) cp_async_wait<0>();                  // issued at the end of the previous pass
             else gather_e(p, sh.x, sh.anch, e, CH, cb, tid, nth);
@@ -931,9 +934,12 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
                 for (int s = 0; s < b; ++s) {
                     const SeqState st = sh.st[s];
                     if (!st.active) continue;
-                    if (kh == 0) mix_block16<0>(e + s * B * CH, Lp, pc + s * B * CH, cop, sh.cown, d, st.m, st.off, rank);
+                    if (kh == 0)
+                        mix_block16<0>(e + s * B * CH, Lp, pc + s * B * CH, cop, sh.cown, d, st.m, st.m + st.cnt,
+                                       st.off, rank);
                     else if (kh == 1)
-                        mix_block16<1>(e + s * B * CH, Lp, pc + s * B * CH, cop, sh.cown, d, st.m, st.off, rank);
+                        mix_block16<1>(e + s * B * CH, Lp, pc + s * B * CH, cop, sh.cown, d, st.m, st.m + st.cnt,
+                                       st.off, rank);
                 }
             } else if (kh < 2)
                 for (int s = 0; s < b; ++s) {
@@ -945,7 +951,7 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
                         er[j2] = j2 < B ? *reinterpret_cast<const float2 *>(e + (s * B + j2) * CH + d)
                                         : make_float2(0.0f, 0.0f);
 #pragma unroll 1
-                    for (int k = st.m + 1; k < B; ++k) {
+                    for (int k = st.m + 1; k <= st.m + st.cnt; ++k) {
                         if ((((B - 1 - k + 1) >> 1) & 1) != kh) continue;
                         const int t = st.off + k - st.m - 1;
                         float2 a0 = *reinterpret_cast<const float2 *>(e + (s * B + k) * CH + d);
@@ -1000,7 +1006,8 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
             __syncthreads();
             if (tid == 0) {
                 red_add_release_gpu(&c->c_ready.v, 1u);
-                sh.go = wait_count(c, &c->c_ready.v, (unsigned)(8 * (pass + (p.draft ? 0 : 1))), p.wait_ns);
+                sh.go = wait_count(c, &c->c_ready.v, (unsigned)(8 * (pass + (p.draft && !p.sequential ? 0 : 1))),
+                                   p.wait_ns);
                 if (trs) trace_mark(p.trace, trs + 2, t_pass);
             }
             __syncthreads();
@@ -1163,7 +1170,7 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
                     if (p.iters) p.iters[lane] = ns.iters;
                     if (p.converged) p.converged[lane] = ns.converged;
                 }
-                cnt = ns.active ? B - 1 - ns.m : 0;
+                cnt = eval_count(p, ns);
             }
             int incl = cnt;
 #pragma unroll

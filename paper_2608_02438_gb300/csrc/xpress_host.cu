@@ -18,7 +18,7 @@ using namespace xp;
 
 namespace {
 
-constexpr int XPRESS_VERSION = 1;
+constexpr int XPRESS_VERSION = 2;
 constexpr int CACHE_SLOTS = 8;
 
 PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder()
@@ -217,6 +217,7 @@ Params make_params(const xpress_refiner *R, const xpress_block_in *in, const xpr
     P.act = R->w.act;
     P.K_max = in->K_max;
     P.fixed_K = in->fixed_K ? 1 : 0;
+    P.sequential = in->mode == XPRESS_MODE_SEQUENTIAL ? 1 : 0;
     P.offset = in->offset;
     P.S = L.S;
     P.use_graph = 1;
@@ -300,7 +301,11 @@ int set_kernel_attributes()
             cudaFuncSetAttribute(k_refine_small, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)kRefineSmallSmemBytes) != cudaSuccess ||
             cudaFuncSetAttribute(k_pre_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kPreTcSmemBytes) !=
-                cudaSuccess) {
+                cudaSuccess ||
+            cudaFuncSetAttribute(k_lm_head32, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kLmHeadSmemBytes[0]) !=
+                cudaSuccess ||
+            cudaFuncSetAttribute(k_lm_head256, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)kLmHeadSmemBytes[1]) != cudaSuccess) {
             (void)cudaGetLastError();
             rc = XPRESS_ERR_CUDA;
         }
@@ -787,6 +792,9 @@ int xpress_refine_block(const xpress_refiner *Rc, const xpress_block_in *in, con
         return XPRESS_ERR_INVALID_ARG;
     if ((reinterpret_cast<uintptr_t>(in->s) & 15) || (reinterpret_cast<uintptr_t>(in->h) & 15))
         return XPRESS_ERR_INVALID_ARG;
+    if ((in->mode != XPRESS_MODE_JACOBI && in->mode != XPRESS_MODE_SEQUENTIAL) ||
+        (in->mode == XPRESS_MODE_SEQUENTIAL && in->K_max < R->w.B))
+        return XPRESS_ERR_INVALID_ARG;
     const Layout L = make_layout(R, in->b);
     if (const int rc = check_ws(ws, ws_bytes, L.total)) return rc;
     Params P = make_params(R, in, out, ws, L);
@@ -994,6 +1002,66 @@ int xpress_get_pass_count(void *ws, void *stream, int32_t *passes_out)
     if (!ws || !passes_out) return XPRESS_ERR_INVALID_ARG;
     XP_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
     XP_CUDA(cudaMemcpy(passes_out, static_cast<char *>(ws) + 64 + CTL_PASS * 4, 4, cudaMemcpyDeviceToHost));
+    return XPRESS_OK;
+}
+
+}  // extern "C"
+
+// ------------------------------------------------------------------ base logits
+
+namespace {
+int lm_grid(int V)
+{
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) !=
+                                                  cudaSuccess) {
+        (void)cudaGetLastError();
+        return 0;
+    }
+    const int nvt = (V + 127) / 128;
+    return nvt < sms ? nvt : sms;
+}
+}  // namespace
+
+extern "C" {
+
+size_t xpress_lm_head_workspace_size(int V, int N)
+{
+    if (V < 1 || N < 1) return 0;
+    const int G = lm_grid(V);
+    if (G < 1) return 0;
+    return 256 + align256((size_t)N * G * sizeof(Partial));
+}
+
+int xpress_lm_head(const void *W_lm, int V, int H, const void *h, int N, void *s_out, int32_t *argmax_out,
+                   void *ws, size_t ws_bytes, void *stream)
+{
+    if (!W_lm || !h || (!s_out && !argmax_out) || V < 1 || N < 1 || H < 8 || (H % 8)) return XPRESS_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(W_lm) & 15) || (reinterpret_cast<uintptr_t>(h) & 15))
+        return XPRESS_ERR_INVALID_ARG;
+    const int G = lm_grid(V);
+    if (G < 1) return XPRESS_ERR_CUDA;
+    if (const int rc = check_ws(ws, ws_bytes, 256 + align256((size_t)N * G * sizeof(Partial)))) return rc;
+    if (set_kernel_attributes() != XPRESS_OK) return XPRESS_ERR_CUDA;
+    const bool wide = N > 32;                       // token chunks of 256, else one chunk of 32
+    CUtensorMap tw{}, th{};
+    if (!make_tmap_bf16(&tw, W_lm, (uint64_t)H, (uint64_t)V, 64, 128) ||
+        !make_tmap_bf16(&th, h, (uint64_t)H, (uint64_t)N, 64, wide ? 256 : 32))
+        return XPRESS_ERR_CUDA;
+    char *w = static_cast<char *>(ws);
+    int32_t *status = reinterpret_cast<int32_t *>(w);
+    Partial *part = reinterpret_cast<Partial *>(w + 256);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    XP_CUDA(cudaMemsetAsync(status, 0, 4, st));
+    if (wide)
+        k_lm_head256<<<G, kLmHeadThreads, kLmHeadSmemBytes[1], st>>>(tw, th, V, H, N,
+                                                                        static_cast<uint16_t *>(s_out), part, status);
+    else
+        k_lm_head32<<<G, kLmHeadThreads, kLmHeadSmemBytes[0], st>>>(tw, th, V, H, N, static_cast<uint16_t *>(s_out),
+                                                                       part, status);
+    XP_CUDA(cudaGetLastError());
+    if (argmax_out) XP_CUDA(launch_pdl(k_lm_head_argmax, dim3((unsigned)((N + 7) / 8)), dim3(256), 0, st,
+                                       (const Partial *)part, G, N, argmax_out));
     return XPRESS_OK;
 }
 

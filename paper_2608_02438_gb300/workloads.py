@@ -188,6 +188,20 @@ def make_inputs(cfg: Config, b: int | None = None, seed_offset: int = 0) -> dict
                 seed=seeds.astype(np.uint64), offset=int(7 + seed_offset), consistent=consistent)
 
 
+def markov_head_weights(weights: dict) -> dict:
+    """The Markov-head comparison head (Sec. 2, Sec. 5 Table 3) in the
+    refiner's notation: the correction for position k depends only on the id
+    of token k-1, through the folded token slot -- the same W_e, W_in and W_r,
+    with the hidden-state slots (W_h, W_g), the mixer L and the Trans MLP
+    (W_1, W_2) switched off (zero).  Then z_k = c_k = W_in[:, 2r:3r] W_e[x_{k-1}]
+    and l_k = s_k + W_r z_k, a rank-r bias table indexed by the previous
+    token, decoded one position after another."""
+    out = dict(weights)
+    for k in ("W_h", "W_g", "L", "W1", "W2"):
+        out[k] = np.zeros_like(weights[k])
+    return out
+
+
 _WEIGHT_CACHE: dict = {}
 
 
