@@ -6,6 +6,14 @@
 
 namespace xp {
 
+// One draw of the lossless acceptance: block seq, position k (< B: the first
+// rejected position, residual draw; = B: the bonus draw from p_{B+1}).
+struct DrawDesc {
+    int seq, k;
+    float invT, lse_p, lse_q;
+    int pad[3];
+};
+
 struct AcceptParams {
     int b, B, V, dtype;
     const void *target, *s;
@@ -17,8 +25,9 @@ struct AcceptParams {
     int32_t *accept_len, *out_tokens;
     int32_t *status;
     Partial *rowpart;   // [b * (B + 1), chunks]
-    int32_t *ticket;    // [b] draw chunks done (cleared by k_acc_rows)
-    Partial *spart;     // [b, chunks]
+    int32_t *ticket;    // [2]: draws listed, draw CTAs done (cleared by k_acc_rows)
+    DrawDesc *draws;    // [b] draws of the sampling blocks (k_acc_decide)
+    unsigned long long *keys;   // [b, 2] best residual / p draw key (argmax_key), cleared by k_acc_decide
 };
 
 // refine_kernels.cu
@@ -72,8 +81,10 @@ extern const size_t kLmHeadSmemBytes[2];
 extern const int kLmHeadThreads;
 
 // accept_kernels.cu
-__global__ void k_acc_rows(AcceptParams p);
-__global__ void k_acc_finalize(AcceptParams p, int chunks);
+__global__ void k_acc_rows(AcceptParams p, int chunks);
+__global__ void k_acc_decide(AcceptParams p, int chunks);
+__global__ void k_acc_draw(AcceptParams p);        // bf16 refiners (tensor-core products)
+__global__ void k_acc_draw_simt(AcceptParams p);   // fp32 refiners
 
 // fp32: c and sigma(W_1 c) of up to 32 tokens in fp32; bf16: the same as
 // bf16 tensor-core operands plus this CTA's share of sigma(W_1 c)

@@ -853,23 +853,31 @@ int xpress_refine_block(const xpress_refiner *Rc, const xpress_block_in *in, con
 
 namespace {
 struct AcceptLayout {
-    size_t status = 0, rowpart = 256, ticket = 0, spart = 0, total = 0;
-    int chunks = 1, chunks2 = 1;
+    size_t status = 0, rowpart = 256, ticket = 0, draws = 0, keys = 0, total = 0;
+    int chunks = 1, row_ctas = 1, draw_ctas = 1;
 };
 
 AcceptLayout accept_layout(const xpress_refiner *R, int b)
 {
     AcceptLayout A;
     const int rows = b * (R->w.B + 1);
+    // chunks per target row: enough items to spread a small batch over the
+    // SMs, and chunks of at most 32768 ids so that a large batch's items
+    // balance over the persistent grid
     int c = (2 * R->num_sms + rows - 1) / rows;
+    const int cv = (R->w.V + 32767) / 32768;
+    c = c > cv ? c : cv;
     A.chunks = c < 1 ? 1 : (c > 64 ? 64 : c);
-    int c2 = (2 * R->num_sms + b - 1) / b;
-    A.chunks2 = c2 < 1 ? 1 : (c2 > 512 ? 512 : c2);
+    const int items = rows * A.chunks;
+    A.row_ctas = items < 4 * R->num_sms ? items : 4 * R->num_sms;
+    A.draw_ctas = 2 * R->num_sms;                 // two CTAs of k_acc_draw fit on an SM
     size_t o = A.rowpart + align256((size_t)rows * A.chunks * sizeof(Partial));
     A.ticket = o;
-    o += align256((size_t)b * 4);
-    A.spart = o;
-    o += align256((size_t)b * A.chunks2 * sizeof(Partial));
+    o += 256;
+    A.draws = o;
+    o += align256((size_t)b * sizeof(DrawDesc));
+    A.keys = o;
+    o += align256((size_t)b * 2 * sizeof(unsigned long long));
     A.total = o;
     return A;
 }
@@ -917,12 +925,15 @@ int accept_launch(const xpress_refiner *R, const xpress_accept_in *in, int32_t *
     P.status = reinterpret_cast<int32_t *>(w + A.status);
     P.rowpart = reinterpret_cast<Partial *>(w + A.rowpart);
     P.ticket = reinterpret_cast<int32_t *>(w + A.ticket);
-    P.spart = reinterpret_cast<Partial *>(w + A.spart);
+    P.draws = reinterpret_cast<DrawDesc *>(w + A.draws);
+    P.keys = reinterpret_cast<unsigned long long *>(w + A.keys);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    // both are chained to their predecessor with programmatic dependent
-    // launch (k_acc_rows clears the status word and the draw tickets)
-    XP_CUDA(launch_pdl(k_acc_rows, dim3(in->b * (R->w.B + 1), A.chunks), dim3(256), 0, st, P));
-    XP_CUDA(launch_pdl(k_acc_finalize, dim3(in->b, A.chunks2), dim3(256), 0, st, P, A.chunks));
+    // each is chained to its predecessor with programmatic dependent launch
+    // (k_acc_rows clears the status word and the draw counters)
+    XP_CUDA(launch_pdl(k_acc_rows, dim3(A.row_ctas), dim3(256), 0, st, P, A.chunks));
+    XP_CUDA(launch_pdl(k_acc_decide, dim3(in->b), dim3(32), 0, st, P, A.chunks));
+    XP_CUDA(launch_pdl(R->w.dtype == XPRESS_BF16 ? k_acc_draw : k_acc_draw_simt, dim3(A.draw_ctas), dim3(256), 0, st,
+                       P));
     XP_CUDA(cudaGetLastError());
     return XPRESS_OK;
 }
