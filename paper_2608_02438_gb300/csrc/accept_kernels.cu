@@ -81,9 +81,14 @@ __global__ void __launch_bounds__(256) k_acc_rows(AcceptParams p, int chunks)
         Partial a{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
         const size_t base = (size_t)row * p.V;
         // four 8-value pieces per thread in flight (the stream is latency-bound
-        // with one); pieces are visited in increasing id order per thread
+        // with one); pieces are visited in increasing id order per thread.
+        // Sampling rows keep the running max in log2 units (y = x log2(e) / T)
+        // and rescale the running sum once per piece, so that each value costs
+        // one multiply, one max, one subtract, one ex2 and one add.
         constexpr int U = 4;
         const int step = 8 * blockDim.x;
+        const float c2 = invT * 1.4426950408889634f;
+        float m2 = -INFINITY, s2 = 0.0f;
         for (int vv = v0 + 8 * threadIdx.x; vv < v1; vv += U * step) {
             float x[U][8];
 #pragma unroll
@@ -96,22 +101,39 @@ __global__ void __launch_bounds__(256) k_acc_rows(AcceptParams p, int chunks)
                 const int v = vv + u * step;
                 if (v >= v1) break;
                 const int nv = min(8, v1 - v);
+                if (nv < 8)                               // the chunk's ragged end: past V reads as -inf
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        if (j >= nv) x[u][j] = -INFINITY;
                 if (invT <= 0.0f) {
+                    const float m8 = fmaxf(fmaxf(fmaxf(x[u][0], x[u][1]), fmaxf(x[u][2], x[u][3])),
+                                           fmaxf(fmaxf(x[u][4], x[u][5]), fmaxf(x[u][6], x[u][7])));
+                    if (m8 > a.best) {                    // the first id of the piece that holds it
+                        int jj = 7;
 #pragma unroll
-                    for (int j = 0; j < 8; ++j)
-                        if (j < nv && x[u][j] > a.best) { a.best = x[u][j]; a.idx = v + j; }
+                        for (int j = 6; j >= 0; --j)
+                            if (x[u][j] == m8) jj = j;
+                        a.best = m8;
+                        a.idx = v + jj;
+                    }
                 } else {
-                    float mx = -INFINITY;
+                    float y[8];
 #pragma unroll
-                    for (int j = 0; j < 8; ++j)
-                        if (j < nv) mx = fmaxf(mx, x[u][j] * invT);
-                    float sum = 0.0f;
+                    for (int j = 0; j < 8; ++j) y[j] = x[u][j] * c2;
+                    const float m8 = fmaxf(fmaxf(fmaxf(y[0], y[1]), fmaxf(y[2], y[3])),
+                                           fmaxf(fmaxf(y[4], y[5]), fmaxf(y[6], y[7])));
+                    const float mn = fmaxf(m2, m8);
+                    float t = 0.0f;
 #pragma unroll
-                    for (int j = 0; j < 8; ++j)
-                        if (j < nv) sum += __expf(x[u][j] * invT - mx);
-                    merge_lse(a.m, a.s, mx, sum);
+                    for (int j = 0; j < 8; ++j) t += ex2_approx(y[j] - mn);
+                    s2 = s2 * ex2_approx(m2 - mn) + t;
+                    m2 = mn;
                 }
             }
+        }
+        if (invT > 0.0f && m2 > -INFINITY) {              // back to natural units: sum e^(x / T - m)
+            a.m = m2 * 0.6931471805599453f;
+            a.s = s2;
         }
         sp[threadIdx.x] = a;
         __syncthreads();
