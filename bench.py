@@ -248,6 +248,20 @@ def run_reference(args):
     return 0
 
 
+def lm_head_line(us, nbytes, flops, hbm, tc_peak, tokens):
+    """The base-logit LM head against its roofline: the weight stream (HBM)
+    for few tokens, the bf16 tensor pipe once the arithmetic intensity nears
+    the ridge point."""
+    gbs = nbytes / (us * 1e-6) / 1e9
+    tfs = flops / (us * 1e-6) / 1e12
+    tensor = flops / nbytes >= 0.75 * tc_peak * 1e3 / hbm
+    return {"kernel": "k_lm_head32" if tokens <= 32 else "k_lm_head256", "us_per_call": us, "tokens": tokens,
+            "bytes_per_call": nbytes, "flops_per_call": flops, "achieved_gbs": gbs, "achieved_tflops": tfs,
+            "bound": "tensor" if tensor else "hbm", "peak": tc_peak if tensor else hbm,
+            "frac": tfs / tc_peak if tensor else gbs / hbm,
+            "note": "s = W_lm h (bf16 out) + Y^(0) = argmax s, L2 flushed; peaks of measured"}
+
+
 def run_xpress(args):
     import torch
     from paper_2608_02438_gb300 import binding as X
@@ -515,11 +529,8 @@ def run_xpress(args):
             "fixed_K_us_per_pass": (fixed_us[8] - fixed_us[1]) / 7.0,
             "sequential_decode_us_per_call": seq_us,
             "markov_head_us_per_call": markov_us,
-            "lm_head": None if lm_us is None else {
-                "kernel": "k_lm_head32" if b * cfg.B <= 32 else "k_lm_head256", "us_per_call": lm_us,
-                "bytes_per_call": lm_bytes, "achieved_gbs": lm_bytes / (lm_us * 1e-6) / 1e9,
-                "frac": lm_bytes / (lm_us * 1e-6) / 1e9 / hbm, "bound": "hbm", "peak_gbs": hbm,
-                "tokens": b * cfg.B, "note": "s = W_lm h (bf16 out) + Y^(0) = argmax s, L2 flushed"},
+            "lm_head": None if lm_us is None else lm_head_line(lm_us, lm_bytes, 2.0 * cfg.V * cfg.H * b * cfg.B, hbm,
+                                                               tc_peak, b * cfg.B),
             "e2e": {"value": e2e_value, "unit": "blocks/s", "h2d_bytes_per_step": int(h2d),
                     "d2h_bytes_per_step": int(d2h), "steps": n_e2e},
             "gpu_launches": per_step_launches * args.steps,
