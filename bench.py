@@ -312,9 +312,12 @@ def run_xpress(args):
         persistent = (dt == X.XPRESS_BF16 and b * cfg.B <= 32 and os.environ.get("XPRESS_SMALL", "1") != "0")
         small = b * cfg.B <= 32
         if persistent:
-            per_step_launches = 1 + 2
+            per_step_launches = 1 + 3
         else:
-            per_step_launches = 1 + (1 if small else 2) + 1 + passes * (2 if small else 3) + 2
+            # per pass: Trans (k_mix_mlp, or k_mix_c + two k_trans_tc for bf16
+            # above 32 tokens), Read, reduce (fused into the Read at <= 32 tokens)
+            per_pass = 2 if small else (5 if dt == X.XPRESS_BF16 else 3)
+            per_step_launches = 1 + (1 if small else 2) + 1 + passes * per_pass + 3
         starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
         ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
         if world > 1:

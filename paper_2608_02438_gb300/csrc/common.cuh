@@ -130,6 +130,8 @@ struct Params {
     int32_t *act_tok;            // [N] packed evaluated tokens (global token ids)
     void *zpack;                 // [N, r] W_r operand of the evaluated tokens
     float *zbuf;                 // [N, r] fp32 z when the caller passes no z_final
+    float *cbuf;                 // [N, r] fp32 c of the evaluated tokens (graph path, bf16, > 32 tokens)
+    uint16_t *ubuf;              // [N, 2r] bf16 sigma(W_1 c) of the evaluated tokens (same)
     RPartial *part;              // [N, S] token-major (a token's ranges are contiguous)
     // persistent small-batch kernel only
     const uint16_t *Fhl;         // [2][2r, H] bf16: hi then lo term of the fp32 rows W_in[:, 0:r] W_h,

@@ -65,6 +65,12 @@ __global__ void k_pack_L(const uint16_t *L, uint16_t *Lpk, int B);
 extern const size_t kRefineSmallSmemBytes;
 constexpr int SMALL_TRANS_CTAS = 8;
 
+// trans_tc.cu (bf16, more than 32 tokens: Fuse + Mix, then Trans on tcgen05)
+__global__ void k_mix_c(const Params *pp);
+__global__ void k_trans_tc(const Params *pp, const __grid_constant__ CUtensorMap tmap_a,
+                           const __grid_constant__ CUtensorMap tmap_b, int K, int mode);
+extern const size_t kTransTcSmemBytes;
+
 // pre_tc.cu (bf16, more than 32 tokens: the hidden projection on tcgen05)
 __global__ void k_pre_tc(const Params *pp, const __grid_constant__ CUtensorMap tmap_h,
                          const __grid_constant__ CUtensorMap tmap_wh, const __grid_constant__ CUtensorMap tmap_wg,

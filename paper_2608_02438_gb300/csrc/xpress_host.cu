@@ -70,7 +70,7 @@ size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 struct Layout {
     size_t status = 0, ctl = 64, params = 256, st = 0, upart = 0, pc = 0, ynew = 0, acttok = 0, zpack = 0,
-           zbuf = 0, part = 0, total = 0;
+           zbuf = 0, part = 0, cbuf = 0, ubuf = 0, total = 0;
     size_t sctl = 0, cx = 0, ux = 0, pcx = 0, c0x = 0, rmax = 0, best64 = 0;
     int ksplit = 1, kchunk = 0, S = 1;
     bool gemv = false;
@@ -90,6 +90,7 @@ struct xpress_refiner {
     CUtensorMap tmap_wr32{};               // W_r boxes of 32 rows (k_refine_small, partial blocks)
     CUtensorMap tmap_wh{}, tmap_wg{};      // W_h, W_g boxes of 256 rows x 64
     CUtensorMap tmap_fhi{}, tmap_flo{};    // folded projection, hi / lo term, boxes of 256 rows x 64 (k_pre_tc)
+    CUtensorMap tmap_w1{}, tmap_w2{};      // W_1 [2r, r], W_2 [r, 2r], boxes of 32 rows x 64 (k_trans_tc)
     int device = 0;
     int num_sms = 0;
     unsigned long long wait_ns = 2000000000ull;   // bound on the persistent kernel's waits for other CTAs
@@ -185,6 +186,12 @@ Layout make_layout(const xpress_refiner *R, int b)
     L.tcv = use_tcv(R, b);
     L.part = o;
     o = align256(o + (size_t)L.S * N * sizeof(RPartial));
+    if (R->use_tc && !L.tcv) {
+        L.cbuf = o;
+        o = align256(o + (size_t)N * RANK * 4);
+        L.ubuf = o;
+        o = align256(o + (size_t)N * 2 * RANK * 2);
+    }
     if (L.small) {
         L.cx = o;
         o = align256(o + (size_t)32 * RANK * 2);
@@ -258,6 +265,10 @@ Params make_params(const xpress_refiner *R, const xpress_block_in *in, const xpr
     P.zpack = w + L.zpack;
     P.zbuf = reinterpret_cast<float *>(w + L.zbuf);
     P.part = reinterpret_cast<RPartial *>(w + L.part);
+    if (L.cbuf) {
+        P.cbuf = reinterpret_cast<float *>(w + L.cbuf);
+        P.ubuf = reinterpret_cast<uint16_t *>(w + L.ubuf);
+    }
     if (L.small) {
         P.use_graph = 0;
         P.Fhl = R->Fhl;
@@ -303,6 +314,8 @@ int set_kernel_attributes()
             cudaFuncSetAttribute(k_pre_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kPreTcSmemBytes) !=
                 cudaSuccess ||
             cudaFuncSetAttribute(k_lm_head32, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kLmHeadSmemBytes[0]) !=
+                cudaSuccess ||
+            cudaFuncSetAttribute(k_trans_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kTransTcSmemBytes) !=
                 cudaSuccess ||
             cudaFuncSetAttribute(k_lm_head256, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)kLmHeadSmemBytes[1]) != cudaSuccess) {
@@ -372,6 +385,34 @@ void launch_pre_gemm(const Layout &L, int N, Params *pdev, cudaStream_t st)
     }
 }
 
+// Tensor maps of the Trans operands on tcgen05 (graph path, bf16, more than
+// 32 tokens): bf16(c) in zpack [N, r] and u in ubuf [N, 2r], boxes of 128
+// token rows x 64.
+bool make_trans_maps(const Params &P, CUtensorMap *tc, CUtensorMap *tu)
+{
+    return make_tmap_bf16(tc, P.zpack, RANK, (uint64_t)P.N, 64, 128) &&
+           make_tmap_bf16(tu, P.ubuf, 2 * RANK, (uint64_t)P.N, 64, 128);
+}
+
+// Fuse + Mix and Trans of one pass: the multi-kernel tcgen05 form (bf16, more
+// than 32 tokens), else k_mix_mlp.
+cudaError_t launch_trans(const xpress_refiner *R, const Layout &L, const Params &P, Params *pdev, cudaStream_t st,
+                         const CUtensorMap &tc, const CUtensorMap &tu)
+{
+    const int b = P.b;
+    if (!(R->use_tc && !L.tcv))
+        return launch_pdl(k_mix_mlp, dim3(8, b), dim3(256), mix_mlp_smem(P.dtype), st, (const Params *)pdev);
+    const unsigned mt = (unsigned)((P.N + 127) / 128);
+    cudaError_t e = launch_pdl(k_mix_c, dim3(8, b), dim3(256), 0, st, (const Params *)pdev);
+    if (e == cudaSuccess)
+        e = launch_pdl(k_trans_tc, dim3(mt, 2 * RANK / 32), dim3(192), kTransTcSmemBytes, st, (const Params *)pdev, tc,
+                       R->tmap_w1, RANK, 1);
+    if (e == cudaSuccess)
+        e = launch_pdl(k_trans_tc, dim3(mt, RANK / 32), dim3(192), kTransTcSmemBytes, st, (const Params *)pdev, tu,
+                       R->tmap_w2, 2 * RANK, 2);
+    return e;
+}
+
 void destroy_entry(GraphEntry &e)
 {
     if (e.exec) cudaGraphExecDestroy(e.exec);
@@ -381,7 +422,8 @@ void destroy_entry(GraphEntry &e)
 
 // Builds the per-(workspace, b) graph:
 //   memset(status) -> k_init -> [k_rowmax] -> k_pre_gemm x2 -> k_pre_mix ->
-//   WHILE (cond) { k_mix_mlp -> k_read_{tc,simt} -> k_reduce (updates cond) }
+//   WHILE (cond) { Trans (k_mix_mlp, or k_mix_c -> k_trans_tc x2) -> k_read_{tc,simt} -> k_reduce
+//                  (updates cond) }
 int build_graph(xpress_refiner *R, GraphEntry &e, const Params &P, const Layout &L, void *ws)
 {
     const int b = P.b, N = P.N;
@@ -454,8 +496,10 @@ int build_graph(xpress_refiner *R, GraphEntry &e, const Params &P, const Layout 
         return XPRESS_ERR_CUDA;
     }
     cudaGraph_t body = cp.conditional.phGraph_out[0];
+    CUtensorMap tmap_c{}, tmap_u{};
+    if (R->use_tc && !L.tcv && !make_trans_maps(P, &tmap_c, &tmap_u)) return XPRESS_ERR_CUDA;
     XP_CUDA(cudaStreamBeginCaptureToGraph(cs, body, nullptr, nullptr, 0, cudaStreamCaptureModeThreadLocal));
-    XP_CUDA(launch_pdl(k_mix_mlp, dim3(8, b), dim3(256), mix_mlp_smem(P.dtype), cs, (const Params *)pdev));
+    XP_CUDA(launch_trans(R, L, P, pdev, cs, tmap_c, tmap_u));
     if (L.tcv) {
         // the small-batch Read kernel also ends the pass (fused reduce)
         XP_CUDA(launch_pdl(k_read_tcv, dim3(L.S), dim3(kReadTcvThreads), kReadTcvSmemBytes, cs, (const Params *)pdev,
@@ -550,9 +594,11 @@ int run_eager(xpress_refiner *R, Params P, const Layout &L, void *ws, cudaStream
     kt.start("pre_mix");
     k_pre_mix<<<dim3(b, RANK / 32), 256, L.pre_tc ? pre_mix_smem_folded(P.B) : pre_mix_smem(P.B), st>>>(pdev);
     kt.stop();
+    CUtensorMap tmap_c{}, tmap_u{};
+    if (R->use_tc && !L.tcv && !make_trans_maps(P, &tmap_c, &tmap_u)) return XPRESS_ERR_CUDA;
     for (int pass = 0; pass < P.K_max; ++pass) {
         kt.start("mix_mlp");
-        k_mix_mlp<<<dim3(8, b), 256, mix_mlp_smem(P.dtype), st>>>(pdev);
+        XP_CUDA(launch_trans(R, L, P, pdev, st, tmap_c, tmap_u));
         kt.stop();
         kt.start("read");
         if (L.tcv)
@@ -737,6 +783,11 @@ int xpress_refiner_create(const xpress_weights *w, void *stream, xpress_refiner 
             k_fold_hidden<<<dim3((w->H + 255) / 256, 2 * RANK / 8), 256, 0, st>>>(
                 static_cast<const uint16_t *>(w->W_h), static_cast<const uint16_t *>(w->W_g),
                 static_cast<const uint16_t *>(w->W_in), R->Fhl, w->H);
+            if (!make_tmap_bf16(&R->tmap_w1, w->W1, RANK, 2 * RANK, 64, 32) ||
+                !make_tmap_bf16(&R->tmap_w2, w->W2, 2 * RANK, RANK, 64, 32)) {
+                rc = XPRESS_ERR_CUDA;
+                break;
+            }
             if (!make_tmap_bf16(&R->tmap_fhi, R->Fhl, (uint64_t)w->H, 2 * RANK, 64, 256) ||
                 !make_tmap_bf16(&R->tmap_flo, R->Fhl + (size_t)2 * RANK * w->H, (uint64_t)w->H, 2 * RANK, 64, 256)) {
                 rc = XPRESS_ERR_CUDA;
