@@ -49,6 +49,8 @@ SMALL_SOURCES = [CSRC + f for f in ("refine_small.cu", "tcv_common.cuh", "mlp_co
 SMALL_SUMMARY = "profiles/k_refine_small_qwen3_8b_greedy.txt"
 READ_SOURCES = [CSRC + "read_tc.cu", CSRC + "common.cuh"]
 READ_SUMMARIES = {"long_b64": "profiles/k_read_tc_long_b64.txt"}
+LM_SOURCES = [CSRC + "lm_head.cu", CSRC + "common.cuh"]
+LM_SUMMARIES = {16: "profiles/k_lm_head32_qwen3_8b_n16.txt"}
 
 
 def dist_env():
@@ -532,8 +534,9 @@ def run_xpress(args):
             "fixed_K_us_per_pass": (fixed_us[8] - fixed_us[1]) / 7.0,
             "sequential_decode_us_per_call": seq_us,
             "markov_head_us_per_call": markov_us,
-            "lm_head": None if lm_us is None else lm_head_line(lm_us, lm_bytes, 2.0 * cfg.V * cfg.H * b * cfg.B, hbm,
-                                                               tc_peak, b * cfg.B),
+            "lm_head": None if lm_us is None else dict(
+                lm_head_line(lm_us, lm_bytes, 2.0 * cfg.V * cfg.H * b * cfg.B, hbm, tc_peak, b * cfg.B),
+                traffic=profiled_traffic(LM_SUMMARIES.get(b * cfg.B, ""), source_hash(LM_SOURCES))),
             "e2e": {"value": e2e_value, "unit": "blocks/s", "h2d_bytes_per_step": int(h2d),
                     "d2h_bytes_per_step": int(d2h), "steps": n_e2e},
             "gpu_launches": per_step_launches * args.steps,
