@@ -282,21 +282,25 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             // s of item k into ring slot k % TC_SPF (cp.async, L2 only; zero-filled
             // past V or for an invalid thread), one commit group per item
             const int et = threadIdx.x - 64;
-            auto issue_s = [&](int k) {
-                if (k < items) {
-                    const int v0 = (vt0 + k / g_count) * TC_BN + (g_first + k % g_count) * GROUP;
+            // the next item to issue, walked forward without divisions
+            int is_k = 0, is_vt = vt0, is_gl = g_first;
+            auto issue_next = [&]() {
+                if (is_k < items) {
+                    const int v0 = is_vt * TC_BN + is_gl * GROUP;
 #pragma unroll
                     for (int c = 0; c < 4; ++c) {
                         const int vv = v0 + 8 * c;
                         const bool in = valid && vv < p.V;
-                        cp_async16(&sS[((k % TC_SPF) * 4 + c) * (TC_EPI_WARPS * 32) + et], in ? srow + vv : srow,
+                        cp_async16(&sS[((is_k % TC_SPF) * 4 + c) * (TC_EPI_WARPS * 32) + et], in ? srow + vv : srow,
                                    in ? 16u : 0u, once);
                     }
                 }
                 cp_async_commit();
+                ++is_k;
+                if (++is_gl == g_first + g_count) { is_gl = g_first; ++is_vt; }
             };
 #pragma unroll
-            for (int k = 0; k < TC_SPF - 1; ++k) issue_s(k);
+            for (int k = 0; k < TC_SPF - 1; ++k) issue_next();
             if (g_count == 0)
                 for (int vt = vt0; vt < vt1; ++vt) {
                     const int buf = t & 1;
@@ -307,8 +311,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     if (lane == 0) mbar_arrive(&sh.tempty[buf]);
                     ++t;
                 }
+            int vt = vt0, gl = g_first;                  // the item being folded
             for (int it = 0; it < items; ++it) {
-                const int vt = vt0 + it / g_count, gl = g_first + it % g_count;
                 const int buf = t & 1;
                 if (gl == g_first) {
                     if (valid && invT > 0.0f)
@@ -316,7 +320,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     if (!mbar_wait(&sh.tfull[buf], (t >> 1) & 1, abort)) { ok = false; break; }
                     tc_fence_after();
                 }
-                issue_s(it + TC_SPF - 1);
+                issue_next();                           // item it + TC_SPF - 1
                 cp_async_wait<TC_SPF - 1>();        // item it has landed
                 uint4 cur[4];
 #pragma unroll
@@ -348,6 +352,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     __syncwarp();
                     if (lane == 0) mbar_arrive(&sh.tempty[buf]);
                     ++t;
+                    gl = g_first;
+                    ++vt;
+                } else {
+                    ++gl;
                 }
             }
             cp_async_wait<0>();                      // nothing in flight into the ring
