@@ -18,6 +18,8 @@ What each entry point follows (see the C file for the details):
 * :func:`accept`      -- greedy / lossless acceptance (Sec. 3.1, Sec. 4.3).
 * :func:`lm_head`     -- the base logits s = W_lm h and Algorithm 1's
   Y^(0) = argmax s (Sec. 4.1, Fig. 2a).
+* :func:`train_step`  -- the training objective of Sec. 4.3 and its gradient
+  with respect to every refiner weight.
 * :func:`philox`, :func:`uniform`, :func:`gumbel` -- Philox4x32-10
   (Salmon et al., SC'11) and the counter layout shared by both sides.
 
@@ -85,8 +87,9 @@ def _load():
             lib.xo_jacobi_seeds.argtypes = [MP, P, P, C.c_int32, P, D, P, I, U32, I, P, P]
             lib.xo_refine_accept_seeds.argtypes = [MP, P, P, P, C.c_int32, P, D, P, I, U32, I, P, P]
             lib.xo_lm_head.argtypes = [P, P, I, I, I, I, P, P, P]
+            lib.xo_train_step.argtypes = [MP, P, P, P, P, C.c_int32, D, D, D, D, D, P] + [P] * 8
             for f in ("xo_forward", "xo_select", "xo_jacobi", "xo_sequential", "xo_accept",
-                      "xo_jacobi_seeds", "xo_refine_accept_seeds", "xo_lm_head"):
+                      "xo_jacobi_seeds", "xo_refine_accept_seeds", "xo_lm_head", "xo_train_step"):
                 getattr(lib, f).restype = I
             _lib = lib
     return _lib
@@ -259,6 +262,30 @@ def lm_head(W_lm, h, dtype):
     if _load().xo_lm_head(_ptr(W_lm), _ptr(h), V, H, N, dtype, _ptr(s_exact), _ptr(s_store), _ptr(am)):
         raise ValueError("invalid arguments")
     return s_exact, s_store, am
+
+
+GRAD_NAMES = ("W_e", "W_h", "W_g", "W_in", "L", "W1", "W2", "W_r")
+
+
+def train_step(m: Model, h, s, target, ystar, anchor, a_ce=1.0, a_l1=1.0, gamma=4.0, lam=0.6, beta=0.3,
+               grads=True):
+    """Sec. 4.3 on one block (T = 1): losses (L(p^r), L(p^b), L(p^r-hat),
+    L_total) and, with grads, dL_total/dtheta for every refiner weight (dict
+    of float64 arrays shaped like the weights).  lam weighs the drafter-anchor
+    term and beta the consistency term, as in the total-loss equation; the
+    defaults are the experimental section's values by role (consistency 0.3,
+    anchor 0.6 at the start of its annealing)."""
+    h = m._a(h, (m.B, m.H))
+    s = m._a(s, (m.B, m.V))
+    tgt = m._a(target, (m.B, m.V))
+    y = np.ascontiguousarray(ystar, dtype=np.int32)
+    loss = np.zeros(4)
+    g = {n: np.zeros(m.w[n].shape) for n in GRAD_NAMES} if grads else None
+    ptrs = [_ptr(g[n]) if grads else None for n in GRAD_NAMES]
+    if _load().xo_train_step(C.byref(m.c), _ptr(h), _ptr(s), _ptr(tgt), _ptr(y), int(anchor), float(a_ce),
+                             float(a_l1), float(gamma), float(lam), float(beta), _ptr(loss), *ptrs):
+        raise ValueError("invalid arguments")
+    return loss, g
 
 
 def jacobi_seeds(m: Model, h, s, anchor, draft, T, seeds, offset, K_max):

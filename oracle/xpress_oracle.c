@@ -18,6 +18,9 @@
  *   greedy acceptance              Sec. 3.1 (longest matching prefix + 1)
  *   lossless acceptance            Sec. 3.1 and Sec. 4.3 (accept w.p.
  *                                  min(1, p/q), else resample max(0, p-q))
+ *   training objective             Sec. 4.3 (cross-entropy + L1 / total
+ *                                  variation, position weights, drafter
+ *                                  anchor, consistency forward)
  *   base logits s = W_lm h         Sec. 4.1 / Fig. 2a (the target-sized LM
  *                                  head that produces s_k; Algorithm 1's
  *                                  Y^(0) = argmax s)
@@ -573,6 +576,247 @@ int xo_lm_head(const void *W_lm, const void *h, int V, int H, int N, int dtype, 
     return 0;
 }
 
+/* ------------------------------------------------------------ training */
+
+/* d sigma / dt for the three readings of sigma. */
+static double sigma_prime(int act, double t)
+{
+    switch (act) {
+    case XO_RELU: return t > 0 ? 1.0 : 0.0;
+    case XO_GELU: return 0.5 * (1.0 + erf(t / sqrt(2.0))) + t * exp(-0.5 * t * t) / sqrt(2.0 * 3.14159265358979323846);
+    default: {
+        const double sg = 1.0 / (1.0 + exp(-t));
+        return sg + t * sg * (1.0 - sg);
+    }
+    }
+}
+
+/* Gradients of the refiner weights (fp64, same shapes and layouts as xo_model's
+ * tensors). */
+typedef struct {
+    double *W_e, *W_h, *W_g, *W_in, *L, *W1, *W2, *W_r;
+} xo_grads;
+
+/* log sum exp and softmax of row[0..n-1]. */
+static double softmax_row(const double *row, int n, double *p)
+{
+    double mx = -INFINITY;
+    for (int v = 0; v < n; ++v) if (row[v] > mx) mx = row[v];
+    double tot = 0.0;
+    for (int v = 0; v < n; ++v) tot += exp(row[v] - mx);
+    const double lse = mx + log(tot);
+    if (p) for (int v = 0; v < n; ++v) p[v] = exp(row[v] - lse);
+    return lse;
+}
+
+/* The per-position loss of Sec. 4.3 for distribution p (softmax of ell) at
+ * position k against the target distribution q = softmax(tgt_k) and the
+ * ground-truth token y*:  a_ce (-log p(y*)) + a_l1 |p - q|_1.  With dl given,
+ * also its gradient with respect to ell, times `scale`:
+ *   a_ce (p_v - [v = y*]) + a_l1 p_v (sgn(p_v - q_v) - sum_u sgn(p_u - q_u) p_u). */
+static double position_loss(const double *ell, const double *tgtrow, int V, int ystar, double a_ce, double a_l1,
+                            double scale, double *dl, double *p, double *q)
+{
+    const double lse = softmax_row(ell, V, p);
+    softmax_row(tgtrow, V, q);
+    double l1 = 0.0, S = 0.0;
+    for (int v = 0; v < V; ++v) {
+        const double d = p[v] - q[v];
+        l1 += fabs(d);
+        S += (d > 0 ? 1.0 : (d < 0 ? -1.0 : 0.0)) * p[v];
+    }
+    if (dl)
+        for (int v = 0; v < V; ++v) {
+            const double d = p[v] - q[v];
+            const double sg = d > 0 ? 1.0 : (d < 0 ? -1.0 : 0.0);
+            dl[v] = scale * (a_ce * (p[v] - (v == ystar ? 1.0 : 0.0)) + a_l1 * p[v] * (sg - S));
+        }
+    return a_ce * (lse - ell[ystar]) + a_l1 * l1;
+}
+
+/* One refiner forward with token inputs x[0..B-1] (x_0 the anchor), the loss
+ * L(p) = sum_k w_k loss_k of its refined distributions p_k = softmax(l_k)
+ * (T = 1) against the ground truth ystar and the target logits, and, with g
+ * given, mult * dL/dtheta added into g.  The bf16 operand roundings of the
+ * forward (c before W_1, sigma(W_1 c) before W_2, z before W_r) pass the
+ * gradient through unchanged (straight-through). */
+static double refiner_loss(const xo_model *M, const void *h, const void *s, const void *tgt, const int32_t *x,
+                           const int32_t *ystar, double a_ce, double a_l1, double gam, double mult, xo_grads *g)
+{
+    const int H = M->H, V = M->V, r = M->r, B = M->B, R2 = 2 * r;
+    double *uh = calloc((size_t)B * r, 8), *ug = calloc(r, 8), *gm = calloc(H, 8);
+    double *a = calloc((size_t)B * r, 8), *c = calloc((size_t)B * r, 8), *cop = calloc((size_t)B * r, 8);
+    double *tp = calloc((size_t)B * R2, 8), *uop = calloc((size_t)B * R2, 8);
+    double *z = calloc((size_t)B * r, 8), *zop = calloc((size_t)B * r, 8);
+    double *ell = malloc(sizeof(double) * V), *tr = malloc(sizeof(double) * V), *dl = malloc(sizeof(double) * V);
+    double *p = malloc(sizeof(double) * V), *q = malloc(sizeof(double) * V);
+    double *dz = calloc((size_t)B * r, 8), *dc = calloc((size_t)B * r, 8), *da = calloc((size_t)B * r, 8);
+    double *du = calloc(R2, 8), *dt = calloc(R2, 8), *dug = calloc(r, 8);
+    /* Fuse: u_h,k = W_h h_k, g = mean_j h_j, u_g = W_g g, a_k = W_in [u_h,k; u_g; W_e[x_k]] */
+    for (int j = 0; j < B; ++j)
+        for (int i = 0; i < H; ++i) gm[i] += ld(h, M->dtype, (size_t)j * H + i);
+    for (int i = 0; i < H; ++i) gm[i] /= B;
+    for (int d = 0; d < r; ++d) {
+        double acc = 0.0;
+        for (int i = 0; i < H; ++i) acc += ld(M->W_g, M->dtype, (size_t)d * H + i) * gm[i];
+        ug[d] = acc;
+        for (int k = 0; k < B; ++k) {
+            double ah = 0.0;
+            for (int i = 0; i < H; ++i) ah += ld(M->W_h, M->dtype, (size_t)d * H + i) * ld(h, M->dtype, (size_t)k * H + i);
+            uh[(size_t)k * r + d] = ah;
+        }
+    }
+    for (int k = 0; k < B; ++k)
+        for (int d = 0; d < r; ++d) {
+            double acc = 0.0;
+            for (int e = 0; e < r; ++e) {
+                acc += ld(M->W_in, M->dtype, (size_t)d * 3 * r + e) * uh[(size_t)k * r + e];
+                acc += ld(M->W_in, M->dtype, (size_t)d * 3 * r + r + e) * ug[e];
+                acc += ld(M->W_in, M->dtype, (size_t)d * 3 * r + 2 * r + e) * ld(M->W_e, M->dtype, (size_t)x[k] * r + e);
+            }
+            a[(size_t)k * r + d] = acc;
+        }
+    /* Mix: c_k = a_k + sum_{j<k} L_kj a_j (per channel) */
+    for (int k = 0; k < B; ++k)
+        for (int d = 0; d < r; ++d) {
+            double acc = a[(size_t)k * r + d];
+            for (int j = 0; j < k; ++j) acc += ld(M->L, M->dtype, ((size_t)d * B + k) * B + j) * a[(size_t)j * r + d];
+            c[(size_t)k * r + d] = acc;
+        }
+    /* Trans: z = c + W_2 sigma(W_1 c) */
+    for (int k = 0; k < B; ++k) {
+        for (int d = 0; d < r; ++d) cop[(size_t)k * r + d] = opround(M, c[(size_t)k * r + d]);
+        for (int o = 0; o < R2; ++o) {
+            double acc = 0.0;
+            for (int d = 0; d < r; ++d) acc += ld(M->W1, M->dtype, (size_t)o * r + d) * cop[(size_t)k * r + d];
+            tp[(size_t)k * R2 + o] = acc;
+            uop[(size_t)k * R2 + o] = opround(M, sigma(M->act, acc));
+        }
+        for (int d = 0; d < r; ++d) {
+            double acc = 0.0;
+            for (int o = 0; o < R2; ++o) acc += ld(M->W2, M->dtype, (size_t)d * R2 + o) * uop[(size_t)k * R2 + o];
+            z[(size_t)k * r + d] = c[(size_t)k * r + d] + acc;
+            zop[(size_t)k * r + d] = opround(M, z[(size_t)k * r + d]);
+        }
+    }
+    /* Read + Correct (Eq. read / correct), the loss, and dL/dl -> W_r, z */
+    double L = 0.0;
+    for (int k = 0; k < B; ++k) {
+        for (int v = 0; v < V; ++v) {
+            double acc = 0.0;
+            for (int d = 0; d < r; ++d) acc += ld(M->W_r, M->dtype, (size_t)v * r + d) * zop[(size_t)k * r + d];
+            ell[v] = ld(s, M->dtype, (size_t)k * V + v) + acc;
+            tr[v] = ld(tgt, M->dtype, (size_t)k * V + v);
+        }
+        const double w = exp(-(double)k / gam);                    /* w_k = exp(-(k-1)/gamma), k from 1 */
+        L += w * position_loss(ell, tr, V, ystar[k], a_ce, a_l1, mult * w, g ? dl : NULL, p, q);
+        if (!g) continue;
+        for (int v = 0; v < V; ++v)
+            for (int d = 0; d < r; ++d) {
+                g->W_r[(size_t)v * r + d] += dl[v] * zop[(size_t)k * r + d];
+                dz[(size_t)k * r + d] += dl[v] * ld(M->W_r, M->dtype, (size_t)v * r + d);
+            }
+    }
+    if (g) {
+        /* Trans backward (Eq. mlp) */
+        for (int k = 0; k < B; ++k) {
+            for (int o = 0; o < R2; ++o) {
+                double acc = 0.0;
+                for (int d = 0; d < r; ++d) {
+                    acc += ld(M->W2, M->dtype, (size_t)d * R2 + o) * dz[(size_t)k * r + d];
+                    g->W2[(size_t)d * R2 + o] += dz[(size_t)k * r + d] * uop[(size_t)k * R2 + o];
+                }
+                du[o] = acc;
+                dt[o] = acc * sigma_prime(M->act, tp[(size_t)k * R2 + o]);
+            }
+            for (int d = 0; d < r; ++d) {
+                double acc = dz[(size_t)k * r + d];
+                for (int o = 0; o < R2; ++o) {
+                    acc += ld(M->W1, M->dtype, (size_t)o * r + d) * dt[o];
+                    g->W1[(size_t)o * r + d] += dt[o] * cop[(size_t)k * r + d];
+                }
+                dc[(size_t)k * r + d] = acc;
+            }
+        }
+        /* Mix backward (Eq. mix) */
+        for (int j = 0; j < B; ++j)
+            for (int d = 0; d < r; ++d) {
+                double acc = dc[(size_t)j * r + d];
+                for (int k = j + 1; k < B; ++k) {
+                    acc += ld(M->L, M->dtype, ((size_t)d * B + k) * B + j) * dc[(size_t)k * r + d];
+                    g->L[((size_t)d * B + k) * B + j] += dc[(size_t)k * r + d] * a[(size_t)j * r + d];
+                }
+                da[(size_t)j * r + d] = acc;
+            }
+        /* Fuse backward (Eq. fuse) */
+        for (int k = 0; k < B; ++k)
+            for (int e = 0; e < r; ++e) {
+                double duh = 0.0, dug_k = 0.0, de = 0.0;
+                const double xe = ld(M->W_e, M->dtype, (size_t)x[k] * r + e);
+                for (int d = 0; d < r; ++d) {
+                    const double dad = da[(size_t)k * r + d];
+                    duh += ld(M->W_in, M->dtype, (size_t)d * 3 * r + e) * dad;
+                    dug_k += ld(M->W_in, M->dtype, (size_t)d * 3 * r + r + e) * dad;
+                    de += ld(M->W_in, M->dtype, (size_t)d * 3 * r + 2 * r + e) * dad;
+                    g->W_in[(size_t)d * 3 * r + e] += dad * uh[(size_t)k * r + e];
+                    g->W_in[(size_t)d * 3 * r + r + e] += dad * ug[e];
+                    g->W_in[(size_t)d * 3 * r + 2 * r + e] += dad * xe;
+                }
+                dug[e] += dug_k;
+                g->W_e[(size_t)x[k] * r + e] += de;
+                for (int i = 0; i < H; ++i) g->W_h[(size_t)e * H + i] += duh * ld(h, M->dtype, (size_t)k * H + i);
+            }
+        for (int e = 0; e < r; ++e)
+            for (int i = 0; i < H; ++i) g->W_g[(size_t)e * H + i] += dug[e] * gm[i];
+    }
+    free(uh); free(ug); free(gm); free(a); free(c); free(cop); free(tp); free(uop); free(z); free(zop);
+    free(ell); free(tr); free(dl); free(p); free(q); free(dz); free(dc); free(da); free(du); free(dt); free(dug);
+    return L;
+}
+
+/* One training step of Sec. 4.3 on one block, T = 1:
+ *   L_total = L(p^r) + lambda L(p^b) + beta L(p^r-hat)
+ * with L(p) = sum_k w_k [a_ce (-log p_k(x*_k)) + a_l1 |p_k - p^t_k|_1],
+ * w_k = exp(-(k-1)/gamma), p^t_k = softmax(target_k):
+ *   p^r      the refiner under teacher forcing (inputs x*_{k-1}, x*_0 = anchor);
+ *   p^b      the drafter's base distribution softmax(s_k) (no refiner weight);
+ *   p^r-hat  the refiner fed the drafter's argmax(s) tokens (consistency).
+ * loss[4] = L(p^r), L(p^b), L(p^r-hat), L_total.  With g given, dL_total /
+ * dtheta of every refiner weight is added into g. */
+int xo_train_step(const xo_model *M, const void *h, const void *s, const void *tgt, const int32_t *ystar,
+                  int32_t anchor, double a_ce, double a_l1, double gam, double lambda, double beta, double *loss,
+                  double *gW_e, double *gW_h, double *gW_g, double *gW_in, double *gL, double *gW1, double *gW2,
+                  double *gW_r)
+{
+    const int B = M->B, V = M->V;
+    if (anchor < 0 || anchor >= V || gam <= 0.0) return -1;
+    for (int k = 0; k < B; ++k)
+        if (ystar[k] < 0 || ystar[k] >= V) return -1;
+    xo_grads gg = {gW_e, gW_h, gW_g, gW_in, gL, gW1, gW2, gW_r};
+    xo_grads *g = gW_r ? &gg : NULL;
+    int32_t *x = malloc(sizeof(int32_t) * B);
+    double *row = malloc(sizeof(double) * V), *tr = malloc(sizeof(double) * V);
+    double *p = malloc(sizeof(double) * V), *q = malloc(sizeof(double) * V);
+    x[0] = anchor;
+    for (int k = 1; k < B; ++k) x[k] = ystar[k - 1];
+    const double Lr = refiner_loss(M, h, s, tgt, x, ystar, a_ce, a_l1, gam, 1.0, g);
+    double Lb = 0.0;
+    for (int k = 0; k < B; ++k) {
+        for (int v = 0; v < V; ++v) {
+            row[v] = ld(s, M->dtype, (size_t)k * V + v);
+            tr[v] = ld(tgt, M->dtype, (size_t)k * V + v);
+        }
+        Lb += exp(-(double)k / gam) * position_loss(row, tr, V, ystar[k], a_ce, a_l1, 0.0, NULL, p, q);
+        if (k + 1 < B) x[k + 1] = argmax_f32(row, V, NULL);   /* the drafter's argmax(s) token */
+    }
+    const double Lc = refiner_loss(M, h, s, tgt, x, ystar, a_ce, a_l1, gam, beta, g);
+    loss[0] = Lr;
+    loss[1] = Lb;
+    loss[2] = Lc;
+    loss[3] = Lr + lambda * Lb + beta * Lc;
+    free(x); free(row); free(tr); free(p); free(q);
+    return 0;
+}
 /* ----------------------------------------------------- batched test helpers */
 
 /* Refine the same block under n different seeds (statistical pins). */
