@@ -264,6 +264,88 @@ def lm_head_line(us, nbytes, flops, hbm, tc_peak, tokens):
             "note": "s = W_lm h (bf16 out) + Y^(0) = argmax s, L2 flushed; peaks of measured"}
 
 
+def train_inputs_device(torch, cfg, dev, seed):
+    """The training workload drawn on the device with the recipe of
+    workloads.make_train_inputs (h ~ N(0, 1); s = W_lm h for a tied-size LM
+    head W_lm ~ N(0, 0.02^2), drawn through the Cholesky factor of each
+    block's B x B covariance; target = s + N(0, 1); y* drawn from
+    softmax(target) by the Gumbel-max trick; anchor uniform), in seconds
+    instead of the half minute the host draw of 2 x 78 M logits takes."""
+    g = torch.Generator(device=dev)
+    g.manual_seed(seed)
+    b, B, H, V = cfg.b, cfg.B, cfg.H, cfg.V
+    h = torch.randn((b, B, H), generator=g, device=dev).to(torch.bfloat16)
+    h64 = h.double()
+    cov = 0.02 ** 2 * (h64 @ h64.transpose(1, 2)) + 1e-12 * torch.eye(B, device=dev, dtype=torch.float64)
+    chol = torch.linalg.cholesky(cov).float()
+    s = torch.empty((b, B, V), dtype=torch.bfloat16, device=dev)
+    tgt = torch.empty_like(s)
+    ystar = torch.empty((b, B), dtype=torch.int32, device=dev)
+    for i in range(b):
+        si = chol[i] @ torch.randn((B, V), generator=g, device=dev)
+        ti = si + torch.randn((B, V), generator=g, device=dev)
+        s[i] = si.to(torch.bfloat16)
+        tgt[i] = ti.to(torch.bfloat16)
+        u = torch.rand((B, V), generator=g, device=dev, dtype=torch.float64) * (1 - 2e-12) + 1e-12
+        ystar[i] = torch.argmax(tgt[i].float() - torch.log(-torch.log(u)).float(), dim=-1).int()
+    anchor = torch.randint(0, V, (b,), generator=g, device=dev, dtype=torch.int32)
+    return dict(h=h, s=s, target=tgt, ystar=ystar, anchor=anchor)
+
+
+def train_pass_line(name, kernel, us, flops, nbytes, hbm, tc_peak):
+    """One vocabulary pass of the training step against its roofline: the
+    bf16 tensor pipe when its arithmetic intensity is at or above the ridge
+    point of the measured peaks, else HBM."""
+    tfs = flops / (us * 1e-6) / 1e12
+    gbs = nbytes / (us * 1e-6) / 1e9
+    tensor = flops / nbytes >= tc_peak * 1e3 / hbm
+    return {"pass": name, "kernel": kernel, "us": us, "flops": flops, "bytes": nbytes, "achieved_tflops": tfs,
+            "achieved_gbs": gbs, "tensor_frac": tfs / tc_peak, "hbm_frac": gbs / hbm,
+            "bound": "tensor" if tensor else "hbm", "frac": tfs / tc_peak if tensor else gbs / hbm}
+
+
+def train_measure(torch, X, W, ref, dev, timed_us, hbm, tc_peak):
+    """The refiner training step (Sec. 4.3) on the training workload: the whole
+    step and each vocabulary pass alone, CUDA events, L2 flushed before each
+    call."""
+    cfg = W.TRAIN_CONFIGS["qwen3_8b_train"]
+    d = train_inputs_device(torch, cfg, dev, 20260005)
+    b, B, V, r = cfg.b, cfg.B, cfg.V, cfg.r
+    grads = ref.alloc_grads()
+    loss = torch.empty((b, 4), dtype=torch.float32, device=dev)
+
+    def call(which=None):
+        ref.train_step(d["h"], d["s"], d["target"], d["ystar"], d["anchor"], grads=grads, loss=loss,
+                       profile_pass=which)
+
+    call()
+    torch.cuda.synchronize()
+    if ref.device_status("train", b) != X.XPRESS_OK or not bool(torch.isfinite(loss).all()):
+        raise RuntimeError("training step: device status error or non-finite loss")
+    step_us = timed_us(call)
+    P = b * B
+    NR = (P + 63) // 64 * 128
+    rows = 2 * P
+    wr, st = V * r * 2, P * V * 2
+    splits = max(1, min((ref.torch.cuda.get_device_properties(dev).multi_processor_count + NR // 256) // (NR // 128),
+                        (V + 63) // 64))
+    f1 = 2.0 * V * r * rows
+    passes = [("lse", "k_train_tok", f1, wr + st + NR * r * 2),
+              ("tv", "k_train_tok", f1, wr + 2 * st + NR * r * 2),
+              ("dz", "k_train_tok", 2 * f1, wr + 2 * st + NR * r * 2 + splits * NR * r * 4),
+              ("dW_r", "k_train_voc", 2 * f1, wr + 2 * st + NR * r * 2 + 2 * V * r * 4)]
+    lines = [train_pass_line(n, k, timed_us(lambda i=i: call(i)), f, nb, hbm, tc_peak)
+             for i, (n, k, f, nb) in enumerate(passes)]
+    launches = 14 + 11 + 4              # 14 products, 11 other kernels, 4 vocabulary passes (and 2 memsets)
+    return {"workload": cfg.name, "blocks": b, "block": B, "positions": P, "refiner_rows": rows, "hidden": cfg.H,
+            "vocab": V, "us_per_step": step_us, "positions_per_s": P / (step_us * 1e-6),
+            "launches_per_step": launches, "passes": lines,
+            "dominant": max(lines, key=lambda x: x["us"])["pass"],
+            "loss_total_mean": float(loss[:, 3].mean().item()),
+            "data": "synthetic, drawn on the device with the workload recipe",
+            "note": "L2 flushed before each call; peaks of measured; gradients added into fp32 buffers"}
+
+
 def run_xpress(args):
     import torch
     from paper_2608_02438_gb300 import binding as X
@@ -464,7 +546,7 @@ def run_xpress(args):
             raise RuntimeError("device status error (Markov head)")
         mref.close()
 
-        lm_us, lm_bytes = None, None
+        lm_us, lm_bytes, train = None, None, None
         if dt == X.XPRESS_BF16:
             # the base logits s = W_lm h of the same hidden states (Fig. 2a), with
             # Y^(0) = argmax s: a tied-size LM head W_lm ~ N(0, 0.02^2) [V, H],
@@ -487,6 +569,9 @@ def run_xpress(args):
             lm_us = timed_us(lm_call, reps=20)
             lm_bytes = cfg.V * cfg.H * 2 + b * cfg.B * cfg.H * 2 + b * cfg.B * cfg.V * 2
             del W_lm, s_lm
+            if cfg.H == 4096 and cfg.V == 151936 and cfg.B == 16:
+                hbm0, tc0, _ = peaks()
+                train = train_measure(torch, X, W, ref, dev, timed_us, hbm0, tc0)
     esz = 2 if dt == X.XPRESS_BF16 else 4
     sms = ref.torch.cuda.get_device_properties(dev).multi_processor_count
     if persistent:
@@ -537,6 +622,7 @@ def run_xpress(args):
             "lm_head": None if lm_us is None else dict(
                 lm_head_line(lm_us, lm_bytes, 2.0 * cfg.V * cfg.H * b * cfg.B, hbm, tc_peak, b * cfg.B),
                 traffic=profiled_traffic(LM_SUMMARIES.get(b * cfg.B, ""), source_hash(LM_SOURCES))),
+            "train_step": train,
             "e2e": {"value": e2e_value, "unit": "blocks/s", "h2d_bytes_per_step": int(h2d),
                     "d2h_bytes_per_step": int(d2h), "steps": n_e2e},
             "gpu_launches": per_step_launches * args.steps,

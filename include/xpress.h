@@ -226,7 +226,7 @@ int xpress_accept_noalloc(const xpress_refiner *refiner, const xpress_accept_in 
                           int32_t *out_tokens, void *stream);
 
 /* Synchronises `stream`, then reads (and clears) the device status word kept
- * in `workspace` by xpress_refine_block / xpress_accept.  *status_out is an
+ * in `workspace` by xpress_refine_block / xpress_accept / xpress_train_step.  *status_out is an
  * xpress_status (XPRESS_OK, XPRESS_ERR_TIMEOUT or XPRESS_ERR_DEVICE_CHECK). */
 int xpress_get_device_status(void *workspace, void *stream, int32_t *status_out);
 
@@ -277,6 +277,83 @@ int xpress_get_pass_count(void *workspace, void *stream, int32_t *passes_out);
 int xpress_profile_read_prepare(const xpress_refiner *refiner, void *workspace, int b, int n_tokens,
                                 void *stream);
 int xpress_profile_read(const xpress_refiner *refiner, void *workspace, int b, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Refiner training step (Sec. 4.3): the loss of one batch of b blocks and its
+ * gradient with respect to every refiner weight, at T = 1:
+ *   L_total = L(p^r) + lambda L(p^b) + beta L(p^r-hat)
+ *   L(p)    = sum_k w_k [a_ce (-log p_k(y*_k)) + a_l1 |p_k - p^t_k|_1],
+ *             w_k = exp(-(k-1)/gamma), k = 1..B, p^t_k = softmax(target_k)
+ *   p^r      the refiner's p_k = softmax(s_k + W_r z_k) under teacher forcing
+ *            (inputs x_0 = anchor, x_k = y*_k for k >= 1, 0-based)
+ *   p^b      the drafter's base distribution softmax(s_k): the drafter-anchor
+ *            term (no refiner weight enters it)
+ *   p^r-hat  the refiner fed the drafter's argmax tokens (x_k = argmax s_{k-1}):
+ *            the consistency term
+ * lambda weighs the anchor term and beta the consistency term, as in the total
+ * loss equation.  The bf16 operand roundings of the forward (c, sigma(W_1 c)
+ * and z, as in refinement) pass the gradient straight through; sgn(0) = 0 in
+ * the L1 subgradient.  u_h and u_g enter W_in as bf16 hi + lo pairs (about 16
+ * bits).  The backward products take bf16 operands (dL/dl, dL/dz, dL/dt,
+ * dL/da and the Fuse operand rounded to bf16) with fp32 accumulation.
+ * Refiner dtype XPRESS_BF16 only (UNSUPPORTED otherwise); in->B must equal the
+ * refiner's B. */
+typedef struct {
+    int b, B;
+    const void *h;           /* [b, B, H] bf16 drafter hidden states */
+    const void *s;           /* [b, B, V] bf16 drafter base logits */
+    const void *target;      /* [b, B, V] bf16 target logits of the same positions */
+    const int32_t *ystar;    /* [b, B] ground-truth tokens */
+    const int32_t *anchor;   /* [b] x_0 */
+    const int32_t *xhat;     /* [b, B] the drafter's argmax tokens, or NULL: the first
+                                argmax of each s row is computed on the device */
+    float a_ce, a_l1;        /* weights of the cross-entropy and L1 terms */
+    float gamma;             /* position-weight decay (> 0) */
+    float lambda, beta;      /* anchor and consistency weights */
+} xpress_train_in;
+
+/* Gradients are ADDED into the caller's fp32 buffers (zero them to start a
+ * step; leave them to accumulate over several batches), each shaped like its
+ * weight (xpress_weights); gL's upper triangle and diagonal are left alone.
+ * loss: [b, 4] per block L(p^r), L(p^b), L(p^r-hat), L_total (overwritten). */
+typedef struct {
+    float *loss;
+    float *gW_e, *gW_h, *gW_g, *gW_in, *gL, *gW1, *gW2, *gW_r;
+} xpress_train_out;
+
+/* Workspace of xpress_train_step for b blocks of B positions. */
+size_t xpress_train_workspace_size(const xpress_refiner *refiner, int b, int B);
+
+/* One training step on `stream` (asynchronous; about 30 kernel launches:
+ * one pass over s and target for the drafter's statistics and argmax, the
+ * forward products, four Read passes over the vocabulary -- log-sum-exp,
+ * total-variation sums, dL/dz, dL/dW_r -- and the backward products).  Token
+ * ids out of [0, V) are clamped to 0 and reported by the status word
+ * (XPRESS_ERR_DEVICE_CHECK); a bounded wait that gives up reports
+ * XPRESS_ERR_TIMEOUT there.
+ * Errors: INVALID_ARG (NULL pointer, b < 1, B mismatch, gamma <= 0),
+ * UNSUPPORTED (fp32 refiner), WORKSPACE, CUDA. */
+int xpress_train_step(const xpress_refiner *refiner, const xpress_train_in *in, const xpress_train_out *out,
+                      void *workspace, size_t ws_bytes, void *stream);
+
+/* Profiling hook (benchmarks only): after an xpress_train_step call on
+ * `workspace` with the same arguments, launches one of its four vocabulary
+ * passes alone on `stream` so that it can be timed with CUDA events:
+ * pass 0 the log-sum-exp statistics, 1 the total-variation sums, 2 dL/dz,
+ * 3 dL/dW_r (which adds into out->gW_r once more).
+ * Errors: as xpress_train_step; INVALID_ARG for another pass number. */
+int xpress_profile_train(const xpress_refiner *refiner, const xpress_train_in *in, const xpress_train_out *out,
+                         void *workspace, size_t ws_bytes, int pass, void *stream);
+
+/* Test hook (not part of the method): C (+)= A B^T for bf16 device matrices
+ * through the tensor-core product the training step uses, A [M, K] stored
+ * with rows along M (a_mn = 0) or as [K, M] (a_mn = 1), B [N, K] or [K, N]
+ * likewise, C [M, N] fp32: overwritten (accumulate = 0) or added into
+ * (accumulate = 1, the K range then split over CTAs).  Rows of an operand
+ * stored with rows along K need a multiple of 8 elements.
+ * Errors: INVALID_ARG, CUDA. */
+int xpress_debug_gemm(const void *A, int a_mn, const void *B, int b_mn, int M, int N, int K, float *C, int accumulate,
+                      void *stream);
 
 const char *xpress_status_string(int status);
 int xpress_version(void);

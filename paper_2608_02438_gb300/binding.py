@@ -50,6 +50,16 @@ class XpressAcceptIn(C.Structure):
         ("offset", C.c_uint32)]
 
 
+class XpressTrainIn(C.Structure):
+    _fields_ = [("b", C.c_int), ("B", C.c_int)] + [(n, C.c_void_p) for n in ("h", "s", "target", "ystar", "anchor",
+                                                                              "xhat")] + [
+        (n, C.c_float) for n in ("a_ce", "a_l1", "gamma", "lambda_", "beta")]
+
+
+class XpressTrainOut(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in ("loss", "gW_e", "gW_h", "gW_g", "gW_in", "gL", "gW1", "gW2", "gW_r")]
+
+
 _lib = None
 
 
@@ -95,6 +105,14 @@ def load(path: str = LIB_PATH):
     lib.xpress_lm_head.restype = I
     lib.xpress_set_wait_limit.argtypes = [P, C.c_uint64]
     lib.xpress_set_wait_limit.restype = I
+    lib.xpress_train_workspace_size.argtypes = [P, I, I]
+    lib.xpress_train_workspace_size.restype = S
+    lib.xpress_train_step.argtypes = [P, C.POINTER(XpressTrainIn), C.POINTER(XpressTrainOut), P, S, P]
+    lib.xpress_train_step.restype = I
+    lib.xpress_profile_train.argtypes = [P, C.POINTER(XpressTrainIn), C.POINTER(XpressTrainOut), P, S, I, P]
+    lib.xpress_profile_train.restype = I
+    lib.xpress_debug_gemm.argtypes = [P, I, P, I, I, I, I, P, I, P]
+    lib.xpress_debug_gemm.restype = I
     lib.xpress_profile_read_prepare.argtypes = [P, P, I, I, P]
     lib.xpress_profile_read_prepare.restype = I
     lib.xpress_profile_read.argtypes = [P, P, I, P]
@@ -200,6 +218,29 @@ def lm_head(W_lm, h, s_out=None, argmax_out=None, stream=None) -> int:
     return XPRESS_OK
 
 
+def xpress_train_workspace_size(handle, b: int, B: int) -> int:
+    return load().xpress_train_workspace_size(handle, b, B)
+
+
+def xpress_train_step(handle, tin: XpressTrainIn, tout: XpressTrainOut, ws_ptr: int, ws_bytes: int,
+                      stream: int) -> None:
+    _check("xpress_train_step", load().xpress_train_step(handle, C.byref(tin), C.byref(tout), C.c_void_p(ws_ptr),
+                                                         ws_bytes, C.c_void_p(stream)))
+
+
+def xpress_profile_train(handle, tin: XpressTrainIn, tout: XpressTrainOut, ws_ptr: int, ws_bytes: int, which: int,
+                         stream: int) -> None:
+    _check("xpress_profile_train", load().xpress_profile_train(handle, C.byref(tin), C.byref(tout),
+                                                               C.c_void_p(ws_ptr), ws_bytes, which,
+                                                               C.c_void_p(stream)))
+
+
+def xpress_debug_gemm(A_ptr: int, a_mn: int, B_ptr: int, b_mn: int, M: int, N: int, K: int, C_ptr: int,
+                      accumulate: int, stream: int) -> None:
+    _check("xpress_debug_gemm", load().xpress_debug_gemm(C.c_void_p(A_ptr), a_mn, C.c_void_p(B_ptr), b_mn, M, N, K,
+                                                         C.c_void_p(C_ptr), accumulate, C.c_void_p(stream)))
+
+
 def xpress_set_wait_limit(handle, limit_ns: int) -> None:
     _check("xpress_set_wait_limit", load().xpress_set_wait_limit(handle, limit_ns))
 
@@ -245,7 +286,11 @@ class Refiner:
     def workspace(self, kind: str, b: int):
         key = (kind, b)
         if key not in self._ws:
-            size = (xpress_refine_workspace_size if kind == "refine" else xpress_accept_workspace_size)(self.handle, b)
+            if kind == "train":
+                size = xpress_train_workspace_size(self.handle, b, self.B)
+            else:
+                size = (xpress_refine_workspace_size if kind == "refine" else xpress_accept_workspace_size)(
+                    self.handle, b)
             self._ws[key] = self.torch.empty(size + 256, dtype=self.torch.uint8, device="cuda")
         buf = self._ws[key]
         ptr = (buf.data_ptr() + 255) & ~255
@@ -298,6 +343,33 @@ class Refiner:
         xpress_accept(self.handle, acc_in, out["accept_len"].data_ptr(), out["out_tokens"].data_ptr(), ws, wsb,
                       self.stream.cuda_stream)
         return out
+
+    GRAD_NAMES = ("W_e", "W_h", "W_g", "W_in", "L", "W1", "W2", "W_r")
+
+    def alloc_grads(self) -> dict:
+        """Zeroed fp32 gradient buffers shaped like the weights."""
+        t = self.torch
+        return {n: t.zeros(self.weights[n].shape, dtype=t.float32, device="cuda") for n in self.GRAD_NAMES}
+
+    def train_step(self, h, s, target, ystar, anchor, xhat=None, a_ce=1.0, a_l1=1.0, gamma=4.0, lam=0.6, beta=0.3,
+                   grads: dict | None = None, loss=None, profile_pass: int | None = None) -> tuple:
+        """One training step (Sec. 4.3) on b blocks: returns (loss [b, 4],
+        grads); the gradients are added into `grads` (allocated zeroed when
+        None).  profile_pass (benchmarks): launch only that vocabulary pass of
+        a step already run with the same arguments."""
+        t = self.torch
+        b = h.shape[0]
+        grads = grads if grads is not None else self.alloc_grads()
+        loss = loss if loss is not None else t.empty((b, 4), dtype=t.float32, device="cuda")
+        tin = XpressTrainIn(b, self.B, h.data_ptr(), s.data_ptr(), target.data_ptr(), ystar.data_ptr(),
+                            anchor.data_ptr(), None if xhat is None else xhat.data_ptr(), a_ce, a_l1, gamma, lam, beta)
+        tout = XpressTrainOut(loss.data_ptr(), *[grads[n].data_ptr() for n in self.GRAD_NAMES])
+        ws, wsb = self.workspace("train", b)
+        if profile_pass is None:
+            xpress_train_step(self.handle, tin, tout, ws, wsb, self.stream.cuda_stream)
+        else:
+            xpress_profile_train(self.handle, tin, tout, ws, wsb, profile_pass, self.stream.cuda_stream)
+        return loss, grads
 
     def device_status(self, kind: str = "refine", b: int = 1) -> int:
         ws, _ = self.workspace(kind, b)

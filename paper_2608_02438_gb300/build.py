@@ -16,7 +16,8 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libxpress.so")
 SOURCES = ["refine_kernels.cu", "read_tc.cu", "read_tcv.cu", "refine_small.cu", "pre_tc.cu", "accept_kernels.cu", "xpress_host.cu",
-           "accept_noalloc.cu", "lm_head.cu", "trans_tc.cu"]
+           "accept_noalloc.cu", "lm_head.cu", "trans_tc.cu", "train_read.cu", "train_gemm.cu",
+           "train_kernels.cu", "train_host.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

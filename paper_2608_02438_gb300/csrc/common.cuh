@@ -450,6 +450,13 @@ __device__ __forceinline__ void fence_proxy_async_global()
     asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
+// Makes this thread's ordinary shared-memory stores visible to the async proxy
+// (a tcgen05.mma that reads the tile as an operand).
+__device__ __forceinline__ void fence_proxy_async_smem()
+{
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 // Programmatic dependent launch: wait for the preceding kernel of the stream
 // (no-op when launched without the attribute) / let the next one start.
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
@@ -679,6 +686,31 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr)
 __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N)
 {
     return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+// Same, with A (bit 15) and / or B (bit 16) given MN-major.
+__host__ __device__ constexpr uint32_t idesc_bf16_mn(int M, int N, bool a_mn, bool b_mn)
+{
+    return idesc_bf16(M, N) | (a_mn ? 1u << 15 : 0u) | (b_mn ? 1u << 16 : 0u);
+}
+
+// Shared-memory matrix descriptor for an MN-major operand stored with the
+// 128-byte swizzle: each 128-byte row holds 64 consecutive M (or N) elements
+// of one K index, 8 consecutive K rows form a 1024-byte swizzle atom, atoms
+// along K are 1024 bytes apart (stride offset) and the next 64 elements along
+// M / N start `mn_stride` bytes further (leading offset).  This is the layout
+// a TMA box of 64 elements (inner) x rows (outer) leaves with SWIZZLE_128B when
+// the rows run along K; advancing K by 16 moves the start by 2048 bytes.
+__device__ __forceinline__ uint64_t smem_desc_sw128_mn(uint32_t saddr, uint32_t mn_stride)
+{
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)((mn_stride >> 4) & 0x3FFFu) << 16) |
+           ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+// Packs two floats as bf16 (round to nearest even): lo in bits 0-15.
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
+{
+    return (uint32_t)f2bf(lo) | ((uint32_t)f2bf(hi) << 16);
 }
 
 }  // namespace xp

@@ -101,10 +101,133 @@ inline int mix_mlp_smem(int dtype)
 }
 constexpr int GEMV_SMEM = 128 * 1024;
 
+// ------------------------------------------------------------ training step
+// Per paired row of the training step (Sec. 4.3): row 128 j + f 64 + l is
+// position 64 j + l under the teacher-forced (f = 0) or the consistency (f = 1)
+// inputs.  dl = p (A0 + A1 sgn(p - q)) - A2 [v = y] with p, q the row's and
+// its position's target softmax; zero coefficients on padding rows.
+struct alignas(16) RowCoef {
+    float lse_p2, lse_q2;   // log2-domain log-sum-exp of the row's logits and of the target row
+    float A0, A1, A2;
+    int y;                  // ground-truth token of the position (-1 on padding rows)
+    float pad[2];
+};
+
+constexpr int TR_STATS = 0, TR_TV = 1, TR_DZ = 2;
+
+struct TrainParams {
+    int P, NR, V, B;        // positions, paired rows (multiple of 128), vocabulary, block
+    int nvt, splits;        // 64-id vocabulary tiles, splits of them (k_train_tok grid.x)
+    const int32_t *ystar;   // [P]
+    float4 *part;           // [splits][NR] per-row partials of the statistics passes
+    float *dzp;             // [splits][NR][r] dL/dz of each vocabulary split
+    float *ly;              // [NR] l at y*
+    const float *lse_p2;    // [NR]
+    const float *lse_q2;    // [P]
+    const float *lse_s2;    // [P]
+    const RowCoef *coef;    // [NR]
+    float *gW_r;            // [V][r] dL/dW_r, added into
+    const void *W_r;
+    int32_t *status;
+    unsigned long long wait_ns;
+};
+
+// train_read.cu
+__global__ void k_train_tok(const __grid_constant__ TrainParams p, const __grid_constant__ CUtensorMap tmap_z,
+                            const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_s,
+                            const __grid_constant__ CUtensorMap tmap_t, int mode);
+__global__ void k_train_voc(const __grid_constant__ TrainParams p, const __grid_constant__ CUtensorMap tmap_z,
+                            const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_s,
+                            const __grid_constant__ CUtensorMap tmap_t);
+extern const size_t kTrainTokSmemBytes, kTrainVocSmemBytes;
+extern const int kTrainTokThreads, kTrainVocThreads;
+
+// train_gemm.cu: C (+)= alpha A B^T on tcgen05, A [M, K] and B [N, K] bf16 given
+// K-major (rows along M / N) or MN-major (rows along K)
+constexpr int GM_STORE = 0, GM_ADD = 1, GM_ACT = 2, GM_RESID = 3, GM_PART = 4;
+struct GemmArgs {
+    int M, N, K;
+    int a_mn, b_mn;         // 1: the operand's rows run along K
+    int kchunks;            // 64-wide K chunks per grid.z slice
+    int mode;               // GM_STORE: C = alpha D; GM_ADD: C += alpha D (atomic);
+                            // GM_ACT: C = D, Cb = bf16(sigma(D)); GM_RESID: x = R + D, C = x, Cb = bf16(x);
+                            // GM_PART: slice z of C (C + z M ldc) = alpha D of K split z (summed later
+                            // in a fixed order, so that the result is reproducible)
+    int act;
+    float alpha;
+    float *C;
+    int ldc;
+    uint16_t *Cb;
+    int ldcb;
+    const float *R;
+    int ldr;
+};
+__global__ void k_gemm(const __grid_constant__ GemmArgs g, const __grid_constant__ CUtensorMap ta,
+                       const __grid_constant__ CUtensorMap tb);
+extern const size_t kGemmSmemBytes;
+
+// train_kernels.cu
+struct TrainMisc {
+    int b, B, P, NR, V, H, act;
+    const void *h, *s, *t;                  // [P, H], [P, V], [P, V] bf16
+    const int32_t *ystar, *anchor, *xhat_in;
+    const uint16_t *W_e, *L;
+    float a_ce, a_l1, gamma, lambda, beta;
+    int nch;                                // vocabulary chunks of k_train_rows
+    float4 *rpart;                          // [P][nch] max / log2-sum of s and of t
+    unsigned long long *rkey;               // [P][nch] argmax key of s
+    float *lse_s2, *lse_q2, *s_y;           // [P]
+    int32_t *xhat;                          // [P] first argmax of s rows
+    int32_t *xrow;                          // [NR] input token of each paired row
+    const float *Uh, *Ug;                   // [usplits][P, r] W_h h_k, W_g h_k per K split
+    int usplits;
+    uint16_t *X;                            // [NR, 3r] bf16 [u_h | u_g | W_e x]
+    uint16_t *Xlo;                          // [NR, 2r] bf16 [u_h - bf16(u_h) | u_g - bf16(u_g)]
+    const float *a;                         // [NR, r]
+    float *c;                               // [NR, r]
+    uint16_t *cop;                          // [NR, r] bf16(c)
+    const float4 *part;                     // [splits][NR]
+    int splits;
+    float *ly, *lse_p2;                     // [NR]
+    RowCoef *coef;                          // [NR]
+    float *loss;                            // [b, 4]
+    const float *dzp;                       // [splits][NR, r] per vocabulary split
+    float *dz;                              // [NR, r]
+    uint16_t *dzb;                          // [NR, r]
+    const float *du, *tpre;                 // [NR, 2r] dL/du, W_1 c
+    uint16_t *dtb;                          // [NR, 2r]
+    const float *dc;                        // [NR, r]
+    uint16_t *dab;                          // [NR, r]
+    float *gL, *gW_e;
+    const float *dX;                        // [NR, 3r]
+    uint16_t *D;                            // [P, 2r] bf16 [dL/du_h | dL/du_g / B]
+    int32_t *status;
+};
+__global__ void k_train_rows(TrainMisc m);
+__global__ void k_train_rows_fin(TrainMisc m);
+__global__ void k_train_fuse(TrainMisc m);
+__global__ void k_train_mix(TrainMisc m);
+__global__ void k_train_stats_fin(TrainMisc m);
+__global__ void k_train_tv_fin(TrainMisc m);
+__global__ void k_train_dz(TrainMisc m);
+__global__ void k_train_dact(TrainMisc m);
+__global__ void k_train_mix_bwd(TrainMisc m);
+__global__ void k_train_gL(TrainMisc m);
+__global__ void k_train_fuse_bwd(TrainMisc m);
+constexpr int TRAIN_ROW_CHUNK = 8192;       // vocabulary ids per k_train_rows CTA
+
 // acceptance launch shared by xpress_accept and xpress_accept_noalloc
 // (xpress_host.cu); `ws` holds the scratch laid out by accept_scratch_bytes
 size_t accept_scratch_bytes(const xpress_refiner *R, int b);
 int refiner_device(const xpress_refiner *R);   // the device the refiner was created on
+const xpress_weights &refiner_weights(const xpress_refiner *R);
+int refiner_sms(const xpress_refiner *R);
+unsigned long long refiner_wait_ns(const xpress_refiner *R);
+const CUtensorMap *refiner_tmap_wr128(const xpress_refiner *R);   // W_r, boxes of 128 rows x 64
+// 2-D bf16 tensor [outer][inner] with a row pitch of `pitch` elements,
+// 128-byte swizzle, zero fill out of bounds
+bool tmap_bf16(CUtensorMap *m, const void *base, uint64_t inner, uint64_t outer, uint64_t pitch, uint32_t box_inner,
+               uint32_t box_outer);
 int accept_launch(const xpress_refiner *R, const xpress_accept_in *in, int32_t *accept_len, int32_t *out_tokens,
                   void *ws, size_t ws_bytes, void *stream);
 constexpr int READ_SIMT_DYN_SMEM = (32 * (RANK + 1) + 8 * 32 * 33) * 4;

@@ -1,0 +1,390 @@
+// train_kernels.cu -- the memory-bound and per-block steps of the refiner
+// training step (Sec. 4.3) around the tensor-core products:
+//
+//   k_train_rows / _fin   one pass over s and the target logits t of every
+//                         position: log-sum-exp of both (log2 domain), s at
+//                         y*, and the first argmax of s (the consistency
+//                         forward's inputs, argmax p^b)
+//   k_train_fuse          the Fuse operand [u_h | u_g | W_e[x]] of both
+//                         forwards (Eq. fuse; u_g = W_g g with g the block
+//                         mean of h, taken as the mean of W_g h_j), u_h and
+//                         u_g as bf16 hi + lo pairs so that W_in sees them to
+//                         about 16 bits
+//   k_train_mix           c_k = a_k + sum_{j<k} L_kj a_j per channel (Eq. mix)
+//   k_train_stats_fin     lse of every row's logits from the split partials
+//   k_train_tv_fin        per block the three losses and L_total; per row the
+//                         coefficients of dL/dl
+//   k_train_dz, _dact     dL/dz from the vocabulary splits and its bf16 copy;
+//                         dL/dt = dL/du sigma'(t)
+//   k_train_mix_bwd, _gL  dL/da_j = dc_j + sum_{k>j} L_kj dc_k; dL/dL_kj
+//   k_train_fuse_bwd      dL/du_h per position (both forwards), dL/du_g / B
+//                         per block, dL/dW_e rows (atomic, both forwards)
+#include "common.cuh"
+#include "kernels.h"
+
+namespace xp {
+
+namespace {
+
+constexpr float L2E = 1.4426950408889634f;
+constexpr float LN2 = 0.69314718055994531f;
+
+__device__ __forceinline__ int pair_row(int i, int f) { return (i >> 6) * 128 + f * 64 + (i & 63); }
+
+__device__ __forceinline__ void lse2_merge(float &m, float &s, float om, float os)
+{
+    const float M = fmaxf(m, om);
+    if (M == -INFINITY) return;
+    s = s * ex2_approx(m - M) + os * ex2_approx(om - M);
+    m = M;
+}
+
+__device__ __forceinline__ float sigma_prime(int act, float t)
+{
+    if (act == 2) return t > 0.0f ? 1.0f : 0.0f;
+    if (act == 1)
+        return 0.5f * (1.0f + erff(t * 0.70710678118654752f)) + t * 0.39894228040143268f * expf(-0.5f * t * t);
+    const float sg = 1.0f / (1.0f + expf(-t));
+    return sg + t * sg * (1.0f - sg);
+}
+
+}  // namespace
+
+// grid (nch, P), 256 threads: ids [ch 8192 + 32 tid, +32) of position blockIdx.y.
+__global__ void __launch_bounds__(256) k_train_rows(TrainMisc m)
+{
+    const int ch = blockIdx.x, i = blockIdx.y, tid = threadIdx.x;
+    const int v0 = ch * TRAIN_ROW_CHUNK + tid * 32;
+    const uint16_t *srow = static_cast<const uint16_t *>(m.s) + (size_t)i * m.V;
+    const uint16_t *trow = static_cast<const uint16_t *>(m.t) + (size_t)i * m.V;
+    float xs[32], xt[32];
+    if (v0 + 32 <= m.V) {
+        const uint4 *sp = reinterpret_cast<const uint4 *>(srow + v0), *tp = reinterpret_cast<const uint4 *>(trow + v0);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const uint4 a = __ldcs(sp + c), b = __ldcs(tp + c);
+            const uint32_t wa[4] = {a.x, a.y, a.z, a.w}, wb[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                xs[8 * c + 2 * q] = __uint_as_float(wa[q] << 16);
+                xs[8 * c + 2 * q + 1] = __uint_as_float(wa[q] & 0xFFFF0000u);
+                xt[8 * c + 2 * q] = __uint_as_float(wb[q] << 16);
+                xt[8 * c + 2 * q + 1] = __uint_as_float(wb[q] & 0xFFFF0000u);
+            }
+        }
+    } else {
+#pragma unroll
+        for (int jj = 0; jj < 32; ++jj) {
+            const bool in = v0 + jj < m.V;
+            xs[jj] = in ? bf2f(srow[v0 + jj]) : -INFINITY;
+            xt[jj] = in ? bf2f(trow[v0 + jj]) : -INFINITY;
+        }
+    }
+    float best = -INFINITY, ms = -INFINITY, mt = -INFINITY;
+    int idx = 0x7fffffff;
+#pragma unroll
+    for (int jj = 0; jj < 32; ++jj) {
+        if (xs[jj] > best) { best = xs[jj]; idx = v0 + jj; }
+        ms = fmaxf(ms, xs[jj]);
+        mt = fmaxf(mt, xt[jj]);
+    }
+    float ss = 0.f, st = 0.f;
+    ms *= L2E;
+    mt *= L2E;
+    if (ms != -INFINITY) {
+#pragma unroll
+        for (int jj = 0; jj < 32; ++jj) {
+            ss += ex2_approx(fmaf(xs[jj], L2E, -ms));
+            st += ex2_approx(fmaf(xt[jj], L2E, -mt));
+        }
+    }
+    // warp, then block
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float oms = __shfl_xor_sync(0xffffffffu, ms, o), oss = __shfl_xor_sync(0xffffffffu, ss, o);
+        const float omt = __shfl_xor_sync(0xffffffffu, mt, o), ost = __shfl_xor_sync(0xffffffffu, st, o);
+        const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+        const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
+        lse2_merge(ms, ss, oms, oss);
+        lse2_merge(mt, st, omt, ost);
+        merge_argmax(best, idx, ob, oi);
+    }
+    __shared__ float4 wp[8];
+    __shared__ float wb[8];
+    __shared__ int wi[8];
+    const int w = tid >> 5;
+    if ((tid & 31) == 0) {
+        wp[w] = make_float4(ms, ss, mt, st);
+        wb[w] = best;
+        wi[w] = idx;
+    }
+    __syncthreads();
+    if (tid == 0) {
+        float4 a = wp[0];
+        float b = wb[0];
+        int bi = wi[0];
+        for (int k = 1; k < 8; ++k) {
+            lse2_merge(a.x, a.y, wp[k].x, wp[k].y);
+            lse2_merge(a.z, a.w, wp[k].z, wp[k].w);
+            merge_argmax(b, bi, wb[k], wi[k]);
+        }
+        m.rpart[(size_t)i * m.nch + ch] = a;
+        m.rkey[(size_t)i * m.nch + ch] = argmax_key(b, bi);
+    }
+}
+
+// grid ceil(P / 8), 256 threads: one warp per position.
+__global__ void __launch_bounds__(256) k_train_rows_fin(TrainMisc m)
+{
+    const int i = blockIdx.x * 8 + threadIdx.x / 32, lane = threadIdx.x % 32;
+    if (i >= m.P) return;
+    float ms = -INFINITY, ss = 0.f, mt = -INFINITY, st = 0.f;
+    unsigned long long key = 0;
+    for (int c = lane; c < m.nch; c += 32) {
+        const float4 a = m.rpart[(size_t)i * m.nch + c];
+        lse2_merge(ms, ss, a.x, a.y);
+        lse2_merge(mt, st, a.z, a.w);
+        key = max(key, m.rkey[(size_t)i * m.nch + c]);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        lse2_merge(ms, ss, __shfl_xor_sync(0xffffffffu, ms, o), __shfl_xor_sync(0xffffffffu, ss, o));
+        lse2_merge(mt, st, __shfl_xor_sync(0xffffffffu, mt, o), __shfl_xor_sync(0xffffffffu, st, o));
+        key = max(key, __shfl_xor_sync(0xffffffffu, key, o));
+    }
+    if (lane == 0) {
+        m.lse_s2[i] = ms + log2f(ss);
+        m.lse_q2[i] = mt + log2f(st);
+        int y = m.ystar[i];
+        if (y < 0 || y >= m.V) {
+            set_status(m.status, ST_BOUNDS);
+            y = 0;
+        }
+        m.s_y[i] = bf2f(static_cast<const uint16_t *>(m.s)[(size_t)i * m.V + y]);
+        if (m.xhat_in) {
+            m.xhat[i] = m.xhat_in[i];
+        } else {
+            float b;
+            int bi;
+            argmax_unkey(key, b, bi);
+            m.xhat[i] = bi;
+        }
+    }
+}
+
+// grid NR / 2 (every position slot of the row tiles), r threads.
+__global__ void __launch_bounds__(RANK) k_train_fuse(TrainMisc m)
+{
+    const int i = blockIdx.x, d = threadIdx.x;
+    const int r3 = 3 * RANK;
+    if (i >= m.P) {
+        // padding rows: zero operands and activations so that every product
+        // over them vanishes
+        for (int f = 0; f < 2; ++f) {
+            const int row = pair_row(i, f);
+            m.X[(size_t)row * r3 + d] = 0;
+            m.X[(size_t)row * r3 + RANK + d] = 0;
+            m.X[(size_t)row * r3 + 2 * RANK + d] = 0;
+            m.Xlo[(size_t)row * 2 * RANK + d] = 0;
+            m.Xlo[(size_t)row * 2 * RANK + RANK + d] = 0;
+            m.c[(size_t)row * RANK + d] = 0.f;
+            m.cop[(size_t)row * RANK + d] = 0;
+            m.dab[(size_t)row * RANK + d] = 0;
+            if (d == 0) m.xrow[row] = -1;
+        }
+        return;
+    }
+    const int blk = i / m.B, k = i % m.B;
+    // the K-split slices of W_h h and W_g h, summed in a fixed order
+    const size_t slice = (size_t)m.P * RANK;
+    float uhv = 0.f, ug = 0.f;
+    for (int sp = 0; sp < m.usplits; ++sp) uhv += m.Uh[sp * slice + (size_t)i * RANK + d];
+    for (int j = 0; j < m.B; ++j) {
+        float uj = 0.f;
+        for (int sp = 0; sp < m.usplits; ++sp) uj += m.Ug[sp * slice + (size_t)(blk * m.B + j) * RANK + d];
+        ug += uj;
+    }
+    ug /= (float)m.B;
+    const uint16_t uh = f2bf(uhv), ugb = f2bf(ug);
+    const uint16_t uhl = f2bf(uhv - bf2f(uh)), ugl = f2bf(ug - bf2f(ugb));
+    for (int f = 0; f < 2; ++f) {
+        const int row = pair_row(i, f);
+        int x = k == 0 ? m.anchor[blk] : (f == 0 ? m.ystar[i - 1] : m.xhat[i - 1]);
+        if (x < 0 || x >= m.V) {
+            if (d == 0) set_status(m.status, ST_BOUNDS);
+            x = 0;
+        }
+        m.X[(size_t)row * r3 + d] = uh;
+        m.X[(size_t)row * r3 + RANK + d] = ugb;
+        m.X[(size_t)row * r3 + 2 * RANK + d] = m.W_e[(size_t)x * RANK + d];
+        m.Xlo[(size_t)row * 2 * RANK + d] = uhl;
+        m.Xlo[(size_t)row * 2 * RANK + RANK + d] = ugl;
+        if (d == 0) m.xrow[row] = x;
+    }
+}
+
+// grid (b, 2), r threads: block blockIdx.x, forward blockIdx.y, channel d.
+__global__ void __launch_bounds__(RANK) k_train_mix(TrainMisc m)
+{
+    const int blk = blockIdx.x, f = blockIdx.y, d = threadIdx.x, B = m.B;
+    float av[MAX_B];
+    for (int k = 0; k < B; ++k) {
+        const int row = pair_row(blk * B + k, f);
+        const float ak = m.a[(size_t)row * RANK + d];
+        float acc = ak;
+        const uint16_t *lr = m.L + ((size_t)d * B + k) * B;
+        for (int j = 0; j < k; ++j) acc = fmaf(bf2f(lr[j]), av[j], acc);
+        av[k] = ak;
+        m.c[(size_t)row * RANK + d] = acc;
+        m.cop[(size_t)row * RANK + d] = f2bf(acc);
+    }
+}
+
+// grid ceil(NR / 256), 256 threads: one row each.
+__global__ void __launch_bounds__(256) k_train_stats_fin(TrainMisc m)
+{
+    const int row = blockIdx.x * 256 + threadIdx.x;
+    if (row >= m.NR) return;
+    const int i = (row >> 7) * 64 + (row & 63);
+    if (i >= m.P) {
+        m.lse_p2[row] = 0.f;
+        return;
+    }
+    float mx = -INFINITY, s = 0.f;
+    for (int sv = 0; sv < m.splits; ++sv) {
+        const float4 a = m.part[(size_t)sv * m.NR + row];
+        lse2_merge(mx, s, a.x, a.y);
+    }
+    m.lse_p2[row] = mx + log2f(s);
+}
+
+// grid b, 32 threads: lane k = position k of block blockIdx.x.
+__global__ void __launch_bounds__(32) k_train_tv_fin(TrainMisc m)
+{
+    const int blk = blockIdx.x, k = threadIdx.x;
+    float lr = 0.f, lb = 0.f, lc = 0.f;
+    if (k < m.B) {
+        const int i = blk * m.B + k;
+        const float w = expf(-(float)k / m.gamma);
+        float anc = 0.f;
+        float lf[2];
+        for (int f = 0; f < 2; ++f) {
+            const int row = pair_row(i, f);
+            float sm = 0.f, lt = 0.f, eq = 0.f;
+            for (int sv = 0; sv < m.splits; ++sv) {
+                const float4 a = m.part[(size_t)sv * m.NR + row];
+                sm += a.x;
+                lt += a.y;
+                eq += a.z;
+                anc += a.w;
+            }
+            const float l1 = 2.0f * (1.0f - sm);
+            const float S = 1.0f - 2.0f * lt - eq;          // sum_v sgn(p_v - q_v) p_v
+            const float ce = m.lse_p2[row] * LN2 - m.ly[row];
+            lf[f] = w * (m.a_ce * ce + m.a_l1 * l1);
+            const float cf = w * (f == 0 ? 1.0f : m.beta);
+            RowCoef rc;
+            rc.lse_p2 = m.lse_p2[row];
+            rc.lse_q2 = m.lse_q2[i];
+            rc.A0 = cf * (m.a_ce - m.a_l1 * S);
+            rc.A1 = cf * m.a_l1;
+            rc.A2 = cf * m.a_ce;
+            rc.y = m.ystar[i];
+            rc.pad[0] = rc.pad[1] = 0.f;
+            m.coef[row] = rc;
+        }
+        lr = lf[0];
+        lc = lf[1];
+        const float ceb = m.lse_s2[i] * LN2 - m.s_y[i];
+        lb = w * (m.a_ce * ceb + m.a_l1 * 2.0f * (1.0f - anc));
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        lr += __shfl_xor_sync(0xffffffffu, lr, o);
+        lb += __shfl_xor_sync(0xffffffffu, lb, o);
+        lc += __shfl_xor_sync(0xffffffffu, lc, o);
+    }
+    if (k == 0) {
+        m.loss[blk * 4 + 0] = lr;
+        m.loss[blk * 4 + 1] = lb;
+        m.loss[blk * 4 + 2] = lc;
+        m.loss[blk * 4 + 3] = lr + m.lambda * lb + m.beta * lc;
+    }
+}
+
+// grid ceil(NR r / 1024), 256 threads, 4 elements each: dL/dz as the sum of
+// the vocabulary splits' slices in a fixed order, and its bf16 copy.
+__global__ void __launch_bounds__(256) k_train_dz(TrainMisc m)
+{
+    const size_t e = ((size_t)blockIdx.x * 256 + threadIdx.x) * 4;
+    const size_t n = (size_t)m.NR * RANK;
+    if (e >= n) return;
+    float4 v = *reinterpret_cast<const float4 *>(m.dzp + e);
+    for (int sp = 1; sp < m.splits; ++sp) {
+        const float4 o = *reinterpret_cast<const float4 *>(m.dzp + sp * n + e);
+        v.x += o.x;
+        v.y += o.y;
+        v.z += o.z;
+        v.w += o.w;
+    }
+    *reinterpret_cast<float4 *>(m.dz + e) = v;
+    *reinterpret_cast<uint2 *>(m.dzb + e) = make_uint2(pack_bf16x2(v.x, v.y), pack_bf16x2(v.z, v.w));
+}
+
+// grid ceil(NR 2r / 1024), 256 threads: dL/dt = dL/du sigma'(t), 4 elements each.
+__global__ void __launch_bounds__(256) k_train_dact(TrainMisc m)
+{
+    const size_t e = ((size_t)blockIdx.x * 256 + threadIdx.x) * 4;
+    if (e >= (size_t)m.NR * 2 * RANK) return;
+    const float4 du = *reinterpret_cast<const float4 *>(m.du + e);
+    const float4 t = *reinterpret_cast<const float4 *>(m.tpre + e);
+    *reinterpret_cast<uint2 *>(m.dtb + e) =
+        make_uint2(pack_bf16x2(du.x * sigma_prime(m.act, t.x), du.y * sigma_prime(m.act, t.y)),
+                   pack_bf16x2(du.z * sigma_prime(m.act, t.z), du.w * sigma_prime(m.act, t.w)));
+}
+
+// grid (b, 2), r threads.
+__global__ void __launch_bounds__(RANK) k_train_mix_bwd(TrainMisc m)
+{
+    const int blk = blockIdx.x, f = blockIdx.y, d = threadIdx.x, B = m.B;
+    float dcv[MAX_B];
+    for (int k = 0; k < B; ++k) dcv[k] = m.dc[(size_t)pair_row(blk * B + k, f) * RANK + d];
+    for (int j = 0; j < B; ++j) {
+        float acc = dcv[j];
+        for (int k = j + 1; k < B; ++k) acc = fmaf(bf2f(m.L[((size_t)d * B + k) * B + j]), dcv[k], acc);
+        m.dab[(size_t)pair_row(blk * B + j, f) * RANK + d] = f2bf(acc);
+    }
+}
+
+// grid B * B ((k, j) = (blockIdx.x / B, blockIdx.x % B), only j < k), r threads:
+// dL/dL_kj^(d) = sum over blocks and both forwards of dc_k^(d) a_j^(d).
+__global__ void __launch_bounds__(RANK) k_train_gL(TrainMisc m)
+{
+    const int k = blockIdx.x / m.B, j = blockIdx.x % m.B, d = threadIdx.x;
+    if (j >= k) return;
+    float acc = 0.f;
+    for (int blk = 0; blk < m.b; ++blk)
+        for (int f = 0; f < 2; ++f)
+            acc = fmaf(m.dc[(size_t)pair_row(blk * m.B + k, f) * RANK + d],
+                       m.a[(size_t)pair_row(blk * m.B + j, f) * RANK + d], acc);
+    m.gL[((size_t)d * m.B + k) * m.B + j] += acc;
+}
+
+// grid P, r threads.
+__global__ void __launch_bounds__(RANK) k_train_fuse_bwd(TrainMisc m)
+{
+    const int i = blockIdx.x, d = threadIdx.x, r3 = 3 * RANK;
+    const int blk = i / m.B;
+    const int rt = pair_row(i, 0), rc = pair_row(i, 1);
+    m.D[(size_t)i * 2 * RANK + d] = f2bf(m.dX[(size_t)rt * r3 + d] + m.dX[(size_t)rc * r3 + d]);
+    float dug = 0.f;
+    for (int jj = 0; jj < m.B; ++jj) {
+        const int p = blk * m.B + jj;
+        dug += m.dX[(size_t)pair_row(p, 0) * r3 + RANK + d] + m.dX[(size_t)pair_row(p, 1) * r3 + RANK + d];
+    }
+    m.D[(size_t)i * 2 * RANK + RANK + d] = f2bf(dug / (float)m.B);
+    atomicAdd(m.gW_e + (size_t)m.xrow[rt] * RANK + d, m.dX[(size_t)rt * r3 + 2 * RANK + d]);
+    atomicAdd(m.gW_e + (size_t)m.xrow[rc] * RANK + d, m.dX[(size_t)rc * r3 + 2 * RANK + d]);
+}
+
+}  // namespace xp

@@ -939,6 +939,24 @@ AcceptLayout accept_layout(const xpress_refiner *R, int b)
 namespace xp {
 
 int refiner_device(const xpress_refiner *R) { return R ? R->device : -1; }
+const xpress_weights &refiner_weights(const xpress_refiner *R) { return R->w; }
+int refiner_sms(const xpress_refiner *R) { return R->num_sms; }
+unsigned long long refiner_wait_ns(const xpress_refiner *R) { return R->wait_ns; }
+const CUtensorMap *refiner_tmap_wr128(const xpress_refiner *R) { return &R->tmap_wr128; }
+
+bool tmap_bf16(CUtensorMap *m, const void *base, uint64_t inner, uint64_t outer, uint64_t pitch, uint32_t box_inner,
+               uint32_t box_outer)
+{
+    auto enc = tensor_map_encoder();
+    if (!enc) return false;
+    cuuint64_t dims[2] = {inner, outer};
+    cuuint64_t strides[1] = {pitch * 2};
+    cuuint32_t box[2] = {box_inner, box_outer};
+    cuuint32_t es[2] = {1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
 
 size_t accept_scratch_bytes(const xpress_refiner *R, int b)
 {

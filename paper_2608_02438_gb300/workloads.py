@@ -188,6 +188,41 @@ def make_inputs(cfg: Config, b: int | None = None, seed_offset: int = 0) -> dict
                 seed=seeds.astype(np.uint64), offset=int(7 + seed_offset), consistent=consistent)
 
 
+# The training workload of Sec. 4.3 (a batch of blocks with target logits and
+# ground-truth tokens); the paper gives no batch size, 32 blocks of 16 is the
+# serving batch of the refinement benchmark.
+TRAIN_CONFIGS = {
+    "qwen3_8b_train": Config("qwen3_8b_train", b=32, B=16, H=4096, V=151936, r=256, dtype=BF16, K_max=16,
+                             seed=20260005, notes="training batch 32 x block 16, Qwen3-8B shape, bf16"),
+}
+
+
+def make_train_inputs(cfg: Config, b: int | None = None, seed_offset: int = 0) -> dict:
+    """Inputs of one training step for ``b`` blocks (default cfg.b): h [b,B,H]
+    and s [b,B,V] as in make_inputs (cfg.logits recipe), target logits of the
+    same positions [b,B,V] = s + N(0, 1) (a target that mostly agrees with the
+    drafter), ground-truth tokens y* [b,B] drawn from softmax(target) (the
+    target model's own samples), anchor [b]."""
+    b = cfg.b if b is None else b
+    rng = np.random.Generator(np.random.PCG64(cfg.seed + 7919 * seed_offset + 3))
+    B, H, V = cfg.B, cfg.H, cfg.V
+    h = _normal(rng, (b, B, H), 1.0)
+    h_st = to_storage(h, cfg.dtype)
+    h32 = to_f32(h_st, cfg.dtype)
+    s = np.empty((b, B, V), np.float32)
+    if cfg.logits == "lm_head":
+        for i in range(b):
+            s[i] = _lm_head_logits(rng, h32[i], V)
+    else:
+        s[:] = _normal(rng, (b, B, V), 4.0)
+    tgt = s + _normal(rng, (b, B, V), 1.0)
+    s_st = to_storage(s, cfg.dtype)
+    tgt_st = to_storage(tgt, cfg.dtype)
+    ystar = _gumbel_sample(rng, to_f32(tgt_st, cfg.dtype))
+    anchor = rng.integers(0, V, size=b).astype(np.int32)
+    return dict(h=h_st, s=s_st, target=tgt_st, ystar=ystar, anchor=anchor)
+
+
 def markov_head_weights(weights: dict) -> dict:
     """The Markov-head comparison head (Sec. 2, Sec. 5 Table 3) in the
     refiner's notation: the correction for position k depends only on the id
