@@ -50,6 +50,7 @@ SMALL_SUMMARY = "profiles/k_refine_small_qwen3_8b_greedy.txt"
 READ_SOURCES = [CSRC + "read_tc.cu", CSRC + "common.cuh"]
 READ_SUMMARIES = {"long_b64": "profiles/k_read_tc_long_b64.txt"}
 LM_SOURCES = [CSRC + "lm_head.cu", CSRC + "common.cuh"]
+TRAIN_SOURCES = [CSRC + f for f in ("train_read.cu", "kernels.h", "common.cuh")]
 LM_SUMMARIES = {16: "profiles/k_lm_head32_qwen3_8b_n16.txt"}
 
 
@@ -275,9 +276,9 @@ def train_inputs_device(torch, cfg, dev, seed):
     g.manual_seed(seed)
     b, B, H, V = cfg.b, cfg.B, cfg.H, cfg.V
     h = torch.randn((b, B, H), generator=g, device=dev).to(torch.bfloat16)
-    h64 = h.double()
-    cov = 0.02 ** 2 * (h64 @ h64.transpose(1, 2)) + 1e-12 * torch.eye(B, device=dev, dtype=torch.float64)
-    chol = torch.linalg.cholesky(cov).float()
+    h64 = h.double().cpu().numpy()              # the B x B factors on the host (numpy)
+    cov = 0.02 ** 2 * (h64 @ h64.transpose(0, 2, 1)) + 1e-12 * np.eye(B)
+    chol = torch.from_numpy(np.linalg.cholesky(cov).astype(np.float32)).to(dev)
     s = torch.empty((b, B, V), dtype=torch.bfloat16, device=dev)
     tgt = torch.empty_like(s)
     ystar = torch.empty((b, B), dtype=torch.int32, device=dev)
@@ -304,12 +305,12 @@ def train_pass_line(name, kernel, us, flops, nbytes, hbm, tc_peak):
             "bound": "tensor" if tensor else "hbm", "frac": tfs / tc_peak if tensor else gbs / hbm}
 
 
-def train_measure(torch, X, W, ref, dev, timed_us, hbm, tc_peak):
+def train_measure(torch, X, W, ref, dev, timed_us, hbm, tc_peak, d=None, cfg=None):
     """The refiner training step (Sec. 4.3) on the training workload: the whole
     step and each vocabulary pass alone, CUDA events, L2 flushed before each
     call."""
-    cfg = W.TRAIN_CONFIGS["qwen3_8b_train"]
-    d = train_inputs_device(torch, cfg, dev, 20260005)
+    cfg = cfg or W.TRAIN_CONFIGS["qwen3_8b_train"]
+    d = d or train_inputs_device(torch, cfg, dev, cfg.seed)
     b, B, V, r = cfg.b, cfg.B, cfg.V, cfg.r
     grads = ref.alloc_grads()
     loss = torch.empty((b, 4), dtype=torch.float32, device=dev)
@@ -336,7 +337,7 @@ def train_measure(torch, X, W, ref, dev, timed_us, hbm, tc_peak):
               ("dW_r", "k_train_voc", 2 * f1, wr + 2 * st + NR * r * 2 + 2 * V * r * 4)]
     lines = [train_pass_line(n, k, timed_us(lambda i=i: call(i)), f, nb, hbm, tc_peak)
              for i, (n, k, f, nb) in enumerate(passes)]
-    launches = 14 + 11 + 4              # 14 products, 11 other kernels, 4 vocabulary passes (and 2 memsets)
+    launches = 14 + 10 + 4              # 14 products, 10 other kernels, 4 vocabulary passes (and 3 memsets)
     return {"workload": cfg.name, "blocks": b, "block": B, "positions": P, "refiner_rows": rows, "hidden": cfg.H,
             "vocab": V, "us_per_step": step_us, "positions_per_s": P / (step_us * 1e-6),
             "launches_per_step": launches, "passes": lines,
@@ -648,6 +649,86 @@ def run_xpress(args):
     return 0
 
 
+def run_train(args):
+    """--config qwen3_8b_train: the refiner training step (Sec. 4.3) alone,
+    K timed steps after W warm-up steps, L2 flushed between steps, one JSON
+    line (training positions/s); the launch list and kernel captures of the
+    training kernels are taken on this command."""
+    import torch
+    from paper_2608_02438_gb300 import binding as X
+    from paper_2608_02438_gb300 import build as BLD
+    from paper_2608_02438_gb300 import workloads as W
+
+    rank, world, local = dist_env()
+    if world > 1:
+        print(json.dumps({"impl": "xpress", "unavailable": "the training line runs on one GPU"}))
+        return 0
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    BLD.build()
+    cfg = W.TRAIN_CONFIGS[args.config]
+    w = W.make_weights(cfg.H, cfg.V, cfg.r, cfg.B, cfg.dtype, cfg.seed, "paper")
+    ref = X.Refiner({k: X.to_device(v, X.XPRESS_BF16) for k, v in w.items()}, cfg.H, cfg.V, cfg.r, cfg.B,
+                    X.XPRESS_BF16)
+    stream = ref.stream
+    flush = torch.empty(512 * 2 ** 20, dtype=torch.uint8, device=dev)
+    hbm, tc_peak, src = peaks()
+
+    def timed_us(call, reps=12):
+        fs = [torch.cuda.Event(enable_timing=True) for _ in range(reps)]
+        fe = [torch.cuda.Event(enable_timing=True) for _ in range(reps)]
+        for i in range(reps):
+            flush.zero_()
+            fs[i].record(stream)
+            call()
+            fe[i].record(stream)
+        torch.cuda.synchronize()
+        return 1000.0 * float(np.mean([s.elapsed_time(e) for s, e in zip(fs[2:], fe[2:])]))
+
+    with torch.cuda.stream(stream):
+        d = train_inputs_device(torch, cfg, dev, cfg.seed)
+        grads = ref.alloc_grads()
+        loss = torch.empty((cfg.b, 4), dtype=torch.float32, device=dev)
+
+        def step():
+            ref.train_step(d["h"], d["s"], d["target"], d["ystar"], d["anchor"], grads=grads, loss=loss)
+
+        for _ in range(max(3, args.warmup)):
+            step()
+        torch.cuda.synchronize()
+        if ref.device_status("train", cfg.b) != X.XPRESS_OK:
+            raise RuntimeError("device status error")
+        st = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        en = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        with ClockSampler(dev.index) as clk:
+            for i in range(args.steps):
+                flush.zero_()
+                st[i].record(stream)
+                step()
+                en[i].record(stream)
+            torch.cuda.synchronize()
+        ms = float(sum(s.elapsed_time(e) for s, e in zip(st, en)))
+        tr = train_measure(torch, X, W, ref, dev, timed_us, hbm, tc_peak, d=d, cfg=cfg)
+    P = cfg.b * cfg.B
+    dom = max(tr["passes"], key=lambda x: x["us"])
+    line = {"metric": "refiner training positions/s (Qwen3-8B shape, block 16)", "value": P * args.steps / (ms / 1e3),
+            "unit": "positions/s", "n_gpus": 1, "steps": args.steps, "warmup": max(3, args.warmup),
+            "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": cfg.name, "blocks": cfg.b, "block": cfg.B, "hidden": cfg.H, "vocab": cfg.V,
+                       "rank": cfg.r, "l2": "flushed between steps (512 MB write)"},
+            "gpu_launches": tr["launches_per_step"] * args.steps,
+            "roofline": {"bound": dom["bound"], "kernel": dom["kernel"], "pass": dom["pass"],
+                         "achieved": dom["achieved_tflops"] if dom["bound"] == "tensor" else dom["achieved_gbs"],
+                         "peak": tc_peak if dom["bound"] == "tensor" else hbm,
+                         "unit": "TFLOP/s" if dom["bound"] == "tensor" else "GB/s", "frac": dom["frac"],
+                         "traffic": None, "peak_source": src, "source_hash": source_hash(TRAIN_SOURCES)},
+            "train_step": tr, "clocks": clk.summary()}
+    print(json.dumps(line), flush=True)
+    ref.close()
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -658,6 +739,9 @@ def main():
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    from paper_2608_02438_gb300 import workloads as W
+    if args.config in W.TRAIN_CONFIGS:
+        return run_train(args)
     return run_xpress(args)
 
 

@@ -104,13 +104,14 @@ constexpr int GEMV_SMEM = 128 * 1024;
 // ------------------------------------------------------------ training step
 // Per paired row of the training step (Sec. 4.3): row 128 j + f 64 + l is
 // position 64 j + l under the teacher-forced (f = 0) or the consistency (f = 1)
-// inputs.  dl = p (A0 + A1 sgn(p - q)) - A2 [v = y] with p, q the row's and
-// its position's target softmax; zero coefficients on padding rows.
+// inputs.  dL/dl_v = p_v A(sgn(p_v - q_v)) - A2 [v = y*] with p, q the row's
+// and its position's target softmax, A(+1) = Apos, A(-1) = Aneg,
+// A(0) = (Apos + Aneg) / 2; the vocabulary passes apply the first term, the
+// -A2 [v = y*] term is applied to dz and dW_r by k_train_dz.  Zero on padding
+// rows.
 struct alignas(16) RowCoef {
     float lse_p2, lse_q2;   // log2-domain log-sum-exp of the row's logits and of the target row
-    float A0, A1, A2;
-    int y;                  // ground-truth token of the position (-1 on padding rows)
-    float pad[2];
+    float Apos, Aneg;
 };
 
 constexpr int TR_STATS = 0, TR_TV = 1, TR_DZ = 2;
@@ -128,6 +129,7 @@ struct TrainParams {
     const RowCoef *coef;    // [NR]
     float *gW_r;            // [V][r] dL/dW_r, added into
     const void *W_r;
+    const uint16_t *zop;    // [NR][r] the W_r operand z of every row (bf16)
     int32_t *status;
     unsigned long long wait_ns;
 };
@@ -190,6 +192,9 @@ struct TrainMisc {
     int splits;
     float *ly, *lse_p2;                     // [NR]
     RowCoef *coef;                          // [NR]
+    float *A2;                              // [NR] coefficient of the -[v = y*] term
+    const uint16_t *W_r, *zop;              // [V, r], [NR, r]
+    float *gW_r;
     float *loss;                            // [b, 4]
     const float *dzp;                       // [splits][NR, r] per vocabulary split
     float *dz;                              // [NR, r]
@@ -212,7 +217,7 @@ __global__ void k_train_tv_fin(TrainMisc m);
 __global__ void k_train_dz(TrainMisc m);
 __global__ void k_train_dact(TrainMisc m);
 __global__ void k_train_mix_bwd(TrainMisc m);
-__global__ void k_train_gL(TrainMisc m);
+size_t train_mix_smem(int B);               // dynamic shared memory of k_train_mix / _mix_bwd
 __global__ void k_train_fuse_bwd(TrainMisc m);
 constexpr int TRAIN_ROW_CHUNK = 8192;       // vocabulary ids per k_train_rows CTA
 

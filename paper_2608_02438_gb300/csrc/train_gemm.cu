@@ -61,6 +61,12 @@ __global__ void __launch_bounds__(192, 1)
         fence_barrier_init();
     }
     if (warp == 1) { tmem_alloc(&sh.tmem_base, G_BN); tmem_relinquish(); }
+    if (threadIdx.x == 0) {
+        tma_prefetch_desc(&ta);
+        tma_prefetch_desc(&tb);
+    }
+    pdl_trigger();                 // the next kernel may start its set-up
+    pdl_wait();                    // the operands of this product are complete
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -69,13 +75,11 @@ __global__ void __launch_bounds__(192, 1)
 
     if (warp == 0) {
         if (lane == 0 && nc > 0) {
-            tma_prefetch_desc(&ta);
-            tma_prefetch_desc(&tb);
             uint32_t pending = 0, pend_par = 0;
             for (int c = 0; c < nc; ++c) {
                 const int st = c % G_STAGES;
                 const uint32_t ph = (uint32_t)((c / G_STAGES) & 1);
-                if (!mbar_wait(&sh.empty[st], ph ^ 1, abort)) break;
+                if (!mbar_wait_spin(&sh.empty[st], ph ^ 1, abort)) break;
                 uint8_t *sa = base + st * G_STAGE, *sb = sa + G_A_STAGE;
                 const int k = (kc0 + c) * G_BK;
                 mbar_expect_tx(&sh.full[st], G_STAGE);
@@ -93,7 +97,7 @@ __global__ void __launch_bounds__(192, 1)
             if (*abort) {
                 int dummy = 0;
                 for (int st = 0; st < G_STAGES; ++st)
-                    if (pending & (1u << st)) mbar_wait(&sh.full[st], (pend_par >> st) & 1, &dummy, 100000000ull);
+                    if (pending & (1u << st)) mbar_wait_spin(&sh.full[st], (pend_par >> st) & 1, &dummy, 100000000ull);
             }
         }
     } else if (warp == 1) {
@@ -101,7 +105,7 @@ __global__ void __launch_bounds__(192, 1)
             bool ok = true;
             for (int c = 0; c < nc && ok; ++c) {
                 const int st = c % G_STAGES;
-                if (!mbar_wait(&sh.full[st], (uint32_t)((c / G_STAGES) & 1), abort)) { ok = false; break; }
+                if (!mbar_wait_spin(&sh.full[st], (uint32_t)((c / G_STAGES) & 1), abort)) { ok = false; break; }
                 tc_fence_after();
                 const uint32_t a0 = smem_u32(base + st * G_STAGE), b0 = a0 + G_A_STAGE;
 #pragma unroll
@@ -119,7 +123,7 @@ __global__ void __launch_bounds__(192, 1)
     } else if (nc > 0) {
         const int q = warp & 3;
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
-        if (mbar_wait(&sh.tfull, 0, abort)) {
+        if (mbar_wait_spin(&sh.tfull, 0, abort)) {
             tc_fence_after();
             const int m = m0 + q * 32 + lane;
             const bool valid = m < g.M && !*abort;

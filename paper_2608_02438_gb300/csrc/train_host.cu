@@ -27,9 +27,28 @@ namespace {
 
 size_t a256(size_t x) { return (x + 255) & ~size_t(255); }
 
+// Launch with programmatic stream serialization: the kernel may start its
+// set-up while its predecessor finishes (every training kernel waits with
+// griddepcontrol.wait before it touches memory).
+template <typename... KArgs, typename... Args>
+cudaError_t launch(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, Args... args)
+{
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 struct TrainLayout {
     int P = 0, NR = 0, nch = 0, nvt = 0, splits = 1, usplits = 1;
-    size_t rpart, rkey, lse_s2, lse_q2, s_y, xhat, xrow, Uh, Ug, X, Xlo, a, c, cop, t, uop, zop, part, ly, lse_p2, coef,
+    size_t rpart, rkey, lse_s2, lse_q2, s_y, xhat, xrow, Uh, Ug, X, Xlo, a, c, cop, t, uop, zop, part, ly, lse_p2, coef, A2,
         dzp, dz, dzb, du, dtb, dc, dab, dX, D, total;
 };
 
@@ -81,6 +100,7 @@ TrainLayout train_layout(const xpress_refiner *R, int b, int B)
     L.ly = take(NR * 4);
     L.lse_p2 = take(NR * 4);
     L.coef = take(NR * sizeof(RowCoef));
+    L.A2 = take(NR * 4);
     L.dzp = take((size_t)L.splits * NR * r * 4);
     L.dz = take(NR * r * 4);
     L.dzb = take(NR * r * 2);
@@ -105,7 +125,11 @@ int train_attributes()
             cudaFuncSetAttribute(k_train_voc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kTrainVocSmemBytes) !=
                 cudaSuccess ||
             cudaFuncSetAttribute(k_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmemBytes) !=
-                cudaSuccess) {
+                cudaSuccess ||
+            cudaFuncSetAttribute(k_train_mix, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)train_mix_smem(MAX_B)) !=
+                cudaSuccess ||
+            cudaFuncSetAttribute(k_train_mix_bwd, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)train_mix_smem(MAX_B)) != cudaSuccess) {
             (void)cudaGetLastError();
             rc = XPRESS_ERR_CUDA;
         }
@@ -151,8 +175,7 @@ int gemm(cudaStream_t st, int sms, int M, int N, int K, Operand A, Operand B, in
     const int splits = (mode == GM_ADD || mode == GM_PART) ? gemm_splits(sms, M, N, K) : 1;
     g.kchunks = (nk + splits - 1) / splits;
     const dim3 grid((M + 127) / 128, (N + 63) / 64, splits);
-    k_gemm<<<grid, 192, kGemmSmemBytes, st>>>(g, ta, tb);
-    XT_CUDA(cudaGetLastError());
+    XT_CUDA(launch(k_gemm, grid, dim3(192), kGemmSmemBytes, st, g, ta, tb));
     return XPRESS_OK;
 }
 
@@ -237,6 +260,10 @@ int train_run(const xpress_refiner *R, const xpress_train_in *in, const xpress_t
     m.ly = F(L.ly);
     m.lse_p2 = F(L.lse_p2);
     m.coef = reinterpret_cast<RowCoef *>(W + L.coef);
+    m.A2 = F(L.A2);
+    m.W_r = static_cast<const uint16_t *>(w.W_r);
+    m.zop = U(L.zop);
+    m.gW_r = out->gW_r;
     m.loss = out->loss;
     m.dzp = F(L.dzp);
     m.dz = F(L.dz);
@@ -269,6 +296,7 @@ int train_run(const xpress_refiner *R, const xpress_train_in *in, const xpress_t
     tp.dzp = F(L.dzp);
     tp.gW_r = out->gW_r;
     tp.W_r = w.W_r;
+    tp.zop = U(L.zop);
     tp.status = m.status;
     tp.wait_ns = refiner_wait_ns(R);
 
@@ -283,22 +311,22 @@ int train_run(const xpress_refiner *R, const xpress_train_in *in, const xpress_t
     const int nvt128 = (V + 127) / 128;
     if (only >= 0) {
         if (only == 0 || only == 1 || only == 2)
-            k_train_tok<<<gtok, kTrainTokThreads, kTrainTokSmemBytes, st>>>(tp, tz128, tw64, ts64, tt64, only);
+            XT_CUDA(launch(k_train_tok, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128, tw64, ts64,
+                           tt64, only));
         else
-            k_train_voc<<<nvt128 < sms ? nvt128 : sms, kTrainVocThreads, kTrainVocSmemBytes, st>>>(
-                tp, tz32, *refiner_tmap_wr128(R), ts32, tt32);
-        XT_CUDA(cudaGetLastError());
+            XT_CUDA(launch(k_train_voc, dim3(nvt128 < sms ? nvt128 : sms), dim3(kTrainVocThreads), kTrainVocSmemBytes,
+                           st, tp, tz32, *refiner_tmap_wr128(R), ts32, tt32));
         return XPRESS_OK;
     }
 
     // the status word and the padding rows' coefficients
     XT_CUDA(cudaMemsetAsync(W, 0, 4, st));
     XT_CUDA(cudaMemsetAsync(W + L.coef, 0, (size_t)NR * sizeof(RowCoef), st));
+    XT_CUDA(cudaMemsetAsync(W + L.A2, 0, (size_t)NR * 4, st));
 
     // the drafter's rows: lse of s and of the target, s at y*, argmax s
-    k_train_rows<<<dim3(L.nch, P), 256, 0, st>>>(m);
-    k_train_rows_fin<<<(P + 7) / 8, 256, 0, st>>>(m);
-    XT_CUDA(cudaGetLastError());
+    XT_CUDA(launch(k_train_rows, dim3(L.nch, P), dim3(256), 0, st, m));
+    XT_CUDA(launch(k_train_rows_fin, dim3((P + 7) / 8), dim3(256), 0, st, m));
 
     // forward: Fuse, Mix, Trans of both input sequences
     int rc;
@@ -309,8 +337,7 @@ int train_run(const xpress_refiner *R, const xpress_train_in *in, const xpress_t
     if ((rc = gemm(st, sms, P, r, H, h_k, {w.W_g, (uint64_t)H, false}, GM_PART, 1.f, F(L.Ug), r, nullptr, 0, nullptr,
                    0, 0)))
         return rc;
-    k_train_fuse<<<NR / 2, RANK, 0, st>>>(m);
-    XT_CUDA(cudaGetLastError());
+    XT_CUDA(launch(k_train_fuse, dim3(4 * in->b + NR / 2 - P), dim3(RANK), 0, st, m));
     if ((rc = gemm(st, sms, NR, r, 3 * r, {U(L.X), (uint64_t)3 * r, false}, {w.W_in, (uint64_t)3 * r, false}, GM_STORE,
                    1.f, F(L.a), r, nullptr, 0, nullptr, 0, 0)))
         return rc;
@@ -318,8 +345,8 @@ int train_run(const xpress_refiner *R, const xpress_train_in *in, const xpress_t
     if ((rc = gemm(st, sms, NR, r, 2 * r, {U(L.Xlo), (uint64_t)2 * r, false}, {w.W_in, (uint64_t)3 * r, false},
                    GM_RESID, 1.f, F(L.a), r, nullptr, 0, F(L.a), r, 0)))
         return rc;
-    k_train_mix<<<dim3(in->b, 2), RANK, 0, st>>>(m);
-    XT_CUDA(cudaGetLastError());
+    const dim3 gmix(RANK / 32, in->b), bmix(32, in->B);     // 2 sequences (both forwards of a block) per CTA
+    XT_CUDA(launch(k_train_mix, gmix, bmix, train_mix_smem(in->B), st, m));
     if ((rc = gemm(st, sms, NR, 2 * r, r, {U(L.cop), (uint64_t)r, false}, {w.W1, (uint64_t)r, false}, GM_ACT, 1.f,
                    F(L.t), 2 * r, U(L.uop), 2 * r, nullptr, 0, w.act)))
         return rc;
@@ -328,23 +355,24 @@ int train_run(const xpress_refiner *R, const xpress_train_in *in, const xpress_t
         return rc;
 
     // the Read passes
-    k_train_tok<<<gtok, kTrainTokThreads, kTrainTokSmemBytes, st>>>(tp, tz128, tw64, ts64, tt64, TR_STATS);
-    k_train_stats_fin<<<(NR + 255) / 256, 256, 0, st>>>(m);
-    k_train_tok<<<gtok, kTrainTokThreads, kTrainTokSmemBytes, st>>>(tp, tz128, tw64, ts64, tt64, TR_TV);
-    k_train_tv_fin<<<in->b, 32, 0, st>>>(m);
-    k_train_tok<<<gtok, kTrainTokThreads, kTrainTokSmemBytes, st>>>(tp, tz128, tw64, ts64, tt64, TR_DZ);
-    k_train_voc<<<nvt128 < sms ? nvt128 : sms, kTrainVocThreads, kTrainVocSmemBytes, st>>>(
-        tp, tz32, *refiner_tmap_wr128(R), ts32, tt32);
-    XT_CUDA(cudaGetLastError());
+    const dim3 gvoc(nvt128 < sms ? nvt128 : sms);
+    XT_CUDA(launch(k_train_tok, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128, tw64, ts64, tt64,
+                   (int)TR_STATS));
+    XT_CUDA(launch(k_train_stats_fin, dim3(NR / 8), dim3(256), 0, st, m));
+    XT_CUDA(launch(k_train_tok, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128, tw64, ts64, tt64,
+                   (int)TR_TV));
+    XT_CUDA(launch(k_train_tv_fin, dim3(in->b), dim3(32), 0, st, m));
+    XT_CUDA(launch(k_train_tok, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128, tw64, ts64, tt64,
+                   (int)TR_DZ));
+    XT_CUDA(launch(k_train_voc, gvoc, dim3(kTrainVocThreads), kTrainVocSmemBytes, st, tp, tz32,
+                   *refiner_tmap_wr128(R), ts32, tt32));
 
     // backward through Trans (Eq. mlp)
-    k_train_dz<<<(NR * r / 4 + 255) / 256, 256, 0, st>>>(m);
-    XT_CUDA(cudaGetLastError());
+    XT_CUDA(launch(k_train_dz, dim3((NR * r / 4 + 255) / 256), dim3(256), 0, st, m));
     if ((rc = gemm(st, sms, NR, 2 * r, r, {U(L.dzb), (uint64_t)r, false}, {w.W2, (uint64_t)2 * r, true}, GM_STORE, 1.f,
                    F(L.du), 2 * r, nullptr, 0, nullptr, 0, 0)))
         return rc;
-    k_train_dact<<<(NR * 2 * r / 4 + 255) / 256, 256, 0, st>>>(m);
-    XT_CUDA(cudaGetLastError());
+    XT_CUDA(launch(k_train_dact, dim3((NR * 2 * r / 4 + 255) / 256), dim3(256), 0, st, m));
     if ((rc = gemm(st, sms, NR, r, 2 * r, {U(L.dtb), (uint64_t)2 * r, false}, {w.W1, (uint64_t)r, true}, GM_RESID, 1.f,
                    F(L.dc), r, nullptr, 0, F(L.dz), r, 0)))
         return rc;
@@ -356,17 +384,14 @@ int train_run(const xpress_refiner *R, const xpress_train_in *in, const xpress_t
         return rc;
 
     // backward through Mix (Eq. mix) and Fuse (Eq. fuse)
-    k_train_mix_bwd<<<dim3(in->b, 2), RANK, 0, st>>>(m);
-    k_train_gL<<<in->B * in->B, RANK, 0, st>>>(m);
-    XT_CUDA(cudaGetLastError());
+    XT_CUDA(launch(k_train_mix_bwd, gmix, bmix, train_mix_smem(in->B), st, m));
     if ((rc = gemm(st, sms, NR, 3 * r, r, {U(L.dab), (uint64_t)r, false}, {w.W_in, (uint64_t)3 * r, true}, GM_STORE,
                    1.f, F(L.dX), 3 * r, nullptr, 0, nullptr, 0, 0)))
         return rc;
     if ((rc = gemm(st, sms, r, 3 * r, NR, {U(L.dab), (uint64_t)r, true}, {U(L.X), (uint64_t)3 * r, true}, GM_ADD, 1.f,
                    out->gW_in, 3 * r, nullptr, 0, nullptr, 0, 0)))
         return rc;
-    k_train_fuse_bwd<<<P, RANK, 0, st>>>(m);
-    XT_CUDA(cudaGetLastError());
+    XT_CUDA(launch(k_train_fuse_bwd, dim3(P), dim3(RANK), 0, st, m));
     if ((rc = gemm(st, sms, r, H, P, {U(L.D), (uint64_t)2 * r, true}, h_mn, GM_ADD, 1.f, out->gW_h, H, nullptr, 0,
                    nullptr, 0, 0)))
         return rc;

@@ -1,5 +1,7 @@
 // train_kernels.cu -- the memory-bound and per-block steps of the refiner
-// training step (Sec. 4.3) around the tensor-core products:
+// training step (Sec. 4.3) around the tensor-core products.  Every kernel of
+// the step is launched with programmatic dependent launch: it signals its
+// successor at once and waits for its predecessor before touching memory.
 //
 //   k_train_rows / _fin   one pass over s and the target logits t of every
 //                         position: log-sum-exp of both (log2 domain), s at
@@ -10,13 +12,14 @@
 //                         mean of h, taken as the mean of W_g h_j), u_h and
 //                         u_g as bf16 hi + lo pairs so that W_in sees them to
 //                         about 16 bits
-//   k_train_mix           c_k = a_k + sum_{j<k} L_kj a_j per channel (Eq. mix)
+//   k_train_mix           c_k = a_k + sum_{j<k} L_kj a_j per channel (Eq. mix),
+//                         L staged in shared memory per 32 channels
 //   k_train_stats_fin     lse of every row's logits from the split partials
 //   k_train_tv_fin        per block the three losses and L_total; per row the
 //                         coefficients of dL/dl
 //   k_train_dz, _dact     dL/dz from the vocabulary splits and its bf16 copy;
 //                         dL/dt = dL/du sigma'(t)
-//   k_train_mix_bwd, _gL  dL/da_j = dc_j + sum_{k>j} L_kj dc_k; dL/dL_kj
+//   k_train_mix_bwd       dL/da_j = dc_j + sum_{k>j} L_kj dc_k and dL/dL_kj
 //   k_train_fuse_bwd      dL/du_h per position (both forwards), dL/du_g / B
 //                         per block, dL/dW_e rows (atomic, both forwards)
 #include "common.cuh"
@@ -53,6 +56,8 @@ __device__ __forceinline__ float sigma_prime(int act, float t)
 // grid (nch, P), 256 threads: ids [ch 8192 + 32 tid, +32) of position blockIdx.y.
 __global__ void __launch_bounds__(256) k_train_rows(TrainMisc m)
 {
+    pdl_trigger();
+    pdl_wait();
     const int ch = blockIdx.x, i = blockIdx.y, tid = threadIdx.x;
     const int v0 = ch * TRAIN_ROW_CHUNK + tid * 32;
     const uint16_t *srow = static_cast<const uint16_t *>(m.s) + (size_t)i * m.V;
@@ -136,6 +141,8 @@ __global__ void __launch_bounds__(256) k_train_rows(TrainMisc m)
 // grid ceil(P / 8), 256 threads: one warp per position.
 __global__ void __launch_bounds__(256) k_train_rows_fin(TrainMisc m)
 {
+    pdl_trigger();
+    pdl_wait();
     const int i = blockIdx.x * 8 + threadIdx.x / 32, lane = threadIdx.x % 32;
     if (i >= m.P) return;
     float ms = -INFINITY, ss = 0.f, mt = -INFINITY, st = 0.f;
@@ -172,14 +179,18 @@ __global__ void __launch_bounds__(256) k_train_rows_fin(TrainMisc m)
     }
 }
 
-// grid NR / 2 (every position slot of the row tiles), r threads.
+// grid b * 4 + (NR / 2 - P), r threads: CTA 4 blk + k4 (< 4 b) builds the
+// rows of positions k4, k4 + 4, ... of block blk (u_g of the block summed by
+// each of its four CTAs), the others zero one padding position each.
 __global__ void __launch_bounds__(RANK) k_train_fuse(TrainMisc m)
 {
-    const int i = blockIdx.x, d = threadIdx.x;
-    const int r3 = 3 * RANK;
-    if (i >= m.P) {
+    pdl_trigger();
+    pdl_wait();
+    const int d = threadIdx.x, r3 = 3 * RANK;
+    if ((int)blockIdx.x >= 4 * m.b) {
         // padding rows: zero operands and activations so that every product
         // over them vanishes
+        const int i = m.P + (int)blockIdx.x - 4 * m.b;
         for (int f = 0; f < 2; ++f) {
             const int row = pair_row(i, f);
             m.X[(size_t)row * r3 + d] = 0;
@@ -194,73 +205,169 @@ __global__ void __launch_bounds__(RANK) k_train_fuse(TrainMisc m)
         }
         return;
     }
-    const int blk = i / m.B, k = i % m.B;
+    const int blk = blockIdx.x >> 2, k4 = blockIdx.x & 3, B = m.B;
     // the K-split slices of W_h h and W_g h, summed in a fixed order
     const size_t slice = (size_t)m.P * RANK;
-    float uhv = 0.f, ug = 0.f;
-    for (int sp = 0; sp < m.usplits; ++sp) uhv += m.Uh[sp * slice + (size_t)i * RANK + d];
-    for (int j = 0; j < m.B; ++j) {
+    float ug = 0.f;
+    for (int j = 0; j < B; ++j) {
         float uj = 0.f;
-        for (int sp = 0; sp < m.usplits; ++sp) uj += m.Ug[sp * slice + (size_t)(blk * m.B + j) * RANK + d];
+        for (int sp = 0; sp < m.usplits; ++sp) uj += m.Ug[sp * slice + (size_t)(blk * B + j) * RANK + d];
         ug += uj;
     }
-    ug /= (float)m.B;
-    const uint16_t uh = f2bf(uhv), ugb = f2bf(ug);
-    const uint16_t uhl = f2bf(uhv - bf2f(uh)), ugl = f2bf(ug - bf2f(ugb));
-    for (int f = 0; f < 2; ++f) {
-        const int row = pair_row(i, f);
-        int x = k == 0 ? m.anchor[blk] : (f == 0 ? m.ystar[i - 1] : m.xhat[i - 1]);
-        if (x < 0 || x >= m.V) {
-            if (d == 0) set_status(m.status, ST_BOUNDS);
-            x = 0;
+    ug /= (float)B;
+    const uint16_t ugb = f2bf(ug), ugl = f2bf(ug - bf2f(ugb));
+    for (int k = k4; k < B; k += 4) {
+        const int i = blk * B + k;
+        float uhv = 0.f;
+        for (int sp = 0; sp < m.usplits; ++sp) uhv += m.Uh[sp * slice + (size_t)i * RANK + d];
+        const uint16_t uh = f2bf(uhv), uhl = f2bf(uhv - bf2f(uh));
+        for (int f = 0; f < 2; ++f) {
+            const int row = pair_row(i, f);
+            int x = k == 0 ? m.anchor[blk] : (f == 0 ? m.ystar[i - 1] : m.xhat[i - 1]);
+            if (x < 0 || x >= m.V) {
+                if (d == 0) set_status(m.status, ST_BOUNDS);
+                x = 0;
+            }
+            m.X[(size_t)row * r3 + d] = uh;
+            m.X[(size_t)row * r3 + RANK + d] = ugb;
+            m.X[(size_t)row * r3 + 2 * RANK + d] = m.W_e[(size_t)x * RANK + d];
+            m.Xlo[(size_t)row * 2 * RANK + d] = uhl;
+            m.Xlo[(size_t)row * 2 * RANK + RANK + d] = ugl;
+            if (d == 0) m.xrow[row] = x;
         }
-        m.X[(size_t)row * r3 + d] = uh;
-        m.X[(size_t)row * r3 + RANK + d] = ugb;
-        m.X[(size_t)row * r3 + 2 * RANK + d] = m.W_e[(size_t)x * RANK + d];
-        m.Xlo[(size_t)row * 2 * RANK + d] = uhl;
-        m.Xlo[(size_t)row * 2 * RANK + RANK + d] = ugl;
-        if (d == 0) m.xrow[row] = x;
     }
 }
 
-// grid (b, 2), r threads: block blockIdx.x, forward blockIdx.y, channel d.
-__global__ void __launch_bounds__(RANK) k_train_mix(TrainMisc m)
+namespace {
+
+// The causal mixer of 32 channels, staged as Ls[(k B + j) 32 + d] (fp32,
+// channel innermost); only j < k is read.
+__device__ __forceinline__ void stage_L(const TrainMisc &m, float *Ls, int d0)
 {
-    const int blk = blockIdx.x, f = blockIdx.y, d = threadIdx.x, B = m.B;
-    float av[MAX_B];
-    for (int k = 0; k < B; ++k) {
+    const int B = m.B, n = 32 * B * B;
+    for (int e = threadIdx.y * 32 + threadIdx.x; e < n; e += 32 * B) {
+        const int dl = e / (B * B), kj = e % (B * B);
+        Ls[kj * 32 + dl] = bf2f(m.L[(size_t)(d0 + dl) * B * B + kj]);
+    }
+}
+
+constexpr int MIX_SEQ = 2;        // sequences (block, forward) per CTA
+
+inline size_t mix_smem(int B) { return (size_t)(32 * B * B + 2 * B * 32) * 4; }
+
+}  // namespace
+
+size_t train_mix_smem(int B) { return mix_smem(B); }
+
+// grid (r / 32, ceil(2 b / MIX_SEQ)), block (32, B): channel d0 + x, position y
+// of the sequences 2 blk + f of the CTA's group: c_k = a_k + sum_{j<k} L_kj a_j.
+__global__ void __launch_bounds__(1024) k_train_mix(TrainMisc m)
+{
+    pdl_trigger();
+    extern __shared__ float smf[];
+    const int B = m.B, dl = threadIdx.x, k = threadIdx.y, d0 = blockIdx.x * 32, d = d0 + dl;
+    float *Ls = smf, *sa = smf + 32 * B * B;
+    stage_L(m, Ls, d0);
+    pdl_wait();
+    for (int q = 0; q < MIX_SEQ; ++q) {
+        const int sq = blockIdx.y * MIX_SEQ + q;
+        if (sq >= 2 * m.b) break;
+        const int blk = sq >> 1, f = sq & 1;
         const int row = pair_row(blk * B + k, f);
         const float ak = m.a[(size_t)row * RANK + d];
+        __syncthreads();                           // Ls staged; the previous sequence's sa read
+        sa[k * 32 + dl] = ak;
+        __syncthreads();
         float acc = ak;
-        const uint16_t *lr = m.L + ((size_t)d * B + k) * B;
-        for (int j = 0; j < k; ++j) acc = fmaf(bf2f(lr[j]), av[j], acc);
-        av[k] = ak;
+        for (int j = 0; j < k; ++j) acc = fmaf(Ls[(k * B + j) * 32 + dl], sa[j * 32 + dl], acc);
         m.c[(size_t)row * RANK + d] = acc;
         m.cop[(size_t)row * RANK + d] = f2bf(acc);
     }
 }
 
-// grid ceil(NR / 256), 256 threads: one row each.
+// Same grid: dL/da_j = dc_j + sum_{k>j} L_kj dc_k, and this group's share of
+// dL/dL_kj = sum over sequences of dc_k a_j (added atomically into gL).
+__global__ void __launch_bounds__(1024) k_train_mix_bwd(TrainMisc m)
+{
+    pdl_trigger();
+    extern __shared__ float smf[];
+    const int B = m.B, dl = threadIdx.x, j = threadIdx.y, d0 = blockIdx.x * 32, d = d0 + dl;
+    float *Ls = smf, *sdc = smf + 32 * B * B, *sa = sdc + B * 32;
+    stage_L(m, Ls, d0);
+    pdl_wait();
+    float gl[MAX_B];                               // thread (d, k = j) holds dL/dL_kj' for j' < k
+    for (int jj = 0; jj < MAX_B; ++jj) gl[jj] = 0.f;
+    for (int q = 0; q < MIX_SEQ; ++q) {
+        const int sq = blockIdx.y * MIX_SEQ + q;
+        if (sq >= 2 * m.b) break;
+        const int blk = sq >> 1, f = sq & 1;
+        const int row = pair_row(blk * B + j, f);
+        const float dcj = m.dc[(size_t)row * RANK + d];
+        const float aj = m.a[(size_t)row * RANK + d];
+        __syncthreads();
+        sdc[j * 32 + dl] = dcj;
+        sa[j * 32 + dl] = aj;
+        __syncthreads();
+        float acc = dcj;
+        for (int k = j + 1; k < B; ++k) acc = fmaf(Ls[(k * B + j) * 32 + dl], sdc[k * 32 + dl], acc);
+        m.dab[(size_t)row * RANK + d] = f2bf(acc);
+#pragma unroll
+        for (int jj = 0; jj < MAX_B; ++jj)
+            if (jj < j) gl[jj] = fmaf(dcj, sa[jj * 32 + dl], gl[jj]);
+    }
+    for (int jj = 0; jj < j; ++jj) atomicAdd(m.gL + ((size_t)d * B + j) * B + jj, gl[jj]);
+}
+
+// grid NR / 8, 256 threads: one warp per row.  The row's log-sum-exp from the
+// split partials, and its logit at y*: s_y* + W_r[y*] . z (the bf16 operands
+// of the Read, fp32 accumulation).
 __global__ void __launch_bounds__(256) k_train_stats_fin(TrainMisc m)
 {
-    const int row = blockIdx.x * 256 + threadIdx.x;
+    pdl_trigger();
+    pdl_wait();
+    const int row = blockIdx.x * 8 + threadIdx.x / 32, lane = threadIdx.x % 32;
     if (row >= m.NR) return;
     const int i = (row >> 7) * 64 + (row & 63);
     if (i >= m.P) {
-        m.lse_p2[row] = 0.f;
+        if (lane == 0) {
+            m.lse_p2[row] = 0.f;
+            m.ly[row] = 0.f;
+        }
         return;
     }
     float mx = -INFINITY, s = 0.f;
-    for (int sv = 0; sv < m.splits; ++sv) {
+    for (int sv = lane; sv < m.splits; sv += 32) {
         const float4 a = m.part[(size_t)sv * m.NR + row];
         lse2_merge(mx, s, a.x, a.y);
     }
-    m.lse_p2[row] = mx + log2f(s);
+    int y = m.ystar[i];
+    if (y < 0 || y >= m.V) y = 0;                 // reported by k_train_rows_fin
+    // lane: 8 consecutive elements of the 256
+    const uint4 a = reinterpret_cast<const uint4 *>(m.W_r + (size_t)y * RANK)[lane];
+    const uint4 b = reinterpret_cast<const uint4 *>(m.zop + (size_t)row * RANK)[lane];
+    const uint32_t wa[4] = {a.x, a.y, a.z, a.w}, wb[4] = {b.x, b.y, b.z, b.w};
+    float acc = 0.f;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        acc = fmaf(__uint_as_float(wa[q] << 16), __uint_as_float(wb[q] << 16), acc);
+        acc = fmaf(__uint_as_float(wa[q] & 0xFFFF0000u), __uint_as_float(wb[q] & 0xFFFF0000u), acc);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        acc += __shfl_xor_sync(0xffffffffu, acc, o);
+        lse2_merge(mx, s, __shfl_xor_sync(0xffffffffu, mx, o), __shfl_xor_sync(0xffffffffu, s, o));
+    }
+    if (lane == 0) {
+        m.lse_p2[row] = mx + log2f(s);
+        m.ly[row] = m.s_y[i] + acc;
+    }
 }
 
 // grid b, 32 threads: lane k = position k of block blockIdx.x.
 __global__ void __launch_bounds__(32) k_train_tv_fin(TrainMisc m)
 {
+    pdl_trigger();
+    pdl_wait();
     const int blk = blockIdx.x, k = threadIdx.x;
     float lr = 0.f, lb = 0.f, lc = 0.f;
     if (k < m.B) {
@@ -278,20 +385,20 @@ __global__ void __launch_bounds__(32) k_train_tv_fin(TrainMisc m)
                 eq += a.z;
                 anc += a.w;
             }
+            // lt: sum of p where p < q plus half of it where p = q (k_train_tok)
             const float l1 = 2.0f * (1.0f - sm);
             const float S = 1.0f - 2.0f * lt - eq;          // sum_v sgn(p_v - q_v) p_v
             const float ce = m.lse_p2[row] * LN2 - m.ly[row];
             lf[f] = w * (m.a_ce * ce + m.a_l1 * l1);
+            // dL/dl_v = cf [a_ce (p_v - [v = y*]) + a_l1 p_v (sgn(p_v - q_v) - S)]
             const float cf = w * (f == 0 ? 1.0f : m.beta);
             RowCoef rc;
             rc.lse_p2 = m.lse_p2[row];
             rc.lse_q2 = m.lse_q2[i];
-            rc.A0 = cf * (m.a_ce - m.a_l1 * S);
-            rc.A1 = cf * m.a_l1;
-            rc.A2 = cf * m.a_ce;
-            rc.y = m.ystar[i];
-            rc.pad[0] = rc.pad[1] = 0.f;
+            rc.Apos = cf * (m.a_ce + m.a_l1 * (1.0f - S));
+            rc.Aneg = cf * (m.a_ce - m.a_l1 * (1.0f + S));
             m.coef[row] = rc;
+            m.A2[row] = cf * m.a_ce;
         }
         lr = lf[0];
         lc = lf[1];
@@ -313,9 +420,13 @@ __global__ void __launch_bounds__(32) k_train_tv_fin(TrainMisc m)
 }
 
 // grid ceil(NR r / 1024), 256 threads, 4 elements each: dL/dz as the sum of
-// the vocabulary splits' slices in a fixed order, and its bf16 copy.
+// the vocabulary splits' slices in a fixed order plus the -A2 [v = y*] term of
+// dL/dl (-A2 W_r[y*]), and its bf16 copy; the same term of dL/dW_r,
+// -A2 z at row y*, is added into gW_r (atomic: positions share ids).
 __global__ void __launch_bounds__(256) k_train_dz(TrainMisc m)
 {
+    pdl_trigger();
+    pdl_wait();
     const size_t e = ((size_t)blockIdx.x * 256 + threadIdx.x) * 4;
     const size_t n = (size_t)m.NR * RANK;
     if (e >= n) return;
@@ -327,6 +438,23 @@ __global__ void __launch_bounds__(256) k_train_dz(TrainMisc m)
         v.z += o.z;
         v.w += o.w;
     }
+    const int row = (int)(e / RANK), d = (int)(e % RANK);
+    const float a2 = m.A2[row];
+    if (a2 != 0.0f) {
+        int y = m.ystar[(row >> 7) * 64 + (row & 63)];
+        if (y < 0 || y >= m.V) y = 0;             // reported by k_train_rows_fin
+        const uint2 wv = *reinterpret_cast<const uint2 *>(m.W_r + (size_t)y * RANK + d);
+        v.x -= a2 * __uint_as_float(wv.x << 16);
+        v.y -= a2 * __uint_as_float(wv.x & 0xFFFF0000u);
+        v.z -= a2 * __uint_as_float(wv.y << 16);
+        v.w -= a2 * __uint_as_float(wv.y & 0xFFFF0000u);
+        const uint2 zv = *reinterpret_cast<const uint2 *>(m.zop + (size_t)row * RANK + d);
+        float *g = m.gW_r + (size_t)y * RANK + d;
+        atomicAdd(g + 0, -a2 * __uint_as_float(zv.x << 16));
+        atomicAdd(g + 1, -a2 * __uint_as_float(zv.x & 0xFFFF0000u));
+        atomicAdd(g + 2, -a2 * __uint_as_float(zv.y << 16));
+        atomicAdd(g + 3, -a2 * __uint_as_float(zv.y & 0xFFFF0000u));
+    }
     *reinterpret_cast<float4 *>(m.dz + e) = v;
     *reinterpret_cast<uint2 *>(m.dzb + e) = make_uint2(pack_bf16x2(v.x, v.y), pack_bf16x2(v.z, v.w));
 }
@@ -334,6 +462,8 @@ __global__ void __launch_bounds__(256) k_train_dz(TrainMisc m)
 // grid ceil(NR 2r / 1024), 256 threads: dL/dt = dL/du sigma'(t), 4 elements each.
 __global__ void __launch_bounds__(256) k_train_dact(TrainMisc m)
 {
+    pdl_trigger();
+    pdl_wait();
     const size_t e = ((size_t)blockIdx.x * 256 + threadIdx.x) * 4;
     if (e >= (size_t)m.NR * 2 * RANK) return;
     const float4 du = *reinterpret_cast<const float4 *>(m.du + e);
@@ -343,36 +473,11 @@ __global__ void __launch_bounds__(256) k_train_dact(TrainMisc m)
                    pack_bf16x2(du.z * sigma_prime(m.act, t.z), du.w * sigma_prime(m.act, t.w)));
 }
 
-// grid (b, 2), r threads.
-__global__ void __launch_bounds__(RANK) k_train_mix_bwd(TrainMisc m)
-{
-    const int blk = blockIdx.x, f = blockIdx.y, d = threadIdx.x, B = m.B;
-    float dcv[MAX_B];
-    for (int k = 0; k < B; ++k) dcv[k] = m.dc[(size_t)pair_row(blk * B + k, f) * RANK + d];
-    for (int j = 0; j < B; ++j) {
-        float acc = dcv[j];
-        for (int k = j + 1; k < B; ++k) acc = fmaf(bf2f(m.L[((size_t)d * B + k) * B + j]), dcv[k], acc);
-        m.dab[(size_t)pair_row(blk * B + j, f) * RANK + d] = f2bf(acc);
-    }
-}
-
-// grid B * B ((k, j) = (blockIdx.x / B, blockIdx.x % B), only j < k), r threads:
-// dL/dL_kj^(d) = sum over blocks and both forwards of dc_k^(d) a_j^(d).
-__global__ void __launch_bounds__(RANK) k_train_gL(TrainMisc m)
-{
-    const int k = blockIdx.x / m.B, j = blockIdx.x % m.B, d = threadIdx.x;
-    if (j >= k) return;
-    float acc = 0.f;
-    for (int blk = 0; blk < m.b; ++blk)
-        for (int f = 0; f < 2; ++f)
-            acc = fmaf(m.dc[(size_t)pair_row(blk * m.B + k, f) * RANK + d],
-                       m.a[(size_t)pair_row(blk * m.B + j, f) * RANK + d], acc);
-    m.gL[((size_t)d * m.B + k) * m.B + j] += acc;
-}
-
 // grid P, r threads.
 __global__ void __launch_bounds__(RANK) k_train_fuse_bwd(TrainMisc m)
 {
+    pdl_trigger();
+    pdl_wait();
     const int i = blockIdx.x, d = threadIdx.x, r3 = 3 * RANK;
     const int blk = i / m.B;
     const int rt = pair_row(i, 0), rc = pair_row(i, 1);

@@ -12,18 +12,25 @@
 //
 // k_train_tok -- token-major: D[row, v] = z_row . W_r[v], M = 128 rows, N = 64
 // vocabulary ids, K = r.  CTA (split, tile) takes one row tile and a
-// contiguous range of vocabulary tiles.  Modes:
-//   TR_STATS  per row the running max / log2-sum of l (log2 domain) and l at y*
+// contiguous range of vocabulary tiles.  The row tile Z sits in tensor memory
+// as the A operand (with N = 64, re-reading a 4 KB A block from shared memory
+// for every MMA would cost more than the product), so shared memory holds
+// only the W_r and s / t rings.  Modes:
+//   TR_STATS  per row the running max / log2-sum of l (log2 domain)
 //   TR_TV     per row sum_v min(p, q), the part where p < q and where p = q
 //             (compared in the log domain: one exp2 per element), and per
 //             position the same sum for the drafter's p^b = softmax(s)
-//   TR_DZ     dl = p (A0 + A1 sgn(p - q)) - A2 [v = y*] as a bf16 tile in
-//             shared memory, then dz += dl W_r on the tensor core (W_r tile
-//             read MN-major); each split stores its dz slice at the end
+//   TR_DZ     dl = p A(sgn(p - q)) as a bf16 tile in shared memory, then
+//             dz += dl W_r on the tensor core (W_r tile read MN-major); each
+//             split stores its dz slice at the end
 // k_train_voc -- vocabulary-major: D[v, row] = W_r[v] . z_row, M = 128 ids,
 // N = 64 rows (32 positions x both forwards); the same dl (transposed) feeds
 // dW_r[v, :] += dl^T Z (Z tile read MN-major), accumulated in TMEM over every
 // row of the step and added into gW_r once per vocabulary tile.
+// The s and t tiles stream from HBM: the producers prefetch them into L2 a
+// few tiles ahead (tensor-map prefetch) so that the TMA loads of the rings
+// hit L2.  The -A2 [v = y*] term of dL/dl and l at y* are left to the small
+// kernels (k_train_dz, k_train_stats_fin), so the loops here carry no id test.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -36,35 +43,53 @@ constexpr float L2E = 1.4426950408889634f;
 // ---------------------------------------------------------------- k_train_tok
 constexpr int TR_BM = 128;
 constexpr int TR_BN = 64;
-constexpr int TR_BSTAGES = 3;
-constexpr int TR_SSTAGES = 2;
-constexpr int TR_EPI_WARPS = 8;                            // 2 per TMEM lane quarter: 32 ids each
+constexpr int TR_BMAX = 5;                                 // most W_r ring stages
+constexpr int TR_SMAX = 8;                                 // most s / t ring stages
+constexpr int TR_PF = 8;                                   // s / t tiles prefetched into L2 ahead
+constexpr int TR_EPI_WARPS = 16;                           // 2 sets (item parity) x 4 lane quarters x 2 id groups
+constexpr int TR_SET = TR_EPI_WARPS / 2;                   // the warps that take one item
 constexpr int TR_THREADS = 32 * (2 + TR_EPI_WARPS);
-constexpr uint32_t TR_A_CHUNK = TR_BM * 64 * 2;            // 16 KB: 128 rows x 64 of r
-constexpr uint32_t TR_A_BYTES = 4 * TR_A_CHUNK;            // 64 KB
 constexpr uint32_t TR_B_CHUNK = TR_BN * 64 * 2;            // 8 KB: 64 ids x 64 of r
 constexpr uint32_t TR_B_STAGE = 4 * TR_B_CHUNK;            // 32 KB: one vocabulary tile of W_r
 constexpr uint32_t TR_ST_TILE = 64 * TR_BN * 2;            // 8 KB: 64 positions x 64 ids of s (or t)
-constexpr uint32_t TR_S_STAGE = 2 * TR_ST_TILE;            // s and t
 constexpr uint32_t TR_D_BUF = TR_BM * TR_BN * 2;           // 16 KB: dl tile, bf16, K-major (K = ids)
+constexpr uint32_t TR_RINGS = 224 * 1024;                  // W_r ring, s / t ring (and the dl tiles in TR_DZ)
 constexpr uint32_t TR_IDESC_F = idesc_bf16(TR_BM, TR_BN);
 constexpr uint32_t TR_IDESC_D = idesc_bf16_mn(TR_BM, RANK, false, true);
-constexpr uint32_t TR_TMEM_COLS = 512;                     // l: 2 x 64 at 0; dz: 256 at 256
+constexpr int TR_NBUF = 4;                                 // most l accumulators in flight
+// TMEM: l accumulators (4, TR_DZ: 2) of 64 columns from 0, then the Z tile (128
+// columns: 256 bf16 per lane, two per column), then in TR_DZ dz (256) at 256
+constexpr uint32_t TR_TMEM_COLS = 512;
 constexpr uint32_t TR_DZ_COL = 256;
 
 struct TrShared {
     uint64_t a_full;
-    uint64_t full[TR_BSTAGES], empty[TR_BSTAGES];
-    uint64_t sfull[TR_SSTAGES], sempty[TR_SSTAGES];
-    uint64_t tfull[2], tempty[2];
+    uint64_t full[TR_BMAX], empty[TR_BMAX];
+    uint64_t sfull[TR_SMAX], sempty[TR_SMAX];
+    uint64_t tfull[TR_NBUF], tempty[TR_NBUF];
     uint64_t dfull[2], dempty[2];
     uint64_t zdone, drain;
     uint32_t tmem_base;
     int abort;
 };
 
-constexpr size_t TR_SMEM = 1024 + TR_A_BYTES + TR_BSTAGES * TR_B_STAGE + TR_SSTAGES * TR_S_STAGE + 2 * TR_D_BUF +
-                           sizeof(TrShared);
+constexpr size_t TR_SMEM = 1024 + TR_RINGS + sizeof(TrShared);
+static_assert(TR_SMEM <= 232448, "k_train_tok shared memory");
+
+// The rings of each mode (TR_RINGS holds them): W_r stages (the W_r loads
+// from L2 take about 2 us under load, so their ring depth sets the pace; the
+// s / t tiles are prefetched into L2 and need fewer), s / t stage bytes and
+// stages, and the two dl tiles in TR_DZ.
+__host__ __device__ constexpr int tr_bstages(int mode) { return mode == TR_DZ ? 4 : 5; }
+__host__ __device__ constexpr int tr_nbuf(int mode) { return mode == TR_DZ ? 2 : TR_NBUF; }
+__host__ __device__ constexpr uint32_t tr_stage_bytes(int mode) { return mode == TR_STATS ? TR_ST_TILE : 2 * TR_ST_TILE; }
+__host__ __device__ constexpr int tr_stages(int mode)
+{
+    return (int)((TR_RINGS - tr_bstages(mode) * TR_B_STAGE - (mode == TR_DZ ? 2 * TR_D_BUF : 0)) / tr_stage_bytes(mode));
+}
+static_assert(tr_stages(TR_STATS) <= TR_SMAX && tr_stages(TR_TV) >= 2 && tr_stages(TR_DZ) >= 2 &&
+                  tr_stages(TR_TV) <= TR_SMAX && tr_stages(TR_DZ) <= TR_SMAX && tr_bstages(TR_STATS) <= TR_BMAX,
+              "ring depths");
 
 __device__ __forceinline__ void tr_epi_bar()
 {
@@ -79,9 +104,6 @@ __device__ __forceinline__ void ld_tile32(const uint8_t *tile, int pr, int h, ui
         r[c] = *reinterpret_cast<const uint4 *>(tile + pr * 128 + (((4 * h + c) ^ (pr & 7)) << 4));
 }
 
-__device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
-
 __device__ __forceinline__ void unpack32(const uint4 (&r)[4], float (&x)[32])
 {
 #pragma unroll
@@ -89,24 +111,33 @@ __device__ __forceinline__ void unpack32(const uint4 (&r)[4], float (&x)[32])
         const uint32_t w[4] = {r[c].x, r[c].y, r[c].z, r[c].w};
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-            x[8 * c + 2 * q] = bf_lo(w[q]);
-            x[8 * c + 2 * q + 1] = bf_hi(w[q]);
+            x[8 * c + 2 * q] = __uint_as_float(w[q] << 16);
+            x[8 * c + 2 * q + 1] = __uint_as_float(w[q] & 0xFFFF0000u);
         }
     }
 }
 
-// log2-domain running log-sum-exp: value = s * 2^m
-__device__ __forceinline__ void lse2_add32(float &m, float &s, const float (&x)[32])
+// log2-domain running log-sum-exp over 16 values: value = s * 2^m.  The max
+// and the sum run as trees (short dependent chains).
+__device__ __forceinline__ void lse2_add16(float &m, float &s, const float (&x)[16])
 {
-    float gm = x[0];
+    float t[8];
 #pragma unroll
-    for (int j = 1; j < 32; ++j) gm = fmaxf(gm, x[j]);
-    const float M = fmaxf(m, gm);
+    for (int j = 0; j < 8; ++j) t[j] = fmaxf(x[j], x[j + 8]);
+#pragma unroll
+    for (int w = 4; w >= 1; w >>= 1)
+#pragma unroll
+        for (int j = 0; j < w; ++j) t[j] = fmaxf(t[j], t[j + w]);
+    const float M = fmaxf(m, t[0]);
     if (M == -INFINITY) return;
-    float acc = 0.0f;
+    float e[8];
 #pragma unroll
-    for (int j = 0; j < 32; ++j) acc += ex2_approx(x[j] - M);
-    s = s * ex2_approx(m - M) + acc;
+    for (int j = 0; j < 8; ++j) e[j] = ex2_approx(x[j] - M) + ex2_approx(x[j + 8] - M);
+#pragma unroll
+    for (int w = 4; w >= 1; w >>= 1)
+#pragma unroll
+        for (int j = 0; j < w; ++j) e[j] += e[j + w];
+    s = s * ex2_approx(m - M) + e[0];
     m = M;
 }
 
@@ -118,12 +149,21 @@ __device__ __forceinline__ void lse2_merge(float &m, float &s, float om, float o
     m = M;
 }
 
+// dL/dl_v without the y* term: p A(sgn(p - q)); A(0) = (Apos + Aneg) / 2
+__device__ __forceinline__ float dl_value(float a2, float b2, float Apos, float Aneg)
+{
+    const float A = a2 > b2 ? Apos : (a2 < b2 ? Aneg : 0.5f * (Apos + Aneg));
+    return ex2_approx(a2) * A;
+}
+
 }  // namespace
 
 const size_t kTrainTokSmemBytes = TR_SMEM;
 const int kTrainTokThreads = TR_THREADS;
 
-// grid (splits, NR / 128), TR_THREADS threads, TR_SMEM bytes.
+// grid (splits, NR / 128), TR_THREADS threads, TR_SMEM bytes.  tmap_z is not
+// read (Z goes to tensor memory from p.zop); the argument keeps the four maps
+// of the vocabulary-major kernel.
 __global__ void __launch_bounds__(TR_THREADS, 1)
     k_train_tok(const __grid_constant__ TrainParams p, const __grid_constant__ CUtensorMap tmap_z,
                 const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_s,
@@ -131,25 +171,29 @@ __global__ void __launch_bounds__(TR_THREADS, 1)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t *sA = base;
-    uint8_t *sB = sA + TR_A_BYTES;
-    uint8_t *sS = sB + TR_BSTAGES * TR_B_STAGE;
-    uint8_t *sD = sS + TR_SSTAGES * TR_S_STAGE;
-    TrShared &sh = *reinterpret_cast<TrShared *>(sD + 2 * TR_D_BUF);
+    uint8_t *sB = base;
+    TrShared &sh = *reinterpret_cast<TrShared *>(sB + TR_RINGS);
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const int j = blockIdx.y, sv = blockIdx.x;
     const int vt0 = (int)((long long)p.nvt * sv / p.splits), vt1 = (int)((long long)p.nvt * (sv + 1) / p.splits);
     const int items = vt1 - vt0;
     const bool dzm = mode == TR_DZ;
+    const int NB = tr_bstages(mode), NS = tr_stages(mode), NBUF = tr_nbuf(mode);
+    const uint32_t ZC = NBUF * TR_BN;              // TMEM column of the Z tile
+    const uint32_t SB = tr_stage_bytes(mode);
+    uint8_t *sS = sB + NB * TR_B_STAGE;            // s / t ring after the W_r ring
+    uint8_t *sD = sS + NS * SB;                    // TR_DZ: the two dl tiles after the s / t ring
 
     if (threadIdx.x == 0) {
-        mbar_init(&sh.a_full, 1);
-        for (int i = 0; i < TR_BSTAGES; ++i) { mbar_init(&sh.full[i], 1); mbar_init(&sh.empty[i], 1); }
-        for (int i = 0; i < TR_SSTAGES; ++i) { mbar_init(&sh.sfull[i], 1); mbar_init(&sh.sempty[i], TR_EPI_WARPS); }
-        for (int i = 0; i < 2; ++i) {
+        mbar_init(&sh.a_full, TR_EPI_WARPS);       // every epilogue warp stores its part of Z
+        for (int i = 0; i < NB; ++i) { mbar_init(&sh.full[i], 1); mbar_init(&sh.empty[i], 1); }
+        for (int i = 0; i < NS; ++i) { mbar_init(&sh.sfull[i], 1); mbar_init(&sh.sempty[i], TR_SET); }
+        for (int i = 0; i < TR_NBUF; ++i) {
             mbar_init(&sh.tfull[i], 1);
-            mbar_init(&sh.tempty[i], TR_EPI_WARPS);
-            mbar_init(&sh.dfull[i], TR_EPI_WARPS);
+            mbar_init(&sh.tempty[i], TR_SET);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&sh.dfull[i], TR_SET);
             mbar_init(&sh.dempty[i], 1);
         }
         mbar_init(&sh.zdone, 1);
@@ -158,6 +202,8 @@ __global__ void __launch_bounds__(TR_THREADS, 1)
         fence_barrier_init();
     }
     if (warp == 1) { tmem_alloc(&sh.tmem_base, TR_TMEM_COLS); tmem_relinquish(); }
+    pdl_trigger();                 // the next kernel may start its set-up
+    pdl_wait();                    // Z, the statistics and the coefficients are complete
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -168,72 +214,102 @@ __global__ void __launch_bounds__(TR_THREADS, 1)
     if (warp == 0) {
         // ------------------------------------------------------- producer
         if (lane == 0 && items > 0) {
-            tma_prefetch_desc(&tmap_z);
             tma_prefetch_desc(&tmap_w);
             tma_prefetch_desc(&tmap_s);
             tma_prefetch_desc(&tmap_t);
             const uint64_t keep = policy_evict_last(), once = policy_evict_first();
             const bool need_t = mode != TR_STATS;
-            mbar_expect_tx(&sh.a_full, TR_A_BYTES);
-            for (int c = 0; c < 4; ++c) tma_load_2d(sA + c * TR_A_CHUNK, &tmap_z, &sh.a_full, c * 64, j * TR_BM);
+            auto prefetch_st = [&](int it) {
+                tma_prefetch_2d(&tmap_s, (vt0 + it) * TR_BN, j * 64);
+                if (need_t) tma_prefetch_2d(&tmap_t, (vt0 + it) * TR_BN, j * 64);
+            };
+            for (int it = 0; it < min(TR_PF, items); ++it) prefetch_st(it);
             uint32_t pend_b = 0, par_b = 0, pend_s = 0, par_s = 0;
+            int ss = 0;
+            uint32_t sph = 0;
             for (int it = 0; it < items && !*abort; ++it) {
                 const int vt = vt0 + it;
-                const int st = it % TR_BSTAGES;
-                const uint32_t ph = (uint32_t)((it / TR_BSTAGES) & 1);
-                if (!mbar_wait(&sh.empty[st], ph ^ 1, abort, lim)) break;
+                if (it + TR_PF < items) prefetch_st(it + TR_PF);
+                const int st = it % NB;
+                const uint32_t ph = (uint32_t)((it / NB) & 1);
+                if (!mbar_wait_spin(&sh.empty[st], ph ^ 1, abort, lim)) break;
                 mbar_expect_tx(&sh.full[st], TR_B_STAGE);
                 for (int c = 0; c < 4; ++c)
                     tma_load_2d_hint(sB + st * TR_B_STAGE + c * TR_B_CHUNK, &tmap_w, &sh.full[st], c * 64, vt * TR_BN,
                                      keep);
                 pend_b |= 1u << st;
                 par_b = (par_b & ~(1u << st)) | (ph << st);
-                const int ss = it & 1;
-                const uint32_t sph = (uint32_t)((it >> 1) & 1);
-                if (!mbar_wait(&sh.sempty[ss], sph ^ 1, abort, lim)) break;
-                mbar_expect_tx(&sh.sfull[ss], need_t ? TR_S_STAGE : TR_ST_TILE);
-                tma_load_2d_hint(sS + ss * TR_S_STAGE, &tmap_s, &sh.sfull[ss], vt * TR_BN, j * 64, once);
+                if (!mbar_wait_spin(&sh.sempty[ss], sph ^ 1, abort, lim)) break;
+                mbar_expect_tx(&sh.sfull[ss], SB);
+                tma_load_2d_hint(sS + ss * SB, &tmap_s, &sh.sfull[ss], vt * TR_BN, j * 64, once);
                 if (need_t)
-                    tma_load_2d_hint(sS + ss * TR_S_STAGE + TR_ST_TILE, &tmap_t, &sh.sfull[ss], vt * TR_BN, j * 64,
-                                     once);
+                    tma_load_2d_hint(sS + ss * SB + TR_ST_TILE, &tmap_t, &sh.sfull[ss], vt * TR_BN, j * 64, once);
                 pend_s |= 1u << ss;
                 par_s = (par_s & ~(1u << ss)) | (sph << ss);
+                if (++ss == NS) { ss = 0; sph ^= 1; }
             }
             if (*abort) {
                 // no copy may still be landing when the CTA leaves
                 int dummy = 0;
-                mbar_wait(&sh.a_full, 0, &dummy, 100000000ull);
-                for (int st = 0; st < TR_BSTAGES; ++st)
-                    if (pend_b & (1u << st)) mbar_wait(&sh.full[st], (par_b >> st) & 1, &dummy, 100000000ull);
-                for (int ss = 0; ss < TR_SSTAGES; ++ss)
-                    if (pend_s & (1u << ss)) mbar_wait(&sh.sfull[ss], (par_s >> ss) & 1, &dummy, 100000000ull);
+                for (int st = 0; st < NB; ++st)
+                    if (pend_b & (1u << st)) mbar_wait_spin(&sh.full[st], (par_b >> st) & 1, &dummy, 100000000ull);
+                for (int s2 = 0; s2 < NS; ++s2)
+                    if (pend_s & (1u << s2)) mbar_wait_spin(&sh.sfull[s2], (par_s >> s2) & 1, &dummy, 100000000ull);
             }
         }
     } else if (warp == 1) {
         // ---------------------------------------------------- MMA issuer
         if (lane == 0 && items > 0) {
-            const uint32_t a0 = smem_u32(sA), b0 = smem_u32(sB), d0 = smem_u32(sD);
+            const uint32_t b0 = smem_u32(sB), d0 = smem_u32(sD);
             // dz += dl(u) W_r(u): A = the dl tile (K-major over ids), B = the W_r
             // tile read MN-major (N = r along the 128-byte rows, K = ids)
             auto dz_step = [&](int u) -> bool {
                 const int db = u & 1;
-                if (!mbar_wait(&sh.dfull[db], (uint32_t)((u >> 1) & 1), abort, lim)) return false;
+                if (!mbar_wait_spin(&sh.dfull[db], (uint32_t)((u >> 1) & 1), abort, lim)) return false;
                 tc_fence_after();
-                const uint32_t bs = b0 + (u % TR_BSTAGES) * TR_B_STAGE;
+                const uint32_t bs = b0 + (u % NB) * TR_B_STAGE;
 #pragma unroll
                 for (int kk = 0; kk < TR_BN / 16; ++kk)
                     tc_mma_bf16(tmem + TR_DZ_COL, smem_desc_sw128(d0 + db * TR_D_BUF + kk * 32),
                                 smem_desc_sw128_mn(bs + kk * 2048, TR_B_CHUNK), TR_IDESC_D, (u | kk) != 0);
-                tc_commit(&sh.empty[u % TR_BSTAGES]);
+                tc_commit(&sh.empty[u % NB]);
                 tc_commit(&sh.dempty[db]);
                 return true;
             };
-            bool ok = mbar_wait(&sh.a_full, 0, abort, lim);
+            bool ok = mbar_wait_spin(&sh.a_full, 0, abort, lim);
             if (ok) tc_fence_after();
-            for (int it = 0; it < items && ok; ++it) {
-                const int st = it % TR_BSTAGES, buf = it & 1;
-                if (!mbar_wait(&sh.full[st], (uint32_t)((it / TR_BSTAGES) & 1), abort, lim) ||
-                    !mbar_wait(&sh.tempty[buf], (uint32_t)(((it >> 1) & 1) ^ 1), abort, lim)) {
+            // without dz: two tiles at a time, their MMA chains interleaved
+            // (two accumulators), so that consecutive MMAs do not depend on
+            // one another
+            for (int it = 0; it + 1 < items && ok && !dzm; it += 2) {
+                const int st0 = it % NB, st1 = (it + 1) % NB, b0_ = it % NBUF, b1_ = (it + 1) % NBUF;
+                if (!mbar_wait_spin(&sh.full[st0], (uint32_t)((it / NB) & 1), abort, lim) ||
+                    !mbar_wait_spin(&sh.full[st1], (uint32_t)(((it + 1) / NB) & 1), abort, lim) ||
+                    !mbar_wait_spin(&sh.tempty[b0_], (uint32_t)(((it / NBUF) & 1) ^ 1), abort, lim) ||
+                    !mbar_wait_spin(&sh.tempty[b1_], (uint32_t)((((it + 1) / NBUF) & 1) ^ 1), abort, lim)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t bs0 = b0 + st0 * TR_B_STAGE, bs1 = b0 + st1 * TR_B_STAGE;
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk) {
+                        tc_mma_bf16_ts(tmem + b0_ * TR_BN, tmem + ZC + c * 32 + kk * 8,
+                                       smem_desc_sw128(bs0 + c * TR_B_CHUNK + kk * 32), TR_IDESC_F, (c | kk) != 0);
+                        tc_mma_bf16_ts(tmem + b1_ * TR_BN, tmem + ZC + c * 32 + kk * 8,
+                                       smem_desc_sw128(bs1 + c * TR_B_CHUNK + kk * 32), TR_IDESC_F, (c | kk) != 0);
+                    }
+                tc_commit(&sh.tfull[b0_]);
+                tc_commit(&sh.tfull[b1_]);
+                tc_commit(&sh.empty[st0]);
+                tc_commit(&sh.empty[st1]);
+            }
+            for (int it = dzm ? 0 : (items & ~1); it < items && ok; ++it) {
+                const int st = it % NB, buf = it % NBUF;
+                if (!mbar_wait_spin(&sh.full[st], (uint32_t)((it / NB) & 1), abort, lim) ||
+                    !mbar_wait_spin(&sh.tempty[buf], (uint32_t)(((it / NBUF) & 1) ^ 1), abort, lim)) {
                     ok = false;
                     break;
                 }
@@ -243,8 +319,8 @@ __global__ void __launch_bounds__(TR_THREADS, 1)
                 for (int c = 0; c < 4; ++c)
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk)
-                        tc_mma_bf16(tmem + buf * TR_BN, smem_desc_sw128(a0 + c * TR_A_CHUNK + kk * 32),
-                                    smem_desc_sw128(bs + c * TR_B_CHUNK + kk * 32), TR_IDESC_F, (c | kk) != 0);
+                        tc_mma_bf16_ts(tmem + buf * TR_BN, tmem + ZC + c * 32 + kk * 8,
+                                       smem_desc_sw128(bs + c * TR_B_CHUNK + kk * 32), TR_IDESC_F, (c | kk) != 0);
                 tc_commit(&sh.tfull[buf]);
                 if (!dzm) tc_commit(&sh.empty[st]);
                 else if (it > 0 && !dz_step(it - 1)) ok = false;
@@ -258,14 +334,16 @@ __global__ void __launch_bounds__(TR_THREADS, 1)
         }
     } else {
         // ------------------------------------------------------ epilogue
-        const int ew = warp - 2, q = warp & 3, g = ew >> 2;
+        // warp set `set` takes the items of its parity (accumulators set and
+        // set + 2, dl tile `set`); within a set, warp (q, g) the 32 rows of
+        // lane quarter q and the 32 ids of group g, in two halves of 16
+        const int ew = warp - 2, q = warp & 3, g = (ew >> 2) & 1, set = ew >> 3;
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
         const int row = q * 32 + lane, f = row >> 6, pl = row & 63;
         const int i = j * 64 + pl;                 // position
         const int rowg = j * TR_BM + row;          // paired row
         const bool valid = i < p.P;
-        const int y = valid ? p.ystar[i] : -1;
-        float lp2 = 0.f, lq2 = 0.f, ls2 = 0.f, A0 = 0.f, A1 = 0.f, A2 = 0.f;
+        float lp2 = 0.f, lq2 = 0.f, ls2 = 0.f, Apos = 0.f, Aneg = 0.f;
         if (valid && mode != TR_STATS) {
             lp2 = p.lse_p2[rowg];
             lq2 = p.lse_q2[i];
@@ -273,118 +351,171 @@ __global__ void __launch_bounds__(TR_THREADS, 1)
         }
         if (valid && dzm) {
             const RowCoef rc = p.coef[rowg];
-            A0 = rc.A0;
-            A1 = rc.A1;
-            A2 = rc.A2;
+            Apos = rc.Apos;
+            Aneg = rc.Aneg;
+        }
+        // Z into TMEM: warp (q, g, set) stores K elements 64 cb .. 64 cb + 63
+        // (columns ZC + 32 cb ..) of its 32 rows, cb = 2 set + g
+        {
+            const int cb = 2 * set + g;
+            const uint4 *src = reinterpret_cast<const uint4 *>(p.zop + (size_t)rowg * RANK + 64 * cb);
+            uint32_t zr[32];
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                const uint4 v = src[c];
+                zr[4 * c] = v.x;
+                zr[4 * c + 1] = v.y;
+                zr[4 * c + 2] = v.z;
+                zr[4 * c + 3] = v.w;
+            }
+            tmem_st32(tmem + lane_base + ZC + 32 * cb, zr);
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sh.a_full);
         }
         // the anchor term's share: the teacher-forced row takes the even
         // 32-id group of each tile, the consistency row the odd one
         const bool anchor = (f == g);
-        float r0 = -INFINITY, r1 = 0.f, r2 = 0.f, r3 = 0.f;   // STATS: m, s; TV: sum min, lt, eq, anchor
-        if (mode == TR_TV) r0 = 0.f;
+        // STATS: running (m, s); TV: 2-way partial sums of min(p, q), of the
+        // part where p < q (+ half of where p = q), and of the anchor's min(p^b, q)
+        float m2 = -INFINITY, s2 = 0.f;
+        float r0[2] = {0.f, 0.f}, r1[2] = {0.f, 0.f}, r3[2] = {0.f, 0.f};
         bool ok = true;
-        for (int it = 0; it < items; ++it) {
-            const int buf = it & 1;
-            const uint32_t ph = (uint32_t)((it >> 1) & 1);
-            if (!mbar_wait(&sh.tfull[buf], ph, abort, lim) || !mbar_wait(&sh.sfull[buf], ph, abort, lim)) {
+        for (int it = set; it < items; it += 2) {
+            const int buf = it % NBUF;
+            const uint32_t ph = (uint32_t)((it >> 1) & 1);      // phase of the dl tile `set`
+            const int ss = it % NS;
+            if (!mbar_wait_spin(&sh.tfull[buf], (uint32_t)((it / NBUF) & 1), abort, lim) ||
+                !mbar_wait_spin(&sh.sfull[ss], (uint32_t)((it / NS) & 1), abort, lim)) {
                 ok = false;
                 break;
             }
             tc_fence_after();
-            float acc[32];
-            tmem_ld32(tmem + lane_base + buf * TR_BN + g * 32, acc);
-            uint4 sr[4], tr[4];
-            const uint8_t *stile = sS + buf * TR_S_STAGE;
-            ld_tile32(stile, pl, g, sr);
-            if (mode != TR_STATS) ld_tile32(stile + TR_ST_TILE, pl, g, tr);
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) {
-                mbar_arrive(&sh.tempty[buf]);
-                mbar_arrive(&sh.sempty[buf]);
-            }
+            const uint8_t *stile = sS + ss * SB;
             const int v0 = (vt0 + it) * TR_BN + g * 32;
-            const int nv = min(32, p.V - v0);
-            float sv32[32];
-            unpack32(sr, sv32);
-            if (mode == TR_STATS) {
-                if (valid) {
-                    float x[32];
+            const int nv = valid ? min(32, p.V - v0) : 0;
+            uint32_t w[16];
 #pragma unroll
-                    for (int jj = 0; jj < 32; ++jj) {
-                        const float l = acc[jj] + sv32[jj];
-                        x[jj] = jj < nv ? l * L2E : -INFINITY;
-                        if (v0 + jj == y) p.ly[rowg] = l;
-                    }
-                    lse2_add32(r0, r1, x);
+            for (int h = 0; h < 2; ++h) {
+                float acc[16];
+                tmem_ld16(tmem + lane_base + buf * TR_BN + g * 32 + h * 16, acc);
+                // this half's 16 ids of s (and t): chunks 4g + 2h, + 1 of the row
+                uint4 sr[2], tr[2];
+#pragma unroll
+                for (int c = 0; c < 2; ++c) {
+                    const int off = pl * 128 + (((4 * g + 2 * h + c) ^ (pl & 7)) << 4);
+                    sr[c] = *reinterpret_cast<const uint4 *>(stile + off);
+                    if (mode != TR_STATS) tr[c] = *reinterpret_cast<const uint4 *>(stile + TR_ST_TILE + off);
                 }
-            } else {
-                float tv32[32];
-                unpack32(tr, tv32);
-                if (mode == TR_TV) {
-                    if (valid) {
+                float sv[16], tv[16];
 #pragma unroll
-                        for (int jj = 0; jj < 32; ++jj) {
-                            if (jj < nv) {
-                                const float a2 = fmaf(acc[jj] + sv32[jj], L2E, -lp2);
-                                const float b2 = fmaf(tv32[jj], L2E, -lq2);
+                for (int c = 0; c < 2; ++c) {
+                    const uint32_t ws_[4] = {sr[c].x, sr[c].y, sr[c].z, sr[c].w};
+                    const uint32_t wt_[4] = {tr[c].x, tr[c].y, tr[c].z, tr[c].w};
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        sv[8 * c + 2 * e] = __uint_as_float(ws_[e] << 16);
+                        sv[8 * c + 2 * e + 1] = __uint_as_float(ws_[e] & 0xFFFF0000u);
+                        tv[8 * c + 2 * e] = __uint_as_float(wt_[e] << 16);
+                        tv[8 * c + 2 * e + 1] = __uint_as_float(wt_[e] & 0xFFFF0000u);
+                    }
+                }
+                const int nh = nv - 16 * h;              // ids of this half that exist (<= 0: none)
+                if (mode == TR_STATS) {
+                    if (nh > 0) {
+                        float x[16];
+#pragma unroll
+                        for (int jj = 0; jj < 16; ++jj) x[jj] = jj < nh ? (acc[jj] + sv[jj]) * L2E : -INFINITY;
+                        lse2_add16(m2, s2, x);
+                    }
+                } else if (mode == TR_TV) {
+                    if (nh >= 16) {
+#pragma unroll
+                        for (int jj = 0; jj < 16; ++jj) {
+                            const float a2 = fmaf(acc[jj] + sv[jj], L2E, -lp2);
+                            const float b2 = fmaf(tv[jj], L2E, -lq2);
+                            const float m = ex2_approx(fminf(a2, b2));
+                            r0[jj & 1] += m;
+                            r1[jj & 1] += a2 < b2 ? m : (a2 == b2 ? 0.5f * m : 0.f);
+                            if (anchor) r3[jj & 1] += ex2_approx(fminf(fmaf(sv[jj], L2E, -ls2), b2));
+                        }
+                    } else if (nh > 0) {
+                        // the vocabulary's last tile: the same, masked
+#pragma unroll
+                        for (int jj = 0; jj < 16; ++jj) {
+                            if (jj < nh) {
+                                const float a2 = fmaf(acc[jj] + sv[jj], L2E, -lp2);
+                                const float b2 = fmaf(tv[jj], L2E, -lq2);
                                 const float m = ex2_approx(fminf(a2, b2));
-                                r0 += m;
-                                r1 += a2 < b2 ? m : 0.f;
-                                r2 += a2 == b2 ? m : 0.f;
-                                if (anchor) r3 += ex2_approx(fminf(fmaf(sv32[jj], L2E, -ls2), b2));
+                                r0[jj & 1] += m;
+                                r1[jj & 1] += a2 < b2 ? m : (a2 == b2 ? 0.5f * m : 0.f);
+                                if (anchor) r3[jj & 1] += ex2_approx(fminf(fmaf(sv[jj], L2E, -ls2), b2));
                             }
                         }
                     }
                 } else {
-                    uint32_t w[16];
 #pragma unroll
-                    for (int jj = 0; jj < 32; jj += 2) {
+                    for (int jj = 0; jj < 16; jj += 2) {
                         float d2[2];
 #pragma unroll
                         for (int e = 0; e < 2; ++e) {
                             const int jv = jj + e;
-                            const float a2 = fmaf(acc[jv] + sv32[jv], L2E, -lp2);
-                            const float b2 = fmaf(tv32[jv], L2E, -lq2);
-                            const float pv = ex2_approx(a2);
-                            const float sg = a2 > b2 ? 1.f : (a2 < b2 ? -1.f : 0.f);
-                            float d = pv * fmaf(A1, sg, A0) - (v0 + jv == y ? A2 : 0.f);
-                            d2[e] = (jv < nv && valid) ? d : 0.f;
+                            const float a2 = fmaf(acc[jv] + sv[jv], L2E, -lp2);
+                            const float b2 = fmaf(tv[jv], L2E, -lq2);
+                            d2[e] = jv < nh ? dl_value(a2, b2, Apos, Aneg) : 0.f;
                         }
-                        w[jj / 2] = pack_bf16x2(d2[0], d2[1]);
+                        w[8 * h + jj / 2] = pack_bf16x2(d2[0], d2[1]);
                     }
-                    if (!mbar_wait(&sh.dempty[buf], ph ^ 1, abort, lim)) { ok = false; break; }
-                    uint8_t *dt = sD + buf * TR_D_BUF + row * 128;
-#pragma unroll
-                    for (int c = 0; c < 4; ++c)
-                        *reinterpret_cast<uint4 *>(dt + (((4 * g + c) ^ (row & 7)) << 4)) =
-                            make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
-                    fence_proxy_async_smem();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(&sh.dfull[buf]);
                 }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive(&sh.tempty[buf]);
+                mbar_arrive(&sh.sempty[ss]);
+            }
+            if (dzm) {
+                if (!mbar_wait_spin(&sh.dempty[set], ph ^ 1, abort, lim)) { ok = false; break; }
+                uint8_t *dt = sD + set * TR_D_BUF + row * 128;
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+                    *reinterpret_cast<uint4 *>(dt + (((4 * g + c) ^ (row & 7)) << 4)) =
+                        make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&sh.dfull[set]);
             }
         }
         if (!dzm) {
-            // merge the two id groups of each row, one partial per (split, row)
-            float4 *scr = reinterpret_cast<float4 *>(sD);
-            if (g == 1) scr[row] = make_float4(r0, r1, r2, r3);
+            // merge the four warps of each row (2 id groups x 2 sets), one
+            // partial per (split, row); the ring is free once every item is read
+            const float4 o4 = mode == TR_STATS ? make_float4(m2, s2, 0.f, 0.f)
+                                               : make_float4(r0[0] + r0[1], r1[0] + r1[1], 0.f, r3[0] + r3[1]);
             tr_epi_bar();
-            if (g == 0 && valid && ok && !*abort) {
-                const float4 o = scr[row];
-                if (mode == TR_STATS) lse2_merge(r0, r1, o.x, o.y);
-                else { r0 += o.x; r1 += o.y; r2 += o.z; r3 += o.w; }
-                p.part[(size_t)sv * p.NR + rowg] = make_float4(r0, r1, r2, r3);
+            float4 *scr = reinterpret_cast<float4 *>(sS);
+            const int slot = 2 * set + g;
+            if (slot != 0) scr[(slot - 1) * TR_BM + row] = o4;
+            tr_epi_bar();
+            if (slot == 0 && valid && ok && !*abort) {
+                float4 a = o4;
+                for (int k = 0; k < 3; ++k) {
+                    const float4 o = scr[k * TR_BM + row];
+                    if (mode == TR_STATS) lse2_merge(a.x, a.y, o.x, o.y);
+                    else { a.x += o.x; a.y += o.y; a.w += o.w; }
+                }
+                p.part[(size_t)sv * p.NR + rowg] = a;
             }
         } else if (ok && items > 0) {
-            if (mbar_wait(&sh.zdone, 0, abort, lim)) {
+            if (mbar_wait_spin(&sh.zdone, 0, abort, lim)) {
                 tc_fence_after();
+                // the 4 warps of a lane quarter take 64 of the 256 columns each
+                const int c0 = (2 * set + g) * 64;
 #pragma unroll 1
-                for (int c4 = 0; c4 < 4; ++c4) {
+                for (int c4 = 0; c4 < 2; ++c4) {
                     float v[32];
-                    tmem_ld32(tmem + lane_base + TR_DZ_COL + g * 128 + c4 * 32, v);
-                    float4 *dst = reinterpret_cast<float4 *>(p.dzp + ((size_t)sv * p.NR + rowg) * RANK + g * 128 +
-                                                             c4 * 32);
+                    tmem_ld32(tmem + lane_base + TR_DZ_COL + c0 + c4 * 32, v);
+                    float4 *dst =
+                        reinterpret_cast<float4 *>(p.dzp + ((size_t)sv * p.NR + rowg) * RANK + c0 + c4 * 32);
 #pragma unroll
                     for (int e = 0; e < 8; ++e)
                         dst[e] = valid ? make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3])
@@ -402,13 +533,14 @@ __global__ void __launch_bounds__(TR_THREADS, 1)
     if (threadIdx.x == 0 && sh.abort) set_status(p.status, ST_TIMEOUT);
 }
 
-
 // ---------------------------------------------------------------- k_train_voc
 namespace {
 
 constexpr int TV_BM = 128;                                 // vocabulary ids
 constexpr int TV_BN = 64;                                  // rows per step: 32 positions x 2 forwards
-constexpr int TV_EPI_WARPS = 8;                            // 2 per lane quarter: teacher / consistency half
+constexpr int TV_PF = 4;                                   // steps whose s / t are prefetched into L2 ahead
+constexpr int TV_EPI_WARPS = 16;                           // 2 sets (step parity) x 4 lane quarters x 2 row halves
+constexpr int TV_SET = TV_EPI_WARPS / 2;
 constexpr int TV_THREADS = 32 * (2 + TV_EPI_WARPS);
 constexpr uint32_t TV_W_CHUNK = TV_BM * 64 * 2;            // 16 KB: 128 ids x 64 of r
 constexpr uint32_t TV_W_BYTES = 4 * TV_W_CHUNK;            // 64 KB
@@ -416,8 +548,9 @@ constexpr uint32_t TV_Z_CHUNK = TV_BN * 64 * 2;            // 8 KB: 64 rows x 64
 constexpr uint32_t TV_Z_BYTES = 4 * TV_Z_CHUNK;            // 32 KB
 constexpr uint32_t TV_ST_BOX = 32 * 64 * 2;                // 4 KB: 32 positions x 64 ids
 constexpr uint32_t TV_ST_TILE = 2 * TV_ST_BOX;             // s (or t) of 32 positions x 128 ids
-constexpr uint32_t TV_INFO = TV_BN * sizeof(RowCoef);      // 2 KB
-constexpr uint32_t TV_STEP = TV_Z_BYTES + 2 * TV_ST_TILE + TV_INFO;   // one ring stage
+constexpr uint32_t TV_INFO = TV_BN * sizeof(RowCoef);      // 1 KB
+constexpr uint32_t TV_STEP = TV_Z_BYTES + 2 * TV_ST_TILE + TV_INFO;   // one ring stage (1024-byte aligned)
+static_assert(TV_STEP % 1024 == 0, "ring stages keep the 128-byte swizzle alignment");
 constexpr uint32_t TV_D_BUF = TV_BM * TV_BN * 2;           // 16 KB: dl^T tile (K-major over rows)
 constexpr uint32_t TV_IDESC_F = idesc_bf16(TV_BM, TV_BN);
 constexpr uint32_t TV_IDESC_D = idesc_bf16_mn(TV_BM, RANK, false, true);
@@ -464,10 +597,10 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
         mbar_init(&sh.a_empty, 1);
         for (int i = 0; i < 2; ++i) {
             mbar_init(&sh.zfull[i], 1);
-            mbar_init(&sh.zempty[i], 1 + TV_EPI_WARPS);    // the dW MMA's commit + every epilogue warp
+            mbar_init(&sh.zempty[i], 1 + TV_SET);          // the dW MMA's commit + the step's epilogue warps
             mbar_init(&sh.tfull[i], 1);
-            mbar_init(&sh.tempty[i], TV_EPI_WARPS);
-            mbar_init(&sh.dfull[i], TV_EPI_WARPS);
+            mbar_init(&sh.tempty[i], TV_SET);
+            mbar_init(&sh.dfull[i], TV_SET);
             mbar_init(&sh.dempty[i], 1);
         }
         mbar_init(&sh.wfull, 1);
@@ -477,6 +610,8 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
         fence_barrier_init();
     }
     if (warp == 1) { tmem_alloc(&sh.tmem_base, TV_TMEM_COLS); tmem_relinquish(); }
+    pdl_trigger();                 // the next kernel may start its set-up
+    pdl_wait();                    // Z and the coefficients are complete
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -493,6 +628,17 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
             tma_prefetch_desc(&tmap_t);
             const uint64_t once = policy_evict_first();
             const char *wr = static_cast<const char *>(p.W_r);
+            // the L2 prefetch cursor of s / t runs TV_PF steps ahead of the loads
+            int pf_vt = blockIdx.x, pf_u = 0;
+            auto advance_pf = [&]() {
+                if (pf_vt >= nvt) return;
+                for (int h2 = 0; h2 < 2; ++h2) {
+                    tma_prefetch_2d(&tmap_s, pf_vt * TV_BM + 64 * h2, 32 * pf_u);
+                    tma_prefetch_2d(&tmap_t, pf_vt * TV_BM + 64 * h2, 32 * pf_u);
+                }
+                if (++pf_u == nsteps) { pf_u = 0; pf_vt += gridDim.x; }
+            };
+            for (int k = 0; k < TV_PF; ++k) advance_pf();
             int gu = 0, lt = 0;
             uint32_t pend = 0, par = 0;
             bool pend_a = false;
@@ -502,14 +648,15 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
                 if (nx < nvt)
                     prefetch_l2_bulk(wr + (size_t)nx * TV_BM * RANK * 2,
                                      (uint32_t)min(TV_BM, p.V - nx * TV_BM) * RANK * 2);
-                if (!mbar_wait(&sh.a_empty, (uint32_t)((lt & 1) ^ 1), abort, lim)) break;
+                if (!mbar_wait_spin(&sh.a_empty, (uint32_t)((lt & 1) ^ 1), abort, lim)) break;
                 mbar_expect_tx(&sh.a_full, TV_W_BYTES);
                 for (int c = 0; c < 4; ++c) tma_load_2d(sW + c * TV_W_CHUNK, &tmap_w, &sh.a_full, c * 64, vt * TV_BM);
                 pend_a = true;
                 for (int u = 0; u < nsteps; ++u, ++gu) {
+                    advance_pf();
                     const int zs = gu & 1;
                     const uint32_t ph = (uint32_t)((gu >> 1) & 1);
-                    if (!mbar_wait(&sh.zempty[zs], ph ^ 1, abort, lim)) break;
+                    if (!mbar_wait_spin(&sh.zempty[zs], ph ^ 1, abort, lim)) break;
                     uint8_t *st = sR + zs * TV_STEP;
                     mbar_expect_tx(&sh.zfull[zs], TV_STEP);
                     const int jt = u >> 1, hh = u & 1;
@@ -533,9 +680,9 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
             }
             if (*abort) {
                 int dummy = 0;
-                if (pend_a) mbar_wait(&sh.a_full, (uint32_t)((lt - 1) & 1), &dummy, 100000000ull);
+                if (pend_a) mbar_wait_spin(&sh.a_full, (uint32_t)((lt - 1) & 1), &dummy, 100000000ull);
                 for (int zs = 0; zs < 2; ++zs)
-                    if (pend & (1u << zs)) mbar_wait(&sh.zfull[zs], (par >> zs) & 1, &dummy, 100000000ull);
+                    if (pend & (1u << zs)) mbar_wait_spin(&sh.zfull[zs], (par >> zs) & 1, &dummy, 100000000ull);
             }
         }
     } else if (warp == 1) {
@@ -548,8 +695,8 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
             // step's Z tile read MN-major (N = r along the 128-byte rows, K = rows)
             auto dw_step = [&](int v, bool first) -> bool {
                 const int db = v & 1;
-                if (!mbar_wait(&sh.dfull[db], (uint32_t)((v >> 1) & 1), abort, lim)) return false;
-                if (first && !mbar_wait(&sh.wempty, (uint32_t)((lt & 1) ^ 1), abort, lim)) return false;
+                if (!mbar_wait_spin(&sh.dfull[db], (uint32_t)((v >> 1) & 1), abort, lim)) return false;
+                if (first && !mbar_wait_spin(&sh.wempty, (uint32_t)((lt & 1) ^ 1), abort, lim)) return false;
                 tc_fence_after();
                 const uint32_t zb = r0 + (v & 1) * TV_STEP;
 #pragma unroll
@@ -561,12 +708,12 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
                 return true;
             };
             for (int vt = blockIdx.x; vt < nvt && ok; vt += gridDim.x, ++lt) {
-                if (!mbar_wait(&sh.a_full, (uint32_t)(lt & 1), abort, lim)) { ok = false; break; }
+                if (!mbar_wait_spin(&sh.a_full, (uint32_t)(lt & 1), abort, lim)) { ok = false; break; }
                 tc_fence_after();
                 for (int u = 0; u < nsteps; ++u, ++gu) {
                     const int zs = gu & 1, buf = gu & 1;
-                    if (!mbar_wait(&sh.zfull[zs], (uint32_t)((gu >> 1) & 1), abort, lim) ||
-                        !mbar_wait(&sh.tempty[buf], (uint32_t)(((gu >> 1) & 1) ^ 1), abort, lim)) {
+                    if (!mbar_wait_spin(&sh.zfull[zs], (uint32_t)((gu >> 1) & 1), abort, lim) ||
+                        !mbar_wait_spin(&sh.tempty[buf], (uint32_t)(((gu >> 1) & 1) ^ 1), abort, lim)) {
                         ok = false;
                         break;
                     }
@@ -592,53 +739,57 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
         }
     } else {
         // ------------------------------------------------------ epilogue
-        const int ew = warp - 2, q = warp & 3, g = ew >> 2;     // g: 0 teacher-forced rows, 1 consistency rows
+        // warp set `set` takes the steps of its parity; within a set, warp
+        // (q, g) the 32 ids of lane quarter q and the 32 rows of half g
+        // (0 teacher-forced, 1 consistency), in two halves of 16
+        const int ew = warp - 2, q = warp & 3, g = (ew >> 2) & 1, set = ew >> 3;
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
         const int vr = q * 32 + lane;                          // id row of the tile
         const int h2 = vr >> 6, cc = vr & 63;                  // s / t box and column within it
+        const int coff = (cc & 7) * 2;
         int gu = 0, lt = 0;
         bool ok = nsteps > 0;
         for (int vt = blockIdx.x; vt < nvt && ok; vt += gridDim.x, ++lt) {
             const int v = vt * TV_BM + vr;
             const bool vvalid = v < p.V;
             for (int u = 0; u < nsteps; ++u, ++gu) {
-                const int buf = gu & 1;
+                if ((gu & 1) != set) continue;
+                const int buf = set;
                 const uint32_t ph = (uint32_t)((gu >> 1) & 1);
-                if (!mbar_wait(&sh.tfull[buf], ph, abort, lim) || !mbar_wait(&sh.zfull[buf], ph, abort, lim)) {
+                if (!mbar_wait_spin(&sh.tfull[buf], ph, abort, lim) || !mbar_wait_spin(&sh.zfull[buf], ph, abort, lim)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                float acc[32];
-                tmem_ld32(tmem + lane_base + buf * TV_BN + g * 32, acc);
+                const uint8_t *st = sR + buf * TV_STEP;
+                const uint8_t *sbox = st + TV_Z_BYTES + h2 * TV_ST_BOX;
+                const float4 *info = reinterpret_cast<const float4 *>(st + TV_Z_BYTES + 2 * TV_ST_TILE) + g * 32;
+                uint32_t w[16];
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    float acc[16];
+                    tmem_ld16(tmem + lane_base + buf * TV_BN + g * 32 + h * 16, acc);
+#pragma unroll
+                    for (int c = 0; c < 16; c += 2) {
+                        float d2[2];
+#pragma unroll
+                        for (int e = 0; e < 2; ++e) {
+                            const int pr = 16 * h + c + e;     // position within the step
+                            const int off = pr * 128 + (((cc >> 3) ^ (pr & 7)) << 4) + coff;
+                            const float sv = bf2f(*reinterpret_cast<const uint16_t *>(sbox + off));
+                            const float tv = bf2f(*reinterpret_cast<const uint16_t *>(sbox + TV_ST_TILE + off));
+                            const float4 rc = info[pr];      // lse_p2, lse_q2, Apos, Aneg
+                            const float a2 = fmaf(acc[c + e] + sv, L2E, -rc.x);
+                            const float b2 = fmaf(tv, L2E, -rc.y);
+                            d2[e] = vvalid ? dl_value(a2, b2, rc.z, rc.w) : 0.f;
+                        }
+                        w[8 * h + c / 2] = pack_bf16x2(d2[0], d2[1]);
+                    }
+                }
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&sh.tempty[buf]);
-                const uint8_t *st = sR + buf * TV_STEP;
-                const uint8_t *sbox = st + TV_Z_BYTES + h2 * TV_ST_BOX;
-                const RowCoef *info = reinterpret_cast<const RowCoef *>(st + TV_Z_BYTES + 2 * TV_ST_TILE) + g * 32;
-                const int coff = (cc & 7) * 2;
-                uint32_t w[16];
-#pragma unroll
-                for (int c = 0; c < 32; c += 2) {
-                    float d2[2];
-#pragma unroll
-                    for (int e = 0; e < 2; ++e) {
-                        const int pr = c + e;                  // position within the step
-                        const int off = pr * 128 + (((cc >> 3) ^ (pr & 7)) << 4) + coff;
-                        const float sv = bf2f(*reinterpret_cast<const uint16_t *>(sbox + off));
-                        const float tv = bf2f(*reinterpret_cast<const uint16_t *>(sbox + TV_ST_TILE + off));
-                        const RowCoef rc = info[pr];
-                        const float a2 = fmaf(acc[pr] + sv, L2E, -rc.lse_p2);
-                        const float b2 = fmaf(tv, L2E, -rc.lse_q2);
-                        const float pv = ex2_approx(a2);
-                        const float sg = a2 > b2 ? 1.f : (a2 < b2 ? -1.f : 0.f);
-                        const float d = pv * fmaf(rc.A1, sg, rc.A0) - (v == rc.y ? rc.A2 : 0.f);
-                        d2[e] = vvalid ? d : 0.f;
-                    }
-                    w[c / 2] = pack_bf16x2(d2[0], d2[1]);
-                }
-                if (!mbar_wait(&sh.dempty[buf], ph ^ 1, abort, lim)) { ok = false; break; }
+                if (!mbar_wait_spin(&sh.dempty[buf], ph ^ 1, abort, lim)) { ok = false; break; }
                 uint8_t *dt = sD + buf * TV_D_BUF + vr * 128;
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
@@ -652,15 +803,17 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
                 }
             }
             if (!ok) break;
-            // this tile's dW_r rows: add into gW_r, then hand the accumulator back
-            if (!mbar_wait(&sh.wfull, (uint32_t)(lt & 1), abort, lim)) { ok = false; break; }
+            // this tile's dW_r rows: add into gW_r (the 4 warps of a lane
+            // quarter take 64 columns each), then hand the accumulator back
+            if (!mbar_wait_spin(&sh.wfull, (uint32_t)(lt & 1), abort, lim)) { ok = false; break; }
             tc_fence_after();
+            const int c0 = (2 * set + g) * 64;
 #pragma unroll 1
-            for (int c4 = 0; c4 < 4; ++c4) {
+            for (int c4 = 0; c4 < 2; ++c4) {
                 float wv[32];
-                tmem_ld32(tmem + lane_base + TV_DW_COL + g * 128 + c4 * 32, wv);
+                tmem_ld32(tmem + lane_base + TV_DW_COL + c0 + c4 * 32, wv);
                 if (vvalid) {
-                    float4 *dst = reinterpret_cast<float4 *>(p.gW_r + (size_t)v * RANK + g * 128 + c4 * 32);
+                    float4 *dst = reinterpret_cast<float4 *>(p.gW_r + (size_t)v * RANK + c0 + c4 * 32);
 #pragma unroll
                     for (int e = 0; e < 8; ++e) {
                         float4 o = dst[e];
