@@ -14,7 +14,7 @@
 //
 // Roles (192 threads): warp 0 TMA producer, warp 1 TMEM allocator and MMA
 // issuer, warps 2-5 epilogue (one TMEM lane quarter each, 32 rows).
-#include "common.cuh"
+#include "train_common.cuh"
 #include "kernels.h"
 
 namespace xp {

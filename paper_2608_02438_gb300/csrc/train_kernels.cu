@@ -22,7 +22,7 @@
 //   k_train_mix_bwd       dL/da_j = dc_j + sum_{k>j} L_kj dc_k and dL/dL_kj
 //   k_train_fuse_bwd      dL/du_h per position (both forwards), dL/du_g / B
 //                         per block, dL/dW_e rows (atomic, both forwards)
-#include "common.cuh"
+#include "train_common.cuh"
 #include "kernels.h"
 
 namespace xp {

@@ -31,7 +31,7 @@
 // few tiles ahead (tensor-map prefetch) so that the TMA loads of the rings
 // hit L2.  The -A2 [v = y*] term of dL/dl and l at y* are left to the small
 // kernels (k_train_dz, k_train_stats_fin), so the loops here carry no id test.
-#include "common.cuh"
+#include "train_common.cuh"
 #include "kernels.h"
 
 namespace xp {
