@@ -96,27 +96,6 @@ __device__ __forceinline__ void tr_epi_bar()
     asm volatile("bar.sync 1, %0;" ::"n"(TR_EPI_WARPS * 32) : "memory");
 }
 
-// 32 consecutive bf16 of row `pr` of a 64-wide SW128 tile (chunks 4h .. 4h+3)
-__device__ __forceinline__ void ld_tile32(const uint8_t *tile, int pr, int h, uint4 (&r)[4])
-{
-#pragma unroll
-    for (int c = 0; c < 4; ++c)
-        r[c] = *reinterpret_cast<const uint4 *>(tile + pr * 128 + (((4 * h + c) ^ (pr & 7)) << 4));
-}
-
-__device__ __forceinline__ void unpack32(const uint4 (&r)[4], float (&x)[32])
-{
-#pragma unroll
-    for (int c = 0; c < 4; ++c) {
-        const uint32_t w[4] = {r[c].x, r[c].y, r[c].z, r[c].w};
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            x[8 * c + 2 * q] = __uint_as_float(w[q] << 16);
-            x[8 * c + 2 * q + 1] = __uint_as_float(w[q] & 0xFFFF0000u);
-        }
-    }
-}
-
 // log2-domain running log-sum-exp over 16 values: value = s * 2^m.  The max
 // and the sum run as trees (short dependent chains).
 __device__ __forceinline__ void lse2_add16(float &m, float &s, const float (&x)[16])
@@ -542,24 +521,28 @@ constexpr int TV_PF = 4;                                   // steps whose s / t 
 constexpr int TV_EPI_WARPS = 16;                           // 2 sets (step parity) x 4 lane quarters x 2 row halves
 constexpr int TV_SET = TV_EPI_WARPS / 2;
 constexpr int TV_THREADS = 32 * (2 + TV_EPI_WARPS);
-constexpr uint32_t TV_W_CHUNK = TV_BM * 64 * 2;            // 16 KB: 128 ids x 64 of r
-constexpr uint32_t TV_W_BYTES = 4 * TV_W_CHUNK;            // 64 KB
+constexpr int TV_ZS = 4;                                   // Z ring (freed by the step's dW MMA)
+constexpr int TV_SS = 3;                                   // s / t / coefficient ring (freed by the epilogue)
 constexpr uint32_t TV_Z_CHUNK = TV_BN * 64 * 2;            // 8 KB: 64 rows x 64 of r
 constexpr uint32_t TV_Z_BYTES = 4 * TV_Z_CHUNK;            // 32 KB
 constexpr uint32_t TV_ST_BOX = 32 * 64 * 2;                // 4 KB: 32 positions x 64 ids
 constexpr uint32_t TV_ST_TILE = 2 * TV_ST_BOX;             // s (or t) of 32 positions x 128 ids
 constexpr uint32_t TV_INFO = TV_BN * sizeof(RowCoef);      // 1 KB
-constexpr uint32_t TV_STEP = TV_Z_BYTES + 2 * TV_ST_TILE + TV_INFO;   // one ring stage (1024-byte aligned)
-static_assert(TV_STEP % 1024 == 0, "ring stages keep the 128-byte swizzle alignment");
+constexpr uint32_t TV_S_STAGE = 2 * TV_ST_TILE + 1024;     // s, t, row coefficients (1024-byte aligned)
 constexpr uint32_t TV_D_BUF = TV_BM * TV_BN * 2;           // 16 KB: dl^T tile (K-major over rows)
 constexpr uint32_t TV_IDESC_F = idesc_bf16(TV_BM, TV_BN);
 constexpr uint32_t TV_IDESC_D = idesc_bf16_mn(TV_BM, RANK, false, true);
-constexpr uint32_t TV_TMEM_COLS = 512;                     // l^T: 2 x 64 at 0; dW_r: 256 at 256
+// TMEM: l^T accumulators 2 x 64 from 0, the W_r tile (A operand: 128 ids x
+// 256 bf16, two per column) at 128, dW_r (256) at 256
+constexpr uint32_t TV_TMEM_COLS = 512;
+constexpr uint32_t TV_WR_COL = 128;
 constexpr uint32_t TV_DW_COL = 256;
+static_assert(TV_INFO <= 1024, "row coefficients of a step");
 
 struct TvShared {
-    uint64_t a_full, a_empty;
-    uint64_t zfull[2], zempty[2];
+    uint64_t a_full, a_empty;                  // the W_r tile in TMEM: written (16 warps), read by the last F
+    uint64_t zfull[TV_ZS], zempty[TV_ZS];
+    uint64_t sfull[TV_SS], sempty[TV_SS];
     uint64_t tfull[2], tempty[2];
     uint64_t dfull[2], dempty[2];
     uint64_t wfull, wempty, drain;
@@ -567,7 +550,8 @@ struct TvShared {
     int abort;
 };
 
-constexpr size_t TV_SMEM = 1024 + TV_W_BYTES + 2 * TV_STEP + 2 * TV_D_BUF + sizeof(TvShared);
+constexpr size_t TV_SMEM = 1024 + TV_ZS * TV_Z_BYTES + TV_SS * TV_S_STAGE + 2 * TV_D_BUF + sizeof(TvShared);
+static_assert(TV_SMEM <= 232448, "k_train_voc shared memory");
 
 }  // namespace
 
@@ -575,8 +559,9 @@ const size_t kTrainVocSmemBytes = TV_SMEM;
 const int kTrainVocThreads = TV_THREADS;
 
 // grid min(SMs, ceil(V / 128)) (persistent over vocabulary tiles), TV_THREADS
-// threads, TV_SMEM bytes.  tmap_w: W_r boxes of 128 rows; tmap_z: Z boxes of 32
-// rows; tmap_s / tmap_t: boxes of 64 ids x 32 positions.
+// threads, TV_SMEM bytes.  tmap_z: Z boxes of 32 rows; tmap_s / tmap_t: boxes
+// of 64 ids x 32 positions.  tmap_w is not read (the W_r tile goes to tensor
+// memory from p.W_r).
 __global__ void __launch_bounds__(TV_THREADS, 1)
     k_train_voc(const __grid_constant__ TrainParams p, const __grid_constant__ CUtensorMap tmap_z,
                 const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_s,
@@ -584,20 +569,26 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t *sW = base;
-    uint8_t *sR = sW + TV_W_BYTES;                 // step ring: Z, s, t, row coefficients
-    uint8_t *sD = sR + 2 * TV_STEP;
+    uint8_t *sZ = base;                            // Z ring
+    uint8_t *sS = sZ + TV_ZS * TV_Z_BYTES;         // s / t / coefficient ring
+    uint8_t *sD = sS + TV_SS * TV_S_STAGE;         // dl^T tiles, one per warp set
     TvShared &sh = *reinterpret_cast<TvShared *>(sD + 2 * TV_D_BUF);
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const int nvt = (p.V + TV_BM - 1) / TV_BM;
     const int nsteps = (p.P + 31) / 32;
 
     if (threadIdx.x == 0) {
-        mbar_init(&sh.a_full, 1);
+        mbar_init(&sh.a_full, TV_EPI_WARPS);
         mbar_init(&sh.a_empty, 1);
-        for (int i = 0; i < 2; ++i) {
+        for (int i = 0; i < TV_ZS; ++i) {
             mbar_init(&sh.zfull[i], 1);
-            mbar_init(&sh.zempty[i], 1 + TV_SET);          // the dW MMA's commit + the step's epilogue warps
+            mbar_init(&sh.zempty[i], 1);               // the step's dW MMA
+        }
+        for (int i = 0; i < TV_SS; ++i) {
+            mbar_init(&sh.sfull[i], 1);
+            mbar_init(&sh.sempty[i], TV_SET);          // the step's epilogue warps
+        }
+        for (int i = 0; i < 2; ++i) {
             mbar_init(&sh.tfull[i], 1);
             mbar_init(&sh.tempty[i], TV_SET);
             mbar_init(&sh.dfull[i], TV_SET);
@@ -623,11 +614,14 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
         // ------------------------------------------------------- producer
         if (lane == 0 && nsteps > 0) {
             tma_prefetch_desc(&tmap_z);
-            tma_prefetch_desc(&tmap_w);
             tma_prefetch_desc(&tmap_s);
             tma_prefetch_desc(&tmap_t);
             const uint64_t once = policy_evict_first();
             const char *wr = static_cast<const char *>(p.W_r);
+            auto prefetch_wr = [&](int vt) {      // a W_r tile into L2 (the epilogue loads it into TMEM)
+                if (vt < nvt)
+                    prefetch_l2_bulk(wr + (size_t)vt * TV_BM * RANK * 2, (uint32_t)min(TV_BM, p.V - vt * TV_BM) * RANK * 2);
+            };
             // the L2 prefetch cursor of s / t runs TV_PF steps ahead of the loads
             int pf_vt = blockIdx.x, pf_u = 0;
             auto advance_pf = [&]() {
@@ -638,100 +632,128 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
                 }
                 if (++pf_u == nsteps) { pf_u = 0; pf_vt += gridDim.x; }
             };
+            prefetch_wr(blockIdx.x);
             for (int k = 0; k < TV_PF; ++k) advance_pf();
-            int gu = 0, lt = 0;
-            uint32_t pend = 0, par = 0;
-            bool pend_a = false;
-            for (int vt = blockIdx.x; vt < nvt && !*abort; vt += gridDim.x, ++lt) {
-                // the next tile's W_r rows go to L2 while this one is consumed
-                const int nx = vt + gridDim.x;
-                if (nx < nvt)
-                    prefetch_l2_bulk(wr + (size_t)nx * TV_BM * RANK * 2,
-                                     (uint32_t)min(TV_BM, p.V - nx * TV_BM) * RANK * 2);
-                if (!mbar_wait_spin(&sh.a_empty, (uint32_t)((lt & 1) ^ 1), abort, lim)) break;
-                mbar_expect_tx(&sh.a_full, TV_W_BYTES);
-                for (int c = 0; c < 4; ++c) tma_load_2d(sW + c * TV_W_CHUNK, &tmap_w, &sh.a_full, c * 64, vt * TV_BM);
-                pend_a = true;
-                for (int u = 0; u < nsteps; ++u, ++gu) {
+            int gu = 0;
+            uint32_t pend_z = 0, par_z = 0, pend_s = 0, par_s = 0;
+            const char *gw = reinterpret_cast<const char *>(p.gW_r);
+            for (int vt = blockIdx.x; vt < nvt && !*abort; vt += gridDim.x) {
+                prefetch_wr(vt + gridDim.x);
+                for (int u = 0; u < nsteps && !*abort; ++u, ++gu) {
                     advance_pf();
-                    const int zs = gu & 1;
-                    const uint32_t ph = (uint32_t)((gu >> 1) & 1);
-                    if (!mbar_wait_spin(&sh.zempty[zs], ph ^ 1, abort, lim)) break;
-                    uint8_t *st = sR + zs * TV_STEP;
-                    mbar_expect_tx(&sh.zfull[zs], TV_STEP);
+                    if (u == max(0, nsteps - 4)) {
+                        // this tile's gW_r rows (fp32, added into at the tile's end)
+                        // into L2, a few steps before the drain needs them
+                        const uint32_t rows = (uint32_t)min(TV_BM, p.V - vt * TV_BM);
+                        for (uint32_t r0 = 0; r0 < rows; r0 += 32)
+                            prefetch_l2_bulk(gw + ((size_t)vt * TV_BM + r0) * RANK * 4,
+                                             min(32u, rows - r0) * RANK * 4);
+                    }
                     const int jt = u >> 1, hh = u & 1;
                     const int rt = jt * 128 + 32 * hh;               // teacher-forced rows of the step
+                    const int zs = gu % TV_ZS;
+                    const uint32_t zph = (uint32_t)((gu / TV_ZS) & 1);
+                    if (!mbar_wait_spin(&sh.zempty[zs], zph ^ 1, abort, lim)) break;
+                    uint8_t *zt = sZ + zs * TV_Z_BYTES;
+                    mbar_expect_tx(&sh.zfull[zs], TV_Z_BYTES);
                     for (int c = 0; c < 4; ++c) {
-                        tma_load_2d(st + c * TV_Z_CHUNK, &tmap_z, &sh.zfull[zs], c * 64, rt);
-                        tma_load_2d(st + c * TV_Z_CHUNK + 4096, &tmap_z, &sh.zfull[zs], c * 64, rt + 64);
+                        tma_load_2d(zt + c * TV_Z_CHUNK, &tmap_z, &sh.zfull[zs], c * 64, rt);
+                        tma_load_2d(zt + c * TV_Z_CHUNK + 4096, &tmap_z, &sh.zfull[zs], c * 64, rt + 64);
                     }
+                    pend_z |= 1u << zs;
+                    par_z = (par_z & ~(1u << zs)) | (zph << zs);
+                    const int ss = gu % TV_SS;
+                    const uint32_t sph = (uint32_t)((gu / TV_SS) & 1);
+                    if (!mbar_wait_spin(&sh.sempty[ss], sph ^ 1, abort, lim)) break;
+                    uint8_t *stg = sS + ss * TV_S_STAGE;
+                    mbar_expect_tx(&sh.sfull[ss], 2 * TV_ST_TILE + TV_INFO);
                     for (int h2 = 0; h2 < 2; ++h2) {
-                        tma_load_2d_hint(st + TV_Z_BYTES + h2 * TV_ST_BOX, &tmap_s, &sh.zfull[zs],
-                                         vt * TV_BM + 64 * h2, 32 * u, once);
-                        tma_load_2d_hint(st + TV_Z_BYTES + TV_ST_TILE + h2 * TV_ST_BOX, &tmap_t, &sh.zfull[zs],
-                                         vt * TV_BM + 64 * h2, 32 * u, once);
+                        tma_load_2d_hint(stg + h2 * TV_ST_BOX, &tmap_s, &sh.sfull[ss], vt * TV_BM + 64 * h2, 32 * u, once);
+                        tma_load_2d_hint(stg + TV_ST_TILE + h2 * TV_ST_BOX, &tmap_t, &sh.sfull[ss], vt * TV_BM + 64 * h2,
+                                         32 * u, once);
                     }
-                    uint8_t *info = st + TV_Z_BYTES + 2 * TV_ST_TILE;
-                    bulk_load_1d(info, p.coef + rt, 32 * sizeof(RowCoef), &sh.zfull[zs]);
-                    bulk_load_1d(info + 32 * sizeof(RowCoef), p.coef + rt + 64, 32 * sizeof(RowCoef), &sh.zfull[zs]);
-                    pend |= 1u << zs;
-                    par = (par & ~(1u << zs)) | (ph << zs);
+                    uint8_t *info = stg + 2 * TV_ST_TILE;
+                    bulk_load_1d(info, p.coef + rt, 32 * sizeof(RowCoef), &sh.sfull[ss]);
+                    bulk_load_1d(info + 32 * sizeof(RowCoef), p.coef + rt + 64, 32 * sizeof(RowCoef), &sh.sfull[ss]);
+                    pend_s |= 1u << ss;
+                    par_s = (par_s & ~(1u << ss)) | (sph << ss);
                 }
             }
             if (*abort) {
+                // no copy may still be landing when the CTA leaves
                 int dummy = 0;
-                if (pend_a) mbar_wait_spin(&sh.a_full, (uint32_t)((lt - 1) & 1), &dummy, 100000000ull);
-                for (int zs = 0; zs < 2; ++zs)
-                    if (pend & (1u << zs)) mbar_wait_spin(&sh.zfull[zs], (par >> zs) & 1, &dummy, 100000000ull);
+                for (int k = 0; k < TV_ZS; ++k)
+                    if (pend_z & (1u << k)) mbar_wait_spin(&sh.zfull[k], (par_z >> k) & 1, &dummy, 100000000ull);
+                for (int k = 0; k < TV_SS; ++k)
+                    if (pend_s & (1u << k)) mbar_wait_spin(&sh.sfull[k], (par_s >> k) & 1, &dummy, 100000000ull);
             }
         }
     } else if (warp == 1) {
         // ---------------------------------------------------- MMA issuer
+        // Issues, in order, the l^T products F(k) and the dW_r products D(k)
+        // of the CTA's steps k = tile * nsteps + u, whichever is ready first:
+        // F(k) needs Z(k) landed, accumulator k % 2 handed back and (first
+        // step of a tile) the tile's W_r rows in TMEM; D(k) needs the dl^T
+        // tile of step k and (first step of a tile) the previous tile's dW_r
+        // drained.  F runs ahead of D while the epilogue works.
         if (lane == 0 && nsteps > 0) {
-            const uint32_t w0 = smem_u32(sW), r0 = smem_u32(sR), d0 = smem_u32(sD);
-            int gu = 0, lt = 0;
+            const uint32_t z0 = smem_u32(sZ), d0 = smem_u32(sD);
+            const int ntiles = ((int)blockIdx.x < nvt) ? (nvt - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+            const int total = ntiles * nsteps;
+            int kf = 0, kd = 0;
             bool ok = true;
-            // dW_r += dl^T(v) Z(v): A = the dl^T tile (K-major over rows), B = the
-            // step's Z tile read MN-major (N = r along the 128-byte rows, K = rows)
-            auto dw_step = [&](int v, bool first) -> bool {
-                const int db = v & 1;
-                if (!mbar_wait_spin(&sh.dfull[db], (uint32_t)((v >> 1) & 1), abort, lim)) return false;
-                if (first && !mbar_wait_spin(&sh.wempty, (uint32_t)((lt & 1) ^ 1), abort, lim)) return false;
-                tc_fence_after();
-                const uint32_t zb = r0 + (v & 1) * TV_STEP;
+            unsigned long long stall0 = 0;          // when the current stall began (bounded by wait_ns)
+            uint32_t spins = 0;
+            while (kd < total && ok) {
+                bool progressed = false;
+                if (kf < total) {
+                    const int lt = kf / nsteps, u = kf - lt * nsteps;
+                    const int zs = kf % TV_ZS, buf = kf & 1;
+                    if ((u != 0 || mbar_try_wait(&sh.a_full, (uint32_t)(lt & 1))) &&
+                        mbar_try_wait(&sh.zfull[zs], (uint32_t)((kf / TV_ZS) & 1)) &&
+                        mbar_try_wait(&sh.tempty[buf], (uint32_t)(((kf >> 1) & 1) ^ 1))) {
+                        tc_fence_after();
+                        const uint32_t zb = z0 + zs * TV_Z_BYTES;
 #pragma unroll
-                for (int kk = 0; kk < TV_BN / 16; ++kk)
-                    tc_mma_bf16(tmem + TV_DW_COL, smem_desc_sw128(d0 + db * TV_D_BUF + kk * 32),
-                                smem_desc_sw128_mn(zb + kk * 2048, TV_Z_CHUNK), TV_IDESC_D, !(first && kk == 0));
-                tc_commit(&sh.zempty[v & 1]);
-                tc_commit(&sh.dempty[db]);
-                return true;
-            };
-            for (int vt = blockIdx.x; vt < nvt && ok; vt += gridDim.x, ++lt) {
-                if (!mbar_wait_spin(&sh.a_full, (uint32_t)(lt & 1), abort, lim)) { ok = false; break; }
-                tc_fence_after();
-                for (int u = 0; u < nsteps; ++u, ++gu) {
-                    const int zs = gu & 1, buf = gu & 1;
-                    if (!mbar_wait_spin(&sh.zfull[zs], (uint32_t)((gu >> 1) & 1), abort, lim) ||
-                        !mbar_wait_spin(&sh.tempty[buf], (uint32_t)(((gu >> 1) & 1) ^ 1), abort, lim)) {
-                        ok = false;
-                        break;
+                        for (int c = 0; c < 4; ++c)
+#pragma unroll
+                            for (int kk = 0; kk < 4; ++kk)
+                                tc_mma_bf16_ts(tmem + buf * TV_BN, tmem + TV_WR_COL + c * 32 + kk * 8,
+                                               smem_desc_sw128(zb + c * TV_Z_CHUNK + kk * 32), TV_IDESC_F,
+                                               (c | kk) != 0);
+                        tc_commit(&sh.tfull[buf]);
+                        if (u == nsteps - 1) tc_commit(&sh.a_empty);
+                        ++kf;
+                        progressed = true;
                     }
-                    tc_fence_after();
-                    const uint32_t zb = r0 + zs * TV_STEP;
-#pragma unroll
-                    for (int c = 0; c < 4; ++c)
-#pragma unroll
-                        for (int kk = 0; kk < 4; ++kk)
-                            tc_mma_bf16(tmem + buf * TV_BN, smem_desc_sw128(w0 + c * TV_W_CHUNK + kk * 32),
-                                        smem_desc_sw128(zb + c * TV_Z_CHUNK + kk * 32), TV_IDESC_F, (c | kk) != 0);
-                    tc_commit(&sh.tfull[buf]);
-                    if (u == nsteps - 1) tc_commit(&sh.a_empty);
-                    if (u > 0 && !dw_step(gu - 1, u == 1)) { ok = false; break; }
                 }
-                if (!ok) break;
-                if (!dw_step(gu - 1, nsteps == 1)) { ok = false; break; }
-                tc_commit(&sh.wfull);
+                if (kd < kf) {
+                    const int lt = kd / nsteps, u = kd - lt * nsteps;
+                    const int db = kd & 1;
+                    if (mbar_try_wait(&sh.dfull[db], (uint32_t)((kd >> 1) & 1)) &&
+                        (u != 0 || mbar_try_wait(&sh.wempty, (uint32_t)((lt & 1) ^ 1)))) {
+                        tc_fence_after();
+                        const uint32_t zb = z0 + (kd % TV_ZS) * TV_Z_BYTES;
+#pragma unroll
+                        for (int kk = 0; kk < TV_BN / 16; ++kk)
+                            tc_mma_bf16(tmem + TV_DW_COL, smem_desc_sw128(d0 + db * TV_D_BUF + kk * 32),
+                                        smem_desc_sw128_mn(zb + kk * 2048, TV_Z_CHUNK), TV_IDESC_D,
+                                        !(u == 0 && kk == 0));
+                        tc_commit(&sh.zempty[kd % TV_ZS]);
+                        tc_commit(&sh.dempty[db]);
+                        if (u == nsteps - 1) tc_commit(&sh.wfull);
+                        ++kd;
+                        progressed = true;
+                    }
+                }
+                if (progressed) {
+                    spins = 0;
+                } else if ((++spins & 63u) == 0) {
+                    const unsigned long long now = globaltimer();
+                    if (spins == 64) stall0 = now;
+                    if (*abort) ok = false;
+                    else if (now - stall0 > lim) { *abort = 1; ok = false; }
+                }
             }
             tc_commit(&sh.drain);
             int dummy = 0;
@@ -741,29 +763,88 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
         // ------------------------------------------------------ epilogue
         // warp set `set` takes the steps of its parity; within a set, warp
         // (q, g) the 32 ids of lane quarter q and the 32 rows of half g
-        // (0 teacher-forced, 1 consistency), in two halves of 16
+        // (0 teacher-forced, 1 consistency), in two halves of 16.  At each
+        // vocabulary tile every warp first stores its part of the tile's W_r
+        // rows into TMEM (K block 2 set + g), then drains the previous tile's
+        // dW_r (64 columns each) while the MMA starts on the new tile.
         const int ew = warp - 2, q = warp & 3, g = (ew >> 2) & 1, set = ew >> 3;
+        const int cb = 2 * set + g;
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
         const int vr = q * 32 + lane;                          // id row of the tile
         const int h2 = vr >> 6, cc = vr & 63;                  // s / t box and column within it
         const int coff = (cc & 7) * 2;
         int gu = 0, lt = 0;
         bool ok = nsteps > 0;
+        // adds the dW_r rows of tile `pvt` (the lt'-th of this CTA) into gW_r
+        auto drain = [&](int pvt, int plt) -> bool {
+            if (!mbar_wait_spin(&sh.wfull, (uint32_t)(plt & 1), abort, lim)) return false;
+            tc_fence_after();
+            const int pv = pvt * TV_BM + vr;
+#pragma unroll 1
+            for (int c4 = 0; c4 < 4; ++c4) {
+                float4 *dst = reinterpret_cast<float4 *>(p.gW_r + (size_t)pv * RANK + 64 * cb + 16 * c4);
+                float4 o[4];
+                if (pv < p.V) {
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) o[e] = dst[e];   // loads in flight before the TMEM read
+                }
+                float wv[16];
+                tmem_ld16(tmem + lane_base + TV_DW_COL + 64 * cb + c4 * 16, wv);
+                if (pv < p.V) {
+#pragma unroll
+                    for (int e = 0; e < 4; ++e)
+                        dst[e] = make_float4(o[e].x + wv[4 * e], o[e].y + wv[4 * e + 1], o[e].z + wv[4 * e + 2],
+                                             o[e].w + wv[4 * e + 3]);
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sh.wempty);
+            return true;
+        };
         for (int vt = blockIdx.x; vt < nvt && ok; vt += gridDim.x, ++lt) {
             const int v = vt * TV_BM + vr;
             const bool vvalid = v < p.V;
+            // this tile's W_r rows into TMEM, once the previous tile's last F is done
+            if (!mbar_wait_spin(&sh.a_empty, (uint32_t)((lt & 1) ^ 1), abort, lim)) { ok = false; break; }
+            {
+                uint32_t wrw[32];
+                if (vvalid) {
+                    const uint4 *src = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.W_r) +
+                                                                       (size_t)v * RANK + 64 * cb);
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        const uint4 x = src[c];
+                        wrw[4 * c] = x.x;
+                        wrw[4 * c + 1] = x.y;
+                        wrw[4 * c + 2] = x.z;
+                        wrw[4 * c + 3] = x.w;
+                    }
+                } else {
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) wrw[c] = 0u;
+                }
+                tc_fence_after();
+                tmem_st32(tmem + lane_base + TV_WR_COL + 32 * cb, wrw);
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&sh.a_full);
+            }
+            if (lt > 0 && !drain(vt - (int)gridDim.x, lt - 1)) { ok = false; break; }
             for (int u = 0; u < nsteps; ++u, ++gu) {
                 if ((gu & 1) != set) continue;
                 const int buf = set;
                 const uint32_t ph = (uint32_t)((gu >> 1) & 1);
-                if (!mbar_wait_spin(&sh.tfull[buf], ph, abort, lim) || !mbar_wait_spin(&sh.zfull[buf], ph, abort, lim)) {
+                const int ss = gu % TV_SS;
+                if (!mbar_wait_spin(&sh.tfull[buf], ph, abort, lim) ||
+                    !mbar_wait_spin(&sh.sfull[ss], (uint32_t)((gu / TV_SS) & 1), abort, lim)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const uint8_t *st = sR + buf * TV_STEP;
-                const uint8_t *sbox = st + TV_Z_BYTES + h2 * TV_ST_BOX;
-                const float4 *info = reinterpret_cast<const float4 *>(st + TV_Z_BYTES + 2 * TV_ST_TILE) + g * 32;
+                const uint8_t *stg = sS + ss * TV_S_STAGE;
+                const uint8_t *sbox = stg + h2 * TV_ST_BOX;
+                const float4 *info = reinterpret_cast<const float4 *>(stg + 2 * TV_ST_TILE) + g * 32;
                 uint32_t w[16];
 #pragma unroll
                 for (int h = 0; h < 2; ++h) {
@@ -788,7 +869,10 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
                 }
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&sh.tempty[buf]);
+                if (lane == 0) {
+                    mbar_arrive(&sh.tempty[buf]);
+                    mbar_arrive(&sh.sempty[ss]);
+                }
                 if (!mbar_wait_spin(&sh.dempty[buf], ph ^ 1, abort, lim)) { ok = false; break; }
                 uint8_t *dt = sD + buf * TV_D_BUF + vr * 128;
 #pragma unroll
@@ -797,38 +881,11 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
                         make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
                 fence_proxy_async_smem();
                 __syncwarp();
-                if (lane == 0) {
-                    mbar_arrive(&sh.dfull[buf]);
-                    mbar_arrive(&sh.zempty[buf]);
-                }
+                if (lane == 0) mbar_arrive(&sh.dfull[buf]);
             }
-            if (!ok) break;
-            // this tile's dW_r rows: add into gW_r (the 4 warps of a lane
-            // quarter take 64 columns each), then hand the accumulator back
-            if (!mbar_wait_spin(&sh.wfull, (uint32_t)(lt & 1), abort, lim)) { ok = false; break; }
-            tc_fence_after();
-            const int c0 = (2 * set + g) * 64;
-#pragma unroll 1
-            for (int c4 = 0; c4 < 2; ++c4) {
-                float wv[32];
-                tmem_ld32(tmem + lane_base + TV_DW_COL + c0 + c4 * 32, wv);
-                if (vvalid) {
-                    float4 *dst = reinterpret_cast<float4 *>(p.gW_r + (size_t)v * RANK + c0 + c4 * 32);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        float4 o = dst[e];
-                        o.x += wv[4 * e];
-                        o.y += wv[4 * e + 1];
-                        o.z += wv[4 * e + 2];
-                        o.w += wv[4 * e + 3];
-                        dst[e] = o;
-                    }
-                }
-            }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&sh.wempty);
         }
+        // the last tile's dW_r
+        if (ok && lt > 0) drain(blockIdx.x + (lt - 1) * (int)gridDim.x, lt - 1);
     }
     tc_fence_before();
     __syncthreads();
