@@ -50,7 +50,8 @@ SMALL_SUMMARY = "profiles/k_refine_small_qwen3_8b_greedy.txt"
 READ_SOURCES = [CSRC + "read_tc.cu", CSRC + "common.cuh"]
 READ_SUMMARIES = {"long_b64": "profiles/k_read_tc_long_b64.txt"}
 LM_SOURCES = [CSRC + "lm_head.cu", CSRC + "common.cuh"]
-TRAIN_SOURCES = [CSRC + f for f in ("train_read.cu", "kernels.h", "common.cuh")]
+TRAIN_SOURCES = [CSRC + f for f in ("train_read.cu", "train_common.cuh", "kernels.h", "common.cuh")]
+TRAIN_SUMMARIES = {"dz": "profiles/k_train_tok_dz_qwen3_8b_train.txt", "dW_r": "profiles/k_train_voc_qwen3_8b_train.txt"}
 LM_SUMMARIES = {16: "profiles/k_lm_head32_qwen3_8b_n16.txt"}
 
 
@@ -337,6 +338,12 @@ def train_measure(torch, X, W, ref, dev, timed_us, hbm, tc_peak, d=None, cfg=Non
               ("dW_r", "k_train_voc", 2 * f1, wr + 2 * st + NR * r * 2 + 2 * V * r * 4)]
     lines = [train_pass_line(n, k, timed_us(lambda i=i: call(i)), f, nb, hbm, tc_peak)
              for i, (n, k, f, nb) in enumerate(passes)]
+    thash = source_hash(TRAIN_SOURCES)
+    for ln in lines:
+        # DRAM bytes of the pass from its committed ncu summary (same sources)
+        ln["traffic"] = profiled_traffic(TRAIN_SUMMARIES.get(ln["pass"], ""), thash) if cfg.name == "qwen3_8b_train" \
+            else None
+        ln["dram_gbs"] = ln["traffic"] / (ln["us"] * 1e-6) / 1e9 if ln["traffic"] else None
     launches = 14 + 10 + 4              # 14 products, 10 other kernels, 4 vocabulary passes (and 3 memsets)
     return {"workload": cfg.name, "blocks": b, "block": B, "positions": P, "refiner_rows": rows, "hidden": cfg.H,
             "vocab": V, "us_per_step": step_us, "positions_per_s": P / (step_us * 1e-6),
@@ -722,7 +729,9 @@ def run_train(args):
                          "achieved": dom["achieved_tflops"] if dom["bound"] == "tensor" else dom["achieved_gbs"],
                          "peak": tc_peak if dom["bound"] == "tensor" else hbm,
                          "unit": "TFLOP/s" if dom["bound"] == "tensor" else "GB/s", "frac": dom["frac"],
-                         "traffic": None, "peak_source": src, "source_hash": source_hash(TRAIN_SOURCES)},
+                         "traffic": dom.get("traffic"), "dram_gbs": dom.get("dram_gbs"),
+                         "dram_frac": dom["dram_gbs"] / hbm if dom.get("dram_gbs") else None, "peak_source": src,
+                         "source_hash": source_hash(TRAIN_SOURCES)},
             "train_step": tr, "clocks": clk.summary()}
     print(json.dumps(line), flush=True)
     ref.close()
