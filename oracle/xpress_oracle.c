@@ -48,6 +48,14 @@
  *   - a decision that floating point turns into an integer (argmax, a Gumbel
  *     comparison, the accept test) is taken on values rounded to fp32, the
  *     precision the kernels decide in; ties resolve to the smallest index.
+ *   - training (Sec. 4.3): lambda weighs the drafter-anchor term and beta the
+ *     consistency term, as in the total-loss equation; every softmax at
+ *     T = 1; the bf16 operand roundings pass the gradient straight through;
+ *     sgn(0) = 0 in the L1 subgradient; the consistency forward takes the
+ *     first argmax of s_{k-1} as x_k (x_0 the anchor); the target logits are
+ *     those of the B positions themselves and w_k = exp(-(k-1)/gamma) for
+ *     k = 1..B; the drafter's own parameters are out of scope, so L(p^b)
+ *     contributes a value and no gradient.
  *
  * Random numbers: Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11), written
  * here from its published definition.  key = (seed low 32, seed high 32),
