@@ -135,9 +135,15 @@ struct TrainParams {
 };
 
 // train_read.cu
-__global__ void k_train_tok(const __grid_constant__ TrainParams p, const __grid_constant__ CUtensorMap tmap_z,
-                            const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_s,
-                            const __grid_constant__ CUtensorMap tmap_t, int mode);
+// k_train_tok_{stats, tv, dz}: the token-major kernel in its three modes
+#define XP_TRAIN_TOK_ARGS                                                                                     \
+    const __grid_constant__ TrainParams p, const __grid_constant__ CUtensorMap tmap_z,                        \
+        const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_s,               \
+        const __grid_constant__ CUtensorMap tmap_t
+__global__ void k_train_tok_stats(XP_TRAIN_TOK_ARGS);
+__global__ void k_train_tok_tv(XP_TRAIN_TOK_ARGS);
+__global__ void k_train_tok_dz(XP_TRAIN_TOK_ARGS);
+#undef XP_TRAIN_TOK_ARGS
 __global__ void k_train_voc(const __grid_constant__ TrainParams p, const __grid_constant__ CUtensorMap tmap_z,
                             const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_s,
                             const __grid_constant__ CUtensorMap tmap_t);

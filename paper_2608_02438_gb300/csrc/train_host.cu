@@ -120,7 +120,11 @@ int train_attributes()
     static std::once_flag once;
     std::call_once(once, [] {
         rc = XPRESS_OK;
-        if (cudaFuncSetAttribute(k_train_tok, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kTrainTokSmemBytes) !=
+        if (cudaFuncSetAttribute(k_train_tok_stats, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)kTrainTokSmemBytes) != cudaSuccess ||
+            cudaFuncSetAttribute(k_train_tok_tv, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kTrainTokSmemBytes) !=
+                cudaSuccess ||
+            cudaFuncSetAttribute(k_train_tok_dz, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kTrainTokSmemBytes) !=
                 cudaSuccess ||
             cudaFuncSetAttribute(k_train_voc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kTrainVocSmemBytes) !=
                 cudaSuccess ||
@@ -310,9 +314,15 @@ int train_run(const xpress_refiner *R, const xpress_train_in *in, const xpress_t
     const dim3 gtok(L.splits, NR / 128);
     const int nvt128 = (V + 127) / 128;
     if (only >= 0) {
-        if (only == 0 || only == 1 || only == 2)
-            XT_CUDA(launch(k_train_tok, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128, tw64, ts64,
-                           tt64, only));
+        if (only == TR_STATS)
+            XT_CUDA(launch(k_train_tok_stats, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128,
+                           *refiner_tmap_wr128(R), ts64, tt64));
+        else if (only == TR_TV)
+            XT_CUDA(launch(k_train_tok_tv, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128, tw64, ts64,
+                           tt64));
+        else if (only == TR_DZ)
+            XT_CUDA(launch(k_train_tok_dz, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128, tw64, ts64,
+                           tt64));
         else
             XT_CUDA(launch(k_train_voc, dim3(nvt128 < sms ? nvt128 : sms), dim3(kTrainVocThreads), kTrainVocSmemBytes,
                            st, tp, tz32, *refiner_tmap_wr128(R), ts32, tt32));
@@ -356,14 +366,15 @@ int train_run(const xpress_refiner *R, const xpress_train_in *in, const xpress_t
 
     // the Read passes
     const dim3 gvoc(nvt128 < sms ? nvt128 : sms);
-    XT_CUDA(launch(k_train_tok, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128, tw64, ts64, tt64,
-                   (int)TR_STATS));
+    // W_r tiles of 128 ids (boxes of 128 rows) for the log-sum-exp pass, of 64 for the others
+    XT_CUDA(launch(k_train_tok_stats, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128,
+                   *refiner_tmap_wr128(R), ts64, tt64));
     XT_CUDA(launch(k_train_stats_fin, dim3(NR / 8), dim3(256), 0, st, m));
-    XT_CUDA(launch(k_train_tok, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128, tw64, ts64, tt64,
-                   (int)TR_TV));
+    XT_CUDA(launch(k_train_tok_tv, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128, tw64, ts64,
+                   tt64));
     XT_CUDA(launch(k_train_tv_fin, dim3(in->b), dim3(32), 0, st, m));
-    XT_CUDA(launch(k_train_tok, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128, tw64, ts64, tt64,
-                   (int)TR_DZ));
+    XT_CUDA(launch(k_train_tok_dz, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128, tw64, ts64,
+                   tt64));
     XT_CUDA(launch(k_train_voc, gvoc, dim3(kTrainVocThreads), kTrainVocSmemBytes, st, tp, tz32,
                    *refiner_tmap_wr128(R), ts32, tt32));
 

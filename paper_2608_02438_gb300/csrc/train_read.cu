@@ -10,8 +10,8 @@
 // the teacher-forced forward and rows 64-127 the consistency forward of the
 // same positions, so that one s / t tile of those 64 positions serves both.
 //
-// k_train_tok -- token-major: D[row, v] = z_row . W_r[v], M = 128 rows, N = 64
-// vocabulary ids, K = r.  CTA (split, tile) takes one row tile and a
+// k_train_tok -- token-major: D[row, v] = z_row . W_r[v], M = 128 rows, N = 128
+// vocabulary ids in TR_STATS, 64 in TR_TV and TR_DZ, K = r.  CTA (split, tile) takes one row tile and a
 // contiguous range of vocabulary tiles.  The row tile Z sits in tensor memory
 // as the A operand (with N = 64, re-reading a 4 KB A block from shared memory
 // for every MMA would cost more than the product), so shared memory holds
@@ -42,22 +42,19 @@ constexpr float L2E = 1.4426950408889634f;
 
 // ---------------------------------------------------------------- k_train_tok
 constexpr int TR_BM = 128;
-constexpr int TR_BN = 64;
-constexpr int TR_BMAX = 5;                                 // most W_r ring stages
+constexpr int TR_BN = 64;                                  // ids per tile in TR_DZ (128 in the other modes)
+constexpr int TR_BMAX = 4;                                 // most W_r ring stages
 constexpr int TR_SMAX = 8;                                 // most s / t ring stages
 constexpr int TR_PF = 8;                                   // s / t tiles prefetched into L2 ahead
 constexpr int TR_EPI_WARPS = 16;                           // 2 sets (item parity) x 4 lane quarters x 2 id groups
 constexpr int TR_SET = TR_EPI_WARPS / 2;                   // the warps that take one item
 constexpr int TR_THREADS = 32 * (2 + TR_EPI_WARPS);
-constexpr uint32_t TR_B_CHUNK = TR_BN * 64 * 2;            // 8 KB: 64 ids x 64 of r
-constexpr uint32_t TR_B_STAGE = 4 * TR_B_CHUNK;            // 32 KB: one vocabulary tile of W_r
-constexpr uint32_t TR_ST_TILE = 64 * TR_BN * 2;            // 8 KB: 64 positions x 64 ids of s (or t)
+constexpr uint32_t TR_BOX = 64 * 64 * 2;                   // 8 KB: a TMA box of 64 rows x 64 bf16 (128 B)
 constexpr uint32_t TR_D_BUF = TR_BM * TR_BN * 2;           // 16 KB: dl tile, bf16, K-major (K = ids)
 constexpr uint32_t TR_RINGS = 224 * 1024;                  // W_r ring, s / t ring (and the dl tiles in TR_DZ)
-constexpr uint32_t TR_IDESC_F = idesc_bf16(TR_BM, TR_BN);
 constexpr uint32_t TR_IDESC_D = idesc_bf16_mn(TR_BM, RANK, false, true);
 constexpr int TR_NBUF = 4;                                 // most l accumulators in flight
-// TMEM: l accumulators (4, TR_DZ: 2) of 64 columns from 0, then the Z tile (128
+// TMEM: the l accumulators (tr_nbuf) of bn columns from 0, then the Z tile (128
 // columns: 256 bf16 per lane, two per column), then in TR_DZ dz (256) at 256
 constexpr uint32_t TR_TMEM_COLS = 512;
 constexpr uint32_t TR_DZ_COL = 256;
@@ -80,15 +77,27 @@ static_assert(TR_SMEM <= 232448, "k_train_tok shared memory");
 // from L2 take about 2 us under load, so their ring depth sets the pace; the
 // s / t tiles are prefetched into L2 and need fewer), s / t stage bytes and
 // stages, and the two dl tiles in TR_DZ.
-__host__ __device__ constexpr int tr_bstages(int mode) { return mode == TR_DZ ? 4 : 5; }
-__host__ __device__ constexpr int tr_nbuf(int mode) { return mode == TR_DZ ? 2 : TR_NBUF; }
-__host__ __device__ constexpr uint32_t tr_stage_bytes(int mode) { return mode == TR_STATS ? TR_ST_TILE : 2 * TR_ST_TILE; }
+// 128-id tiles where the epilogue is light (the log-sum-exp pass: the MMA of a
+// 16-instruction tile costs the same for N = 64 and N = 128), 64 otherwise
+__host__ __device__ constexpr int tr_bn(int mode) { return mode == TR_STATS ? 2 * TR_BN : TR_BN; }
+__host__ __device__ constexpr uint32_t tr_bstage(int mode) { return 4u * tr_bn(mode) * 128u; }   // a W_r tile
+__host__ __device__ constexpr int tr_bstages(int mode) { return mode == TR_STATS ? 2 : 4; }
+__host__ __device__ constexpr int tr_nbuf(int mode) { return mode == TR_TV ? 4 : 2; }
+static_assert(tr_nbuf(TR_STATS) * 2 * 64 + 128 <= 512 && tr_nbuf(TR_TV) * 64 + 128 <= 512 &&
+                  tr_nbuf(TR_DZ) * 64 + 128 <= 256,
+              "tensor memory: accumulators + Z (+ dz)");
+__host__ __device__ constexpr uint32_t tr_st_tile(int mode) { return (uint32_t)tr_bn(mode) * 64u * 2u; }   // s or t
+__host__ __device__ constexpr uint32_t tr_stage_bytes(int mode)
+{
+    return mode == TR_STATS ? tr_st_tile(mode) : 2 * tr_st_tile(mode);
+}
 __host__ __device__ constexpr int tr_stages(int mode)
 {
-    return (int)((TR_RINGS - tr_bstages(mode) * TR_B_STAGE - (mode == TR_DZ ? 2 * TR_D_BUF : 0)) / tr_stage_bytes(mode));
+    return (int)((TR_RINGS - tr_bstages(mode) * tr_bstage(mode) - (mode == TR_DZ ? 2 * TR_D_BUF : 0)) /
+                 tr_stage_bytes(mode));
 }
 static_assert(tr_stages(TR_STATS) <= TR_SMAX && tr_stages(TR_TV) >= 2 && tr_stages(TR_DZ) >= 2 &&
-                  tr_stages(TR_TV) <= TR_SMAX && tr_stages(TR_DZ) <= TR_SMAX && tr_bstages(TR_STATS) <= TR_BMAX,
+                  tr_stages(TR_TV) <= TR_SMAX && tr_stages(TR_DZ) <= TR_SMAX && tr_bstages(TR_DZ) <= TR_BMAX,
               "ring depths");
 
 __device__ __forceinline__ void tr_epi_bar()
@@ -140,13 +149,12 @@ __device__ __forceinline__ float dl_value(float a2, float b2, float Apos, float 
 const size_t kTrainTokSmemBytes = TR_SMEM;
 const int kTrainTokThreads = TR_THREADS;
 
-// grid (splits, NR / 128), TR_THREADS threads, TR_SMEM bytes.  tmap_z is not
-// read (Z goes to tensor memory from p.zop); the argument keeps the four maps
-// of the vocabulary-major kernel.
-__global__ void __launch_bounds__(TR_THREADS, 1)
-    k_train_tok(const __grid_constant__ TrainParams p, const __grid_constant__ CUtensorMap tmap_z,
-                const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_s,
-                const __grid_constant__ CUtensorMap tmap_t, int mode)
+// The token-major kernel for one mode (compiled once per mode, so that its
+// tile width, ring depths and epilogue are constants).  tmap_w: W_r boxes of
+// bn rows x 64; tmap_s / tmap_t: boxes of 64 ids x 64 positions.
+template <int mode>
+__device__ __forceinline__ void train_tok_body(const TrainParams &p, const CUtensorMap &tmap_w,
+                                               const CUtensorMap &tmap_s, const CUtensorMap &tmap_t)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -154,13 +162,17 @@ __global__ void __launch_bounds__(TR_THREADS, 1)
     TrShared &sh = *reinterpret_cast<TrShared *>(sB + TR_RINGS);
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const int j = blockIdx.y, sv = blockIdx.x;
-    const int vt0 = (int)((long long)p.nvt * sv / p.splits), vt1 = (int)((long long)p.nvt * (sv + 1) / p.splits);
+    constexpr int bn = tr_bn(mode);                // ids per tile
+    const int nvtm = (p.V + bn - 1) / bn;
+    const int vt0 = (int)((long long)nvtm * sv / p.splits), vt1 = (int)((long long)nvtm * (sv + 1) / p.splits);
     const int items = vt1 - vt0;
-    const bool dzm = mode == TR_DZ;
-    const int NB = tr_bstages(mode), NS = tr_stages(mode), NBUF = tr_nbuf(mode);
-    const uint32_t ZC = NBUF * TR_BN;              // TMEM column of the Z tile
-    const uint32_t SB = tr_stage_bytes(mode);
-    uint8_t *sS = sB + NB * TR_B_STAGE;            // s / t ring after the W_r ring
+    constexpr bool dzm = mode == TR_DZ;
+    constexpr int NB = tr_bstages(mode), NS = tr_stages(mode);
+    constexpr uint32_t BST = tr_bstage(mode), BCH = (uint32_t)tr_bn(mode) * 128, STT = tr_st_tile(mode);
+    constexpr int NBUF = tr_nbuf(mode);
+    constexpr uint32_t ZC = NBUF * bn;             // TMEM column of the Z tile
+    constexpr uint32_t SB = tr_stage_bytes(mode);
+    uint8_t *sS = sB + NB * BST;                   // s / t ring after the W_r ring
     uint8_t *sD = sS + NS * SB;                    // TR_DZ: the two dl tiles after the s / t ring
 
     if (threadIdx.x == 0) {
@@ -197,10 +209,12 @@ __global__ void __launch_bounds__(TR_THREADS, 1)
             tma_prefetch_desc(&tmap_s);
             tma_prefetch_desc(&tmap_t);
             const uint64_t keep = policy_evict_last(), once = policy_evict_first();
-            const bool need_t = mode != TR_STATS;
+            constexpr bool need_t = mode != TR_STATS;
             auto prefetch_st = [&](int it) {
-                tma_prefetch_2d(&tmap_s, (vt0 + it) * TR_BN, j * 64);
-                if (need_t) tma_prefetch_2d(&tmap_t, (vt0 + it) * TR_BN, j * 64);
+                for (int x = 0; x < bn; x += 64) {
+                    tma_prefetch_2d(&tmap_s, (vt0 + it) * bn + x, j * 64);
+                    if (need_t) tma_prefetch_2d(&tmap_t, (vt0 + it) * bn + x, j * 64);
+                }
             };
             for (int it = 0; it < min(TR_PF, items); ++it) prefetch_st(it);
             uint32_t pend_b = 0, par_b = 0, pend_s = 0, par_s = 0;
@@ -212,17 +226,19 @@ __global__ void __launch_bounds__(TR_THREADS, 1)
                 const int st = it % NB;
                 const uint32_t ph = (uint32_t)((it / NB) & 1);
                 if (!mbar_wait_spin(&sh.empty[st], ph ^ 1, abort, lim)) break;
-                mbar_expect_tx(&sh.full[st], TR_B_STAGE);
-                for (int c = 0; c < 4; ++c)
-                    tma_load_2d_hint(sB + st * TR_B_STAGE + c * TR_B_CHUNK, &tmap_w, &sh.full[st], c * 64, vt * TR_BN,
-                                     keep);
+                mbar_expect_tx(&sh.full[st], BST);
+                for (int c = 0; c < 4; ++c)      // tmap_w: boxes of bn rows x 64
+                    tma_load_2d_hint(sB + st * BST + c * BCH, &tmap_w, &sh.full[st], c * 64, vt * bn, keep);
                 pend_b |= 1u << st;
                 par_b = (par_b & ~(1u << st)) | (ph << st);
                 if (!mbar_wait_spin(&sh.sempty[ss], sph ^ 1, abort, lim)) break;
                 mbar_expect_tx(&sh.sfull[ss], SB);
-                tma_load_2d_hint(sS + ss * SB, &tmap_s, &sh.sfull[ss], vt * TR_BN, j * 64, once);
-                if (need_t)
-                    tma_load_2d_hint(sS + ss * SB + TR_ST_TILE, &tmap_t, &sh.sfull[ss], vt * TR_BN, j * 64, once);
+                for (int x = 0; x < bn; x += 64) {   // boxes of 64 ids x 64 positions
+                    tma_load_2d_hint(sS + ss * SB + x * 128, &tmap_s, &sh.sfull[ss], vt * bn + x, j * 64, once);
+                    if (need_t)
+                        tma_load_2d_hint(sS + ss * SB + STT + x * 128, &tmap_t, &sh.sfull[ss], vt * bn + x, j * 64,
+                                         once);
+                }
                 pend_s |= 1u << ss;
                 par_s = (par_s & ~(1u << ss)) | (sph << ss);
                 if (++ss == NS) { ss = 0; sph ^= 1; }
@@ -246,46 +262,47 @@ __global__ void __launch_bounds__(TR_THREADS, 1)
                 const int db = u & 1;
                 if (!mbar_wait_spin(&sh.dfull[db], (uint32_t)((u >> 1) & 1), abort, lim)) return false;
                 tc_fence_after();
-                const uint32_t bs = b0 + (u % NB) * TR_B_STAGE;
+                const uint32_t bs = b0 + (u % NB) * BST;
 #pragma unroll
                 for (int kk = 0; kk < TR_BN / 16; ++kk)
                     tc_mma_bf16(tmem + TR_DZ_COL, smem_desc_sw128(d0 + db * TR_D_BUF + kk * 32),
-                                smem_desc_sw128_mn(bs + kk * 2048, TR_B_CHUNK), TR_IDESC_D, (u | kk) != 0);
+                                smem_desc_sw128_mn(bs + kk * 2048, BCH), TR_IDESC_D, (u | kk) != 0);
                 tc_commit(&sh.empty[u % NB]);
                 tc_commit(&sh.dempty[db]);
                 return true;
             };
             bool ok = mbar_wait_spin(&sh.a_full, 0, abort, lim);
             if (ok) tc_fence_after();
-            // without dz: two tiles at a time, their MMA chains interleaved
-            // (two accumulators), so that consecutive MMAs do not depend on
-            // one another
-            for (int it = 0; it + 1 < items && ok && !dzm; it += 2) {
-                const int st0 = it % NB, st1 = (it + 1) % NB, b0_ = it % NBUF, b1_ = (it + 1) % NBUF;
+            const uint32_t idesc_f = idesc_bf16(TR_BM, bn);
+            // TR_TV: two tiles at a time, their MMA chains interleaved (two
+            // accumulators), so that consecutive MMAs do not depend on one another
+            constexpr bool pairs = mode == TR_TV;
+            for (int it = 0; pairs && it + 1 < items && ok; it += 2) {
+                const int st0 = it % NB, st1 = (it + 1) % NB, q0 = it % NBUF, q1 = (it + 1) % NBUF;
                 if (!mbar_wait_spin(&sh.full[st0], (uint32_t)((it / NB) & 1), abort, lim) ||
                     !mbar_wait_spin(&sh.full[st1], (uint32_t)(((it + 1) / NB) & 1), abort, lim) ||
-                    !mbar_wait_spin(&sh.tempty[b0_], (uint32_t)(((it / NBUF) & 1) ^ 1), abort, lim) ||
-                    !mbar_wait_spin(&sh.tempty[b1_], (uint32_t)((((it + 1) / NBUF) & 1) ^ 1), abort, lim)) {
+                    !mbar_wait_spin(&sh.tempty[q0], (uint32_t)(((it / NBUF) & 1) ^ 1), abort, lim) ||
+                    !mbar_wait_spin(&sh.tempty[q1], (uint32_t)((((it + 1) / NBUF) & 1) ^ 1), abort, lim)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const uint32_t bs0 = b0 + st0 * TR_B_STAGE, bs1 = b0 + st1 * TR_B_STAGE;
+                const uint32_t bs0 = b0 + st0 * BST, bs1 = b0 + st1 * BST;
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk) {
-                        tc_mma_bf16_ts(tmem + b0_ * TR_BN, tmem + ZC + c * 32 + kk * 8,
-                                       smem_desc_sw128(bs0 + c * TR_B_CHUNK + kk * 32), TR_IDESC_F, (c | kk) != 0);
-                        tc_mma_bf16_ts(tmem + b1_ * TR_BN, tmem + ZC + c * 32 + kk * 8,
-                                       smem_desc_sw128(bs1 + c * TR_B_CHUNK + kk * 32), TR_IDESC_F, (c | kk) != 0);
+                        tc_mma_bf16_ts(tmem + q0 * bn, tmem + ZC + c * 32 + kk * 8,
+                                       smem_desc_sw128(bs0 + c * BCH + kk * 32), idesc_f, (c | kk) != 0);
+                        tc_mma_bf16_ts(tmem + q1 * bn, tmem + ZC + c * 32 + kk * 8,
+                                       smem_desc_sw128(bs1 + c * BCH + kk * 32), idesc_f, (c | kk) != 0);
                     }
-                tc_commit(&sh.tfull[b0_]);
-                tc_commit(&sh.tfull[b1_]);
+                tc_commit(&sh.tfull[q0]);
+                tc_commit(&sh.tfull[q1]);
                 tc_commit(&sh.empty[st0]);
                 tc_commit(&sh.empty[st1]);
             }
-            for (int it = dzm ? 0 : (items & ~1); it < items && ok; ++it) {
+            for (int it = pairs ? (items & ~1) : 0; it < items && ok; ++it) {
                 const int st = it % NB, buf = it % NBUF;
                 if (!mbar_wait_spin(&sh.full[st], (uint32_t)((it / NB) & 1), abort, lim) ||
                     !mbar_wait_spin(&sh.tempty[buf], (uint32_t)(((it / NBUF) & 1) ^ 1), abort, lim)) {
@@ -293,13 +310,13 @@ __global__ void __launch_bounds__(TR_THREADS, 1)
                     break;
                 }
                 tc_fence_after();
-                const uint32_t bs = b0 + st * TR_B_STAGE;
+                const uint32_t bs = b0 + st * BST;
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk)
-                        tc_mma_bf16_ts(tmem + buf * TR_BN, tmem + ZC + c * 32 + kk * 8,
-                                       smem_desc_sw128(bs + c * TR_B_CHUNK + kk * 32), TR_IDESC_F, (c | kk) != 0);
+                        tc_mma_bf16_ts(tmem + buf * bn, tmem + ZC + c * 32 + kk * 8,
+                                       smem_desc_sw128(bs + c * BCH + kk * 32), idesc_f, (c | kk) != 0);
                 tc_commit(&sh.tfull[buf]);
                 if (!dzm) tc_commit(&sh.empty[st]);
                 else if (it > 0 && !dz_step(it - 1)) ok = false;
@@ -313,9 +330,9 @@ __global__ void __launch_bounds__(TR_THREADS, 1)
         }
     } else {
         // ------------------------------------------------------ epilogue
-        // warp set `set` takes the items of its parity (accumulators set and
-        // set + 2, dl tile `set`); within a set, warp (q, g) the 32 rows of
-        // lane quarter q and the 32 ids of group g, in two halves of 16
+        // warp set `set` takes the items of its parity (accumulators it %
+        // NBUF, dl tile `set`); within a set, warp (q, g) the 32 rows of lane
+        // quarter q and ids [g bn / 2, (g + 1) bn / 2) of the tile, 16 at a time
         const int ew = warp - 2, q = warp & 3, g = (ew >> 2) & 1, set = ew >> 3;
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
         const int row = q * 32 + lane, f = row >> 6, pl = row & 63;
@@ -352,14 +369,15 @@ __global__ void __launch_bounds__(TR_THREADS, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive(&sh.a_full);
         }
-        // the anchor term's share: the teacher-forced row takes the even
-        // 32-id group of each tile, the consistency row the odd one
+        // the anchor term's share: the teacher-forced row takes the first half
+        // of each tile's ids, the consistency row the second
         const bool anchor = (f == g);
         // STATS: running (m, s); TV: 2-way partial sums of min(p, q), of the
         // part where p < q (+ half of where p = q), and of the anchor's min(p^b, q)
         float m2 = -INFINITY, s2 = 0.f;
         float r0[2] = {0.f, 0.f}, r1[2] = {0.f, 0.f}, r3[2] = {0.f, 0.f};
         bool ok = true;
+        constexpr int nq = bn / 32;                // 16-id pieces per warp and tile
         for (int it = set; it < items; it += 2) {
             const int buf = it % NBUF;
             const uint32_t ph = (uint32_t)((it >> 1) & 1);      // phase of the dl tile `set`
@@ -371,20 +389,24 @@ __global__ void __launch_bounds__(TR_THREADS, 1)
             }
             tc_fence_after();
             const uint8_t *stile = sS + ss * SB;
-            const int v0 = (vt0 + it) * TR_BN + g * 32;
-            const int nv = valid ? min(32, p.V - v0) : 0;
+            const int v0 = (vt0 + it) * bn + g * (bn / 2);
+            const int nv = valid ? min(bn / 2, p.V - v0) : 0;
             uint32_t w[16];
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
+            for (int h = 0; h < 4; ++h) {
+                if (h >= nq) break;
+                const int idoff = g * (bn / 2) + 16 * h;        // first id of the piece within the tile
                 float acc[16];
-                tmem_ld16(tmem + lane_base + buf * TR_BN + g * 32 + h * 16, acc);
-                // this half's 16 ids of s (and t): chunks 4g + 2h, + 1 of the row
+                tmem_ld16(tmem + lane_base + buf * bn + idoff, acc);
+                // the piece's 16 ids of s (and t): two 16-byte chunks of row pl
+                // of the 64-id box idoff / 64
                 uint4 sr[2], tr[2];
 #pragma unroll
                 for (int c = 0; c < 2; ++c) {
-                    const int off = pl * 128 + (((4 * g + 2 * h + c) ^ (pl & 7)) << 4);
+                    const int off = (idoff >> 6) * (int)TR_BOX + pl * 128 +
+                                    (((((idoff & 63) >> 3) + c) ^ (pl & 7)) << 4);
                     sr[c] = *reinterpret_cast<const uint4 *>(stile + off);
-                    if (mode != TR_STATS) tr[c] = *reinterpret_cast<const uint4 *>(stile + TR_ST_TILE + off);
+                    if (mode != TR_STATS) tr[c] = *reinterpret_cast<const uint4 *>(stile + STT + off);
                 }
                 float sv[16], tv[16];
 #pragma unroll
@@ -399,7 +421,7 @@ __global__ void __launch_bounds__(TR_THREADS, 1)
                         tv[8 * c + 2 * e + 1] = __uint_as_float(wt_[e] & 0xFFFF0000u);
                     }
                 }
-                const int nh = nv - 16 * h;              // ids of this half that exist (<= 0: none)
+                const int nh = nv - 16 * h;              // ids of this piece that exist (<= 0: none)
                 if (mode == TR_STATS) {
                     if (nh > 0) {
                         float x[16];
@@ -443,7 +465,7 @@ __global__ void __launch_bounds__(TR_THREADS, 1)
                             const float b2 = fmaf(tv[jv], L2E, -lq2);
                             d2[e] = jv < nh ? dl_value(a2, b2, Apos, Aneg) : 0.f;
                         }
-                        w[8 * h + jj / 2] = pack_bf16x2(d2[0], d2[1]);
+                        w[8 * (h & 1) + jj / 2] = pack_bf16x2(d2[0], d2[1]);
                     }
                 }
             }
@@ -510,6 +532,30 @@ __global__ void __launch_bounds__(TR_THREADS, 1)
         tmem_dealloc(tmem, TR_TMEM_COLS);
     }
     if (threadIdx.x == 0 && sh.abort) set_status(p.status, ST_TIMEOUT);
+}
+
+// grid (splits, NR / 128), TR_THREADS threads, TR_SMEM bytes; one kernel per
+// mode.  tmap_z is not read (Z goes to tensor memory from p.zop).
+__global__ void __launch_bounds__(TR_THREADS, 1)
+    k_train_tok_stats(const __grid_constant__ TrainParams p, const __grid_constant__ CUtensorMap tmap_z,
+                      const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_s,
+                      const __grid_constant__ CUtensorMap tmap_t)
+{
+    train_tok_body<TR_STATS>(p, tmap_w, tmap_s, tmap_t);
+}
+__global__ void __launch_bounds__(TR_THREADS, 1)
+    k_train_tok_tv(const __grid_constant__ TrainParams p, const __grid_constant__ CUtensorMap tmap_z,
+                   const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_s,
+                   const __grid_constant__ CUtensorMap tmap_t)
+{
+    train_tok_body<TR_TV>(p, tmap_w, tmap_s, tmap_t);
+}
+__global__ void __launch_bounds__(TR_THREADS, 1)
+    k_train_tok_dz(const __grid_constant__ TrainParams p, const __grid_constant__ CUtensorMap tmap_z,
+                   const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_s,
+                   const __grid_constant__ CUtensorMap tmap_t)
+{
+    train_tok_body<TR_DZ>(p, tmap_w, tmap_s, tmap_t);
 }
 
 // ---------------------------------------------------------------- k_train_voc
