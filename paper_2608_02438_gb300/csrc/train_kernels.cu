@@ -53,73 +53,83 @@ __device__ __forceinline__ float sigma_prime(int act, float t)
 
 }  // namespace
 
-// grid (nch, P), 256 threads: ids [ch 8192 + 32 tid, +32) of position blockIdx.y.
-__global__ void __launch_bounds__(256) k_train_rows(TrainMisc m)
+// grid (nch, P), 256 threads: warp w of chunk ch takes the 2048 ids from
+// ch TRAIN_ROW_CHUNK + 2048 w of position blockIdx.y; lane l reads the 8-id
+// pieces l, l + 32, ..., l + 224 of it (each load instruction of the warp one
+// coalesced 512-byte run).  The warp's maxima are reduced first, so every
+// exponential is taken against the warp maximum and the sums need no rescale.
+__global__ void __launch_bounds__(256, 2) k_train_rows(TrainMisc m)
 {
     pdl_trigger();
     pdl_wait();
-    const int ch = blockIdx.x, i = blockIdx.y, tid = threadIdx.x;
-    const int v0 = ch * TRAIN_ROW_CHUNK + tid * 32;
+    const int ch = blockIdx.x, i = blockIdx.y, tid = threadIdx.x, w = tid >> 5, lane = tid & 31;
+    const int vw = ch * TRAIN_ROW_CHUNK + w * (TRAIN_ROW_CHUNK / 8) + 8 * lane;
     const uint16_t *srow = static_cast<const uint16_t *>(m.s) + (size_t)i * m.V;
     const uint16_t *trow = static_cast<const uint16_t *>(m.t) + (size_t)i * m.V;
-    float xs[32], xt[32];
-    if (v0 + 32 <= m.V) {
-        const uint4 *sp = reinterpret_cast<const uint4 *>(srow + v0), *tp = reinterpret_cast<const uint4 *>(trow + v0);
+    constexpr uint32_t NEG2 = 0xFF80FF80u;     // two bf16 -inf
+    uint4 ps[8], pt[8];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            const uint4 a = __ldcs(sp + c), b = __ldcs(tp + c);
-            const uint32_t wa[4] = {a.x, a.y, a.z, a.w}, wb[4] = {b.x, b.y, b.z, b.w};
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                xs[8 * c + 2 * q] = __uint_as_float(wa[q] << 16);
-                xs[8 * c + 2 * q + 1] = __uint_as_float(wa[q] & 0xFFFF0000u);
-                xt[8 * c + 2 * q] = __uint_as_float(wb[q] << 16);
-                xt[8 * c + 2 * q + 1] = __uint_as_float(wb[q] & 0xFFFF0000u);
-            }
-        }
-    } else {
-#pragma unroll
-        for (int jj = 0; jj < 32; ++jj) {
-            const bool in = v0 + jj < m.V;
-            xs[jj] = in ? bf2f(srow[v0 + jj]) : -INFINITY;
-            xt[jj] = in ? bf2f(trow[v0 + jj]) : -INFINITY;
+    for (int c = 0; c < 8; ++c) {
+        const int v = vw + 256 * c;
+        if (v < m.V) {                         // V % 8 == 0: a piece is wholly inside or wholly past the end
+            ps[c] = __ldcs(reinterpret_cast<const uint4 *>(srow + v));
+            pt[c] = __ldcs(reinterpret_cast<const uint4 *>(trow + v));
+        } else {
+            ps[c] = pt[c] = make_uint4(NEG2, NEG2, NEG2, NEG2);
         }
     }
-    float best = -INFINITY, ms = -INFINITY, mt = -INFINITY;
+    // the thread's ids increase along (c, word, half): a strict > keeps the first
+    float best = -INFINITY, mt = -INFINITY;
     int idx = 0x7fffffff;
 #pragma unroll
-    for (int jj = 0; jj < 32; ++jj) {
-        if (xs[jj] > best) { best = xs[jj]; idx = v0 + jj; }
-        ms = fmaxf(ms, xs[jj]);
-        mt = fmaxf(mt, xt[jj]);
-    }
-    float ss = 0.f, st = 0.f;
-    ms *= L2E;
-    mt *= L2E;
-    if (ms != -INFINITY) {
+    for (int c = 0; c < 8; ++c) {
+        const uint32_t ws[4] = {ps[c].x, ps[c].y, ps[c].z, ps[c].w}, wt[4] = {pt[c].x, pt[c].y, pt[c].z, pt[c].w};
 #pragma unroll
-        for (int jj = 0; jj < 32; ++jj) {
-            ss += ex2_approx(fmaf(xs[jj], L2E, -ms));
-            st += ex2_approx(fmaf(xt[jj], L2E, -mt));
+        for (int q = 0; q < 4; ++q) {
+            const float s0 = __uint_as_float(ws[q] << 16), s1 = __uint_as_float(ws[q] & 0xFFFF0000u);
+            const int v = vw + 256 * c + 2 * q;
+            if (s0 > best) { best = s0; idx = v; }
+            if (s1 > best) { best = s1; idx = v + 1; }
+            mt = fmaxf(mt, fmaxf(__uint_as_float(wt[q] << 16), __uint_as_float(wt[q] & 0xFFFF0000u)));
         }
     }
-    // warp, then block
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
-        const float oms = __shfl_xor_sync(0xffffffffu, ms, o), oss = __shfl_xor_sync(0xffffffffu, ss, o);
-        const float omt = __shfl_xor_sync(0xffffffffu, mt, o), ost = __shfl_xor_sync(0xffffffffu, st, o);
         const float ob = __shfl_xor_sync(0xffffffffu, best, o);
         const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
-        lse2_merge(ms, ss, oms, oss);
-        lse2_merge(mt, st, omt, ost);
+        mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, o));
         merge_argmax(best, idx, ob, oi);
+    }
+    // best is now the warp's maximum of s (log2 domain below)
+    const float ms2 = best * L2E, mt2 = mt * L2E;
+    float ss[2] = {0.f, 0.f}, st[2] = {0.f, 0.f};
+    const bool has_s = best != -INFINITY, has_t = mt != -INFINITY;
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+        const uint32_t ws[4] = {ps[c].x, ps[c].y, ps[c].z, ps[c].w}, wt[4] = {pt[c].x, pt[c].y, pt[c].z, pt[c].w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            if (has_s) {
+                ss[q & 1] += ex2_approx(fmaf(__uint_as_float(ws[q] << 16), L2E, -ms2));
+                ss[q & 1] += ex2_approx(fmaf(__uint_as_float(ws[q] & 0xFFFF0000u), L2E, -ms2));
+            }
+            if (has_t) {
+                st[q & 1] += ex2_approx(fmaf(__uint_as_float(wt[q] << 16), L2E, -mt2));
+                st[q & 1] += ex2_approx(fmaf(__uint_as_float(wt[q] & 0xFFFF0000u), L2E, -mt2));
+            }
+        }
+    }
+    float sum_s = ss[0] + ss[1], sum_t = st[0] + st[1];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        sum_s += __shfl_xor_sync(0xffffffffu, sum_s, o);
+        sum_t += __shfl_xor_sync(0xffffffffu, sum_t, o);
     }
     __shared__ float4 wp[8];
     __shared__ float wb[8];
     __shared__ int wi[8];
-    const int w = tid >> 5;
-    if ((tid & 31) == 0) {
-        wp[w] = make_float4(ms, ss, mt, st);
+    if (lane == 0) {
+        wp[w] = make_float4(has_s ? ms2 : -INFINITY, sum_s, has_t ? mt2 : -INFINITY, sum_t);
         wb[w] = best;
         wi[w] = idx;
     }
@@ -211,6 +221,7 @@ __global__ void __launch_bounds__(RANK) k_train_fuse(TrainMisc m)
     float ug = 0.f;
     for (int j = 0; j < B; ++j) {
         float uj = 0.f;
+#pragma unroll 8
         for (int sp = 0; sp < m.usplits; ++sp) uj += m.Ug[sp * slice + (size_t)(blk * B + j) * RANK + d];
         ug += uj;
     }
@@ -219,6 +230,7 @@ __global__ void __launch_bounds__(RANK) k_train_fuse(TrainMisc m)
     for (int k = k4; k < B; k += 4) {
         const int i = blk * B + k;
         float uhv = 0.f;
+#pragma unroll 8
         for (int sp = 0; sp < m.usplits; ++sp) uhv += m.Uh[sp * slice + (size_t)i * RANK + d];
         const uint16_t uh = f2bf(uhv), uhl = f2bf(uhv - bf2f(uh));
         for (int f = 0; f < 2; ++f) {
