@@ -103,6 +103,20 @@ def test_bf16_ragged_vocabulary(X, b, B, temps):
     _check(X, cfg, w, inp)
 
 
+# Read ranges of several 128-row blocks (V = 40008 over 144 Read CTAs: 256 or
+# 288 rows each, i.e. 2 full blocks and possibly a partial third, the last
+# range ending in a partial quarter),
+# so that the W_r ring of the persistent kernel wraps within a pass and runs
+# ahead across passes (16 of them) at a size the oracle finishes in seconds.
+@pytest.mark.parametrize("b,temps", [(1, (0.0,)), (2, (1.0, 0.0))])
+def test_bf16_multi_block_read_ranges(X, b, temps):
+    cfg = W.tiny_config("bf16r", b=b, B=16, H=128, V=40008, r=256, dtype=W.BF16, temps=temps, seed=1700 + b)
+    w = W.make_weights(cfg.H, cfg.V, cfg.r, cfg.B, cfg.dtype, 2700 + b, "strong")
+    inp = W.make_inputs(cfg)
+    _, _, _, _, orc = _check(X, cfg, w, inp)
+    assert max(o["iters"] for o in orc.values()) >= 2
+
+
 def test_bf16_fixed_k_and_cap(X):
     cfg = W.tiny_config("bf16k", b=6, B=16, H=128, V=2080, r=256, dtype=W.BF16, temps=(0.0, 1.0), seed=31)
     w = W.make_weights(cfg.H, cfg.V, cfg.r, cfg.B, cfg.dtype, 32, "strong")
