@@ -331,8 +331,8 @@ size_t xpress_train_workspace_size(const xpress_refiner *refiner, int b, int B);
  * ids out of [0, V) are clamped to 0 and reported by the status word
  * (XPRESS_ERR_DEVICE_CHECK); a bounded wait that gives up reports
  * XPRESS_ERR_TIMEOUT there.
- * Errors: INVALID_ARG (NULL pointer, b < 1, B mismatch, gamma <= 0),
- * UNSUPPORTED (fp32 refiner), WORKSPACE, CUDA. */
+ * Errors: INVALID_ARG (NULL pointer, h / s / target not 16-byte aligned,
+ * b < 1, B mismatch, gamma <= 0), UNSUPPORTED (fp32 refiner), WORKSPACE, CUDA. */
 int xpress_train_step(const xpress_refiner *refiner, const xpress_train_in *in, const xpress_train_out *out,
                       void *workspace, size_t ws_bytes, void *stream);
 

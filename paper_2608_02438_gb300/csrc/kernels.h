@@ -225,7 +225,9 @@ __global__ void k_train_dact(TrainMisc m);
 __global__ void k_train_mix_bwd(TrainMisc m);
 size_t train_mix_smem(int B);               // dynamic shared memory of k_train_mix / _mix_bwd
 __global__ void k_train_fuse_bwd(TrainMisc m);
-constexpr int TRAIN_ROW_CHUNK = 16384;      // vocabulary ids per k_train_rows CTA (8 warps x 32 lanes x 64)
+constexpr int TRAIN_ROW_CHUNK = 16384;      // vocabulary ids per k_train_rows item (8 warps x 32 lanes x 64)
+extern const size_t kTrainRowsSmemBytes;
+extern const int kTrainRowsThreads;
 
 // acceptance launch shared by xpress_accept and xpress_accept_noalloc
 // (xpress_host.cu); `ws` holds the scratch laid out by accept_scratch_bytes

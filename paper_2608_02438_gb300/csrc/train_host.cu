@@ -126,6 +126,8 @@ int train_attributes()
                 cudaSuccess ||
             cudaFuncSetAttribute(k_train_tok_dz, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kTrainTokSmemBytes) !=
                 cudaSuccess ||
+            cudaFuncSetAttribute(k_train_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kTrainRowsSmemBytes) !=
+                cudaSuccess ||
             cudaFuncSetAttribute(k_train_voc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kTrainVocSmemBytes) !=
                 cudaSuccess ||
             cudaFuncSetAttribute(k_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmemBytes) !=
@@ -208,6 +210,10 @@ int train_run(const xpress_refiner *R, const xpress_train_in *in, const xpress_t
     if (in->b < 1 || in->B != w.B || !in->h || !in->s || !in->target || !in->ystar || !in->anchor ||
         !(in->gamma > 0.0f) || !out->loss || !out->gW_e || !out->gW_h || !out->gW_g || !out->gW_in || !out->gL ||
         !out->gW1 || !out->gW2 || !out->gW_r)
+        return XPRESS_ERR_INVALID_ARG;
+    // h, s and target are read by bulk copies, tensor maps and 16-byte loads
+    if (((reinterpret_cast<uintptr_t>(in->h) | reinterpret_cast<uintptr_t>(in->s) |
+          reinterpret_cast<uintptr_t>(in->target)) & 15) != 0)
         return XPRESS_ERR_INVALID_ARG;
     if (refiner_device(R) >= 0) {
         int dev = -1;
@@ -335,7 +341,9 @@ int train_run(const xpress_refiner *R, const xpress_train_in *in, const xpress_t
     XT_CUDA(cudaMemsetAsync(W + L.A2, 0, (size_t)NR * 4, st));
 
     // the drafter's rows: lse of s and of the target, s at y*, argmax s
-    XT_CUDA(launch(k_train_rows, dim3(L.nch, P), dim3(256), 0, st, m));
+    const int row_items = L.nch * P;
+    XT_CUDA(launch(k_train_rows, dim3(row_items < sms ? row_items : sms), dim3(kTrainRowsThreads), kTrainRowsSmemBytes,
+                   st, m));
     XT_CUDA(launch(k_train_rows_fin, dim3((P + 7) / 8), dim3(256), 0, st, m));
 
     // forward: Fuse, Mix, Trans of both input sequences

@@ -53,99 +53,197 @@ __device__ __forceinline__ float sigma_prime(int act, float t)
 
 }  // namespace
 
-// grid (nch, P), 256 threads: warp w of chunk ch takes the 2048 ids from
-// ch TRAIN_ROW_CHUNK + 2048 w of position blockIdx.y; lane l reads the 8-id
-// pieces l, l + 32, ..., l + 224 of it (each load instruction of the warp one
-// coalesced 512-byte run).  The warp's maxima are reduced first, so every
-// exponential is taken against the warp maximum and the sums need no rescale.
-__global__ void __launch_bounds__(256, 2) k_train_rows(TrainMisc m)
+namespace {
+
+constexpr int ROWS_STAGES = 3;
+constexpr uint32_t ROWS_SEG = TRAIN_ROW_CHUNK * 2;          // bytes of one s (or t) segment
+constexpr int ROWS_THREADS = 32 * 9;                         // a copy warp, 8 reducing warps
+
+struct RowsShared {
+    uint64_t full[ROWS_STAGES], empty[ROWS_STAGES];
+    float4 wp[2][8];                                          // per item parity and warp: max / sum of s and t
+    float wb[2][8];
+    int wi[2][8];
+    int abort;
+};
+
+constexpr size_t ROWS_SMEM = 128 + ROWS_STAGES * 2 * ROWS_SEG + sizeof(RowsShared);
+
+// OR of `pred` over the 256 reducing threads (named barrier 1): every one of
+// them takes the same decision.
+__device__ __forceinline__ bool rows_bar_or(bool pred)
 {
-    pdl_trigger();
-    pdl_wait();
-    const int ch = blockIdx.x, i = blockIdx.y, tid = threadIdx.x, w = tid >> 5, lane = tid & 31;
-    const int vw = ch * TRAIN_ROW_CHUNK + w * (TRAIN_ROW_CHUNK / 8) + 8 * lane;
-    const uint16_t *srow = static_cast<const uint16_t *>(m.s) + (size_t)i * m.V;
-    const uint16_t *trow = static_cast<const uint16_t *>(m.t) + (size_t)i * m.V;
-    constexpr uint32_t NEG2 = 0xFF80FF80u;     // two bf16 -inf
-    uint4 ps[8], pt[8];
-#pragma unroll
-    for (int c = 0; c < 8; ++c) {
-        const int v = vw + 256 * c;
-        if (v < m.V) {                         // V % 8 == 0: a piece is wholly inside or wholly past the end
-            ps[c] = __ldcs(reinterpret_cast<const uint4 *>(srow + v));
-            pt[c] = __ldcs(reinterpret_cast<const uint4 *>(trow + v));
-        } else {
-            ps[c] = pt[c] = make_uint4(NEG2, NEG2, NEG2, NEG2);
+    uint32_t res;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "bar.red.or.pred q, 1, 256, p;\n\t"
+        "selp.u32 %0, 1, 0, q;\n\t}"
+        : "=r"(res)
+        : "r"((uint32_t)pred)
+        : "memory");
+    return res != 0;
+}
+
+}  // namespace
+
+const size_t kTrainRowsSmemBytes = ROWS_SMEM;
+const int kTrainRowsThreads = ROWS_THREADS;
+
+// grid min(SMs, P nch), ROWS_THREADS threads, ROWS_SMEM bytes: persistent
+// over the (position, chunk of TRAIN_ROW_CHUNK ids) items, position-major.
+// Warp 0 streams each item's s and t segments into a ROWS_STAGES-deep ring by
+// bulk copies; reducing warp w takes the 8-id pieces 32 w + lane + 256 c
+// (c < 8), so each of its shared-memory reads is one 512-byte run, and
+// releases the stage as soon as its pieces are in registers.  The warp's
+// maxima are reduced first, so every exponential is taken against the warp
+// maximum and the sums need no rescale.
+__global__ void __launch_bounds__(ROWS_THREADS, 1) k_train_rows(TrainMisc m)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
+    RowsShared &sh = *reinterpret_cast<RowsShared *>(base + ROWS_STAGES * 2 * ROWS_SEG);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int items = m.P * m.nch;
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < ROWS_STAGES; ++i) {
+            mbar_init(&sh.full[i], 1);
+            mbar_init(&sh.empty[i], 8);
         }
-    }
-    // the thread's ids increase along (c, word, half): a strict > keeps the first
-    float best = -INFINITY, mt = -INFINITY;
-    int idx = 0x7fffffff;
-#pragma unroll
-    for (int c = 0; c < 8; ++c) {
-        const uint32_t ws[4] = {ps[c].x, ps[c].y, ps[c].z, ps[c].w}, wt[4] = {pt[c].x, pt[c].y, pt[c].z, pt[c].w};
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const float s0 = __uint_as_float(ws[q] << 16), s1 = __uint_as_float(ws[q] & 0xFFFF0000u);
-            const int v = vw + 256 * c + 2 * q;
-            if (s0 > best) { best = s0; idx = v; }
-            if (s1 > best) { best = s1; idx = v + 1; }
-            mt = fmaxf(mt, fmaxf(__uint_as_float(wt[q] << 16), __uint_as_float(wt[q] & 0xFFFF0000u)));
-        }
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        const float ob = __shfl_xor_sync(0xffffffffu, best, o);
-        const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
-        mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, o));
-        merge_argmax(best, idx, ob, oi);
-    }
-    // best is now the warp's maximum of s (log2 domain below)
-    const float ms2 = best * L2E, mt2 = mt * L2E;
-    float ss[2] = {0.f, 0.f}, st[2] = {0.f, 0.f};
-    const bool has_s = best != -INFINITY, has_t = mt != -INFINITY;
-#pragma unroll
-    for (int c = 0; c < 8; ++c) {
-        const uint32_t ws[4] = {ps[c].x, ps[c].y, ps[c].z, ps[c].w}, wt[4] = {pt[c].x, pt[c].y, pt[c].z, pt[c].w};
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            if (has_s) {
-                ss[q & 1] += ex2_approx(fmaf(__uint_as_float(ws[q] << 16), L2E, -ms2));
-                ss[q & 1] += ex2_approx(fmaf(__uint_as_float(ws[q] & 0xFFFF0000u), L2E, -ms2));
-            }
-            if (has_t) {
-                st[q & 1] += ex2_approx(fmaf(__uint_as_float(wt[q] << 16), L2E, -mt2));
-                st[q & 1] += ex2_approx(fmaf(__uint_as_float(wt[q] & 0xFFFF0000u), L2E, -mt2));
-            }
-        }
-    }
-    float sum_s = ss[0] + ss[1], sum_t = st[0] + st[1];
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        sum_s += __shfl_xor_sync(0xffffffffu, sum_s, o);
-        sum_t += __shfl_xor_sync(0xffffffffu, sum_t, o);
-    }
-    __shared__ float4 wp[8];
-    __shared__ float wb[8];
-    __shared__ int wi[8];
-    if (lane == 0) {
-        wp[w] = make_float4(has_s ? ms2 : -INFINITY, sum_s, has_t ? mt2 : -INFINITY, sum_t);
-        wb[w] = best;
-        wi[w] = idx;
+        sh.abort = 0;
+        fence_barrier_init();
     }
     __syncthreads();
-    if (tid == 0) {
-        float4 a = wp[0];
-        float b = wb[0];
-        int bi = wi[0];
-        for (int k = 1; k < 8; ++k) {
-            lse2_merge(a.x, a.y, wp[k].x, wp[k].y);
-            lse2_merge(a.z, a.w, wp[k].z, wp[k].w);
-            merge_argmax(b, bi, wb[k], wi[k]);
+    pdl_trigger();
+    pdl_wait();
+    volatile int *abort = &sh.abort;
+    if (warp == 0) {
+        if (lane == 0) {
+            uint32_t pending = 0, pend_par = 0;
+            int k = 0;
+            for (int it = blockIdx.x; it < items; it += gridDim.x, ++k) {
+                const int st = k % ROWS_STAGES;
+                const uint32_t ph = (uint32_t)((k / ROWS_STAGES) & 1);
+                if (!mbar_wait(&sh.empty[st], ph ^ 1, abort)) break;
+                const int i = it / m.nch, v0 = (it % m.nch) * TRAIN_ROW_CHUNK;
+                // V % 8 == 0: the segment's bytes are a multiple of 16
+                const uint32_t bytes = (uint32_t)min(TRAIN_ROW_CHUNK, m.V - v0) * 2u;
+                uint8_t *dst = base + st * 2 * ROWS_SEG;
+                mbar_expect_tx(&sh.full[st], 2 * bytes);
+                bulk_load_1d(dst, static_cast<const uint16_t *>(m.s) + (size_t)i * m.V + v0, bytes, &sh.full[st]);
+                bulk_load_1d(dst + ROWS_SEG, static_cast<const uint16_t *>(m.t) + (size_t)i * m.V + v0, bytes,
+                             &sh.full[st]);
+                pending |= 1u << st;
+                pend_par = (pend_par & ~(1u << st)) | (ph << st);
+            }
+            if (*abort) {
+                // no copy may still be landing when the CTA leaves
+                int dummy = 0;
+                for (int st = 0; st < ROWS_STAGES; ++st)
+                    if (pending & (1u << st)) mbar_wait(&sh.full[st], (pend_par >> st) & 1, &dummy, 100000000ull);
+            }
         }
-        m.rpart[(size_t)i * m.nch + ch] = a;
-        m.rkey[(size_t)i * m.nch + ch] = argmax_key(b, bi);
+    } else {
+        const int w = warp - 1;
+        constexpr uint32_t NEG2 = 0xFF80FF80u;   // two bf16 -inf
+        int k = 0;
+        for (int it = blockIdx.x; it < items; it += gridDim.x, ++k) {
+            const int st = k % ROWS_STAGES;
+            const bool got = mbar_wait(&sh.full[st], (uint32_t)((k / ROWS_STAGES) & 1), abort);
+            if (rows_bar_or(!got)) break;
+            const int i = it / m.nch, ch = it % m.nch;
+            const int v0 = ch * TRAIN_ROW_CHUNK, n = min(TRAIN_ROW_CHUNK, m.V - v0);
+            const uint4 *ss = reinterpret_cast<const uint4 *>(base + st * 2 * ROWS_SEG);
+            const uint4 *tt = ss + ROWS_SEG / 16;
+            uint4 ps[8], pt[8];
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                const int pc = 32 * w + lane + 256 * c;
+                if (8 * pc < n) {
+                    ps[c] = ss[pc];
+                    pt[c] = tt[pc];
+                } else {
+                    ps[c] = pt[c] = make_uint4(NEG2, NEG2, NEG2, NEG2);
+                }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sh.empty[st]);
+            // the thread's ids increase along (c, word, half): a strict > keeps the first
+            const int vt = v0 + 8 * (32 * w + lane);
+            float best = -INFINITY, mt = -INFINITY;
+            int idx = 0x7fffffff;
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                const uint32_t ws[4] = {ps[c].x, ps[c].y, ps[c].z, ps[c].w};
+                const uint32_t wt[4] = {pt[c].x, pt[c].y, pt[c].z, pt[c].w};
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float s0 = __uint_as_float(ws[q] << 16), s1 = __uint_as_float(ws[q] & 0xFFFF0000u);
+                    const int v = vt + 2048 * c + 2 * q;
+                    if (s0 > best) { best = s0; idx = v; }
+                    if (s1 > best) { best = s1; idx = v + 1; }
+                    mt = fmaxf(mt, fmaxf(__uint_as_float(wt[q] << 16), __uint_as_float(wt[q] & 0xFFFF0000u)));
+                }
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+                const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
+                mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, o));
+                merge_argmax(best, idx, ob, oi);
+            }
+            // best is now the warp's maximum of s (log2 domain below)
+            const float ms2 = best * L2E, mt2 = mt * L2E;
+            const bool has_s = best != -INFINITY, has_t = mt != -INFINITY;
+            float sa[2] = {0.f, 0.f}, ta[2] = {0.f, 0.f};
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                const uint32_t ws[4] = {ps[c].x, ps[c].y, ps[c].z, ps[c].w};
+                const uint32_t wt[4] = {pt[c].x, pt[c].y, pt[c].z, pt[c].w};
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    if (has_s) {
+                        sa[q & 1] += ex2_approx(fmaf(__uint_as_float(ws[q] << 16), L2E, -ms2));
+                        sa[q & 1] += ex2_approx(fmaf(__uint_as_float(ws[q] & 0xFFFF0000u), L2E, -ms2));
+                    }
+                    if (has_t) {
+                        ta[q & 1] += ex2_approx(fmaf(__uint_as_float(wt[q] << 16), L2E, -mt2));
+                        ta[q & 1] += ex2_approx(fmaf(__uint_as_float(wt[q] & 0xFFFF0000u), L2E, -mt2));
+                    }
+                }
+            }
+            float sum_s = sa[0] + sa[1], sum_t = ta[0] + ta[1];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                sum_s += __shfl_xor_sync(0xffffffffu, sum_s, o);
+                sum_t += __shfl_xor_sync(0xffffffffu, sum_t, o);
+            }
+            // the 8 warps' partials (double-buffered by item parity: the
+            // merge of item k reads buffer k & 1 before the barrier of
+            // item k + 1, the writes of item k + 2 come after it)
+            const int pb = k & 1;
+            if (lane == 0) {
+                sh.wp[pb][w] = make_float4(has_s ? ms2 : -INFINITY, sum_s, has_t ? mt2 : -INFINITY, sum_t);
+                sh.wb[pb][w] = best;
+                sh.wi[pb][w] = idx;
+            }
+            asm volatile("bar.sync 1, 256;" ::: "memory");
+            if (w == 0 && lane == 0) {
+                float4 a = sh.wp[pb][0];
+                float b = sh.wb[pb][0];
+                int bi = sh.wi[pb][0];
+                for (int k2 = 1; k2 < 8; ++k2) {
+                    lse2_merge(a.x, a.y, sh.wp[pb][k2].x, sh.wp[pb][k2].y);
+                    lse2_merge(a.z, a.w, sh.wp[pb][k2].z, sh.wp[pb][k2].w);
+                    merge_argmax(b, bi, sh.wb[pb][k2], sh.wi[pb][k2]);
+                }
+                m.rpart[(size_t)i * m.nch + ch] = a;
+                m.rkey[(size_t)i * m.nch + ch] = argmax_key(b, bi);
+            }
+        }
     }
+    __syncthreads();
+    if (threadIdx.x == 0 && sh.abort) set_status(m.status, ST_TIMEOUT);
 }
 
 // grid ceil(P / 8), 256 threads: one warp per position.
