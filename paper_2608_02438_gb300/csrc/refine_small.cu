@@ -46,7 +46,7 @@ namespace {
 // ------------------------------------------------------------- shared memory
 
 struct RsShared {                              // Read CTA, after the W_r stages and z
-    uint64_t full[TV_STAGES], empty[TV_STAGES];
+    uint64_t full[RS_BSTAGES], empty[RS_BSTAGES];   // W_r blocks (64 KB stages)
     uint64_t z_full, z_empty, go;
     uint64_t tfull[TV_NBUF], tempty[TV_NBUF];
     uint64_t drain;
@@ -362,7 +362,7 @@ __device__ __forceinline__ void rowmax_item(const Params &p, int item, int lane)
 
 // ------------------------------------------------------------- Read role
 
-__device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tmap_wr, const CUtensorMap *tmap_wr32,
+__device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tmap_wrb, const CUtensorMap *tmap_wr32,
                                           const CUtensorMap *tmap_z, SmallCtl *c,
                           uint8_t *base, unsigned long long t_start)
 {
@@ -378,13 +378,12 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
     const int R1 = min(32 * (int)((long long)NQ * (r + 1) / S), V);
     const int nblk = (R1 - R0 + TV_BM - 1) / TV_BM;        // >= 1: S <= V / 128
     const int last_q = (R1 - R0 - (nblk - 1) * TV_BM + 31) / 32;   // quarters of the last block (1..4)
-    const int per_pass = nblk * TV_KCH;                    // W_r chunks per pass
-    const int ahead = min(TV_STAGES, per_pass);
+    const int ahead = min(RS_BSTAGES, nblk);               // W_r blocks issued ahead of the pass
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const bool tr = p.trace && r == 0;
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < TV_STAGES; ++i) { mbar_init(&sh.full[i], 1); mbar_init(&sh.empty[i], 1); }
+        for (int i = 0; i < RS_BSTAGES; ++i) { mbar_init(&sh.full[i], 1); mbar_init(&sh.empty[i], 1); }
         mbar_init(&sh.z_full, 1);
         mbar_init(&sh.z_empty, 1);
         mbar_init(&sh.go, 1);
@@ -397,7 +396,7 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
     if (warp == 1) { tmem_alloc(&sh.tmem_base, TV_TMEM_COLS); tmem_relinquish(); }
     const uint64_t keep = policy_evict_last();
     if (warp == 0 && lane == 0) {
-        tma_prefetch_desc(tmap_wr);
+        tma_prefetch_desc(tmap_wrb);
         tma_prefetch_desc(tmap_z);
     }
     tc_fence_before();
@@ -439,21 +438,24 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
             uint32_t pending = 0, pend_par = 0;            // last issue per stage (for the drain)
             bool z_issued = false;
             uint32_t z_par = 0;
+            // ci counts W_r blocks over the passes: block ci % nblk of the range
             auto issue = [&](long long ci) -> bool {
-                const int stage = (int)(ci % TV_STAGES);
-                const uint32_t ph = (uint32_t)((ci / TV_STAGES) & 1);
+                const int stage = (int)(ci % RS_BSTAGES);
+                const uint32_t ph = (uint32_t)((ci / RS_BSTAGES) & 1);
                 if (!mbar_wait(&sh.empty[stage], ph ^ 1, abort)) return false;
-                const int within = (int)(ci % per_pass), blk = within / TV_KCH, kx = (within % TV_KCH) * TV_BK;
+                const int blk = (int)(ci % nblk);
+                uint8_t *dst = sA + stage * RS_B_STAGE;
                 if (blk == nblk - 1 && last_q < 4) {
-                    // partial last block: its quarters only (the MMA's other rows
-                    // are stale and the epilogue leaves them out)
-                    mbar_expect_tx(&sh.full[stage], (uint32_t)last_q * (TV_A_STAGE / 4));
-                    for (int qq = 0; qq < last_q; ++qq)
-                        tma_load_2d_hint(sA + stage * TV_A_STAGE + qq * (TV_A_STAGE / 4), tmap_wr32, &sh.full[stage], kx,
-                                         R0 + blk * TV_BM + 32 * qq, keep);
+                    // partial last block: its quarters only, per K chunk (the
+                    // MMA's other rows are stale and the epilogue leaves them out)
+                    mbar_expect_tx(&sh.full[stage], (uint32_t)(last_q * TV_KCH) * (TV_A_STAGE / 4));
+                    for (int kc = 0; kc < TV_KCH; ++kc)
+                        for (int qq = 0; qq < last_q; ++qq)
+                            tma_load_2d_hint(dst + kc * TV_A_STAGE + qq * (TV_A_STAGE / 4), tmap_wr32, &sh.full[stage],
+                                             kc * TV_BK, R0 + blk * TV_BM + 32 * qq, keep);
                 } else {
-                    mbar_expect_tx(&sh.full[stage], TV_A_STAGE);
-                    tma_load_2d_hint(sA + stage * TV_A_STAGE, tmap_wr, &sh.full[stage], kx, R0 + blk * TV_BM, keep);
+                    mbar_expect_tx(&sh.full[stage], RS_B_STAGE);
+                    tma_load_3d_hint(dst, tmap_wrb, &sh.full[stage], 0, R0 + blk * TV_BM, 0, keep);
                 }
                 pending |= 1u << stage;
                 pend_par = (pend_par & ~(1u << stage)) | (ph << stage);
@@ -464,7 +466,7 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
             for (; next < ahead && ok; ++next) ok = issue(next);
             // while the first Trans runs, the rest of this CTA's W_r range
             // (past the chunks the ring holds) goes into L2 a slice at a time
-            const int pf_row0 = R0 + (ahead / TV_KCH) * TV_BM;
+            const int pf_row0 = R0 + ahead * TV_BM;
             const int pf_rows = max(0, R1 - pf_row0);
             const uint32_t pf_bytes = (uint32_t)pf_rows * RANK * 2;
             for (int pass = 0; ok; ++pass) {
@@ -488,13 +490,13 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
                 z_issued = true;
                 z_par = (uint32_t)(pass & 1);
                 // the rest of this pass, then the first chunks of the next one
-                const long long end = (long long)(pass + 1) * per_pass + ahead;
+                const long long end = (long long)(pass + 1) * nblk + ahead;
                 for (; next < end; ++next)
                     if (!issue(next)) { ok = false; break; }
             }
             // no copy may still be landing when the CTA leaves
             int dummy = 0;
-            for (int st = 0; st < TV_STAGES; ++st)
+            for (int st = 0; st < RS_BSTAGES; ++st)
                 if (pending & (1u << st)) mbar_wait(&sh.full[st], (pend_par >> st) & 1, &dummy, 100000000ull);
             if (z_issued) mbar_wait(&sh.z_full, z_par, &dummy, 100000000ull);
         }
@@ -514,19 +516,19 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
                     if (!mbar_wait(&sh.tempty[buf], (uint32_t)(((ib / TV_NBUF) & 1) ^ 1), abort)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t d = tmem + buf * TV_BN;
-                    for (int kc = 0; kc < TV_KCH; ++kc) {
-                        const long long ci = (long long)pass * per_pass + i * TV_KCH + kc;
-                        const int stage = (int)(ci % TV_STAGES);
-                        if (!mbar_wait(&sh.full[stage], (uint32_t)((ci / TV_STAGES) & 1), abort)) { ok = false; break; }
-                        tc_fence_after();
-                        const uint32_t a0 = smem_u32(sA + stage * TV_A_STAGE);
+                    const long long ci = (long long)pass * nblk + i;
+                    const int stage = (int)(ci % RS_BSTAGES);
+                    if (!mbar_wait(&sh.full[stage], (uint32_t)((ci / RS_BSTAGES) & 1), abort)) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t ab = smem_u32(sA + stage * RS_B_STAGE);
+#pragma unroll
+                    for (int kc = 0; kc < TV_KCH; ++kc)
 #pragma unroll
                         for (int kk = 0; kk < TV_BK / 16; ++kk)
-                            tc_mma_bf16(d, smem_desc_sw128(a0 + kk * 32), smem_desc_sw128(z0 + kc * TV_Z_CHUNK + kk * 32),
-                                        TV_IDESC, (kc | kk) != 0);
-                        tc_commit(&sh.empty[stage]);
-                    }
-                    if (ok) tc_commit(&sh.tfull[buf]);
+                            tc_mma_bf16(d, smem_desc_sw128(ab + kc * TV_A_STAGE + kk * 32),
+                                        smem_desc_sw128(z0 + kc * TV_Z_CHUNK + kk * 32), TV_IDESC, (kc | kk) != 0);
+                    tc_commit(&sh.empty[stage]);
+                    tc_commit(&sh.tfull[buf]);
                 }
                 if (!ok) break;
                 tc_commit(&sh.z_empty);
@@ -1221,7 +1223,7 @@ const size_t kRefineSmallSmemBytes = SMALL_SMEM;
 // one CTA per SM (10 warps: 3 on some of the 4 sub-partitions, hence <= 168
 // registers per thread).
 __global__ void __launch_bounds__(TV_THREADS, 1)
-    k_refine_small(const __grid_constant__ Params p, const __grid_constant__ CUtensorMap tmap_wr128,
+    k_refine_small(const __grid_constant__ Params p, const __grid_constant__ CUtensorMap tmap_wrb,
                    const __grid_constant__ CUtensorMap tmap_wr32, const __grid_constant__ CUtensorMap tmap_z)
 {
     const unsigned long long t_start = globaltimer_ns();
@@ -1239,7 +1241,7 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
         CtlLine *nxt = reinterpret_cast<CtlLine *>(&area->blk[par ^ 1]);
         nxt[threadIdx.x].v = 0;
     }
-    if ((int)blockIdx.x < p.S) read_role(p, &tmap_wr128, &tmap_wr32, &tmap_z, c, base, t_start);
+    if ((int)blockIdx.x < p.S) read_role(p, &tmap_wrb, &tmap_wr32, &tmap_z, c, base, t_start);
     else trans_role(p, c, base, t_start);
     __syncthreads();
     if (threadIdx.x == 0) leave(p, area, c, par);

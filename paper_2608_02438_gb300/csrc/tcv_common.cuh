@@ -21,6 +21,24 @@ constexpr uint32_t TV_Z_BYTES = TV_Z_CHUNK * TV_KCH;      // 16 KB
 constexpr uint32_t TV_TMEM_COLS = TV_NBUF * TV_BN;        // 128
 constexpr uint32_t TV_IDESC = idesc_bf16(TV_BM, TV_BN);
 
+// The persistent kernel streams W_r one 128-row block (all four 64-column K
+// chunks, 64 KB) per copy: a 3D tensor map (64 columns, rows, K chunk) whose
+// box lands as the four 16 KB K-chunk tiles of the 2D boxes, back to back.
+// Copies of 64 KB keep one issuing thread's stream well above what 16 KB
+// boxes reach.
+constexpr int RS_BSTAGES = TV_STAGES / TV_KCH;          // W_r blocks in flight
+constexpr uint32_t RS_B_STAGE = TV_KCH * TV_A_STAGE;   // 64 KB
+
+__device__ __forceinline__ void tma_load_3d_hint(void *smem_dst, const CUtensorMap *map, uint64_t *bar, int x, int y,
+                                                 int z, uint64_t policy)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1, {%2, "
+        "%3, %4}], [%5], %6;" ::"r"(smem_u32(smem_dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)), "l"(policy)
+        : "memory");
+}
+
 __device__ __forceinline__ void tv_epi_bar() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
 
 __device__ __forceinline__ bool tv_epi_bar_or(bool pred)

@@ -1,8 +1,8 @@
 // train_common.cuh -- device helpers of the training-step kernels
 // (train_read.cu, train_gemm.cu, train_kernels.cu) on top of common.cuh:
 // MN-major shared-memory descriptors, the A-from-tensor-memory MMA, TMEM
-// stores and 16-column loads, a tensor-map L2 prefetch and a polling
-// bounded wait.
+// stores and 16-column loads, a tensor-map L2 prefetch, a polling bounded
+// wait and a vector reduction into global memory.
 #pragma once
 
 #include "common.cuh"
@@ -103,6 +103,15 @@ __device__ __forceinline__ uint64_t smem_desc_sw128_mn(uint32_t saddr, uint32_t 
 {
     return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)((mn_stride >> 4) & 0x3FFFu) << 16) |
            ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+// Adds four floats into 16-byte aligned global memory with one vector
+// reduction (relaxed, GPU scope).
+__device__ __forceinline__ void red_add_v4(float *dst, float a, float b, float c, float d)
+{
+    asm volatile("red.relaxed.gpu.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(dst), "f"(a), "f"(b), "f"(c),
+                 "f"(d)
+                 : "memory");
 }
 
 // Packs two floats as bf16 (round to nearest even): lo in bits 0-15.

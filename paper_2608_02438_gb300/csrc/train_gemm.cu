@@ -136,7 +136,16 @@ __global__ void __launch_bounds__(192, 1)
                 const int nv = min(32, g.N - n);
                 if (g.mode == GM_ADD) {
                     float *dst = g.C + (size_t)m * g.ldc + n;
-                    for (int jj = 0; jj < nv; ++jj) atomicAdd(dst + jj, g.alpha * v[jj]);
+                    if (nv == 32 && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
+#pragma unroll
+                        for (int e = 0; e < 8; ++e)
+                            red_add_v4(dst + 4 * e, g.alpha * v[4 * e], g.alpha * v[4 * e + 1], g.alpha * v[4 * e + 2],
+                                       g.alpha * v[4 * e + 3]);
+                    } else {
+#pragma unroll
+                        for (int jj = 0; jj < 32; ++jj)
+                            if (jj < nv) atomicAdd(dst + jj, g.alpha * v[jj]);
+                    }
                     continue;
                 }
                 float x[32];
@@ -157,7 +166,9 @@ __global__ void __launch_bounds__(192, 1)
                             reinterpret_cast<float4 *>(dst)[e] =
                                 make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
                     } else {
-                        for (int jj = 0; jj < nv; ++jj) dst[jj] = x[jj];
+#pragma unroll
+                        for (int jj = 0; jj < 32; ++jj)
+                            if (jj < nv) dst[jj] = x[jj];
                     }
                 }
                 if (g.Cb) {
@@ -174,7 +185,9 @@ __global__ void __launch_bounds__(192, 1)
                                            pack_bf16x2(x[8 * e + 4], x[8 * e + 5]),
                                            pack_bf16x2(x[8 * e + 6], x[8 * e + 7]));
                     } else {
-                        for (int jj = 0; jj < nv; ++jj) dst[jj] = f2bf(x[jj]);
+#pragma unroll
+                        for (int jj = 0; jj < 32; ++jj)
+                            if (jj < nv) dst[jj] = f2bf(x[jj]);
                     }
                 }
             }

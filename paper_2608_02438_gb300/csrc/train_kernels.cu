@@ -425,7 +425,9 @@ __global__ void __launch_bounds__(1024) k_train_mix_bwd(TrainMisc m)
         for (int jj = 0; jj < MAX_B; ++jj)
             if (jj < j) gl[jj] = fmaf(dcj, sa[jj * 32 + dl], gl[jj]);
     }
-    for (int jj = 0; jj < j; ++jj) atomicAdd(m.gL + ((size_t)d * B + j) * B + jj, gl[jj]);
+#pragma unroll
+    for (int jj = 0; jj < MAX_B; ++jj)
+        if (jj < j) atomicAdd(m.gL + ((size_t)d * B + j) * B + jj, gl[jj]);
 }
 
 // grid NR / 8, 256 threads: one warp per row.  The row's log-sum-exp from the

@@ -51,6 +51,23 @@ bool make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t inner, uint64_t o
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// W_r [rows][r] bf16 viewed as (64 columns, rows, r / 64 K chunks of 64
+// columns, 128 bytes apart): a box of 64 x box_rows x r / 64 lands in shared
+// memory as the K-chunk tiles of 2D boxes of 64 x box_rows, back to back, with
+// the same 128-byte swizzle.
+bool make_tmap_bf16_kblocks(CUtensorMap *m, const void *base, uint64_t rows, uint32_t box_rows)
+{
+    auto enc = tensor_map_encoder();
+    if (!enc) return false;
+    cuuint64_t dims[3] = {64, rows, RANK / 64};
+    cuuint64_t strides[2] = {RANK * 2, 128};
+    cuuint32_t box[3] = {64, box_rows, RANK / 64};
+    cuuint32_t es[3] = {1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 struct GraphEntry {
     bool used = false;
     void *ws = nullptr;
@@ -86,7 +103,8 @@ struct xpress_refiner {
     float *Ep = nullptr;
     unsigned long long *trace = nullptr;   // profiling timeline (XPRESS_TRACE=1)
     CUtensorMap tmap_wr{};                 // W_r boxes of 256 rows (k_read_tc)
-    CUtensorMap tmap_wr128{};              // W_r boxes of 128 rows (k_read_tcv, k_refine_small)
+    CUtensorMap tmap_wr128{};              // W_r boxes of 128 rows (k_read_tcv, the training step)
+    CUtensorMap tmap_wrb{};                // W_r as (64 columns, rows, 4 K chunks): one 128-row block per box (k_refine_small)
     CUtensorMap tmap_wr32{};               // W_r boxes of 32 rows (k_refine_small, partial blocks)
     CUtensorMap tmap_wh{}, tmap_wg{};      // W_h, W_g boxes of 256 rows x 64
     CUtensorMap tmap_fhi{}, tmap_flo{};    // folded projection, hi / lo term, boxes of 256 rows x 64 (k_pre_tc)
@@ -653,7 +671,7 @@ int run_small(xpress_refiner *R, const Params &P, const Layout &L, void *ws, cud
     cfg.stream = st;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    XP_CUDA(cudaLaunchKernelEx(&cfg, k_refine_small, P, R->tmap_wr128, R->tmap_wr32, tmap_z));
+    XP_CUDA(cudaLaunchKernelEx(&cfg, k_refine_small, P, R->tmap_wrb, R->tmap_wr32, tmap_z));
     if (R->trace) print_trace(R, st);
     return XPRESS_OK;
 }
@@ -748,6 +766,7 @@ int xpress_refiner_create(const xpress_weights *w, void *stream, xpress_refiner 
         if (R->use_tc && (!make_tmap_bf16(&R->tmap_wr, w->W_r, RANK, (uint64_t)w->V, 64, 256) ||
                           !make_tmap_bf16(&R->tmap_wr128, w->W_r, RANK, (uint64_t)w->V, 64, 128) ||
                           !make_tmap_bf16(&R->tmap_wr32, w->W_r, RANK, (uint64_t)w->V, 64, 32) ||
+                          !make_tmap_bf16_kblocks(&R->tmap_wrb, w->W_r, (uint64_t)w->V, 128) ||
                           !make_tmap_bf16(&R->tmap_wh, w->W_h, (uint64_t)w->H, RANK, 64, 256) ||
                           !make_tmap_bf16(&R->tmap_wg, w->W_g, (uint64_t)w->H, RANK, 64, 256))) {
             rc = XPRESS_ERR_CUDA;
