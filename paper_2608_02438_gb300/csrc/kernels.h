@@ -59,11 +59,13 @@ constexpr int TCV_MAX_TOKENS = 32;
 // refine_small.cu (at most 32 evaluated tokens, bf16: the whole call in one
 // persistent cooperative kernel of S Read CTAs + SMALL_TRANS_CTAS Trans CTAs)
 __global__ void k_refine_small(const __grid_constant__ Params p, const __grid_constant__ CUtensorMap tmap_wrb,
-                               const __grid_constant__ CUtensorMap tmap_wr32, const __grid_constant__ CUtensorMap tmap_z);
+                               const __grid_constant__ CUtensorMap tmap_wr32, const __grid_constant__ CUtensorMap tmap_z,
+                               const __grid_constant__ CUtensorMap tmap_f, const __grid_constant__ CUtensorMap tmap_h);
 __global__ void k_fold_hidden(const uint16_t *W_h, const uint16_t *W_g, const uint16_t *W_in, uint16_t *Fhl, int H);
 __global__ void k_pack_L(const uint16_t *L, uint16_t *Lpk, int B);
 extern const size_t kRefineSmallSmemBytes;
 constexpr int SMALL_TRANS_CTAS = 8;
+constexpr int SMALL_PC_KT = 8;              // 64-wide K tiles per precompute copy of the persistent kernel
 
 // trans_tc.cu (bf16, more than 32 tokens: Fuse + Mix, then Trans on tcgen05)
 __global__ void k_mix_c(const Params *pp);

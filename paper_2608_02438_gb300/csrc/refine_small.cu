@@ -16,8 +16,9 @@
 //     (Algorithm 1's Y^(0)).  In every pass they run Read + Correct +
 //     selection (Eq. read / correct, the argmax or the fixed-noise group
 //     draw) over a fixed range of vocabulary rows (128-row blocks): W_r rows
-//     are the tcgen05 M dimension, the <= 32 tokens N, and an 8-stage TMA ring
-//     streams W_r, running ahead into the next pass while the Trans CTAs work.
+//     are the tcgen05 M dimension, the <= 32 tokens N, and a TMA ring of two
+//     64 KB blocks (one copy per block) streams W_r, running ahead into the
+//     next pass while the Trans CTAs work.
 //     Each range leaves one result per token (greedy: an argmax key; T > 0: a
 //     partial with the member draw of its best group already taken).
 //   Trans CTAs (S .. S + 7).  CTA j owns channels [32 j, 32 j + 32).  In every
@@ -45,12 +46,14 @@ namespace {
 
 // ------------------------------------------------------------- shared memory
 
+constexpr int PC_BUFS_MAX = 5;                 // precompute ring buffers (at most)
+
 struct RsShared {                              // Read CTA, after the W_r stages and z
     uint64_t full[RS_BSTAGES], empty[RS_BSTAGES];   // W_r blocks (64 KB stages)
     uint64_t z_full, z_empty, go;
     uint64_t tfull[TV_NBUF], tempty[TV_NBUF];
     uint64_t drain;
-    uint64_t pfull[3], pempty[3];              // precompute ring (h and F chunks)
+    uint64_t pfull[PC_BUFS_MAX], pempty[PC_BUFS_MAX];   // precompute ring (h and F chunks)
     uint32_t tmem_base;
     int abort;
     int pass_n, pass_stop;                     // published by the producer with `go`
@@ -178,55 +181,63 @@ __device__ __forceinline__ void leave(const Params &p, SmallCtlArea *a, SmallCtl
 //   Pc_k = P_k + sum_{j<k} L_kj P_j (Eq. mix, per channel), written to pcx;
 //   with a draft also the first pass's c_k = Pc_k + e_k + sum_{j<k} L_kj e_j
 //   (e_k = E'[x_{k-1}], Eq. fuse / mix), written to c0x.
-// K is streamed through a 3-buffer ring of bulk copies (warp 0 issues them):
-// per chunk the unit's 8 F rows ([lo][slot h / g][channel]) and the N rows of
-// h, each row at a pitch of 64 mod 128 bytes so that the fragment loads below
-// hit distinct banks.
-constexpr int PC_BUFS = 3;
+// K is streamed through a ring of TMA copies (warp 0 issues them), two per
+// chunk of PC_KT 64-wide K tiles: the unit's 8 F rows ([lo][slot h / g]
+// [channel], one 5D box of the folded projection) and the NT rows of h (one 3D
+// box; rows past N and tiles past H are zero-filled).  Both land as
+// [K tile][row][128 bytes] with the 128-byte swizzle: the 16-byte piece j of
+// row i of a tile sits at piece j ^ (i & 7).
 constexpr int PC_ROWS = 8;
+constexpr int PC_KT = SMALL_PC_KT;                            // 64-wide K tiles per chunk
+constexpr int PC_KC = 64 * PC_KT;                             // K per chunk (a multiple of 8 warps x 32)
 template <int NT>
 struct PcShape {
-    static constexpr int KC = NT <= 16 ? 768 : 512;          // K per chunk (a multiple of 8 warps x 32)
-    static constexpr int PITCH = 2 * KC + 64;                // bytes per row
-    static constexpr int BUF = (PC_ROWS + NT) * PITCH;
+    static constexpr int F_BYTES = PC_KT * PC_ROWS * 128;        // 8 KB
+    static constexpr int H_BYTES = PC_KT * NT * 128;             // 16 or 32 KB
+    static constexpr int BUF = F_BYTES + H_BYTES;
+    static constexpr int BUFS = NT <= 16 ? 5 : 3;
 };
-static_assert(PC_BUFS * PcShape<16>::BUF <= (int)(TV_STAGES * TV_A_STAGE + TV_Z_BYTES), "precompute ring");
-static_assert(PC_BUFS * PcShape<32>::BUF <= (int)(TV_STAGES * TV_A_STAGE + TV_Z_BYTES), "precompute ring");
+static_assert(PcShape<16>::BUFS * PcShape<16>::BUF <= (int)(TV_STAGES * TV_A_STAGE + TV_Z_BYTES), "precompute ring");
+static_assert(PcShape<32>::BUFS * PcShape<32>::BUF <= (int)(TV_STAGES * TV_A_STAGE + TV_Z_BYTES), "precompute ring");
+static_assert(PcShape<16>::BUFS <= PC_BUFS_MAX && PcShape<32>::BUFS <= PC_BUFS_MAX, "precompute barriers");
 
-// Warp 0, one lane: the chunk copies of every unit of this CTA.
+__device__ __forceinline__ void tma_load_5d(void *smem_dst, const CUtensorMap *map, uint64_t *bar, int c0, int c1, int c2,
+                                            int c3, int c4)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.5d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5, %6}], "
+        "[%7];" ::"r"(smem_u32(smem_dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4), "r"(smem_u32(bar))
+        : "memory");
+}
+
+// Warp 0, one lane: the chunk copies of every unit of this CTA.  tmap_f: the
+// folded projection as (64 columns, 2r rows of a slot, slot, term, K tile);
+// tmap_h: h as (64 columns, N rows, K tile).
 template <int NT>
-__device__ __forceinline__ void pc_produce(const Params &p, uint8_t *ring, RsShared &sh, int r, int S,
-                                           volatile int *abort)
+__device__ __forceinline__ void pc_produce(const Params &p, const CUtensorMap *tmap_f, const CUtensorMap *tmap_h,
+                                           uint8_t *ring, RsShared &sh, int r, int S, volatile int *abort)
 {
     using Sh = PcShape<NT>;
-    const int H = p.H, N = p.N, nchk = (H + Sh::KC - 1) / Sh::KC;
-    const uint16_t *h = static_cast<const uint16_t *>(p.h);
-    const size_t lo_off = (size_t)2 * RANK * H;
+    const int nchk = (p.H + PC_KC - 1) / PC_KC;
     uint32_t pending = 0, pend_par = 0;
     int ci = 0;
     bool ok = true;
     for (int unit = r; unit < RANK / 2 && ok; unit += S)
         for (int kc = 0; kc < nchk; ++kc, ++ci) {
-            const int buf = ci % PC_BUFS;
-            const uint32_t ph = (uint32_t)((ci / PC_BUFS) & 1);
+            const int buf = ci % Sh::BUFS;
+            const uint32_t ph = (uint32_t)((ci / Sh::BUFS) & 1);
             if (!mbar_wait(&sh.pempty[buf], ph ^ 1, abort)) { ok = false; break; }
-            const int kb = kc * Sh::KC, kl = min(Sh::KC, H - kb);
-            const uint32_t bytes = (uint32_t)kl * 2;
             uint8_t *dst = ring + buf * Sh::BUF;
-            mbar_expect_tx(&sh.pfull[buf], bytes * (uint32_t)(PC_ROWS + N));
-            for (int m = 0; m < PC_ROWS; ++m) {
-                const int lo = m >> 2, slot = (m >> 1) & 1, ch = m & 1;
-                bulk_load_1d(dst + m * Sh::PITCH, p.Fhl + lo * lo_off + (size_t)(slot * RANK + 2 * unit + ch) * H + kb,
-                             bytes, &sh.pfull[buf]);
-            }
-            for (int t = 0; t < N; ++t)
-                bulk_load_1d(dst + (PC_ROWS + t) * Sh::PITCH, h + (size_t)t * H + kb, bytes, &sh.pfull[buf]);
+            mbar_expect_tx(&sh.pfull[buf], (uint32_t)Sh::BUF);
+            tma_load_5d(dst, tmap_f, &sh.pfull[buf], 0, 2 * unit, 0, 0, kc * PC_KT);
+            tma_load_3d(dst + Sh::F_BYTES, tmap_h, &sh.pfull[buf], 0, 0, kc * PC_KT);
             pending |= 1u << buf;
             pend_par = (pend_par & ~(1u << buf)) | (ph << buf);
         }
     // no copy may still be landing when the ring is reused
     int dummy = 0;
-    for (int b2 = 0; b2 < PC_BUFS; ++b2)
+    for (int b2 = 0; b2 < Sh::BUFS; ++b2)
         if (pending & (1u << b2)) mbar_wait(&sh.pfull[b2], (pend_par >> b2) & 1, &dummy, 100000000ull);
 }
 
@@ -234,13 +245,13 @@ __device__ __forceinline__ void pc_produce(const Params &p, uint8_t *ring, RsSha
 // w, w + 8, ... of every chunk (m16n8k16: A = the unit's F rows, hi in rows
 // 0-7 and lo in rows 8-15, B = h, tokens in 8-column tiles).  The 16 K values
 // of one product are taken from 32 consecutive ones, the same for A and B, so
-// each operand is one 16-byte load per lane.
+// each operand is one 16-byte load per lane (one swizzled piece of a row).
 template <int NT>
 __device__ __forceinline__ void pc_consume(const Params &p, uint8_t *ring, RsShared &sh, int r, int S, int w,
                                            int lane, volatile int *abort, bool tm, unsigned long long t_start)
 {
     using Sh = PcShape<NT>;
-    const int H = p.H, N = p.N, B = p.B, V = p.V, nchk = (H + Sh::KC - 1) / Sh::KC;
+    const int H = p.H, N = p.N, B = p.B, V = p.V, nchk = (H + PC_KC - 1) / PC_KC;
     const int g = lane >> 2, tq = lane & 3, et = w * 32 + lane;
     const int TRI = B * (B - 1) / 2;
     float *us = &sh.bestx[0][0][0];                               // U [4][32]: rows (slot, channel)
@@ -263,26 +274,28 @@ __device__ __forceinline__ void pc_consume(const Params &p, uint8_t *ring, RsSha
 #pragma unroll
         for (int nt = 0; nt < NT / 8; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.0f;
         for (int kc = 0; kc < nchk; ++kc, ++ci) {
-            const int buf = ci % PC_BUFS;
-            if (ok && !mbar_wait(&sh.pfull[buf], (uint32_t)((ci / PC_BUFS) & 1), abort)) ok = false;
+            const int buf = ci % Sh::BUFS;
+            if (ok && !mbar_wait(&sh.pfull[buf], (uint32_t)((ci / Sh::BUFS) & 1), abort)) ok = false;
             if (ok) {
                 if (tm && kc == 0) trace_mark(p.trace, 5, t_start);
-                const int kl = min(Sh::KC, H - kc * Sh::KC);
-                const uint8_t *fb = ring + buf * Sh::BUF;
-                const uint8_t *fhi = fb + (g & 3) * Sh::PITCH, *flo = fb + (4 + (g & 3)) * Sh::PITCH;
-                const uint8_t *hr = fb + (PC_ROWS + g) * Sh::PITCH;
+                const int kl = min(PC_KC, H - kc * PC_KC);
+                const uint8_t *fb = ring + buf * Sh::BUF, *hb = fb + Sh::F_BYTES;
+                const int mh = g & 3, ml = 4 + (g & 3);             // F rows of the hi and lo terms
 #pragma unroll 1
                 for (int ks = w; ks * 32 < kl; ks += 8) {
                     const int ko = ks * 32 + 8 * tq;
                     const bool v = ko < kl;
+                    const int tile = ko >> 6, pc = (ko >> 3) & 7;
                     const uint4 z4 = make_uint4(0u, 0u, 0u, 0u);
-                    const uint4 ah = v ? *reinterpret_cast<const uint4 *>(fhi + 2 * ko) : z4;
-                    const uint4 al = v ? *reinterpret_cast<const uint4 *>(flo + 2 * ko) : z4;
+                    const uint8_t *ft = fb + tile * (PC_ROWS * 128);
+                    const uint4 ah = v ? *reinterpret_cast<const uint4 *>(ft + mh * 128 + ((pc ^ mh) << 4)) : z4;
+                    const uint4 al = v ? *reinterpret_cast<const uint4 *>(ft + ml * 128 + ((pc ^ ml) << 4)) : z4;
                     const uint32_t a0[4] = {ah.x, al.x, ah.y, al.y}, a1[4] = {ah.z, al.z, ah.w, al.w};
+                    const uint8_t *ht = hb + tile * (NT * 128) + g * 128 + ((pc ^ g) << 4);
 #pragma unroll
                     for (int nt = 0; nt < NT / 8; ++nt) {
                         const uint4 bb = (v && nt * 8 + g < N)
-                                             ? *reinterpret_cast<const uint4 *>(hr + nt * 8 * Sh::PITCH + 2 * ko)
+                                             ? *reinterpret_cast<const uint4 *>(ht + nt * 8 * 128)
                                              : z4;
                         mma_bf16_16816(acc[nt], a0, bb.x, bb.y);
                         mma_bf16_16816(acc[nt], a1, bb.z, bb.w);
@@ -363,7 +376,8 @@ __device__ __forceinline__ void rowmax_item(const Params &p, int item, int lane)
 // ------------------------------------------------------------- Read role
 
 __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tmap_wrb, const CUtensorMap *tmap_wr32,
-                                          const CUtensorMap *tmap_z, SmallCtl *c,
+                                          const CUtensorMap *tmap_z, const CUtensorMap *tmap_f, const CUtensorMap *tmap_h,
+                                          SmallCtl *c,
                           uint8_t *base, unsigned long long t_start)
 {
     uint8_t *sA = base;                                    // W_r stages (h slices before the first pass)
@@ -389,13 +403,15 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
         mbar_init(&sh.go, 1);
         for (int i = 0; i < TV_NBUF; ++i) { mbar_init(&sh.tfull[i], 1); mbar_init(&sh.tempty[i], 4); }
         mbar_init(&sh.drain, 1);
-        for (int i = 0; i < PC_BUFS; ++i) { mbar_init(&sh.pfull[i], 1); mbar_init(&sh.pempty[i], TV_EPI_WARPS); }
+        for (int i = 0; i < PC_BUFS_MAX; ++i) { mbar_init(&sh.pfull[i], 1); mbar_init(&sh.pempty[i], TV_EPI_WARPS); }
         sh.abort = 0;
         fence_barrier_init();
     }
     if (warp == 1) { tmem_alloc(&sh.tmem_base, TV_TMEM_COLS); tmem_relinquish(); }
     const uint64_t keep = policy_evict_last();
     if (warp == 0 && lane == 0) {
+        tma_prefetch_desc(tmap_f);
+        tma_prefetch_desc(tmap_h);
         tma_prefetch_desc(tmap_wrb);
         tma_prefetch_desc(tmap_z);
     }
@@ -410,8 +426,8 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
     // argmaxes of s
     if (warp == 0) {
         if (lane == 0) {
-            if (N <= 16) pc_produce<16>(p, sA, sh, r, S, abort);
-            else pc_produce<32>(p, sA, sh, r, S, abort);
+            if (N <= 16) pc_produce<16>(p, tmap_f, tmap_h, sA, sh, r, S, abort);
+            else pc_produce<32>(p, tmap_f, tmap_h, sA, sh, r, S, abort);
         }
     } else if (warp >= 2) {
         const int w = warp - 2;
@@ -806,13 +822,22 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
     const int g = lane >> 2, tq = lane & 3, khalf = (warp >> 2) & 1;
     const bool lead = rank == 0;
 
-    // static operands: W_1 / W_2 fragments (warps 0-7) and L's strictly lower
-    // part for the kept channels
+    // static operands: W_1 / W_2 fragments and L's strictly lower part for the
+    // kept channels (warps 0-7).  Meanwhile warps 8 and 9 run the B = 16 mix
+    // once on scratch operands, so that its code (a non-inlined function) is
+    // cached before the first pass needs it (cop and cown are rewritten before
+    // their first use; e, pc and Lp hold whatever is there).
     MlpFrags fr;
-    if (warp < 8) load_mlp_frags(p, rank, fr);
-    for (int i = tid; i < TRI * CH / 8; i += nth) {            // 16-byte pieces of the kept channels
-        const int q = i / (CH / 8), c8 = i % (CH / 8);
-        reinterpret_cast<uint4 *>(Lp)[i] = __ldg(reinterpret_cast<const uint4 *>(p.Lpk + (size_t)q * RANK + cb) + c8);
+    if (warp < 8) {
+        load_mlp_frags(p, rank, fr);
+        for (int i = tid; i < TRI * CH / 8; i += 256) {          // 16-byte pieces of the kept channels
+            const int q = i / (CH / 8), c8 = i % (CH / 8);
+            reinterpret_cast<uint4 *>(Lp)[i] = __ldg(reinterpret_cast<const uint4 *>(p.Lpk + (size_t)q * RANK + cb) + c8);
+        }
+    } else if (full && B == FULL_C_MAX_B) {
+        const int d = 2 * (tid & 127);
+        if (warp == 8) mix_block16<0>(e, Lp, pc, cop, sh.cown, d, -1, B - 1, 0, rank);
+        else mix_block16<1>(e, Lp, pc, cop, sh.cown, d, -1, B - 1, 0, rank);
     }
     if (tid < N) { sh.tpos[tid] = tid % B; sh.tseq[tid] = tid / B; }
     // Y^(0) from the draft; the lead CTA writes the state of the first pass
@@ -854,13 +879,6 @@ __device__ __forceinline__ void trans_role(const Params &p, SmallCtl *c, uint8_t
         sh.anch[tid] = p.anchor[tid];
         const float T = p.temperature[tid];
         sh.invT[tid] = T > 0.0f ? 1.0f / T : 0.0f;
-    }
-    if (full && B == FULL_C_MAX_B && tid < 2 * 128) {
-        // warm the mix's code on scratch operands (cop and cown are rewritten
-        // before their first use; e and pc hold whatever is there)
-        const int d = 2 * (tid & 127);
-        if (tid < 128) mix_block16<0>(e, Lp, pc, cop, sh.cown, d, -1, B - 1, 0, rank);
-        else mix_block16<1>(e, Lp, pc, cop, sh.cown, d, -1, B - 1, 0, rank);
     }
     if (lead && tid == 0 && p.trace) trace_mark(p.trace, 250, t_start);
     if (tid == 0) sh.go = wait_count(c, &c->pre_done.v, (unsigned)p.S, p.wait_ns);
@@ -1224,7 +1242,8 @@ const size_t kRefineSmallSmemBytes = SMALL_SMEM;
 // registers per thread).
 __global__ void __launch_bounds__(TV_THREADS, 1)
     k_refine_small(const __grid_constant__ Params p, const __grid_constant__ CUtensorMap tmap_wrb,
-                   const __grid_constant__ CUtensorMap tmap_wr32, const __grid_constant__ CUtensorMap tmap_z)
+                   const __grid_constant__ CUtensorMap tmap_wr32, const __grid_constant__ CUtensorMap tmap_z,
+                   const __grid_constant__ CUtensorMap tmap_f, const __grid_constant__ CUtensorMap tmap_h)
 {
     const unsigned long long t_start = globaltimer_ns();
     // a kernel launched after this one with programmatic dependent launch may
@@ -1241,7 +1260,7 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
         CtlLine *nxt = reinterpret_cast<CtlLine *>(&area->blk[par ^ 1]);
         nxt[threadIdx.x].v = 0;
     }
-    if ((int)blockIdx.x < p.S) read_role(p, &tmap_wrb, &tmap_wr32, &tmap_z, c, base, t_start);
+    if ((int)blockIdx.x < p.S) read_role(p, &tmap_wrb, &tmap_wr32, &tmap_z, &tmap_f, &tmap_h, c, base, t_start);
     else trans_role(p, c, base, t_start);
     __syncthreads();
     if (threadIdx.x == 0) leave(p, area, c, par);

@@ -29,6 +29,14 @@ constexpr uint32_t TV_IDESC = idesc_bf16(TV_BM, TV_BN);
 constexpr int RS_BSTAGES = TV_STAGES / TV_KCH;          // W_r blocks in flight
 constexpr uint32_t RS_B_STAGE = TV_KCH * TV_A_STAGE;   // 64 KB
 
+__device__ __forceinline__ void tma_load_3d(void *smem_dst, const CUtensorMap *map, uint64_t *bar, int x, int y, int z)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];"
+        ::"r"(smem_u32(smem_dst)), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+        : "memory");
+}
+
 __device__ __forceinline__ void tma_load_3d_hint(void *smem_dst, const CUtensorMap *map, uint64_t *bar, int x, int y,
                                                  int z, uint64_t policy)
 {

@@ -68,6 +68,38 @@ bool make_tmap_bf16_kblocks(CUtensorMap *m, const void *base, uint64_t rows, uin
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The folded projection Fhl [term 2][slot 2][r rows][H] bf16 as a 5D map
+// (64 columns, r rows of a slot, slot, term, H / 64 K tiles of 128 bytes): a
+// box of 64 x 2 x 2 x 2 x kt holds the 8 rows (term, slot, channel pair) of
+// one unit over kt K tiles, landing as [K tile][row][128 bytes].
+bool make_tmap_fold_k(CUtensorMap *m, const void *Fhl, uint64_t H, uint32_t kt)
+{
+    auto enc = tensor_map_encoder();
+    if (!enc) return false;
+    cuuint64_t dims[5] = {64, RANK, 2, 2, H / 64};
+    cuuint64_t strides[4] = {H * 2, (cuuint64_t)RANK * H * 2, (cuuint64_t)2 * RANK * H * 2, 128};
+    cuuint32_t box[5] = {64, 2, 2, 2, kt};
+    cuuint32_t es[5] = {1, 1, 1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void *>(Fhl), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// h [N][H] bf16 as (64 columns, N rows, H / 64 K tiles): a box of
+// 64 x rows x kt lands as [K tile][row][128 bytes] (rows past N zero).
+bool make_tmap_rows_k(CUtensorMap *m, const void *h, uint64_t N, uint64_t H, uint32_t rows, uint32_t kt)
+{
+    auto enc = tensor_map_encoder();
+    if (!enc) return false;
+    cuuint64_t dims[3] = {64, N, H / 64};
+    cuuint64_t strides[2] = {H * 2, 128};
+    cuuint32_t box[3] = {64, rows, kt};
+    cuuint32_t es[3] = {1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(h), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 struct GraphEntry {
     bool used = false;
     void *ws = nullptr;
@@ -105,6 +137,7 @@ struct xpress_refiner {
     CUtensorMap tmap_wr{};                 // W_r boxes of 256 rows (k_read_tc)
     CUtensorMap tmap_wr128{};              // W_r boxes of 128 rows (k_read_tcv, the training step)
     CUtensorMap tmap_wrb{};                // W_r as (64 columns, rows, 4 K chunks): one 128-row block per box (k_refine_small)
+    CUtensorMap tmap_fk{};                 // folded projection as (64 columns, rows of a slot, slot, term, K tile) (k_refine_small)
     CUtensorMap tmap_wr32{};               // W_r boxes of 32 rows (k_refine_small, partial blocks)
     CUtensorMap tmap_wh{}, tmap_wg{};      // W_h, W_g boxes of 256 rows x 64
     CUtensorMap tmap_fhi{}, tmap_flo{};    // folded projection, hi / lo term, boxes of 256 rows x 64 (k_pre_tc)
@@ -655,8 +688,10 @@ int run_small(xpress_refiner *R, const Params &P, const Layout &L, void *ws, cud
         R->small_ws[R->small_ws_next] = ws;
         R->small_ws_next = (R->small_ws_next + 1) % CACHE_SLOTS;
     }
-    CUtensorMap tmap_z{};
-    if (!make_tmap_bf16(&tmap_z, P.zpack, RANK, (uint64_t)P.N, 64, 32)) return XPRESS_ERR_CUDA;
+    CUtensorMap tmap_z{}, tmap_h{};
+    if (!make_tmap_bf16(&tmap_z, P.zpack, RANK, (uint64_t)P.N, 64, 32) ||
+        !make_tmap_rows_k(&tmap_h, P.h, (uint64_t)P.N, (uint64_t)P.H, P.N <= 16 ? 16 : 32, SMALL_PC_KT))
+        return XPRESS_ERR_CUDA;
     if (R->trace) {
         XP_CUDA(cudaMemsetAsync(R->trace, 0xFF, TRACE_SLOTS * sizeof(unsigned long long), st));
         XP_CUDA(cudaMemsetAsync(R->trace + TRACE_SLOTS, 0, TRACE_SLOTS * sizeof(unsigned long long), st));
@@ -671,7 +706,7 @@ int run_small(xpress_refiner *R, const Params &P, const Layout &L, void *ws, cud
     cfg.stream = st;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    XP_CUDA(cudaLaunchKernelEx(&cfg, k_refine_small, P, R->tmap_wrb, R->tmap_wr32, tmap_z));
+    XP_CUDA(cudaLaunchKernelEx(&cfg, k_refine_small, P, R->tmap_wrb, R->tmap_wr32, tmap_z, R->tmap_fk, tmap_h));
     if (R->trace) print_trace(R, st);
     return XPRESS_OK;
 }
@@ -820,7 +855,9 @@ int xpress_refiner_create(const xpress_weights *w, void *stream, xpress_refiner 
             }
             if (tri > 0)
                 k_pack_L<<<(tri + 7) / 8, 256, 0, st>>>(static_cast<const uint16_t *>(w->L), R->Lpk, w->B);
-            if (coop && per_sm >= 1 && R->num_sms > SMALL_TRANS_CTAS) R->small_ok = true;
+            // the persistent kernel reads h and F by K tiles of 64 (H % 64 == 0)
+            const bool fk = w->H % 64 == 0 && make_tmap_fold_k(&R->tmap_fk, R->Fhl, (uint64_t)w->H, SMALL_PC_KT);
+            if (coop && per_sm >= 1 && R->num_sms > SMALL_TRANS_CTAS && fk) R->small_ok = true;
         }
         if (cudaGetLastError() != cudaSuccess || cudaStreamSynchronize(st) != cudaSuccess) rc = XPRESS_ERR_CUDA;
     } while (0);
