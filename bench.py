@@ -403,13 +403,14 @@ def run_xpress(args):
         # acceptance kernels.
         persistent = (dt == X.XPRESS_BF16 and b * cfg.B <= 32 and os.environ.get("XPRESS_SMALL", "1") != "0")
         small = b * cfg.B <= 32
+        acc_launches = 2 if b <= 8 else 3         # rows, (decide,) draw: small batches decide in the draw kernel
         if persistent:
-            per_step_launches = 1 + 3
+            per_step_launches = 1 + acc_launches
         else:
             # per pass: Trans (k_mix_mlp, or k_mix_c + two k_trans_tc for bf16
             # above 32 tokens), Read, reduce (fused into the Read at <= 32 tokens)
             per_pass = 2 if small else (5 if dt == X.XPRESS_BF16 else 3)
-            per_step_launches = 1 + (1 if small else 2) + 1 + passes * per_pass + 3
+            per_step_launches = 1 + (1 if small else 2) + 1 + passes * per_pass + acc_launches
         starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
         ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
         if world > 1:

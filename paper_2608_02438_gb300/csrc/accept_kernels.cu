@@ -8,6 +8,9 @@
 //                 accept y_k while u_k q_k(y_k) < p_k(y_k), q from the
 //                 refinement pass (exp(l_y/T - lse)), p = softmax(target_k / T))
 //                 and, for a sampling block, its draw descriptor
+//                 (batches of at most ACCEPT_FUSED_MAX_B blocks skip this
+//                 kernel: every CTA of k_acc_draw takes the decisions itself,
+//                 which saves a dependent launch on the latency-bound path)
 //   k_acc_draw    every draw of the batch over every vocabulary range:
 //                 Gumbel-max over log max(0, p_k - q_k) at the first rejected
 //                 position (q_k recomputed from z_final through W_r, read once
@@ -62,10 +65,13 @@ __device__ __forceinline__ Partial ldcg_partial16(const Partial *q)
 __global__ void __launch_bounds__(256) k_acc_rows(AcceptParams p, int chunks)
 {
     pdl_trigger();
-    if (blockIdx.x == 0 && threadIdx.x == 0) {
-        *p.status = 0;
-        p.ticket[0] = 0;                          // draws listed by k_acc_decide
-        p.ticket[1] = 0;                          // CTAs of k_acc_draw done
+    if (blockIdx.x == 0) {
+        if (threadIdx.x == 0) {
+            *p.status = 0;
+            p.ticket[0] = 0;                      // draws listed by k_acc_decide
+            p.ticket[1] = 0;                      // CTAs of k_acc_draw done
+        }
+        for (int i = threadIdx.x; i < 2 * p.b; i += blockDim.x) p.keys[i] = 0ull;   // draw keys
     }
     __shared__ Partial sp[256];
     const int items = p.b * (p.B + 1) * chunks;
@@ -151,24 +157,22 @@ __global__ void __launch_bounds__(256) k_acc_rows(AcceptParams p, int chunks)
     pdl_wait();
 }
 
-// grid b, 32 threads (one warp per block).  The block's decision: lane k
-// combines the chunk partials of target row k and decides position k (greedy:
-// y_k equals the target argmax; lossless: u_k q_k(y_k) < p_k(y_k), q from the
-// refinement pass, p = softmax(target_k / T)); a ballot finds the first
-// position not accepted.  Writes the accepted prefix and the accept length;
-// greedy blocks also the target's token after it.  A sampling block appends
-// one draw descriptor (its rejected position, or B for the bonus draw) for
-// k_acc_draw and clears its two draw keys.
-__global__ void __launch_bounds__(32) k_acc_decide(AcceptParams p, int chunks)
+// One warp: the decision of block `seq`.  Lane k combines the chunk partials
+// of target row k and decides position k (greedy: y_k equals the target
+// argmax; lossless: u_k q_k(y_k) < p_k(y_k), q from the refinement pass,
+// p = softmax(target_k / T)); a ballot finds the first position not
+// accepted.  With `write`, the warp writes the accepted prefix, -1 past it
+// and the accept length; a greedy block also the target's token after the
+// prefix (a sampling block's token there is the draw's).  Returns whether the
+// block samples and, for a sampling block, fills its draw descriptor (its
+// rejected position, or B for the bonus draw).
+__device__ __forceinline__ bool decide_block(const AcceptParams &p, int seq, int lane, Partial *rows, bool write,
+                                             DrawDesc &dd)
 {
-    pdl_trigger();                                // k_acc_draw may start its prologue
-    pdl_wait();                                   // the row partials (and the refinement before them)
-    const int seq = blockIdx.x, lane = threadIdx.x;
-    const int B = p.B;
+    const int B = p.B, chunks = p.chunks;
     const float T = p.temperature[seq];
     const bool sampling = T > 0.0f;
     const float invT = sampling ? 1.0f / T : 0.0f;
-    __shared__ Partial rows[MAX_B + 1];
     for (int k = lane; k <= B; k += 32) {
         Partial a{-INFINITY, 0x7fffffff, -INFINITY, 0.0f};
         const size_t r = (size_t)seq * (B + 1) + k;
@@ -206,25 +210,63 @@ __global__ void __launch_bounds__(32) k_acc_decide(AcceptParams p, int chunks)
     }
     const unsigned rejected = __ballot_sync(0xffffffffu, lane < B && !ok);
     const int n = rejected ? __ffs(rejected) - 1 : B;
-    int32_t *out = p.out_tokens + (size_t)seq * (B + 1);
-    for (int k = lane; k <= B; k += 32) out[k] = k < n ? p.tokens[(size_t)seq * B + k] : -1;
-    __syncwarp();
-    if (lane == 0) {
-        p.accept_len[seq] = n;
-        if (!sampling) {
-            out[n] = rows[n].idx;
-        } else {
-            p.keys[2 * seq] = 0ull;
-            p.keys[2 * seq + 1] = 0ull;
-            DrawDesc dd;
-            dd.seq = seq;
-            dd.k = n;
-            dd.invT = invT;
-            dd.lse_p = rows[n].m + logf(rows[n].s);
-            dd.lse_q = n < B ? p.lse[(size_t)seq * B + n] : 0.0f;
-            p.draws[atomicAdd(p.ticket, 1)] = dd;
+    if (write) {
+        int32_t *out = p.out_tokens + (size_t)seq * (B + 1);
+        for (int k = lane; k <= B; k += 32)
+            if (k != n) out[k] = k < n ? p.tokens[(size_t)seq * B + k] : -1;
+        if (lane == 0) {
+            p.accept_len[seq] = n;
+            if (!sampling) out[n] = rows[n].idx;
         }
     }
+    if (sampling) {
+        dd.seq = seq;
+        dd.k = n;
+        dd.invT = invT;
+        dd.lse_p = rows[n].m + logf(rows[n].s);
+        dd.lse_q = n < B ? p.lse[(size_t)seq * B + n] : 0.0f;
+    }
+    __syncwarp();                                 // rows is reused by the warp's next block
+    return sampling;
+}
+
+// grid b, 32 threads (one warp per block): the block's decision
+// (decide_block); a sampling block appends its draw descriptor for
+// k_acc_draw.
+__global__ void __launch_bounds__(32) k_acc_decide(AcceptParams p)
+{
+    pdl_trigger();                                // k_acc_draw may start its prologue
+    pdl_wait();                                   // the row partials (and the refinement before them)
+    __shared__ Partial rows[MAX_B + 1];
+    DrawDesc dd{};
+    if (decide_block(p, blockIdx.x, threadIdx.x, rows, true, dd) && threadIdx.x == 0) p.draws[atomicAdd(p.ticket, 1)] = dd;
+}
+
+// Small batches (fused): every CTA of the draw kernel takes all the
+// decisions itself (warp w: blocks w, w + 8, ...), CTA 0 writes the accepted
+// prefixes, and the sampling blocks' draw descriptors are listed in block
+// order in shared memory (the same list in every CTA).  Returns their count.
+__device__ __forceinline__ int decide_all(const AcceptParams &p, DrawDesc *list, Partial (*rows)[MAX_B + 1],
+                                          int *sflag)
+{
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32, nwarps = blockDim.x / 32;
+    for (int seq = warp; seq < p.b; seq += nwarps) {
+        DrawDesc dd{};
+        const bool s = decide_block(p, seq, lane, rows[warp], blockIdx.x == 0, dd);
+        if (lane == 0) {
+            sflag[seq] = s;
+            if (s) list[seq] = dd;
+        }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int nd = 0;
+        for (int seq = 0; seq < p.b; ++seq)
+            if (sflag[seq]) list[nd++] = list[seq];
+        sflag[ACCEPT_FUSED_MAX_B] = nd;
+    }
+    __syncthreads();
+    return sflag[ACCEPT_FUSED_MAX_B];
 }
 
 namespace {
@@ -260,7 +302,7 @@ __device__ __forceinline__ void load_row32(float (&w)[32], const void *W_r, int 
 // The end of the draw kernel, every thread of every CTA: the CTA counts
 // itself done; the last one emits each drawn token (the residual's draw, or
 // the draw from p when the residual is empty or after B acceptances).
-__device__ __forceinline__ void draw_finish(const AcceptParams &p, int nd, int G, int *s_last)
+__device__ __forceinline__ void draw_finish(const AcceptParams &p, const DrawDesc *list, int nd, int G, int *s_last)
 {
     if (threadIdx.x == 0) {
         __threadfence();
@@ -270,7 +312,7 @@ __device__ __forceinline__ void draw_finish(const AcceptParams &p, int nd, int G
     if (!*s_last) return;
     __threadfence();
     for (int j = threadIdx.x; j < nd; j += blockDim.x) {
-        const DrawDesc dd = p.draws[j];
+        const DrawDesc dd = list[j];
         const unsigned long long kr = __ldcg(p.keys + 2 * dd.seq), kp = __ldcg(p.keys + 2 * dd.seq + 1);
         float best;
         int idx;
@@ -323,8 +365,12 @@ __device__ __forceinline__ void draw_element(const AcceptParams &p, const DrawDe
 // so it must not start until every CTA of this kernel has exited.
 __global__ void __launch_bounds__(DRAW_THREADS) k_acc_draw_simt(AcceptParams p)
 {
-    pdl_wait();                                   // the draw list of k_acc_decide
-    const int nd = __ldcg(p.ticket);
+    pdl_wait();                                   // the draw list of k_acc_decide (or the row partials)
+    __shared__ DrawDesc flist[ACCEPT_FUSED_MAX_B];
+    __shared__ Partial frows[DRAW_THREADS / 32][MAX_B + 1];
+    __shared__ int fflag[ACCEPT_FUSED_MAX_B + 1];
+    const int nd = p.fused ? decide_all(p, flist, frows, fflag) : __ldcg(p.ticket);
+    const DrawDesc *list = p.fused ? flist : p.draws;
     if (nd == 0) return;
     const int G = gridDim.x, r = blockIdx.x, warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const int nwarps = DRAW_THREADS / 32, B = p.B;
@@ -335,7 +381,7 @@ __global__ void __launch_bounds__(DRAW_THREADS) k_acc_draw_simt(AcceptParams p)
     __shared__ int s_any_resid, s_last;
     for (int g0 = 0; g0 < nd; g0 += DRAW_NZ) {
         const int nz = min(DRAW_NZ, nd - g0);
-        if (threadIdx.x < nz) dsc[threadIdx.x] = p.draws[g0 + threadIdx.x];
+        if (threadIdx.x < nz) dsc[threadIdx.x] = list[g0 + threadIdx.x];
         if (threadIdx.x == 0) s_any_resid = 0;
         __syncthreads();
         for (int i = threadIdx.x; i < nz * RANK; i += DRAW_THREADS) {
@@ -418,7 +464,7 @@ __global__ void __launch_bounds__(DRAW_THREADS) k_acc_draw_simt(AcceptParams p)
         }
         __syncthreads();
     }
-    draw_finish(p, nd, G, &s_last);
+    draw_finish(p, list, nd, G, &s_last);
 }
 
 
@@ -434,8 +480,12 @@ __global__ void __launch_bounds__(DRAW_THREADS) k_acc_draw_simt(AcceptParams p)
 // CTA ranges start at multiples of 8 ids.
 __global__ void __launch_bounds__(DRAW_THREADS, 2) k_acc_draw(AcceptParams p)
 {
-    pdl_wait();                                   // the draw list of k_acc_decide
-    const int nd = __ldcg(p.ticket);
+    pdl_wait();                                   // the draw list of k_acc_decide (or the row partials)
+    __shared__ DrawDesc flist[ACCEPT_FUSED_MAX_B];
+    __shared__ Partial frows[DRAW_THREADS / 32][MAX_B + 1];
+    __shared__ int fflag[ACCEPT_FUSED_MAX_B + 1];
+    const int nd = p.fused ? decide_all(p, flist, frows, fflag) : __ldcg(p.ticket);
+    const DrawDesc *list = p.fused ? flist : p.draws;
     if (nd == 0) return;
     const int G = gridDim.x, r = blockIdx.x, warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const int nwarps = DRAW_THREADS / 32, B = p.B;
@@ -454,7 +504,7 @@ __global__ void __launch_bounds__(DRAW_THREADS, 2) k_acc_draw(AcceptParams p)
         if (threadIdx.x < DRAW_NZ) {
             DrawDesc dd{};
             dd.k = B;                                 // padding draws: no residual, never read
-            if (threadIdx.x < nz) dd = p.draws[g0 + threadIdx.x];
+            if (threadIdx.x < nz) dd = list[g0 + threadIdx.x];
             dsc[threadIdx.x] = dd;
             dseed[threadIdx.x] = threadIdx.x < nz ? p.seed[dd.seq] : 0ull;
         }
@@ -540,7 +590,7 @@ __global__ void __launch_bounds__(DRAW_THREADS, 2) k_acc_draw(AcceptParams p)
         }
         __syncthreads();
     }
-    draw_finish(p, nd, G, &s_last);
+    draw_finish(p, list, nd, G, &s_last);
 }
 
 }  // namespace xp

@@ -27,8 +27,11 @@ struct AcceptParams {
     Partial *rowpart;   // [b * (B + 1), chunks]
     int32_t *ticket;    // [2]: draws listed, draw CTAs done (cleared by k_acc_rows)
     DrawDesc *draws;    // [b] draws of the sampling blocks (k_acc_decide)
-    unsigned long long *keys;   // [b, 2] best residual / p draw key (argmax_key), cleared by k_acc_decide
+    unsigned long long *keys;   // [b, 2] best residual / p draw key (argmax_key), cleared by k_acc_rows
+    int chunks;         // vocabulary chunks per target row (k_acc_rows)
+    int fused;          // 1: no k_acc_decide; every k_acc_draw CTA takes the decisions itself (b <= 8)
 };
+constexpr int ACCEPT_FUSED_MAX_B = 8;       // batches up to this size skip k_acc_decide
 
 // refine_kernels.cu
 __global__ void k_init(Params pin, Params *pdev, cudaGraphConditionalHandle handle);
@@ -90,7 +93,7 @@ extern const int kLmHeadThreads;
 
 // accept_kernels.cu
 __global__ void k_acc_rows(AcceptParams p, int chunks);
-__global__ void k_acc_decide(AcceptParams p, int chunks);
+__global__ void k_acc_decide(AcceptParams p);
 __global__ void k_acc_draw(AcceptParams p);        // bf16 refiners (tensor-core products)
 __global__ void k_acc_draw_simt(AcceptParams p);   // fp32 refiners
 

@@ -56,6 +56,8 @@ struct RsShared {                              // Read CTA, after the W_r stages
     uint64_t pfull[PC_BUFS_MAX], pempty[PC_BUFS_MAX];   // precompute ring (h and F chunks)
     uint32_t tmem_base;
     int abort;
+    int pc_end;                                // the epilogue warps are done with the precompute
+    uint32_t pf_early;                         // bytes of the W_r range prefetched during the precompute
     int pass_n, pass_stop;                     // published by the producer with `go`
     int tok[TV_BN], pos[TV_BN];
     float invT[TV_BN];
@@ -405,6 +407,8 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
         mbar_init(&sh.drain, 1);
         for (int i = 0; i < PC_BUFS_MAX; ++i) { mbar_init(&sh.pfull[i], 1); mbar_init(&sh.pempty[i], TV_EPI_WARPS); }
         sh.abort = 0;
+        sh.pc_end = 0;
+        sh.pf_early = 0;
         fence_barrier_init();
     }
     if (warp == 1) { tmem_alloc(&sh.tmem_base, TV_TMEM_COLS); tmem_relinquish(); }
@@ -429,12 +433,35 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
             if (N <= 16) pc_produce<16>(p, tmap_f, tmap_h, sA, sh, r, S, abort);
             else pc_produce<32>(p, tmap_f, tmap_h, sA, sh, r, S, abort);
         }
+    } else if (warp == 1) {
+        // meanwhile the idle MMA thread streams the start of this CTA's W_r
+        // range into L2 at a gentle pace (the first pass reads it cold), until
+        // the precompute ends
+        if (lane == 0) {
+            const char *wr = static_cast<const char *>(p.W_r) + (size_t)R0 * RANK * 2;
+            const uint32_t total = (uint32_t)(R1 - R0) * RANK * 2, slice = 64 * RANK * 2;
+            const unsigned long long t0 = globaltimer();
+            unsigned long long t_next = t0;
+            uint32_t done = 0;
+            while (!*reinterpret_cast<volatile int *>(&sh.pc_end) && done < total) {
+                const unsigned long long now = globaltimer();
+                if (now >= t_next) {
+                    prefetch_l2_bulk(wr + done, min(slice, total - done));
+                    done += min(slice, total - done);
+                    t_next = now + 1500u;
+                }
+                if (now - t0 > 100000000ull) break;          // a bound; the precompute takes microseconds
+                __nanosleep(200);
+            }
+            sh.pf_early = done;
+        }
     } else if (warp >= 2) {
         const int w = warp - 2;
         const bool tm = tr && w == 0 && lane == 0;
         if (tm) trace_mark(p.trace, 4, t_start);
         if (N <= 16) pc_consume<16>(p, sA, sh, r, S, w, lane, abort, tm, t_start);
         else pc_consume<32>(p, sA, sh, r, S, w, lane, abort, tm, t_start);
+        if (w == 0 && lane == 0) *reinterpret_cast<volatile int *>(&sh.pc_end) = 1;
         if (!p.draft)
             for (int item = r * TV_EPI_WARPS + w; item < N * RMAX_SEG; item += S * TV_EPI_WARPS)
                 rowmax_item(p, item, lane);
@@ -482,7 +509,7 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
             for (; next < ahead && ok; ++next) ok = issue(next);
             // while the first Trans runs, the rest of this CTA's W_r range
             // (past the chunks the ring holds) goes into L2 a slice at a time
-            const int pf_row0 = R0 + ahead * TV_BM;
+            const int pf_row0 = max(R0 + ahead * TV_BM, R0 + (int)(sh.pf_early / (RANK * 2)));
             const int pf_rows = max(0, R1 - pf_row0);
             const uint32_t pf_bytes = (uint32_t)pf_rows * RANK * 2;
             for (int pass = 0; ok; ++pass) {

@@ -1052,11 +1052,14 @@ int accept_launch(const xpress_refiner *R, const xpress_accept_in *in, int32_t *
     P.ticket = reinterpret_cast<int32_t *>(w + A.ticket);
     P.draws = reinterpret_cast<DrawDesc *>(w + A.draws);
     P.keys = reinterpret_cast<unsigned long long *>(w + A.keys);
+    P.chunks = A.chunks;
+    P.fused = in->b <= ACCEPT_FUSED_MAX_B;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     // each is chained to its predecessor with programmatic dependent launch
-    // (k_acc_rows clears the status word and the draw counters)
+    // (k_acc_rows clears the status word, the draw counters and keys); small
+    // batches skip k_acc_decide (the draw kernel's CTAs decide)
     XP_CUDA(launch_pdl(k_acc_rows, dim3(A.row_ctas), dim3(256), 0, st, P, A.chunks));
-    XP_CUDA(launch_pdl(k_acc_decide, dim3(in->b), dim3(32), 0, st, P, A.chunks));
+    if (!P.fused) XP_CUDA(launch_pdl(k_acc_decide, dim3(in->b), dim3(32), 0, st, P));
     XP_CUDA(launch_pdl(R->w.dtype == XPRESS_BF16 ? k_acc_draw : k_acc_draw_simt, dim3(A.draw_ctas), dim3(256), 0, st,
                        P));
     XP_CUDA(cudaGetLastError());
