@@ -246,6 +246,9 @@ const CUtensorMap *refiner_tmap_wr128(const xpress_refiner *R);   // W_r, boxes 
 // 128-byte swizzle, zero fill out of bounds
 bool tmap_bf16(CUtensorMap *m, const void *base, uint64_t inner, uint64_t outer, uint64_t pitch, uint32_t box_inner,
                uint32_t box_outer);
+// [rows][r] bf16 as (64 columns, rows, r / 64 K chunks): a box of 64 x box_rows
+// x r / 64 lands as the K-chunk tiles of 2D boxes of 64 x box_rows, back to back
+bool tmap_bf16_kblocks(CUtensorMap *m, const void *base, uint64_t rows, uint32_t box_rows);
 int accept_launch(const xpress_refiner *R, const xpress_accept_in *in, int32_t *accept_len, int32_t *out_tokens,
                   void *ws, size_t ws_bytes, void *stream);
 constexpr int READ_SIMT_DYN_SMEM = (32 * (RANK + 1) + 8 * 32 * 33) * 4;

@@ -105,6 +105,21 @@ __device__ __forceinline__ uint64_t smem_desc_sw128_mn(uint32_t saddr, uint32_t 
            ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
 }
 
+// TMA load of a 3D box with an L2 cache policy: the readout weights viewed as
+// (64 columns, rows, K chunk of 64), so that one copy brings a tile's four K
+// chunks ([chunk][row][128 bytes], each chunk as a 2D box of 64 x rows would
+// land).  One large copy per tile instead of four keeps the TMA unit's
+// per-copy cost off the critical path.
+__device__ __forceinline__ void tma_load_w3d(void *smem_dst, const CUtensorMap *map, uint64_t *bar, int row,
+                                             uint64_t policy)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1, {%2, "
+        "%3, %4}], [%5], %6;" ::"r"(smem_u32(smem_dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(row), "r"(0), "r"(smem_u32(bar)), "l"(policy)
+        : "memory");
+}
+
 // Adds four floats into 16-byte aligned global memory with one vector
 // reduction (relaxed, GPU scope).
 __device__ __forceinline__ void red_add_v4(float *dst, float a, float b, float c, float d)

@@ -310,9 +310,10 @@ int train_run(const xpress_refiner *R, const xpress_train_in *in, const xpress_t
     tp.status = m.status;
     tp.wait_ns = refiner_wait_ns(R);
 
-    CUtensorMap tz128, tz32, tw64, ts64, tt64, ts32, tt32;
+    CUtensorMap tz128, tz32, tw64, tw128, ts64, tt64, ts32, tt32;
     if (!tmap_bf16(&tz128, U(L.zop), r, NR, r, 64, 128) || !tmap_bf16(&tz32, U(L.zop), r, NR, r, 64, 32) ||
-        !tmap_bf16(&tw64, w.W_r, r, V, r, 64, 64) || !tmap_bf16(&ts64, in->s, V, P, V, 64, 64) ||
+        !tmap_bf16_kblocks(&tw64, w.W_r, V, 64) || !tmap_bf16_kblocks(&tw128, w.W_r, V, 128) ||
+        !tmap_bf16(&ts64, in->s, V, P, V, 64, 64) ||
         !tmap_bf16(&tt64, in->target, V, P, V, 64, 64) || !tmap_bf16(&ts32, in->s, V, P, V, 64, 32) ||
         !tmap_bf16(&tt32, in->target, V, P, V, 64, 32))
         return XPRESS_ERR_CUDA;
@@ -322,7 +323,7 @@ int train_run(const xpress_refiner *R, const xpress_train_in *in, const xpress_t
     if (only >= 0) {
         if (only == TR_STATS)
             XT_CUDA(launch(k_train_tok_stats, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128,
-                           *refiner_tmap_wr128(R), ts64, tt64));
+                           tw128, ts64, tt64));
         else if (only == TR_TV)
             XT_CUDA(launch(k_train_tok_tv, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128, tw64, ts64,
                            tt64));
@@ -375,8 +376,8 @@ int train_run(const xpress_refiner *R, const xpress_train_in *in, const xpress_t
     // the Read passes
     const dim3 gvoc(nvt128 < sms ? nvt128 : sms);
     // W_r tiles of 128 ids (boxes of 128 rows) for the log-sum-exp pass, of 64 for the others
-    XT_CUDA(launch(k_train_tok_stats, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128,
-                   *refiner_tmap_wr128(R), ts64, tt64));
+    XT_CUDA(launch(k_train_tok_stats, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128, tw128,
+                   ts64, tt64));
     XT_CUDA(launch(k_train_stats_fin, dim3(NR / 8), dim3(256), 0, st, m));
     XT_CUDA(launch(k_train_tok_tv, gtok, dim3(kTrainTokThreads), kTrainTokSmemBytes, st, tp, tz128, tw64, ts64,
                    tt64));

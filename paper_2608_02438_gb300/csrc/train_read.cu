@@ -150,8 +150,9 @@ const size_t kTrainTokSmemBytes = TR_SMEM;
 const int kTrainTokThreads = TR_THREADS;
 
 // The token-major kernel for one mode (compiled once per mode, so that its
-// tile width, ring depths and epilogue are constants).  tmap_w: W_r boxes of
-// bn rows x 64; tmap_s / tmap_t: boxes of 64 ids x 64 positions.
+// tile width, ring depths and epilogue are constants).  tmap_w: W_r as (64
+// columns, rows, 4 K chunks), boxes of 64 x bn x 4 (one copy per tile);
+// tmap_s / tmap_t: boxes of 64 ids x 64 positions.
 template <int mode>
 __device__ __forceinline__ void train_tok_body(const TrainParams &p, const CUtensorMap &tmap_w,
                                                const CUtensorMap &tmap_s, const CUtensorMap &tmap_t)
@@ -226,9 +227,8 @@ __device__ __forceinline__ void train_tok_body(const TrainParams &p, const CUten
                 const int st = it % NB;
                 const uint32_t ph = (uint32_t)((it / NB) & 1);
                 if (!mbar_wait_spin(&sh.empty[st], ph ^ 1, abort, lim)) break;
-                mbar_expect_tx(&sh.full[st], BST);
-                for (int c = 0; c < 4; ++c)      // tmap_w: boxes of bn rows x 64
-                    tma_load_2d_hint(sB + st * BST + c * BCH, &tmap_w, &sh.full[st], c * 64, vt * bn, keep);
+                mbar_expect_tx(&sh.full[st], BST);   // tmap_w: (64 columns, rows, K chunk), boxes of bn rows
+                tma_load_w3d(sB + st * BST, &tmap_w, &sh.full[st], vt * bn, keep);
                 pend_b |= 1u << st;
                 par_b = (par_b & ~(1u << st)) | (ph << st);
                 if (!mbar_wait_spin(&sh.sempty[ss], sph ^ 1, abort, lim)) break;

@@ -1000,6 +1000,11 @@ int refiner_sms(const xpress_refiner *R) { return R->num_sms; }
 unsigned long long refiner_wait_ns(const xpress_refiner *R) { return R->wait_ns; }
 const CUtensorMap *refiner_tmap_wr128(const xpress_refiner *R) { return &R->tmap_wr128; }
 
+bool tmap_bf16_kblocks(CUtensorMap *m, const void *base, uint64_t rows, uint32_t box_rows)
+{
+    return make_tmap_bf16_kblocks(m, base, rows, box_rows);
+}
+
 bool tmap_bf16(CUtensorMap *m, const void *base, uint64_t inner, uint64_t outer, uint64_t pitch, uint32_t box_inner,
                uint32_t box_outer)
 {
