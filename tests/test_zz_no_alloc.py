@@ -78,6 +78,35 @@ def test_noalloc_accept_matches_workspace_accept_on_two_calls(X):
         ref.close()
 
 
+def test_noalloc_accept_replayed_from_a_cuda_graph(X):
+    # the entry point exists for stream capture: one call captured (after a
+    # warm-up call that caches the scratch address), then replayed twice
+    cfg, inp, ref, d, out = _setup(X, (1.0, 0.0), 83)
+    want = ref.accept(d["target"], d["s"], out["tokens"], out["lse"], out["logit_sel"], out["z_final"],
+                      d["temperature"], d["seed"], inp["offset"])
+    torch.cuda.synchronize()
+    want = {k: v.cpu().numpy().copy() for k, v in want.items()}
+    alen = torch.full((cfg.b,), -7, dtype=torch.int32, device="cuda")
+    otok = torch.full((cfg.b, cfg.B + 1), -7, dtype=torch.int32, device="cuda")
+    acc_in = _accept_in(X, cfg, inp, d, out)
+    X.xpress_accept_noalloc(ref.handle, acc_in, alen.data_ptr(), otok.data_ptr(), ref.stream.cuda_stream)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):                 # captured on torch's side stream
+        X.xpress_accept_noalloc(ref.handle, acc_in, alen.data_ptr(), otok.data_ptr(),
+                                torch.cuda.current_stream().cuda_stream)
+    for replay in range(2):
+        alen.fill_(-7)
+        otok.fill_(-7)
+        torch.cuda.synchronize()
+        graph.replay()
+        torch.cuda.synchronize()
+        np.testing.assert_array_equal(alen.cpu().numpy(), want["accept_len"], err_msg=f"replay {replay}")
+        np.testing.assert_array_equal(otok.cpu().numpy(), want["out_tokens"], err_msg=f"replay {replay}")
+    del graph
+    ref.close()
+
+
 def test_noalloc_rejects_a_batch_beyond_its_scratch(X):
     cfg = W.tiny_config("noalloc_big", b=1, B=32, H=64, V=64, r=256, dtype=W.BF16, seed=79)
     w = W.make_weights(cfg.H, cfg.V, cfg.r, cfg.B, cfg.dtype, 80, "paper")
