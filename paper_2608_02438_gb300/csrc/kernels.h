@@ -242,6 +242,9 @@ const xpress_weights &refiner_weights(const xpress_refiner *R);
 int refiner_sms(const xpress_refiner *R);
 unsigned long long refiner_wait_ns(const xpress_refiner *R);
 const CUtensorMap *refiner_tmap_wr128(const xpress_refiner *R);   // W_r, boxes of 128 rows x 64
+// the refiner's second stream and four events, on which the training step
+// runs its weight-gradient products beside the input-gradient chain
+cudaStream_t refiner_train_aux(const xpress_refiner *R, cudaEvent_t (&ev)[4]);
 // 2-D bf16 tensor [outer][inner] with a row pitch of `pitch` elements,
 // 128-byte swizzle, zero fill out of bounds
 bool tmap_bf16(CUtensorMap *m, const void *base, uint64_t inner, uint64_t outer, uint64_t pitch, uint32_t box_inner,

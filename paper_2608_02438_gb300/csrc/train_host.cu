@@ -393,31 +393,45 @@ int train_run(const xpress_refiner *R, const xpress_train_in *in, const xpress_t
                    F(L.du), 2 * r, nullptr, 0, nullptr, 0, 0)))
         return rc;
     XT_CUDA(launch(k_train_dact, dim3((NR * 2 * r / 4 + 255) / 256), dim3(256), 0, st, m));
-    if ((rc = gemm(st, sms, NR, r, 2 * r, {U(L.dtb), (uint64_t)2 * r, false}, {w.W1, (uint64_t)r, true}, GM_RESID, 1.f,
-                   F(L.dc), r, nullptr, 0, F(L.dz), r, 0)))
-        return rc;
-    if ((rc = gemm(st, sms, r, 2 * r, NR, {U(L.dzb), (uint64_t)r, true}, {U(L.uop), (uint64_t)2 * r, true}, GM_ADD,
+    // The weight-gradient products run on the refiner's second stream beside
+    // the input-gradient chain (dz -> dc -> Mix backward -> dX -> Fuse
+    // backward), each forked once its operands exist and joined at the end;
+    // none of their operands is written again in the step.
+    cudaEvent_t ev[4];
+    const cudaStream_t aux = refiner_train_aux(R, ev);
+    XT_CUDA(cudaEventRecord(ev[0], st));                        // dz and dt
+    XT_CUDA(cudaStreamWaitEvent(aux, ev[0], 0));
+    if ((rc = gemm(aux, sms, r, 2 * r, NR, {U(L.dzb), (uint64_t)r, true}, {U(L.uop), (uint64_t)2 * r, true}, GM_ADD,
                    1.f, out->gW2, 2 * r, nullptr, 0, nullptr, 0, 0)))
         return rc;
-    if ((rc = gemm(st, sms, 2 * r, r, NR, {U(L.dtb), (uint64_t)2 * r, true}, {U(L.cop), (uint64_t)r, true}, GM_ADD,
+    if ((rc = gemm(aux, sms, 2 * r, r, NR, {U(L.dtb), (uint64_t)2 * r, true}, {U(L.cop), (uint64_t)r, true}, GM_ADD,
                    1.f, out->gW1, r, nullptr, 0, nullptr, 0, 0)))
+        return rc;
+    if ((rc = gemm(st, sms, NR, r, 2 * r, {U(L.dtb), (uint64_t)2 * r, false}, {w.W1, (uint64_t)r, true}, GM_RESID, 1.f,
+                   F(L.dc), r, nullptr, 0, F(L.dz), r, 0)))
         return rc;
 
     // backward through Mix (Eq. mix) and Fuse (Eq. fuse)
     XT_CUDA(launch(k_train_mix_bwd, gmix, bmix, train_mix_smem(in->B), st, m));
+    XT_CUDA(cudaEventRecord(ev[1], st));                        // dL/da
+    XT_CUDA(cudaStreamWaitEvent(aux, ev[1], 0));
+    if ((rc = gemm(aux, sms, r, 3 * r, NR, {U(L.dab), (uint64_t)r, true}, {U(L.X), (uint64_t)3 * r, true}, GM_ADD, 1.f,
+                   out->gW_in, 3 * r, nullptr, 0, nullptr, 0, 0)))
+        return rc;
     if ((rc = gemm(st, sms, NR, 3 * r, r, {U(L.dab), (uint64_t)r, false}, {w.W_in, (uint64_t)3 * r, true}, GM_STORE,
                    1.f, F(L.dX), 3 * r, nullptr, 0, nullptr, 0, 0)))
         return rc;
-    if ((rc = gemm(st, sms, r, 3 * r, NR, {U(L.dab), (uint64_t)r, true}, {U(L.X), (uint64_t)3 * r, true}, GM_ADD, 1.f,
-                   out->gW_in, 3 * r, nullptr, 0, nullptr, 0, 0)))
-        return rc;
     XT_CUDA(launch(k_train_fuse_bwd, dim3(P), dim3(RANK), 0, st, m));
+    XT_CUDA(cudaEventRecord(ev[2], st));                        // dL/du_h, dL/du_g
+    XT_CUDA(cudaStreamWaitEvent(aux, ev[2], 0));
+    if ((rc = gemm(aux, sms, r, H, P, {U(L.D) + r, (uint64_t)2 * r, true}, h_mn, GM_ADD, 1.f, out->gW_g, H, nullptr, 0,
+                   nullptr, 0, 0)))
+        return rc;
     if ((rc = gemm(st, sms, r, H, P, {U(L.D), (uint64_t)2 * r, true}, h_mn, GM_ADD, 1.f, out->gW_h, H, nullptr, 0,
                    nullptr, 0, 0)))
         return rc;
-    if ((rc = gemm(st, sms, r, H, P, {U(L.D) + r, (uint64_t)2 * r, true}, h_mn, GM_ADD, 1.f, out->gW_g, H, nullptr, 0,
-                   nullptr, 0, 0)))
-        return rc;
+    XT_CUDA(cudaEventRecord(ev[3], aux));                       // join
+    XT_CUDA(cudaStreamWaitEvent(st, ev[3], 0));
     return XPRESS_OK;
 }
 

@@ -147,6 +147,8 @@ struct xpress_refiner {
     unsigned long long wait_ns = 2000000000ull;   // bound on the persistent kernel's waits for other CTAs
     bool use_tc = false;
     cudaStream_t cs = nullptr;
+    cudaStream_t train_aux = nullptr;      // the training step's weight-gradient products (forked, then joined)
+    cudaEvent_t train_ev[4] = {};
     uint16_t *Fhl = nullptr;               // [2][2r, H] folded hidden projection, bf16 hi / lo (bf16 refiners)
     uint16_t *Lpk = nullptr;               // [B(B-1)/2, r] L's strictly lower part, channel innermost
     bool small_ok = false;                 // the small-batch kernel can run co-resident on this GPU
@@ -813,10 +815,14 @@ int xpress_refiner_create(const xpress_weights *w, void *stream, xpress_refiner 
                 break;
             }
         if (cudaMalloc(&R->Ep, (size_t)w->V * RANK * sizeof(float)) != cudaSuccess ||
-            cudaStreamCreateWithFlags(&R->cs, cudaStreamNonBlocking) != cudaSuccess) {
+            cudaStreamCreateWithFlags(&R->cs, cudaStreamNonBlocking) != cudaSuccess ||
+            cudaStreamCreateWithFlags(&R->train_aux, cudaStreamNonBlocking) != cudaSuccess) {
             rc = XPRESS_ERR_CUDA;
             break;
         }
+        for (auto &ev : R->train_ev)
+            if (cudaEventCreateWithFlags(&ev, cudaEventDisableTiming) != cudaSuccess) rc = XPRESS_ERR_CUDA;
+        if (rc != XPRESS_OK) break;
         const dim3 grid(RANK / 64, (w->V + 63) / 64);
         k_build_ep<<<grid, 256, 0, st>>>(w->W_e, w->W_in, R->Ep, w->V, w->dtype);
         if (R->use_tc) {
@@ -878,6 +884,9 @@ int xpress_refiner_destroy(xpress_refiner *R)
     if (R->Fhl) cudaFree(R->Fhl);
     if (R->Lpk) cudaFree(R->Lpk);
     if (R->cs) cudaStreamDestroy(R->cs);
+    if (R->train_aux) cudaStreamDestroy(R->train_aux);
+    for (auto &ev : R->train_ev)
+        if (ev) cudaEventDestroy(ev);
     if (R->trace) cudaFree(R->trace);
     delete R;
     return XPRESS_OK;
@@ -999,6 +1008,11 @@ const xpress_weights &refiner_weights(const xpress_refiner *R) { return R->w; }
 int refiner_sms(const xpress_refiner *R) { return R->num_sms; }
 unsigned long long refiner_wait_ns(const xpress_refiner *R) { return R->wait_ns; }
 const CUtensorMap *refiner_tmap_wr128(const xpress_refiner *R) { return &R->tmap_wr128; }
+cudaStream_t refiner_train_aux(const xpress_refiner *R, cudaEvent_t (&ev)[4])
+{
+    for (int i = 0; i < 4; ++i) ev[i] = R->train_ev[i];
+    return R->train_aux;
+}
 
 bool tmap_bf16_kblocks(CUtensorMap *m, const void *base, uint64_t rows, uint32_t box_rows)
 {

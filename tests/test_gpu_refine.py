@@ -196,6 +196,28 @@ def test_accept_tiny(X, temps):
     _accept_check(X, cfg, w, inp)
 
 
+# Batches of at most 8 blocks take the decisions inside the draw kernel (no
+# separate decision launch): greedy and sampling blocks mixed, and a batch of
+# one of each kind.
+@pytest.mark.parametrize("b,temps", [(8, (0.0, 1.0)), (1, (1.0,)), (1, (0.0,))])
+def test_accept_small_batches(X, b, temps):
+    cfg = W.tiny_config("accs", b=b, B=16, H=128, V=2080, r=256, dtype=W.BF16, temps=temps, seed=63 + b,
+                        logits="gauss4_spike", draft="sample")
+    w = W.make_weights(cfg.H, cfg.V, cfg.r, cfg.B, cfg.dtype, 64 + b, "strong")
+    inp = W.make_inputs(cfg)
+    _accept_check(X, cfg, w, inp)
+
+
+# A hidden size that is not a multiple of 64: the persistent kernel reads h
+# and the folded projection by 64-wide K tiles, so these calls take the
+# multi-kernel path; results must not change.
+def test_hidden_size_not_a_multiple_of_64(X):
+    cfg = W.tiny_config("h136", b=1, B=16, H=136, V=2080, r=256, dtype=W.BF16, temps=(0.0,), seed=1900)
+    w = W.make_weights(cfg.H, cfg.V, cfg.r, cfg.B, cfg.dtype, 1901, "strong")
+    inp = W.make_inputs(cfg)
+    _check(X, cfg, w, inp)
+
+
 @pytest.mark.parametrize("name", ["qwen3_8b_greedy", "qwen3_8b_t1"])
 def test_accept_qwen3_shape(X, name):
     cfg, w, inp = W.make_workload(name)
