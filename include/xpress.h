@@ -151,9 +151,10 @@ typedef struct {
 size_t xpress_refine_workspace_size(const xpress_refiner *refiner, int b);
 
 /* Runs Algorithm 1 on all b blocks with no host synchronisation: the
- * iteration loop runs on the device.  Calls of a bf16 refiner that evaluate at
- * most 32 tokens (b * B <= 32) run as one persistent cooperative kernel whose
- * CTAs apply the stopping rule themselves; other calls run a CUDA graph whose
+ * iteration loop runs on the device.  Calls of a bf16 refiner (H a multiple of
+ * 64) that evaluate at most 32 tokens (b * B <= 32) run as one persistent
+ * cooperative kernel whose CTAs apply the stopping rule themselves; other
+ * calls run a CUDA graph whose
  * WHILE conditional node repeats the per-pass kernels until the device clears
  * its condition.  Blocks that have converged drop out of later passes, and a
  * pass re-evaluates only the positions after the first token the previous
