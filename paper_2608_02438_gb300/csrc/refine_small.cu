@@ -546,7 +546,9 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
     } else if (warp == 1) {
         // ---------------------------------------------------- MMA issuer
         if (lane == 0) {
-            const uint32_t z0 = smem_u32(sZ);
+            // descriptors formed once, advanced per MMA
+            const uint64_t zdesc0 = smem_desc_sw128(smem_u32(sZ));
+            const uint64_t adesc0 = smem_desc_sw128(smem_u32(sA));
             for (int pass = 0;; ++pass) {
                 if (!mbar_wait(&sh.go, (uint32_t)(pass & 1), abort)) break;
                 if (*reinterpret_cast<volatile int *>(&sh.pass_stop)) break;
@@ -563,13 +565,13 @@ __device__ __forceinline__ void read_role(const Params &p, const CUtensorMap *tm
                     const int stage = (int)(ci % RS_BSTAGES);
                     if (!mbar_wait(&sh.full[stage], (uint32_t)((ci / RS_BSTAGES) & 1), abort)) { ok = false; break; }
                     tc_fence_after();
-                    const uint32_t ab = smem_u32(sA + stage * RS_B_STAGE);
+                    const uint64_t ad = smem_desc_advance(adesc0, stage * RS_B_STAGE);
 #pragma unroll
                     for (int kc = 0; kc < TV_KCH; ++kc)
 #pragma unroll
                         for (int kk = 0; kk < TV_BK / 16; ++kk)
-                            tc_mma_bf16(d, smem_desc_sw128(ab + kc * TV_A_STAGE + kk * 32),
-                                        smem_desc_sw128(z0 + kc * TV_Z_CHUNK + kk * 32), TV_IDESC, (kc | kk) != 0);
+                            tc_mma_bf16(d, smem_desc_advance(ad, kc * TV_A_STAGE + kk * 32),
+                                        smem_desc_advance(zdesc0, kc * TV_Z_CHUNK + kk * 32), TV_IDESC, (kc | kk) != 0);
                     tc_commit(&sh.empty[stage]);
                     tc_commit(&sh.tfull[buf]);
                 }

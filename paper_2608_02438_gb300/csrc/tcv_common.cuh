@@ -85,4 +85,10 @@ __device__ __forceinline__ void load_s_group(uint4 (&r)[4], const uint16_t *row,
     for (int c = 0; c < 4; ++c) r[c] = make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
 }
 
+// The descriptor of the same operand layout `bytes` further on (a multiple of
+// 16): only the start-address field (bits 0-13, address >> 4) moves, and it
+// cannot overflow for shared-memory addresses below 256 KB.  One thread issues
+// every MMA, so descriptors are formed once and advanced with one add per MMA.
+__device__ __forceinline__ uint64_t smem_desc_advance(uint64_t desc, uint32_t bytes) { return desc + (bytes >> 4); }
+
 }  // namespace xp

@@ -135,4 +135,10 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
     return (uint32_t)f2bf(lo) | ((uint32_t)f2bf(hi) << 16);
 }
 
+// The descriptor of the same operand layout `bytes` further on (a multiple of
+// 16): only the start-address field (bits 0-13, address >> 4) moves, and it
+// cannot overflow for shared-memory addresses below 256 KB.  One thread issues
+// every MMA, so descriptors are formed once and advanced with one add per MMA.
+__device__ __forceinline__ uint64_t smem_desc_advance(uint64_t desc, uint32_t bytes) { return desc + (bytes >> 4); }
+
 }  // namespace xp

@@ -256,17 +256,21 @@ __device__ __forceinline__ void train_tok_body(const TrainParams &p, const CUten
         // ---------------------------------------------------- MMA issuer
         if (lane == 0 && items > 0) {
             const uint32_t b0 = smem_u32(sB), d0 = smem_u32(sD);
+            // descriptors formed once, advanced per MMA
+            const uint64_t bdesc0 = smem_desc_sw128(b0), ddesc0 = smem_desc_sw128(d0);
+            const uint64_t bmn0 = smem_desc_sw128_mn(b0, BCH);
             // dz += dl(u) W_r(u): A = the dl tile (K-major over ids), B = the W_r
             // tile read MN-major (N = r along the 128-byte rows, K = ids)
             auto dz_step = [&](int u) -> bool {
                 const int db = u & 1;
                 if (!mbar_wait_spin(&sh.dfull[db], (uint32_t)((u >> 1) & 1), abort, lim)) return false;
                 tc_fence_after();
-                const uint32_t bs = b0 + (u % NB) * BST;
+                const uint64_t bs = smem_desc_advance(bmn0, (u % NB) * BST);
+                const uint64_t ds = smem_desc_advance(ddesc0, db * TR_D_BUF);
 #pragma unroll
                 for (int kk = 0; kk < TR_BN / 16; ++kk)
-                    tc_mma_bf16(tmem + TR_DZ_COL, smem_desc_sw128(d0 + db * TR_D_BUF + kk * 32),
-                                smem_desc_sw128_mn(bs + kk * 2048, BCH), TR_IDESC_D, (u | kk) != 0);
+                    tc_mma_bf16(tmem + TR_DZ_COL, smem_desc_advance(ds, kk * 32), smem_desc_advance(bs, kk * 2048),
+                                TR_IDESC_D, (u | kk) != 0);
                 tc_commit(&sh.empty[u % NB]);
                 tc_commit(&sh.dempty[db]);
                 return true;
@@ -287,15 +291,15 @@ __device__ __forceinline__ void train_tok_body(const TrainParams &p, const CUten
                     break;
                 }
                 tc_fence_after();
-                const uint32_t bs0 = b0 + st0 * BST, bs1 = b0 + st1 * BST;
+                const uint64_t bs0 = smem_desc_advance(bdesc0, st0 * BST), bs1 = smem_desc_advance(bdesc0, st1 * BST);
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk) {
                         tc_mma_bf16_ts(tmem + q0 * bn, tmem + ZC + c * 32 + kk * 8,
-                                       smem_desc_sw128(bs0 + c * BCH + kk * 32), idesc_f, (c | kk) != 0);
+                                       smem_desc_advance(bs0, c * BCH + kk * 32), idesc_f, (c | kk) != 0);
                         tc_mma_bf16_ts(tmem + q1 * bn, tmem + ZC + c * 32 + kk * 8,
-                                       smem_desc_sw128(bs1 + c * BCH + kk * 32), idesc_f, (c | kk) != 0);
+                                       smem_desc_advance(bs1, c * BCH + kk * 32), idesc_f, (c | kk) != 0);
                     }
                 tc_commit(&sh.tfull[q0]);
                 tc_commit(&sh.tfull[q1]);
@@ -310,13 +314,13 @@ __device__ __forceinline__ void train_tok_body(const TrainParams &p, const CUten
                     break;
                 }
                 tc_fence_after();
-                const uint32_t bs = b0 + st * BST;
+                const uint64_t bs = smem_desc_advance(bdesc0, st * BST);
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk)
                         tc_mma_bf16_ts(tmem + buf * bn, tmem + ZC + c * 32 + kk * 8,
-                                       smem_desc_sw128(bs + c * BCH + kk * 32), idesc_f, (c | kk) != 0);
+                                       smem_desc_advance(bs, c * BCH + kk * 32), idesc_f, (c | kk) != 0);
                 tc_commit(&sh.tfull[buf]);
                 if (!dzm) tc_commit(&sh.empty[st]);
                 else if (it > 0 && !dz_step(it - 1)) ok = false;
@@ -744,6 +748,9 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
         // drained.  F runs ahead of D while the epilogue works.
         if (lane == 0 && nsteps > 0) {
             const uint32_t z0 = smem_u32(sZ), d0 = smem_u32(sD);
+            // descriptors formed once, advanced per MMA
+            const uint64_t zdesc0 = smem_desc_sw128(z0), ddesc0 = smem_desc_sw128(d0);
+            const uint64_t zmn0 = smem_desc_sw128_mn(z0, TV_Z_CHUNK);
             const int ntiles = ((int)blockIdx.x < nvt) ? (nvt - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
             const int total = ntiles * nsteps;
             int kf = 0, kd = 0;
@@ -759,13 +766,13 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
                         mbar_try_wait(&sh.zfull[zs], (uint32_t)((kf / TV_ZS) & 1)) &&
                         mbar_try_wait(&sh.tempty[buf], (uint32_t)(((kf >> 1) & 1) ^ 1))) {
                         tc_fence_after();
-                        const uint32_t zb = z0 + zs * TV_Z_BYTES;
+                        const uint64_t zb = smem_desc_advance(zdesc0, zs * TV_Z_BYTES);
 #pragma unroll
                         for (int c = 0; c < 4; ++c)
 #pragma unroll
                             for (int kk = 0; kk < 4; ++kk)
                                 tc_mma_bf16_ts(tmem + buf * TV_BN, tmem + TV_WR_COL + c * 32 + kk * 8,
-                                               smem_desc_sw128(zb + c * TV_Z_CHUNK + kk * 32), TV_IDESC_F,
+                                               smem_desc_advance(zb, c * TV_Z_CHUNK + kk * 32), TV_IDESC_F,
                                                (c | kk) != 0);
                         tc_commit(&sh.tfull[buf]);
                         if (u == nsteps - 1) tc_commit(&sh.a_empty);
@@ -779,12 +786,12 @@ __global__ void __launch_bounds__(TV_THREADS, 1)
                     if (mbar_try_wait(&sh.dfull[db], (uint32_t)((kd >> 1) & 1)) &&
                         (u != 0 || mbar_try_wait(&sh.wempty, (uint32_t)((lt & 1) ^ 1)))) {
                         tc_fence_after();
-                        const uint32_t zb = z0 + (kd % TV_ZS) * TV_Z_BYTES;
+                        const uint64_t zb = smem_desc_advance(zmn0, (kd % TV_ZS) * TV_Z_BYTES);
+                        const uint64_t ds = smem_desc_advance(ddesc0, db * TV_D_BUF);
 #pragma unroll
                         for (int kk = 0; kk < TV_BN / 16; ++kk)
-                            tc_mma_bf16(tmem + TV_DW_COL, smem_desc_sw128(d0 + db * TV_D_BUF + kk * 32),
-                                        smem_desc_sw128_mn(zb + kk * 2048, TV_Z_CHUNK), TV_IDESC_D,
-                                        !(u == 0 && kk == 0));
+                            tc_mma_bf16(tmem + TV_DW_COL, smem_desc_advance(ds, kk * 32), smem_desc_advance(zb, kk * 2048),
+                                        TV_IDESC_D, !(u == 0 && kk == 0));
                         tc_commit(&sh.zempty[kd % TV_ZS]);
                         tc_commit(&sh.dempty[db]);
                         if (u == nsteps - 1) tc_commit(&sh.wfull);
