@@ -49,7 +49,8 @@ def test_profiled_traffic_needs_matching_hash(bench, tmp_path, monkeypatch):
 
 def test_committed_summaries_name_their_kernel_sources(bench):
     # every summary the bench can cite exists and carries the fields it reads
-    paths = [bench.SMALL_SUMMARY] + list(bench.READ_SUMMARIES.values())
+    paths = ([bench.SMALL_SUMMARY] + list(bench.READ_SUMMARIES.values()) + list(bench.LM_SUMMARIES.values()) +
+             list(bench.TRAIN_SUMMARIES.values()))
     for rel in paths:
         path = os.path.join(ROOT, rel)
         assert os.path.isfile(path), rel
